@@ -1,0 +1,174 @@
+"""fp64 CPU oracle for exact attention backward-over-backward (test infrastructure).
+
+Only tests/, ``__graft_entry__.smoke()`` and bench.py's CPU-baseline / reference
+leg may import this package.  The product (paper_2609_24089_gb300) never does.
+
+The arithmetic lives in ``fbob_oracle.c`` (plain fp64 C, OpenMP over rows); this
+module only builds that file, marshals numpy float64 arrays into it and loops
+over heads.  Every input is [B, H, N, d] (or [N, d] for one head) float64.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import tempfile
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "fbob_oracle.c")
+_LIBS = {}
+
+
+def lib_path(mutant: int = 0, out_dir: str | None = None) -> str:
+    name = "libfbob_oracle.so" if mutant == 0 else f"libfbob_oracle_mutant{mutant}.so"
+    return os.path.join(out_dir or _HERE, name)
+
+
+def build(mutant: int = 0, out_dir: str | None = None, force: bool = False) -> str:
+    """Compile the oracle with gcc (-O2, OpenMP, no fast-math)."""
+    path = lib_path(mutant, out_dir)
+    if (not force and os.path.exists(path)
+            and os.path.getmtime(path) >= os.path.getmtime(_SRC)):
+        return path
+    tmp = path + f".tmp{os.getpid()}"
+    cmd = ["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-fopenmp",
+           "-fno-fast-math", "-ffp-contract=off", f"-DFBOB_MUTANT={int(mutant)}",
+           _SRC, "-o", tmp, "-lm"]
+    subprocess.run(cmd, check=True)
+    os.replace(tmp, path)
+    return path
+
+
+def _load(mutant: int = 0, out_dir: str | None = None):
+    key = (mutant, out_dir)
+    if key in _LIBS:
+        return _LIBS[key]
+    lib = ctypes.CDLL(build(mutant, out_dir))
+    i64, dbl, cint = ctypes.c_int64, ctypes.c_double, ctypes.c_int
+    p = ctypes.c_void_p
+    lib.fbob_oracle_fwd.argtypes = [i64, i64, dbl, cint, p, p, p, p, p, cint]
+    lib.fbob_oracle_bwd.argtypes = [i64, i64, dbl, cint, p, p, p, p, p, p, p, p, cint]
+    lib.fbob_oracle_bob.argtypes = [i64, i64, dbl, cint, p, p, p, p, p, p, p,
+                                    p, i64, i64, i64, p, p, p, p, p, p, p, p, cint]
+    for f in (lib.fbob_oracle_fwd, lib.fbob_oracle_bwd, lib.fbob_oracle_bob):
+        f.restype = cint
+    _LIBS[key] = lib
+    return lib
+
+
+def _c(x):
+    return np.ascontiguousarray(x, dtype=np.float64)
+
+
+def _ptr(x):
+    return None if x is None else x.ctypes.data_as(ctypes.c_void_p)
+
+
+def _heads(x):
+    x = np.asarray(x)
+    if x.ndim == 2:
+        return x[None, None]
+    return x
+
+
+def fwd(q, k, v, scale, causal, nthreads=0):
+    """Forward attention (eq. 1).  Returns O [B,H,N,d] and natural-log L [B,H,N]."""
+    q, k, v = (_c(_heads(t)) for t in (q, k, v))
+    B, H, N, d = q.shape
+    lib = _load()
+    O = np.zeros_like(q)
+    L = np.zeros((B, H, N))
+    for b in range(B):
+        for h in range(H):
+            o_ = np.zeros((N, d)); l_ = np.zeros(N)
+            rc = lib.fbob_oracle_fwd(N, d, float(scale), int(bool(causal)),
+                                     _ptr(_c(q[b, h])), _ptr(_c(k[b, h])), _ptr(_c(v[b, h])),
+                                     _ptr(o_), _ptr(l_), int(nthreads))
+            assert rc == 0, rc
+            O[b, h], L[b, h] = o_, l_
+    return O, L
+
+
+def bwd(q, k, v, dout, scale, causal, nthreads=0):
+    """First backward (eqs. 2-3).  Returns dQ, dK, dV [B,H,N,d] and D [B,H,N]."""
+    q, k, v, dout = (_c(_heads(t)) for t in (q, k, v, dout))
+    B, H, N, d = q.shape
+    lib = _load()
+    outs = [np.zeros_like(q) for _ in range(3)]
+    D = np.zeros((B, H, N))
+    for b in range(B):
+        for h in range(H):
+            dq, dk, dv, dd = np.zeros((N, d)), np.zeros((N, d)), np.zeros((N, d)), np.zeros(N)
+            rc = lib.fbob_oracle_bwd(N, d, float(scale), int(bool(causal)),
+                                     _ptr(_c(q[b, h])), _ptr(_c(k[b, h])), _ptr(_c(v[b, h])),
+                                     _ptr(_c(dout[b, h])), _ptr(dq), _ptr(dk), _ptr(dv),
+                                     _ptr(dd), int(nthreads))
+            assert rc == 0, rc
+            outs[0][b, h], outs[1][b, h], outs[2][b, h], D[b, h] = dq, dk, dv, dd
+    return outs[0], outs[1], outs[2], D
+
+
+def bob_head(q, k, v, dout, gq, gk, gv, scale, causal, rows=None, cols=None,
+             nthreads=0, mutant=0, mutant_dir=None):
+    """Backward-over-backward of one head ([N, d] float64 arrays).
+
+    rows: query rows whose row-owned outputs are wanted (default: all).
+    cols: (c0, c1) key columns receiving the listed rows' contributions to
+          Ktil, Vtil (default: all columns when rows is all rows, else none).
+    Returns a dict with qbar, dobar, alpha, E, D, L (indexed like rows) and
+    kbar, vbar ((c1-c0) x d; complete only if every contributing row is listed).
+    """
+    q, k, v, dout, gq, gk, gv = (_c(t) for t in (q, k, v, dout, gq, gk, gv))
+    N, d = q.shape
+    if rows is None:
+        rows = np.arange(N, dtype=np.int64)
+        if cols is None:
+            cols = (0, N)
+    rows = np.ascontiguousarray(rows, dtype=np.int64)
+    if cols is None:
+        cols = (0, 0)
+    c0, c1 = int(cols[0]), int(cols[1])
+    nr = rows.shape[0]
+    nc = max(c1 - c0, 0)
+    res = {
+        "qbar": np.zeros((nr, d)), "dobar": np.zeros((nr, d)),
+        "alpha": np.zeros(nr), "E": np.zeros(nr), "D": np.zeros(nr), "L": np.zeros(nr),
+        "kbar": np.zeros((nc, d)), "vbar": np.zeros((nc, d)),
+    }
+    lib = _load(mutant, mutant_dir)
+    rc = lib.fbob_oracle_bob(N, d, float(scale), int(bool(causal)),
+                             _ptr(q), _ptr(k), _ptr(v), _ptr(dout), _ptr(gq), _ptr(gk), _ptr(gv),
+                             _ptr(rows), nr, c0, c1,
+                             _ptr(res["qbar"]), _ptr(res["dobar"]), _ptr(res["alpha"]),
+                             _ptr(res["E"]), _ptr(res["D"]), _ptr(res["L"]),
+                             _ptr(res["kbar"]), _ptr(res["vbar"]), int(nthreads))
+    assert rc == 0, rc
+    return res
+
+
+def bob(q, k, v, dout, gq, gk, gv, scale, causal, nthreads=0, mutant=0, mutant_dir=None):
+    """Full backward-over-backward on [B,H,N,d] (or [N,d]) float64 arrays.
+
+    Returns (qbar, kbar, vbar, dobar, alpha, E, D) with the input's batch shape.
+    """
+    ts = [_c(_heads(t)) for t in (q, k, v, dout, gq, gk, gv)]
+    B, H, N, d = ts[0].shape
+    out = {n: np.zeros((B, H, N, d)) for n in ("qbar", "kbar", "vbar", "dobar")}
+    for n in ("alpha", "E", "D"):
+        out[n] = np.zeros((B, H, N))
+    for b in range(B):
+        for h in range(H):
+            r = bob_head(*(t[b, h] for t in ts), scale, causal, nthreads=nthreads,
+                         mutant=mutant, mutant_dir=mutant_dir)
+            for n in ("qbar", "kbar", "vbar", "dobar", "alpha", "E", "D"):
+                out[n][b, h] = r[n]
+    return (out["qbar"], out["kbar"], out["vbar"], out["dobar"],
+            out["alpha"], out["E"], out["D"])
+
+
+def mutant_build_dir():
+    d = os.path.join(tempfile.gettempdir(), "fbob_oracle_mutants")
+    os.makedirs(d, exist_ok=True)
+    return d

@@ -1,0 +1,334 @@
+/*
+ * fbob_oracle.c -- plain fp64 CPU oracle for exact attention backward-over-backward.
+ *
+ * TEST INFRASTRUCTURE ONLY.  Nothing on the product path may load or call this
+ * file: only tests/, __graft_entry__.smoke() and bench.py's cpu_baseline /
+ * reference leg use it.  It shares no code, header, table or helper with the
+ * CUDA library under paper_2609_24089_gb300/csrc.
+ *
+ * What it computes, all per single attention head, on row-major [N x d] fp64
+ * arrays (the bf16 test inputs up-cast exactly):
+ *
+ *   fbob_oracle_fwd : forward attention, Sec. 2 eq. (1):
+ *                     S = tau Q K^T + M,  P = softmax_row(S),  O = P V,
+ *                     L_i = log sum_{j in V_i} exp(S_ij)  (natural log).
+ *   fbob_oracle_bwd : first backward, eqs. (2)-(3):
+ *                     dP = dO V^T, dV = P^T dO, D_i = sum_j P_ij dP_ij,
+ *                     dS = P o (dP - D 1^T), dQ = tau dS K, dK = tau dS^T Q.
+ *   fbob_oracle_bob : backward-over-backward, eqs. (4)-(7), App. C steps 1-7
+ *                     and the assembled identities closing App. C:
+ *                     F = tau (U_Q K^T + Q U_K^T)           (App. C step 1)
+ *                     alpha_i = sum_j P_ij F_ij              (step 2)
+ *                     Vtil = (P o h)^T dO, h = F - alpha 1^T (step 3)
+ *                     C = dO U_V^T,  dOtil = P U_V + (P o h) V   (step 4)
+ *                     Ptil = C + F o (dP - D 1^T) - alpha o dP    (step 5)
+ *                     E_i = sum_j P_ij Ptil_ij, Stil = P o (Ptil - E 1^T)  (step 6)
+ *                     Qtil = tau (Stil K + dS U_K), Ktil = tau (Stil^T Q + dS^T U_Q) (step 7)
+ *
+ * The oracle deliberately does NOT use the affine fusion of Prop. 3.1 nor the
+ * two-pass schedule of Algorithm 1: every row is materialised in full (all N
+ * scores of that row), alpha and E are formed as plain row sums before they are
+ * used, and every output is the plain sum its defining equation states.
+ *
+ * Masking (Sec. 2): the valid column set of row i is V_i = {j < N} without a
+ * mask and {j <= i} with the causal mask (square, top-left aligned, diagonal
+ * included).  Entries outside V_i have P = 0 and contribute nothing.
+ *
+ * Threads: rows are independent, so OpenMP splits rows across threads.  The
+ * column-owned sums (Ktil, Vtil, dV, dK) are accumulated into one private
+ * buffer per thread and reduced in thread order at the end.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+/* Optional deliberately planted mistakes, used only by the test that checks
+ * the pins have the power to catch them (tests/test_oracle_mutants.py).  The
+ * default build has FBOB_MUTANT == 0 and none of these branches exist. */
+#ifndef FBOB_MUTANT
+#define FBOB_MUTANT 0
+#endif
+
+static double dot(const double* a, const double* b, int64_t d) {
+    double s = 0.0;
+    for (int64_t t = 0; t < d; ++t) s += a[t] * b[t];
+    return s;
+}
+
+static int64_t valid_cols(int64_t i, int64_t N, int causal) {
+    return causal ? (i + 1 < N ? i + 1 : N) : N;
+}
+
+static int pick_threads(int nthreads) {
+#ifdef _OPENMP
+    return nthreads > 0 ? nthreads : omp_get_max_threads();
+#else
+    (void)nthreads;
+    return 1;
+#endif
+}
+
+static int thread_id(void) {
+#ifdef _OPENMP
+    return omp_get_thread_num();
+#else
+    return 0;
+#endif
+}
+
+/* Row i of S and P (eq. 1): S_ij = tau q_i.k_j for j in V_i, L_i the
+ * natural-log normaliser, P_ij = exp(S_ij - L_i).  Returns |V_i|. */
+static int64_t softmax_row(int64_t i, int64_t N, int64_t d, double tau, int causal,
+                           const double* Q, const double* K, double* S, double* P,
+                           double* L_out) {
+    const int64_t nv = valid_cols(i, N, causal);
+    double m = -INFINITY;
+    for (int64_t j = 0; j < nv; ++j) {
+        S[j] = tau * dot(Q + i * d, K + j * d, d);
+        if (S[j] > m) m = S[j];
+    }
+    double z = 0.0;
+    for (int64_t j = 0; j < nv; ++j) z += exp(S[j] - m);
+    const double L = m + log(z);
+    for (int64_t j = 0; j < nv; ++j) P[j] = exp(S[j] - L);
+    *L_out = L;
+    return nv;
+}
+
+/* ---------------------------------------------------------------- forward */
+int fbob_oracle_fwd(int64_t N, int64_t d, double tau, int causal,
+                    const double* Q, const double* K, const double* V,
+                    double* O, double* L, int nthreads) {
+    if (N < 0 || d <= 0) return 1;
+    const int nt = pick_threads(nthreads);
+#pragma omp parallel num_threads(nt)
+    {
+        double* S = (double*)malloc(sizeof(double) * (size_t)(N > 0 ? N : 1));
+        double* P = (double*)malloc(sizeof(double) * (size_t)(N > 0 ? N : 1));
+#pragma omp for schedule(static)
+        for (int64_t i = 0; i < N; ++i) {
+            double Li;
+            const int64_t nv = softmax_row(i, N, d, tau, causal, Q, K, S, P, &Li);
+            L[i] = Li;
+            for (int64_t a = 0; a < d; ++a) {
+                double acc = 0.0;
+                for (int64_t j = 0; j < nv; ++j) acc += P[j] * V[j * d + a];
+                O[i * d + a] = acc;
+            }
+        }
+        free(S);
+        free(P);
+    }
+    return 0;
+}
+
+/* ------------------------------------------------------- first backward */
+int fbob_oracle_bwd(int64_t N, int64_t d, double tau, int causal,
+                    const double* Q, const double* K, const double* V, const double* dO,
+                    double* dQ, double* dK, double* dV, double* Dvec, int nthreads) {
+    if (N < 0 || d <= 0) return 1;
+    const int nt = pick_threads(nthreads);
+    const size_t nd = (size_t)N * (size_t)d;
+    double* part = (double*)calloc((size_t)nt * 2 * (nd > 0 ? nd : 1), sizeof(double));
+    if (!part) return 2;
+#pragma omp parallel num_threads(nt)
+    {
+        double* S = (double*)malloc(sizeof(double) * (size_t)(N > 0 ? N : 1));
+        double* P = (double*)malloc(sizeof(double) * (size_t)(N > 0 ? N : 1));
+        double* dP = (double*)malloc(sizeof(double) * (size_t)(N > 0 ? N : 1));
+        double* my_dK = part + (size_t)thread_id() * 2 * nd;
+        double* my_dV = my_dK + nd;
+#pragma omp for schedule(static)
+        for (int64_t i = 0; i < N; ++i) {
+            double Li;
+            const int64_t nv = softmax_row(i, N, d, tau, causal, Q, K, S, P, &Li);
+            double D = 0.0;                                   /* D_i = sum_j P_ij dP_ij */
+            for (int64_t j = 0; j < nv; ++j) {
+                dP[j] = dot(dO + i * d, V + j * d, d);        /* dP = dO V^T */
+                D += P[j] * dP[j];
+            }
+            Dvec[i] = D;
+            for (int64_t a = 0; a < d; ++a) dQ[i * d + a] = 0.0;
+            for (int64_t j = 0; j < nv; ++j) {
+                const double dS = P[j] * (dP[j] - D);         /* dS = P o (dP - D) */
+                for (int64_t a = 0; a < d; ++a) {
+                    dQ[i * d + a] += tau * dS * K[j * d + a];     /* dQ = tau dS K   */
+                    my_dK[j * d + a] += tau * dS * Q[i * d + a];  /* dK = tau dS^T Q */
+                    my_dV[j * d + a] += P[j] * dO[i * d + a];     /* dV = P^T dO     */
+                }
+            }
+        }
+        free(S);
+        free(P);
+        free(dP);
+    }
+    for (size_t e = 0; e < nd; ++e) {
+        double k = 0.0, v = 0.0;
+        for (int t = 0; t < nt; ++t) {
+            k += part[(size_t)t * 2 * nd + e];
+            v += part[(size_t)t * 2 * nd + nd + e];
+        }
+        dK[e] = k;
+        dV[e] = v;
+    }
+    free(part);
+    return 0;
+}
+
+/* ----------------------------------------------- backward-over-backward
+ *
+ * rows[0..nrows): the query rows whose row-owned outputs are produced
+ *   (Qtil, dOtil, alpha, E, D, L are written at positions 0..nrows of the
+ *   corresponding output arrays, in the order of rows[]).
+ * [c0, c1): the key columns whose column-owned outputs Ktil, Vtil receive the
+ *   contributions of the listed rows (written as a (c1-c0) x d block).  They
+ *   are the complete Ktil_j, Vtil_j only when every row i with j in V_i is
+ *   listed: all rows without a mask, rows i >= j with the causal mask.
+ * Any output pointer may be NULL; c1 <= c0 skips the column-owned sums.
+ */
+int fbob_oracle_bob(int64_t N, int64_t d, double tau, int causal,
+                    const double* Q, const double* K, const double* V, const double* dO,
+                    const double* UQ, const double* UK, const double* UV,
+                    const int64_t* rows, int64_t nrows, int64_t c0, int64_t c1,
+                    double* Qt, double* dOt, double* alpha_out, double* E_out,
+                    double* D_out, double* L_out, double* Kt, double* Vt, int nthreads) {
+    if (N < 0 || d <= 0 || nrows < 0) return 1;
+    for (int64_t r = 0; r < nrows; ++r)
+        if (rows[r] < 0 || rows[r] >= N) return 1;
+    if (c0 < 0) c0 = 0;
+    if (c1 > N) c1 = N;
+    const int64_t ncols = c1 > c0 ? c1 - c0 : 0;
+    const int nt = pick_threads(nthreads);
+    const size_t cd = (size_t)ncols * (size_t)d;
+    double* part = NULL;
+    if (cd > 0) {
+        part = (double*)calloc((size_t)nt * 2 * cd, sizeof(double));
+        if (!part) return 2;
+    }
+#pragma omp parallel num_threads(nt)
+    {
+        const size_t n1 = (size_t)(N > 0 ? N : 1);
+        double* S = (double*)malloc(sizeof(double) * n1);
+        double* P = (double*)malloc(sizeof(double) * n1);
+        double* dP = (double*)malloc(sizeof(double) * n1);
+        double* F = (double*)malloc(sizeof(double) * n1);
+        double* C = (double*)malloc(sizeof(double) * n1);
+        double* Pt = (double*)malloc(sizeof(double) * n1);
+        double* St = (double*)malloc(sizeof(double) * n1);
+        double* dS = (double*)malloc(sizeof(double) * n1);
+        double* h = (double*)malloc(sizeof(double) * n1);
+        double* my_Kt = part ? part + (size_t)thread_id() * 2 * cd : NULL;
+        double* my_Vt = part ? my_Kt + cd : NULL;
+#pragma omp for schedule(static)
+        for (int64_t r = 0; r < nrows; ++r) {
+            const int64_t i = rows[r];
+            const double* q = Q + i * d;
+            const double* dout = dO + i * d;
+            const double* uq = UQ + i * d;
+            double Li;
+            /* eq. (1): scores and probabilities of row i */
+            const int64_t nv = softmax_row(i, N, d, tau, causal, Q, K, S, P, &Li);
+            /* eq. (2): dP = dO V^T and D_i = sum_j P_ij dP_ij */
+            double D = 0.0;
+            for (int64_t j = 0; j < nv; ++j) {
+                dP[j] = dot(dout, V + j * d, d);
+                D += P[j] * dP[j];
+            }
+            /* App. C step 1: F = tau (U_Q K^T + Q U_K^T); step 4: C = dO U_V^T */
+            for (int64_t j = 0; j < nv; ++j) {
+#if FBOB_MUTANT == 1 /* planted: dropped Q U_K^T term */
+                F[j] = tau * dot(uq, K + j * d, d);
+#elif FBOB_MUTANT == 2 /* planted: transposed operand, U_Q paired with U_K */
+                F[j] = tau * (dot(uq, UK + j * d, d) + dot(q, UK + j * d, d));
+#else
+                F[j] = tau * (dot(uq, K + j * d, d) + dot(q, UK + j * d, d));
+#endif
+                C[j] = dot(dout, UV + j * d, d);
+            }
+            /* step 2: alpha_i = sum_j P_ij F_ij */
+            double alpha = 0.0;
+            for (int64_t j = 0; j < nv; ++j) alpha += P[j] * F[j];
+            /* step 5: Ptil = C + F o (dP - D) - alpha dP */
+            for (int64_t j = 0; j < nv; ++j) {
+#if FBOB_MUTANT == 3 /* planted: wrong sign on the alpha term */
+                Pt[j] = C[j] + F[j] * (dP[j] - D) + alpha * dP[j];
+#elif FBOB_MUTANT == 4 /* planted: dropped C (the dV-child contribution) */
+                Pt[j] = F[j] * (dP[j] - D) - alpha * dP[j];
+#else
+                Pt[j] = C[j] + F[j] * (dP[j] - D) - alpha * dP[j];
+#endif
+            }
+            /* step 6: E_i = sum_j P_ij Ptil_ij, Stil = P o (Ptil - E) */
+            double E = 0.0;
+            for (int64_t j = 0; j < nv; ++j) E += P[j] * Pt[j];
+            for (int64_t j = 0; j < nv; ++j) {
+#if FBOB_MUTANT == 5 /* planted: E row scalar dropped */
+                St[j] = P[j] * Pt[j];
+#else
+                St[j] = P[j] * (Pt[j] - E);
+#endif
+                dS[j] = P[j] * (dP[j] - D);                  /* eq. (2) */
+                h[j] = F[j] - alpha;                          /* step 3 */
+            }
+            /* step 7: Qtil_i = tau sum_j (Stil_ij k_j + dS_ij u_K,j);
+             * step 4: dOtil_i = sum_j (P_ij u_V,j + P_ij h_ij v_j) */
+            if (Qt || dOt) {
+                for (int64_t a = 0; a < d; ++a) {
+                    double qa = 0.0, oa = 0.0;
+                    for (int64_t j = 0; j < nv; ++j) {
+                        qa += St[j] * K[j * d + a] + dS[j] * UK[j * d + a];
+#if FBOB_MUTANT == 6 /* planted: h replaced by F (alpha dropped from h) */
+                        oa += P[j] * UV[j * d + a] + P[j] * F[j] * V[j * d + a];
+#elif FBOB_MUTANT == 7 /* planted: wrong index, value row i used for every j */
+                        oa += P[j] * UV[j * d + a] + P[j] * h[j] * V[i * d + a];
+#else
+                        oa += P[j] * UV[j * d + a] + P[j] * h[j] * V[j * d + a];
+#endif
+                    }
+                    if (Qt) Qt[r * d + a] = tau * qa;
+                    if (dOt) dOt[r * d + a] = oa;
+                }
+            }
+            if (alpha_out) alpha_out[r] = alpha;
+            if (E_out) E_out[r] = E;
+            if (D_out) D_out[r] = D;
+            if (L_out) L_out[r] = Li;
+            /* step 7 / step 3: column-owned sums over the listed rows:
+             * Ktil_j += tau (Stil_ij q_i + dS_ij u_Q,i),  Vtil_j += P_ij h_ij do_i */
+            if (my_Kt) {
+                const int64_t jend = nv < c1 ? nv : c1;
+                for (int64_t j = c0; j < jend; ++j) {
+                    double* kt = my_Kt + (size_t)(j - c0) * d;
+                    double* vt = my_Vt + (size_t)(j - c0) * d;
+                    const double ph = P[j] * h[j];
+                    for (int64_t a = 0; a < d; ++a) {
+#if FBOB_MUTANT == 8 /* planted: U_Q term replaced by U_K of row i */
+                        kt[a] += tau * (St[j] * q[a] + dS[j] * UK[i * d + a]);
+#else
+                        kt[a] += tau * (St[j] * q[a] + dS[j] * uq[a]);
+#endif
+                        vt[a] += ph * dout[a];
+                    }
+                }
+            }
+        }
+        free(S); free(P); free(dP); free(F); free(C); free(Pt); free(St); free(dS); free(h);
+    }
+    if (part) {
+        for (size_t e = 0; e < cd; ++e) {
+            double k = 0.0, v = 0.0;
+            for (int t = 0; t < nt; ++t) {
+                k += part[(size_t)t * 2 * cd + e];
+                v += part[(size_t)t * 2 * cd + cd + e];
+            }
+            if (Kt) Kt[e] = k;
+            if (Vt) Vt[e] = v;
+        }
+        free(part);
+    }
+    return 0;
+}

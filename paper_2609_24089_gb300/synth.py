@@ -1,0 +1,100 @@
+"""Seeded synthetic inputs for attention backward-over-backward.
+
+This module draws random numbers and rounds them to bf16; it holds none of the
+method's arithmetic, so the CUDA path and the CPU oracle can both consume its
+output without sharing any computation.
+
+Recipe (the paper's isolated-kernel benchmark uses fixed-seed random inputs at
+GPT-2 head shape, Sec. 4.1; the shapes below stand in for it):
+  * numpy ``Generator(PCG64(seed))``;
+  * draw order Q, K, V, dO, U_Q, U_K, U_V, each ``standard_normal`` in fp32
+    times the tensor's standard deviation;
+  * round to nearest-even bf16 on the host.  Tensors are carried as uint16
+    bit patterns ([B, H, N, d], row-major) so that both sides see identical
+    values; ``to_f64`` up-casts them exactly.
+"""
+from __future__ import annotations
+
+import dataclasses
+import math
+
+import numpy as np
+
+NAMES = ("q", "k", "v", "dout", "gq", "gk", "gv")
+
+
+@dataclasses.dataclass(frozen=True)
+class Workload:
+    name: str
+    B: int
+    H: int
+    N: int
+    d: int
+    causal: bool
+    seed: int
+    sigma: tuple  # per tensor in NAMES order
+
+    @property
+    def scale(self) -> float:
+        return 1.0 / math.sqrt(self.d)
+
+    @property
+    def shape(self) -> tuple:
+        return (self.B, self.H, self.N, self.d)
+
+
+def _s(*v):
+    return tuple(float(x) for x in v)
+
+
+# The five synthetic workloads.  Standard deviations follow each workload's
+# stated distribution; seeds are the workload index minus one.
+WORKLOADS = {
+    "n128_d64": Workload("n128_d64", 1, 1, 128, 64, False, 0, _s(1, 1, 1, 1, 1, 1, 1)),
+    "n4k_d64": Workload("n4k_d64", 4, 16, 4096, 64, False, 1, _s(1, 1, 1, 1, 1, 1, 1)),
+    "n16k_d128_causal": Workload(
+        "n16k_d128_causal", 2, 16, 16384, 128, True, 2,
+        _s(1, 1, 1, *(4 * [1 / math.sqrt(128)]))),
+    "n64k_d128_causal_peaky": Workload(
+        "n64k_d128_causal_peaky", 1, 8, 65536, 128, True, 3, _s(1.5, 1.5, 1, 1, 1, 1, 1)),
+    "n256k_d64": Workload("n256k_d64", 1, 4, 262144, 64, False, 4, _s(1, 1, 1, 1, 1, 1, 1)),
+}
+
+
+def bf16_bits(x: np.ndarray) -> np.ndarray:
+    """Round fp32 values to bf16 (round to nearest, ties to even); return uint16 bits."""
+    u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32)
+    rounded = (u + np.uint32(0x7FFF) + ((u >> np.uint32(16)) & np.uint32(1))) >> np.uint32(16)
+    return rounded.astype(np.uint16)
+
+
+def to_f64(bits: np.ndarray) -> np.ndarray:
+    """Exact up-cast of bf16 bit patterns to float64."""
+    return (bits.astype(np.uint32) << np.uint32(16)).view(np.float32).astype(np.float64)
+
+
+def to_f32(bits: np.ndarray) -> np.ndarray:
+    return (bits.astype(np.uint32) << np.uint32(16)).view(np.float32)
+
+
+def make_inputs(B, H, N, d, seed, sigma=(1.0,) * 7, heads=None):
+    """Draw the seven bf16 inputs.  ``heads`` (list of flat b*H+h indices)
+    keeps only those heads after drawing, so a slice sees exactly the values
+    the full tensor holds."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    out = {}
+    for name, s in zip(NAMES, sigma):
+        x = rng.standard_normal((B, H, N, d), dtype=np.float32)
+        if s != 1.0:
+            x *= np.float32(s)
+        bits = bf16_bits(x)
+        if heads is not None:
+            bits = np.ascontiguousarray(bits.reshape(B * H, N, d)[list(heads)])
+            bits = bits.reshape(1, len(heads), N, d)
+        out[name] = bits
+        del x
+    return out
+
+
+def workload_inputs(w: Workload, heads=None):
+    return make_inputs(w.B, w.H, w.N, w.d, w.seed, w.sigma, heads=heads)

@@ -1,0 +1,109 @@
+"""Independent references used to pin the fp64 oracle.
+
+Nothing here imports the oracle.  The first backward below is written in
+matrix form from Sec. 2 eqs. (1)-(3) (numpy, batched, real or complex), so
+finite differences and complex-step derivatives of
+
+    Phi = <dQ, U_Q> + <dK, U_K> + <dV, U_V>          (eq. 4)
+
+give backward-over-backward results that owe nothing to the oracle's
+closed-form App. C walk.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+
+def mask(N, causal):
+    if causal:
+        return np.tril(np.ones((N, N)))
+    return np.ones((N, N))
+
+
+def softmax_probs(Q, K, tau, causal):
+    """P = softmax_row(tau Q K^T + M) for [..., N, d] inputs (real or complex).
+
+    The shift uses the real part of the row max so the function stays
+    complex-analytic (the shift cancels exactly in the ratio)."""
+    N = Q.shape[-2]
+    S = tau * (Q @ np.swapaxes(K, -1, -2))
+    Mk = mask(N, causal)
+    shift = np.max(np.where(Mk > 0, S.real, -np.inf), axis=-1, keepdims=True)
+    Ex = np.exp(S - shift) * Mk
+    return Ex / Ex.sum(axis=-1, keepdims=True)
+
+
+def first_backward(Q, K, V, dO, tau, causal):
+    """g(Q, K, V, dO) = (dQ, dK, dV), eqs. (2)-(3), batched over leading dims."""
+    P = softmax_probs(Q, K, tau, causal)
+    dP = dO @ np.swapaxes(V, -1, -2)
+    D = (P * dP).sum(axis=-1, keepdims=True)
+    dS = P * (dP - D)
+    dQ = tau * dS @ K
+    dK = tau * np.swapaxes(dS, -1, -2) @ Q
+    dV = np.swapaxes(P, -1, -2) @ dO
+    return dQ, dK, dV
+
+
+def attention(Q, K, V, tau, causal):
+    return softmax_probs(Q, K, tau, causal) @ V
+
+
+def phi(Q, K, V, dO, UQ, UK, UV, tau, causal):
+    dQ, dK, dV = first_backward(Q, K, V, dO, tau, causal)
+    return ((dQ * UQ).sum(axis=(-1, -2)) + (dK * UK).sum(axis=(-1, -2))
+            + (dV * UV).sum(axis=(-1, -2)))
+
+
+def _perturbed(X, which, deltas):
+    """Stack of copies of the 4 primal inputs with input `which` perturbed
+    entrywise: returns list of 4 arrays shaped [N*d, N, d]."""
+    N, d = X[0].shape
+    out = []
+    for t in range(4):
+        base = np.broadcast_to(X[t], (N * d, N, d)).astype(np.result_type(X[t], deltas))
+        if t == which:
+            base = base.copy()
+            idx = np.arange(N * d)
+            base[idx, idx // d, idx % d] += deltas
+        out.append(base)
+    return out
+
+
+def bob_central_fd(Q, K, V, dO, UQ, UK, UV, tau, causal, rel_h=1e-5):
+    """grad_{Q,K,V,dO} Phi by central differences, one entry at a time."""
+    X = [Q, K, V, dO]
+    grads = []
+    for which in range(4):
+        x = X[which].reshape(-1)
+        h = rel_h * np.maximum(1.0, np.abs(x))
+        plus = _perturbed(X, which, h)
+        minus = _perturbed(X, which, -h)
+        fp = phi(*plus, UQ, UK, UV, tau, causal)
+        fm = phi(*minus, UQ, UK, UV, tau, causal)
+        grads.append(((fp - fm) / (2 * h)).reshape(X[which].shape))
+    return grads
+
+
+def jacobian_complex_step(Q, K, V, dO, tau, causal, h=1e-30):
+    """Explicit Jacobian of g: rows index vec(dQ, dK, dV) (3Nd), columns index
+    vec(Q, K, V, dO) (4Nd); built column by column by complex step."""
+    N, d = Q.shape
+    X = [Q.astype(complex), K.astype(complex), V.astype(complex), dO.astype(complex)]
+    cols = []
+    for which in range(4):
+        pert = _perturbed(X, which, np.full(N * d, 1j * h))
+        dQ, dK, dV = first_backward(*pert, tau, causal)
+        J = np.concatenate([dQ.reshape(N * d, -1), dK.reshape(N * d, -1),
+                            dV.reshape(N * d, -1)], axis=1).imag / h   # [Nd(in), 3Nd(out)]
+        cols.append(J.T)
+    return np.concatenate(cols, axis=1)                                 # [3Nd, 4Nd]
+
+
+def inner(a, b):
+    return float(np.sum(np.asarray(a) * np.asarray(b)))
+
+
+def rel_fro(x, ref):
+    den = np.linalg.norm(ref)
+    return np.linalg.norm(x - ref) / (den if den > 0 else 1.0)
