@@ -1,0 +1,147 @@
+/*
+ * fbob.h -- C ABI of libfbob: exact backward-over-backward (BoB) of softmax
+ * attention on one NVIDIA GB300 (sm_103a).
+ *
+ * Notation follows the paper (FlashBoB, arXiv 2609.24089): per attention head
+ * Q, K, V, dO, U_Q, U_K, U_V are N x d matrices, tau is the softmax scale,
+ * P = softmax_row(tau Q K^T + M) (Sec. 2, eq. 1).  U_Q, U_K, U_V are the
+ * cotangents on the first-backward outputs dQ, dK, dV; this header calls
+ * them gq, gk, gv.
+ *
+ * Common conventions for every entry point
+ * ----------------------------------------
+ *  Layout     All matrices are contiguous row-major [B, H, N, d] bf16
+ *             (element (b,h,i,a) at ((b*H + h)*N + i)*d + a).  Row vectors
+ *             (lse, dstat, alpha, E, D) are contiguous fp32 [B, H, N].
+ *  Pointers   Device pointers (global memory of the current device), each
+ *             16-byte aligned.  Outputs must not overlap any input or each
+ *             other.
+ *  Shapes     d in {64, 128}; other head dims return FBOB_ERR_UNSUPPORTED.
+ *             N >= 0 is arbitrary (tails are masked); B*H*N == 0 is a valid
+ *             empty problem that launches nothing and returns FBOB_OK.
+ *             N <= 2^24 and B*H <= 2^24.  scale must be finite and > 0
+ *             (1/sqrt(d) in the paper).  causal is 0 or 1; with 1 the mask
+ *             keeps j <= i (square, top-left aligned, diagonal included).
+ *  Stream     Every call enqueues its kernels on `stream` (NULL = legacy
+ *             default stream) and returns without synchronising.
+ *  Memory     The library allocates and frees no device memory.  The caller
+ *             owns every buffer.  Library state is one device-side error word
+ *             per device plus cached driver entry points.
+ *  Errors     Host-side validation failures return immediately, before any
+ *             CUDA call, and launch nothing.  A failed launch returns
+ *             FBOB_ERR_CUDA.  Kernels never trap: every device-side wait is
+ *             bounded, and on expiry the kernel records FBOB_ERR_DEVICE_TIMEOUT
+ *             in the device error word and exits cleanly; fbob_device_status()
+ *             reports it.
+ *  Determinism  No floating-point atomics; every output element has one
+ *             writer, so results are bitwise reproducible run to run.
+ */
+#ifndef FBOB_H_
+#define FBOB_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+struct CUstream_st; /* cudaStream_t == struct CUstream_st* */
+
+typedef enum fbob_status {
+    FBOB_OK = 0,
+    FBOB_ERR_INVALID_ARGUMENT = 1, /* null/misaligned/overlapping pointer, bad shape, scale */
+    FBOB_ERR_UNSUPPORTED = 2,      /* valid request this build does not implement (d) */
+    FBOB_ERR_CUDA = 3,             /* a CUDA runtime/driver call or launch failed */
+    FBOB_ERR_DEVICE_TIMEOUT = 4,   /* a bounded device-side wait expired */
+    FBOB_ERR_DEVICE_FAULT = 5      /* the device reported an error while synchronising */
+} fbob_status;
+
+typedef struct fbob_shape {
+    int64_t B, H, N, d;
+    float scale;    /* tau */
+    int32_t causal; /* 0 or 1 */
+} fbob_shape;
+
+/*
+ * Forward attention, Sec. 2 eq. (1):
+ *   S = scale * Q K^T + M,  P = softmax_row(S),  O = P V,
+ *   lse_i = L_i = log sum_{j valid} exp(S_ij)   (natural log, fp32).
+ * In:  q, k, v  bf16 [B,H,N,d].   Out: o bf16 [B,H,N,d], lse fp32 [B,H,N].
+ */
+int fbob_attn_fwd(const fbob_shape* shape, const void* q, const void* k, const void* v,
+                  void* o, float* lse, struct CUstream_st* stream);
+
+/*
+ * First backward, Sec. 2 eqs. (2)-(3):
+ *   dP = dO V^T, dV = P^T dO, D_i = do_i . o_i, dS = P o (dP - D 1^T),
+ *   dQ = scale dS K, dK = scale dS^T Q.
+ * P is recomputed from q, k and lse.  D (fp32, from the given o and dout) is
+ * written to dstat [B,H,N].
+ * In:  q, k, v, o, dout bf16; lse fp32.   Out: dq, dk, dv bf16; dstat fp32.
+ */
+int fbob_attn_bwd(const fbob_shape* shape, const void* q, const void* k, const void* v,
+                  const void* o, const float* lse, const void* dout,
+                  void* dq, void* dk, void* dv, float* dstat, struct CUstream_st* stream);
+
+/*
+ * Backward-over-backward, Sec. 3.1 eqs. (4)-(5) and closed form eqs. (6)-(7):
+ *   Phi = <dQ, U_Q> + <dK, U_K> + <dV, U_V>,
+ *   (q_bar, k_bar, v_bar, dout_bar) = grad_{Q, K, V, dO} Phi,
+ * computed by the two-pass schedule of Algorithm 1 (row-block pass, then
+ * column-block pass) with the affine fusion of Prop. 3.1 / eq. (8).  No N x N
+ * tensor is written to memory.
+ * In:  q, k, v, o, dout, gq, gk, gv  bf16 [B,H,N,d]; lse fp32 [B,H,N] (natural
+ *      log, as written by fbob_attn_fwd).
+ * Out: q_bar, k_bar, v_bar, dout_bar bf16 [B,H,N,d];
+ *      row_stats fp32 [3,B,H,N] = (alpha, E, D): the two BoB row scalars of
+ *      eq. (6) (alpha_i = sum_j P_ij F_ij, E_i = sum_j P_ij Ptil_ij) and
+ *      D_i = do_i . o_i.  Pass 1 writes it, pass 2 reads it; it is required.
+ */
+int fbob_attn_bob(const fbob_shape* shape, const void* q, const void* k, const void* v,
+                  const void* o, const float* lse, const void* dout,
+                  const void* gq, const void* gk, const void* gv,
+                  void* q_bar, void* k_bar, void* v_bar, void* dout_bar,
+                  float* row_stats, struct CUstream_st* stream);
+
+/*
+ * Pass 1 of Algorithm 1 alone (row-block outer; Alg. 2, first loop):
+ * writes q_bar, dout_bar and row_stats (alpha, E, D).  Same arguments and
+ * rules as fbob_attn_bob; k_bar/v_bar are not touched.
+ */
+int fbob_attn_bob_pass1(const fbob_shape* shape, const void* q, const void* k, const void* v,
+                        const void* o, const float* lse, const void* dout,
+                        const void* gq, const void* gk, const void* gv,
+                        void* q_bar, void* dout_bar, float* row_stats,
+                        struct CUstream_st* stream);
+
+/*
+ * Pass 2 of Algorithm 1 alone (column-block outer; Alg. 2, second loop):
+ * reads row_stats (alpha, E, D, as pass 1 writes them) and lse, writes
+ * k_bar and v_bar.  row_stats is an input here.
+ */
+int fbob_attn_bob_pass2(const fbob_shape* shape, const void* q, const void* k, const void* v,
+                        const float* lse, const void* dout,
+                        const void* gq, const void* gk, const void* gv,
+                        const float* row_stats, void* k_bar, void* v_bar,
+                        struct CUstream_st* stream);
+
+/*
+ * Synchronises `stream`, then returns and clears the device error word of the
+ * current device: FBOB_OK, FBOB_ERR_DEVICE_TIMEOUT (a bounded wait expired in
+ * some kernel since the last call), or FBOB_ERR_DEVICE_FAULT / FBOB_ERR_CUDA
+ * if synchronisation itself failed.
+ */
+int fbob_device_status(struct CUstream_st* stream);
+
+/* Number of kernels the last successful call of the named entry point
+ * enqueued ("fwd", "bwd", "bob", "bob_pass1", "bob_pass2"); -1 if unknown. */
+int fbob_launch_count(const char* entry);
+
+/* Static, human-readable name of a status code. */
+const char* fbob_status_string(int status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FBOB_H_ */

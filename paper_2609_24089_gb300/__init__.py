@@ -1,0 +1,179 @@
+"""Python binding of libfbob (include/fbob.h): exact backward-over-backward of
+softmax attention on GB300.
+
+The functions named like the C entry points (``fbob_attn_fwd``, ...) only
+marshal torch tensors into device pointers and the current CUDA stream; every
+step of the computation runs in the library's kernels.  There is no fallback:
+if libfbob.so is missing or a call fails, an exception is raised.
+The ``attn_*`` helpers additionally allocate the outputs with torch.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libfbob.so")
+HEADER = os.path.join(os.path.dirname(_HERE), "include", "fbob.h")
+
+FBOB_OK = 0
+STATUS = {0: "FBOB_OK", 1: "FBOB_ERR_INVALID_ARGUMENT", 2: "FBOB_ERR_UNSUPPORTED",
+          3: "FBOB_ERR_CUDA", 4: "FBOB_ERR_DEVICE_TIMEOUT", 5: "FBOB_ERR_DEVICE_FAULT"}
+
+
+class FbobError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        super().__init__(f"{where}: {STATUS.get(status, status)}")
+        self.status = status
+
+
+class fbob_shape(ctypes.Structure):
+    _fields_ = [("B", ctypes.c_int64), ("H", ctypes.c_int64), ("N", ctypes.c_int64),
+                ("d", ctypes.c_int64), ("scale", ctypes.c_float), ("causal", ctypes.c_int32)]
+
+
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    from . import buildlib
+    return buildlib.build(force=force)
+
+
+def load():
+    """Load libfbob.so (raises if it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError(f"libfbob.so not built ({LIB_PATH}); run paper_2609_24089_gb300.build()")
+    lib = ctypes.CDLL(LIB_PATH)
+    P = ctypes.c_void_p
+    S = ctypes.POINTER(fbob_shape)
+    sig = {
+        "fbob_attn_fwd": [S, P, P, P, P, P, P],
+        "fbob_attn_bwd": [S, P, P, P, P, P, P, P, P, P, P, P],
+        "fbob_attn_bob": [S, P, P, P, P, P, P, P, P, P, P, P, P, P, P, P],
+        "fbob_attn_bob_pass1": [S, P, P, P, P, P, P, P, P, P, P, P, P, P],
+        "fbob_attn_bob_pass2": [S, P, P, P, P, P, P, P, P, P, P, P, P],
+        "fbob_device_status": [P],
+        "fbob_launch_count": [ctypes.c_char_p],
+        "fbob_status_string": [ctypes.c_int],
+    }
+    for name, argt in sig.items():
+        f = getattr(lib, name)
+        f.argtypes = argt
+        f.restype = ctypes.c_char_p if name == "fbob_status_string" else ctypes.c_int
+    _lib = lib
+    return lib
+
+
+def header_symbols() -> list:
+    """Entry points declared in include/fbob.h."""
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?\w+\**\s+\**(fbob_\w+)\s*\(", text, re.M)))
+
+
+def make_shape(B, H, N, d, scale, causal) -> fbob_shape:
+    return fbob_shape(int(B), int(H), int(N), int(d), float(scale), int(causal))
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    if not t.is_contiguous():
+        raise ValueError("tensors must be contiguous")
+    return t.data_ptr()
+
+
+def _stream(stream):
+    if stream is not None:
+        return stream if isinstance(stream, int) else stream.cuda_stream
+    import torch
+    return torch.cuda.current_stream().cuda_stream
+
+
+def _check(rc, where):
+    if rc != FBOB_OK:
+        raise FbobError(rc, where)
+
+
+def _shape_of(q, scale, causal):
+    B, H, N, d = q.shape
+    return make_shape(B, H, N, d, scale, causal)
+
+
+# ------------------------------------------------ entry points, same names as the C ABI
+def fbob_attn_fwd(shape, q, k, v, o, lse, stream=None):
+    _check(load().fbob_attn_fwd(ctypes.byref(shape), *map(_ptr, (q, k, v, o, lse)),
+                                _stream(stream)), "fbob_attn_fwd")
+
+
+def fbob_attn_bwd(shape, q, k, v, o, lse, dout, dq, dk, dv, dstat, stream=None):
+    _check(load().fbob_attn_bwd(ctypes.byref(shape),
+                                *map(_ptr, (q, k, v, o, lse, dout, dq, dk, dv, dstat)),
+                                _stream(stream)), "fbob_attn_bwd")
+
+
+def fbob_attn_bob(shape, q, k, v, o, lse, dout, gq, gk, gv, q_bar, k_bar, v_bar, dout_bar,
+                  row_stats, stream=None):
+    _check(load().fbob_attn_bob(
+        ctypes.byref(shape),
+        *map(_ptr, (q, k, v, o, lse, dout, gq, gk, gv, q_bar, k_bar, v_bar, dout_bar, row_stats)),
+        _stream(stream)), "fbob_attn_bob")
+
+
+def fbob_attn_bob_pass1(shape, q, k, v, o, lse, dout, gq, gk, gv, q_bar, dout_bar, row_stats,
+                        stream=None):
+    _check(load().fbob_attn_bob_pass1(
+        ctypes.byref(shape),
+        *map(_ptr, (q, k, v, o, lse, dout, gq, gk, gv, q_bar, dout_bar, row_stats)),
+        _stream(stream)), "fbob_attn_bob_pass1")
+
+
+def fbob_attn_bob_pass2(shape, q, k, v, lse, dout, gq, gk, gv, row_stats, k_bar, v_bar,
+                        stream=None):
+    _check(load().fbob_attn_bob_pass2(
+        ctypes.byref(shape),
+        *map(_ptr, (q, k, v, lse, dout, gq, gk, gv, row_stats, k_bar, v_bar)),
+        _stream(stream)), "fbob_attn_bob_pass2")
+
+
+def fbob_device_status(stream=None) -> int:
+    return load().fbob_device_status(_stream(stream))
+
+
+def fbob_launch_count(entry: str) -> int:
+    return load().fbob_launch_count(entry.encode())
+
+
+# ------------------------------------------------ allocating helpers
+def attn_fwd(q, k, v, scale, causal):
+    import torch
+    B, H, N, d = q.shape
+    o = torch.empty_like(q)
+    lse = torch.empty((B, H, N), dtype=torch.float32, device=q.device)
+    fbob_attn_fwd(_shape_of(q, scale, causal), q, k, v, o, lse)
+    return o, lse
+
+
+def attn_bwd(q, k, v, o, lse, dout, scale, causal):
+    import torch
+    B, H, N, d = q.shape
+    dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
+    dstat = torch.empty((B, H, N), dtype=torch.float32, device=q.device)
+    fbob_attn_bwd(_shape_of(q, scale, causal), q, k, v, o, lse, dout, dq, dk, dv, dstat)
+    return dq, dk, dv, dstat
+
+
+def attn_bob(q, k, v, o, lse, dout, gq, gk, gv, scale, causal):
+    """Returns (q_bar, k_bar, v_bar, dout_bar, row_stats[3,B,H,N] = alpha, E, D)."""
+    import torch
+    B, H, N, d = q.shape
+    outs = [torch.empty_like(q) for _ in range(4)]
+    row_stats = torch.empty((3, B, H, N), dtype=torch.float32, device=q.device)
+    fbob_attn_bob(_shape_of(q, scale, causal), q, k, v, o, lse, dout, gq, gk, gv, *outs, row_stats)
+    return (*outs, row_stats)

@@ -1,0 +1,75 @@
+// engine_params.h -- host-visible tile constants, operation kinds, kernel
+// parameter block and per-kernel shared-memory plans of the tile engines.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+namespace fbob {
+
+// Bits of the device-side error word.
+enum : uint32_t { kDevErrTimeout = 1u, kDevErrBadLaunch = 2u };
+
+constexpr int BM = 128;
+constexpr int BN = 64;
+constexpr int kThreads = 320;
+constexpr int kProducerWarp = 8;
+constexpr int kMmaWarp = 9;
+constexpr int kEwThreads = 256;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kColA = 256;  // first stage-A column
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
+
+enum class RowOp { Fwd, BwdDQ, BobPass1 };
+enum class ColOp { BwdDKDV, BobPass2 };
+
+// ---------------------------------------------------------------- parameters
+struct EngineParams {
+  CUtensorMap tm[7];  // stationary maps first (box rows BM), then streamed (box rows BN)
+  const __nv_bfloat16* o;     // forward output O (row engine: D and dOtil)
+  const __nv_bfloat16* dout;  // dO (row engine: D = do.o)
+  const float* lse;           // natural-log L [BH, N]
+  const float* vec_in;        // column engine: D (bwd) or row_stats (alpha,E,D) (pass 2)
+  __nv_bfloat16* out0;        // O | dQ | Qtil  ||  dK | Ktil
+  __nv_bfloat16* out1;        // dOtil          ||  dV | Vtil
+  float* vec_out;             // lse | D | row_stats(alpha, E, D)
+  int N;
+  int BH;
+  int nblk;  // stationary blocks per head
+  int causal;
+  float scale;
+  long long bhn;  // BH * N (row_stats plane stride)
+};
+
+// ---------------------------------------------------------------- configs
+template <RowOp OP, int D>
+struct RowCfg {
+  static constexpr int KB = D / 64;  // 64-wide boxes per row
+  static constexpr int NSTAT = OP == RowOp::Fwd ? 1 : OP == RowOp::BwdDQ ? 2 : 3;
+  static constexpr int NSTREAM = OP == RowOp::BobPass1 ? 4 : 2;
+  static constexpr int DOUT = OP == RowOp::BobPass1 ? 64 : D;  // accumulator width per CTA
+  static constexpr int NSPLIT = D / DOUT;
+  static constexpr int STAT_BYTES = NSTAT * KB * BM * 128;
+  static constexpr int STAGE_BYTES = NSTREAM * KB * BN * 128;
+  static constexpr int NSTAGES = OP == RowOp::BobPass1 ? (D == 64 ? 3 : 2) : 4;
+  static constexpr int MISC_BYTES = 2304;
+  static constexpr int SMEM_BYTES = STAT_BYTES + NSTAGES * STAGE_BYTES + MISC_BYTES;
+};
+
+template <ColOp OP, int D>
+struct ColCfg {
+  static constexpr int KB = D / 64;
+  static constexpr int NSTAT = OP == ColOp::BwdDKDV ? 2 : 4;
+  static constexpr int NSTREAM = OP == ColOp::BwdDKDV ? 2 : 3;
+  static constexpr int NVEC = OP == ColOp::BwdDKDV ? 2 : 4;  // L2, D (, alpha, E)
+  static constexpr int STAT_BYTES = NSTAT * KB * BM * 128;
+  static constexpr int TILE_BYTES = NSTREAM * KB * BN * 128;
+  static constexpr int STAGE_BYTES = TILE_BYTES + 1024;  // + row vectors
+  static constexpr int NSTAGES = (OP == ColOp::BobPass2 && D == 128) ? 2 : (D == 64 ? 4 : 3);
+  static constexpr int MISC_BYTES = 256;
+  static constexpr int SMEM_BYTES = STAT_BYTES + NSTAGES * STAGE_BYTES + MISC_BYTES;
+};
+
+}  // namespace fbob

@@ -1,0 +1,341 @@
+// fbob_api.cu -- the C ABI declared in include/fbob.h: argument validation,
+// TMA tensor-map construction and kernel launches.  Allocates no device memory.
+#include <cudaTypedefs.h>
+#include <cuda_runtime.h>
+
+#include <atomic>
+#include <cmath>
+#include <cstring>
+#include <mutex>
+
+#include "../../include/fbob.h"
+#include "launch.h"
+
+namespace fbob {
+namespace {
+
+constexpr int64_t kMaxN = int64_t(1) << 24;
+constexpr int64_t kMaxBH = int64_t(1) << 24;
+
+std::atomic<int> g_launches[5] = {{-1}, {-1}, {-1}, {-1}, {-1}};
+enum Entry { kEntFwd = 0, kEntBwd, kEntBob, kEntPass1, kEntPass2 };
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static std::once_flag once;
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// [BH, N, d] bf16 tensor viewed as 3-D (d innermost), box = 64 columns x `rows`,
+// 128-byte swizzle, zero fill out of bounds.
+bool make_map(CUtensorMap* m, const void* base, int64_t BH, int64_t N, int64_t d, int rows) {
+  auto enc = encode_fn();
+  if (!enc) return false;
+  cuuint64_t dims[3] = {(cuuint64_t)d, (cuuint64_t)N, (cuuint64_t)BH};
+  cuuint64_t strides[2] = {(cuuint64_t)(d * 2), (cuuint64_t)(N * d * 2)};
+  cuuint32_t box[3] = {64, (cuuint32_t)rows, 1};
+  cuuint32_t es[3] = {1, 1, 1};
+  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides,
+                   box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+struct Span {
+  uintptr_t lo, hi;
+};
+
+bool overlaps(const Span& a, const Span& b) { return a.lo < b.hi && b.lo < a.hi; }
+
+// Shape rules of include/fbob.h.  Returns FBOB_OK, or the status to report;
+// *empty is set when B*H*N == 0.
+int check_shape(const fbob_shape* s, bool* empty) {
+  if (!s) return FBOB_ERR_INVALID_ARGUMENT;
+  if (s->B < 0 || s->H < 0 || s->N < 0 || s->d <= 0) return FBOB_ERR_INVALID_ARGUMENT;
+  if (!(std::isfinite(s->scale) && s->scale > 0.f)) return FBOB_ERR_INVALID_ARGUMENT;
+  if (s->causal != 0 && s->causal != 1) return FBOB_ERR_INVALID_ARGUMENT;
+  if (s->d != 64 && s->d != 128) return FBOB_ERR_UNSUPPORTED;
+  if (s->N > kMaxN) return FBOB_ERR_INVALID_ARGUMENT;
+  if (s->B > kMaxBH || s->H > kMaxBH || s->B * s->H > kMaxBH) return FBOB_ERR_INVALID_ARGUMENT;
+  *empty = (s->B * s->H * s->N) == 0;
+  return FBOB_OK;
+}
+
+// Null / alignment / overlap checks: `in` and `out` are (pointer, bytes) lists.
+int check_ptrs(const void* const* in, const int64_t* in_bytes, int nin, void* const* out,
+               const int64_t* out_bytes, int nout) {
+  Span spans[16];
+  int ns = 0;
+  for (int t = 0; t < nin; ++t) {
+    if (!in[t] || (reinterpret_cast<uintptr_t>(in[t]) & 15u)) return FBOB_ERR_INVALID_ARGUMENT;
+    spans[ns++] = {reinterpret_cast<uintptr_t>(in[t]),
+                   reinterpret_cast<uintptr_t>(in[t]) + (uintptr_t)in_bytes[t]};
+  }
+  const int first_out = ns;
+  for (int t = 0; t < nout; ++t) {
+    if (!out[t] || (reinterpret_cast<uintptr_t>(out[t]) & 15u)) return FBOB_ERR_INVALID_ARGUMENT;
+    spans[ns++] = {reinterpret_cast<uintptr_t>(out[t]),
+                   reinterpret_cast<uintptr_t>(out[t]) + (uintptr_t)out_bytes[t]};
+  }
+  for (int a = first_out; a < ns; ++a)
+    for (int b = 0; b < ns; ++b)
+      if (a != b && overlaps(spans[a], spans[b])) return FBOB_ERR_INVALID_ARGUMENT;
+  return FBOB_OK;
+}
+
+EngineParams base_params(const fbob_shape* s) {
+  EngineParams p;
+  std::memset(&p, 0, sizeof(p));
+  p.N = (int)s->N;
+  p.BH = (int)(s->B * s->H);
+  p.causal = s->causal;
+  p.scale = s->scale;
+  p.bhn = s->B * s->H * s->N;
+  return p;
+}
+
+int n_blocks(int64_t N, int rows) { return (int)((N + rows - 1) / rows); }
+
+int launch_status(cudaError_t e) { return e == cudaSuccess ? FBOB_OK : FBOB_ERR_CUDA; }
+
+// ---- the individual launches (arguments already validated)
+int run_pass1(const fbob_shape* s, const void* q, const void* k, const void* v, const void* o,
+              const float* lse, const void* dout, const void* gq, const void* gk,
+              const void* gv, void* q_bar, void* dout_bar, float* row_stats,
+              cudaStream_t st) {
+  EngineParams p = base_params(s);
+  const int64_t BH = s->B * s->H, N = s->N, d = s->d;
+  const void* stat[3] = {q, gq, dout};
+  const void* strm[4] = {k, gk, v, gv};
+  for (int t = 0; t < 3; ++t)
+    if (!make_map(&p.tm[t], stat[t], BH, N, d, BM)) return FBOB_ERR_CUDA;
+  for (int t = 0; t < 4; ++t)
+    if (!make_map(&p.tm[3 + t], strm[t], BH, N, d, BN)) return FBOB_ERR_CUDA;
+  p.o = static_cast<const __nv_bfloat16*>(o);
+  p.dout = static_cast<const __nv_bfloat16*>(dout);
+  p.lse = lse;
+  p.out0 = static_cast<__nv_bfloat16*>(q_bar);
+  p.out1 = static_cast<__nv_bfloat16*>(dout_bar);
+  p.vec_out = row_stats;
+  p.nblk = n_blocks(N, BM);
+  const int nb = p.nblk * p.BH * row_nsplit(RowOp::BobPass1, (int)d);
+  return launch_status(launch_row(RowOp::BobPass1, (int)d, p, nb, st));
+}
+
+int run_pass2(const fbob_shape* s, const void* q, const void* k, const void* v, const float* lse,
+              const void* dout, const void* gq, const void* gk, const void* gv,
+              const float* row_stats, void* k_bar, void* v_bar, cudaStream_t st) {
+  EngineParams p = base_params(s);
+  const int64_t BH = s->B * s->H, N = s->N, d = s->d;
+  const void* stat[4] = {k, v, gk, gv};
+  const void* strm[3] = {q, gq, dout};
+  for (int t = 0; t < 4; ++t)
+    if (!make_map(&p.tm[t], stat[t], BH, N, d, BM)) return FBOB_ERR_CUDA;
+  for (int t = 0; t < 3; ++t)
+    if (!make_map(&p.tm[4 + t], strm[t], BH, N, d, BN)) return FBOB_ERR_CUDA;
+  p.lse = lse;
+  p.vec_in = row_stats;
+  p.out0 = static_cast<__nv_bfloat16*>(k_bar);
+  p.out1 = static_cast<__nv_bfloat16*>(v_bar);
+  p.nblk = n_blocks(N, BM);
+  return launch_status(launch_col(ColOp::BobPass2, (int)d, p, p.nblk * p.BH, st));
+}
+
+}  // namespace
+}  // namespace fbob
+
+using namespace fbob;
+
+extern "C" {
+
+const char* fbob_status_string(int status) {
+  switch (status) {
+    case FBOB_OK: return "FBOB_OK";
+    case FBOB_ERR_INVALID_ARGUMENT: return "FBOB_ERR_INVALID_ARGUMENT";
+    case FBOB_ERR_UNSUPPORTED: return "FBOB_ERR_UNSUPPORTED";
+    case FBOB_ERR_CUDA: return "FBOB_ERR_CUDA";
+    case FBOB_ERR_DEVICE_TIMEOUT: return "FBOB_ERR_DEVICE_TIMEOUT";
+    case FBOB_ERR_DEVICE_FAULT: return "FBOB_ERR_DEVICE_FAULT";
+    default: return "FBOB_UNKNOWN_STATUS";
+  }
+}
+
+int fbob_launch_count(const char* entry) {
+  if (!entry) return -1;
+  static const char* names[5] = {"fwd", "bwd", "bob", "bob_pass1", "bob_pass2"};
+  for (int t = 0; t < 5; ++t)
+    if (std::strcmp(entry, names[t]) == 0) return g_launches[t].load();
+  return -1;
+}
+
+int fbob_attn_fwd(const fbob_shape* s, const void* q, const void* k, const void* v, void* o,
+                  float* lse, struct CUstream_st* stream) {
+  bool empty = false;
+  int rc = check_shape(s, &empty);
+  if (rc != FBOB_OK) return rc;
+  if (empty) {
+    g_launches[kEntFwd] = 0;
+    return FBOB_OK;
+  }
+  const int64_t mat = s->B * s->H * s->N * s->d * 2, vec = s->B * s->H * s->N * 4;
+  const void* in[3] = {q, k, v};
+  const int64_t inb[3] = {mat, mat, mat};
+  void* out[2] = {o, lse};
+  const int64_t outb[2] = {mat, vec};
+  rc = check_ptrs(in, inb, 3, out, outb, 2);
+  if (rc != FBOB_OK) return rc;
+  EngineParams p = base_params(s);
+  const int64_t BH = s->B * s->H;
+  if (!make_map(&p.tm[0], q, BH, s->N, s->d, BM) || !make_map(&p.tm[1], k, BH, s->N, s->d, BN) ||
+      !make_map(&p.tm[2], v, BH, s->N, s->d, BN))
+    return FBOB_ERR_CUDA;
+  p.out0 = static_cast<__nv_bfloat16*>(o);
+  p.vec_out = lse;
+  p.nblk = n_blocks(s->N, BM);
+  rc = launch_status(launch_row(RowOp::Fwd, (int)s->d, p, p.nblk * p.BH, stream));
+  if (rc == FBOB_OK) g_launches[kEntFwd] = 1;
+  return rc;
+}
+
+int fbob_attn_bwd(const fbob_shape* s, const void* q, const void* k, const void* v, const void* o,
+                  const float* lse, const void* dout, void* dq, void* dk, void* dv, float* dstat,
+                  struct CUstream_st* stream) {
+  bool empty = false;
+  int rc = check_shape(s, &empty);
+  if (rc != FBOB_OK) return rc;
+  if (empty) {
+    g_launches[kEntBwd] = 0;
+    return FBOB_OK;
+  }
+  const int64_t mat = s->B * s->H * s->N * s->d * 2, vec = s->B * s->H * s->N * 4;
+  const void* in[6] = {q, k, v, o, lse, dout};
+  const int64_t inb[6] = {mat, mat, mat, mat, vec, mat};
+  void* out[4] = {dq, dk, dv, dstat};
+  const int64_t outb[4] = {mat, mat, mat, vec};
+  rc = check_ptrs(in, inb, 6, out, outb, 4);
+  if (rc != FBOB_OK) return rc;
+  const int64_t BH = s->B * s->H, N = s->N, d = s->d;
+  // dQ and D: row-block pass (writes D, which the column pass reads)
+  EngineParams p = base_params(s);
+  if (!make_map(&p.tm[0], q, BH, N, d, BM) || !make_map(&p.tm[1], dout, BH, N, d, BM) ||
+      !make_map(&p.tm[2], k, BH, N, d, BN) || !make_map(&p.tm[3], v, BH, N, d, BN))
+    return FBOB_ERR_CUDA;
+  p.o = static_cast<const __nv_bfloat16*>(o);
+  p.dout = static_cast<const __nv_bfloat16*>(dout);
+  p.lse = lse;
+  p.out0 = static_cast<__nv_bfloat16*>(dq);
+  p.vec_out = dstat;
+  p.nblk = n_blocks(N, BM);
+  rc = launch_status(launch_row(RowOp::BwdDQ, (int)d, p, p.nblk * p.BH, stream));
+  if (rc != FBOB_OK) return rc;
+  // dK and dV: column-block pass
+  EngineParams c = base_params(s);
+  if (!make_map(&c.tm[0], k, BH, N, d, BM) || !make_map(&c.tm[1], v, BH, N, d, BM) ||
+      !make_map(&c.tm[2], q, BH, N, d, BN) || !make_map(&c.tm[3], dout, BH, N, d, BN))
+    return FBOB_ERR_CUDA;
+  c.lse = lse;
+  c.vec_in = dstat;
+  c.out0 = static_cast<__nv_bfloat16*>(dk);
+  c.out1 = static_cast<__nv_bfloat16*>(dv);
+  c.nblk = n_blocks(N, BM);
+  rc = launch_status(launch_col(ColOp::BwdDKDV, (int)d, c, c.nblk * c.BH, stream));
+  if (rc == FBOB_OK) g_launches[kEntBwd] = 2;
+  return rc;
+}
+
+int fbob_attn_bob_pass1(const fbob_shape* s, const void* q, const void* k, const void* v,
+                        const void* o, const float* lse, const void* dout, const void* gq,
+                        const void* gk, const void* gv, void* q_bar, void* dout_bar,
+                        float* row_stats, struct CUstream_st* stream) {
+  bool empty = false;
+  int rc = check_shape(s, &empty);
+  if (rc != FBOB_OK) return rc;
+  if (empty) {
+    g_launches[kEntPass1] = 0;
+    return FBOB_OK;
+  }
+  const int64_t mat = s->B * s->H * s->N * s->d * 2, vec = s->B * s->H * s->N * 4;
+  const void* in[9] = {q, k, v, o, lse, dout, gq, gk, gv};
+  const int64_t inb[9] = {mat, mat, mat, mat, vec, mat, mat, mat, mat};
+  void* out[3] = {q_bar, dout_bar, row_stats};
+  const int64_t outb[3] = {mat, mat, 3 * vec};
+  rc = check_ptrs(in, inb, 9, out, outb, 3);
+  if (rc != FBOB_OK) return rc;
+  rc = run_pass1(s, q, k, v, o, lse, dout, gq, gk, gv, q_bar, dout_bar, row_stats, stream);
+  if (rc == FBOB_OK) g_launches[kEntPass1] = 1;
+  return rc;
+}
+
+int fbob_attn_bob_pass2(const fbob_shape* s, const void* q, const void* k, const void* v,
+                        const float* lse, const void* dout, const void* gq, const void* gk,
+                        const void* gv, const float* row_stats, void* k_bar, void* v_bar,
+                        struct CUstream_st* stream) {
+  bool empty = false;
+  int rc = check_shape(s, &empty);
+  if (rc != FBOB_OK) return rc;
+  if (empty) {
+    g_launches[kEntPass2] = 0;
+    return FBOB_OK;
+  }
+  const int64_t mat = s->B * s->H * s->N * s->d * 2, vec = s->B * s->H * s->N * 4;
+  // row_stats is an input of pass 2; check it with the inputs
+  const void* in2[9] = {q, k, v, lse, dout, gq, gk, gv, row_stats};
+  const int64_t inb2[9] = {mat, mat, mat, vec, mat, mat, mat, mat, 3 * vec};
+  void* out[2] = {k_bar, v_bar};
+  const int64_t outb[2] = {mat, mat};
+  rc = check_ptrs(in2, inb2, 9, out, outb, 2);
+  if (rc != FBOB_OK) return rc;
+  rc = run_pass2(s, q, k, v, lse, dout, gq, gk, gv, row_stats, k_bar, v_bar, stream);
+  if (rc == FBOB_OK) g_launches[kEntPass2] = 1;
+  return rc;
+}
+
+int fbob_attn_bob(const fbob_shape* s, const void* q, const void* k, const void* v, const void* o,
+                  const float* lse, const void* dout, const void* gq, const void* gk,
+                  const void* gv, void* q_bar, void* k_bar, void* v_bar, void* dout_bar,
+                  float* row_stats, struct CUstream_st* stream) {
+  bool empty = false;
+  int rc = check_shape(s, &empty);
+  if (rc != FBOB_OK) return rc;
+  if (empty) {
+    g_launches[kEntBob] = 0;
+    return FBOB_OK;
+  }
+  const int64_t mat = s->B * s->H * s->N * s->d * 2, vec = s->B * s->H * s->N * 4;
+  const void* in[9] = {q, k, v, o, lse, dout, gq, gk, gv};
+  const int64_t inb[9] = {mat, mat, mat, mat, vec, mat, mat, mat, mat};
+  void* out[5] = {q_bar, k_bar, v_bar, dout_bar, row_stats};
+  const int64_t outb[5] = {mat, mat, mat, mat, 3 * vec};
+  rc = check_ptrs(in, inb, 9, out, outb, 5);
+  if (rc != FBOB_OK) return rc;
+  // Pass 1 (row blocks): Qtil, dOtil and the row scalars alpha, E, D.
+  rc = run_pass1(s, q, k, v, o, lse, dout, gq, gk, gv, q_bar, dout_bar, row_stats, stream);
+  if (rc != FBOB_OK) return rc;
+  // Pass 2 (column blocks): Ktil, Vtil from the saved row state.  Stream
+  // order is the only synchronisation between the passes.
+  rc = run_pass2(s, q, k, v, lse, dout, gq, gk, gv, row_stats, k_bar, v_bar, stream);
+  if (rc == FBOB_OK) g_launches[kEntBob] = 2;
+  return rc;
+}
+
+int fbob_device_status(struct CUstream_st* stream) {
+  cudaError_t e = cudaStreamSynchronize(stream);
+  if (e != cudaSuccess) return FBOB_ERR_DEVICE_FAULT;
+  uint32_t w1 = 0, w2 = 0;
+  if (take_row_error(&w1, stream) != cudaSuccess || take_col_error(&w2, stream) != cudaSuccess)
+    return FBOB_ERR_CUDA;
+  const uint32_t w = w1 | w2;
+  if (w & kDevErrTimeout) return FBOB_ERR_DEVICE_TIMEOUT;
+  if (w) return FBOB_ERR_DEVICE_FAULT;
+  return FBOB_OK;
+}
+
+}  // extern "C"

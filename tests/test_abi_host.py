@@ -1,0 +1,87 @@
+"""Host-only checks of the C ABI: the library builds, loads, exports every
+entry point include/fbob.h declares, and validates arguments before touching
+CUDA (so these run without a GPU)."""
+import ctypes
+
+import pytest
+
+import paper_2609_24089_gb300 as fbob
+
+
+@pytest.fixture(scope="module")
+def lib():
+    fbob.build()
+    return fbob.load()
+
+
+def test_exports_every_declared_symbol(lib):
+    names = fbob.header_symbols()
+    assert {"fbob_attn_fwd", "fbob_attn_bwd", "fbob_attn_bob", "fbob_attn_bob_pass1",
+            "fbob_attn_bob_pass2", "fbob_device_status", "fbob_status_string",
+            "fbob_launch_count"} <= set(names)
+    for n in names:
+        assert getattr(lib, n) is not None
+
+
+def test_status_strings(lib):
+    assert lib.fbob_status_string(0) == b"FBOB_OK"
+    assert lib.fbob_status_string(2) == b"FBOB_ERR_UNSUPPORTED"
+    assert lib.fbob_status_string(99) == b"FBOB_UNKNOWN_STATUS"
+
+
+# fake, 16-byte aligned, non-overlapping "device" addresses: validation never
+# dereferences them, and every call below fails or returns before any CUDA call
+BASE = 1 << 40
+STRIDE = 1 << 34
+
+
+def ptrs(n, misalign=None):
+    out = [BASE + t * STRIDE for t in range(n)]
+    if misalign is not None:
+        out[misalign] += 8
+    return [ctypes.c_void_p(p) for p in out]
+
+
+def bob(lib, shape, ps):
+    return lib.fbob_attn_bob(ctypes.byref(shape), *ps, None)
+
+
+def test_rejects_bad_shapes(lib):
+    S = fbob.make_shape
+    assert bob(lib, S(1, 1, 128, 32, 0.17, 0), ptrs(14)) == 2          # d unsupported
+    assert bob(lib, S(1, 1, 128, 256, 0.06, 1), ptrs(14)) == 2
+    assert bob(lib, S(1, 1, 128, 64, 0.0, 0), ptrs(14)) == 1           # scale <= 0
+    assert bob(lib, S(1, 1, 128, 64, float("nan"), 0), ptrs(14)) == 1
+    assert bob(lib, S(1, 1, 128, 64, float("inf"), 0), ptrs(14)) == 1
+    assert bob(lib, S(1, 1, 128, 64, 0.125, 2), ptrs(14)) == 1         # causal not 0/1
+    assert bob(lib, S(-1, 1, 128, 64, 0.125, 0), ptrs(14)) == 1
+    assert bob(lib, S(1, 1, (1 << 24) + 1, 64, 0.125, 0), ptrs(14)) == 1
+    assert lib.fbob_attn_bob(None, *ptrs(14), None) == 1               # null shape
+
+
+def test_empty_problems_launch_nothing(lib):
+    S = fbob.make_shape
+    for shp in (S(0, 4, 128, 64, 0.125, 0), S(2, 0, 128, 64, 0.125, 1), S(2, 4, 0, 128, 0.09, 0)):
+        assert bob(lib, shp, ptrs(14)) == 0
+        assert lib.fbob_launch_count(b"bob") == 0
+        assert lib.fbob_attn_fwd(ctypes.byref(shp), *ptrs(5), None) == 0
+        assert lib.fbob_attn_bwd(ctypes.byref(shp), *ptrs(10), None) == 0
+
+
+def test_rejects_null_misaligned_and_overlapping_pointers(lib):
+    S = fbob.make_shape(1, 2, 100, 64, 0.125, 1)
+    for t in range(14):
+        ps = ptrs(14)
+        ps[t] = ctypes.c_void_p(0)
+        assert bob(lib, S, ps) == 1, t
+        assert bob(lib, S, ptrs(14, misalign=t)) == 1, t
+    ps = ptrs(14)
+    ps[10] = ps[0]                      # k_bar aliases q
+    assert bob(lib, S, ps) == 1
+    ps = ptrs(14)
+    ps[13] = ctypes.c_void_p(ps[12].value + 64)   # row_stats overlaps dout_bar
+    assert bob(lib, S, ps) == 1
+    # pass 2 reads row_stats: it may not alias its outputs
+    ps = ptrs(11)          # q k v lse dout gq gk gv row_stats k_bar v_bar
+    ps[9] = ps[8]
+    assert lib.fbob_attn_bob_pass2(ctypes.byref(S), *ps, None) == 1

@@ -1,0 +1,134 @@
+"""Parity on the five synthetic workloads, run on the GPU at full size in the
+launch configuration the benchmark times.
+
+  n128_d64               full oracle; O and L from the oracle's forward
+  n4k_d64                full oracle on a seeded set of heads (all heads: FBOB_SLOW=1)
+  n16k_d128_causal       full oracle on two seeded heads
+  n64k_d128_causal_peaky oracle on sampled rows (row-owned outputs) and on the
+                         causal tail: key columns >= N - 256 are complete once
+                         rows >= N - 256 are summed
+  n256k_d64              oracle on sampled rows; Ktil, Vtil through identities that
+                         hold at any size (column sums vanish, Euler identities)
+"""
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+import paper_2609_24089_gb300 as fbob
+from paper_2609_24089_gb300 import synth
+from tests import gpu_util as G
+
+pytestmark = pytest.mark.gpu
+
+ROWS_OUT = ("qbar", "dobar", "alpha", "E", "D")
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    fbob.build()
+    fbob.load()
+
+
+def sample_rows(N, seed, n=40):
+    rng = np.random.default_rng(seed)
+    fixed = [0, 1, 2, 63, 64, 127, 128, 129, N // 2, N - 129, N - 128, N - 2, N - 1]
+    rows = set(r for r in fixed if 0 <= r < N)
+    rows.update(rng.integers(0, N, n).tolist())
+    return np.array(sorted(rows), dtype=np.int64)
+
+
+def check_rows(r, refs, heads, H, rows):
+    for hh, ref in zip(heads, refs):
+        for name in ROWS_OUT:
+            got = G.flat(r[name], hh, H)[rows]
+            G.check(f"{name}[head {hh}]", got, ref[name])
+
+
+def test_n128_d64_full_with_oracle_forward():
+    w = synth.WORKLOADS["n128_d64"]
+    bits = synth.workload_inputs(w)
+    r = G.run_bob(bits, w.scale, w.causal, o_l=G.oracle_o_l(bits, w.scale, w.causal))
+    assert r["status"] == 0
+    ref = oracle.bob(*(G.f64(bits[n]) for n in synth.NAMES), w.scale, w.causal)
+    for name, x in zip(("qbar", "kbar", "vbar", "dobar", "alpha", "E", "D"), ref):
+        G.check(name, r[name], x)
+
+
+def test_n4k_d64_heads():
+    w = synth.WORKLOADS["n4k_d64"]
+    bits = synth.workload_inputs(w)
+    r = G.run_bob(bits, w.scale, w.causal)
+    assert r["status"] == 0
+    BH = w.B * w.H
+    heads = list(range(BH)) if os.environ.get("FBOB_SLOW") == "1" else [0, 21, 42, 63]
+    refs = G.oracle_bob_heads(bits, w.scale, w.causal, heads)
+    for hh, ref in zip(heads, refs):
+        for name in ("qbar", "kbar", "vbar", "dobar", "alpha", "E", "D"):
+            G.check(f"{name}[head {hh}]", G.flat(r[name], hh, w.H), ref[name])
+
+
+def test_n16k_d128_causal_two_heads():
+    w = synth.WORKLOADS["n16k_d128_causal"]
+    bits = synth.workload_inputs(w)
+    r = G.run_bob(bits, w.scale, w.causal)
+    assert r["status"] == 0
+    heads = [0, w.B * w.H - 1]
+    refs = G.oracle_bob_heads(bits, w.scale, w.causal, heads)
+    for hh, ref in zip(heads, refs):
+        for name in ("qbar", "kbar", "vbar", "dobar", "alpha", "E", "D"):
+            G.check(f"{name}[head {hh}]", G.flat(r[name], hh, w.H), ref[name])
+
+
+def test_n64k_d128_causal_peaky_rows_and_tail():
+    w = synth.WORKLOADS["n64k_d128_causal_peaky"]
+    bits = synth.workload_inputs(w)
+    r = G.run_bob(bits, w.scale, w.causal)
+    assert r["status"] == 0
+    N = w.N
+    heads = [3]
+    rows = sample_rows(N, 64)
+    check_rows(r, G.oracle_bob_heads(bits, w.scale, w.causal, heads, rows=rows), heads, w.H, rows)
+    t0 = N - 256
+    tail = G.oracle_bob_heads(bits, w.scale, w.causal, heads, rows=np.arange(t0, N), cols=(t0, N))
+    for hh, ref in zip(heads, tail):
+        G.check("kbar[tail]", G.flat(r["kbar"], hh, w.H)[t0:], ref["kbar"])
+        G.check("vbar[tail]", G.flat(r["vbar"], hh, w.H)[t0:], ref["vbar"])
+
+
+def test_n256k_d64_rows_and_identities():
+    w = synth.WORKLOADS["n256k_d64"]
+    bits = synth.workload_inputs(w)
+    t = G.torch()
+    q, k, v, do, gq, gk, gv = (G.dev(bits[n]) for n in synth.NAMES)
+    o, lse = fbob.attn_fwd(q, k, v, w.scale, w.causal)
+    qb, kb, vb, dob, rs = fbob.attn_bob(q, k, v, o, lse, do, gq, gk, gv, w.scale, w.causal)
+    dq, dk, dv, _ = fbob.attn_bwd(q, k, v, o, lse, do, w.scale, w.causal)
+    assert fbob.fbob_device_status() == 0
+    H = w.H
+    heads = [1]
+    rows = sample_rows(w.N, 256)
+    r = {"qbar": G.host(qb), "dobar": G.host(dob), "alpha": rs[0].cpu().numpy(),
+         "E": rs[1].cpu().numpy(), "D": rs[2].cpu().numpy()}
+    check_rows(r, G.oracle_bob_heads(bits, w.scale, w.causal, heads, rows=rows), heads, H, rows)
+    # identities, per head, in fp64 over the bf16 outputs
+    for hh in range(w.B * H):
+        b, h = divmod(hh, H)
+        X = {n: G.f64(bits[n][b, h]) for n in synth.NAMES}
+        Kt, Vt = G.host(kb[b, h]), G.host(vb[b, h])
+        Qt, dOt = G.host(qb[b, h]), G.host(dob[b, h])
+        dQ, dK, dV = G.host(dq[b, h]), G.host(dk[b, h]), G.host(dv[b, h])
+        for name, M in (("kbar", Kt), ("vbar", Vt)):   # shift invariance of Phi
+            colsum = np.abs(M.sum(0))
+            assert np.all(colsum <= 3e-2 * np.linalg.norm(M, axis=0)), name
+        a = float((dQ * X["gq"]).sum())
+        bk = float((dK * X["gk"]).sum())
+        c = float((dV * X["gv"]).sum())
+        phi = a + bk + c
+        # Euler identities (degree 1 in dO; V -> sV; Q -> sQ, K -> K/s)
+        sc = abs(a) + abs(bk) + abs(c)
+        assert abs(float((dOt * X["dout"]).sum()) - phi) <= 2e-2 * sc
+        assert abs(float((Vt * X["v"]).sum()) - (a + bk)) <= 2e-2 * (abs(a) + abs(bk))
+        lhs = float((Qt * X["q"]).sum()) - float((Kt * X["k"]).sum())
+        assert abs(lhs - (bk - a)) <= 2e-2 * (abs(a) + abs(bk))

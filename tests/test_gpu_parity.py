@@ -1,0 +1,164 @@
+"""GPU parity against the fp64 oracle at sizes the oracle finishes in seconds:
+several tiles, ragged tails, both masks, both head dims, every kernel alone
+and the whole pipeline.  All calls go through the C ABI."""
+import numpy as np
+import pytest
+
+import oracle
+import paper_2609_24089_gb300 as fbob
+from paper_2609_24089_gb300 import synth
+from tests import gpu_util as G
+
+pytestmark = pytest.mark.gpu
+
+SHAPES = [  # B, H, N, d, causal
+    (1, 1, 128, 64, False),
+    (1, 2, 17, 64, True),
+    (2, 1, 100, 128, False),
+    (1, 1, 129, 64, True),
+    (1, 2, 300, 128, True),
+    (1, 3, 257, 64, False),
+    (1, 1, 2, 64, False),
+    (1, 1, 3, 128, True),
+    (2, 2, 384, 128, False),
+    (1, 2, 520, 64, True),
+]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    fbob.build()
+    fbob.load()
+
+
+def ids(s):
+    return "B{}H{}N{}d{}{}".format(*s[:4], "c" if s[4] else "")
+
+
+@pytest.mark.parametrize("shape", SHAPES, ids=ids)
+def test_forward_and_first_backward(shape):
+    B, H, N, d, causal = shape
+    bits = G.inputs(B, H, N, d, seed=N + d)
+    scale = 1 / np.sqrt(d)
+    q, k, v, do = (G.dev(bits[n]) for n in ("q", "k", "v", "dout"))
+    o, lse = fbob.attn_fwd(q, k, v, scale, causal)
+    dq, dk, dv, dstat = fbob.attn_bwd(q, k, v, o, lse, do, scale, causal)
+    assert fbob.fbob_device_status() == 0
+    X = [G.f64(bits[n]) for n in ("q", "k", "v", "dout")]
+    O, L = oracle.fwd(*X[:3], scale, causal)
+    G.check("O", G.host(o), O)
+    assert np.abs(lse.cpu().numpy() - L).max() <= 1e-3
+    dQ, dK, dV, Dv = oracle.bwd(*X, scale, causal)
+    G.check("dQ", G.host(dq), dQ)
+    G.check("dK", G.host(dk), dK)
+    G.check("dV", G.host(dv), dV)
+    G.check("D", dstat.cpu().numpy(), Dv)
+
+
+@pytest.mark.parametrize("shape", SHAPES, ids=ids)
+def test_bob_end_to_end(shape):
+    B, H, N, d, causal = shape
+    bits = G.inputs(B, H, N, d, seed=7 * N + d)
+    scale = 1 / np.sqrt(d)
+    r = G.run_bob(bits, scale, causal)
+    assert r["status"] == 0
+    ref = oracle.bob(*(G.f64(bits[n]) for n in synth.NAMES), scale, causal)
+    for name, x in zip(("qbar", "kbar", "vbar", "dobar", "alpha", "E", "D"), ref):
+        G.check(name, r[name], x)
+
+
+@pytest.mark.parametrize("shape", [(1, 2, 300, 64, True), (2, 1, 200, 128, False)], ids=ids)
+def test_pass2_alone_on_oracle_row_state(shape):
+    """Algorithm 2's second loop fed the oracle's L, D, alpha, E."""
+    B, H, N, d, causal = shape
+    bits = G.inputs(B, H, N, d, seed=3)
+    scale = 1 / np.sqrt(d)
+    X = [G.f64(bits[n]) for n in synth.NAMES]
+    qb, kb, vb, dob, al, E, D = oracle.bob(*X, scale, causal)
+    _, L = oracle.fwd(*X[:3], scale, causal)
+    rs = np.stack([al, E, D]).astype(np.float32)
+    t = G.torch()
+    q, k, v, do, gq, gk, gv = (G.dev(bits[n]) for n in synth.NAMES)
+    k_bar, v_bar = t.empty_like(k), t.empty_like(v)
+    shp = fbob.make_shape(B, H, N, d, scale, causal)
+    fbob.fbob_attn_bob_pass2(shp, q, k, v, G.dev_f32(L), do, gq, gk, gv, G.dev_f32(rs),
+                             k_bar, v_bar)
+    assert fbob.fbob_device_status() == 0
+    G.check("kbar", G.host(k_bar), kb)
+    G.check("vbar", G.host(v_bar), vb)
+
+
+@pytest.mark.parametrize("shape", [(1, 2, 300, 64, True), (2, 1, 200, 128, False)], ids=ids)
+def test_pass1_alone(shape):
+    """Algorithm 2's first loop: Qtil, dOtil and the row scalars alpha, E, D."""
+    B, H, N, d, causal = shape
+    bits = G.inputs(B, H, N, d, seed=4)
+    scale = 1 / np.sqrt(d)
+    X = [G.f64(bits[n]) for n in synth.NAMES]
+    qb, kb, vb, dob, al, E, D = oracle.bob(*X, scale, causal)
+    o_bits, L = G.oracle_o_l(bits, scale, causal)
+    t = G.torch()
+    q, k, v, do, gq, gk, gv = (G.dev(bits[n]) for n in synth.NAMES)
+    q_bar, dout_bar = t.empty_like(q), t.empty_like(q)
+    rs = t.empty((3, B, H, N), dtype=t.float32, device="cuda")
+    shp = fbob.make_shape(B, H, N, d, scale, causal)
+    fbob.fbob_attn_bob_pass1(shp, q, k, v, G.dev(o_bits), G.dev_f32(L), do, gq, gk, gv,
+                             q_bar, dout_bar, rs)
+    assert fbob.fbob_device_status() == 0
+    rs = rs.cpu().numpy().astype(np.float64)
+    G.check("alpha", rs[0], al)
+    G.check("E", rs[1], E)
+    G.check("D", rs[2], D)
+    G.check("qbar", G.host(q_bar), qb)
+    G.check("dobar", G.host(dout_bar), dob)
+
+
+def test_runs_are_bitwise_identical():
+    bits = G.inputs(1, 4, 777, 128, seed=9)
+    scale = 1 / np.sqrt(128)
+    a = G.run_bob(bits, scale, True)
+    b = G.run_bob(bits, scale, True)
+    for n in ("qbar", "kbar", "vbar", "dobar", "alpha", "E", "D"):
+        assert np.array_equal(a[n], b[n]), n
+
+
+def test_lemma_d2_embedding_on_gpu():
+    """V = dO = U_Q = U_K = 0, U_V = W: dOtil = softmax(tau Q K^T) W exactly
+    (Lemma D.2) and the other outputs vanish."""
+    B, H, N, d = 1, 2, 200, 64
+    bits = G.inputs(B, H, N, d, seed=21)
+    z = np.zeros_like(bits["q"])
+    for n in ("v", "dout", "gq", "gk"):
+        bits[n] = z
+    scale = 1 / np.sqrt(d)
+    r = G.run_bob(bits, scale, True)
+    O, _ = oracle.fwd(G.f64(bits["q"]), G.f64(bits["k"]), G.f64(bits["gv"]), scale, True)
+    G.check("dobar", r["dobar"], O)
+    for n in ("qbar", "kbar", "vbar"):
+        assert np.abs(r[n]).max() == 0.0, n
+
+
+@pytest.mark.parametrize("d,causal", [(64, False), (128, True)])
+def test_single_key_degenerate(d, causal):
+    """N = 1: P = 1, so Qtil = Ktil = Vtil = 0 and dOtil = U_V exactly.  The
+    fused form Qtil = tau (Omega - alpha R - E B) cancels to zero only up to
+    the bf16 rounding of its operand tiles: with N = 1 it equals
+    tau [(bf16(C) - C) - F (bf16(dP) - dP)] k, so |Qtil| is bounded by
+    tau 2^-8 (|C| + |F dP|) max|k| (bf16 relative rounding <= 2^-9, factor 2
+    of margin).  Ktil and Vtil cancel in fp32 (alpha and E are fp32)."""
+    B, H, N = 1, 3, 1
+    bits = G.inputs(B, H, N, d, seed=5 + d)
+    scale = 1 / np.sqrt(d)
+    r = G.run_bob(bits, scale, causal)
+    assert r["status"] == 0
+    X = {n: G.f64(bits[n]) for n in synth.NAMES}
+    for h in range(H):
+        q, k, v, do, uq, uk, uv = (X[n][0, h, 0] for n in synth.NAMES)
+        C = do @ uv
+        F = scale * (uq @ k + q @ uk)
+        dP = do @ v
+        bound = scale * 2.0 ** -8 * (abs(C) + abs(F * dP)) * np.abs(k).max()
+        assert np.abs(r["qbar"][0, h, 0]).max() <= bound, h
+        G.check("dobar", r["dobar"][0, h, 0], uv)
+    assert np.abs(r["kbar"]).max() <= 1e-4 * scale * np.abs(X["q"]).max() * np.abs(X["gv"]).max() * d
+    assert np.abs(r["vbar"]).max() <= 1e-4 * np.abs(X["dout"]).max() * np.abs(X["gq"]).max() * d
