@@ -1,0 +1,382 @@
+"""Benchmark of exact attention backward-over-backward (BoB) on GB300.
+
+One step = one BoB of the whole workload (Pass 1 + Pass 2 of Algorithm 1)
+on inputs already resident in HBM.  Throughput is reported in TFLOP/s by the
+fixed contraction-count formula
+
+    FLOPs = 2 * 19 * B*H * N^2 * d * rho,    rho = 1 (no mask) or 1/2 (causal),
+
+19 being the N x N x d contractions of Algorithm 2 (11 in Pass 1, 8 in Pass 2).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl reference]
+
+Multi-GPU (torchrun): every rank runs an independent replica of the workload
+(no data-path collective); the value is the sum over ranks of the work
+divided by the slowest rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2609_24089_gb300 import synth  # noqa: E402
+
+METRIC = "BoB TFLOP/s and tensor-pipe % of bf16 peak at N=16K-262K; peak HBM bytes"
+DEFAULT_WORKLOAD = "n16k_d128_causal"
+CONTRACTIONS = {"pass1": 11, "pass2": 8}
+KERNEL_NAMES = {"pass1": "row_engine<BobPass1>", "pass2": "col_engine<BobPass2>"}
+CSRC = os.path.join(ROOT, "paper_2609_24089_gb300", "csrc")
+
+
+def bob_flops(w, contractions=19):
+    rho = 0.5 if w.causal else 1.0
+    return 2.0 * contractions * w.B * w.H * float(w.N) ** 2 * w.d * rho
+
+
+def valid_pairs_rows(w, rows):
+    return float(sum(min(r + 1, w.N) if w.causal else w.N for r in rows))
+
+
+def source_hash() -> str:
+    h = hashlib.sha256()
+    for f in sorted(os.listdir(CSRC)):
+        with open(os.path.join(CSRC, f), "rb") as fh:
+            h.update(f.encode() + fh.read())
+    return h.hexdigest()[:16]
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as fh:
+            j = json.load(fh)
+        return {"bf16": j["bf16_tflops"], "bf16_sustained": j["bf16_tflops_sustained"],
+                "hbm": j["hbm_gbs"], "source": "measured"}
+    return {"bf16": 1900.0, "bf16_sustained": 1700.0, "hbm": 6800.0, "source": "fallback"}
+
+
+def ncu_traffic(kernel_key, workload):
+    """Per-launch DRAM bytes from the committed ncu summary, if it was taken on
+    the current kernel source (else None)."""
+    p = os.path.join(ROOT, "profiles", "traffic.txt")
+    if not os.path.exists(p):
+        return None
+    cur = source_hash()
+    with open(p) as fh:
+        for line in fh:
+            f = line.split()
+            if len(f) >= 4 and not line.startswith("#") and f[0] == kernel_key and f[1] == workload:
+                return float(f[2]) if f[3] == cur else None
+    return None
+
+
+# ----------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        self.out = ""
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                self.out, _ = self.proc.communicate()
+
+    def summary(self):
+        rows = [r.split(",") for r in (self.out or "").strip().splitlines() if r.count(",") >= 7]
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        sm, mx, reasons = [], [], set()
+        for r in rows:
+            try:
+                sm.append(float(r[0]))
+                mx.append(float(r[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, r[4:8]):
+                if v.strip().lower().startswith("active"):
+                    reasons.add(n)
+        under_load = [s for s in sm if s > 0.5 * max(mx or [1])] or sm
+        return {"sm_mhz": statistics.median(under_load) if under_load else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ----------------------------------------------------------------- oracle
+def oracle_sample(w, bits_head, target_s, seed=0):
+    """Time the fp64 oracle on a bounded, evenly spread sample of query rows of
+    one head (their row-owned outputs plus their contributions to every
+    column-owned sum).  Returns (fixed-formula FLOPs of the sample, seconds,
+    description)."""
+    import oracle
+    X = [synth.to_f64(bits_head[n]) for n in synth.NAMES]
+    rows_probe = np.linspace(0, w.N - 1, 16).astype(np.int64)
+    t0 = time.perf_counter()
+    oracle.bob_head(*X, w.scale, w.causal, rows=rows_probe, cols=(0, w.N))
+    dt = time.perf_counter() - t0
+    n = int(max(16, min(w.N, 16 * target_s / max(dt, 1e-6))))
+    rows = np.unique(np.linspace(0, w.N - 1, n).astype(np.int64))
+    t0 = time.perf_counter()
+    oracle.bob_head(*X, w.scale, w.causal, rows=rows, cols=(0, w.N))
+    dt = time.perf_counter() - t0
+    flops = 2.0 * 19 * valid_pairs_rows(w, rows) * w.d
+    return flops, dt, f"{len(rows)} evenly spaced query rows of head 0 (of {w.N}), all key columns"
+
+
+def cores():
+    return len(os.sched_getaffinity(0))
+
+
+# ----------------------------------------------------------------- reference arm
+def run_reference(args, w):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    import oracle
+    oracle.build()
+    bits = synth.workload_inputs(w, heads=[0])
+    bits = {n: b[0, 0] for n, b in bits.items()}
+    per = []
+    for s in range(args.warmup + args.steps):
+        fl, dt, desc = oracle_sample(w, bits, target_s=args.ref_step_s)
+        if s >= args.warmup:
+            per.append((fl, dt))
+    fl = sum(f for f, _ in per)
+    dt = sum(t for _, t in per)
+    val = fl / dt / 1e12
+    line = {"impl": "reference", "metric": METRIC, "value": val, "unit": "TFLOP/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 * dt / len(per), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": w.name, "B": w.B, "H": w.H, "N": w.N, "d": w.d,
+                       "causal": w.causal},
+            "cpu_baseline": {"value": val, "unit": "TFLOP/s", "cores": cores(), "kind": "oracle",
+                             "sample": desc + " per step"},
+            "e2e": {"value": val, "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ----------------------------------------------------------------- GPU arm
+def run_gpu(args, w):
+    import torch
+    import torch.distributed as dist
+
+    import paper_2609_24089_gb300 as fbob
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    fbob.build()
+    fbob.load()
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    bits = synth.workload_inputs(w)
+    dev = {n: torch.from_numpy(bits[n].view(np.int16)).view(torch.bfloat16).cuda()
+           for n in synth.NAMES}
+    q, k, v, do, gq, gk, gv = (dev[n] for n in synth.NAMES)
+    o, lse = fbob.attn_fwd(q, k, v, w.scale, w.causal)
+    shp = fbob.make_shape(w.B, w.H, w.N, w.d, w.scale, w.causal)
+    outs = [torch.empty_like(q) for _ in range(4)]
+    rs = torch.empty((3, w.B, w.H, w.N), dtype=torch.float32, device="cuda")
+    torch.cuda.synchronize()
+    stream = torch.cuda.current_stream()
+
+    def step():
+        fbob.fbob_attn_bob(shp, q, k, v, o, lse, do, gq, gk, gv, *outs, rs)
+
+    # peak HBM of one call: the library allocates nothing, so the footprint is
+    # the caller's tensors (inputs, O, L, outputs, row_stats)
+    torch.cuda.reset_peak_memory_stats()
+    base = torch.cuda.memory_allocated()
+    step()
+    torch.cuda.synchronize()
+    call_delta = torch.cuda.max_memory_allocated() - base
+    footprint = sum(t.numel() * t.element_size()
+                    for t in (q, k, v, do, gq, gk, gv, o, lse, *outs, rs))
+
+    for _ in range(args.warmup):
+        step()
+    if fbob.fbob_device_status() != 0:
+        raise RuntimeError("device status not OK after warm-up")
+
+    # ---- timed region: K steps, each as its two launches with events between
+    K = args.steps
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier()
+    with ClockSampler(local) as clk:
+        start.record(stream)
+        for s in range(K):
+            ev[s][0].record(stream)
+            fbob.fbob_attn_bob_pass1(shp, q, k, v, o, lse, do, gq, gk, gv, outs[0], outs[3], rs)
+            ev[s][1].record(stream)
+            fbob.fbob_attn_bob_pass2(shp, q, k, v, lse, do, gq, gk, gv, rs, outs[1], outs[2])
+            ev[s][2].record(stream)
+        stop.record(stream)
+        barrier()
+    status = fbob.fbob_device_status()
+    if status != 0:
+        raise RuntimeError(f"device status {status} in timed region")
+    ms = start.elapsed_time(stop)
+    t1 = [e[0].elapsed_time(e[1]) for e in ev]
+    t2 = [e[1].elapsed_time(e[2]) for e in ev]
+    ms_t = torch.tensor([ms], device="cuda")
+    if world > 1:
+        dist.all_reduce(ms_t, op=dist.ReduceOp.MAX)
+    ms_max = float(ms_t.item())
+    flops = bob_flops(w)
+    value = world * flops * K / (ms_max * 1e-3) / 1e12
+
+    # ---- end to end through the public call with host buffers
+    pin = {n: torch.from_numpy(bits[n].view(np.int16)).view(torch.bfloat16).pin_memory()
+           for n in synth.NAMES}
+    o_h, lse_h = o.cpu().pin_memory(), lse.cpu().pin_memory()
+    res_h = [torch.empty(q.shape, dtype=torch.bfloat16).pin_memory() for _ in range(4)]
+    rs_h = torch.empty(rs.shape, dtype=torch.float32).pin_memory()
+    h2d = sum(t.numel() * t.element_size() for t in (*pin.values(), o_h, lse_h))
+    d2h = sum(t.numel() * t.element_size() for t in (*res_h, rs_h))
+    e2e_bufs = {n: torch.empty_like(dev[n]) for n in synth.NAMES}
+    o_d, lse_d = torch.empty_like(o), torch.empty_like(lse)
+
+    def e2e_step():
+        for n in synth.NAMES:
+            e2e_bufs[n].copy_(pin[n], non_blocking=True)
+        o_d.copy_(o_h, non_blocking=True)
+        lse_d.copy_(lse_h, non_blocking=True)
+        fbob.fbob_attn_bob(shp, e2e_bufs["q"], e2e_bufs["k"], e2e_bufs["v"], o_d, lse_d,
+                           e2e_bufs["dout"], e2e_bufs["gq"], e2e_bufs["gk"], e2e_bufs["gv"],
+                           *outs, rs)
+        for hbuf, dbuf in zip(res_h, outs):
+            hbuf.copy_(dbuf, non_blocking=True)
+        rs_h.copy_(rs, non_blocking=True)
+
+    for _ in range(max(1, args.warmup)):
+        e2e_step()
+    barrier()
+    es, ee = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    es.record(stream)
+    for _ in range(K):
+        e2e_step()
+    ee.record(stream)
+    barrier()
+    e2e_ms = es.elapsed_time(ee)
+    e_t = torch.tensor([e2e_ms], device="cuda")
+    if world > 1:
+        dist.all_reduce(e_t, op=dist.ReduceOp.MAX)
+    e2e_val = world * flops * K / (float(e_t.item()) * 1e-3) / 1e12
+
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return
+
+    peaks = measured_peaks()
+    a1, a2 = sum(t1) / K, sum(t2) / K
+    dom = "pass1" if a1 >= a2 else "pass2"
+    dur = a1 if dom == "pass1" else a2
+    dflops = bob_flops(w, CONTRACTIONS[dom])
+    achieved = dflops / (dur * 1e-3) / 1e12
+    peak = peaks["bf16_sustained"]
+    roofline = {"bound": "tensor", "kernel": KERNEL_NAMES[dom], "achieved": achieved,
+                "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
+                "peak_kind": f"bf16 sustained ({peaks['source']})",
+                "traffic": ncu_traffic(dom, w.name),
+                "launch_ms": dur, "share_of_step": dur / (a1 + a2),
+                "other_kernel_ms": a2 if dom == "pass1" else a1}
+    cpu = None
+    if world == 1 and not args.no_cpu_baseline:
+        bits0 = {n: b[0, 0] for n, b in bits.items()}
+        fl, dt, desc = oracle_sample(w, bits0, target_s=args.cpu_s)
+        cpu = {"value": fl / dt / 1e12, "unit": "TFLOP/s", "cores": cores(), "kind": "oracle",
+               "sample": desc, "seconds": dt}
+    line = {
+        "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": K,
+        "warmup": args.warmup, "ms_per_step": ms_max / K, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": w.name, "B": w.B, "H": w.H, "N": w.N, "d": w.d,
+                   "causal": w.causal, "seed": w.seed,
+                   "l2": "no flush: inputs (%.2f GB) exceed the 129 MB L2" % (footprint / 1e9),
+                   "parallelism": "replicas" if world > 1 else "single GPU",
+                   "flop_formula": "2*19*B*H*N^2*d*(1/2 if causal)"},
+        "frac_of_bf16_peak": value / world / peak,
+        "roofline": roofline,
+        "cpu_baseline": cpu,
+        "e2e": {"value": e2e_val, "unit": "TFLOP/s", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "ms_per_step": float(e_t.item()) / K},
+        "gpu_launches": 2 * K,
+        "clocks": clk.summary(),
+        "peak_hbm_bytes": footprint,
+        "call_alloc_bytes": call_delta,
+        "pass_ms": {"pass1": a1, "pass2": a2},
+    }
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(synth.WORKLOADS))
+    ap.add_argument("--impl", default="fbob", choices=["fbob", "reference"])
+    ap.add_argument("--cpu-s", type=float, default=15.0, help="target seconds of the CPU baseline")
+    ap.add_argument("--ref-step-s", type=float, default=5.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--bh", default=None,
+                    help="B,H override (smaller profiling captures of the same kernels)")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)  # at least 3 untimed warm-up steps
+    w = synth.WORKLOADS[args.workload]
+    if args.bh:
+        import dataclasses
+        B, H = (int(x) for x in args.bh.split(","))
+        w = dataclasses.replace(w, B=B, H=H, name=f"{w.name}_B{B}H{H}")
+    if args.impl == "reference":
+        run_reference(args, w)
+    else:
+        run_gpu(args, w)
+
+
+if __name__ == "__main__":
+    main()
