@@ -3,29 +3,40 @@
 //
 // Two engines share one schedule skeleton:
 //   * row engine: a CTA owns BM = 128 query rows (TMEM lanes) and streams key
-//     blocks of BN = 64 rows.  Used by the forward (eq. 1), the dQ half of the
+//     tiles of BN = 64 rows.  Used by the forward (eq. 1), the dQ half of the
 //     first backward (eqs. 2-3) and BoB Pass 1 (Alg. 2, first loop).
-//   * column engine: a CTA owns BM = 128 key rows and streams query blocks of
+//   * column engine: a CTA owns BM = 128 key rows and streams query tiles of
 //     BN = 64 rows, computing transposed tiles (key rows on lanes).  Used by
 //     the dK/dV half of the first backward and BoB Pass 2 (Alg. 2, second loop).
 //
-// Roles (320 threads):
+// Roles (352 threads):
 //   warps 0-7  elementwise: two warpgroups; warp w reads TMEM lanes
-//              32*(w%4) .. +31, one stationary row per thread.  Each 64-column
-//              tile is processed as 4 K-steps of 16 columns, warpgroup g taking
-//              K-steps 2h+g of chunk h = 0, 1.
+//              32*(w%4) .. +31, one stationary row per thread.  Warpgroup g
+//              takes columns 16g .. 16g+15 of every 32-column half tile.
 //   warp 8     TMA producer: stationary tiles once, then a ring of NSTAGES
 //              stream stages (mbarrier full/empty pairs).  In the column engine
 //              it also stages the streamed rows' fp32 row vectors in shared memory.
-//   warp 9     TMEM allocator and MMA issuer (one lane).
+//   warps 9,10 MMA issuers X and Y (one lane each; warp 9 also allocates
+//              TMEM).  A single thread issues at most one tcgen05.mma about
+//              every 53 cycles, so the tile's MMAs are split between two
+//              issuers by tensor-memory ownership: X owns stage-A columns
+//              0..63 of each half region, Y columns 64..127, and each reads
+//              operand tiles only inside its own columns.
 //
-// Per streamed tile: stage A (scores and friends, fp32 in TMEM, A and B from
+// Half-tile pipeline.  Every streamed tile is split into two halves of 32
+// rows, each with its own stage-A region of tensor memory (128 columns at
+// kColA + 128 h).  Per half: stage A (scores and friends, fp32, A and B from
 // shared memory) -> elementwise (TMEM -> registers -> bf16 operand tiles
-// written back into TMEM over stage-A columns already consumed) -> stage B
-// (accumulators += bf16 tile (TMEM) x streamed tile (shared memory,
-// MN-major)).  Stage B of chunk 0 runs while the elementwise warps work on
-// chunk 1.  Tensor-memory map (512 columns): accumulators at 0..255,
-// stage-A tiles at 256..511.
+// written back into the columns of that region already read) -> stage B
+// (accumulators += bf16 tile (TMEM) x streamed half tile (shared memory,
+// MN-major)).  Each issuer runs  B_0(t), A_0(t+1), B_1(t), A_1(t+1), ...
+// so the tensor pipe works on one half while the elementwise warps work on the
+// other.  Accumulators live at TMEM columns 0..255.
+//
+// Shared memory: stationary tensors as 128-row x 64-column swizzled boxes;
+// each stream stage as 32-row x 64-column chunks ordered (box, half, tensor),
+// so that two tensors streamed side by side (K and U_K, V and U_V, Q and U_Q)
+// form one 64-row operand of a fused N = 64 stage-A MMA.
 //
 // Every wait is bounded (tc_ptx.cuh); on expiry the CTA records a timeout in
 // the device error word, drains its own asynchronous work and exits.
@@ -41,7 +52,7 @@ struct Misc {
   uint64_t bar_stat;
   uint64_t bar_full[4];
   uint64_t bar_empty[4];
-  uint64_t bar_sa;
+  uint64_t bar_sa[2];
   uint64_t bar_ew[2];
   uint64_t bar_acc;
   uint32_t tmem_base;
@@ -50,6 +61,12 @@ struct Misc {
 
 __device__ __forceinline__ uint32_t lane_base_addr(uint32_t tmem_base, int warp) {
   return tmem_base + ((uint32_t)(32 * (warp & 3)) << 16);
+}
+
+// Offset of streamed tensor t, half h, 64-column box b inside a stream stage.
+template <int NSTREAM>
+__device__ __forceinline__ uint32_t chunk_off(int t, int h, int b) {
+  return (uint32_t)(((b * 2 + h) * NSTREAM + t) * kChunk);
 }
 
 // Second-chance drain used only on the abort path: waits (bounded, ignoring
@@ -62,6 +79,10 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
 }
 
 __device__ __forceinline__ float bits_f(uint32_t u) { return __uint_as_float(u); }
+__device__ __forceinline__ float2 pair(const uint32_t (&r)[16], int c) {
+  return make_float2(__uint_as_float(r[c]), __uint_as_float(r[c + 1]));
+}
+__device__ __forceinline__ float2 splat(float x) { return make_float2(x, x); }
 
 // 16 bf16 values -> two 16-byte global stores.
 __device__ __forceinline__ void store_row16(__nv_bfloat16* dst, const float (&v)[16]) {
@@ -104,6 +125,12 @@ __device__ __forceinline__ float row_dot(const __nv_bfloat16* a, const __nv_bflo
   return acc;
 }
 
+// p = exp2(s * sl2 - L2) for a pair of scores; masked entries are 0.
+__device__ __forceinline__ float2 probs2(float2 s, float2 sl2, float2 nL2) {
+  const float2 a = __ffma2_rn(s, sl2, nL2);
+  return make_float2(ex2(a.x), ex2(a.y));
+}
+
 // ============================================================== row engine
 template <RowOp OP, int D>
 __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant__ EngineParams p) {
@@ -134,18 +161,20 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
   const int last_row = min(i0 + BM, N) - 1;
   const int ntiles = p.causal ? (last_row / BN + 1) : (N + BN - 1) / BN;
   const int nsteps = OP == RowOp::Fwd ? 2 * ntiles : ntiles;
+  const int first_b = OP == RowOp::Fwd ? ntiles : 0;  // first step with stage-B MMAs
 
   if (tid == 0) {
     m->abort_flag = 0;
     mbar_init(&m->bar_stat, 1);
     for (int s = 0; s < C::NSTAGES; ++s) {
       mbar_init(&m->bar_full[s], 1);
-      mbar_init(&m->bar_empty[s], 1);
+      mbar_init(&m->bar_empty[s], 2);  // released by both MMA issuers
     }
-    mbar_init(&m->bar_sa, 1);
-    mbar_init(&m->bar_ew[0], kEwThreads);
-    mbar_init(&m->bar_ew[1], kEwThreads);
-    mbar_init(&m->bar_acc, 1);
+    for (int h = 0; h < 2; ++h) {
+      mbar_init(&m->bar_sa[h], 2);  // one commit per MMA issuer
+      mbar_init(&m->bar_ew[h], kEwThreads);
+    }
+    mbar_init(&m->bar_acc, 2);
     fence_mbar_init();
   }
   if (warp == kMmaWarp) {
@@ -173,15 +202,16 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         if (st >= C::NSTAGES) {
           if (!mbar_wait(&m->bar_empty[stage], ((st / C::NSTAGES) - 1) & 1, abort_flag)) break;
         }
-        const int j = st % ntiles;
+        const int j0 = (st % ntiles) * BN;
         const bool k_only = (OP == RowOp::Fwd) && st < ntiles;
+        const int nt = k_only ? 1 : C::NSTREAM;
         uint8_t* dst = s_stream + stage * C::STAGE_BYTES;
-        mbar_arrive_expect_tx(&m->bar_full[stage],
-                              k_only ? C::KB * BN * 128 : C::STAGE_BYTES);
-        for (int t = 0; t < (k_only ? 1 : C::NSTREAM); ++t)
-          for (int b = 0; b < C::KB; ++b)
-            tma_load_3d(dst + (b * C::NSTREAM + t) * (BN * 128), &p.tm[C::NSTAT + t],
-                        &m->bar_full[stage], 64 * b, j * BN, bh);
+        mbar_arrive_expect_tx(&m->bar_full[stage], nt * C::KB * 2 * kChunk);
+        for (int b = 0; b < C::KB; ++b)
+          for (int h = 0; h < 2; ++h)
+            for (int t = 0; t < nt; ++t)
+              tma_load_3d(dst + chunk_off<C::NSTREAM>(t, h, b), &p.tm[C::NSTAT + t],
+                          &m->bar_full[stage], 64 * b, j0 + HB * h, bh);
         issued[stage] = st;
       }
       if (*abort_flag) {  // drain loads still in flight
@@ -190,95 +220,141 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         drain_wait(&m->bar_stat, 0);
       }
     }
-  } else if (warp == kMmaWarp) {
-    // ------------------------------------------------------------ MMA issuer
+  } else if (warp == kMmaWarp || warp == kMmaWarpY) {
+    // ------------------------------------------------------------ MMA issuers
+    // Issuer X (warp 9) owns stage-A columns 0..63 of each half region and the
+    // accumulators it feeds from them; issuer Y (warp 10) owns columns 64..127.
+    // Each issuer reads only operand tiles inside the columns it overwrites
+    // itself, so the two never race on tensor memory and every accumulator
+    // has one issuer (fixed summation order).
     if (elect_lane0()) {
-      const uint32_t id_n64 = idesc_bf16(128, 64, false);
-      const uint32_t id_n128 = idesc_bf16(128, 128, false);
-      const uint32_t id_b = idesc_bf16(128, C::DOUT, true);
-      const uint32_t tA = tmem + kColA;
-      bool ok = mbar_wait(&m->bar_stat, 0, abort_flag);
-      for (int st = 0; ok && st < nsteps; ++st) {
-        const int stage = st % C::NSTAGES;
-        if (!mbar_wait(&m->bar_full[stage], (st / C::NSTAGES) & 1, abort_flag)) break;
-        tc_fence_after();
-        const uint32_t sbase = smem_u32(s_stream + stage * C::STAGE_BYTES);
-        const uint32_t stat = smem_u32(s_stat);
-        auto stat_desc = [&](int t, int k) {
-          return sdesc_sw128(stat + (t * C::KB + k / 4) * (BM * 128) + (k % 4) * 32, 16, 1024);
+      const int role = warp == kMmaWarp ? 0 : 1;
+      constexpr uint32_t id_n32 = idesc_bf16(128, 32, false);
+      constexpr uint32_t id_n64 = idesc_bf16(128, 64, false);
+      constexpr uint32_t id_b = idesc_bf16(128, C::DOUT, true);
+      constexpr uint32_t id_b2 = idesc_bf16(128, 2 * C::DOUT, true);
+      // descriptors are formed once; per MMA only the start-address field moves
+      const uint64_t sd0 = sdesc_sw128(smem_u32(s_stat), 16, 1024);
+      auto sd = [&](int t, int k) -> uint64_t {
+        return sd0 + (uint64_t)(((t * C::KB + k / 4) * (BM * 128) + (k % 4) * 32) >> 4);
+      };
+      auto stage_a = [&](uint32_t sb, int h) {
+        const uint64_t kd0 = sdesc_sw128(sb, 16, 1024);
+        auto kd = [&](int t, int k) -> uint64_t {
+          return kd0 + (uint64_t)((chunk_off<C::NSTREAM>(t, h, k / 4) + (k % 4) * 32) >> 4);
         };
-        auto strm_desc = [&](int t, int k) {
-          return sdesc_sw128(sbase + ((k / 4) * C::NSTREAM + t) * (BN * 128) + (k % 4) * 32, 16,
-                             1024);
-        };
-        // ---- stage A
+        const uint32_t R = tmem + kColA + 128 * h;
         if constexpr (OP == RowOp::BobPass1) {
           // stationary: 0 Q, 1 U_Q, 2 dO ; stream: 0 K, 1 U_K, 2 V, 3 U_V
-          for (int k = 0; k < D / 16; ++k)  // [S | F2] = Q [K ; U_K]^T
-            mma_ss(tA + 0, stat_desc(0, k), strm_desc(0, k), id_n128, k > 0);
-          for (int k = 0; k < D / 16; ++k)  // [dP | C] = dO [V ; U_V]^T
-            mma_ss(tA + 128, stat_desc(2, k), strm_desc(2, k), id_n128, k > 0);
-          for (int k = 0; k < D / 16; ++k)  // F += U_Q K^T
-            mma_ss(tA + 64, stat_desc(1, k), strm_desc(0, k), id_n64, 1);
+          if (role == 0) {
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k)  // [S | F] = Q [K ; U_K]^T
+              mma_ss(R + 0, sd(0, k), kd(0, k), id_n64, k > 0);
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k)  // F += U_Q K^T
+              mma_ss(R + 32, sd(1, k), kd(0, k), id_n32, 1);
+          } else {
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k)  // [dP | C] = dO [V ; U_V]^T
+              mma_ss(R + 64, sd(2, k), kd(2, k), id_n64, k > 0);
+          }
         } else if constexpr (OP == RowOp::BwdDQ) {
-          // stationary: 0 Q, 1 dO ; stream: 0 K, 1 V
-          for (int k = 0; k < D / 16; ++k)
-            mma_ss(tA + 0, stat_desc(0, k), strm_desc(0, k), id_n64, k > 0);
-          for (int k = 0; k < D / 16; ++k)
-            mma_ss(tA + 64, stat_desc(1, k), strm_desc(1, k), id_n64, k > 0);
+          if (role == 0) {
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k)  // S = Q K^T
+              mma_ss(R + 0, sd(0, k), kd(0, k), id_n32, k > 0);
+          } else {
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k)  // dP = dO V^T
+              mma_ss(R + 32, sd(1, k), kd(1, k), id_n32, k > 0);
+          }
         } else {
-          for (int k = 0; k < D / 16; ++k)
-            mma_ss(tA + 0, stat_desc(0, k), strm_desc(0, k), id_n64, k > 0);
+          if (role == 0) {
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k)  // S = Q K^T
+              mma_ss(R + 0, sd(0, k), kd(0, k), id_n32, k > 0);
+          }
         }
-        mma_commit(&m->bar_sa);
-        // ---- stage B, per chunk, once the elementwise warps have written it
+      };
+      auto stage_b = [&](uint32_t sb, int h, int st) {
+        if (st < first_b) return;
+        // MN-major views: rows 16*sub.. of streamed tensor t (box bo) ; the fused
+        // view spans [K | U_V] (second 64-wide block three chunks further on)
+        const uint64_t md0 = sdesc_sw128(sb, 2 * C::NSTREAM * kChunk, 1024);
+        const uint64_t mf0 = sdesc_sw128(sb, 3 * kChunk, 1024);
+#pragma unroll
+        for (int sub = 0; sub < 2; ++sub) {
+          auto md = [&](int t, int bo) -> uint64_t {
+            return md0 + (uint64_t)((chunk_off<C::NSTREAM>(t, h, bo) + sub * 2048) >> 4);
+          };
+          const uint32_t first = (st == first_b && h == 0 && sub == 0) ? 0u : 1u;
+          const uint32_t A = tmem + kColA + 128 * h + 16 * sub;
+          if constexpr (OP == RowOp::BobPass1) {
+            if (role == 0) {
+              // [B | dOtil0] += P [K | U_V] ;  dOtil0 += (P o F) V
+              const uint64_t fused =
+                  mf0 + (uint64_t)((chunk_off<C::NSTREAM>(0, h, split) + sub * 2048) >> 4);
+              mma_ts(tmem + 0, A + 0, fused, id_b2, first);
+              mma_ts(tmem + 64, A + 8, md(2, split), id_b, 1);
+            } else {
+              mma_ts(tmem + 128, A + 64, md(0, split), id_b, first);  // Omega += (P o Pt0) K
+              mma_ts(tmem + 128, A + 72, md(1, split), id_b, 1);      //   += dS U_K
+              mma_ts(tmem + 192, A + 96, md(0, split), id_b, first);  // R += (P o dP) K
+            }
+          } else if constexpr (OP == RowOp::BwdDQ) {
+            if (role == 0) mma_ts(tmem + 0, A, md(0, 0), id_b, first);  // dQ += dS K
+          } else {
+            if (role == 0) mma_ts(tmem + 0, A, md(1, 0), id_b, first);  // O += P V
+          }
+        }
+      };
+      bool ok = mbar_wait(&m->bar_stat, 0, abort_flag) &&
+                mbar_wait(&m->bar_full[0], 0, abort_flag);
+      if (ok) {
+        tc_fence_after();
+        const uint32_t sb0 = smem_u32(s_stream);
+        stage_a(sb0, 0);
+        mma_commit(&m->bar_sa[0]);
+        stage_a(sb0, 1);
+        mma_commit(&m->bar_sa[1]);
+      }
+      for (int st = 0; ok && st < nsteps; ++st) {
+        const int stage = st % C::NSTAGES;
+        const uint32_t sb = smem_u32(s_stream + stage * C::STAGE_BYTES);
+        const int nstage = (st + 1) % C::NSTAGES;
+        const uint32_t nsb = smem_u32(s_stream + nstage * C::STAGE_BYTES);
+        const bool more = st + 1 < nsteps;
+#pragma unroll
         for (int h = 0; h < 2; ++h) {
           if (!mbar_wait(&m->bar_ew[h], st & 1, abort_flag)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          for (int s = 2 * h; s < 2 * h + 2; ++s) {
-            const uint32_t first = (st == 0 && s == 0) ? 0u : 1u;
-            auto mn_desc = [&](int t) {  // streamed tile t, output block `split`, rows 16s..
-              return sdesc_sw128(
-                  sbase + (split * C::NSTREAM + t) * (BN * 128) + s * 2048,
-                  C::NSTREAM * BN * 128, 1024);
-            };
-            if constexpr (OP == RowOp::BobPass1) {
-              const uint32_t aP = tA + 16 * s, aPF = tA + 16 * s + 8;
-              const uint32_t aPPt = tA + 128 + 16 * s, adS = tA + 128 + 16 * s + 8;
-              const uint32_t aPdP = tA + 192 + 16 * s;
-              mma_ts(tmem + 0, aP, mn_desc(3), id_b, first);     // dOtil0 += P U_V
-              mma_ts(tmem + 0, aPF, mn_desc(2), id_b, 1);        //        += (P o F) V
-              mma_ts(tmem + 64, aPPt, mn_desc(0), id_b, first);  // Omega  += (P o Pt0) K
-              mma_ts(tmem + 64, adS, mn_desc(1), id_b, 1);       //        += dS U_K
-              mma_ts(tmem + 128, aP, mn_desc(0), id_b, first);   // B      += P K
-              mma_ts(tmem + 192, aPdP, mn_desc(0), id_b, first); // R      += (P o dP) K
-            } else if constexpr (OP == RowOp::BwdDQ) {
-              mma_ts(tmem + 0, tA + 16 * s, mn_desc(0), id_b, first);  // dQ += dS K
-            } else {
-              if (st >= ntiles) {  // second sweep: O += P V
-                const uint32_t f2 = (st == ntiles && s == 0) ? 0u : 1u;
-                mma_ts(tmem + 0, tA + 16 * s, mn_desc(1), id_b, f2);
-              }
+          stage_b(sb, h, st);
+          if (h == 1) mma_commit(&m->bar_empty[stage]);
+          if (more) {
+            if (h == 0 && !mbar_wait(&m->bar_full[nstage], ((st + 1) / C::NSTAGES) & 1,
+                                     abort_flag)) {
+              ok = false;
+              break;
             }
+            tc_fence_after();
+            stage_a(nsb, h);
+            mma_commit(&m->bar_sa[h]);
           }
         }
-        if (!ok) break;
-        mma_commit(&m->bar_empty[stage]);
       }
       mma_commit(&m->bar_acc);
       if (*abort_flag) drain_wait(&m->bar_acc, 0);
     }
   } else {
     // ------------------------------------------------------------ elementwise
-    const int wg = warp >> 2;                 // warpgroup 0/1
+    const int wg = warp >> 2;                    // warpgroup 0/1
     const int r = 32 * (warp & 3) + (tid & 31);  // stationary row in the block
     const int gi = i0 + r;
     const bool row_ok = gi < N;
     const uint32_t ta = lane_base_addr(tmem, warp);
-    const uint32_t tA = ta + kColA;
     const size_t rowoff = ((size_t)bh * N + (size_t)(row_ok ? gi : 0)) * D;
     const float tau = p.scale;
     const float sl2 = tau * kLog2e;
@@ -289,107 +365,106 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         Dr = row_dot<D>(p.dout + rowoff, p.o + rowoff);
       }
     }
-    float mrow = -INFINITY, lrow = 0.f;  // forward sweep-1 running max / sum (log2 domain)
-    float a_part = 0.f, e_part = 0.f;    // Pass 1 partial row sums
+    float mrow = -INFINITY, lrow = 0.f;               // forward sweep 1 (log2 domain)
+    float2 acc_a = splat(0.f), acc_e = splat(0.f);    // Pass 1 partial row sums
     bool ok = true;
-    for (int st = 0; st < nsteps; ++st) {
-      if (!mbar_wait(&m->bar_sa, st & 1, abort_flag)) {
-        ok = false;
-        break;
-      }
-      tc_fence_after();
-      const int j0 = (st % ntiles) * BN;
-      const bool need_mask = (!row_ok) || (j0 + BN > N) || (p.causal && j0 + BN - 1 > gi);
-      if constexpr (OP == RowOp::Fwd) {
-        if (st == ntiles) {  // end of sweep 1: combine the two warpgroups' (max, sum)
-          s_xchg[wg * BM + r] = mrow;
-          s_xchg[(2 + wg) * BM + r] = lrow;
-          named_bar_sync(1, kEwThreads);
-          const float m0 = s_xchg[r], m1 = s_xchg[BM + r];
-          const float l0 = s_xchg[2 * BM + r], l1 = s_xchg[3 * BM + r];
-          const float mm = fmaxf(m0, m1);
-          const float l = (m0 == -INFINITY ? 0.f : l0 * ex2(m0 - mm)) +
-                          (m1 == -INFINITY ? 0.f : l1 * ex2(m1 - mm));
-          L2 = row_ok ? mm + __log2f(l) : 0.f;
-        }
-      }
+    for (int st = 0; ok && st < nsteps; ++st) {
       for (int h = 0; h < 2; ++h) {
-        const int s = 2 * h + wg;  // K-step handled by this warpgroup
-        const int c0 = 16 * s;
+        if (!mbar_wait(&m->bar_sa[h], st & 1, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        if constexpr (OP == RowOp::Fwd) {
+          if (st == ntiles && h == 0) {  // end of sweep 1: combine the warpgroups' (max, sum)
+            s_xchg[wg * BM + r] = mrow;
+            s_xchg[(2 + wg) * BM + r] = lrow;
+            named_bar_sync(1, kEwThreads);
+            const float m0 = s_xchg[r], m1 = s_xchg[BM + r];
+            const float l0 = s_xchg[2 * BM + r], l1 = s_xchg[3 * BM + r];
+            const float mm = fmaxf(m0, m1);
+            const float l = (m0 == -INFINITY ? 0.f : l0 * ex2(m0 - mm)) +
+                            (m1 == -INFINITY ? 0.f : l1 * ex2(m1 - mm));
+            L2 = row_ok ? mm + __log2f(l) : 0.f;
+          }
+        }
+        const int c0 = 16 * wg;                                // column within the half
+        const int j0 = (st % ntiles) * BN + HB * h + c0;       // first key of this thread's 16
+        const bool need_mask = (!row_ok) || (j0 + 16 > N) || (p.causal && j0 + 15 > gi);
+        const int lim = need_mask ? (row_ok ? (p.causal ? min(N, gi + 1) : N) - j0 : 0) : 16;
+        const uint32_t R = ta + kColA + 128 * h + c0;  // this thread's 16 columns, region X0
+        const float2 sl2v = splat(sl2), nL2v = splat(-L2);
         if constexpr (OP == RowOp::BobPass1) {
           uint32_t rS[16], rF[16], rdP[16], rC[16];
-          tmem_ld16(tA + 0 + c0, rS);
-          tmem_ld16(tA + 64 + c0, rF);
-          tmem_ld16(tA + 128 + c0, rdP);
-          tmem_ld16(tA + 192 + c0, rC);
+          tmem_ld16(R + 0, rS);
+          tmem_ld16(R + 32, rF);
+          tmem_ld16(R + 64, rdP);
+          tmem_ld16(R + 96, rC);
           tmem_ld_wait(rS);
           reg_dep(rF);
           reg_dep(rdP);
           reg_dep(rC);
+          const float2 tauv = splat(tau), nDv = splat(-Dr);
           uint32_t oP[8], oPF[8], oPPt[8], odS[8], oPdP[8];
 #pragma unroll
           for (int c = 0; c < 16; c += 2) {
-            float pv[2], pf[2], ppt[2], ds[2], pdp[2];
-#pragma unroll
-            for (int e = 0; e < 2; ++e) {
-              const int gj = j0 + c0 + c + e;
-              float pr = ex2(fmaf(bits_f(rS[c + e]), sl2, -L2));
-              if (need_mask && !(row_ok && gj < N && (!p.causal || gj <= gi))) pr = 0.f;
-              const float f = tau * bits_f(rF[c + e]);
-              const float dp = bits_f(rdP[c + e]);
-              const float t = dp - Dr;
-              const float pt0 = fmaf(f, t, bits_f(rC[c + e]));  // Ptil0 = C + F (dP - D)
-              pv[e] = pr;
-              pf[e] = pr * f;
-              ppt[e] = pr * pt0;
-              ds[e] = pr * t;
-              pdp[e] = pr * dp;
-              a_part += pf[e];
-              e_part += ppt[e];
+            float2 pr = probs2(pair(rS, c), sl2v, nL2v);
+            if (need_mask) {
+              if (c >= lim) pr.x = 0.f;
+              if (c + 1 >= lim) pr.y = 0.f;
             }
-            oP[c / 2] = pack_bf16(pv[0], pv[1]);
-            oPF[c / 2] = pack_bf16(pf[0], pf[1]);
-            oPPt[c / 2] = pack_bf16(ppt[0], ppt[1]);
-            odS[c / 2] = pack_bf16(ds[0], ds[1]);
-            oPdP[c / 2] = pack_bf16(pdp[0], pdp[1]);
+            const float2 f = __fmul2_rn(pair(rF, c), tauv);
+            const float2 dp = pair(rdP, c);
+            const float2 t = __fadd2_rn(dp, nDv);
+            const float2 pt0 = __ffma2_rn(f, t, pair(rC, c));  // Ptil0 = C + F (dP - D)
+            const float2 pf = __fmul2_rn(pr, f);
+            const float2 ppt = __fmul2_rn(pr, pt0);
+            const float2 ds = __fmul2_rn(pr, t);
+            const float2 pdp = __fmul2_rn(pr, dp);
+            acc_a = __fadd2_rn(acc_a, pf);
+            acc_e = __fadd2_rn(acc_e, ppt);
+            oP[c / 2] = pack_bf16(pr.x, pr.y);
+            oPF[c / 2] = pack_bf16(pf.x, pf.y);
+            oPPt[c / 2] = pack_bf16(ppt.x, ppt.y);
+            odS[c / 2] = pack_bf16(ds.x, ds.y);
+            oPdP[c / 2] = pack_bf16(pdp.x, pdp.y);
           }
-          tmem_st8(tA + 0 + c0, oP);
-          tmem_st8(tA + 0 + c0 + 8, oPF);
-          tmem_st8(tA + 128 + c0, oPPt);
-          tmem_st8(tA + 128 + c0 + 8, odS);
-          tmem_st8(tA + 192 + c0, oPdP);
+          // operand tiles: issuer X reads columns 0..63, issuer Y 64..127
+          tmem_st8(R + 0, oP);
+          tmem_st8(R + 8, oPF);
+          tmem_st8(R + 64, oPPt);
+          tmem_st8(R + 72, odS);
+          tmem_st8(R + 96, oPdP);
         } else if constexpr (OP == RowOp::BwdDQ) {
           uint32_t rS[16], rdP[16];
-          tmem_ld16(tA + 0 + c0, rS);
-          tmem_ld16(tA + 64 + c0, rdP);
+          tmem_ld16(R + 0, rS);
+          tmem_ld16(R + 32, rdP);
           tmem_ld_wait(rS);
           reg_dep(rdP);
+          const float2 nDv = splat(-Dr);
           uint32_t odS[8];
 #pragma unroll
           for (int c = 0; c < 16; c += 2) {
-            float ds[2];
-#pragma unroll
-            for (int e = 0; e < 2; ++e) {
-              const int gj = j0 + c0 + c + e;
-              float pr = ex2(fmaf(bits_f(rS[c + e]), sl2, -L2));
-              if (need_mask && !(row_ok && gj < N && (!p.causal || gj <= gi))) pr = 0.f;
-              ds[e] = pr * (bits_f(rdP[c + e]) - Dr);
+            float2 pr = probs2(pair(rS, c), sl2v, nL2v);
+            if (need_mask) {
+              if (c >= lim) pr.x = 0.f;
+              if (c + 1 >= lim) pr.y = 0.f;
             }
-            odS[c / 2] = pack_bf16(ds[0], ds[1]);
+            const float2 ds = __fmul2_rn(pr, __fadd2_rn(pair(rdP, c), nDv));
+            odS[c / 2] = pack_bf16(ds.x, ds.y);
           }
-          tmem_st8(tA + c0, odS);
+          tmem_st8(R, odS);
         } else {
           uint32_t rS[16];
-          tmem_ld16(tA + c0, rS);
+          tmem_ld16(R, rS);
           tmem_ld_wait(rS);
           if (st < ntiles) {  // sweep 1: running max and sum in the log2 domain
             float x[16];
             float mx = mrow;
 #pragma unroll
             for (int c = 0; c < 16; ++c) {
-              const int gj = j0 + c0 + c;
               x[c] = bits_f(rS[c]) * sl2;
-              if (need_mask && !(row_ok && gj < N && (!p.causal || gj <= gi))) x[c] = -INFINITY;
+              if (need_mask && c >= lim) x[c] = -INFINITY;
               mx = fmaxf(mx, x[c]);
             }
             if (mx != -INFINITY) {
@@ -403,17 +478,14 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
             uint32_t oP[8];
 #pragma unroll
             for (int c = 0; c < 16; c += 2) {
-              float pv[2];
-#pragma unroll
-              for (int e = 0; e < 2; ++e) {
-                const int gj = j0 + c0 + c + e;
-                float pr = ex2(fmaf(bits_f(rS[c + e]), sl2, -L2));
-                if (need_mask && !(row_ok && gj < N && (!p.causal || gj <= gi))) pr = 0.f;
-                pv[e] = pr;
+              float2 pr = probs2(pair(rS, c), sl2v, nL2v);
+              if (need_mask) {
+                if (c >= lim) pr.x = 0.f;
+                if (c + 1 >= lim) pr.y = 0.f;
               }
-              oP[c / 2] = pack_bf16(pv[0], pv[1]);
+              oP[c / 2] = pack_bf16(pr.x, pr.y);
             }
-            tmem_st8(tA + c0, oP);
+            tmem_st8(R, oP);
           }
         }
         tmem_st_wait();
@@ -423,10 +495,11 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
     }
     // ---------------------------------------------------------- epilogue
     if (ok) ok = mbar_wait(&m->bar_acc, 0, abort_flag);
+    if (ok && *abort_flag) ok = false;
     tc_fence_after();
     if constexpr (OP == RowOp::BobPass1) {
-      s_xchg[wg * BM + r] = a_part;
-      s_xchg[(2 + wg) * BM + r] = e_part;
+      s_xchg[wg * BM + r] = acc_a.x + acc_a.y;
+      s_xchg[(2 + wg) * BM + r] = acc_e.x + acc_e.y;
       named_bar_sync(1, kEwThreads);
     }
     if (ok) {
@@ -438,10 +511,11 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
 #pragma unroll 1
         for (int q = 0; q < 2; ++q) {
           const int cc = 32 * wg + 16 * q;  // accumulator column (0..63)
+          // accumulators: B at 0, dOtil0 at 64, Omega at 128, R at 192
           uint32_t rO[16], rW[16], rB[16], rR[16];
-          tmem_ld16(ta + 0 + cc, rO);
-          tmem_ld16(ta + 64 + cc, rW);
-          tmem_ld16(ta + 128 + cc, rB);
+          tmem_ld16(ta + 64 + cc, rO);
+          tmem_ld16(ta + 128 + cc, rW);
+          tmem_ld16(ta + 0 + cc, rB);
           tmem_ld16(ta + 192 + cc, rR);
           tmem_ld_wait(rO);
           reg_dep(rW);
@@ -514,7 +588,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
     return;
   }
   const int N = p.N;
-  int lin = blockIdx.x;
+  const int lin = blockIdx.x;
   const int bh = lin % p.BH;
   const int cb = lin / p.BH;  // key block; block 0 has the most work under the causal mask
   const int j0 = cb * BM;
@@ -527,12 +601,13 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
     mbar_init(&m->bar_stat, 1);
     for (int s = 0; s < C::NSTAGES; ++s) {
       mbar_init(&m->bar_full[s], 1 + 32);  // TMA bytes + 32 producer lanes' row vectors
-      mbar_init(&m->bar_empty[s], 1);
+      mbar_init(&m->bar_empty[s], 2);      // released by both MMA issuers
     }
-    mbar_init(&m->bar_sa, 1);
-    mbar_init(&m->bar_ew[0], kEwThreads);
-    mbar_init(&m->bar_ew[1], kEwThreads);
-    mbar_init(&m->bar_acc, 1);
+    for (int h = 0; h < 2; ++h) {
+      mbar_init(&m->bar_sa[h], 2);  // one commit per MMA issuer
+      mbar_init(&m->bar_ew[h], kEwThreads);
+    }
+    mbar_init(&m->bar_acc, 2);
     fence_mbar_init();
   }
   if (warp == kMmaWarp) {
@@ -566,12 +641,14 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
       uint8_t* dst = s_stream + stage * C::STAGE_BYTES;
       if (lane == 0) {
         mbar_arrive_expect_tx(&m->bar_full[stage], C::TILE_BYTES);
-        for (int t = 0; t < C::NSTREAM; ++t)
-          for (int b = 0; b < C::KB; ++b)
-            tma_load_3d(dst + (b * C::NSTREAM + t) * (BN * 128), &p.tm[C::NSTAT + t],
-                        &m->bar_full[stage], 64 * b, ib, bh);
+        for (int b = 0; b < C::KB; ++b)
+          for (int h = 0; h < 2; ++h)
+            for (int t = 0; t < C::NSTREAM; ++t)
+              tma_load_3d(dst + chunk_off<C::NSTREAM>(t, h, b), &p.tm[C::NSTAT + t],
+                          &m->bar_full[stage], 64 * b, ib + HB * h, bh);
       }
-      // row vectors of the streamed query rows: [0] L*log2e, [1] D, [2] alpha, [3] E
+      // negated row vectors of the streamed query rows:
+      // [0] -L*log2e, [1] -D, [2] -alpha, [3] -E
       float* vec = reinterpret_cast<float*>(dst + C::TILE_BYTES);
 #pragma unroll
       for (int q = 0; q < 2; ++q) {
@@ -579,14 +656,13 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
         const int gi = ib + c;
         const bool ok = gi < N;
         const size_t ri = (size_t)bh * N + (ok ? gi : 0);
+        vec[c] = ok ? -p.lse[ri] * kLog2e : 0.f;
         if constexpr (OP == ColOp::BwdDKDV) {
-          vec[c] = ok ? p.lse[ri] * kLog2e : 0.f;
-          vec[64 + c] = ok ? p.vec_in[ri] : 0.f;
+          vec[64 + c] = ok ? -p.vec_in[ri] : 0.f;
         } else {
-          vec[c] = ok ? p.lse[ri] * kLog2e : 0.f;
-          vec[64 + c] = ok ? p.vec_in[2 * p.bhn + ri] : 0.f;  // D
-          vec[128 + c] = ok ? p.vec_in[ri] : 0.f;             // alpha
-          vec[192 + c] = ok ? p.vec_in[p.bhn + ri] : 0.f;     // E
+          vec[64 + c] = ok ? -p.vec_in[2 * p.bhn + ri] : 0.f;  // D
+          vec[128 + c] = ok ? -p.vec_in[ri] : 0.f;             // alpha
+          vec[192 + c] = ok ? -p.vec_in[p.bhn + ri] : 0.f;     // E
         }
       }
       mbar_arrive(&m->bar_full[stage]);
@@ -597,68 +673,113 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
         if (issued[s] >= 0) drain_wait(&m->bar_full[s], (issued[s] / C::NSTAGES) & 1);
       drain_wait(&m->bar_stat, 0);
     }
-  } else if (warp == kMmaWarp) {
-    // ------------------------------------------------------------ MMA issuer
+  } else if (warp == kMmaWarp || warp == kMmaWarpY) {
+    // ------------------------------------------------------------ MMA issuers
+    // Same ownership split as the row engine: issuer X owns stage-A columns
+    // 0..63 of each half region, issuer Y columns 64..127.
     if (elect_lane0()) {
-      const uint32_t id_n64 = idesc_bf16(128, 64, false);
-      const uint32_t id_n128 = idesc_bf16(128, 128, false);
-      const uint32_t id_b = idesc_bf16(128, D, true);
-      const uint32_t tA = tmem + kColA;
-      bool ok = mbar_wait(&m->bar_stat, 0, abort_flag);
-      for (int st = 0; ok && st < nsteps; ++st) {
-        const int stage = st % C::NSTAGES;
-        if (!mbar_wait(&m->bar_full[stage], (st / C::NSTAGES) & 1, abort_flag)) break;
-        tc_fence_after();
-        const uint32_t sbase = smem_u32(s_stream + stage * C::STAGE_BYTES);
-        const uint32_t stat = smem_u32(s_stat);
-        auto stat_desc = [&](int t, int k) {
-          return sdesc_sw128(stat + (t * C::KB + k / 4) * (BM * 128) + (k % 4) * 32, 16, 1024);
+      const int role = warp == kMmaWarp ? 0 : 1;
+      constexpr uint32_t id_n32 = idesc_bf16(128, 32, false);
+      constexpr uint32_t id_n64 = idesc_bf16(128, 64, false);
+      constexpr uint32_t id_b = idesc_bf16(128, D, true);
+      const uint64_t sd0 = sdesc_sw128(smem_u32(s_stat), 16, 1024);
+      auto sd = [&](int t, int k) -> uint64_t {
+        return sd0 + (uint64_t)(((t * C::KB + k / 4) * (BM * 128) + (k % 4) * 32) >> 4);
+      };
+      auto stage_a = [&](uint32_t sb, int h) {
+        const uint64_t kd0 = sdesc_sw128(sb, 16, 1024);
+        auto kd = [&](int t, int k) -> uint64_t {
+          return kd0 + (uint64_t)((chunk_off<C::NSTREAM>(t, h, k / 4) + (k % 4) * 32) >> 4);
         };
-        auto strm_desc = [&](int t, int k) {
-          return sdesc_sw128(sbase + ((k / 4) * C::NSTREAM + t) * (BN * 128) + (k % 4) * 32, 16,
-                             1024);
-        };
+        const uint32_t R = tmem + kColA + 128 * h;
         if constexpr (OP == ColOp::BobPass2) {
           // stationary: 0 K, 1 V, 2 U_K, 3 U_V ; stream: 0 Q, 1 U_Q, 2 dO
-          for (int k = 0; k < D / 16; ++k)  // [S^T | F1^T] = K [Q ; U_Q]^T
-            mma_ss(tA + 0, stat_desc(0, k), strm_desc(0, k), id_n128, k > 0);
-          for (int k = 0; k < D / 16; ++k)  // F^T += U_K Q^T
-            mma_ss(tA + 64, stat_desc(2, k), strm_desc(0, k), id_n64, 1);
-          for (int k = 0; k < D / 16; ++k)  // dP^T = V dO^T
-            mma_ss(tA + 128, stat_desc(1, k), strm_desc(2, k), id_n64, k > 0);
-          for (int k = 0; k < D / 16; ++k)  // C^T = U_V dO^T
-            mma_ss(tA + 192, stat_desc(3, k), strm_desc(2, k), id_n64, k > 0);
+          if (role == 0) {
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k)  // [S^T | F^T] = K [Q ; U_Q]^T
+              mma_ss(R + 0, sd(0, k), kd(0, k), id_n64, k > 0);
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k)  // F^T += U_K Q^T
+              mma_ss(R + 32, sd(2, k), kd(0, k), id_n32, 1);
+          } else {
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k)  // dP^T = V dO^T
+              mma_ss(R + 64, sd(1, k), kd(2, k), id_n32, k > 0);
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k)  // C^T = U_V dO^T
+              mma_ss(R + 96, sd(3, k), kd(2, k), id_n32, k > 0);
+          }
         } else {
           // stationary: 0 K, 1 V ; stream: 0 Q, 1 dO
-          for (int k = 0; k < D / 16; ++k)
-            mma_ss(tA + 0, stat_desc(0, k), strm_desc(0, k), id_n64, k > 0);
-          for (int k = 0; k < D / 16; ++k)
-            mma_ss(tA + 64, stat_desc(1, k), strm_desc(1, k), id_n64, k > 0);
+          if (role == 0) {
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k)  // S^T = K Q^T
+              mma_ss(R + 0, sd(0, k), kd(0, k), id_n32, k > 0);
+          } else {
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k)  // dP^T = V dO^T
+              mma_ss(R + 64, sd(1, k), kd(1, k), id_n32, k > 0);
+          }
         }
-        mma_commit(&m->bar_sa);
+      };
+      auto stage_b = [&](uint32_t sb, int h, int st) {
+        const uint64_t md0 = sdesc_sw128(sb, 2 * C::NSTREAM * kChunk, 1024);
+#pragma unroll
+        for (int sub = 0; sub < 2; ++sub) {
+          auto md = [&](int t) -> uint64_t {
+            return md0 + (uint64_t)((chunk_off<C::NSTREAM>(t, h, 0) + sub * 2048) >> 4);
+          };
+          const uint32_t first = (st == 0 && h == 0 && sub == 0) ? 0u : 1u;
+          const uint32_t A = tmem + kColA + 128 * h + 16 * sub;
+          if constexpr (OP == ColOp::BobPass2) {
+            if (role == 0) {
+              mma_ts(tmem + D, A + 0, md(2), id_b, first);    // Vtil += (P o h)^T dO
+            } else {
+              mma_ts(tmem + 0, A + 64, md(0), id_b, first);   // Ktil += Stil^T Q
+              mma_ts(tmem + 0, A + 72, md(1), id_b, 1);       //      += dS^T U_Q
+            }
+          } else {
+            if (role == 0) mma_ts(tmem + D, A + 0, md(1), id_b, first);   // dV += P^T dO
+            else mma_ts(tmem + 0, A + 64, md(0), id_b, first);            // dK += dS^T Q
+          }
+        }
+      };
+      bool ok = mbar_wait(&m->bar_stat, 0, abort_flag) &&
+                mbar_wait(&m->bar_full[0], 0, abort_flag);
+      if (ok) {
+        tc_fence_after();
+        const uint32_t sb0 = smem_u32(s_stream);
+        stage_a(sb0, 0);
+        mma_commit(&m->bar_sa[0]);
+        stage_a(sb0, 1);
+        mma_commit(&m->bar_sa[1]);
+      }
+      for (int st = 0; ok && st < nsteps; ++st) {
+        const int stage = st % C::NSTAGES;
+        const uint32_t sb = smem_u32(s_stream + stage * C::STAGE_BYTES);
+        const int nstage = (st + 1) % C::NSTAGES;
+        const uint32_t nsb = smem_u32(s_stream + nstage * C::STAGE_BYTES);
+        const bool more = st + 1 < nsteps;
+#pragma unroll
         for (int h = 0; h < 2; ++h) {
           if (!mbar_wait(&m->bar_ew[h], st & 1, abort_flag)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          for (int s = 2 * h; s < 2 * h + 2; ++s) {
-            const uint32_t first = (st == 0 && s == 0) ? 0u : 1u;
-            auto mn_desc = [&](int t) {
-              return sdesc_sw128(sbase + t * (BN * 128) + s * 2048, C::NSTREAM * BN * 128, 1024);
-            };
-            if constexpr (OP == ColOp::BobPass2) {
-              mma_ts(tmem + D, tA + 16 * s, mn_desc(2), id_b, first);       // Vtil += (P o h)^T dO
-              mma_ts(tmem + 0, tA + 16 * s + 8, mn_desc(0), id_b, first);   // Ktil += Stil^T Q
-              mma_ts(tmem + 0, tA + 128 + 16 * s, mn_desc(1), id_b, 1);     //      += dS^T U_Q
-            } else {
-              mma_ts(tmem + D, tA + 16 * s, mn_desc(1), id_b, first);       // dV += P^T dO
-              mma_ts(tmem + 0, tA + 16 * s + 8, mn_desc(0), id_b, first);   // dK += dS^T Q
+          stage_b(sb, h, st);
+          if (h == 1) mma_commit(&m->bar_empty[stage]);
+          if (more) {
+            if (h == 0 && !mbar_wait(&m->bar_full[nstage], ((st + 1) / C::NSTAGES) & 1,
+                                     abort_flag)) {
+              ok = false;
+              break;
             }
+            tc_fence_after();
+            stage_a(nsb, h);
+            mma_commit(&m->bar_sa[h]);
           }
         }
-        if (!ok) break;
-        mma_commit(&m->bar_empty[stage]);
       }
       mma_commit(&m->bar_acc);
       if (*abort_flag) drain_wait(&m->bar_acc, 0);
@@ -670,32 +791,38 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
     const int gj = j0 + r;  // stationary key row
     const bool row_ok = gj < N;
     const uint32_t ta = lane_base_addr(tmem, warp);
-    const uint32_t tA = ta + kColA;
     const float tau = p.scale;
-    const float sl2 = tau * kLog2e;
+    const float2 sl2v = splat(tau * kLog2e), tauv = splat(tau);
     bool ok = true;
-    for (int st = 0; st < nsteps; ++st) {
+    for (int st = 0; ok && st < nsteps; ++st) {
       const int stage = st % C::NSTAGES;
       // the row vectors were written by the producer: acquire them explicitly
-      if (!mbar_wait(&m->bar_full[stage], (st / C::NSTAGES) & 1, abort_flag) ||
-          !mbar_wait(&m->bar_sa, st & 1, abort_flag)) {
+      if (!mbar_wait(&m->bar_full[stage], (st / C::NSTAGES) & 1, abort_flag)) {
         ok = false;
         break;
       }
-      tc_fence_after();
       const float* vec = reinterpret_cast<const float*>(s_stream + stage * C::STAGE_BYTES +
                                                         C::TILE_BYTES);
-      const int ib = (first_tile + st) * BN;
-      const bool need_mask = (!row_ok) || (ib + BN > N) || (p.causal && ib < gj);
       for (int h = 0; h < 2; ++h) {
-        const int s = 2 * h + wg;
-        const int c0 = 16 * s;
+        if (!mbar_wait(&m->bar_sa[h], st & 1, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const int c0 = 16 * wg;
+        const int cv = HB * h + c0;                    // tile column of this thread's first
+        const int ib = (first_tile + st) * BN + cv;    // first query row of this thread's 16
+        const bool need_mask = (!row_ok) || (ib + 16 > N) || (p.causal && ib < gj);
+        // valid query columns c satisfy  lo <= c < hi
+        const int lo = p.causal ? gj - ib : 0;
+        const int hi = row_ok ? N - ib : 0;
+        const uint32_t R = ta + kColA + 128 * h + c0;
         if constexpr (OP == ColOp::BobPass2) {
           uint32_t rS[16], rF[16], rdP[16], rC[16];
-          tmem_ld16(tA + 0 + c0, rS);
-          tmem_ld16(tA + 64 + c0, rF);
-          tmem_ld16(tA + 128 + c0, rdP);
-          tmem_ld16(tA + 192 + c0, rC);
+          tmem_ld16(R + 0, rS);
+          tmem_ld16(R + 32, rF);
+          tmem_ld16(R + 64, rdP);
+          tmem_ld16(R + 96, rC);
           tmem_ld_wait(rS);
           reg_dep(rF);
           reg_dep(rdP);
@@ -703,54 +830,53 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
           uint32_t oPh[8], oSt[8], odS[8];
 #pragma unroll
           for (int c = 0; c < 16; c += 2) {
-            float ph[2], stl[2], ds[2];
-#pragma unroll
-            for (int e = 0; e < 2; ++e) {
-              const int cc = c0 + c + e;
-              const int gi = ib + cc;
-              float pr = ex2(fmaf(bits_f(rS[c + e]), sl2, -vec[cc]));
-              if (need_mask && !(row_ok && gi < N && (!p.causal || gj <= gi))) pr = 0.f;
-              const float Dv = vec[64 + cc], al = vec[128 + cc], Ev = vec[192 + cc];
-              const float f = tau * bits_f(rF[c + e]);
-              const float dp = bits_f(rdP[c + e]);
-              const float t = dp - Dv;
-              // Ptil = C + F (dP - D) - alpha dP ; Stil = P (Ptil - E) ; h = F - alpha
-              const float pt = fmaf(-al, dp, fmaf(f, t, bits_f(rC[c + e])));
-              ph[e] = pr * (f - al);
-              stl[e] = pr * (pt - Ev);
-              ds[e] = pr * t;
+            const float2 nL2 = *reinterpret_cast<const float2*>(vec + cv + c);
+            const float2 nD = *reinterpret_cast<const float2*>(vec + 64 + cv + c);
+            const float2 nal = *reinterpret_cast<const float2*>(vec + 128 + cv + c);
+            const float2 nE = *reinterpret_cast<const float2*>(vec + 192 + cv + c);
+            float2 pr = probs2(pair(rS, c), sl2v, nL2);
+            if (need_mask) {
+              if (c < lo || c >= hi) pr.x = 0.f;
+              if (c + 1 < lo || c + 1 >= hi) pr.y = 0.f;
             }
-            oPh[c / 2] = pack_bf16(ph[0], ph[1]);
-            oSt[c / 2] = pack_bf16(stl[0], stl[1]);
-            odS[c / 2] = pack_bf16(ds[0], ds[1]);
+            const float2 f = __fmul2_rn(pair(rF, c), tauv);
+            const float2 dp = pair(rdP, c);
+            const float2 t = __fadd2_rn(dp, nD);
+            // Ptil = C + F (dP - D) - alpha dP ; Stil = P (Ptil - E) ; h = F - alpha
+            const float2 pt = __ffma2_rn(nal, dp, __ffma2_rn(f, t, pair(rC, c)));
+            const float2 ph = __fmul2_rn(pr, __fadd2_rn(f, nal));
+            const float2 stl = __fmul2_rn(pr, __fadd2_rn(pt, nE));
+            const float2 ds = __fmul2_rn(pr, t);
+            oPh[c / 2] = pack_bf16(ph.x, ph.y);
+            oSt[c / 2] = pack_bf16(stl.x, stl.y);
+            odS[c / 2] = pack_bf16(ds.x, ds.y);
           }
-          tmem_st8(tA + c0, oPh);
-          tmem_st8(tA + c0 + 8, oSt);
-          tmem_st8(tA + 128 + c0, odS);
+          // operand tiles: issuer X reads columns 0..63, issuer Y 64..127
+          tmem_st8(R + 0, oPh);
+          tmem_st8(R + 64, oSt);
+          tmem_st8(R + 72, odS);
         } else {
           uint32_t rS[16], rdP[16];
-          tmem_ld16(tA + 0 + c0, rS);
-          tmem_ld16(tA + 64 + c0, rdP);
+          tmem_ld16(R + 0, rS);
+          tmem_ld16(R + 64, rdP);
           tmem_ld_wait(rS);
           reg_dep(rdP);
           uint32_t oP[8], odS[8];
 #pragma unroll
           for (int c = 0; c < 16; c += 2) {
-            float pv[2], ds[2];
-#pragma unroll
-            for (int e = 0; e < 2; ++e) {
-              const int cc = c0 + c + e;
-              const int gi = ib + cc;
-              float pr = ex2(fmaf(bits_f(rS[c + e]), sl2, -vec[cc]));
-              if (need_mask && !(row_ok && gi < N && (!p.causal || gj <= gi))) pr = 0.f;
-              pv[e] = pr;
-              ds[e] = pr * (bits_f(rdP[c + e]) - vec[64 + cc]);
+            const float2 nL2 = *reinterpret_cast<const float2*>(vec + cv + c);
+            const float2 nD = *reinterpret_cast<const float2*>(vec + 64 + cv + c);
+            float2 pr = probs2(pair(rS, c), sl2v, nL2);
+            if (need_mask) {
+              if (c < lo || c >= hi) pr.x = 0.f;
+              if (c + 1 < lo || c + 1 >= hi) pr.y = 0.f;
             }
-            oP[c / 2] = pack_bf16(pv[0], pv[1]);
-            odS[c / 2] = pack_bf16(ds[0], ds[1]);
+            const float2 ds = __fmul2_rn(pr, __fadd2_rn(pair(rdP, c), nD));
+            oP[c / 2] = pack_bf16(pr.x, pr.y);
+            odS[c / 2] = pack_bf16(ds.x, ds.y);
           }
-          tmem_st8(tA + c0, oP);
-          tmem_st8(tA + c0 + 8, odS);
+          tmem_st8(R + 0, oP);
+          tmem_st8(R + 64, odS);
         }
         tmem_st_wait();
         tc_fence_before();
@@ -758,6 +884,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
       }
     }
     if (ok) ok = mbar_wait(&m->bar_acc, 0, abort_flag);
+    if (ok && *abort_flag) ok = false;
     tc_fence_after();
     if (ok) {
       const size_t rowoff = ((size_t)bh * N + (size_t)(row_ok ? gj : 0)) * D;

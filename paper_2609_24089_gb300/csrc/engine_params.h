@@ -11,14 +11,17 @@ namespace fbob {
 // Bits of the device-side error word.
 enum : uint32_t { kDevErrTimeout = 1u, kDevErrBadLaunch = 2u };
 
-constexpr int BM = 128;
-constexpr int BN = 64;
-constexpr int kThreads = 320;
+constexpr int BM = 128;          // stationary rows per CTA (TMEM lanes)
+constexpr int BN = 64;           // streamed rows per tile
+constexpr int HB = 32;           // streamed rows per half tile (TMA box rows of streamed maps)
+constexpr int kChunk = HB * 128; // bytes of one 32-row x 64-column bf16 chunk
+constexpr int kThreads = 352;
 constexpr int kProducerWarp = 8;
-constexpr int kMmaWarp = 9;
+constexpr int kMmaWarp = 9;   // MMA issuer X (and TMEM allocator)
+constexpr int kMmaWarpY = 10; // MMA issuer Y
 constexpr int kEwThreads = 256;
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kColA = 256;  // first stage-A column
+constexpr uint32_t kColA = 256;  // stage-A region of half h starts at kColA + 128 h
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 
@@ -27,7 +30,7 @@ enum class ColOp { BwdDKDV, BobPass2 };
 
 // ---------------------------------------------------------------- parameters
 struct EngineParams {
-  CUtensorMap tm[7];  // stationary maps first (box rows BM), then streamed (box rows BN)
+  CUtensorMap tm[7];  // stationary maps first (box rows BM), then streamed (box rows HB)
   const __nv_bfloat16* o;     // forward output O (row engine: D and dOtil)
   const __nv_bfloat16* dout;  // dO (row engine: D = do.o)
   const float* lse;           // natural-log L [BH, N]
