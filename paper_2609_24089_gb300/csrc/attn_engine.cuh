@@ -23,20 +23,17 @@
 //              0..63 of each half region, Y columns 64..127, and each reads
 //              operand tiles only inside its own columns.
 //
-// Half-tile pipeline.  Every streamed tile is split into two halves of 32
-// rows, each with its own stage-A region of tensor memory (128 columns at
-// kColA + 128 h).  Per half: stage A (scores and friends, fp32, A and B from
-// shared memory) -> elementwise (TMEM -> registers -> bf16 operand tiles
-// written back into the columns of that region already read) -> stage B
-// (accumulators += bf16 tile (TMEM) x streamed half tile (shared memory,
-// MN-major)).  Each issuer runs  B_0(t), A_0(t+1), B_1(t), A_1(t+1), ...
-// so the tensor pipe works on one half while the elementwise warps work on the
-// other.  Accumulators live at TMEM columns 0..255.
+// Per streamed tile: stage A (scores and friends, fp32 in the 256 stage-A
+// columns of TMEM; A and B from shared memory; tensors streamed side by side
+// -- K and U_K, V and U_V, Q and U_Q -- form one 128-row B operand, so the
+// main stage-A MMAs have N = 128) -> elementwise in two halves of 32 columns
+// (TMEM -> registers -> bf16 operand tiles written back into columns already
+// read) -> stage B per half (accumulators += bf16 tile (TMEM) x streamed tile
+// (shared memory, MN-major)).  Stage B of half 0 runs while the elementwise
+// warps work on half 1.  Accumulators live at TMEM columns 0..255.
 //
 // Shared memory: stationary tensors as 128-row x 64-column swizzled boxes;
-// each stream stage as 32-row x 64-column chunks ordered (box, half, tensor),
-// so that two tensors streamed side by side (K and U_K, V and U_V, Q and U_Q)
-// form one 64-row operand of a fused N = 64 stage-A MMA.
+// each stream stage as 64-row x 64-column boxes ordered (box, tensor).
 //
 // Every wait is bounded (tc_ptx.cuh); on expiry the CTA records a timeout in
 // the device error word, drains its own asynchronous work and exits.
@@ -63,10 +60,10 @@ __device__ __forceinline__ uint32_t lane_base_addr(uint32_t tmem_base, int warp)
   return tmem_base + ((uint32_t)(32 * (warp & 3)) << 16);
 }
 
-// Offset of streamed tensor t, half h, 64-column box b inside a stream stage.
+// Offset of streamed tensor t, 64-column box b inside a stream stage.
 template <int NSTREAM>
-__device__ __forceinline__ uint32_t chunk_off(int t, int h, int b) {
-  return (uint32_t)(((b * 2 + h) * NSTREAM + t) * kChunk);
+__device__ __forceinline__ uint32_t tile_off(int t, int b) {
+  return (uint32_t)((b * NSTREAM + t) * (BN * 128));
 }
 
 // Second-chance drain used only on the abort path: waits (bounded, ignoring
@@ -206,12 +203,11 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         const bool k_only = (OP == RowOp::Fwd) && st < ntiles;
         const int nt = k_only ? 1 : C::NSTREAM;
         uint8_t* dst = s_stream + stage * C::STAGE_BYTES;
-        mbar_arrive_expect_tx(&m->bar_full[stage], nt * C::KB * 2 * kChunk);
+        mbar_arrive_expect_tx(&m->bar_full[stage], nt * C::KB * BN * 128);
         for (int b = 0; b < C::KB; ++b)
-          for (int h = 0; h < 2; ++h)
-            for (int t = 0; t < nt; ++t)
-              tma_load_3d(dst + chunk_off<C::NSTREAM>(t, h, b), &p.tm[C::NSTAT + t],
-                          &m->bar_full[stage], 64 * b, j0 + HB * h, bh);
+          for (int t = 0; t < nt; ++t)
+            tma_load_3d(dst + tile_off<C::NSTREAM>(t, b), &p.tm[C::NSTAT + t],
+                        &m->bar_full[stage], 64 * b, j0, bh);
         issued[stage] = st;
       }
       if (*abort_flag) {  // drain loads still in flight
@@ -222,15 +218,15 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
     }
   } else if (warp == kMmaWarp || warp == kMmaWarpY) {
     // ------------------------------------------------------------ MMA issuers
-    // Issuer X (warp 9) owns stage-A columns 0..63 of each half region and the
-    // accumulators it feeds from them; issuer Y (warp 10) owns columns 64..127.
-    // Each issuer reads only operand tiles inside the columns it overwrites
-    // itself, so the two never race on tensor memory and every accumulator
-    // has one issuer (fixed summation order).
+    // Issuer X (warp 9) owns stage-A columns 0..127 and the accumulators it
+    // feeds from them; issuer Y (warp 10) owns columns 128..255.  Each issuer
+    // reads operand tiles only inside the columns it overwrites itself, so the
+    // two never race on tensor memory and every accumulator has one issuer
+    // (fixed summation order).
     if (elect_lane0()) {
       const int role = warp == kMmaWarp ? 0 : 1;
-      constexpr uint32_t id_n32 = idesc_bf16(128, 32, false);
       constexpr uint32_t id_n64 = idesc_bf16(128, 64, false);
+      constexpr uint32_t id_n128 = idesc_bf16(128, 128, false);
       constexpr uint32_t id_b = idesc_bf16(128, C::DOUT, true);
       constexpr uint32_t id_b2 = idesc_bf16(128, 2 * C::DOUT, true);
       // descriptors are formed once; per MMA only the start-address field moves
@@ -238,68 +234,68 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
       auto sd = [&](int t, int k) -> uint64_t {
         return sd0 + (uint64_t)(((t * C::KB + k / 4) * (BM * 128) + (k % 4) * 32) >> 4);
       };
-      auto stage_a = [&](uint32_t sb, int h) {
+      auto stage_a = [&](uint32_t sb) {
         const uint64_t kd0 = sdesc_sw128(sb, 16, 1024);
         auto kd = [&](int t, int k) -> uint64_t {
-          return kd0 + (uint64_t)((chunk_off<C::NSTREAM>(t, h, k / 4) + (k % 4) * 32) >> 4);
+          return kd0 + (uint64_t)((tile_off<C::NSTREAM>(t, k / 4) + (k % 4) * 32) >> 4);
         };
-        const uint32_t R = tmem + kColA + 128 * h;
+        const uint32_t R = tmem + kColA;
         if constexpr (OP == RowOp::BobPass1) {
           // stationary: 0 Q, 1 U_Q, 2 dO ; stream: 0 K, 1 U_K, 2 V, 3 U_V
           if (role == 0) {
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)  // [S | F] = Q [K ; U_K]^T
-              mma_ss(R + 0, sd(0, k), kd(0, k), id_n64, k > 0);
+              mma_ss(R + 0, sd(0, k), kd(0, k), id_n128, k > 0);
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)  // F += U_Q K^T
-              mma_ss(R + 32, sd(1, k), kd(0, k), id_n32, 1);
+              mma_ss(R + 64, sd(1, k), kd(0, k), id_n64, 1);
           } else {
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)  // [dP | C] = dO [V ; U_V]^T
-              mma_ss(R + 64, sd(2, k), kd(2, k), id_n64, k > 0);
+              mma_ss(R + 128, sd(2, k), kd(2, k), id_n128, k > 0);
           }
         } else if constexpr (OP == RowOp::BwdDQ) {
           if (role == 0) {
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)  // S = Q K^T
-              mma_ss(R + 0, sd(0, k), kd(0, k), id_n32, k > 0);
+              mma_ss(R + 0, sd(0, k), kd(0, k), id_n64, k > 0);
           } else {
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)  // dP = dO V^T
-              mma_ss(R + 32, sd(1, k), kd(1, k), id_n32, k > 0);
+              mma_ss(R + 128, sd(1, k), kd(1, k), id_n64, k > 0);
           }
         } else {
           if (role == 0) {
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)  // S = Q K^T
-              mma_ss(R + 0, sd(0, k), kd(0, k), id_n32, k > 0);
+              mma_ss(R + 0, sd(0, k), kd(0, k), id_n64, k > 0);
           }
         }
       };
+      // stage B of half h: K-steps s = 2h, 2h+1 (16 streamed rows each)
       auto stage_b = [&](uint32_t sb, int h, int st) {
         if (st < first_b) return;
-        // MN-major views: rows 16*sub.. of streamed tensor t (box bo) ; the fused
-        // view spans [K | U_V] (second 64-wide block three chunks further on)
-        const uint64_t md0 = sdesc_sw128(sb, 2 * C::NSTREAM * kChunk, 1024);
-        const uint64_t mf0 = sdesc_sw128(sb, 3 * kChunk, 1024);
+        const uint64_t md0 = sdesc_sw128(sb, C::NSTREAM * BN * 128, 1024);
+        const uint64_t mf0 = sdesc_sw128(sb, 3 * BN * 128, 1024);  // [K | U_V]
 #pragma unroll
         for (int sub = 0; sub < 2; ++sub) {
+          const int s = 2 * h + sub;
           auto md = [&](int t, int bo) -> uint64_t {
-            return md0 + (uint64_t)((chunk_off<C::NSTREAM>(t, h, bo) + sub * 2048) >> 4);
+            return md0 + (uint64_t)((tile_off<C::NSTREAM>(t, bo) + s * 2048) >> 4);
           };
-          const uint32_t first = (st == first_b && h == 0 && sub == 0) ? 0u : 1u;
-          const uint32_t A = tmem + kColA + 128 * h + 16 * sub;
+          const uint32_t first = (st == first_b && s == 0) ? 0u : 1u;
+          const uint32_t A = tmem + kColA + 16 * s;
           if constexpr (OP == RowOp::BobPass1) {
             if (role == 0) {
               // [B | dOtil0] += P [K | U_V] ;  dOtil0 += (P o F) V
               const uint64_t fused =
-                  mf0 + (uint64_t)((chunk_off<C::NSTREAM>(0, h, split) + sub * 2048) >> 4);
+                  mf0 + (uint64_t)((tile_off<C::NSTREAM>(0, split) + s * 2048) >> 4);
               mma_ts(tmem + 0, A + 0, fused, id_b2, first);
               mma_ts(tmem + 64, A + 8, md(2, split), id_b, 1);
             } else {
-              mma_ts(tmem + 128, A + 64, md(0, split), id_b, first);  // Omega += (P o Pt0) K
-              mma_ts(tmem + 128, A + 72, md(1, split), id_b, 1);      //   += dS U_K
-              mma_ts(tmem + 192, A + 96, md(0, split), id_b, first);  // R += (P o dP) K
+              mma_ts(tmem + 128, A + 128, md(0, split), id_b, first);  // Omega += (P o Pt0) K
+              mma_ts(tmem + 128, A + 136, md(1, split), id_b, 1);      //   += dS U_K
+              mma_ts(tmem + 192, A + 192, md(0, split), id_b, first);  // R += (P o dP) K
             }
           } else if constexpr (OP == RowOp::BwdDQ) {
             if (role == 0) mma_ts(tmem + 0, A, md(0, 0), id_b, first);  // dQ += dS K
@@ -312,18 +308,12 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
                 mbar_wait(&m->bar_full[0], 0, abort_flag);
       if (ok) {
         tc_fence_after();
-        const uint32_t sb0 = smem_u32(s_stream);
-        stage_a(sb0, 0);
+        stage_a(smem_u32(s_stream));
         mma_commit(&m->bar_sa[0]);
-        stage_a(sb0, 1);
-        mma_commit(&m->bar_sa[1]);
       }
       for (int st = 0; ok && st < nsteps; ++st) {
         const int stage = st % C::NSTAGES;
         const uint32_t sb = smem_u32(s_stream + stage * C::STAGE_BYTES);
-        const int nstage = (st + 1) % C::NSTAGES;
-        const uint32_t nsb = smem_u32(s_stream + nstage * C::STAGE_BYTES);
-        const bool more = st + 1 < nsteps;
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
           if (!mbar_wait(&m->bar_ew[h], st & 1, abort_flag)) {
@@ -332,17 +322,15 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
           }
           tc_fence_after();
           stage_b(sb, h, st);
-          if (h == 1) mma_commit(&m->bar_empty[stage]);
-          if (more) {
-            if (h == 0 && !mbar_wait(&m->bar_full[nstage], ((st + 1) / C::NSTAGES) & 1,
-                                     abort_flag)) {
-              ok = false;
-              break;
-            }
-            tc_fence_after();
-            stage_a(nsb, h);
-            mma_commit(&m->bar_sa[h]);
-          }
+        }
+        if (!ok) break;
+        mma_commit(&m->bar_empty[stage]);
+        if (st + 1 < nsteps) {
+          const int nstage = (st + 1) % C::NSTAGES;
+          if (!mbar_wait(&m->bar_full[nstage], ((st + 1) / C::NSTAGES) & 1, abort_flag)) break;
+          tc_fence_after();
+          stage_a(smem_u32(s_stream + nstage * C::STAGE_BYTES));
+          mma_commit(&m->bar_sa[0]);
         }
       }
       mma_commit(&m->bar_acc);
@@ -369,12 +357,12 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
     float2 acc_a = splat(0.f), acc_e = splat(0.f);    // Pass 1 partial row sums
     bool ok = true;
     for (int st = 0; ok && st < nsteps; ++st) {
+      if (!mbar_wait(&m->bar_sa[0], st & 1, abort_flag)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
       for (int h = 0; h < 2; ++h) {
-        if (!mbar_wait(&m->bar_sa[h], st & 1, abort_flag)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
         if constexpr (OP == RowOp::Fwd) {
           if (st == ntiles && h == 0) {  // end of sweep 1: combine the warpgroups' (max, sum)
             s_xchg[wg * BM + r] = mrow;
@@ -388,18 +376,18 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
             L2 = row_ok ? mm + __log2f(l) : 0.f;
           }
         }
-        const int c0 = 16 * wg;                                // column within the half
-        const int j0 = (st % ntiles) * BN + HB * h + c0;       // first key of this thread's 16
+        const int c0 = HB * h + 16 * wg;                       // tile column of this thread's 16
+        const int j0 = (st % ntiles) * BN + c0;                // first key of this thread's 16
         const bool need_mask = (!row_ok) || (j0 + 16 > N) || (p.causal && j0 + 15 > gi);
         const int lim = need_mask ? (row_ok ? (p.causal ? min(N, gi + 1) : N) - j0 : 0) : 16;
-        const uint32_t R = ta + kColA + 128 * h + c0;  // this thread's 16 columns, region X0
+        const uint32_t R = ta + kColA + c0;  // this thread's 16 columns of the first stage-A tile
         const float2 sl2v = splat(sl2), nL2v = splat(-L2);
         if constexpr (OP == RowOp::BobPass1) {
           uint32_t rS[16], rF[16], rdP[16], rC[16];
           tmem_ld16(R + 0, rS);
-          tmem_ld16(R + 32, rF);
-          tmem_ld16(R + 64, rdP);
-          tmem_ld16(R + 96, rC);
+          tmem_ld16(R + 64, rF);
+          tmem_ld16(R + 128, rdP);
+          tmem_ld16(R + 192, rC);
           tmem_ld_wait(rS);
           reg_dep(rF);
           reg_dep(rdP);
@@ -429,16 +417,16 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
             odS[c / 2] = pack_bf16(ds.x, ds.y);
             oPdP[c / 2] = pack_bf16(pdp.x, pdp.y);
           }
-          // operand tiles: issuer X reads columns 0..63, issuer Y 64..127
+          // operand tiles: issuer X reads columns 0..127, issuer Y 128..255
           tmem_st8(R + 0, oP);
           tmem_st8(R + 8, oPF);
-          tmem_st8(R + 64, oPPt);
-          tmem_st8(R + 72, odS);
-          tmem_st8(R + 96, oPdP);
+          tmem_st8(R + 128, oPPt);
+          tmem_st8(R + 136, odS);
+          tmem_st8(R + 192, oPdP);
         } else if constexpr (OP == RowOp::BwdDQ) {
           uint32_t rS[16], rdP[16];
           tmem_ld16(R + 0, rS);
-          tmem_ld16(R + 32, rdP);
+          tmem_ld16(R + 128, rdP);
           tmem_ld_wait(rS);
           reg_dep(rdP);
           const float2 nDv = splat(-Dr);
@@ -642,10 +630,9 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
       if (lane == 0) {
         mbar_arrive_expect_tx(&m->bar_full[stage], C::TILE_BYTES);
         for (int b = 0; b < C::KB; ++b)
-          for (int h = 0; h < 2; ++h)
-            for (int t = 0; t < C::NSTREAM; ++t)
-              tma_load_3d(dst + chunk_off<C::NSTREAM>(t, h, b), &p.tm[C::NSTAT + t],
-                          &m->bar_full[stage], 64 * b, ib + HB * h, bh);
+          for (int t = 0; t < C::NSTREAM; ++t)
+            tma_load_3d(dst + tile_off<C::NSTREAM>(t, b), &p.tm[C::NSTAT + t],
+                        &m->bar_full[stage], 64 * b, ib, bh);
       }
       // negated row vectors of the streamed query rows:
       // [0] -L*log2e, [1] -D, [2] -alpha, [3] -E
@@ -676,71 +663,72 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
   } else if (warp == kMmaWarp || warp == kMmaWarpY) {
     // ------------------------------------------------------------ MMA issuers
     // Same ownership split as the row engine: issuer X owns stage-A columns
-    // 0..63 of each half region, issuer Y columns 64..127.
+    // 0..127, issuer Y columns 128..255.
     if (elect_lane0()) {
       const int role = warp == kMmaWarp ? 0 : 1;
-      constexpr uint32_t id_n32 = idesc_bf16(128, 32, false);
       constexpr uint32_t id_n64 = idesc_bf16(128, 64, false);
+      constexpr uint32_t id_n128 = idesc_bf16(128, 128, false);
       constexpr uint32_t id_b = idesc_bf16(128, D, true);
       const uint64_t sd0 = sdesc_sw128(smem_u32(s_stat), 16, 1024);
       auto sd = [&](int t, int k) -> uint64_t {
         return sd0 + (uint64_t)(((t * C::KB + k / 4) * (BM * 128) + (k % 4) * 32) >> 4);
       };
-      auto stage_a = [&](uint32_t sb, int h) {
+      auto stage_a = [&](uint32_t sb) {
         const uint64_t kd0 = sdesc_sw128(sb, 16, 1024);
         auto kd = [&](int t, int k) -> uint64_t {
-          return kd0 + (uint64_t)((chunk_off<C::NSTREAM>(t, h, k / 4) + (k % 4) * 32) >> 4);
+          return kd0 + (uint64_t)((tile_off<C::NSTREAM>(t, k / 4) + (k % 4) * 32) >> 4);
         };
-        const uint32_t R = tmem + kColA + 128 * h;
+        const uint32_t R = tmem + kColA;
         if constexpr (OP == ColOp::BobPass2) {
           // stationary: 0 K, 1 V, 2 U_K, 3 U_V ; stream: 0 Q, 1 U_Q, 2 dO
           if (role == 0) {
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)  // [S^T | F^T] = K [Q ; U_Q]^T
-              mma_ss(R + 0, sd(0, k), kd(0, k), id_n64, k > 0);
+              mma_ss(R + 0, sd(0, k), kd(0, k), id_n128, k > 0);
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)  // F^T += U_K Q^T
-              mma_ss(R + 32, sd(2, k), kd(0, k), id_n32, 1);
+              mma_ss(R + 64, sd(2, k), kd(0, k), id_n64, 1);
           } else {
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)  // dP^T = V dO^T
-              mma_ss(R + 64, sd(1, k), kd(2, k), id_n32, k > 0);
+              mma_ss(R + 128, sd(1, k), kd(2, k), id_n64, k > 0);
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)  // C^T = U_V dO^T
-              mma_ss(R + 96, sd(3, k), kd(2, k), id_n32, k > 0);
+              mma_ss(R + 192, sd(3, k), kd(2, k), id_n64, k > 0);
           }
         } else {
           // stationary: 0 K, 1 V ; stream: 0 Q, 1 dO
           if (role == 0) {
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)  // S^T = K Q^T
-              mma_ss(R + 0, sd(0, k), kd(0, k), id_n32, k > 0);
+              mma_ss(R + 0, sd(0, k), kd(0, k), id_n64, k > 0);
           } else {
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)  // dP^T = V dO^T
-              mma_ss(R + 64, sd(1, k), kd(1, k), id_n32, k > 0);
+              mma_ss(R + 128, sd(1, k), kd(1, k), id_n64, k > 0);
           }
         }
       };
       auto stage_b = [&](uint32_t sb, int h, int st) {
-        const uint64_t md0 = sdesc_sw128(sb, 2 * C::NSTREAM * kChunk, 1024);
+        const uint64_t md0 = sdesc_sw128(sb, C::NSTREAM * BN * 128, 1024);
 #pragma unroll
         for (int sub = 0; sub < 2; ++sub) {
+          const int s = 2 * h + sub;
           auto md = [&](int t) -> uint64_t {
-            return md0 + (uint64_t)((chunk_off<C::NSTREAM>(t, h, 0) + sub * 2048) >> 4);
+            return md0 + (uint64_t)((tile_off<C::NSTREAM>(t, 0) + s * 2048) >> 4);
           };
-          const uint32_t first = (st == 0 && h == 0 && sub == 0) ? 0u : 1u;
-          const uint32_t A = tmem + kColA + 128 * h + 16 * sub;
+          const uint32_t first = (st == 0 && s == 0) ? 0u : 1u;
+          const uint32_t A = tmem + kColA + 16 * s;
           if constexpr (OP == ColOp::BobPass2) {
             if (role == 0) {
-              mma_ts(tmem + D, A + 0, md(2), id_b, first);    // Vtil += (P o h)^T dO
+              mma_ts(tmem + D, A + 0, md(2), id_b, first);      // Vtil += (P o h)^T dO
             } else {
-              mma_ts(tmem + 0, A + 64, md(0), id_b, first);   // Ktil += Stil^T Q
-              mma_ts(tmem + 0, A + 72, md(1), id_b, 1);       //      += dS^T U_Q
+              mma_ts(tmem + 0, A + 128, md(0), id_b, first);    // Ktil += Stil^T Q
+              mma_ts(tmem + 0, A + 136, md(1), id_b, 1);        //      += dS^T U_Q
             }
           } else {
             if (role == 0) mma_ts(tmem + D, A + 0, md(1), id_b, first);   // dV += P^T dO
-            else mma_ts(tmem + 0, A + 64, md(0), id_b, first);            // dK += dS^T Q
+            else mma_ts(tmem + 0, A + 128, md(0), id_b, first);           // dK += dS^T Q
           }
         }
       };
@@ -748,18 +736,12 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
                 mbar_wait(&m->bar_full[0], 0, abort_flag);
       if (ok) {
         tc_fence_after();
-        const uint32_t sb0 = smem_u32(s_stream);
-        stage_a(sb0, 0);
+        stage_a(smem_u32(s_stream));
         mma_commit(&m->bar_sa[0]);
-        stage_a(sb0, 1);
-        mma_commit(&m->bar_sa[1]);
       }
       for (int st = 0; ok && st < nsteps; ++st) {
         const int stage = st % C::NSTAGES;
         const uint32_t sb = smem_u32(s_stream + stage * C::STAGE_BYTES);
-        const int nstage = (st + 1) % C::NSTAGES;
-        const uint32_t nsb = smem_u32(s_stream + nstage * C::STAGE_BYTES);
-        const bool more = st + 1 < nsteps;
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
           if (!mbar_wait(&m->bar_ew[h], st & 1, abort_flag)) {
@@ -768,17 +750,15 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
           }
           tc_fence_after();
           stage_b(sb, h, st);
-          if (h == 1) mma_commit(&m->bar_empty[stage]);
-          if (more) {
-            if (h == 0 && !mbar_wait(&m->bar_full[nstage], ((st + 1) / C::NSTAGES) & 1,
-                                     abort_flag)) {
-              ok = false;
-              break;
-            }
-            tc_fence_after();
-            stage_a(nsb, h);
-            mma_commit(&m->bar_sa[h]);
-          }
+        }
+        if (!ok) break;
+        mma_commit(&m->bar_empty[stage]);
+        if (st + 1 < nsteps) {
+          const int nstage = (st + 1) % C::NSTAGES;
+          if (!mbar_wait(&m->bar_full[nstage], ((st + 1) / C::NSTAGES) & 1, abort_flag)) break;
+          tc_fence_after();
+          stage_a(smem_u32(s_stream + nstage * C::STAGE_BYTES));
+          mma_commit(&m->bar_sa[0]);
         }
       }
       mma_commit(&m->bar_acc);
@@ -803,12 +783,12 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
       }
       const float* vec = reinterpret_cast<const float*>(s_stream + stage * C::STAGE_BYTES +
                                                         C::TILE_BYTES);
+      if (!mbar_wait(&m->bar_sa[0], st & 1, abort_flag)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
       for (int h = 0; h < 2; ++h) {
-        if (!mbar_wait(&m->bar_sa[h], st & 1, abort_flag)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
         const int c0 = 16 * wg;
         const int cv = HB * h + c0;                    // tile column of this thread's first
         const int ib = (first_tile + st) * BN + cv;    // first query row of this thread's 16
@@ -816,13 +796,13 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
         // valid query columns c satisfy  lo <= c < hi
         const int lo = p.causal ? gj - ib : 0;
         const int hi = row_ok ? N - ib : 0;
-        const uint32_t R = ta + kColA + 128 * h + c0;
+        const uint32_t R = ta + kColA + cv;
         if constexpr (OP == ColOp::BobPass2) {
           uint32_t rS[16], rF[16], rdP[16], rC[16];
           tmem_ld16(R + 0, rS);
-          tmem_ld16(R + 32, rF);
-          tmem_ld16(R + 64, rdP);
-          tmem_ld16(R + 96, rC);
+          tmem_ld16(R + 64, rF);
+          tmem_ld16(R + 128, rdP);
+          tmem_ld16(R + 192, rC);
           tmem_ld_wait(rS);
           reg_dep(rF);
           reg_dep(rdP);
@@ -851,14 +831,14 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
             oSt[c / 2] = pack_bf16(stl.x, stl.y);
             odS[c / 2] = pack_bf16(ds.x, ds.y);
           }
-          // operand tiles: issuer X reads columns 0..63, issuer Y 64..127
+          // operand tiles: issuer X reads columns 0..127, issuer Y 128..255
           tmem_st8(R + 0, oPh);
-          tmem_st8(R + 64, oSt);
-          tmem_st8(R + 72, odS);
+          tmem_st8(R + 128, oSt);
+          tmem_st8(R + 136, odS);
         } else {
           uint32_t rS[16], rdP[16];
           tmem_ld16(R + 0, rS);
-          tmem_ld16(R + 64, rdP);
+          tmem_ld16(R + 128, rdP);
           tmem_ld_wait(rS);
           reg_dep(rdP);
           uint32_t oP[8], odS[8];
@@ -876,7 +856,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
             odS[c / 2] = pack_bf16(ds.x, ds.y);
           }
           tmem_st8(R + 0, oP);
-          tmem_st8(R + 64, odS);
+          tmem_st8(R + 128, odS);
         }
         tmem_st_wait();
         tc_fence_before();

@@ -30,7 +30,7 @@ enum class ColOp { BwdDKDV, BobPass2 };
 
 // ---------------------------------------------------------------- parameters
 struct EngineParams {
-  CUtensorMap tm[7];  // stationary maps first (box rows BM), then streamed (box rows HB)
+  CUtensorMap tm[7];  // stationary maps first (box rows BM), then streamed (box rows BN)
   const __nv_bfloat16* o;     // forward output O (row engine: D and dOtil)
   const __nv_bfloat16* dout;  // dO (row engine: D = do.o)
   const float* lse;           // natural-log L [BH, N]

@@ -118,7 +118,7 @@ int run_pass1(const fbob_shape* s, const void* q, const void* k, const void* v, 
   for (int t = 0; t < 3; ++t)
     if (!make_map(&p.tm[t], stat[t], BH, N, d, BM)) return FBOB_ERR_CUDA;
   for (int t = 0; t < 4; ++t)
-    if (!make_map(&p.tm[3 + t], strm[t], BH, N, d, HB)) return FBOB_ERR_CUDA;
+    if (!make_map(&p.tm[3 + t], strm[t], BH, N, d, BN)) return FBOB_ERR_CUDA;
   p.o = static_cast<const __nv_bfloat16*>(o);
   p.dout = static_cast<const __nv_bfloat16*>(dout);
   p.lse = lse;
@@ -140,7 +140,7 @@ int run_pass2(const fbob_shape* s, const void* q, const void* k, const void* v, 
   for (int t = 0; t < 4; ++t)
     if (!make_map(&p.tm[t], stat[t], BH, N, d, BM)) return FBOB_ERR_CUDA;
   for (int t = 0; t < 3; ++t)
-    if (!make_map(&p.tm[4 + t], strm[t], BH, N, d, HB)) return FBOB_ERR_CUDA;
+    if (!make_map(&p.tm[4 + t], strm[t], BH, N, d, BN)) return FBOB_ERR_CUDA;
   p.lse = lse;
   p.vec_in = row_stats;
   p.out0 = static_cast<__nv_bfloat16*>(k_bar);
@@ -194,8 +194,8 @@ int fbob_attn_fwd(const fbob_shape* s, const void* q, const void* k, const void*
   if (rc != FBOB_OK) return rc;
   EngineParams p = base_params(s);
   const int64_t BH = s->B * s->H;
-  if (!make_map(&p.tm[0], q, BH, s->N, s->d, BM) || !make_map(&p.tm[1], k, BH, s->N, s->d, HB) ||
-      !make_map(&p.tm[2], v, BH, s->N, s->d, HB))
+  if (!make_map(&p.tm[0], q, BH, s->N, s->d, BM) || !make_map(&p.tm[1], k, BH, s->N, s->d, BN) ||
+      !make_map(&p.tm[2], v, BH, s->N, s->d, BN))
     return FBOB_ERR_CUDA;
   p.out0 = static_cast<__nv_bfloat16*>(o);
   p.vec_out = lse;
@@ -226,7 +226,7 @@ int fbob_attn_bwd(const fbob_shape* s, const void* q, const void* k, const void*
   // dQ and D: row-block pass (writes D, which the column pass reads)
   EngineParams p = base_params(s);
   if (!make_map(&p.tm[0], q, BH, N, d, BM) || !make_map(&p.tm[1], dout, BH, N, d, BM) ||
-      !make_map(&p.tm[2], k, BH, N, d, HB) || !make_map(&p.tm[3], v, BH, N, d, HB))
+      !make_map(&p.tm[2], k, BH, N, d, BN) || !make_map(&p.tm[3], v, BH, N, d, BN))
     return FBOB_ERR_CUDA;
   p.o = static_cast<const __nv_bfloat16*>(o);
   p.dout = static_cast<const __nv_bfloat16*>(dout);
@@ -239,7 +239,7 @@ int fbob_attn_bwd(const fbob_shape* s, const void* q, const void* k, const void*
   // dK and dV: column-block pass
   EngineParams c = base_params(s);
   if (!make_map(&c.tm[0], k, BH, N, d, BM) || !make_map(&c.tm[1], v, BH, N, d, BM) ||
-      !make_map(&c.tm[2], q, BH, N, d, HB) || !make_map(&c.tm[3], dout, BH, N, d, HB))
+      !make_map(&c.tm[2], q, BH, N, d, BN) || !make_map(&c.tm[3], dout, BH, N, d, BN))
     return FBOB_ERR_CUDA;
   c.lse = lse;
   c.vec_in = dstat;
