@@ -33,6 +33,12 @@
  *             bounded, and on expiry the kernel records FBOB_ERR_DEVICE_TIMEOUT
  *             in the device error word and exits cleanly; fbob_device_status()
  *             reports it.
+ *  Debug      Two environment variables, read at every call, control the
+ *             bounded waits: FBOB_WAIT_LIMIT_MS (1..60000, default 2000) is the
+ *             limit of each wait, and FBOB_INJECT_STALL=1 injects a stall (the
+ *             kernels load nothing, every wait expires, the outputs are left
+ *             unspecified and fbob_device_status() then reports
+ *             FBOB_ERR_DEVICE_TIMEOUT) for testing failure detection.
  *  Determinism  No floating-point atomics; every output element has one
  *             writer, so results are bitwise reproducible run to run.
  */

@@ -20,6 +20,7 @@ HEADER = os.path.join(os.path.dirname(_HERE), "include", "fbob.h")
 FBOB_OK = 0
 STATUS = {0: "FBOB_OK", 1: "FBOB_ERR_INVALID_ARGUMENT", 2: "FBOB_ERR_UNSUPPORTED",
           3: "FBOB_ERR_CUDA", 4: "FBOB_ERR_DEVICE_TIMEOUT", 5: "FBOB_ERR_DEVICE_FAULT"}
+STATUS_CODES = {v: k for k, v in STATUS.items()}
 
 
 class FbobError(RuntimeError):

@@ -53,7 +53,8 @@ struct Misc {
   uint64_t bar_ew[2];
   uint64_t bar_acc;
   uint32_t tmem_base;
-  int abort_flag;
+  uint32_t pad;
+  WaitCtl wctl;
 };
 
 __device__ __forceinline__ uint32_t lane_base_addr(uint32_t tmem_base, int warp) {
@@ -161,7 +162,8 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
   const int first_b = OP == RowOp::Fwd ? ntiles : 0;  // first step with stage-B MMAs
 
   if (tid == 0) {
-    m->abort_flag = 0;
+    m->wctl.abort = 0;
+    m->wctl.limit_ns = p.wait_limit_ns;
     mbar_init(&m->bar_stat, 1);
     for (int s = 0; s < C::NSTAGES; ++s) {
       mbar_init(&m->bar_full[s], 1);
@@ -182,11 +184,14 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = m->tmem_base;
-  volatile int* abort_flag = &m->abort_flag;
+  WaitCtl* wctl = &m->wctl;
+  volatile int* abort_flag = &m->wctl.abort;
 
   if (warp == kProducerWarp) {
     // ------------------------------------------------------------ producer
-    if (elect_lane0()) {
+    // p.inject_stall (host-side fault injection, off by default): issue no
+    // loads at all, so every consumer wait runs into its bounded limit.
+    if (elect_lane0() && !p.inject_stall) {
       for (int t = 0; t < C::NSTAT + C::NSTREAM; ++t) tma_prefetch_desc(&p.tm[t]);
       mbar_arrive_expect_tx(&m->bar_stat, C::STAT_BYTES);
       for (int t = 0; t < C::NSTAT; ++t)
@@ -197,7 +202,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
       for (int st = 0; st < nsteps; ++st) {
         const int stage = st % C::NSTAGES;
         if (st >= C::NSTAGES) {
-          if (!mbar_wait(&m->bar_empty[stage], ((st / C::NSTAGES) - 1) & 1, abort_flag)) break;
+          if (!mbar_wait(&m->bar_empty[stage], ((st / C::NSTAGES) - 1) & 1, wctl)) break;
         }
         const int j0 = (st % ntiles) * BN;
         const bool k_only = (OP == RowOp::Fwd) && st < ntiles;
@@ -304,8 +309,8 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
           }
         }
       };
-      bool ok = mbar_wait(&m->bar_stat, 0, abort_flag) &&
-                mbar_wait(&m->bar_full[0], 0, abort_flag);
+      bool ok = mbar_wait(&m->bar_stat, 0, wctl) &&
+                mbar_wait(&m->bar_full[0], 0, wctl);
       if (ok) {
         tc_fence_after();
         stage_a(smem_u32(s_stream));
@@ -316,7 +321,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         const uint32_t sb = smem_u32(s_stream + stage * C::STAGE_BYTES);
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
-          if (!mbar_wait(&m->bar_ew[h], st & 1, abort_flag)) {
+          if (!mbar_wait(&m->bar_ew[h], st & 1, wctl)) {
             ok = false;
             break;
           }
@@ -327,7 +332,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         mma_commit(&m->bar_empty[stage]);
         if (st + 1 < nsteps) {
           const int nstage = (st + 1) % C::NSTAGES;
-          if (!mbar_wait(&m->bar_full[nstage], ((st + 1) / C::NSTAGES) & 1, abort_flag)) break;
+          if (!mbar_wait(&m->bar_full[nstage], ((st + 1) / C::NSTAGES) & 1, wctl)) break;
           tc_fence_after();
           stage_a(smem_u32(s_stream + nstage * C::STAGE_BYTES));
           mma_commit(&m->bar_sa[0]);
@@ -357,7 +362,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
     float2 acc_a = splat(0.f), acc_e = splat(0.f);    // Pass 1 partial row sums
     bool ok = true;
     for (int st = 0; ok && st < nsteps; ++st) {
-      if (!mbar_wait(&m->bar_sa[0], st & 1, abort_flag)) {
+      if (!mbar_wait(&m->bar_sa[0], st & 1, wctl)) {
         ok = false;
         break;
       }
@@ -482,7 +487,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
       }
     }
     // ---------------------------------------------------------- epilogue
-    if (ok) ok = mbar_wait(&m->bar_acc, 0, abort_flag);
+    if (ok) ok = mbar_wait(&m->bar_acc, 0, wctl);
     if (ok && *abort_flag) ok = false;
     tc_fence_after();
     if constexpr (OP == RowOp::BobPass1) {
@@ -585,7 +590,8 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
   const int nsteps = ntotal - first_tile;
 
   if (tid == 0) {
-    m->abort_flag = 0;
+    m->wctl.abort = 0;
+    m->wctl.limit_ns = p.wait_limit_ns;
     mbar_init(&m->bar_stat, 1);
     for (int s = 0; s < C::NSTAGES; ++s) {
       mbar_init(&m->bar_full[s], 1 + 32);  // TMA bytes + 32 producer lanes' row vectors
@@ -606,12 +612,15 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = m->tmem_base;
-  volatile int* abort_flag = &m->abort_flag;
+  WaitCtl* wctl = &m->wctl;
+  volatile int* abort_flag = &m->wctl.abort;
 
   if (warp == kProducerWarp) {
     // ------------------------------------------------------------ producer
+    // (p.inject_stall: no loads at all, as in the row engine)
     const int lane = tid & 31;
-    if (lane == 0) {
+    const int nprod = p.inject_stall ? 0 : nsteps;
+    if (lane == 0 && !p.inject_stall) {
       for (int t = 0; t < C::NSTAT + C::NSTREAM; ++t) tma_prefetch_desc(&p.tm[t]);
       mbar_arrive_expect_tx(&m->bar_stat, C::STAT_BYTES);
       for (int t = 0; t < C::NSTAT; ++t)
@@ -620,10 +629,10 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
                       bh);
     }
     int issued[4] = {-1, -1, -1, -1};
-    for (int st = 0; st < nsteps; ++st) {
+    for (int st = 0; st < nprod; ++st) {
       const int stage = st % C::NSTAGES;
       if (st >= C::NSTAGES) {
-        if (!mbar_wait(&m->bar_empty[stage], ((st / C::NSTAGES) - 1) & 1, abort_flag)) break;
+        if (!mbar_wait(&m->bar_empty[stage], ((st / C::NSTAGES) - 1) & 1, wctl)) break;
       }
       const int ib = (first_tile + st) * BN;
       uint8_t* dst = s_stream + stage * C::STAGE_BYTES;
@@ -732,8 +741,8 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
           }
         }
       };
-      bool ok = mbar_wait(&m->bar_stat, 0, abort_flag) &&
-                mbar_wait(&m->bar_full[0], 0, abort_flag);
+      bool ok = mbar_wait(&m->bar_stat, 0, wctl) &&
+                mbar_wait(&m->bar_full[0], 0, wctl);
       if (ok) {
         tc_fence_after();
         stage_a(smem_u32(s_stream));
@@ -744,7 +753,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
         const uint32_t sb = smem_u32(s_stream + stage * C::STAGE_BYTES);
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
-          if (!mbar_wait(&m->bar_ew[h], st & 1, abort_flag)) {
+          if (!mbar_wait(&m->bar_ew[h], st & 1, wctl)) {
             ok = false;
             break;
           }
@@ -755,7 +764,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
         mma_commit(&m->bar_empty[stage]);
         if (st + 1 < nsteps) {
           const int nstage = (st + 1) % C::NSTAGES;
-          if (!mbar_wait(&m->bar_full[nstage], ((st + 1) / C::NSTAGES) & 1, abort_flag)) break;
+          if (!mbar_wait(&m->bar_full[nstage], ((st + 1) / C::NSTAGES) & 1, wctl)) break;
           tc_fence_after();
           stage_a(smem_u32(s_stream + nstage * C::STAGE_BYTES));
           mma_commit(&m->bar_sa[0]);
@@ -777,13 +786,13 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
     for (int st = 0; ok && st < nsteps; ++st) {
       const int stage = st % C::NSTAGES;
       // the row vectors were written by the producer: acquire them explicitly
-      if (!mbar_wait(&m->bar_full[stage], (st / C::NSTAGES) & 1, abort_flag)) {
+      if (!mbar_wait(&m->bar_full[stage], (st / C::NSTAGES) & 1, wctl)) {
         ok = false;
         break;
       }
       const float* vec = reinterpret_cast<const float*>(s_stream + stage * C::STAGE_BYTES +
                                                         C::TILE_BYTES);
-      if (!mbar_wait(&m->bar_sa[0], st & 1, abort_flag)) {
+      if (!mbar_wait(&m->bar_sa[0], st & 1, wctl)) {
         ok = false;
         break;
       }
@@ -863,7 +872,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
         mbar_arrive(&m->bar_ew[h]);
       }
     }
-    if (ok) ok = mbar_wait(&m->bar_acc, 0, abort_flag);
+    if (ok) ok = mbar_wait(&m->bar_acc, 0, wctl);
     if (ok && *abort_flag) ok = false;
     tc_fence_after();
     if (ok) {

@@ -44,6 +44,8 @@ struct EngineParams {
   int causal;
   float scale;
   long long bhn;  // BH * N (row_stats plane stride)
+  unsigned long long wait_limit_ns;  // bound of every device-side wait
+  int inject_stall;                  // fault injection: producers issue nothing
 };
 
 // ---------------------------------------------------------------- configs

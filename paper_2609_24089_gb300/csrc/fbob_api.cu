@@ -5,6 +5,7 @@
 
 #include <atomic>
 #include <cmath>
+#include <cstdlib>
 #include <cstring>
 #include <mutex>
 
@@ -91,6 +92,21 @@ int check_ptrs(const void* const* in, const int64_t* in_bytes, int nin, void* co
   return FBOB_OK;
 }
 
+// Bound of every device-side wait (FBOB_WAIT_LIMIT_MS, default 2000 ms) and
+// the host-side stall injection used to test failure detection
+// (FBOB_INJECT_STALL=1: the kernels' producers issue no loads, so every wait
+// expires and the call reports FBOB_ERR_DEVICE_TIMEOUT).  Read at each call.
+void debug_controls(EngineParams* p) {
+  unsigned long long ms = 2000;
+  if (const char* e = std::getenv("FBOB_WAIT_LIMIT_MS")) {
+    const long long v = std::atoll(e);
+    if (v > 0 && v <= 60000) ms = (unsigned long long)v;
+  }
+  p->wait_limit_ns = ms * 1000000ull;
+  const char* inj = std::getenv("FBOB_INJECT_STALL");
+  p->inject_stall = (inj && inj[0] == '1') ? 1 : 0;
+}
+
 EngineParams base_params(const fbob_shape* s) {
   EngineParams p;
   std::memset(&p, 0, sizeof(p));
@@ -99,6 +115,7 @@ EngineParams base_params(const fbob_shape* s) {
   p.causal = s->causal;
   p.scale = s->scale;
   p.bhn = s->B * s->H * s->N;
+  debug_controls(&p);
   return p;
 }
 

@@ -20,11 +20,15 @@ namespace fbob {
 // reads and clears every copy (see launch.h).
 static __device__ uint32_t g_fbob_error_word = 0;
 
-// A single bounded wait never legitimately lasts long: every wait in these
-// kernels is a CTA-local producer/consumer hand-off of a few microseconds.
-#ifndef FBOB_WAIT_LIMIT_NS
-#define FBOB_WAIT_LIMIT_NS 2000000000ull
-#endif
+// Per-CTA wait control in shared memory.  A single bounded wait never
+// legitimately lasts long: every wait in these kernels is a CTA-local
+// producer/consumer hand-off of a few microseconds; the limit (default 2 s)
+// comes with the launch.
+struct WaitCtl {
+  int abort;  // set once any thread of the CTA gave up
+  int pad;
+  unsigned long long limit_ns;
+};
 
 __device__ __forceinline__ uint64_t global_timer_ns() {
   uint64_t t;
@@ -69,20 +73,21 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
-// Bounded wait on phase `parity`.  `abort` is a CTA-shared flag: once any
-// thread of the CTA has given up, every later wait returns false at once so
-// all roles reach the teardown.  On expiry the error word gets the timeout bit.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
+// Bounded wait on phase `parity`.  Once any thread of the CTA has given up
+// (ctl->abort), every later wait returns false at once so all roles reach the
+// teardown.  On expiry the error word gets the timeout bit.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, WaitCtl* ctl) {
   if (mbar_try_wait(bar, parity)) return true;
+  volatile WaitCtl* c = ctl;
   const uint64_t t0 = global_timer_ns();
   uint32_t n = 0;
   while (true) {
     if (mbar_try_wait(bar, parity)) return true;
     if ((++n & 63u) == 0) {
-      if (*abort) return false;
-      if (global_timer_ns() - t0 > FBOB_WAIT_LIMIT_NS) {
+      if (c->abort) return false;
+      if (global_timer_ns() - t0 > c->limit_ns) {
         atomicOr(&g_fbob_error_word, kDevErrTimeout);
-        *abort = 1;
+        c->abort = 1;
         return false;
       }
     }

@@ -7,6 +7,8 @@ max |got - ref| <= 5e-2 * max |ref|.
 """
 from __future__ import annotations
 
+import os
+
 import numpy as np
 
 import oracle
@@ -15,6 +17,10 @@ from paper_2609_24089_gb300 import synth
 
 REL_FRO = 1e-2
 MAX_ABS = 5e-2
+
+# every check appends (test id, tensor, rel_fro, max_abs/max|ref|); the session
+# hook in conftest.py writes them out when FBOB_PARITY_REPORT names a file
+RECORD = []
 
 
 def torch():
@@ -47,6 +53,7 @@ def check(name, got, ref, rel=REL_FRO, mx=MAX_ABS, zero_atol=1e-6):
         return 0.0, 0.0
     r = np.linalg.norm(got - ref) / np.linalg.norm(ref)
     m = np.abs(got - ref).max() / scale
+    RECORD.append((os.environ.get("PYTEST_CURRENT_TEST", "").split(" ")[0], name, float(r), float(m)))
     assert r <= rel and m <= mx, f"{name}: rel_fro={r:.3e} (<= {rel}) max_abs/max|ref|={m:.3e} (<= {mx})"
     return r, m
 

@@ -162,3 +162,25 @@ def test_single_key_degenerate(d, causal):
         G.check("dobar", r["dobar"][0, h, 0], uv)
     assert np.abs(r["kbar"]).max() <= 1e-4 * scale * np.abs(X["q"]).max() * np.abs(X["gv"]).max() * d
     assert np.abs(r["vbar"]).max() <= 1e-4 * np.abs(X["dout"]).max() * np.abs(X["gq"]).max() * d
+
+
+def test_bounded_wait_timeout_is_reported_and_context_survives(monkeypatch):
+    """Failure detection without a GPU fault: with the producers' loads
+    suppressed (FBOB_INJECT_STALL=1) every consumer wait runs into its bounded
+    limit; the kernels record FBOB_ERR_DEVICE_TIMEOUT, release tensor memory
+    and exit, and the next call on the same context computes correct results."""
+    B, H, N, d = 1, 1, 256, 64
+    bits = G.inputs(B, H, N, d, seed=77)
+    scale = 1 / np.sqrt(d)
+    o_l = G.oracle_o_l(bits, scale, False)
+    monkeypatch.setenv("FBOB_WAIT_LIMIT_MS", "50")
+    monkeypatch.setenv("FBOB_INJECT_STALL", "1")
+    r = G.run_bob(bits, scale, False, o_l=o_l)
+    assert r["status"] == fbob.STATUS_CODES["FBOB_ERR_DEVICE_TIMEOUT"]
+    monkeypatch.delenv("FBOB_INJECT_STALL")
+    monkeypatch.delenv("FBOB_WAIT_LIMIT_MS")
+    r = G.run_bob(bits, scale, False, o_l=o_l)
+    assert r["status"] == 0
+    ref = oracle.bob(*(G.f64(bits[n]) for n in synth.NAMES), scale, False)
+    for name, x in zip(("qbar", "kbar", "vbar", "dobar"), ref):
+        G.check(name, r[name], x)
