@@ -16,24 +16,35 @@
 //   warp 8     TMA producer: stationary tiles once, then a ring of NSTAGES
 //              stream stages (mbarrier full/empty pairs).  In the column engine
 //              it also stages the streamed rows' fp32 row vectors in shared memory.
-//   warps 9,10 MMA issuers X and Y (one lane each; warp 9 also allocates
-//              TMEM).  A single thread issues at most one tcgen05.mma about
-//              every 53 cycles, so the tile's MMAs are split between two
-//              issuers by tensor-memory ownership: X owns stage-A columns
-//              0..63 of each half region, Y columns 64..127, and each reads
-//              operand tiles only inside its own columns.
+//   warp 9     MMA issuer X (one lane; the warp also allocates TMEM).
+//   warp 10    MMA issuer Y (one lane).
 //
-// Per streamed tile: stage A (scores and friends, fp32 in the 256 stage-A
-// columns of TMEM; A and B from shared memory; tensors streamed side by side
-// -- K and U_K, V and U_V, Q and U_Q -- form one 128-row B operand, so the
-// main stage-A MMAs have N = 128) -> elementwise in two halves of 32 columns
-// (TMEM -> registers -> bf16 operand tiles written back into columns already
-// read) -> stage B per half (accumulators += bf16 tile (TMEM) x streamed tile
-// (shared memory, MN-major)).  Stage B of half 0 runs while the elementwise
-// warps work on half 1.  Accumulators live at TMEM columns 0..255.
+// Tensor memory (512 columns): accumulators at 0..255; stage-A area "SF" at
+// 256..383 (scores, and F in the BoB passes), owned by issuer X; stage-A area
+// "DC" at 384..511 (dP, and C in the BoB passes), owned by issuer Y.
+//
+// Per streamed tile t:
+//   X  issues SF(t) as soon as the elementwise warps have copied SF(t-1)
+//      into registers, so the next tile's largest stage-A contractions run
+//      while the elementwise warps still work on tile t.
+//   Y  issues DC(t) (per 32-column half in Pass 1) and all stage-B MMAs.
+//   elementwise: copy SF to registers and release it; then per half read DC,
+//      compute, and write the bf16 operand tiles of stage B over the DC
+//      columns just read; stage B of half 0 overlaps the elementwise work on
+//      half 1.
+// Every TMEM region has one writer issuer and the MMAs reading a region are
+// issued by that same thread, so no cross-issuer hazard exists and every
+// accumulator is summed in a fixed order (bitwise reproducible results).
+//
+// A single thread issues at most one tcgen05.mma about every 53 cycles and
+// the tensor core needs N >= 128 per instruction to stay busy, so MMAs that
+// share an operand are fused to N = 128 ([S|F] = Q [K;U_K]^T,
+// [B|dOtil0] += P [K|U_V], [G|Omega] += dS [K|U_K], ...).
 //
 // Shared memory: stationary tensors as 128-row x 64-column swizzled boxes;
-// each stream stage as 64-row x 64-column boxes ordered (box, tensor).
+// each stream stage as, per 64-column box, 64-row tiles in tensor order.  In
+// Pass 1, V and U_V are stored as 32-row chunks V_0 U_V_0 V_1 U_V_1 so that
+// [V_h ; U_V_h] is one 64-row operand.
 //
 // Every wait is bounded (tc_ptx.cuh); on expiry the CTA records a timeout in
 // the device error word, drains its own asynchronous work and exits.
@@ -44,12 +55,17 @@
 
 namespace fbob {
 
+constexpr uint32_t kColSF = 256;  // stage-A area of issuer X
+constexpr uint32_t kColDC = 384;  // stage-A area of issuer Y
+
 // Shared-memory bookkeeping block (in the MISC area).
 struct Misc {
   uint64_t bar_stat;
   uint64_t bar_full[4];
   uint64_t bar_empty[4];
-  uint64_t bar_sa[2];
+  uint64_t bar_sa_sf;   // X's stage A of a tile completed
+  uint64_t bar_sf_free; // elementwise warps copied SF to registers
+  uint64_t bar_sa_dc[2];
   uint64_t bar_ew[2];
   uint64_t bar_acc;
   uint32_t tmem_base;
@@ -61,10 +77,15 @@ __device__ __forceinline__ uint32_t lane_base_addr(uint32_t tmem_base, int warp)
   return tmem_base + ((uint32_t)(32 * (warp & 3)) << 16);
 }
 
-// Offset of streamed tensor t, 64-column box b inside a stream stage.
-template <int NSTREAM>
-__device__ __forceinline__ uint32_t tile_off(int t, int b) {
-  return (uint32_t)((b * NSTREAM + t) * (BN * 128));
+// Offset inside a stream stage of rows 32h .. 32h+31 of streamed tensor t,
+// 64-column box b.  Tensors are 64-row tiles in order, except that with
+// kHalvesVUV (Pass 1) tensors 2 and 3 (V, U_V) are interleaved 32-row chunks.
+template <int NSTREAM, bool kHalvesVUV>
+__device__ __forceinline__ uint32_t soff(int t, int h, int b) {
+  constexpr int kBox = NSTREAM * BN * 128;
+  if (kHalvesVUV && t >= 2)
+    return (uint32_t)(b * kBox + 2 * BN * 128 + h * 2 * kChunk + (t - 2) * kChunk);
+  return (uint32_t)(b * kBox + t * BN * 128 + h * kChunk);
 }
 
 // Second-chance drain used only on the abort path: waits (bounded, ignoring
@@ -123,7 +144,7 @@ __device__ __forceinline__ float row_dot(const __nv_bfloat16* a, const __nv_bflo
   return acc;
 }
 
-// p = exp2(s * sl2 - L2) for a pair of scores; masked entries are 0.
+// p = exp2(s * sl2 - L2) for a pair of scores.
 __device__ __forceinline__ float2 probs2(float2 s, float2 sl2, float2 nL2) {
   const float2 a = __ffma2_rn(s, sl2, nL2);
   return make_float2(ex2(a.x), ex2(a.y));
@@ -133,6 +154,8 @@ __device__ __forceinline__ float2 probs2(float2 s, float2 sl2, float2 nL2) {
 template <RowOp OP, int D>
 __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant__ EngineParams p) {
   using C = RowCfg<OP, D>;
+  constexpr bool kBob = OP == RowOp::BobPass1;
+  constexpr bool kDcHalves = kBob;  // Pass 1 issues DC per 32-column half
   extern __shared__ __align__(1024) uint8_t smem[];
   uint8_t* s_stat = smem;
   uint8_t* s_stream = smem + C::STAT_BYTES;
@@ -169,8 +192,10 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
       mbar_init(&m->bar_full[s], 1);
       mbar_init(&m->bar_empty[s], 2);  // released by both MMA issuers
     }
+    mbar_init(&m->bar_sa_sf, 1);
+    mbar_init(&m->bar_sf_free, kEwThreads);
     for (int h = 0; h < 2; ++h) {
-      mbar_init(&m->bar_sa[h], 2);  // one commit per MMA issuer
+      mbar_init(&m->bar_sa_dc[h], 1);
       mbar_init(&m->bar_ew[h], kEwThreads);
     }
     mbar_init(&m->bar_acc, 2);
@@ -210,9 +235,16 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         uint8_t* dst = s_stream + stage * C::STAGE_BYTES;
         mbar_arrive_expect_tx(&m->bar_full[stage], nt * C::KB * BN * 128);
         for (int b = 0; b < C::KB; ++b)
-          for (int t = 0; t < nt; ++t)
-            tma_load_3d(dst + tile_off<C::NSTREAM>(t, b), &p.tm[C::NSTAT + t],
-                        &m->bar_full[stage], 64 * b, j0, bh);
+          for (int t = 0; t < nt; ++t) {
+            if (kBob && t >= 2) {  // 32-row chunks (map box rows HB)
+              for (int h = 0; h < 2; ++h)
+                tma_load_3d(dst + soff<C::NSTREAM, kBob>(t, h, b), &p.tm[C::NSTAT + t],
+                            &m->bar_full[stage], 64 * b, j0 + HB * h, bh);
+            } else {
+              tma_load_3d(dst + soff<C::NSTREAM, kBob>(t, 0, b), &p.tm[C::NSTAT + t],
+                          &m->bar_full[stage], 64 * b, j0, bh);
+            }
+          }
         issued[stage] = st;
       }
       if (*abort_flag) {  // drain loads still in flight
@@ -223,13 +255,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
     }
   } else if (warp == kMmaWarp || warp == kMmaWarpY) {
     // ------------------------------------------------------------ MMA issuers
-    // Issuer X (warp 9) owns stage-A columns 0..127 and the accumulators it
-    // feeds from them; issuer Y (warp 10) owns columns 128..255.  Each issuer
-    // reads operand tiles only inside the columns it overwrites itself, so the
-    // two never race on tensor memory and every accumulator has one issuer
-    // (fixed summation order).
     if (elect_lane0()) {
-      const int role = warp == kMmaWarp ? 0 : 1;
       constexpr uint32_t id_n64 = idesc_bf16(128, 64, false);
       constexpr uint32_t id_n128 = idesc_bf16(128, 128, false);
       constexpr uint32_t id_b = idesc_bf16(128, C::DOUT, true);
@@ -239,107 +265,130 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
       auto sd = [&](int t, int k) -> uint64_t {
         return sd0 + (uint64_t)(((t * C::KB + k / 4) * (BM * 128) + (k % 4) * 32) >> 4);
       };
-      auto stage_a = [&](uint32_t sb) {
-        const uint64_t kd0 = sdesc_sw128(sb, 16, 1024);
-        auto kd = [&](int t, int k) -> uint64_t {
-          return kd0 + (uint64_t)((tile_off<C::NSTREAM>(t, k / 4) + (k % 4) * 32) >> 4);
-        };
-        const uint32_t R = tmem + kColA;
-        if constexpr (OP == RowOp::BobPass1) {
-          // stationary: 0 Q, 1 U_Q, 2 dO ; stream: 0 K, 1 U_K, 2 V, 3 U_V
-          if (role == 0) {
+      // K-major view of streamed rows 32h.. (64 of them) of tensor t, K-step k
+      auto kd = [&](uint64_t kd0, int t, int h, int k) -> uint64_t {
+        return kd0 + (uint64_t)((soff<C::NSTREAM, kBob>(t, h, k / 4) + (k % 4) * 32) >> 4);
+      };
+      if (warp == kMmaWarp) {
+        // ---------------- issuer X: SF(t) = scores (and F) of tile t
+        bool ok = mbar_wait(&m->bar_stat, 0, wctl);
+        for (int st = 0; ok && st < nsteps; ++st) {
+          if (st > 0 && !mbar_wait(&m->bar_sf_free, (st - 1) & 1, wctl)) break;
+          const int stage = st % C::NSTAGES;
+          if (!mbar_wait(&m->bar_full[stage], (st / C::NSTAGES) & 1, wctl)) break;
+          tc_fence_after();
+          const uint64_t kd0 = sdesc_sw128(smem_u32(s_stream + stage * C::STAGE_BYTES), 16, 1024);
+          const uint32_t R = tmem + kColSF;
+          if constexpr (kBob) {
+            // stationary: 0 Q, 1 U_Q, 2 dO ; stream: 0 K, 1 U_K, 2 V, 3 U_V
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)  // [S | F] = Q [K ; U_K]^T
-              mma_ss(R + 0, sd(0, k), kd(0, k), id_n128, k > 0);
+              mma_ss(R + 0, sd(0, k), kd(kd0, 0, 0, k), id_n128, k > 0);
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)  // F += U_Q K^T
-              mma_ss(R + 64, sd(1, k), kd(0, k), id_n64, 1);
+              mma_ss(R + 64, sd(1, k), kd(kd0, 0, 0, k), id_n64, 1);
           } else {
 #pragma unroll
-            for (int k = 0; k < D / 16; ++k)  // [dP | C] = dO [V ; U_V]^T
-              mma_ss(R + 128, sd(2, k), kd(2, k), id_n128, k > 0);
-          }
-        } else if constexpr (OP == RowOp::BwdDQ) {
-          if (role == 0) {
-#pragma unroll
             for (int k = 0; k < D / 16; ++k)  // S = Q K^T
-              mma_ss(R + 0, sd(0, k), kd(0, k), id_n64, k > 0);
-          } else {
-#pragma unroll
-            for (int k = 0; k < D / 16; ++k)  // dP = dO V^T
-              mma_ss(R + 128, sd(1, k), kd(1, k), id_n64, k > 0);
+              mma_ss(R + 0, sd(0, k), kd(kd0, 0, 0, k), id_n64, k > 0);
           }
-        } else {
-          if (role == 0) {
-#pragma unroll
-            for (int k = 0; k < D / 16; ++k)  // S = Q K^T
-              mma_ss(R + 0, sd(0, k), kd(0, k), id_n64, k > 0);
-          }
+          mma_commit(&m->bar_sa_sf);
+          mma_commit(&m->bar_empty[stage]);
         }
-      };
-      // stage B of half h: K-steps s = 2h, 2h+1 (16 streamed rows each)
-      auto stage_b = [&](uint32_t sb, int h, int st) {
-        if (st < first_b) return;
-        const uint64_t md0 = sdesc_sw128(sb, C::NSTREAM * BN * 128, 1024);
-        const uint64_t mf0 = sdesc_sw128(sb, 3 * BN * 128, 1024);  // [K | U_V]
+        mma_commit(&m->bar_acc);
+        if (*abort_flag) drain_wait(&m->bar_acc, 0);
+      } else {
+        // ---------------- issuer Y: DC(t) and every stage-B MMA
+        auto stage_dc = [&](uint32_t sb, int h) {
+          const uint64_t kd0 = sdesc_sw128(sb, 16, 1024);
+          if constexpr (kBob) {  // [dP_h | C_h] = dO [V_h ; U_V_h]^T
 #pragma unroll
-        for (int sub = 0; sub < 2; ++sub) {
-          const int s = 2 * h + sub;
-          auto md = [&](int t, int bo) -> uint64_t {
-            return md0 + (uint64_t)((tile_off<C::NSTREAM>(t, bo) + s * 2048) >> 4);
-          };
-          const uint32_t first = (st == first_b && s == 0) ? 0u : 1u;
-          const uint32_t A = tmem + kColA + 16 * s;
-          if constexpr (OP == RowOp::BobPass1) {
-            if (role == 0) {
-              // [B | dOtil0] += P [K | U_V] ;  dOtil0 += (P o F) V
-              const uint64_t fused =
-                  mf0 + (uint64_t)((tile_off<C::NSTREAM>(0, split) + s * 2048) >> 4);
-              mma_ts(tmem + 0, A + 0, fused, id_b2, first);
-              mma_ts(tmem + 64, A + 8, md(2, split), id_b, 1);
+            for (int k = 0; k < D / 16; ++k)
+              mma_ss(tmem + kColDC + 64 * h, sd(2, k), kd(kd0, 2, h, k), id_n64, k > 0);
+          } else if constexpr (OP == RowOp::BwdDQ) {  // dP = dO V^T (whole tile)
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k)
+              mma_ss(tmem + kColDC, sd(1, k), kd(kd0, 1, 0, k), id_n64, k > 0);
+          }
+        };
+        // stage B of half h: K-steps s = 2h + sub, 16 streamed rows each; the
+        // operand tiles of K-step s sit at DC columns written by warpgroup sub
+        auto stage_b = [&](uint32_t sb, int h, int st) {
+          if (st < first_b) return;
+          constexpr uint32_t kBoxBytes = C::NSTREAM * BN * 128;
+          const uint64_t md0 = sdesc_sw128(sb, kBoxBytes, 1024);
+#pragma unroll
+          for (int sub = 0; sub < 2; ++sub) {
+            const int s = 2 * h + sub;
+            auto md = [&](int t, int bo) -> uint64_t {
+              return md0 + (uint64_t)((soff<C::NSTREAM, kBob>(t, h, bo) + sub * 2048) >> 4);
+            };
+            const uint32_t first = (st == first_b && s == 0) ? 0u : 1u;
+            if constexpr (kBob) {
+              const uint32_t A = tmem + kColDC + 64 * h + 16 * sub;
+              const uint32_t k_rows = sb + soff<C::NSTREAM, kBob>(0, h, split) + sub * 2048;
+              // [B | dOtil0] += P [K | U_V]   (second 64-wide block at U_V)
+              const uint64_t fKUV = sdesc_sw128(
+                  k_rows,
+                  soff<C::NSTREAM, kBob>(3, h, split) - soff<C::NSTREAM, kBob>(0, h, split),
+                  1024);
+              mma_ts(tmem + 0, A + 0, fKUV, id_b2, first);
+              mma_ts(tmem + 64, A + 8, md(2, split), id_b, 1);  // dOtil0 += (P o F) V
+              // [G | Omega] += dS [K | U_K] ;  Omega += (P o Pt0) K
+              const uint64_t fKUK = sdesc_sw128(
+                  k_rows,
+                  soff<C::NSTREAM, kBob>(1, h, split) - soff<C::NSTREAM, kBob>(0, h, split),
+                  1024);
+              mma_ts(tmem + 128, A + 40, fKUK, id_b2, first);
+              mma_ts(tmem + 192, A + 32, md(0, split), id_b, 1);
+            } else if constexpr (OP == RowOp::BwdDQ) {
+              mma_ts(tmem + 0, tmem + kColDC + 16 * s, md(0, 0), id_b, first);  // dQ += dS K
             } else {
-              mma_ts(tmem + 128, A + 128, md(0, split), id_b, first);  // Omega += (P o Pt0) K
-              mma_ts(tmem + 128, A + 136, md(1, split), id_b, 1);      //   += dS U_K
-              mma_ts(tmem + 192, A + 192, md(0, split), id_b, first);  // R += (P o dP) K
+              mma_ts(tmem + 0, tmem + kColDC + 16 * s, md(1, 0), id_b, first);  // O += P V
             }
-          } else if constexpr (OP == RowOp::BwdDQ) {
-            if (role == 0) mma_ts(tmem + 0, A, md(0, 0), id_b, first);  // dQ += dS K
-          } else {
-            if (role == 0) mma_ts(tmem + 0, A, md(1, 0), id_b, first);  // O += P V
           }
-        }
-      };
-      bool ok = mbar_wait(&m->bar_stat, 0, wctl) &&
-                mbar_wait(&m->bar_full[0], 0, wctl);
-      if (ok) {
-        tc_fence_after();
-        stage_a(smem_u32(s_stream));
-        mma_commit(&m->bar_sa[0]);
-      }
-      for (int st = 0; ok && st < nsteps; ++st) {
-        const int stage = st % C::NSTAGES;
-        const uint32_t sb = smem_u32(s_stream + stage * C::STAGE_BYTES);
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          if (!mbar_wait(&m->bar_ew[h], st & 1, wctl)) {
-            ok = false;
-            break;
-          }
+        };
+        bool ok = mbar_wait(&m->bar_stat, 0, wctl) && mbar_wait(&m->bar_full[0], 0, wctl);
+        if (ok) {
           tc_fence_after();
-          stage_b(sb, h, st);
+          const uint32_t sb0 = smem_u32(s_stream);
+          stage_dc(sb0, 0);
+          mma_commit(&m->bar_sa_dc[0]);
+          if (kDcHalves) {
+            stage_dc(sb0, 1);
+            mma_commit(&m->bar_sa_dc[1]);
+          }
         }
-        if (!ok) break;
-        mma_commit(&m->bar_empty[stage]);
-        if (st + 1 < nsteps) {
+        for (int st = 0; ok && st < nsteps; ++st) {
+          const int stage = st % C::NSTAGES;
+          const uint32_t sb = smem_u32(s_stream + stage * C::STAGE_BYTES);
           const int nstage = (st + 1) % C::NSTAGES;
-          if (!mbar_wait(&m->bar_full[nstage], ((st + 1) / C::NSTAGES) & 1, wctl)) break;
-          tc_fence_after();
-          stage_a(smem_u32(s_stream + nstage * C::STAGE_BYTES));
-          mma_commit(&m->bar_sa[0]);
+          const uint32_t nsb = smem_u32(s_stream + nstage * C::STAGE_BYTES);
+          const bool more = st + 1 < nsteps;
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            if (!mbar_wait(&m->bar_ew[h], st & 1, wctl)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            stage_b(sb, h, st);
+            if (h == 1) mma_commit(&m->bar_empty[stage]);
+            if (more && (kDcHalves || h == 1)) {
+              if ((h == 0 || !kDcHalves) &&
+                  !mbar_wait(&m->bar_full[nstage], ((st + 1) / C::NSTAGES) & 1, wctl)) {
+                ok = false;
+                break;
+              }
+              tc_fence_after();
+              stage_dc(nsb, kDcHalves ? h : 0);
+              mma_commit(&m->bar_sa_dc[kDcHalves ? h : 0]);
+            }
+          }
         }
+        mma_commit(&m->bar_acc);
+        if (*abort_flag) drain_wait(&m->bar_acc, 0);
       }
-      mma_commit(&m->bar_acc);
-      if (*abort_flag) drain_wait(&m->bar_acc, 0);
     }
   } else {
     // ------------------------------------------------------------ elementwise
@@ -358,87 +407,102 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         Dr = row_dot<D>(p.dout + rowoff, p.o + rowoff);
       }
     }
-    float mrow = -INFINITY, lrow = 0.f;               // forward sweep 1 (log2 domain)
-    float2 acc_a = splat(0.f), acc_e = splat(0.f);    // Pass 1 partial row sums
+    float mrow = -INFINITY, lrow = 0.f;             // forward sweep 1 (log2 domain)
+    float2 acc_a = splat(0.f), acc_e = splat(0.f);  // Pass 1 partial row sums
     bool ok = true;
     for (int st = 0; ok && st < nsteps; ++st) {
-      if (!mbar_wait(&m->bar_sa[0], st & 1, wctl)) {
+      if (!mbar_wait(&m->bar_sa_sf, st & 1, wctl)) {
         ok = false;
         break;
       }
       tc_fence_after();
-      for (int h = 0; h < 2; ++h) {
-        if constexpr (OP == RowOp::Fwd) {
-          if (st == ntiles && h == 0) {  // end of sweep 1: combine the warpgroups' (max, sum)
-            s_xchg[wg * BM + r] = mrow;
-            s_xchg[(2 + wg) * BM + r] = lrow;
-            named_bar_sync(1, kEwThreads);
-            const float m0 = s_xchg[r], m1 = s_xchg[BM + r];
-            const float l0 = s_xchg[2 * BM + r], l1 = s_xchg[3 * BM + r];
-            const float mm = fmaxf(m0, m1);
-            const float l = (m0 == -INFINITY ? 0.f : l0 * ex2(m0 - mm)) +
-                            (m1 == -INFINITY ? 0.f : l1 * ex2(m1 - mm));
-            L2 = row_ok ? mm + __log2f(l) : 0.f;
-          }
+      if constexpr (OP == RowOp::Fwd) {
+        if (st == ntiles) {  // end of sweep 1: combine the two warpgroups' (max, sum)
+          s_xchg[wg * BM + r] = mrow;
+          s_xchg[(2 + wg) * BM + r] = lrow;
+          named_bar_sync(1, kEwThreads);
+          const float m0 = s_xchg[r], m1 = s_xchg[BM + r];
+          const float l0 = s_xchg[2 * BM + r], l1 = s_xchg[3 * BM + r];
+          const float mm = fmaxf(m0, m1);
+          const float l = (m0 == -INFINITY ? 0.f : l0 * ex2(m0 - mm)) +
+                          (m1 == -INFINITY ? 0.f : l1 * ex2(m1 - mm));
+          L2 = row_ok ? mm + __log2f(l) : 0.f;
         }
-        const int c0 = HB * h + 16 * wg;                       // tile column of this thread's 16
-        const int j0 = (st % ntiles) * BN + c0;                // first key of this thread's 16
+      }
+      // ---- copy this thread's SF columns of both halves, then release SF
+      uint32_t rS[2][16], rF[2][16];
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        tmem_ld16(ta + kColSF + HB * h + 16 * wg, rS[h]);
+        if constexpr (kBob) tmem_ld16(ta + kColSF + 64 + HB * h + 16 * wg, rF[h]);
+      }
+      tmem_ld_wait(rS[0]);
+      reg_dep(rS[1]);
+      if constexpr (kBob) {
+        reg_dep(rF[0]);
+        reg_dep(rF[1]);
+      }
+      tc_fence_before();
+      mbar_arrive(&m->bar_sf_free);
+      const int jt = (st % ntiles) * BN;
+      const float2 sl2v = splat(sl2), nL2v = splat(-L2);
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        if (kDcHalves || h == 0) {
+          if (!mbar_wait(&m->bar_sa_dc[kDcHalves ? h : 0], st & 1, wctl)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+        }
+        const int c0 = HB * h + 16 * wg;  // tile column of this thread's 16
+        const int j0 = jt + c0;           // first key of this thread's 16
         const bool need_mask = (!row_ok) || (j0 + 16 > N) || (p.causal && j0 + 15 > gi);
         const int lim = need_mask ? (row_ok ? (p.causal ? min(N, gi + 1) : N) - j0 : 0) : 16;
-        const uint32_t R = ta + kColA + c0;  // this thread's 16 columns of the first stage-A tile
-        const float2 sl2v = splat(sl2), nL2v = splat(-L2);
-        if constexpr (OP == RowOp::BobPass1) {
-          uint32_t rS[16], rF[16], rdP[16], rC[16];
-          tmem_ld16(R + 0, rS);
-          tmem_ld16(R + 64, rF);
-          tmem_ld16(R + 128, rdP);
-          tmem_ld16(R + 192, rC);
-          tmem_ld_wait(rS);
-          reg_dep(rF);
-          reg_dep(rdP);
+        if constexpr (kBob) {
+          const uint32_t R = ta + kColDC + 64 * h + 16 * wg;  // [dP_h | C_h] columns
+          uint32_t rdP[16], rC[16];
+          tmem_ld16(R + 0, rdP);
+          tmem_ld16(R + 32, rC);
+          tmem_ld_wait(rdP);
           reg_dep(rC);
           const float2 tauv = splat(tau), nDv = splat(-Dr);
-          uint32_t oP[8], oPF[8], oPPt[8], odS[8], oPdP[8];
+          uint32_t oP[8], oPF[8], oPPt[8], odS[8];
 #pragma unroll
           for (int c = 0; c < 16; c += 2) {
-            float2 pr = probs2(pair(rS, c), sl2v, nL2v);
+            float2 pr = probs2(pair(rS[h], c), sl2v, nL2v);
             if (need_mask) {
               if (c >= lim) pr.x = 0.f;
               if (c + 1 >= lim) pr.y = 0.f;
             }
-            const float2 f = __fmul2_rn(pair(rF, c), tauv);
+            const float2 f = __fmul2_rn(pair(rF[h], c), tauv);
             const float2 dp = pair(rdP, c);
             const float2 t = __fadd2_rn(dp, nDv);
             const float2 pt0 = __ffma2_rn(f, t, pair(rC, c));  // Ptil0 = C + F (dP - D)
             const float2 pf = __fmul2_rn(pr, f);
             const float2 ppt = __fmul2_rn(pr, pt0);
             const float2 ds = __fmul2_rn(pr, t);
-            const float2 pdp = __fmul2_rn(pr, dp);
             acc_a = __fadd2_rn(acc_a, pf);
             acc_e = __fadd2_rn(acc_e, ppt);
             oP[c / 2] = pack_bf16(pr.x, pr.y);
             oPF[c / 2] = pack_bf16(pf.x, pf.y);
             oPPt[c / 2] = pack_bf16(ppt.x, ppt.y);
             odS[c / 2] = pack_bf16(ds.x, ds.y);
-            oPdP[c / 2] = pack_bf16(pdp.x, pdp.y);
           }
-          // operand tiles: issuer X reads columns 0..127, issuer Y 128..255
           tmem_st8(R + 0, oP);
           tmem_st8(R + 8, oPF);
-          tmem_st8(R + 128, oPPt);
-          tmem_st8(R + 136, odS);
-          tmem_st8(R + 192, oPdP);
+          tmem_st8(R + 32, oPPt);
+          tmem_st8(R + 40, odS);
         } else if constexpr (OP == RowOp::BwdDQ) {
-          uint32_t rS[16], rdP[16];
-          tmem_ld16(R + 0, rS);
-          tmem_ld16(R + 128, rdP);
-          tmem_ld_wait(rS);
-          reg_dep(rdP);
+          const uint32_t R = ta + kColDC + c0;
+          uint32_t rdP[16];
+          tmem_ld16(R, rdP);
+          tmem_ld_wait(rdP);
           const float2 nDv = splat(-Dr);
           uint32_t odS[8];
 #pragma unroll
           for (int c = 0; c < 16; c += 2) {
-            float2 pr = probs2(pair(rS, c), sl2v, nL2v);
+            float2 pr = probs2(pair(rS[h], c), sl2v, nL2v);
             if (need_mask) {
               if (c >= lim) pr.x = 0.f;
               if (c + 1 >= lim) pr.y = 0.f;
@@ -448,15 +512,12 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
           }
           tmem_st8(R, odS);
         } else {
-          uint32_t rS[16];
-          tmem_ld16(R, rS);
-          tmem_ld_wait(rS);
           if (st < ntiles) {  // sweep 1: running max and sum in the log2 domain
             float x[16];
             float mx = mrow;
 #pragma unroll
             for (int c = 0; c < 16; ++c) {
-              x[c] = bits_f(rS[c]) * sl2;
+              x[c] = bits_f(rS[h][c]) * sl2;
               if (need_mask && c >= lim) x[c] = -INFINITY;
               mx = fmaxf(mx, x[c]);
             }
@@ -467,18 +528,18 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
               lrow = l;
               mrow = mx;
             }
-          } else {  // sweep 2: normalised probabilities
+          } else {  // sweep 2: normalised probabilities into DC for O += P V
             uint32_t oP[8];
 #pragma unroll
             for (int c = 0; c < 16; c += 2) {
-              float2 pr = probs2(pair(rS, c), sl2v, nL2v);
+              float2 pr = probs2(pair(rS[h], c), sl2v, nL2v);
               if (need_mask) {
                 if (c >= lim) pr.x = 0.f;
                 if (c + 1 >= lim) pr.y = 0.f;
               }
               oP[c / 2] = pack_bf16(pr.x, pr.y);
             }
-            tmem_st8(R, oP);
+            tmem_st8(ta + kColDC + c0, oP);
           }
         }
         tmem_st_wait();
@@ -504,23 +565,24 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
 #pragma unroll 1
         for (int q = 0; q < 2; ++q) {
           const int cc = 32 * wg + 16 * q;  // accumulator column (0..63)
-          // accumulators: B at 0, dOtil0 at 64, Omega at 128, R at 192
-          uint32_t rO[16], rW[16], rB[16], rR[16];
-          tmem_ld16(ta + 64 + cc, rO);
-          tmem_ld16(ta + 128 + cc, rW);
+          // accumulators: B at 0, dOtil0 at 64, G at 128, Omega at 192
+          uint32_t rB[16], rO[16], rG[16], rW[16];
           tmem_ld16(ta + 0 + cc, rB);
-          tmem_ld16(ta + 192 + cc, rR);
-          tmem_ld_wait(rO);
+          tmem_ld16(ta + 64 + cc, rO);
+          tmem_ld16(ta + 128 + cc, rG);
+          tmem_ld16(ta + 192 + cc, rW);
+          tmem_ld_wait(rB);
+          reg_dep(rO);
+          reg_dep(rG);
           reg_dep(rW);
-          reg_dep(rB);
-          reg_dep(rR);
           if (row_ok) {
             float ov[16], qt[16], dot[16];
             load_row16(p.o + rowoff + cbase + 16 * q, ov);
 #pragma unroll
             for (int c = 0; c < 16; ++c) {
-              // eq. (8): Qtil = tau (Omega - alpha R - E B), dOtil = dOtil0 - alpha o
-              qt[c] = tau * (bits_f(rW[c]) - alpha * bits_f(rR[c]) - E * bits_f(rB[c]));
+              // eq. (8) with R = G + D B (G = sum_j dS_ij k_j) and E + alpha D = E0:
+              // Qtil = tau (Omega - alpha G - E0 B), dOtil = dOtil0 - alpha o
+              qt[c] = tau * (bits_f(rW[c]) - alpha * bits_f(rG[c]) - E0 * bits_f(rB[c]));
               dot[c] = bits_f(rO[c]) - alpha * ov[c];
             }
             store_row16(p.out0 + rowoff + cbase + 16 * q, qt);
@@ -569,6 +631,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
 template <ColOp OP, int D>
 __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant__ EngineParams p) {
   using C = ColCfg<OP, D>;
+  constexpr bool kBob = OP == ColOp::BobPass2;
   extern __shared__ __align__(1024) uint8_t smem[];
   uint8_t* s_stat = smem;
   uint8_t* s_stream = smem + C::STAT_BYTES;
@@ -597,8 +660,10 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
       mbar_init(&m->bar_full[s], 1 + 32);  // TMA bytes + 32 producer lanes' row vectors
       mbar_init(&m->bar_empty[s], 2);      // released by both MMA issuers
     }
+    mbar_init(&m->bar_sa_sf, 1);
+    mbar_init(&m->bar_sf_free, kEwThreads);
     for (int h = 0; h < 2; ++h) {
-      mbar_init(&m->bar_sa[h], 2);  // one commit per MMA issuer
+      mbar_init(&m->bar_sa_dc[h], 1);
       mbar_init(&m->bar_ew[h], kEwThreads);
     }
     mbar_init(&m->bar_acc, 2);
@@ -640,7 +705,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
         mbar_arrive_expect_tx(&m->bar_full[stage], C::TILE_BYTES);
         for (int b = 0; b < C::KB; ++b)
           for (int t = 0; t < C::NSTREAM; ++t)
-            tma_load_3d(dst + tile_off<C::NSTREAM>(t, b), &p.tm[C::NSTAT + t],
+            tma_load_3d(dst + soff<C::NSTREAM, false>(t, 0, b), &p.tm[C::NSTAT + t],
                         &m->bar_full[stage], 64 * b, ib, bh);
       }
       // negated row vectors of the streamed query rows:
@@ -671,10 +736,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
     }
   } else if (warp == kMmaWarp || warp == kMmaWarpY) {
     // ------------------------------------------------------------ MMA issuers
-    // Same ownership split as the row engine: issuer X owns stage-A columns
-    // 0..127, issuer Y columns 128..255.
     if (elect_lane0()) {
-      const int role = warp == kMmaWarp ? 0 : 1;
       constexpr uint32_t id_n64 = idesc_bf16(128, 64, false);
       constexpr uint32_t id_n128 = idesc_bf16(128, 128, false);
       constexpr uint32_t id_b = idesc_bf16(128, D, true);
@@ -682,96 +744,106 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
       auto sd = [&](int t, int k) -> uint64_t {
         return sd0 + (uint64_t)(((t * C::KB + k / 4) * (BM * 128) + (k % 4) * 32) >> 4);
       };
-      auto stage_a = [&](uint32_t sb) {
-        const uint64_t kd0 = sdesc_sw128(sb, 16, 1024);
-        auto kd = [&](int t, int k) -> uint64_t {
-          return kd0 + (uint64_t)((tile_off<C::NSTREAM>(t, k / 4) + (k % 4) * 32) >> 4);
-        };
-        const uint32_t R = tmem + kColA;
-        if constexpr (OP == ColOp::BobPass2) {
-          // stationary: 0 K, 1 V, 2 U_K, 3 U_V ; stream: 0 Q, 1 U_Q, 2 dO
-          if (role == 0) {
+      auto kd = [&](uint64_t kd0, int t, int k) -> uint64_t {
+        return kd0 + (uint64_t)((soff<C::NSTREAM, false>(t, 0, k / 4) + (k % 4) * 32) >> 4);
+      };
+      if (warp == kMmaWarp) {
+        // ---------------- issuer X: SF(t) = transposed scores (and F)
+        bool ok = mbar_wait(&m->bar_stat, 0, wctl);
+        for (int st = 0; ok && st < nsteps; ++st) {
+          if (st > 0 && !mbar_wait(&m->bar_sf_free, (st - 1) & 1, wctl)) break;
+          const int stage = st % C::NSTAGES;
+          if (!mbar_wait(&m->bar_full[stage], (st / C::NSTAGES) & 1, wctl)) break;
+          tc_fence_after();
+          const uint64_t kd0 = sdesc_sw128(smem_u32(s_stream + stage * C::STAGE_BYTES), 16, 1024);
+          const uint32_t R = tmem + kColSF;
+          if constexpr (kBob) {
+            // stationary: 0 K, 1 V, 2 U_K, 3 U_V ; stream: 0 Q, 1 U_Q, 2 dO
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)  // [S^T | F^T] = K [Q ; U_Q]^T
-              mma_ss(R + 0, sd(0, k), kd(0, k), id_n128, k > 0);
+              mma_ss(R + 0, sd(0, k), kd(kd0, 0, k), id_n128, k > 0);
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)  // F^T += U_K Q^T
-              mma_ss(R + 64, sd(2, k), kd(0, k), id_n64, 1);
+              mma_ss(R + 64, sd(2, k), kd(kd0, 0, k), id_n64, 1);
           } else {
-#pragma unroll
-            for (int k = 0; k < D / 16; ++k)  // dP^T = V dO^T
-              mma_ss(R + 128, sd(1, k), kd(2, k), id_n64, k > 0);
-#pragma unroll
-            for (int k = 0; k < D / 16; ++k)  // C^T = U_V dO^T
-              mma_ss(R + 192, sd(3, k), kd(2, k), id_n64, k > 0);
-          }
-        } else {
-          // stationary: 0 K, 1 V ; stream: 0 Q, 1 dO
-          if (role == 0) {
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)  // S^T = K Q^T
-              mma_ss(R + 0, sd(0, k), kd(0, k), id_n64, k > 0);
+              mma_ss(R + 0, sd(0, k), kd(kd0, 0, k), id_n64, k > 0);
+          }
+          mma_commit(&m->bar_sa_sf);
+          mma_commit(&m->bar_empty[stage]);
+        }
+        mma_commit(&m->bar_acc);
+        if (*abort_flag) drain_wait(&m->bar_acc, 0);
+      } else {
+        // ---------------- issuer Y: DC(t) and every stage-B MMA
+        auto stage_dc = [&](uint32_t sb) {
+          const uint64_t kd0 = sdesc_sw128(sb, 16, 1024);
+          if constexpr (kBob) {
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k)  // dP^T = V dO^T
+              mma_ss(tmem + kColDC, sd(1, k), kd(kd0, 2, k), id_n64, k > 0);
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k)  // C^T = U_V dO^T
+              mma_ss(tmem + kColDC + 64, sd(3, k), kd(kd0, 2, k), id_n64, k > 0);
           } else {
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)  // dP^T = V dO^T
-              mma_ss(R + 128, sd(1, k), kd(1, k), id_n64, k > 0);
+              mma_ss(tmem + kColDC, sd(1, k), kd(kd0, 1, k), id_n64, k > 0);
           }
-        }
-      };
-      auto stage_b = [&](uint32_t sb, int h, int st) {
-        const uint64_t md0 = sdesc_sw128(sb, C::NSTREAM * BN * 128, 1024);
+        };
+        auto stage_b = [&](uint32_t sb, int h, int st) {
+          constexpr uint32_t kBoxBytes = C::NSTREAM * BN * 128;
+          const uint64_t md0 = sdesc_sw128(sb, kBoxBytes, 1024);
 #pragma unroll
-        for (int sub = 0; sub < 2; ++sub) {
-          const int s = 2 * h + sub;
-          auto md = [&](int t) -> uint64_t {
-            return md0 + (uint64_t)((tile_off<C::NSTREAM>(t, 0) + s * 2048) >> 4);
-          };
-          const uint32_t first = (st == 0 && s == 0) ? 0u : 1u;
-          const uint32_t A = tmem + kColA + 16 * s;
-          if constexpr (OP == ColOp::BobPass2) {
-            if (role == 0) {
-              mma_ts(tmem + D, A + 0, md(2), id_b, first);      // Vtil += (P o h)^T dO
+          for (int sub = 0; sub < 2; ++sub) {
+            const int s = 2 * h + sub;
+            auto md = [&](int t) -> uint64_t {
+              return md0 + (uint64_t)((soff<C::NSTREAM, false>(t, h, 0) + sub * 2048) >> 4);
+            };
+            const uint32_t first = (st == 0 && s == 0) ? 0u : 1u;
+            const uint32_t A = tmem + kColDC + 16 * s;
+            if constexpr (kBob) {
+              mma_ts(tmem + D, A + 0, md(2), id_b, first);    // Vtil += (P o h)^T dO
+              mma_ts(tmem + 0, A + 8, md(0), id_b, first);    // Ktil += Stil^T Q
+              mma_ts(tmem + 0, A + 64, md(1), id_b, 1);       //      += dS^T U_Q
             } else {
-              mma_ts(tmem + 0, A + 128, md(0), id_b, first);    // Ktil += Stil^T Q
-              mma_ts(tmem + 0, A + 136, md(1), id_b, 1);        //      += dS^T U_Q
+              mma_ts(tmem + D, A + 0, md(1), id_b, first);    // dV += P^T dO
+              mma_ts(tmem + 0, A + 8, md(0), id_b, first);    // dK += dS^T Q
             }
-          } else {
-            if (role == 0) mma_ts(tmem + D, A + 0, md(1), id_b, first);   // dV += P^T dO
-            else mma_ts(tmem + 0, A + 128, md(0), id_b, first);           // dK += dS^T Q
           }
+        };
+        bool ok = mbar_wait(&m->bar_stat, 0, wctl) && mbar_wait(&m->bar_full[0], 0, wctl);
+        if (ok) {
+          tc_fence_after();
+          stage_dc(smem_u32(s_stream));
+          mma_commit(&m->bar_sa_dc[0]);
         }
-      };
-      bool ok = mbar_wait(&m->bar_stat, 0, wctl) &&
-                mbar_wait(&m->bar_full[0], 0, wctl);
-      if (ok) {
-        tc_fence_after();
-        stage_a(smem_u32(s_stream));
-        mma_commit(&m->bar_sa[0]);
-      }
-      for (int st = 0; ok && st < nsteps; ++st) {
-        const int stage = st % C::NSTAGES;
-        const uint32_t sb = smem_u32(s_stream + stage * C::STAGE_BYTES);
+        for (int st = 0; ok && st < nsteps; ++st) {
+          const int stage = st % C::NSTAGES;
+          const uint32_t sb = smem_u32(s_stream + stage * C::STAGE_BYTES);
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          if (!mbar_wait(&m->bar_ew[h], st & 1, wctl)) {
-            ok = false;
-            break;
+          for (int h = 0; h < 2; ++h) {
+            if (!mbar_wait(&m->bar_ew[h], st & 1, wctl)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            stage_b(sb, h, st);
           }
-          tc_fence_after();
-          stage_b(sb, h, st);
+          if (!ok) break;
+          mma_commit(&m->bar_empty[stage]);
+          if (st + 1 < nsteps) {
+            const int nstage = (st + 1) % C::NSTAGES;
+            if (!mbar_wait(&m->bar_full[nstage], ((st + 1) / C::NSTAGES) & 1, wctl)) break;
+            tc_fence_after();
+            stage_dc(smem_u32(s_stream + nstage * C::STAGE_BYTES));
+            mma_commit(&m->bar_sa_dc[0]);
+          }
         }
-        if (!ok) break;
-        mma_commit(&m->bar_empty[stage]);
-        if (st + 1 < nsteps) {
-          const int nstage = (st + 1) % C::NSTAGES;
-          if (!mbar_wait(&m->bar_full[nstage], ((st + 1) / C::NSTAGES) & 1, wctl)) break;
-          tc_fence_after();
-          stage_a(smem_u32(s_stream + nstage * C::STAGE_BYTES));
-          mma_commit(&m->bar_sa[0]);
-        }
+        mma_commit(&m->bar_acc);
+        if (*abort_flag) drain_wait(&m->bar_acc, 0);
       }
-      mma_commit(&m->bar_acc);
-      if (*abort_flag) drain_wait(&m->bar_acc, 0);
     }
   } else {
     // ------------------------------------------------------------ elementwise
@@ -786,35 +858,48 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
     for (int st = 0; ok && st < nsteps; ++st) {
       const int stage = st % C::NSTAGES;
       // the row vectors were written by the producer: acquire them explicitly
-      if (!mbar_wait(&m->bar_full[stage], (st / C::NSTAGES) & 1, wctl)) {
-        ok = false;
-        break;
-      }
-      const float* vec = reinterpret_cast<const float*>(s_stream + stage * C::STAGE_BYTES +
-                                                        C::TILE_BYTES);
-      if (!mbar_wait(&m->bar_sa[0], st & 1, wctl)) {
+      if (!mbar_wait(&m->bar_full[stage], (st / C::NSTAGES) & 1, wctl) ||
+          !mbar_wait(&m->bar_sa_sf, st & 1, wctl)) {
         ok = false;
         break;
       }
       tc_fence_after();
+      const float* vec = reinterpret_cast<const float*>(s_stream + stage * C::STAGE_BYTES +
+                                                        C::TILE_BYTES);
+      // ---- copy this thread's SF columns of both halves, then release SF
+      uint32_t rS[2][16], rF[2][16];
+#pragma unroll
       for (int h = 0; h < 2; ++h) {
-        const int c0 = 16 * wg;
-        const int cv = HB * h + c0;                    // tile column of this thread's first
-        const int ib = (first_tile + st) * BN + cv;    // first query row of this thread's 16
+        tmem_ld16(ta + kColSF + HB * h + 16 * wg, rS[h]);
+        if constexpr (kBob) tmem_ld16(ta + kColSF + 64 + HB * h + 16 * wg, rF[h]);
+      }
+      tmem_ld_wait(rS[0]);
+      reg_dep(rS[1]);
+      if constexpr (kBob) {
+        reg_dep(rF[0]);
+        reg_dep(rF[1]);
+      }
+      tc_fence_before();
+      mbar_arrive(&m->bar_sf_free);
+      if (!mbar_wait(&m->bar_sa_dc[0], st & 1, wctl)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int cv = HB * h + 16 * wg;             // tile column of this thread's first
+        const int ib = (first_tile + st) * BN + cv;  // first query row of this thread's 16
         const bool need_mask = (!row_ok) || (ib + 16 > N) || (p.causal && ib < gj);
         // valid query columns c satisfy  lo <= c < hi
         const int lo = p.causal ? gj - ib : 0;
         const int hi = row_ok ? N - ib : 0;
-        const uint32_t R = ta + kColA + cv;
-        if constexpr (OP == ColOp::BobPass2) {
-          uint32_t rS[16], rF[16], rdP[16], rC[16];
-          tmem_ld16(R + 0, rS);
-          tmem_ld16(R + 64, rF);
-          tmem_ld16(R + 128, rdP);
-          tmem_ld16(R + 192, rC);
-          tmem_ld_wait(rS);
-          reg_dep(rF);
-          reg_dep(rdP);
+        const uint32_t R = ta + kColDC + cv;
+        if constexpr (kBob) {
+          uint32_t rdP[16], rC[16];
+          tmem_ld16(R + 0, rdP);
+          tmem_ld16(R + 64, rC);
+          tmem_ld_wait(rdP);
           reg_dep(rC);
           uint32_t oPh[8], oSt[8], odS[8];
 #pragma unroll
@@ -823,12 +908,12 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
             const float2 nD = *reinterpret_cast<const float2*>(vec + 64 + cv + c);
             const float2 nal = *reinterpret_cast<const float2*>(vec + 128 + cv + c);
             const float2 nE = *reinterpret_cast<const float2*>(vec + 192 + cv + c);
-            float2 pr = probs2(pair(rS, c), sl2v, nL2);
+            float2 pr = probs2(pair(rS[h], c), sl2v, nL2);
             if (need_mask) {
               if (c < lo || c >= hi) pr.x = 0.f;
               if (c + 1 < lo || c + 1 >= hi) pr.y = 0.f;
             }
-            const float2 f = __fmul2_rn(pair(rF, c), tauv);
+            const float2 f = __fmul2_rn(pair(rF[h], c), tauv);
             const float2 dp = pair(rdP, c);
             const float2 t = __fadd2_rn(dp, nD);
             // Ptil = C + F (dP - D) - alpha dP ; Stil = P (Ptil - E) ; h = F - alpha
@@ -840,22 +925,19 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
             oSt[c / 2] = pack_bf16(stl.x, stl.y);
             odS[c / 2] = pack_bf16(ds.x, ds.y);
           }
-          // operand tiles: issuer X reads columns 0..127, issuer Y 128..255
           tmem_st8(R + 0, oPh);
-          tmem_st8(R + 128, oSt);
-          tmem_st8(R + 136, odS);
+          tmem_st8(R + 8, oSt);
+          tmem_st8(R + 64, odS);
         } else {
-          uint32_t rS[16], rdP[16];
-          tmem_ld16(R + 0, rS);
-          tmem_ld16(R + 128, rdP);
-          tmem_ld_wait(rS);
-          reg_dep(rdP);
+          uint32_t rdP[16];
+          tmem_ld16(R, rdP);
+          tmem_ld_wait(rdP);
           uint32_t oP[8], odS[8];
 #pragma unroll
           for (int c = 0; c < 16; c += 2) {
             const float2 nL2 = *reinterpret_cast<const float2*>(vec + cv + c);
             const float2 nD = *reinterpret_cast<const float2*>(vec + 64 + cv + c);
-            float2 pr = probs2(pair(rS, c), sl2v, nL2);
+            float2 pr = probs2(pair(rS[h], c), sl2v, nL2);
             if (need_mask) {
               if (c < lo || c >= hi) pr.x = 0.f;
               if (c + 1 < lo || c + 1 >= hi) pr.y = 0.f;
@@ -865,7 +947,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
             odS[c / 2] = pack_bf16(ds.x, ds.y);
           }
           tmem_st8(R + 0, oP);
-          tmem_st8(R + 128, odS);
+          tmem_st8(R + 8, odS);
         }
         tmem_st_wait();
         tc_fence_before();

@@ -134,8 +134,10 @@ int run_pass1(const fbob_shape* s, const void* q, const void* k, const void* v, 
   const void* strm[4] = {k, gk, v, gv};
   for (int t = 0; t < 3; ++t)
     if (!make_map(&p.tm[t], stat[t], BH, N, d, BM)) return FBOB_ERR_CUDA;
+  // K and U_K as 64-row tiles; V and U_V as 32-row chunks (interleaved in the
+  // stream stage so that [V_h ; U_V_h] is one operand)
   for (int t = 0; t < 4; ++t)
-    if (!make_map(&p.tm[3 + t], strm[t], BH, N, d, BN)) return FBOB_ERR_CUDA;
+    if (!make_map(&p.tm[3 + t], strm[t], BH, N, d, t < 2 ? BN : HB)) return FBOB_ERR_CUDA;
   p.o = static_cast<const __nv_bfloat16*>(o);
   p.dout = static_cast<const __nv_bfloat16*>(dout);
   p.lse = lse;
