@@ -61,7 +61,8 @@ constexpr uint32_t kColDC = 384;  // stage-A area of issuer Y
 // Shared-memory bookkeeping block (in the MISC area).
 struct Misc {
   uint64_t bar_stat;
-  uint64_t bar_full[4];
+  uint64_t bar_full[4];    // stream stage landed (in Pass 1: K and U_K only)
+  uint64_t bar_full_b[4];  // Pass 1: V and U_V of the stage landed
   uint64_t bar_empty[4];
   uint64_t bar_sa_sf;   // X's stage A of a tile completed
   uint64_t bar_sf_free; // elementwise warps copied SF to registers
@@ -190,6 +191,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
     mbar_init(&m->bar_stat, 1);
     for (int s = 0; s < C::NSTAGES; ++s) {
       mbar_init(&m->bar_full[s], 1);
+      mbar_init(&m->bar_full_b[s], 1);
       mbar_init(&m->bar_empty[s], 2);  // released by both MMA issuers
     }
     mbar_init(&m->bar_sa_sf, 1);
@@ -233,23 +235,30 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         const bool k_only = (OP == RowOp::Fwd) && st < ntiles;
         const int nt = k_only ? 1 : C::NSTREAM;
         uint8_t* dst = s_stream + stage * C::STAGE_BYTES;
-        mbar_arrive_expect_tx(&m->bar_full[stage], nt * C::KB * BN * 128);
+        // Pass 1: K and U_K first on bar_full (all issuer X needs), then V and
+        // U_V on bar_full_b; the other operations use bar_full alone
+        const int nt_a = kBob ? 2 : nt;
+        mbar_arrive_expect_tx(&m->bar_full[stage], nt_a * C::KB * BN * 128);
         for (int b = 0; b < C::KB; ++b)
-          for (int t = 0; t < nt; ++t) {
-            if (kBob && t >= 2) {  // 32-row chunks (map box rows HB)
+          for (int t = 0; t < nt_a; ++t)
+            tma_load_3d(dst + soff<C::NSTREAM, kBob>(t, 0, b), &p.tm[C::NSTAT + t],
+                        &m->bar_full[stage], 64 * b, j0, bh);
+        if (kBob) {  // 32-row chunks (map box rows HB)
+          mbar_arrive_expect_tx(&m->bar_full_b[stage], 2 * C::KB * BN * 128);
+          for (int b = 0; b < C::KB; ++b)
+            for (int t = 2; t < 4; ++t)
               for (int h = 0; h < 2; ++h)
                 tma_load_3d(dst + soff<C::NSTREAM, kBob>(t, h, b), &p.tm[C::NSTAT + t],
-                            &m->bar_full[stage], 64 * b, j0 + HB * h, bh);
-            } else {
-              tma_load_3d(dst + soff<C::NSTREAM, kBob>(t, 0, b), &p.tm[C::NSTAT + t],
-                          &m->bar_full[stage], 64 * b, j0, bh);
-            }
-          }
+                            &m->bar_full_b[stage], 64 * b, j0 + HB * h, bh);
+        }
         issued[stage] = st;
       }
       if (*abort_flag) {  // drain loads still in flight
         for (int s = 0; s < C::NSTAGES; ++s)
-          if (issued[s] >= 0) drain_wait(&m->bar_full[s], (issued[s] / C::NSTAGES) & 1);
+          if (issued[s] >= 0) {
+            drain_wait(&m->bar_full[s], (issued[s] / C::NSTAGES) & 1);
+            if (kBob) drain_wait(&m->bar_full_b[s], (issued[s] / C::NSTAGES) & 1);
+          }
         drain_wait(&m->bar_stat, 0);
       }
     }
@@ -348,7 +357,12 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
             }
           }
         };
-        bool ok = mbar_wait(&m->bar_stat, 0, wctl) && mbar_wait(&m->bar_full[0], 0, wctl);
+        // issuer Y reads every streamed tensor: wait for both halves of a stage
+        auto wait_stage = [&](int stg, uint32_t par) {
+          return mbar_wait(&m->bar_full[stg], par, wctl) &&
+                 (!kBob || mbar_wait(&m->bar_full_b[stg], par, wctl));
+        };
+        bool ok = mbar_wait(&m->bar_stat, 0, wctl) && wait_stage(0, 0);
         if (ok) {
           tc_fence_after();
           const uint32_t sb0 = smem_u32(s_stream);
@@ -375,8 +389,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
             stage_b(sb, h, st);
             if (h == 1) mma_commit(&m->bar_empty[stage]);
             if (more && (kDcHalves || h == 1)) {
-              if ((h == 0 || !kDcHalves) &&
-                  !mbar_wait(&m->bar_full[nstage], ((st + 1) / C::NSTAGES) & 1, wctl)) {
+              if ((h == 0 || !kDcHalves) && !wait_stage(nstage, ((st + 1) / C::NSTAGES) & 1)) {
                 ok = false;
                 break;
               }
