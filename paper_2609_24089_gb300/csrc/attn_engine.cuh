@@ -61,8 +61,8 @@ constexpr uint32_t kColDC = 384;  // stage-A area of issuer Y
 // Shared-memory bookkeeping block (in the MISC area).
 struct Misc {
   uint64_t bar_stat;
-  uint64_t bar_full[4];    // stream stage landed (in Pass 1: K and U_K only)
-  uint64_t bar_full_b[4];  // Pass 1: V and U_V of the stage landed
+  uint64_t bar_full[4];    // first part of a stream stage landed (all issuer X reads)
+  uint64_t bar_full_b[4];  // rest of the stage (and, column engine, the row vectors)
   uint64_t bar_empty[4];
   uint64_t bar_sa_sf;   // X's stage A of a tile completed
   uint64_t bar_sf_free; // elementwise warps copied SF to registers
@@ -170,14 +170,17 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
     return;
   }
 
-  // ---- tile decode: consecutive CTAs take different heads of one row block;
-  // with the causal mask the longest row blocks go first.
+  // ---- tile decode.  The two output halves of a row block (d = 128) are
+  // adjacent.  Head-major order: the CTAs in flight work on the row blocks of
+  // one or two heads and stream the same K/V tiles, which then stay in L2.
+  // Otherwise heads are innermost, so with the causal mask the longest row
+  // blocks of all heads go first (better balance, less sharing).
   const int N = p.N;
   int lin = blockIdx.x;
-  const int bh = lin % p.BH;
-  lin /= p.BH;
   const int split = lin % C::NSPLIT;
-  const int rbi = lin / C::NSPLIT;
+  lin /= C::NSPLIT;
+  const int rbi = p.head_major ? lin % p.nblk : lin / p.BH;
+  const int bh = p.head_major ? lin / p.nblk : lin % p.BH;
   const int rb = p.causal ? (p.nblk - 1 - rbi) : rbi;
   const int i0 = rb * BM;
   const int last_row = min(i0 + BM, N) - 1;
@@ -656,10 +659,12 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
     if (tid == 0) atomicOr(&g_fbob_error_word, kDevErrBadLaunch);
     return;
   }
+  // ---- tile decode (as in the row engine); key block 0 has the most work
+  // under the causal mask
   const int N = p.N;
   const int lin = blockIdx.x;
-  const int bh = lin % p.BH;
-  const int cb = lin / p.BH;  // key block; block 0 has the most work under the causal mask
+  const int cb = p.head_major ? lin % p.nblk : lin / p.BH;
+  const int bh = p.head_major ? lin / p.nblk : lin % p.BH;
   const int j0 = cb * BM;
   const int first_tile = p.causal ? (j0 / BN) : 0;
   const int ntotal = (N + BN - 1) / BN;
@@ -670,8 +675,9 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
     m->wctl.limit_ns = p.wait_limit_ns;
     mbar_init(&m->bar_stat, 1);
     for (int s = 0; s < C::NSTAGES; ++s) {
-      mbar_init(&m->bar_full[s], 1 + 32);  // TMA bytes + 32 producer lanes' row vectors
-      mbar_init(&m->bar_empty[s], 2);      // released by both MMA issuers
+      mbar_init(&m->bar_full[s], 1);         // Q (and U_Q): all issuer X needs
+      mbar_init(&m->bar_full_b[s], 1 + 32);  // dO + 32 producer lanes' row vectors
+      mbar_init(&m->bar_empty[s], 2);        // released by both MMA issuers
     }
     mbar_init(&m->bar_sa_sf, 1);
     mbar_init(&m->bar_sf_free, kEwThreads);
@@ -715,11 +721,17 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
       const int ib = (first_tile + st) * BN;
       uint8_t* dst = s_stream + stage * C::STAGE_BYTES;
       if (lane == 0) {
-        mbar_arrive_expect_tx(&m->bar_full[stage], C::TILE_BYTES);
+        // Q (and U_Q) first on bar_full, dO on bar_full_b
+        constexpr int na = C::NSTREAM - 1;
+        mbar_arrive_expect_tx(&m->bar_full[stage], na * C::KB * BN * 128);
         for (int b = 0; b < C::KB; ++b)
-          for (int t = 0; t < C::NSTREAM; ++t)
+          for (int t = 0; t < na; ++t)
             tma_load_3d(dst + soff<C::NSTREAM, false>(t, 0, b), &p.tm[C::NSTAT + t],
                         &m->bar_full[stage], 64 * b, ib, bh);
+        mbar_arrive_expect_tx(&m->bar_full_b[stage], C::KB * BN * 128);
+        for (int b = 0; b < C::KB; ++b)
+          tma_load_3d(dst + soff<C::NSTREAM, false>(na, 0, b), &p.tm[C::NSTAT + na],
+                      &m->bar_full_b[stage], 64 * b, ib, bh);
       }
       // negated row vectors of the streamed query rows:
       // [0] -L*log2e, [1] -D, [2] -alpha, [3] -E
@@ -739,12 +751,15 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
           vec[192 + c] = ok ? -p.vec_in[p.bhn + ri] : 0.f;     // E
         }
       }
-      mbar_arrive(&m->bar_full[stage]);
+      mbar_arrive(&m->bar_full_b[stage]);
       issued[stage] = st;
     }
     if (lane == 0 && *abort_flag) {
       for (int s = 0; s < C::NSTAGES; ++s)
-        if (issued[s] >= 0) drain_wait(&m->bar_full[s], (issued[s] / C::NSTAGES) & 1);
+        if (issued[s] >= 0) {
+          drain_wait(&m->bar_full[s], (issued[s] / C::NSTAGES) & 1);
+          drain_wait(&m->bar_full_b[s], (issued[s] / C::NSTAGES) & 1);
+        }
       drain_wait(&m->bar_stat, 0);
     }
   } else if (warp == kMmaWarp || warp == kMmaWarpY) {
@@ -826,7 +841,11 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
             }
           }
         };
-        bool ok = mbar_wait(&m->bar_stat, 0, wctl) && mbar_wait(&m->bar_full[0], 0, wctl);
+        auto wait_stage = [&](int stg, uint32_t par) {
+          return mbar_wait(&m->bar_full[stg], par, wctl) &&
+                 mbar_wait(&m->bar_full_b[stg], par, wctl);
+        };
+        bool ok = mbar_wait(&m->bar_stat, 0, wctl) && wait_stage(0, 0);
         if (ok) {
           tc_fence_after();
           stage_dc(smem_u32(s_stream));
@@ -848,7 +867,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
           mma_commit(&m->bar_empty[stage]);
           if (st + 1 < nsteps) {
             const int nstage = (st + 1) % C::NSTAGES;
-            if (!mbar_wait(&m->bar_full[nstage], ((st + 1) / C::NSTAGES) & 1, wctl)) break;
+            if (!wait_stage(nstage, ((st + 1) / C::NSTAGES) & 1)) break;
             tc_fence_after();
             stage_dc(smem_u32(s_stream + nstage * C::STAGE_BYTES));
             mma_commit(&m->bar_sa_dc[0]);
@@ -871,7 +890,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
     for (int st = 0; ok && st < nsteps; ++st) {
       const int stage = st % C::NSTAGES;
       // the row vectors were written by the producer: acquire them explicitly
-      if (!mbar_wait(&m->bar_full[stage], (st / C::NSTAGES) & 1, wctl) ||
+      if (!mbar_wait(&m->bar_full_b[stage], (st / C::NSTAGES) & 1, wctl) ||
           !mbar_wait(&m->bar_sa_sf, st & 1, wctl)) {
         ok = false;
         break;

@@ -46,6 +46,7 @@ struct EngineParams {
   long long bhn;  // BH * N (row_stats plane stride)
   unsigned long long wait_limit_ns;  // bound of every device-side wait
   int inject_stall;                  // fault injection: producers issue nothing
+  int head_major;                    // CTA order: 1 = head-major, 0 = heads innermost
 };
 
 // ---------------------------------------------------------------- configs

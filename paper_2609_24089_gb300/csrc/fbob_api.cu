@@ -107,6 +107,11 @@ void debug_controls(EngineParams* p) {
   p->inject_stall = (inj && inj[0] == '1') ? 1 : 0;
 }
 
+// CTA order per kernel, from measurements on GB300: head-major helps Pass 1
+// (CTAs in flight share one head's K/V stream in L2); Pass 2 and the helper
+// kernels balance the causal work better with heads innermost.
+void choose_order(EngineParams* p, int head_major) { p->head_major = head_major; }
+
 EngineParams base_params(const fbob_shape* s) {
   EngineParams p;
   std::memset(&p, 0, sizeof(p));
@@ -145,6 +150,7 @@ int run_pass1(const fbob_shape* s, const void* q, const void* k, const void* v, 
   p.out1 = static_cast<__nv_bfloat16*>(dout_bar);
   p.vec_out = row_stats;
   p.nblk = n_blocks(N, BM);
+  choose_order(&p, 1);
   const int nb = p.nblk * p.BH * row_nsplit(RowOp::BobPass1, (int)d);
   return launch_status(launch_row(RowOp::BobPass1, (int)d, p, nb, st));
 }
@@ -165,6 +171,7 @@ int run_pass2(const fbob_shape* s, const void* q, const void* k, const void* v, 
   p.out0 = static_cast<__nv_bfloat16*>(k_bar);
   p.out1 = static_cast<__nv_bfloat16*>(v_bar);
   p.nblk = n_blocks(N, BM);
+  choose_order(&p, 0);
   return launch_status(launch_col(ColOp::BobPass2, (int)d, p, p.nblk * p.BH, st));
 }
 
@@ -219,6 +226,7 @@ int fbob_attn_fwd(const fbob_shape* s, const void* q, const void* k, const void*
   p.out0 = static_cast<__nv_bfloat16*>(o);
   p.vec_out = lse;
   p.nblk = n_blocks(s->N, BM);
+  choose_order(&p, 0);
   rc = launch_status(launch_row(RowOp::Fwd, (int)s->d, p, p.nblk * p.BH, stream));
   if (rc == FBOB_OK) g_launches[kEntFwd] = 1;
   return rc;
@@ -253,6 +261,7 @@ int fbob_attn_bwd(const fbob_shape* s, const void* q, const void* k, const void*
   p.out0 = static_cast<__nv_bfloat16*>(dq);
   p.vec_out = dstat;
   p.nblk = n_blocks(N, BM);
+  choose_order(&p, 0);
   rc = launch_status(launch_row(RowOp::BwdDQ, (int)d, p, p.nblk * p.BH, stream));
   if (rc != FBOB_OK) return rc;
   // dK and dV: column-block pass
@@ -265,6 +274,7 @@ int fbob_attn_bwd(const fbob_shape* s, const void* q, const void* k, const void*
   c.out0 = static_cast<__nv_bfloat16*>(dk);
   c.out1 = static_cast<__nv_bfloat16*>(dv);
   c.nblk = n_blocks(N, BM);
+  choose_order(&c, 0);
   rc = launch_status(launch_col(ColOp::BwdDKDV, (int)d, c, c.nblk * c.BH, stream));
   if (rc == FBOB_OK) g_launches[kEntBwd] = 2;
   return rc;
