@@ -24,17 +24,21 @@
 // "DC" at 384..511 (dP, and C in the BoB passes), owned by issuer Y.
 //
 // Per streamed tile t:
-//   X  issues SF(t) as soon as the elementwise warps have copied SF(t-1)
+//   X  issues SF(t+1) as soon as the elementwise warps have copied SF(t)
 //      into registers, so the next tile's largest stage-A contractions run
 //      while the elementwise warps still work on tile t.
-//   Y  issues DC(t) (per 32-column half in Pass 1) and all stage-B MMAs.
+//   Y  issues DC(t) (per 32-column half in Pass 1).
 //   elementwise: copy SF to registers and release it; then per half read DC,
 //      compute, and write the bf16 operand tiles of stage B over the DC
 //      columns just read; stage B of half 0 overlaps the elementwise work on
 //      half 1.
-// Every TMEM region has one writer issuer and the MMAs reading a region are
-// issued by that same thread, so no cross-issuer hazard exists and every
-// accumulator is summed in a fixed order (bitwise reproducible results).
+//   stage B is issued by Y, or (config flag XSHARE) split between the
+//      issuers by accumulator: X then owns B and dOtil0 (Pass 1) or the value
+//      gradient (column engine) and Y the rest.
+// Every accumulator has one writer issuer, so it is summed in a fixed order
+// (bitwise reproducible results).  With XSHARE the one cross-issuer hazard is
+// that DC(t+1) overwrites operand tiles X's stage-B MMAs of tile t read: X
+// commits those MMAs to bar_xb and Y waits for that before issuing DC(t+1).
 //
 // A single thread issues at most one tcgen05.mma about every 53 cycles and
 // the tensor core needs N >= 128 per instruction to stay busy, so MMAs that
@@ -55,8 +59,9 @@
 
 namespace fbob {
 
-constexpr uint32_t kColSF = 256;  // stage-A area of issuer X
-constexpr uint32_t kColDC = 384;  // stage-A area of issuer Y
+constexpr uint32_t kColSF = 256;   // stage-A area of issuer X
+constexpr uint32_t kColDC = 384;   // stage-A area of issuer Y
+constexpr uint32_t kColDC1 = 128;  // second DC buffer (column engine, d = 64)
 
 // Shared-memory bookkeeping block (in the MISC area).
 struct Misc {
@@ -67,12 +72,14 @@ struct Misc {
   uint64_t bar_sa_sf;   // X's stage A of a tile completed
   uint64_t bar_sf_free; // elementwise warps copied SF to registers
   uint64_t bar_sa_dc[2];
-  uint64_t bar_ew[2];
+  uint64_t bar_ew[4];   // [DC buffer][half]; a single DC buffer uses [0..1]
+  uint64_t bar_xb[2];   // issuer X's stage-B MMAs completed (per half, or per DC buffer)
   uint64_t bar_acc;
   uint32_t tmem_base;
   uint32_t pad;
   WaitCtl wctl;
 };
+static_assert(sizeof(Misc) <= 256, "Misc must fit the first 256 bytes of the MISC area");
 
 __device__ __forceinline__ uint32_t lane_base_addr(uint32_t tmem_base, int warp) {
   return tmem_base + ((uint32_t)(32 * (warp & 3)) << 16);
@@ -201,8 +208,9 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
     mbar_init(&m->bar_sf_free, kEwThreads);
     for (int h = 0; h < 2; ++h) {
       mbar_init(&m->bar_sa_dc[h], 1);
-      mbar_init(&m->bar_ew[h], kEwThreads);
+      mbar_init(&m->bar_xb[h], 1);
     }
+    for (int h = 0; h < 4; ++h) mbar_init(&m->bar_ew[h], kEwThreads);
     mbar_init(&m->bar_acc, 2);
     fence_mbar_init();
   }
@@ -281,14 +289,55 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
       auto kd = [&](uint64_t kd0, int t, int h, int k) -> uint64_t {
         return kd0 + (uint64_t)((soff<C::NSTREAM, kBob>(t, h, k / 4) + (k % 4) * 32) >> 4);
       };
+      // stage B of half h: K-steps s = 2h + sub, 16 streamed rows each; the
+      // operand tiles of K-step s sit at DC columns written by warpgroup sub.
+      // With C::XSHARE issuer X takes the MMAs into B and dOtil0 (part 0) and
+      // issuer Y those into G and Omega (part 1); otherwise Y takes them all
+      // (part 2).
+      auto stage_b = [&](uint32_t sb, int h, int st, int part) {
+        if (st < first_b) return;
+        constexpr uint32_t kBoxBytes = C::NSTREAM * BN * 128;
+        const uint64_t md0 = sdesc_sw128(sb, kBoxBytes, 1024);
+#pragma unroll
+        for (int sub = 0; sub < 2; ++sub) {
+          const int s = 2 * h + sub;
+          auto md = [&](int t, int bo) -> uint64_t {
+            return md0 + (uint64_t)((soff<C::NSTREAM, kBob>(t, h, bo) + sub * 2048) >> 4);
+          };
+          const uint32_t first = (st == first_b && s == 0) ? 0u : 1u;
+          if constexpr (kBob) {
+            const uint32_t A = tmem + kColDC + 64 * h + 16 * sub;
+            const uint32_t k_rows = sb + soff<C::NSTREAM, kBob>(0, h, split) + sub * 2048;
+            if (part != 1) {
+              // [B | dOtil0] += P [K | U_V]   (second 64-wide block at U_V)
+              const uint64_t fKUV = sdesc_sw128(
+                  k_rows,
+                  soff<C::NSTREAM, kBob>(3, h, split) - soff<C::NSTREAM, kBob>(0, h, split),
+                  1024);
+              mma_ts(tmem + 0, A + 0, fKUV, id_b2, first);
+              mma_ts(tmem + 64, A + 8, md(2, split), id_b, 1);  // dOtil0 += (P o F) V
+            }
+            if (part != 0) {
+              // [G | Omega] += dS [K | U_K] ;  Omega += (P o Pt0) K
+              const uint64_t fKUK = sdesc_sw128(
+                  k_rows,
+                  soff<C::NSTREAM, kBob>(1, h, split) - soff<C::NSTREAM, kBob>(0, h, split),
+                  1024);
+              mma_ts(tmem + 128, A + 40, fKUK, id_b2, first);
+              mma_ts(tmem + 192, A + 32, md(0, split), id_b, 1);
+            }
+          } else if constexpr (OP == RowOp::BwdDQ) {
+            mma_ts(tmem + 0, tmem + kColDC + 16 * s, md(0, 0), id_b, first);  // dQ += dS K
+          } else {
+            mma_ts(tmem + 0, tmem + kColDC + 16 * s, md(1, 0), id_b, first);  // O += P V
+          }
+        }
+      };
       if (warp == kMmaWarp) {
-        // ---------------- issuer X: SF(t) = scores (and F) of tile t
-        bool ok = mbar_wait(&m->bar_stat, 0, wctl);
-        for (int st = 0; ok && st < nsteps; ++st) {
-          if (st > 0 && !mbar_wait(&m->bar_sf_free, (st - 1) & 1, wctl)) break;
+        // ---------------- issuer X: SF(t) = scores (and F) of tile t, and
+        // with C::XSHARE the stage-B MMAs into its accumulators B and dOtil0
+        auto stage_sf = [&](int st) {
           const int stage = st % C::NSTAGES;
-          if (!mbar_wait(&m->bar_full[stage], (st / C::NSTAGES) & 1, wctl)) break;
-          tc_fence_after();
           const uint64_t kd0 = sdesc_sw128(smem_u32(s_stream + stage * C::STAGE_BYTES), 16, 1024);
           const uint32_t R = tmem + kColSF;
           if constexpr (kBob) {
@@ -304,13 +353,46 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
             for (int k = 0; k < D / 16; ++k)  // S = Q K^T
               mma_ss(R + 0, sd(0, k), kd(kd0, 0, 0, k), id_n64, k > 0);
           }
+        };
+        bool ok = mbar_wait(&m->bar_stat, 0, wctl) && mbar_wait(&m->bar_full[0], 0, wctl);
+        if (ok) {
+          tc_fence_after();
+          stage_sf(0);
           mma_commit(&m->bar_sa_sf);
+        }
+        for (int st = 0; ok && st < nsteps; ++st) {
+          const int stage = st % C::NSTAGES;
+          if (st + 1 < nsteps) {  // SF(t+1) once the elementwise warps hold SF(t)
+            if (!mbar_wait(&m->bar_sf_free, st & 1, wctl) ||
+                !mbar_wait(&m->bar_full[(st + 1) % C::NSTAGES], ((st + 1) / C::NSTAGES) & 1, wctl))
+              break;
+            tc_fence_after();
+            stage_sf(st + 1);
+            mma_commit(&m->bar_sa_sf);
+          }
+          if constexpr (C::XSHARE) {
+            // V and U_V of this stage (already observed by issuer Y; the wait
+            // makes the acquire explicit)
+            if (!mbar_wait(&m->bar_full_b[stage], (st / C::NSTAGES) & 1, wctl)) break;
+            const uint32_t sb = smem_u32(s_stream + stage * C::STAGE_BYTES);
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              if (!mbar_wait(&m->bar_ew[h], st & 1, wctl)) {
+                ok = false;
+                break;
+              }
+              tc_fence_after();
+              stage_b(sb, h, st, 0);
+              mma_commit(&m->bar_xb[h]);
+            }
+            if (!ok) break;
+          }
           mma_commit(&m->bar_empty[stage]);
         }
         mma_commit(&m->bar_acc);
         if (*abort_flag) drain_wait(&m->bar_acc, 0);
       } else {
-        // ---------------- issuer Y: DC(t) and every stage-B MMA
+        // ---------------- issuer Y: DC(t) and the remaining stage-B MMAs
         auto stage_dc = [&](uint32_t sb, int h) {
           const uint64_t kd0 = sdesc_sw128(sb, 16, 1024);
           if constexpr (kBob) {  // [dP_h | C_h] = dO [V_h ; U_V_h]^T
@@ -321,43 +403,6 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)
               mma_ss(tmem + kColDC, sd(1, k), kd(kd0, 1, 0, k), id_n64, k > 0);
-          }
-        };
-        // stage B of half h: K-steps s = 2h + sub, 16 streamed rows each; the
-        // operand tiles of K-step s sit at DC columns written by warpgroup sub
-        auto stage_b = [&](uint32_t sb, int h, int st) {
-          if (st < first_b) return;
-          constexpr uint32_t kBoxBytes = C::NSTREAM * BN * 128;
-          const uint64_t md0 = sdesc_sw128(sb, kBoxBytes, 1024);
-#pragma unroll
-          for (int sub = 0; sub < 2; ++sub) {
-            const int s = 2 * h + sub;
-            auto md = [&](int t, int bo) -> uint64_t {
-              return md0 + (uint64_t)((soff<C::NSTREAM, kBob>(t, h, bo) + sub * 2048) >> 4);
-            };
-            const uint32_t first = (st == first_b && s == 0) ? 0u : 1u;
-            if constexpr (kBob) {
-              const uint32_t A = tmem + kColDC + 64 * h + 16 * sub;
-              const uint32_t k_rows = sb + soff<C::NSTREAM, kBob>(0, h, split) + sub * 2048;
-              // [B | dOtil0] += P [K | U_V]   (second 64-wide block at U_V)
-              const uint64_t fKUV = sdesc_sw128(
-                  k_rows,
-                  soff<C::NSTREAM, kBob>(3, h, split) - soff<C::NSTREAM, kBob>(0, h, split),
-                  1024);
-              mma_ts(tmem + 0, A + 0, fKUV, id_b2, first);
-              mma_ts(tmem + 64, A + 8, md(2, split), id_b, 1);  // dOtil0 += (P o F) V
-              // [G | Omega] += dS [K | U_K] ;  Omega += (P o Pt0) K
-              const uint64_t fKUK = sdesc_sw128(
-                  k_rows,
-                  soff<C::NSTREAM, kBob>(1, h, split) - soff<C::NSTREAM, kBob>(0, h, split),
-                  1024);
-              mma_ts(tmem + 128, A + 40, fKUK, id_b2, first);
-              mma_ts(tmem + 192, A + 32, md(0, split), id_b, 1);
-            } else if constexpr (OP == RowOp::BwdDQ) {
-              mma_ts(tmem + 0, tmem + kColDC + 16 * s, md(0, 0), id_b, first);  // dQ += dS K
-            } else {
-              mma_ts(tmem + 0, tmem + kColDC + 16 * s, md(1, 0), id_b, first);  // O += P V
-            }
           }
         };
         // issuer Y reads every streamed tensor: wait for both halves of a stage
@@ -389,10 +434,16 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
               break;
             }
             tc_fence_after();
-            stage_b(sb, h, st);
+            stage_b(sb, h, st, C::XSHARE ? 1 : 2);
             if (h == 1) mma_commit(&m->bar_empty[stage]);
             if (more && (kDcHalves || h == 1)) {
               if ((h == 0 || !kDcHalves) && !wait_stage(nstage, ((st + 1) / C::NSTAGES) & 1)) {
+                ok = false;
+                break;
+              }
+              // DC(t+1) of half h overwrites the operand tiles that issuer
+              // X's stage-B MMAs of half h read; wait for their completion
+              if (C::XSHARE && !mbar_wait(&m->bar_xb[h], st & 1, wctl)) {
                 ok = false;
                 break;
               }
@@ -661,6 +712,10 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
   }
   // ---- tile decode (as in the row engine); key block 0 has the most work
   // under the causal mask
+  // DC buffer of tile t, and the phase parity of its per-buffer barriers
+  auto dc_sel = [](int t) -> int { return C::DC2 ? (t & 1) : 0; };
+  auto dc_col = [](int t) -> uint32_t { return (C::DC2 && (t & 1)) ? kColDC1 : kColDC; };
+  auto dc_par = [](int t) -> uint32_t { return C::DC2 ? ((t >> 1) & 1) : (t & 1); };
   const int N = p.N;
   const int lin = blockIdx.x;
   const int cb = p.head_major ? lin % p.nblk : lin / p.BH;
@@ -683,8 +738,9 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
     mbar_init(&m->bar_sf_free, kEwThreads);
     for (int h = 0; h < 2; ++h) {
       mbar_init(&m->bar_sa_dc[h], 1);
-      mbar_init(&m->bar_ew[h], kEwThreads);
+      mbar_init(&m->bar_xb[h], 1);
     }
+    for (int h = 0; h < 4; ++h) mbar_init(&m->bar_ew[h], kEwThreads);
     mbar_init(&m->bar_acc, 2);
     fence_mbar_init();
   }
@@ -775,14 +831,38 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
       auto kd = [&](uint64_t kd0, int t, int k) -> uint64_t {
         return kd0 + (uint64_t)((soff<C::NSTREAM, false>(t, 0, k / 4) + (k % 4) * 32) >> 4);
       };
+      // stage B of half h (K-steps s = 2h + sub).  With C::XSHARE issuer X
+      // takes the MMAs into the value accumulator (part 0) and issuer Y those
+      // into the key accumulator (part 1); otherwise Y takes them all (part 2).
+      auto stage_b = [&](uint32_t sb, int h, int st, int part) {
+        constexpr uint32_t kBoxBytes = C::NSTREAM * BN * 128;
+        const uint32_t dcol = dc_col(st);
+        const uint64_t md0 = sdesc_sw128(sb, kBoxBytes, 1024);
+#pragma unroll
+        for (int sub = 0; sub < 2; ++sub) {
+          const int s = 2 * h + sub;
+          auto md = [&](int t) -> uint64_t {
+            return md0 + (uint64_t)((soff<C::NSTREAM, false>(t, h, 0) + sub * 2048) >> 4);
+          };
+          const uint32_t first = (st == 0 && s == 0) ? 0u : 1u;
+          const uint32_t A = tmem + dcol + 16 * s;
+          if constexpr (kBob) {
+            if (part != 1) mma_ts(tmem + D, A + 0, md(2), id_b, first);  // Vtil += (P o h)^T dO
+            if (part != 0) {
+              mma_ts(tmem + 0, A + 8, md(0), id_b, first);  // Ktil += Stil^T Q
+              mma_ts(tmem + 0, A + 64, md(1), id_b, 1);     //      += dS^T U_Q
+            }
+          } else {
+            if (part != 1) mma_ts(tmem + D, A + 0, md(1), id_b, first);  // dV += P^T dO
+            if (part != 0) mma_ts(tmem + 0, A + 8, md(0), id_b, first);  // dK += dS^T Q
+          }
+        }
+      };
       if (warp == kMmaWarp) {
-        // ---------------- issuer X: SF(t) = transposed scores (and F)
-        bool ok = mbar_wait(&m->bar_stat, 0, wctl);
-        for (int st = 0; ok && st < nsteps; ++st) {
-          if (st > 0 && !mbar_wait(&m->bar_sf_free, (st - 1) & 1, wctl)) break;
+        // ---------------- issuer X: SF(t) = transposed scores (and F), and
+        // with C::XSHARE the stage-B MMAs into the value accumulator
+        auto stage_sf = [&](int st) {
           const int stage = st % C::NSTAGES;
-          if (!mbar_wait(&m->bar_full[stage], (st / C::NSTAGES) & 1, wctl)) break;
-          tc_fence_after();
           const uint64_t kd0 = sdesc_sw128(smem_u32(s_stream + stage * C::STAGE_BYTES), 16, 1024);
           const uint32_t R = tmem + kColSF;
           if constexpr (kBob) {
@@ -798,79 +878,102 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
             for (int k = 0; k < D / 16; ++k)  // S^T = K Q^T
               mma_ss(R + 0, sd(0, k), kd(kd0, 0, k), id_n64, k > 0);
           }
+        };
+        bool ok = mbar_wait(&m->bar_stat, 0, wctl) && mbar_wait(&m->bar_full[0], 0, wctl);
+        if (ok) {
+          tc_fence_after();
+          stage_sf(0);
           mma_commit(&m->bar_sa_sf);
+        }
+        for (int st = 0; ok && st < nsteps; ++st) {
+          const int stage = st % C::NSTAGES;
+          if (st + 1 < nsteps) {  // SF(t+1) once the elementwise warps hold SF(t)
+            if (!mbar_wait(&m->bar_sf_free, st & 1, wctl) ||
+                !mbar_wait(&m->bar_full[(st + 1) % C::NSTAGES], ((st + 1) / C::NSTAGES) & 1, wctl))
+              break;
+            tc_fence_after();
+            stage_sf(st + 1);
+            mma_commit(&m->bar_sa_sf);
+          }
+          if constexpr (C::XSHARE) {
+            // dO of this stage (already observed by issuer Y; explicit acquire)
+            if (!mbar_wait(&m->bar_full_b[stage], (st / C::NSTAGES) & 1, wctl)) break;
+            const uint32_t sb = smem_u32(s_stream + stage * C::STAGE_BYTES);
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              if (!mbar_wait(&m->bar_ew[2 * dc_sel(st) + h], dc_par(st), wctl)) {
+                ok = false;
+                break;
+              }
+              tc_fence_after();
+              stage_b(sb, h, st, 0);
+            }
+            if (!ok) break;
+            mma_commit(&m->bar_xb[dc_sel(st)]);
+          }
           mma_commit(&m->bar_empty[stage]);
         }
         mma_commit(&m->bar_acc);
         if (*abort_flag) drain_wait(&m->bar_acc, 0);
       } else {
-        // ---------------- issuer Y: DC(t) and every stage-B MMA
-        auto stage_dc = [&](uint32_t sb) {
-          const uint64_t kd0 = sdesc_sw128(sb, 16, 1024);
+        // ---------------- issuer Y: DC(t) and the key-accumulator MMAs
+        // DC(t) of streamed tile t (stage buffer of tile t) into its DC buffer
+        auto stage_dc = [&](int t) {
+          const uint64_t kd0 =
+              sdesc_sw128(smem_u32(s_stream + (t % C::NSTAGES) * C::STAGE_BYTES), 16, 1024);
+          const uint32_t dcol = tmem + dc_col(t);
           if constexpr (kBob) {
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)  // dP^T = V dO^T
-              mma_ss(tmem + kColDC, sd(1, k), kd(kd0, 2, k), id_n64, k > 0);
+              mma_ss(dcol, sd(1, k), kd(kd0, 2, k), id_n64, k > 0);
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)  // C^T = U_V dO^T
-              mma_ss(tmem + kColDC + 64, sd(3, k), kd(kd0, 2, k), id_n64, k > 0);
+              mma_ss(dcol + 64, sd(3, k), kd(kd0, 2, k), id_n64, k > 0);
           } else {
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)  // dP^T = V dO^T
-              mma_ss(tmem + kColDC, sd(1, k), kd(kd0, 1, k), id_n64, k > 0);
+              mma_ss(dcol, sd(1, k), kd(kd0, 1, k), id_n64, k > 0);
           }
-        };
-        auto stage_b = [&](uint32_t sb, int h, int st) {
-          constexpr uint32_t kBoxBytes = C::NSTREAM * BN * 128;
-          const uint64_t md0 = sdesc_sw128(sb, kBoxBytes, 1024);
-#pragma unroll
-          for (int sub = 0; sub < 2; ++sub) {
-            const int s = 2 * h + sub;
-            auto md = [&](int t) -> uint64_t {
-              return md0 + (uint64_t)((soff<C::NSTREAM, false>(t, h, 0) + sub * 2048) >> 4);
-            };
-            const uint32_t first = (st == 0 && s == 0) ? 0u : 1u;
-            const uint32_t A = tmem + kColDC + 16 * s;
-            if constexpr (kBob) {
-              mma_ts(tmem + D, A + 0, md(2), id_b, first);    // Vtil += (P o h)^T dO
-              mma_ts(tmem + 0, A + 8, md(0), id_b, first);    // Ktil += Stil^T Q
-              mma_ts(tmem + 0, A + 64, md(1), id_b, 1);       //      += dS^T U_Q
-            } else {
-              mma_ts(tmem + D, A + 0, md(1), id_b, first);    // dV += P^T dO
-              mma_ts(tmem + 0, A + 8, md(0), id_b, first);    // dK += dS^T Q
-            }
-          }
+          mma_commit(&m->bar_sa_dc[dc_sel(t)]);
         };
         auto wait_stage = [&](int stg, uint32_t par) {
           return mbar_wait(&m->bar_full[stg], par, wctl) &&
                  mbar_wait(&m->bar_full_b[stg], par, wctl);
         };
-        bool ok = mbar_wait(&m->bar_stat, 0, wctl) && wait_stage(0, 0);
-        if (ok) {
-          tc_fence_after();
-          stage_dc(smem_u32(s_stream));
-          mma_commit(&m->bar_sa_dc[0]);
+        // with two DC buffers DC runs two tiles ahead of stage B: DC(t+2) is
+        // issued right after stage B(t), whose operand tiles it overwrites
+        constexpr int kAhead = C::DC2 ? 2 : 1;
+        bool ok = mbar_wait(&m->bar_stat, 0, wctl);
+        for (int t = 0; ok && t < kAhead && t < nsteps; ++t) {
+          ok = wait_stage(t % C::NSTAGES, (t / C::NSTAGES) & 1);
+          if (ok) {
+            tc_fence_after();
+            stage_dc(t);
+          }
         }
         for (int st = 0; ok && st < nsteps; ++st) {
           const int stage = st % C::NSTAGES;
           const uint32_t sb = smem_u32(s_stream + stage * C::STAGE_BYTES);
 #pragma unroll
           for (int h = 0; h < 2; ++h) {
-            if (!mbar_wait(&m->bar_ew[h], st & 1, wctl)) {
+            if (!mbar_wait(&m->bar_ew[2 * dc_sel(st) + h], dc_par(st), wctl)) {
               ok = false;
               break;
             }
             tc_fence_after();
-            stage_b(sb, h, st);
+            stage_b(sb, h, st, C::XSHARE ? 1 : 2);
           }
           if (!ok) break;
           mma_commit(&m->bar_empty[stage]);
-          if (st + 1 < nsteps) {
-            const int nstage = (st + 1) % C::NSTAGES;
-            if (!wait_stage(nstage, ((st + 1) / C::NSTAGES) & 1)) break;
+          const int nx = st + kAhead;
+          if (nx < nsteps) {
+            // DC(nx) overwrites the operand tiles of tile st; with XSHARE wait
+            // for issuer X's stage-B MMAs on them as well as for the stage
+            if (!wait_stage(nx % C::NSTAGES, (nx / C::NSTAGES) & 1) ||
+                (C::XSHARE && !mbar_wait(&m->bar_xb[dc_sel(st)], dc_par(st), wctl)))
+              break;
             tc_fence_after();
-            stage_dc(smem_u32(s_stream + nstage * C::STAGE_BYTES));
-            mma_commit(&m->bar_sa_dc[0]);
+            stage_dc(nx);
           }
         }
         mma_commit(&m->bar_acc);
@@ -913,11 +1016,12 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
       }
       tc_fence_before();
       mbar_arrive(&m->bar_sf_free);
-      if (!mbar_wait(&m->bar_sa_dc[0], st & 1, wctl)) {
+      if (!mbar_wait(&m->bar_sa_dc[dc_sel(st)], dc_par(st), wctl)) {
         ok = false;
         break;
       }
       tc_fence_after();
+      const uint32_t dcol = dc_col(st);
 #pragma unroll
       for (int h = 0; h < 2; ++h) {
         const int cv = HB * h + 16 * wg;             // tile column of this thread's first
@@ -926,7 +1030,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
         // valid query columns c satisfy  lo <= c < hi
         const int lo = p.causal ? gj - ib : 0;
         const int hi = row_ok ? N - ib : 0;
-        const uint32_t R = ta + kColDC + cv;
+        const uint32_t R = ta + dcol + cv;
         if constexpr (kBob) {
           uint32_t rdP[16], rC[16];
           tmem_ld16(R + 0, rdP);
@@ -983,7 +1087,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
         }
         tmem_st_wait();
         tc_fence_before();
-        mbar_arrive(&m->bar_ew[h]);
+        mbar_arrive(&m->bar_ew[2 * dc_sel(st) + h]);
       }
     }
     if (ok) ok = mbar_wait(&m->bar_acc, 0, wctl);

@@ -60,6 +60,9 @@ struct RowCfg {
   static constexpr int STAT_BYTES = NSTAT * KB * BM * 128;
   static constexpr int STAGE_BYTES = NSTREAM * KB * BN * 128;
   static constexpr int NSTAGES = OP == RowOp::BobPass1 ? (D == 64 ? 3 : 2) : 4;
+  // issuer X also issues the stage-B MMAs into B and dOtil0 (measured faster
+  // at d = 64 only: at d = 128 the extra cross-issuer wait costs more)
+  static constexpr bool XSHARE = OP == RowOp::BobPass1 && D == 64;
   static constexpr int MISC_BYTES = 2304;
   static constexpr int SMEM_BYTES = STAT_BYTES + NSTAGES * STAGE_BYTES + MISC_BYTES;
 };
@@ -74,6 +77,13 @@ struct ColCfg {
   static constexpr int TILE_BYTES = NSTREAM * KB * BN * 128;
   static constexpr int STAGE_BYTES = TILE_BYTES + 1024;  // + row vectors
   static constexpr int NSTAGES = (OP == ColOp::BobPass2 && D == 128) ? 2 : (D == 64 ? 4 : 3);
+  // two DC buffers in TMEM (DC(t+1) is issued before stage B(t)): possible
+  // when the accumulators (2 D columns) leave columns 128..255 free
+  static constexpr bool DC2 = D == 64;
+  // issuer X takes the value-accumulator MMAs of stage B.  With one DC buffer
+  // issuer Y would have to wait for them before the next DC (measured slower);
+  // with two that wait is two tiles back and off the critical path.
+  static constexpr bool XSHARE = DC2;
   static constexpr int MISC_BYTES = 256;
   static constexpr int SMEM_BYTES = STAT_BYTES + NSTAGES * STAGE_BYTES + MISC_BYTES;
 };
