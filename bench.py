@@ -35,8 +35,13 @@ from paper_2609_24089_gb300 import synth  # noqa: E402
 
 METRIC = "BoB TFLOP/s and tensor-pipe % of bf16 peak at N=16K-262K; peak HBM bytes"
 DEFAULT_WORKLOAD = "n16k_d128_causal"
-CONTRACTIONS = {"pass1": 11, "pass2": 8}
-KERNEL_NAMES = {"pass1": "row_engine<BobPass1>", "pass2": "col_engine<BobPass2>"}
+# Contractions of the fixed formula credited to each kernel: Pass 1 is 11 (Alg. 2,
+# first loop) and Pass 2 is 8.  At d = 128 Pass 1 runs as two kernels: the
+# row-statistics kernel is credited with the 5 stage-A contractions and the
+# direct-form kernel with the other 6 (its stage-A recompute is not credited).
+CONTRACTIONS = {"pass1": 11, "row_stats": 5, "pass1_direct": 6, "pass2": 8}
+KERNEL_NAMES = {"pass1": "row_engine<BobPass1>", "row_stats": "row_engine<BobStats>",
+                "pass1_direct": "row_engine<BobPass1D>", "pass2": "col_engine<BobPass2>"}
 CSRC = os.path.join(ROOT, "paper_2609_24089_gb300", "csrc")
 
 
@@ -238,27 +243,40 @@ def run_gpu(args, w):
     if fbob.fbob_device_status() != 0:
         raise RuntimeError("device status not OK after warm-up")
 
-    # ---- timed region: K steps, each as its two launches with events between
+    # ---- timed region: K steps, each as its kernels (through their C-ABI
+    # calls, the same ones fbob_attn_bob makes) with events between them
+    if w.d == 64:
+        parts = [("pass1", lambda: fbob.fbob_attn_bob_pass1(
+            shp, q, k, v, o, lse, do, gq, gk, gv, outs[0], outs[3], rs))]
+    else:
+        parts = [("row_stats", lambda: fbob.fbob_attn_bob_row_stats(
+                     shp, q, k, v, o, lse, do, gq, gk, gv, rs)),
+                 ("pass1_direct", lambda: fbob.fbob_attn_bob_pass1_direct(
+                     shp, q, k, v, lse, do, gq, gk, gv, rs, outs[0], outs[3]))]
+    parts.append(("pass2", lambda: fbob.fbob_attn_bob_pass2(
+        shp, q, k, v, lse, do, gq, gk, gv, rs, outs[1], outs[2])))
     K = args.steps
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(len(parts) + 1)] for _ in range(K)]
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     barrier()
     with ClockSampler(local) as clk:
         start.record(stream)
         for s in range(K):
             ev[s][0].record(stream)
-            fbob.fbob_attn_bob_pass1(shp, q, k, v, o, lse, do, gq, gk, gv, outs[0], outs[3], rs)
-            ev[s][1].record(stream)
-            fbob.fbob_attn_bob_pass2(shp, q, k, v, lse, do, gq, gk, gv, rs, outs[1], outs[2])
-            ev[s][2].record(stream)
+            for j, (_, call) in enumerate(parts):
+                call()
+                ev[s][j + 1].record(stream)
         stop.record(stream)
         barrier()
     status = fbob.fbob_device_status()
     if status != 0:
         raise RuntimeError(f"device status {status} in timed region")
+    launches_per_step = sum(fbob.fbob_launch_count(
+        {"pass1": "bob_pass1", "row_stats": "bob_row_stats", "pass1_direct": "bob_pass1_direct",
+         "pass2": "bob_pass2"}[name]) for name, _ in parts)
     ms = start.elapsed_time(stop)
-    t1 = [e[0].elapsed_time(e[1]) for e in ev]
-    t2 = [e[1].elapsed_time(e[2]) for e in ev]
+    part_ms = {name: sum(e[j].elapsed_time(e[j + 1]) for e in ev) / K
+               for j, (name, _) in enumerate(parts)}
     ms_t = torch.tensor([ms], device="cuda")
     if world > 1:
         dist.all_reduce(ms_t, op=dist.ReduceOp.MAX)
@@ -310,9 +328,9 @@ def run_gpu(args, w):
         return
 
     peaks = measured_peaks()
-    a1, a2 = sum(t1) / K, sum(t2) / K
-    dom = "pass1" if a1 >= a2 else "pass2"
-    dur = a1 if dom == "pass1" else a2
+    dom = max(part_ms, key=part_ms.get)
+    dur = part_ms[dom]
+    total = sum(part_ms.values())
     dflops = bob_flops(w, CONTRACTIONS[dom])
     achieved = dflops / (dur * 1e-3) / 1e12
     peak = peaks["bf16_sustained"]
@@ -320,8 +338,9 @@ def run_gpu(args, w):
                 "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
                 "peak_kind": f"bf16 sustained ({peaks['source']})",
                 "traffic": ncu_traffic(dom, w.name),
-                "launch_ms": dur, "share_of_step": dur / (a1 + a2),
-                "other_kernel_ms": a2 if dom == "pass1" else a1}
+                "credited_contractions": CONTRACTIONS[dom],
+                "launch_ms": dur, "share_of_step": dur / total,
+                "other_kernels_ms": {n: t for n, t in part_ms.items() if n != dom}}
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
         bits0 = {n: b[0, 0] for n, b in bits.items()}
@@ -342,11 +361,12 @@ def run_gpu(args, w):
         "cpu_baseline": cpu,
         "e2e": {"value": e2e_val, "unit": "TFLOP/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "ms_per_step": float(e_t.item()) / K},
-        "gpu_launches": 2 * K,
+        "gpu_launches": launches_per_step * K,
         "clocks": clk.summary(),
         "peak_hbm_bytes": footprint,
         "call_alloc_bytes": call_delta,
-        "pass_ms": {"pass1": a1, "pass2": a2},
+        "pass_ms": {"pass1": total - part_ms["pass2"], "pass2": part_ms["pass2"]},
+        "kernel_ms": part_ms,
     }
     print(json.dumps(line), flush=True)
     if world > 1:

@@ -112,7 +112,9 @@ int fbob_attn_bob(const fbob_shape* shape, const void* q, const void* k, const v
 /*
  * Pass 1 of Algorithm 1 alone (row-block outer; Alg. 2, first loop):
  * writes q_bar, dout_bar and row_stats (alpha, E, D).  Same arguments and
- * rules as fbob_attn_bob; k_bar/v_bar are not touched.
+ * rules as fbob_attn_bob; k_bar/v_bar are not touched.  d = 64 runs one
+ * sweep with the affine fusion of Prop. 3.1 (one kernel); d = 128 runs
+ * fbob_attn_bob_row_stats then fbob_attn_bob_pass1_direct (two kernels).
  */
 int fbob_attn_bob_pass1(const fbob_shape* shape, const void* q, const void* k, const void* v,
                         const void* o, const float* lse, const void* dout,
@@ -132,6 +134,32 @@ int fbob_attn_bob_pass2(const fbob_shape* shape, const void* q, const void* k, c
                         struct CUstream_st* stream);
 
 /*
+ * Row scalars of BoB alone (eq. 6): writes row_stats [3,B,H,N] = (alpha, E, D)
+ * with alpha_i = sum_j P_ij F_ij, E_i = sum_j P_ij Ptil_ij and D_i = do_i . o_i,
+ * exactly as pass 1 writes them (stage A only; no N x d output).  At d = 128
+ * fbob_attn_bob_pass1 is this call followed by fbob_attn_bob_pass1_direct.
+ * Same arguments and rules as fbob_attn_bob_pass1.
+ */
+int fbob_attn_bob_row_stats(const fbob_shape* shape, const void* q, const void* k,
+                            const void* v, const void* o, const float* lse, const void* dout,
+                            const void* gq, const void* gk, const void* gv, float* row_stats,
+                            struct CUstream_st* stream);
+
+/*
+ * Pass 1 given its row scalars: q_bar and dout_bar from eqs. (6)-(7) directly,
+ *   q_bar = scale (Stil K + dS U_K),  dout_bar = P U_V + (P o h) V,
+ * with alpha, E, D read from row_stats (as fbob_attn_bob_row_stats or pass 1
+ * writes them; input here) and P from lse.  O is not needed.
+ * In:  q, k, v, dout, gq, gk, gv bf16; lse fp32; row_stats fp32 [3,B,H,N].
+ * Out: q_bar, dout_bar bf16 [B,H,N,d].
+ */
+int fbob_attn_bob_pass1_direct(const fbob_shape* shape, const void* q, const void* k,
+                               const void* v, const float* lse, const void* dout,
+                               const void* gq, const void* gk, const void* gv,
+                               const float* row_stats, void* q_bar, void* dout_bar,
+                               struct CUstream_st* stream);
+
+/*
  * Synchronises `stream`, then returns and clears the device error word of the
  * current device: FBOB_OK, FBOB_ERR_DEVICE_TIMEOUT (a bounded wait expired in
  * some kernel since the last call), or FBOB_ERR_DEVICE_FAULT / FBOB_ERR_CUDA
@@ -140,7 +168,8 @@ int fbob_attn_bob_pass2(const fbob_shape* shape, const void* q, const void* k, c
 int fbob_device_status(struct CUstream_st* stream);
 
 /* Number of kernels the last successful call of the named entry point
- * enqueued ("fwd", "bwd", "bob", "bob_pass1", "bob_pass2"); -1 if unknown. */
+ * enqueued ("fwd", "bwd", "bob", "bob_pass1", "bob_pass2", "bob_row_stats",
+ * "bob_pass1_direct"); -1 if unknown. */
 int fbob_launch_count(const char* entry);
 
 /* Static, human-readable name of a status code. */

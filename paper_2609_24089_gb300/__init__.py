@@ -58,6 +58,8 @@ def load():
         "fbob_attn_bob": [S, P, P, P, P, P, P, P, P, P, P, P, P, P, P, P],
         "fbob_attn_bob_pass1": [S, P, P, P, P, P, P, P, P, P, P, P, P, P],
         "fbob_attn_bob_pass2": [S, P, P, P, P, P, P, P, P, P, P, P, P],
+        "fbob_attn_bob_row_stats": [S, P, P, P, P, P, P, P, P, P, P, P],
+        "fbob_attn_bob_pass1_direct": [S, P, P, P, P, P, P, P, P, P, P, P, P],
         "fbob_device_status": [P],
         "fbob_launch_count": [ctypes.c_char_p],
         "fbob_status_string": [ctypes.c_int],
@@ -141,6 +143,21 @@ def fbob_attn_bob_pass2(shape, q, k, v, lse, dout, gq, gk, gv, row_stats, k_bar,
         ctypes.byref(shape),
         *map(_ptr, (q, k, v, lse, dout, gq, gk, gv, row_stats, k_bar, v_bar)),
         _stream(stream)), "fbob_attn_bob_pass2")
+
+
+def fbob_attn_bob_row_stats(shape, q, k, v, o, lse, dout, gq, gk, gv, row_stats, stream=None):
+    _check(load().fbob_attn_bob_row_stats(
+        ctypes.byref(shape),
+        *map(_ptr, (q, k, v, o, lse, dout, gq, gk, gv, row_stats)),
+        _stream(stream)), "fbob_attn_bob_row_stats")
+
+
+def fbob_attn_bob_pass1_direct(shape, q, k, v, lse, dout, gq, gk, gv, row_stats, q_bar, dout_bar,
+                               stream=None):
+    _check(load().fbob_attn_bob_pass1_direct(
+        ctypes.byref(shape),
+        *map(_ptr, (q, k, v, lse, dout, gq, gk, gv, row_stats, q_bar, dout_bar)),
+        _stream(stream)), "fbob_attn_bob_pass1_direct")
 
 
 def fbob_device_status(stream=None) -> int:

@@ -4,7 +4,10 @@
 // Two engines share one schedule skeleton:
 //   * row engine: a CTA owns BM = 128 query rows (TMEM lanes) and streams key
 //     tiles of BN = 64 rows.  Used by the forward (eq. 1), the dQ half of the
-//     first backward (eqs. 2-3) and BoB Pass 1 (Alg. 2, first loop).
+//     first backward (eqs. 2-3) and BoB Pass 1 (Alg. 2, first loop): at
+//     d = 64 in one sweep with the affine fusion of Prop. 3.1 (four
+//     accumulators); at d = 128 as a row-statistics kernel (alpha, E, D; stage
+//     A only) followed by the direct form of eqs. (6)-(7) (two accumulators).
 //   * column engine: a CTA owns BM = 128 key rows and streams query tiles of
 //     BN = 64 rows, computing transposed tiles (key rows on lanes).  Used by
 //     the dK/dV half of the first backward and BoB Pass 2 (Alg. 2, second loop).
@@ -71,6 +74,7 @@ struct Misc {
   uint64_t bar_empty[4];
   uint64_t bar_sa_sf;   // X's stage A of a tile completed
   uint64_t bar_sf_free; // elementwise warps copied SF to registers
+  uint64_t bar_dc_free; // elementwise warps copied DC to registers (row statistics kernel)
   uint64_t bar_sa_dc[2];
   uint64_t bar_ew[4];   // [DC buffer][half]; a single DC buffer uses [0..1]
   uint64_t bar_xb[2];   // issuer X's stage-B MMAs completed (per half, or per DC buffer)
@@ -162,8 +166,11 @@ __device__ __forceinline__ float2 probs2(float2 s, float2 sl2, float2 nL2) {
 template <RowOp OP, int D>
 __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant__ EngineParams p) {
   using C = RowCfg<OP, D>;
-  constexpr bool kBob = OP == RowOp::BobPass1;
-  constexpr bool kDcHalves = kBob;  // Pass 1 issues DC per 32-column half
+  constexpr bool kBob = OP == RowOp::BobPass1;      // Pass 1, one sweep (Prop. 3.1)
+  constexpr bool kStats = OP == RowOp::BobStats;    // row scalars alpha, E, D only
+  constexpr bool kDirect = OP == RowOp::BobPass1D;  // Pass 1 with alpha, E given
+  constexpr bool kB4 = row_bob(OP);                 // streamed K, U_K, V, U_V
+  constexpr bool kDcHalves = kBob || kDirect;       // DC issued per 32-column half
   extern __shared__ __align__(1024) uint8_t smem[];
   uint8_t* s_stat = smem;
   uint8_t* s_stream = smem + C::STAT_BYTES;
@@ -177,15 +184,12 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
     return;
   }
 
-  // ---- tile decode.  The two output halves of a row block (d = 128) are
-  // adjacent.  Head-major order: the CTAs in flight work on the row blocks of
-  // one or two heads and stream the same K/V tiles, which then stay in L2.
-  // Otherwise heads are innermost, so with the causal mask the longest row
-  // blocks of all heads go first (better balance, less sharing).
+  // ---- tile decode.  Head-major order: the CTAs in flight work on the row
+  // blocks of one or two heads and stream the same K/V tiles, which then stay
+  // in L2.  Otherwise heads are innermost, so with the causal mask the longest
+  // row blocks of all heads go first (better balance, less sharing).
   const int N = p.N;
-  int lin = blockIdx.x;
-  const int split = lin % C::NSPLIT;
-  lin /= C::NSPLIT;
+  const int lin = blockIdx.x;
   const int rbi = p.head_major ? lin % p.nblk : lin / p.BH;
   const int bh = p.head_major ? lin / p.nblk : lin % p.BH;
   const int rb = p.causal ? (p.nblk - 1 - rbi) : rbi;
@@ -206,6 +210,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
     }
     mbar_init(&m->bar_sa_sf, 1);
     mbar_init(&m->bar_sf_free, kEwThreads);
+    mbar_init(&m->bar_dc_free, kEwThreads);
     for (int h = 0; h < 2; ++h) {
       mbar_init(&m->bar_sa_dc[h], 1);
       mbar_init(&m->bar_xb[h], 1);
@@ -246,20 +251,20 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         const bool k_only = (OP == RowOp::Fwd) && st < ntiles;
         const int nt = k_only ? 1 : C::NSTREAM;
         uint8_t* dst = s_stream + stage * C::STAGE_BYTES;
-        // Pass 1: K and U_K first on bar_full (all issuer X needs), then V and
+        // BoB: K and U_K first on bar_full (all issuer X needs), then V and
         // U_V on bar_full_b; the other operations use bar_full alone
-        const int nt_a = kBob ? 2 : nt;
+        const int nt_a = kB4 ? 2 : nt;
         mbar_arrive_expect_tx(&m->bar_full[stage], nt_a * C::KB * BN * 128);
         for (int b = 0; b < C::KB; ++b)
           for (int t = 0; t < nt_a; ++t)
-            tma_load_3d(dst + soff<C::NSTREAM, kBob>(t, 0, b), &p.tm[C::NSTAT + t],
+            tma_load_3d(dst + soff<C::NSTREAM, kB4>(t, 0, b), &p.tm[C::NSTAT + t],
                         &m->bar_full[stage], 64 * b, j0, bh);
-        if (kBob) {  // 32-row chunks (map box rows HB)
+        if (kB4) {  // 32-row chunks (map box rows HB)
           mbar_arrive_expect_tx(&m->bar_full_b[stage], 2 * C::KB * BN * 128);
           for (int b = 0; b < C::KB; ++b)
             for (int t = 2; t < 4; ++t)
               for (int h = 0; h < 2; ++h)
-                tma_load_3d(dst + soff<C::NSTREAM, kBob>(t, h, b), &p.tm[C::NSTAT + t],
+                tma_load_3d(dst + soff<C::NSTREAM, kB4>(t, h, b), &p.tm[C::NSTAT + t],
                             &m->bar_full_b[stage], 64 * b, j0 + HB * h, bh);
         }
         issued[stage] = st;
@@ -268,7 +273,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         for (int s = 0; s < C::NSTAGES; ++s)
           if (issued[s] >= 0) {
             drain_wait(&m->bar_full[s], (issued[s] / C::NSTAGES) & 1);
-            if (kBob) drain_wait(&m->bar_full_b[s], (issued[s] / C::NSTAGES) & 1);
+            if (kB4) drain_wait(&m->bar_full_b[s], (issued[s] / C::NSTAGES) & 1);
           }
         drain_wait(&m->bar_stat, 0);
       }
@@ -278,8 +283,8 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
     if (elect_lane0()) {
       constexpr uint32_t id_n64 = idesc_bf16(128, 64, false);
       constexpr uint32_t id_n128 = idesc_bf16(128, 128, false);
-      constexpr uint32_t id_b = idesc_bf16(128, C::DOUT, true);
-      constexpr uint32_t id_b2 = idesc_bf16(128, 2 * C::DOUT, true);
+      constexpr uint32_t id_b = idesc_bf16(128, D, true);
+      constexpr uint32_t id_b2 = idesc_bf16(128, 2 * D, true);
       // descriptors are formed once; per MMA only the start-address field moves
       const uint64_t sd0 = sdesc_sw128(smem_u32(s_stat), 16, 1024);
       auto sd = [&](int t, int k) -> uint64_t {
@@ -287,7 +292,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
       };
       // K-major view of streamed rows 32h.. (64 of them) of tensor t, K-step k
       auto kd = [&](uint64_t kd0, int t, int h, int k) -> uint64_t {
-        return kd0 + (uint64_t)((soff<C::NSTREAM, kBob>(t, h, k / 4) + (k % 4) * 32) >> 4);
+        return kd0 + (uint64_t)((soff<C::NSTREAM, kB4>(t, h, k / 4) + (k % 4) * 32) >> 4);
       };
       // stage B of half h: K-steps s = 2h + sub, 16 streamed rows each; the
       // operand tiles of K-step s sit at DC columns written by warpgroup sub.
@@ -302,30 +307,37 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         for (int sub = 0; sub < 2; ++sub) {
           const int s = 2 * h + sub;
           auto md = [&](int t, int bo) -> uint64_t {
-            return md0 + (uint64_t)((soff<C::NSTREAM, kBob>(t, h, bo) + sub * 2048) >> 4);
+            return md0 + (uint64_t)((soff<C::NSTREAM, kB4>(t, h, bo) + sub * 2048) >> 4);
           };
           const uint32_t first = (st == first_b && s == 0) ? 0u : 1u;
           if constexpr (kBob) {
             const uint32_t A = tmem + kColDC + 64 * h + 16 * sub;
-            const uint32_t k_rows = sb + soff<C::NSTREAM, kBob>(0, h, split) + sub * 2048;
+            const uint32_t k_rows = sb + soff<C::NSTREAM, kB4>(0, h, 0) + sub * 2048;
             if (part != 1) {
               // [B | dOtil0] += P [K | U_V]   (second 64-wide block at U_V)
               const uint64_t fKUV = sdesc_sw128(
                   k_rows,
-                  soff<C::NSTREAM, kBob>(3, h, split) - soff<C::NSTREAM, kBob>(0, h, split),
+                  soff<C::NSTREAM, kB4>(3, h, 0) - soff<C::NSTREAM, kB4>(0, h, 0),
                   1024);
               mma_ts(tmem + 0, A + 0, fKUV, id_b2, first);
-              mma_ts(tmem + 64, A + 8, md(2, split), id_b, 1);  // dOtil0 += (P o F) V
+              mma_ts(tmem + 64, A + 8, md(2, 0), id_b, 1);  // dOtil0 += (P o F) V
             }
             if (part != 0) {
               // [G | Omega] += dS [K | U_K] ;  Omega += (P o Pt0) K
               const uint64_t fKUK = sdesc_sw128(
                   k_rows,
-                  soff<C::NSTREAM, kBob>(1, h, split) - soff<C::NSTREAM, kBob>(0, h, split),
+                  soff<C::NSTREAM, kB4>(1, h, 0) - soff<C::NSTREAM, kB4>(0, h, 0),
                   1024);
               mma_ts(tmem + 128, A + 40, fKUK, id_b2, first);
-              mma_ts(tmem + 192, A + 32, md(0, split), id_b, 1);
+              mma_ts(tmem + 192, A + 32, md(0, 0), id_b, 1);
             }
+          } else if constexpr (kDirect) {
+            // eqs. (6)-(7): Qtil += Stil K + dS U_K ; dOtil += P U_V + (P o h) V
+            const uint32_t A = tmem + kColDC + 64 * h + 16 * sub;
+            mma_ts(tmem + 0, A + 32, md(0, 0), id_b, first);
+            mma_ts(tmem + 0, A + 40, md(1, 0), id_b, 1);
+            mma_ts(tmem + D, A + 0, md(3, 0), id_b, first);
+            mma_ts(tmem + D, A + 8, md(2, 0), id_b, 1);
           } else if constexpr (OP == RowOp::BwdDQ) {
             mma_ts(tmem + 0, tmem + kColDC + 16 * s, md(0, 0), id_b, first);  // dQ += dS K
           } else {
@@ -340,7 +352,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
           const int stage = st % C::NSTAGES;
           const uint64_t kd0 = sdesc_sw128(smem_u32(s_stream + stage * C::STAGE_BYTES), 16, 1024);
           const uint32_t R = tmem + kColSF;
-          if constexpr (kBob) {
+          if constexpr (kB4) {
             // stationary: 0 Q, 1 U_Q, 2 dO ; stream: 0 K, 1 U_K, 2 V, 3 U_V
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)  // [S | F] = Q [K ; U_K]^T
@@ -354,11 +366,14 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
               mma_ss(R + 0, sd(0, k), kd(kd0, 0, 0, k), id_n64, k > 0);
           }
         };
+        // (the statistics kernel has no stage B: a stage is released as soon
+        // as the MMAs reading it complete)
         bool ok = mbar_wait(&m->bar_stat, 0, wctl) && mbar_wait(&m->bar_full[0], 0, wctl);
         if (ok) {
           tc_fence_after();
           stage_sf(0);
           mma_commit(&m->bar_sa_sf);
+          if (kStats) mma_commit(&m->bar_empty[0]);
         }
         for (int st = 0; ok && st < nsteps; ++st) {
           const int stage = st % C::NSTAGES;
@@ -369,6 +384,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
             tc_fence_after();
             stage_sf(st + 1);
             mma_commit(&m->bar_sa_sf);
+            if (kStats) mma_commit(&m->bar_empty[(st + 1) % C::NSTAGES]);
           }
           if constexpr (C::XSHARE) {
             // V and U_V of this stage (already observed by issuer Y; the wait
@@ -387,7 +403,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
             }
             if (!ok) break;
           }
-          mma_commit(&m->bar_empty[stage]);
+          if (!kStats) mma_commit(&m->bar_empty[stage]);
         }
         mma_commit(&m->bar_acc);
         if (*abort_flag) drain_wait(&m->bar_acc, 0);
@@ -395,7 +411,11 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         // ---------------- issuer Y: DC(t) and the remaining stage-B MMAs
         auto stage_dc = [&](uint32_t sb, int h) {
           const uint64_t kd0 = sdesc_sw128(sb, 16, 1024);
-          if constexpr (kBob) {  // [dP_h | C_h] = dO [V_h ; U_V_h]^T
+          if constexpr (kStats) {  // whole tile: [dP_0|C_0|dP_1|C_1] = dO [V_0;U_V_0;V_1;U_V_1]^T
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k)
+              mma_ss(tmem + kColDC, sd(2, k), kd(kd0, 2, 0, k), id_n128, k > 0);
+          } else if constexpr (kB4) {  // [dP_h | C_h] = dO [V_h ; U_V_h]^T
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)
               mma_ss(tmem + kColDC + 64 * h, sd(2, k), kd(kd0, 2, h, k), id_n64, k > 0);
@@ -408,9 +428,29 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         // issuer Y reads every streamed tensor: wait for both halves of a stage
         auto wait_stage = [&](int stg, uint32_t par) {
           return mbar_wait(&m->bar_full[stg], par, wctl) &&
-                 (!kBob || mbar_wait(&m->bar_full_b[stg], par, wctl));
+                 (!kB4 || mbar_wait(&m->bar_full_b[stg], par, wctl));
         };
         bool ok = mbar_wait(&m->bar_stat, 0, wctl) && wait_stage(0, 0);
+        if constexpr (kStats) {
+          // DC(t+1) once the elementwise warps hold DC(t) in registers
+          if (ok) {
+            tc_fence_after();
+            stage_dc(smem_u32(s_stream), 0);
+            mma_commit(&m->bar_sa_dc[0]);
+            mma_commit(&m->bar_empty[0]);
+          }
+          for (int st = 0; ok && st + 1 < nsteps; ++st) {
+            const int ns = (st + 1) % C::NSTAGES;
+            if (!mbar_wait(&m->bar_dc_free, st & 1, wctl) ||
+                !wait_stage(ns, ((st + 1) / C::NSTAGES) & 1))
+              break;
+            tc_fence_after();
+            stage_dc(smem_u32(s_stream + ns * C::STAGE_BYTES), 0);
+            mma_commit(&m->bar_sa_dc[0]);
+            mma_commit(&m->bar_empty[ns]);
+          }
+          ok = false;  // no stage B
+        }
         if (ok) {
           tc_fence_after();
           const uint32_t sb0 = smem_u32(s_stream);
@@ -467,11 +507,18 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
     const size_t rowoff = ((size_t)bh * N + (size_t)(row_ok ? gi : 0)) * D;
     const float tau = p.scale;
     const float sl2 = tau * kLog2e;
-    float L2 = 0.f, Dr = 0.f;
+    float L2 = 0.f, Dr = 0.f, nal = 0.f, nE = 0.f;  // nal = -alpha, nE = -E (direct form)
     if constexpr (OP != RowOp::Fwd) {
       if (row_ok) {
-        L2 = p.lse[(size_t)bh * N + gi] * kLog2e;
-        Dr = row_dot<D>(p.dout + rowoff, p.o + rowoff);
+        const size_t ri = (size_t)bh * N + gi;
+        L2 = p.lse[ri] * kLog2e;
+        if constexpr (kDirect) {  // row scalars written by the statistics kernel
+          nal = -p.vec_in[ri];
+          nE = -p.vec_in[p.bhn + ri];
+          Dr = p.vec_in[2 * p.bhn + ri];
+        } else {
+          Dr = row_dot<D>(p.dout + rowoff, p.o + rowoff);
+        }
       }
     }
     float mrow = -INFINITY, lrow = 0.f;             // forward sweep 1 (log2 domain)
@@ -501,11 +548,11 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
 #pragma unroll
       for (int h = 0; h < 2; ++h) {
         tmem_ld16(ta + kColSF + HB * h + 16 * wg, rS[h]);
-        if constexpr (kBob) tmem_ld16(ta + kColSF + 64 + HB * h + 16 * wg, rF[h]);
+        if constexpr (kB4) tmem_ld16(ta + kColSF + 64 + HB * h + 16 * wg, rF[h]);
       }
       tmem_ld_wait(rS[0]);
       reg_dep(rS[1]);
-      if constexpr (kBob) {
+      if constexpr (kB4) {
         reg_dep(rF[0]);
         reg_dep(rF[1]);
       }
@@ -513,28 +560,32 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
       mbar_arrive(&m->bar_sf_free);
       const int jt = (st % ntiles) * BN;
       const float2 sl2v = splat(sl2), nL2v = splat(-L2);
-#pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        if (kDcHalves || h == 0) {
-          if (!mbar_wait(&m->bar_sa_dc[kDcHalves ? h : 0], st & 1, wctl)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
+      if constexpr (kStats) {
+        // ---- row statistics: copy DC of the whole tile, release it, then
+        // accumulate alpha = sum P F and E0 = sum P (C + F (dP - D))  (eq. 6)
+        if (!mbar_wait(&m->bar_sa_dc[0], st & 1, wctl)) {
+          ok = false;
+          break;
         }
-        const int c0 = HB * h + 16 * wg;  // tile column of this thread's 16
-        const int j0 = jt + c0;           // first key of this thread's 16
-        const bool need_mask = (!row_ok) || (j0 + 16 > N) || (p.causal && j0 + 15 > gi);
-        const int lim = need_mask ? (row_ok ? (p.causal ? min(N, gi + 1) : N) - j0 : 0) : 16;
-        if constexpr (kBob) {
-          const uint32_t R = ta + kColDC + 64 * h + 16 * wg;  // [dP_h | C_h] columns
-          uint32_t rdP[16], rC[16];
-          tmem_ld16(R + 0, rdP);
-          tmem_ld16(R + 32, rC);
-          tmem_ld_wait(rdP);
-          reg_dep(rC);
-          const float2 tauv = splat(tau), nDv = splat(-Dr);
-          uint32_t oP[8], oPF[8], oPPt[8], odS[8];
+        tc_fence_after();
+        uint32_t rdP[2][16], rC[2][16];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          tmem_ld16(ta + kColDC + 64 * h + 16 * wg, rdP[h]);
+          tmem_ld16(ta + kColDC + 64 * h + 32 + 16 * wg, rC[h]);
+        }
+        tmem_ld_wait(rdP[0]);
+        reg_dep(rdP[1]);
+        reg_dep(rC[0]);
+        reg_dep(rC[1]);
+        tc_fence_before();
+        mbar_arrive(&m->bar_dc_free);
+        const float2 tauv = splat(tau), nDv = splat(-Dr);
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const int j0 = jt + HB * h + 16 * wg;
+          const bool need_mask = (!row_ok) || (j0 + 16 > N) || (p.causal && j0 + 15 > gi);
+          const int lim = need_mask ? (row_ok ? (p.causal ? min(N, gi + 1) : N) - j0 : 0) : 16;
 #pragma unroll
           for (int c = 0; c < 16; c += 2) {
             float2 pr = probs2(pair(rS[h], c), sl2v, nL2v);
@@ -543,60 +594,35 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
               if (c + 1 >= lim) pr.y = 0.f;
             }
             const float2 f = __fmul2_rn(pair(rF[h], c), tauv);
-            const float2 dp = pair(rdP, c);
-            const float2 t = __fadd2_rn(dp, nDv);
-            const float2 pt0 = __ffma2_rn(f, t, pair(rC, c));  // Ptil0 = C + F (dP - D)
-            const float2 pf = __fmul2_rn(pr, f);
-            const float2 ppt = __fmul2_rn(pr, pt0);
-            const float2 ds = __fmul2_rn(pr, t);
-            acc_a = __fadd2_rn(acc_a, pf);
-            acc_e = __fadd2_rn(acc_e, ppt);
-            oP[c / 2] = pack_bf16(pr.x, pr.y);
-            oPF[c / 2] = pack_bf16(pf.x, pf.y);
-            oPPt[c / 2] = pack_bf16(ppt.x, ppt.y);
-            odS[c / 2] = pack_bf16(ds.x, ds.y);
+            const float2 t = __fadd2_rn(pair(rdP[h], c), nDv);
+            const float2 pt0 = __ffma2_rn(f, t, pair(rC[h], c));  // Ptil0 = C + F (dP - D)
+            acc_a = __ffma2_rn(pr, f, acc_a);
+            acc_e = __ffma2_rn(pr, pt0, acc_e);
           }
-          tmem_st8(R + 0, oP);
-          tmem_st8(R + 8, oPF);
-          tmem_st8(R + 32, oPPt);
-          tmem_st8(R + 40, odS);
-        } else if constexpr (OP == RowOp::BwdDQ) {
-          const uint32_t R = ta + kColDC + c0;
-          uint32_t rdP[16];
-          tmem_ld16(R, rdP);
-          tmem_ld_wait(rdP);
-          const float2 nDv = splat(-Dr);
-          uint32_t odS[8];
+        }
+      } else {
 #pragma unroll
-          for (int c = 0; c < 16; c += 2) {
-            float2 pr = probs2(pair(rS[h], c), sl2v, nL2v);
-            if (need_mask) {
-              if (c >= lim) pr.x = 0.f;
-              if (c + 1 >= lim) pr.y = 0.f;
+        for (int h = 0; h < 2; ++h) {
+          if (kDcHalves || h == 0) {
+            if (!mbar_wait(&m->bar_sa_dc[kDcHalves ? h : 0], st & 1, wctl)) {
+              ok = false;
+              break;
             }
-            const float2 ds = __fmul2_rn(pr, __fadd2_rn(pair(rdP, c), nDv));
-            odS[c / 2] = pack_bf16(ds.x, ds.y);
+            tc_fence_after();
           }
-          tmem_st8(R, odS);
-        } else {
-          if (st < ntiles) {  // sweep 1: running max and sum in the log2 domain
-            float x[16];
-            float mx = mrow;
-#pragma unroll
-            for (int c = 0; c < 16; ++c) {
-              x[c] = bits_f(rS[h][c]) * sl2;
-              if (need_mask && c >= lim) x[c] = -INFINITY;
-              mx = fmaxf(mx, x[c]);
-            }
-            if (mx != -INFINITY) {
-              float l = (mrow == -INFINITY) ? 0.f : lrow * ex2(mrow - mx);
-#pragma unroll
-              for (int c = 0; c < 16; ++c) l += ex2(x[c] - mx);
-              lrow = l;
-              mrow = mx;
-            }
-          } else {  // sweep 2: normalised probabilities into DC for O += P V
-            uint32_t oP[8];
+          const int c0 = HB * h + 16 * wg;  // tile column of this thread's 16
+          const int j0 = jt + c0;           // first key of this thread's 16
+          const bool need_mask = (!row_ok) || (j0 + 16 > N) || (p.causal && j0 + 15 > gi);
+          const int lim = need_mask ? (row_ok ? (p.causal ? min(N, gi + 1) : N) - j0 : 0) : 16;
+          if constexpr (kBob) {
+            const uint32_t R = ta + kColDC + 64 * h + 16 * wg;  // [dP_h | C_h] columns
+            uint32_t rdP[16], rC[16];
+            tmem_ld16(R + 0, rdP);
+            tmem_ld16(R + 32, rC);
+            tmem_ld_wait(rdP);
+            reg_dep(rC);
+            const float2 tauv = splat(tau), nDv = splat(-Dr);
+            uint32_t oP[8], oPF[8], oPPt[8], odS[8];
 #pragma unroll
             for (int c = 0; c < 16; c += 2) {
               float2 pr = probs2(pair(rS[h], c), sl2v, nL2v);
@@ -604,21 +630,117 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
                 if (c >= lim) pr.x = 0.f;
                 if (c + 1 >= lim) pr.y = 0.f;
               }
+              const float2 f = __fmul2_rn(pair(rF[h], c), tauv);
+              const float2 dp = pair(rdP, c);
+              const float2 t = __fadd2_rn(dp, nDv);
+              const float2 pt0 = __ffma2_rn(f, t, pair(rC, c));  // Ptil0 = C + F (dP - D)
+              const float2 pf = __fmul2_rn(pr, f);
+              const float2 ppt = __fmul2_rn(pr, pt0);
+              const float2 ds = __fmul2_rn(pr, t);
+              acc_a = __fadd2_rn(acc_a, pf);
+              acc_e = __fadd2_rn(acc_e, ppt);
               oP[c / 2] = pack_bf16(pr.x, pr.y);
+              oPF[c / 2] = pack_bf16(pf.x, pf.y);
+              oPPt[c / 2] = pack_bf16(ppt.x, ppt.y);
+              odS[c / 2] = pack_bf16(ds.x, ds.y);
             }
-            tmem_st8(ta + kColDC + c0, oP);
+            tmem_st8(R + 0, oP);
+            tmem_st8(R + 8, oPF);
+            tmem_st8(R + 32, oPPt);
+            tmem_st8(R + 40, odS);
+          } else if constexpr (kDirect) {
+            const uint32_t R = ta + kColDC + 64 * h + 16 * wg;  // [dP_h | C_h] columns
+            uint32_t rdP[16], rC[16];
+            tmem_ld16(R + 0, rdP);
+            tmem_ld16(R + 32, rC);
+            tmem_ld_wait(rdP);
+            reg_dep(rC);
+            const float2 tauv = splat(tau), nDv = splat(-Dr), nalv = splat(nal), nEv = splat(nE);
+            uint32_t oP[8], oPh[8], oSt[8], odS[8];
+#pragma unroll
+            for (int c = 0; c < 16; c += 2) {
+              float2 pr = probs2(pair(rS[h], c), sl2v, nL2v);
+              if (need_mask) {
+                if (c >= lim) pr.x = 0.f;
+                if (c + 1 >= lim) pr.y = 0.f;
+              }
+              const float2 f = __fmul2_rn(pair(rF[h], c), tauv);
+              const float2 dp = pair(rdP, c);
+              const float2 t = __fadd2_rn(dp, nDv);
+              // Ptil = C + F (dP - D) - alpha dP ; Stil = P (Ptil - E) ; h = F - alpha
+              const float2 pt = __ffma2_rn(nalv, dp, __ffma2_rn(f, t, pair(rC, c)));
+              const float2 ph = __fmul2_rn(pr, __fadd2_rn(f, nalv));
+              const float2 stl = __fmul2_rn(pr, __fadd2_rn(pt, nEv));
+              const float2 ds = __fmul2_rn(pr, t);
+              oP[c / 2] = pack_bf16(pr.x, pr.y);
+              oPh[c / 2] = pack_bf16(ph.x, ph.y);
+              oSt[c / 2] = pack_bf16(stl.x, stl.y);
+              odS[c / 2] = pack_bf16(ds.x, ds.y);
+            }
+            tmem_st8(R + 0, oP);
+            tmem_st8(R + 8, oPh);
+            tmem_st8(R + 32, oSt);
+            tmem_st8(R + 40, odS);
+          } else if constexpr (OP == RowOp::BwdDQ) {
+            const uint32_t R = ta + kColDC + c0;
+            uint32_t rdP[16];
+            tmem_ld16(R, rdP);
+            tmem_ld_wait(rdP);
+            const float2 nDv = splat(-Dr);
+            uint32_t odS[8];
+#pragma unroll
+            for (int c = 0; c < 16; c += 2) {
+              float2 pr = probs2(pair(rS[h], c), sl2v, nL2v);
+              if (need_mask) {
+                if (c >= lim) pr.x = 0.f;
+                if (c + 1 >= lim) pr.y = 0.f;
+              }
+              const float2 ds = __fmul2_rn(pr, __fadd2_rn(pair(rdP, c), nDv));
+              odS[c / 2] = pack_bf16(ds.x, ds.y);
+            }
+            tmem_st8(R, odS);
+          } else {
+            if (st < ntiles) {  // sweep 1: running max and sum in the log2 domain
+              float x[16];
+              float mx = mrow;
+#pragma unroll
+              for (int c = 0; c < 16; ++c) {
+                x[c] = bits_f(rS[h][c]) * sl2;
+                if (need_mask && c >= lim) x[c] = -INFINITY;
+                mx = fmaxf(mx, x[c]);
+              }
+              if (mx != -INFINITY) {
+                float l = (mrow == -INFINITY) ? 0.f : lrow * ex2(mrow - mx);
+#pragma unroll
+                for (int c = 0; c < 16; ++c) l += ex2(x[c] - mx);
+                lrow = l;
+                mrow = mx;
+              }
+            } else {  // sweep 2: normalised probabilities into DC for O += P V
+              uint32_t oP[8];
+#pragma unroll
+              for (int c = 0; c < 16; c += 2) {
+                float2 pr = probs2(pair(rS[h], c), sl2v, nL2v);
+                if (need_mask) {
+                  if (c >= lim) pr.x = 0.f;
+                  if (c + 1 >= lim) pr.y = 0.f;
+                }
+                oP[c / 2] = pack_bf16(pr.x, pr.y);
+              }
+              tmem_st8(ta + kColDC + c0, oP);
+            }
           }
+          tmem_st_wait();
+          tc_fence_before();
+          mbar_arrive(&m->bar_ew[h]);
         }
-        tmem_st_wait();
-        tc_fence_before();
-        mbar_arrive(&m->bar_ew[h]);
       }
     }
     // ---------------------------------------------------------- epilogue
     if (ok) ok = mbar_wait(&m->bar_acc, 0, wctl);
     if (ok && *abort_flag) ok = false;
     tc_fence_after();
-    if constexpr (OP == RowOp::BobPass1) {
+    if constexpr (kBob || kStats) {
       s_xchg[wg * BM + r] = acc_a.x + acc_a.y;
       s_xchg[(2 + wg) * BM + r] = acc_e.x + acc_e.y;
       named_bar_sync(1, kEwThreads);
@@ -628,7 +750,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         const float alpha = s_xchg[r] + s_xchg[BM + r];
         const float E0 = s_xchg[2 * BM + r] + s_xchg[3 * BM + r];
         const float E = E0 - alpha * Dr;  // eq. (8): E = E0 - alpha D
-        const int cbase = split * 64 + 32 * wg;
+        const int cbase = 32 * wg;
 #pragma unroll 1
         for (int q = 0; q < 2; ++q) {
           const int cc = 32 * wg + 16 * q;  // accumulator column (0..63)
@@ -656,11 +778,41 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
             store_row16(p.out1 + rowoff + cbase + 16 * q, dot);
           }
         }
-        if (row_ok && split == 0 && wg == 0) {
+        if (row_ok && wg == 0) {
           const size_t ri = (size_t)bh * N + gi;
           p.vec_out[ri] = alpha;
           p.vec_out[p.bhn + ri] = E;
           p.vec_out[2 * p.bhn + ri] = Dr;
+        }
+      } else if constexpr (kStats) {
+        if (row_ok && wg == 0) {
+          const float alpha = s_xchg[r] + s_xchg[BM + r];
+          const float E0 = s_xchg[2 * BM + r] + s_xchg[3 * BM + r];
+          const size_t ri = (size_t)bh * N + gi;
+          p.vec_out[ri] = alpha;
+          p.vec_out[p.bhn + ri] = E0 - alpha * Dr;  // E = E0 - alpha D
+          p.vec_out[2 * p.bhn + ri] = Dr;
+        }
+      } else if constexpr (kDirect) {
+        // Qtil = tau * acc[0, D), dOtil = acc[D, 2D); columns [wg*D/2, +D/2)
+#pragma unroll 1
+        for (int q = 0; q < D / 32; ++q) {
+          const int cc = wg * (D / 2) + 16 * q;
+          uint32_t rQ[16], rO[16];
+          tmem_ld16(ta + cc, rQ);
+          tmem_ld16(ta + D + cc, rO);
+          tmem_ld_wait(rQ);
+          reg_dep(rO);
+          if (row_ok) {
+            float qt[16], dot[16];
+#pragma unroll
+            for (int c = 0; c < 16; ++c) {
+              qt[c] = tau * bits_f(rQ[c]);
+              dot[c] = bits_f(rO[c]);
+            }
+            store_row16(p.out0 + rowoff + cc, qt);
+            store_row16(p.out1 + rowoff + cc, dot);
+          }
         }
       } else {
         // O (forward) or dQ = tau * acc (first backward), columns [wg*D/2, +D/2)

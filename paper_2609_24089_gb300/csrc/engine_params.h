@@ -25,7 +25,10 @@ constexpr uint32_t kColA = 256;  // stage-A region of half h starts at kColA + 1
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 
-enum class RowOp { Fwd, BwdDQ, BobPass1 };
+// BobPass1: Pass 1 in one sweep with the affine fusion of Prop. 3.1 (d = 64).
+// BobStats + BobPass1D: Pass 1 in two kernels (d = 128): the row scalars
+// alpha, E (and D) first, then Qtil and dOtil directly from eqs. (6)-(7).
+enum class RowOp { Fwd, BwdDQ, BobPass1, BobStats, BobPass1D };
 enum class ColOp { BwdDKDV, BobPass2 };
 
 // ---------------------------------------------------------------- parameters
@@ -50,16 +53,21 @@ struct EngineParams {
 };
 
 // ---------------------------------------------------------------- configs
+// BoB row kernels: stationary Q, U_Q, dO; streamed K, U_K, V, U_V
+constexpr bool row_bob(RowOp op) {
+  return op == RowOp::BobPass1 || op == RowOp::BobStats || op == RowOp::BobPass1D;
+}
+
 template <RowOp OP, int D>
 struct RowCfg {
   static constexpr int KB = D / 64;  // 64-wide boxes per row
   static constexpr int NSTAT = OP == RowOp::Fwd ? 1 : OP == RowOp::BwdDQ ? 2 : 3;
-  static constexpr int NSTREAM = OP == RowOp::BobPass1 ? 4 : 2;
-  static constexpr int DOUT = OP == RowOp::BobPass1 ? 64 : D;  // accumulator width per CTA
-  static constexpr int NSPLIT = D / DOUT;
+  static constexpr int NSTREAM = row_bob(OP) ? 4 : 2;
+  // the one-sweep Pass 1 holds four D-column accumulators: d = 64 only
+  static_assert(OP != RowOp::BobPass1 || D == 64, "one-sweep Pass 1 needs d = 64");
   static constexpr int STAT_BYTES = NSTAT * KB * BM * 128;
   static constexpr int STAGE_BYTES = NSTREAM * KB * BN * 128;
-  static constexpr int NSTAGES = OP == RowOp::BobPass1 ? (D == 64 ? 3 : 2) : 4;
+  static constexpr int NSTAGES = row_bob(OP) ? (D == 64 ? 3 : 2) : 4;
   // issuer X also issues the stage-B MMAs into B and dOtil0 (measured faster
   // at d = 64 only: at d = 128 the extra cross-issuer wait costs more)
   static constexpr bool XSHARE = OP == RowOp::BobPass1 && D == 64;

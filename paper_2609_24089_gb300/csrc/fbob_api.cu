@@ -18,8 +18,9 @@ namespace {
 constexpr int64_t kMaxN = int64_t(1) << 24;
 constexpr int64_t kMaxBH = int64_t(1) << 24;
 
-std::atomic<int> g_launches[5] = {{-1}, {-1}, {-1}, {-1}, {-1}};
-enum Entry { kEntFwd = 0, kEntBwd, kEntBob, kEntPass1, kEntPass2 };
+constexpr int kNumEntries = 7;
+std::atomic<int> g_launches[kNumEntries] = {{-1}, {-1}, {-1}, {-1}, {-1}, {-1}, {-1}};
+enum Entry { kEntFwd = 0, kEntBwd, kEntBob, kEntPass1, kEntPass2, kEntRowStats, kEntPass1D };
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   static std::once_flag once;
@@ -129,31 +130,66 @@ int n_blocks(int64_t N, int rows) { return (int)((N + rows - 1) / rows); }
 int launch_status(cudaError_t e) { return e == cudaSuccess ? FBOB_OK : FBOB_ERR_CUDA; }
 
 // ---- the individual launches (arguments already validated)
-int run_pass1(const fbob_shape* s, const void* q, const void* k, const void* v, const void* o,
-              const float* lse, const void* dout, const void* gq, const void* gk,
-              const void* gv, void* q_bar, void* dout_bar, float* row_stats,
-              cudaStream_t st) {
-  EngineParams p = base_params(s);
+
+// Tensor maps and pointers shared by the row-block BoB kernels: stationary
+// Q, U_Q, dO; streamed K, U_K (64-row tiles) and V, U_V (32-row chunks,
+// interleaved in the stream stage so that [V_h ; U_V_h] is one operand).
+bool row_bob_params(const fbob_shape* s, const void* q, const void* k, const void* v,
+                    const void* o, const float* lse, const void* dout, const void* gq,
+                    const void* gk, const void* gv, EngineParams* p) {
+  *p = base_params(s);
   const int64_t BH = s->B * s->H, N = s->N, d = s->d;
   const void* stat[3] = {q, gq, dout};
   const void* strm[4] = {k, gk, v, gv};
   for (int t = 0; t < 3; ++t)
-    if (!make_map(&p.tm[t], stat[t], BH, N, d, BM)) return FBOB_ERR_CUDA;
-  // K and U_K as 64-row tiles; V and U_V as 32-row chunks (interleaved in the
-  // stream stage so that [V_h ; U_V_h] is one operand)
+    if (!make_map(&p->tm[t], stat[t], BH, N, d, BM)) return false;
   for (int t = 0; t < 4; ++t)
-    if (!make_map(&p.tm[3 + t], strm[t], BH, N, d, t < 2 ? BN : HB)) return FBOB_ERR_CUDA;
-  p.o = static_cast<const __nv_bfloat16*>(o);
-  p.dout = static_cast<const __nv_bfloat16*>(dout);
-  p.lse = lse;
+    if (!make_map(&p->tm[3 + t], strm[t], BH, N, d, t < 2 ? BN : HB)) return false;
+  p->o = static_cast<const __nv_bfloat16*>(o);
+  p->dout = static_cast<const __nv_bfloat16*>(dout);
+  p->lse = lse;
+  p->nblk = n_blocks(N, BM);
+  choose_order(p, 1);
+  return true;
+}
+
+// Row scalars alpha, E, D (eq. 6) into row_stats.
+int run_row_stats(EngineParams p, int d, float* row_stats, cudaStream_t st) {
+  p.vec_out = row_stats;
+  return launch_status(launch_row(RowOp::BobStats, d, p, p.nblk * p.BH, st));
+}
+
+// Qtil, dOtil from eqs. (6)-(7) with the row scalars given in row_stats.
+int run_pass1_direct(EngineParams p, int d, const float* row_stats, void* q_bar,
+                     void* dout_bar, cudaStream_t st) {
+  p.vec_in = row_stats;
   p.out0 = static_cast<__nv_bfloat16*>(q_bar);
   p.out1 = static_cast<__nv_bfloat16*>(dout_bar);
-  p.vec_out = row_stats;
-  p.nblk = n_blocks(N, BM);
-  choose_order(&p, 1);
-  const int nb = p.nblk * p.BH * row_nsplit(RowOp::BobPass1, (int)d);
-  return launch_status(launch_row(RowOp::BobPass1, (int)d, p, nb, st));
+  return launch_status(launch_row(RowOp::BobPass1D, d, p, p.nblk * p.BH, st));
 }
+
+int run_pass1(const fbob_shape* s, const void* q, const void* k, const void* v, const void* o,
+              const float* lse, const void* dout, const void* gq, const void* gk,
+              const void* gv, void* q_bar, void* dout_bar, float* row_stats,
+              cudaStream_t st) {
+  EngineParams p;
+  if (!row_bob_params(s, q, k, v, o, lse, dout, gq, gk, gv, &p)) return FBOB_ERR_CUDA;
+  if (s->d == 64) {  // one sweep, affine fusion (Prop. 3.1)
+    p.out0 = static_cast<__nv_bfloat16*>(q_bar);
+    p.out1 = static_cast<__nv_bfloat16*>(dout_bar);
+    p.vec_out = row_stats;
+    return launch_status(launch_row(RowOp::BobPass1, (int)s->d, p, p.nblk * p.BH, st));
+  }
+  // d = 128: the four accumulators of the one-sweep form do not fit TMEM next
+  // to the stage-A tiles.  First the row scalars (alpha, E, D), then Qtil and
+  // dOtil from eqs. (6)-(7) with those scalars known (two accumulators).
+  const int rc = run_row_stats(p, (int)s->d, row_stats, st);
+  if (rc != FBOB_OK) return rc;
+  return run_pass1_direct(p, (int)s->d, row_stats, q_bar, dout_bar, st);
+}
+
+// kernels one pass-1 call enqueues
+int pass1_launches(int64_t d) { return d == 64 ? 1 : 2; }
 
 int run_pass2(const fbob_shape* s, const void* q, const void* k, const void* v, const float* lse,
               const void* dout, const void* gq, const void* gk, const void* gv,
@@ -196,8 +232,10 @@ const char* fbob_status_string(int status) {
 
 int fbob_launch_count(const char* entry) {
   if (!entry) return -1;
-  static const char* names[5] = {"fwd", "bwd", "bob", "bob_pass1", "bob_pass2"};
-  for (int t = 0; t < 5; ++t)
+  static const char* names[kNumEntries] = {"fwd",       "bwd",           "bob",
+                                          "bob_pass1", "bob_pass2",     "bob_row_stats",
+                                          "bob_pass1_direct"};
+  for (int t = 0; t < kNumEntries; ++t)
     if (std::strcmp(entry, names[t]) == 0) return g_launches[t].load();
   return -1;
 }
@@ -299,7 +337,7 @@ int fbob_attn_bob_pass1(const fbob_shape* s, const void* q, const void* k, const
   rc = check_ptrs(in, inb, 9, out, outb, 3);
   if (rc != FBOB_OK) return rc;
   rc = run_pass1(s, q, k, v, o, lse, dout, gq, gk, gv, q_bar, dout_bar, row_stats, stream);
-  if (rc == FBOB_OK) g_launches[kEntPass1] = 1;
+  if (rc == FBOB_OK) g_launches[kEntPass1] = pass1_launches(s->d);
   return rc;
 }
 
@@ -327,6 +365,57 @@ int fbob_attn_bob_pass2(const fbob_shape* s, const void* q, const void* k, const
   return rc;
 }
 
+int fbob_attn_bob_row_stats(const fbob_shape* s, const void* q, const void* k, const void* v,
+                            const void* o, const float* lse, const void* dout, const void* gq,
+                            const void* gk, const void* gv, float* row_stats,
+                            struct CUstream_st* stream) {
+  bool empty = false;
+  int rc = check_shape(s, &empty);
+  if (rc != FBOB_OK) return rc;
+  if (empty) {
+    g_launches[kEntRowStats] = 0;
+    return FBOB_OK;
+  }
+  const int64_t mat = s->B * s->H * s->N * s->d * 2, vec = s->B * s->H * s->N * 4;
+  const void* in[9] = {q, k, v, o, lse, dout, gq, gk, gv};
+  const int64_t inb[9] = {mat, mat, mat, mat, vec, mat, mat, mat, mat};
+  void* out[1] = {row_stats};
+  const int64_t outb[1] = {3 * vec};
+  rc = check_ptrs(in, inb, 9, out, outb, 1);
+  if (rc != FBOB_OK) return rc;
+  EngineParams p;
+  if (!row_bob_params(s, q, k, v, o, lse, dout, gq, gk, gv, &p)) return FBOB_ERR_CUDA;
+  rc = run_row_stats(p, (int)s->d, row_stats, stream);
+  if (rc == FBOB_OK) g_launches[kEntRowStats] = 1;
+  return rc;
+}
+
+int fbob_attn_bob_pass1_direct(const fbob_shape* s, const void* q, const void* k, const void* v,
+                               const float* lse, const void* dout, const void* gq,
+                               const void* gk, const void* gv, const float* row_stats,
+                               void* q_bar, void* dout_bar, struct CUstream_st* stream) {
+  bool empty = false;
+  int rc = check_shape(s, &empty);
+  if (rc != FBOB_OK) return rc;
+  if (empty) {
+    g_launches[kEntPass1D] = 0;
+    return FBOB_OK;
+  }
+  const int64_t mat = s->B * s->H * s->N * s->d * 2, vec = s->B * s->H * s->N * 4;
+  const void* in[9] = {q, k, v, lse, dout, gq, gk, gv, row_stats};
+  const int64_t inb[9] = {mat, mat, mat, vec, mat, mat, mat, mat, 3 * vec};
+  void* out[2] = {q_bar, dout_bar};
+  const int64_t outb[2] = {mat, mat};
+  rc = check_ptrs(in, inb, 9, out, outb, 2);
+  if (rc != FBOB_OK) return rc;
+  EngineParams p;
+  // (o is not read: D comes from row_stats)
+  if (!row_bob_params(s, q, k, v, nullptr, lse, dout, gq, gk, gv, &p)) return FBOB_ERR_CUDA;
+  rc = run_pass1_direct(p, (int)s->d, row_stats, q_bar, dout_bar, stream);
+  if (rc == FBOB_OK) g_launches[kEntPass1D] = 1;
+  return rc;
+}
+
 int fbob_attn_bob(const fbob_shape* s, const void* q, const void* k, const void* v, const void* o,
                   const float* lse, const void* dout, const void* gq, const void* gk,
                   const void* gv, void* q_bar, void* k_bar, void* v_bar, void* dout_bar,
@@ -351,7 +440,7 @@ int fbob_attn_bob(const fbob_shape* s, const void* q, const void* k, const void*
   // Pass 2 (column blocks): Ktil, Vtil from the saved row state.  Stream
   // order is the only synchronisation between the passes.
   rc = run_pass2(s, q, k, v, lse, dout, gq, gk, gv, row_stats, k_bar, v_bar, stream);
-  if (rc == FBOB_OK) g_launches[kEntBob] = 2;
+  if (rc == FBOB_OK) g_launches[kEntBob] = pass1_launches(s->d) + 1;
   return rc;
 }
 

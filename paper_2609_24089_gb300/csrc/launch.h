@@ -12,7 +12,6 @@ namespace fbob {
 // least 120 KB, so that one CTA (holding all 512 TMEM columns) runs per SM.
 inline int launch_smem(int plan_bytes) { return plan_bytes > 120 * 1024 ? plan_bytes : 120 * 1024; }
 
-int row_nsplit(RowOp op, int d);
 cudaError_t launch_row(RowOp op, int d, const EngineParams& p, int nblocks, cudaStream_t s);
 cudaError_t launch_col(ColOp op, int d, const EngineParams& p, int nblocks, cudaStream_t s);
 

@@ -1,6 +1,6 @@
 // row_kernels.cu -- instantiations and launcher of the row-block engine:
 // forward (eq. 1), first-backward dQ (eqs. 2-3), BoB Pass 1 (Algorithm 2,
-// first loop).
+// first loop): one sweep at d = 64, row statistics + direct form at d = 128.
 #include "attn_engine.cuh"
 #include "launch.h"
 
@@ -16,11 +16,6 @@ static cudaError_t launch_one(const EngineParams& p, int nblocks, cudaStream_t s
   return cudaGetLastError();
 }
 
-int row_nsplit(RowOp op, int d) {
-  if (op == RowOp::BobPass1) return d / 64;
-  return 1;
-}
-
 cudaError_t launch_row(RowOp op, int d, const EngineParams& p, int nblocks, cudaStream_t s) {
   switch (op) {
     case RowOp::Fwd:
@@ -29,9 +24,14 @@ cudaError_t launch_row(RowOp op, int d, const EngineParams& p, int nblocks, cuda
     case RowOp::BwdDQ:
       return d == 64 ? launch_one<RowOp::BwdDQ, 64>(p, nblocks, s)
                      : launch_one<RowOp::BwdDQ, 128>(p, nblocks, s);
-    case RowOp::BobPass1:
-      return d == 64 ? launch_one<RowOp::BobPass1, 64>(p, nblocks, s)
-                     : launch_one<RowOp::BobPass1, 128>(p, nblocks, s);
+    case RowOp::BobPass1:  // the one-sweep form serves d = 64 only
+      return d == 64 ? launch_one<RowOp::BobPass1, 64>(p, nblocks, s) : cudaErrorInvalidValue;
+    case RowOp::BobStats:
+      return d == 64 ? launch_one<RowOp::BobStats, 64>(p, nblocks, s)
+                     : launch_one<RowOp::BobStats, 128>(p, nblocks, s);
+    case RowOp::BobPass1D:
+      return d == 64 ? launch_one<RowOp::BobPass1D, 64>(p, nblocks, s)
+                     : launch_one<RowOp::BobPass1D, 128>(p, nblocks, s);
   }
   return cudaErrorInvalidValue;
 }

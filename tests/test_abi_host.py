@@ -17,8 +17,8 @@ def lib():
 def test_exports_every_declared_symbol(lib):
     names = fbob.header_symbols()
     assert {"fbob_attn_fwd", "fbob_attn_bwd", "fbob_attn_bob", "fbob_attn_bob_pass1",
-            "fbob_attn_bob_pass2", "fbob_device_status", "fbob_status_string",
-            "fbob_launch_count"} <= set(names)
+            "fbob_attn_bob_pass2", "fbob_attn_bob_row_stats", "fbob_attn_bob_pass1_direct",
+            "fbob_device_status", "fbob_status_string", "fbob_launch_count"} <= set(names)
     for n in names:
         assert getattr(lib, n) is not None
 
@@ -85,3 +85,29 @@ def test_rejects_null_misaligned_and_overlapping_pointers(lib):
     ps = ptrs(11)          # q k v lse dout gq gk gv row_stats k_bar v_bar
     ps[9] = ps[8]
     assert lib.fbob_attn_bob_pass2(ctypes.byref(S), *ps, None) == 1
+
+
+def test_row_stats_and_direct_validate_like_pass1(lib):
+    S = fbob.make_shape(1, 2, 100, 128, 0.088, 1)
+    rs = lib.fbob_attn_bob_row_stats      # q k v o lse dout gq gk gv row_stats
+    pd = lib.fbob_attn_bob_pass1_direct   # q k v lse dout gq gk gv row_stats q_bar dout_bar
+    for t in range(10):
+        ps = ptrs(10)
+        ps[t] = ctypes.c_void_p(0)
+        assert rs(ctypes.byref(S), *ps, None) == 1, t
+        assert rs(ctypes.byref(S), *ptrs(10, misalign=t), None) == 1, t
+    for t in range(11):
+        ps = ptrs(11)
+        ps[t] = ctypes.c_void_p(0)
+        assert pd(ctypes.byref(S), *ps, None) == 1, t
+    ps = ptrs(11)
+    ps[9] = ps[8]                       # q_bar aliases row_stats (an input here)
+    assert pd(ctypes.byref(S), *ps, None) == 1
+    bad = fbob.make_shape(1, 2, 100, 96, 0.1, 0)
+    assert rs(ctypes.byref(bad), *ptrs(10), None) == 2
+    assert pd(ctypes.byref(bad), *ptrs(11), None) == 2
+    empty = fbob.make_shape(1, 2, 0, 128, 0.088, 0)
+    assert rs(ctypes.byref(empty), *ptrs(10), None) == 0
+    assert lib.fbob_launch_count(b"bob_row_stats") == 0
+    assert pd(ctypes.byref(empty), *ptrs(11), None) == 0
+    assert lib.fbob_launch_count(b"bob_pass1_direct") == 0

@@ -113,6 +113,76 @@ def test_pass1_alone(shape):
     G.check("dobar", G.host(dout_bar), dob)
 
 
+@pytest.mark.parametrize("shape", [(1, 2, 300, 64, True), (2, 1, 200, 128, False),
+                                   (1, 1, 129, 128, True)], ids=ids)
+def test_row_stats_alone(shape):
+    """The row scalars of eq. (6) from the statistics kernel alone."""
+    B, H, N, d, causal = shape
+    bits = G.inputs(B, H, N, d, seed=5)
+    scale = 1 / np.sqrt(d)
+    X = [G.f64(bits[n]) for n in synth.NAMES]
+    _, _, _, _, al, E, D = oracle.bob(*X, scale, causal)
+    o_bits, L = G.oracle_o_l(bits, scale, causal)
+    t = G.torch()
+    q, k, v, do, gq, gk, gv = (G.dev(bits[n]) for n in synth.NAMES)
+    rs = t.empty((3, B, H, N), dtype=t.float32, device="cuda")
+    shp = fbob.make_shape(B, H, N, d, scale, causal)
+    fbob.fbob_attn_bob_row_stats(shp, q, k, v, G.dev(o_bits), G.dev_f32(L), do, gq, gk, gv, rs)
+    assert fbob.fbob_device_status() == 0
+    assert fbob.fbob_launch_count("bob_row_stats") == 1
+    rs = rs.cpu().numpy().astype(np.float64)
+    G.check("alpha", rs[0], al)
+    G.check("E", rs[1], E)
+    G.check("D", rs[2], D)
+
+
+@pytest.mark.parametrize("shape", [(1, 2, 300, 64, True), (2, 1, 200, 128, False),
+                                   (1, 1, 257, 128, True)], ids=ids)
+def test_pass1_direct_on_oracle_row_state(shape):
+    """Qtil, dOtil from eqs. (6)-(7) given the oracle's alpha, E, D and L."""
+    B, H, N, d, causal = shape
+    bits = G.inputs(B, H, N, d, seed=6)
+    scale = 1 / np.sqrt(d)
+    X = [G.f64(bits[n]) for n in synth.NAMES]
+    qb, _, _, dob, al, E, D = oracle.bob(*X, scale, causal)
+    _, L = oracle.fwd(*X[:3], scale, causal)
+    rs = np.stack([al, E, D]).astype(np.float32)
+    t = G.torch()
+    q, k, v, do, gq, gk, gv = (G.dev(bits[n]) for n in synth.NAMES)
+    q_bar, dout_bar = t.empty_like(q), t.empty_like(q)
+    shp = fbob.make_shape(B, H, N, d, scale, causal)
+    fbob.fbob_attn_bob_pass1_direct(shp, q, k, v, G.dev_f32(L), do, gq, gk, gv, G.dev_f32(rs),
+                                    q_bar, dout_bar)
+    assert fbob.fbob_device_status() == 0
+    assert fbob.fbob_launch_count("bob_pass1_direct") == 1
+    G.check("qbar", G.host(q_bar), qb)
+    G.check("dobar", G.host(dout_bar), dob)
+
+
+def test_one_sweep_and_two_kernel_pass1_agree_at_d64():
+    """At d = 64 both Pass-1 schedules exist; they compute the same outputs."""
+    B, H, N, d, causal = 1, 2, 333, 64, True
+    bits = G.inputs(B, H, N, d, seed=8)
+    scale = 1 / np.sqrt(d)
+    o_bits, L = G.oracle_o_l(bits, scale, causal)
+    t = G.torch()
+    q, k, v, do, gq, gk, gv = (G.dev(bits[n]) for n in synth.NAMES)
+    o, lse = G.dev(o_bits), G.dev_f32(L)
+    shp = fbob.make_shape(B, H, N, d, scale, causal)
+    qa, da = t.empty_like(q), t.empty_like(q)
+    ra = t.empty((3, B, H, N), dtype=t.float32, device="cuda")
+    fbob.fbob_attn_bob_pass1(shp, q, k, v, o, lse, do, gq, gk, gv, qa, da, ra)
+    assert fbob.fbob_launch_count("bob_pass1") == 1
+    qb, db = t.empty_like(q), t.empty_like(q)
+    rb = t.empty((3, B, H, N), dtype=t.float32, device="cuda")
+    fbob.fbob_attn_bob_row_stats(shp, q, k, v, o, lse, do, gq, gk, gv, rb)
+    fbob.fbob_attn_bob_pass1_direct(shp, q, k, v, lse, do, gq, gk, gv, rb, qb, db)
+    assert fbob.fbob_device_status() == 0
+    G.check("row_stats", G.host(rb), G.host(ra), rel=1e-4, mx=1e-3)
+    G.check("qbar", G.host(qb), G.host(qa))
+    G.check("dobar", G.host(db), G.host(da))
+
+
 def test_runs_are_bitwise_identical():
     bits = G.inputs(1, 4, 777, 128, seed=9)
     scale = 1 / np.sqrt(128)
