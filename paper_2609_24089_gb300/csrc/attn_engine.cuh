@@ -65,6 +65,10 @@ namespace fbob {
 constexpr uint32_t kColSF = 256;   // stage-A area of issuer X
 constexpr uint32_t kColDC = 384;   // stage-A area of issuer Y
 constexpr uint32_t kColDC1 = 128;  // second DC buffer (column engine, d = 64)
+// row statistics kernel: Q and U_Q as MMA A operands in TMEM (bf16 pairs per
+// column, D/2 columns each) at kColQT and kColQT + D/2; second SF buffer
+constexpr uint32_t kColQT = 0;
+constexpr uint32_t kColSF1 = 128;
 
 // Shared-memory bookkeeping block (in the MISC area).
 struct Misc {
@@ -72,8 +76,8 @@ struct Misc {
   uint64_t bar_full[4];    // first part of a stream stage landed (all issuer X reads)
   uint64_t bar_full_b[4];  // rest of the stage (and, column engine, the row vectors)
   uint64_t bar_empty[4];
-  uint64_t bar_sa_sf;   // X's stage A of a tile completed
-  uint64_t bar_sf_free; // elementwise warps copied SF to registers
+  uint64_t bar_sa_sf[2];   // X's stage A of a tile completed (per SF buffer)
+  uint64_t bar_sf_free[2]; // elementwise warps copied SF to registers (per SF buffer)
   uint64_t bar_dc_free; // elementwise warps copied DC to registers (row statistics kernel)
   uint64_t bar_sa_dc[2];
   uint64_t bar_ew[4];   // [DC buffer][half]; a single DC buffer uses [0..1]
@@ -202,14 +206,18 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
   if (tid == 0) {
     m->wctl.abort = 0;
     m->wctl.limit_ns = p.wait_limit_ns;
-    mbar_init(&m->bar_stat, 1);
+    // stationary tiles: one TMA transaction (plus, with C::STAT_TMEM, the
+    // elementwise threads' stores of Q and U_Q into TMEM)
+    mbar_init(&m->bar_stat, C::STAT_TMEM ? 1 + kEwThreads : 1);
     for (int s = 0; s < C::NSTAGES; ++s) {
       mbar_init(&m->bar_full[s], 1);
       mbar_init(&m->bar_full_b[s], 1);
       mbar_init(&m->bar_empty[s], 2);  // released by both MMA issuers
     }
-    mbar_init(&m->bar_sa_sf, 1);
-    mbar_init(&m->bar_sf_free, kEwThreads);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&m->bar_sa_sf[b], 1);
+      mbar_init(&m->bar_sf_free[b], kEwThreads);
+    }
     mbar_init(&m->bar_dc_free, kEwThreads);
     for (int h = 0; h < 2; ++h) {
       mbar_init(&m->bar_sa_dc[h], 1);
@@ -236,11 +244,12 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
     // loads at all, so every consumer wait runs into its bounded limit.
     if (elect_lane0() && !p.inject_stall) {
       for (int t = 0; t < C::NSTAT + C::NSTREAM; ++t) tma_prefetch_desc(&p.tm[t]);
+      // (with C::STAT_TMEM only dO, map 2, goes to shared memory)
       mbar_arrive_expect_tx(&m->bar_stat, C::STAT_BYTES);
-      for (int t = 0; t < C::NSTAT; ++t)
+      for (int t = C::STAT_TMEM ? 2 : 0; t < C::NSTAT; ++t)
         for (int b = 0; b < C::KB; ++b)
-          tma_load_3d(s_stat + (t * C::KB + b) * (BM * 128), &p.tm[t], &m->bar_stat, 64 * b, i0,
-                      bh);
+          tma_load_3d(s_stat + ((C::STAT_TMEM ? 0 : t) * C::KB + b) * (BM * 128), &p.tm[t],
+                      &m->bar_stat, 64 * b, i0, bh);
       int issued[4] = {-1, -1, -1, -1};
       for (int st = 0; st < nsteps; ++st) {
         const int stage = st % C::NSTAGES;
@@ -348,11 +357,18 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
       if (warp == kMmaWarp) {
         // ---------------- issuer X: SF(t) = scores (and F) of tile t, and
         // with C::XSHARE the stage-B MMAs into its accumulators B and dOtil0
-        auto stage_sf = [&](int st) {
+        auto stage_sf = [&](int st, uint32_t col) {
           const int stage = st % C::NSTAGES;
           const uint64_t kd0 = sdesc_sw128(smem_u32(s_stream + stage * C::STAGE_BYTES), 16, 1024);
-          const uint32_t R = tmem + kColSF;
-          if constexpr (kB4) {
+          const uint32_t R = tmem + col;
+          if constexpr (C::STAT_TMEM) {  // the same with Q and U_Q from TMEM
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k)  // [S | F] = Q [K ; U_K]^T
+              mma_ts(R + 0, tmem + kColQT + 8 * k, kd(kd0, 0, 0, k), id_n128, k > 0);
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k)  // F += U_Q K^T
+              mma_ts(R + 64, tmem + kColQT + D / 2 + 8 * k, kd(kd0, 0, 0, k), id_n64, 1);
+          } else if constexpr (kB4) {
             // stationary: 0 Q, 1 U_Q, 2 dO ; stream: 0 K, 1 U_K, 2 V, 3 U_V
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)  // [S | F] = Q [K ; U_K]^T
@@ -366,25 +382,39 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
               mma_ss(R + 0, sd(0, k), kd(kd0, 0, 0, k), id_n64, k > 0);
           }
         };
-        // (the statistics kernel has no stage B: a stage is released as soon
-        // as the MMAs reading it complete)
-        bool ok = mbar_wait(&m->bar_stat, 0, wctl) && mbar_wait(&m->bar_full[0], 0, wctl);
+        bool ok = mbar_wait(&m->bar_stat, 0, wctl);
+        if constexpr (kStats) {
+          // two SF buffers (tile t in buffer t & 1), so X runs up to a tile
+          // ahead of the elementwise warps; no stage B, so a stage is released
+          // as soon as the MMAs reading it complete
+          for (int st = 0; ok && st < nsteps; ++st) {
+            const int b = st & 1;
+            const int stage = st % C::NSTAGES;
+            if ((st >= 2 && !mbar_wait(&m->bar_sf_free[b], ((st - 2) >> 1) & 1, wctl)) ||
+                !mbar_wait(&m->bar_full[stage], (st / C::NSTAGES) & 1, wctl))
+              break;
+            tc_fence_after();
+            stage_sf(st, b ? kColSF1 : kColSF);
+            mma_commit(&m->bar_sa_sf[b]);
+            mma_commit(&m->bar_empty[stage]);
+          }
+          ok = false;
+        }
+        ok = ok && mbar_wait(&m->bar_full[0], 0, wctl);
         if (ok) {
           tc_fence_after();
-          stage_sf(0);
-          mma_commit(&m->bar_sa_sf);
-          if (kStats) mma_commit(&m->bar_empty[0]);
+          stage_sf(0, kColSF);
+          mma_commit(&m->bar_sa_sf[0]);
         }
         for (int st = 0; ok && st < nsteps; ++st) {
           const int stage = st % C::NSTAGES;
           if (st + 1 < nsteps) {  // SF(t+1) once the elementwise warps hold SF(t)
-            if (!mbar_wait(&m->bar_sf_free, st & 1, wctl) ||
+            if (!mbar_wait(&m->bar_sf_free[0], st & 1, wctl) ||
                 !mbar_wait(&m->bar_full[(st + 1) % C::NSTAGES], ((st + 1) / C::NSTAGES) & 1, wctl))
               break;
             tc_fence_after();
-            stage_sf(st + 1);
-            mma_commit(&m->bar_sa_sf);
-            if (kStats) mma_commit(&m->bar_empty[(st + 1) % C::NSTAGES]);
+            stage_sf(st + 1, kColSF);
+            mma_commit(&m->bar_sa_sf[0]);
           }
           if constexpr (C::XSHARE) {
             // V and U_V of this stage (already observed by issuer Y; the wait
@@ -403,7 +433,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
             }
             if (!ok) break;
           }
-          if (!kStats) mma_commit(&m->bar_empty[stage]);
+          mma_commit(&m->bar_empty[stage]);
         }
         mma_commit(&m->bar_acc);
         if (*abort_flag) drain_wait(&m->bar_acc, 0);
@@ -413,8 +443,8 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
           const uint64_t kd0 = sdesc_sw128(sb, 16, 1024);
           if constexpr (kStats) {  // whole tile: [dP_0|C_0|dP_1|C_1] = dO [V_0;U_V_0;V_1;U_V_1]^T
 #pragma unroll
-            for (int k = 0; k < D / 16; ++k)
-              mma_ss(tmem + kColDC, sd(2, k), kd(kd0, 2, 0, k), id_n128, k > 0);
+            for (int k = 0; k < D / 16; ++k)  // (dO is the one stationary tile in shared memory)
+              mma_ss(tmem + kColDC, sd(0, k), kd(kd0, 2, 0, k), id_n128, k > 0);
           } else if constexpr (kB4) {  // [dP_h | C_h] = dO [V_h ; U_V_h]^T
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)
@@ -521,11 +551,36 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         }
       }
     }
+    if constexpr (C::STAT_TMEM) {
+      // stationary rows straight into TMEM as MMA A operands (word c of a
+      // bf16 row = elements 2c, 2c+1 = column c of its operand): warpgroup 0
+      // writes Q, warpgroup 1 U_Q
+      auto put_row = [&](const __nv_bfloat16* row, uint32_t col, int c0, int ncols) {
+        const uint4* src = reinterpret_cast<const uint4*>(row);
+#pragma unroll 1
+        for (int c = c0; c < c0 + ncols; c += 8) {
+          uint4 a = make_uint4(0, 0, 0, 0), b = a;
+          if (row_ok) {
+            a = src[c / 4];
+            b = src[c / 4 + 1];
+          }
+          const uint32_t w[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+          tmem_st8(ta + col + c, w);
+        }
+      };
+      put_row((wg == 0 ? p.q : p.uq) + rowoff, kColQT + wg * (D / 2), 0, D / 2);
+      tmem_st_wait();
+      tc_fence_before();
+      mbar_arrive(&m->bar_stat);
+    }
     float mrow = -INFINITY, lrow = 0.f;             // forward sweep 1 (log2 domain)
     float2 acc_a = splat(0.f), acc_e = splat(0.f);  // Pass 1 partial row sums
     bool ok = true;
     for (int st = 0; ok && st < nsteps; ++st) {
-      if (!mbar_wait(&m->bar_sa_sf, st & 1, wctl)) {
+      // SF buffer of this tile (the statistics kernel alternates two)
+      const int sfb = kStats ? (st & 1) : 0;
+      const uint32_t sfcol = sfb ? kColSF1 : kColSF;
+      if (!mbar_wait(&m->bar_sa_sf[sfb], kStats ? ((st >> 1) & 1) : (st & 1), wctl)) {
         ok = false;
         break;
       }
@@ -547,8 +602,8 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
       uint32_t rS[2][16], rF[2][16];
 #pragma unroll
       for (int h = 0; h < 2; ++h) {
-        tmem_ld16(ta + kColSF + HB * h + 16 * wg, rS[h]);
-        if constexpr (kB4) tmem_ld16(ta + kColSF + 64 + HB * h + 16 * wg, rF[h]);
+        tmem_ld16(ta + sfcol + HB * h + 16 * wg, rS[h]);
+        if constexpr (kB4) tmem_ld16(ta + sfcol + 64 + HB * h + 16 * wg, rF[h]);
       }
       tmem_ld_wait(rS[0]);
       reg_dep(rS[1]);
@@ -557,7 +612,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         reg_dep(rF[1]);
       }
       tc_fence_before();
-      mbar_arrive(&m->bar_sf_free);
+      mbar_arrive(&m->bar_sf_free[sfb]);
       const int jt = (st % ntiles) * BN;
       const float2 sl2v = splat(sl2), nL2v = splat(-L2);
       if constexpr (kStats) {
@@ -886,8 +941,10 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
       mbar_init(&m->bar_full_b[s], 1 + 32);  // dO + 32 producer lanes' row vectors
       mbar_init(&m->bar_empty[s], 2);        // released by both MMA issuers
     }
-    mbar_init(&m->bar_sa_sf, 1);
-    mbar_init(&m->bar_sf_free, kEwThreads);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&m->bar_sa_sf[b], 1);
+      mbar_init(&m->bar_sf_free[b], kEwThreads);
+    }
     for (int h = 0; h < 2; ++h) {
       mbar_init(&m->bar_sa_dc[h], 1);
       mbar_init(&m->bar_xb[h], 1);
@@ -1035,17 +1092,17 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
         if (ok) {
           tc_fence_after();
           stage_sf(0);
-          mma_commit(&m->bar_sa_sf);
+          mma_commit(&m->bar_sa_sf[0]);
         }
         for (int st = 0; ok && st < nsteps; ++st) {
           const int stage = st % C::NSTAGES;
           if (st + 1 < nsteps) {  // SF(t+1) once the elementwise warps hold SF(t)
-            if (!mbar_wait(&m->bar_sf_free, st & 1, wctl) ||
+            if (!mbar_wait(&m->bar_sf_free[0], st & 1, wctl) ||
                 !mbar_wait(&m->bar_full[(st + 1) % C::NSTAGES], ((st + 1) / C::NSTAGES) & 1, wctl))
               break;
             tc_fence_after();
             stage_sf(st + 1);
-            mma_commit(&m->bar_sa_sf);
+            mma_commit(&m->bar_sa_sf[0]);
           }
           if constexpr (C::XSHARE) {
             // dO of this stage (already observed by issuer Y; explicit acquire)
@@ -1146,7 +1203,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
       const int stage = st % C::NSTAGES;
       // the row vectors were written by the producer: acquire them explicitly
       if (!mbar_wait(&m->bar_full_b[stage], (st / C::NSTAGES) & 1, wctl) ||
-          !mbar_wait(&m->bar_sa_sf, st & 1, wctl)) {
+          !mbar_wait(&m->bar_sa_sf[0], st & 1, wctl)) {
         ok = false;
         break;
       }
@@ -1167,7 +1224,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
         reg_dep(rF[1]);
       }
       tc_fence_before();
-      mbar_arrive(&m->bar_sf_free);
+      mbar_arrive(&m->bar_sf_free[0]);
       if (!mbar_wait(&m->bar_sa_dc[dc_sel(st)], dc_par(st), wctl)) {
         ok = false;
         break;

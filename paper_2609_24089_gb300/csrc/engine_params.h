@@ -34,6 +34,8 @@ enum class ColOp { BwdDKDV, BobPass2 };
 // ---------------------------------------------------------------- parameters
 struct EngineParams {
   CUtensorMap tm[7];  // stationary maps first (box rows BM), then streamed (box rows BN)
+  const __nv_bfloat16* q;     // Q and U_Q (row statistics kernel: stationary A operands)
+  const __nv_bfloat16* uq;
   const __nv_bfloat16* o;     // forward output O (row engine: D and dOtil)
   const __nv_bfloat16* dout;  // dO (row engine: D = do.o)
   const float* lse;           // natural-log L [BH, N]
@@ -65,9 +67,13 @@ struct RowCfg {
   static constexpr int NSTREAM = row_bob(OP) ? 4 : 2;
   // the one-sweep Pass 1 holds four D-column accumulators: d = 64 only
   static_assert(OP != RowOp::BobPass1 || D == 64, "one-sweep Pass 1 needs d = 64");
-  static constexpr int STAT_BYTES = NSTAT * KB * BM * 128;
+  // the row statistics kernel has no accumulators: Q and U_Q live in TMEM as
+  // MMA A operands next to two SF buffers; only dO stays in shared memory,
+  // which leaves room for another stream stage
+  static constexpr bool STAT_TMEM = OP == RowOp::BobStats;
+  static constexpr int STAT_BYTES = (STAT_TMEM ? 1 : NSTAT) * KB * BM * 128;
   static constexpr int STAGE_BYTES = NSTREAM * KB * BN * 128;
-  static constexpr int NSTAGES = row_bob(OP) ? (D == 64 ? 3 : 2) : 4;
+  static constexpr int NSTAGES = STAT_TMEM ? (D == 64 ? 4 : 3) : row_bob(OP) ? (D == 64 ? 3 : 2) : 4;
   // issuer X also issues the stage-B MMAs into B and dOtil0 (measured faster
   // at d = 64 only: at d = 128 the extra cross-issuer wait costs more)
   static constexpr bool XSHARE = OP == RowOp::BobPass1 && D == 64;

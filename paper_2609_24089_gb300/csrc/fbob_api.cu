@@ -145,6 +145,8 @@ bool row_bob_params(const fbob_shape* s, const void* q, const void* k, const voi
     if (!make_map(&p->tm[t], stat[t], BH, N, d, BM)) return false;
   for (int t = 0; t < 4; ++t)
     if (!make_map(&p->tm[3 + t], strm[t], BH, N, d, t < 2 ? BN : HB)) return false;
+  p->q = static_cast<const __nv_bfloat16*>(q);
+  p->uq = static_cast<const __nv_bfloat16*>(gq);
   p->o = static_cast<const __nv_bfloat16*>(o);
   p->dout = static_cast<const __nv_bfloat16*>(dout);
   p->lse = lse;
