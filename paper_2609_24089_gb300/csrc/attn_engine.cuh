@@ -305,9 +305,9 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
       };
       // stage B of half h: K-steps s = 2h + sub, 16 streamed rows each; the
       // operand tiles of K-step s sit at DC columns written by warpgroup sub.
-      // With C::XSHARE issuer X takes the MMAs into B and dOtil0 (part 0) and
-      // issuer Y those into G and Omega (part 1); otherwise Y takes them all
-      // (part 2).
+      // With C::XSHARE issuer X takes the MMAs into B and dOtil0 (one sweep)
+      // or dOtil (direct form) (part 0) and issuer Y the rest (part 1);
+      // otherwise Y takes them all (part 2).
       auto stage_b = [&](uint32_t sb, int h, int st, int part) {
         if (st < first_b) return;
         constexpr uint32_t kBoxBytes = C::NSTREAM * BN * 128;
@@ -341,12 +341,17 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
               mma_ts(tmem + 192, A + 32, md(0, 0), id_b, 1);
             }
           } else if constexpr (kDirect) {
-            // eqs. (6)-(7): Qtil += Stil K + dS U_K ; dOtil += P U_V + (P o h) V
+            // eqs. (6)-(7): Qtil += Stil K + dS U_K (part 1) ; dOtil += P U_V +
+            // (P o h) V (part 0, issuer X's share with XSHARE)
             const uint32_t A = tmem + kColDC + 64 * h + 16 * sub;
-            mma_ts(tmem + 0, A + 32, md(0, 0), id_b, first);
-            mma_ts(tmem + 0, A + 40, md(1, 0), id_b, 1);
-            mma_ts(tmem + D, A + 0, md(3, 0), id_b, first);
-            mma_ts(tmem + D, A + 8, md(2, 0), id_b, 1);
+            if (part != 0) {
+              mma_ts(tmem + 0, A + 32, md(0, 0), id_b, first);
+              mma_ts(tmem + 0, A + 40, md(1, 0), id_b, 1);
+            }
+            if (part != 1) {
+              mma_ts(tmem + D, A + 0, md(3, 0), id_b, first);
+              mma_ts(tmem + D, A + 8, md(2, 0), id_b, 1);
+            }
           } else if constexpr (OP == RowOp::BwdDQ) {
             mma_ts(tmem + 0, tmem + kColDC + 16 * s, md(0, 0), id_b, first);  // dQ += dS K
           } else {
@@ -356,8 +361,9 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
       };
       if (warp == kMmaWarp) {
         // ---------------- issuer X: SF(t) = scores (and F) of tile t, and
-        // with C::XSHARE the stage-B MMAs into its accumulators B and dOtil0
-        auto stage_sf = [&](int st, uint32_t col) {
+        // with C::XSHARE its share of stage B
+        // part 1: [S | F] (and S alone); part 2: F += U_Q K^T; 0: both
+        auto stage_sf = [&](int st, uint32_t col, int part = 0) {
           const int stage = st % C::NSTAGES;
           const uint64_t kd0 = sdesc_sw128(smem_u32(s_stream + stage * C::STAGE_BYTES), 16, 1024);
           const uint32_t R = tmem + col;
@@ -370,12 +376,16 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
               mma_ts(R + 64, tmem + kColQT + D / 2 + 8 * k, kd(kd0, 0, 0, k), id_n64, 1);
           } else if constexpr (kB4) {
             // stationary: 0 Q, 1 U_Q, 2 dO ; stream: 0 K, 1 U_K, 2 V, 3 U_V
+            if (part != 2) {
 #pragma unroll
-            for (int k = 0; k < D / 16; ++k)  // [S | F] = Q [K ; U_K]^T
-              mma_ss(R + 0, sd(0, k), kd(kd0, 0, 0, k), id_n128, k > 0);
+              for (int k = 0; k < D / 16; ++k)  // [S | F] = Q [K ; U_K]^T
+                mma_ss(R + 0, sd(0, k), kd(kd0, 0, 0, k), id_n128, k > 0);
+            }
+            if (part != 1) {
 #pragma unroll
-            for (int k = 0; k < D / 16; ++k)  // F += U_Q K^T
-              mma_ss(R + 64, sd(1, k), kd(kd0, 0, 0, k), id_n64, 1);
+              for (int k = 0; k < D / 16; ++k)  // F += U_Q K^T
+                mma_ss(R + 64, sd(1, k), kd(kd0, 0, 0, k), id_n64, 1);
+            }
           } else {
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)  // S = Q K^T
@@ -408,13 +418,17 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         }
         for (int st = 0; ok && st < nsteps; ++st) {
           const int stage = st % C::NSTAGES;
-          if (st + 1 < nsteps) {  // SF(t+1) once the elementwise warps hold SF(t)
+          const bool more = st + 1 < nsteps;
+          if (more) {  // SF(t+1) once the elementwise warps hold SF(t)
             if (!mbar_wait(&m->bar_sf_free[0], st & 1, wctl) ||
                 !mbar_wait(&m->bar_full[(st + 1) % C::NSTAGES], ((st + 1) / C::NSTAGES) & 1, wctl))
               break;
             tc_fence_after();
-            stage_sf(st + 1, kColSF);
-            mma_commit(&m->bar_sa_sf[0]);
+            // with XSHARE only [S | F] now: X's stage-B share of half 0 goes
+            // between the two parts, so that issuer Y's next DC (which waits
+            // for that share) does not queue behind all of SF(t+1)
+            stage_sf(st + 1, kColSF, C::XSHARE ? 1 : 0);
+            if (!C::XSHARE) mma_commit(&m->bar_sa_sf[0]);
           }
           if constexpr (C::XSHARE) {
             // V and U_V of this stage (already observed by issuer Y; the wait
@@ -430,6 +444,10 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
               tc_fence_after();
               stage_b(sb, h, st, 0);
               mma_commit(&m->bar_xb[h]);
+              if (h == 0 && more) {
+                stage_sf(st + 1, kColSF, 2);
+                mma_commit(&m->bar_sa_sf[0]);
+              }
             }
             if (!ok) break;
           }

@@ -74,8 +74,10 @@ struct RowCfg {
   static constexpr int STAT_BYTES = (STAT_TMEM ? 1 : NSTAT) * KB * BM * 128;
   static constexpr int STAGE_BYTES = NSTREAM * KB * BN * 128;
   static constexpr int NSTAGES = STAT_TMEM ? (D == 64 ? 4 : 3) : row_bob(OP) ? (D == 64 ? 3 : 2) : 4;
-  // issuer X also issues the stage-B MMAs into B and dOtil0 (measured faster
-  // at d = 64 only: at d = 128 the extra cross-issuer wait costs more)
+  // issuer X also issues the stage-B MMAs into B and dOtil0, between the two
+  // parts of SF(t+1).  Measured faster for the one-sweep Pass 1 (d = 64); for
+  // the direct form at d = 128 (dOtil on X) Y's wait for X's share before
+  // each DC cost 5 % more than it saved.
   static constexpr bool XSHARE = OP == RowOp::BobPass1 && D == 64;
   static constexpr int MISC_BYTES = 2304;
   static constexpr int SMEM_BYTES = STAT_BYTES + NSTAGES * STAGE_BYTES + MISC_BYTES;
