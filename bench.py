@@ -373,6 +373,58 @@ def run_gpu(args, w):
         dist.destroy_process_group()
 
 
+def run_gpu_op(args, w):
+    """Forward (eq. 1) or first backward (eqs. 2-3) alone, for their own
+    tuning: K timed calls after W warm-up calls, CUDA events on the stream.
+    FLOPs: 2 contractions (Q K^T, P V) for the forward, 5 (S, dP, dV, dQ, dK)
+    for the backward, times 2*B*H*N^2*d*rho."""
+    import torch
+
+    import paper_2609_24089_gb300 as fbob
+
+    torch.cuda.set_device(0)
+    fbob.build()
+    fbob.load()
+    bits = synth.workload_inputs(w)
+    dev = {n: torch.from_numpy(bits[n].view(np.int16)).view(torch.bfloat16).cuda()
+           for n in ("q", "k", "v", "dout")}
+    q, k, v, do = dev["q"], dev["k"], dev["v"], dev["dout"]
+    shp = fbob.make_shape(w.B, w.H, w.N, w.d, w.scale, w.causal)
+    o, lse = fbob.attn_fwd(q, k, v, w.scale, w.causal)
+    dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
+    dstat = torch.empty_like(lse)
+    if args.op == "fwd":
+        call, contractions, entry = (lambda: fbob.fbob_attn_fwd(shp, q, k, v, o, lse)), 2, "fwd"
+    else:
+        call, contractions, entry = (lambda: fbob.fbob_attn_bwd(
+            shp, q, k, v, o, lse, do, dq, dk, dv, dstat)), 5, "bwd"
+    for _ in range(args.warmup):
+        call()
+    torch.cuda.synchronize()
+    stream = torch.cuda.current_stream()
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(0) as clk:
+        start.record(stream)
+        for _ in range(args.steps):
+            call()
+        stop.record(stream)
+        torch.cuda.synchronize()
+    if fbob.fbob_device_status() != 0:
+        raise RuntimeError("device status not OK")
+    ms = start.elapsed_time(stop) / args.steps
+    value = bob_flops(w, contractions) / (ms * 1e-3) / 1e12
+    peak = measured_peaks()["bf16_sustained"]
+    print(json.dumps({
+        "metric": f"attention {args.op} TFLOP/s ({contractions} contractions x 2*B*H*N^2*d*rho)",
+        "value": value, "unit": "TFLOP/s", "n_gpus": 1, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "dtype": "bf16",
+        "data": "synthetic", "frac_of_bf16_peak": value / peak,
+        "gpu_launches": fbob.fbob_launch_count(entry) * args.steps,
+        "config": {"workload": w.name, "B": w.B, "H": w.H, "N": w.N, "d": w.d,
+                   "causal": w.causal},
+        "clocks": clk.summary()}), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -383,6 +435,8 @@ def main():
     ap.add_argument("--cpu-s", type=float, default=15.0, help="target seconds of the CPU baseline")
     ap.add_argument("--ref-step-s", type=float, default=5.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--op", default="bob", choices=["bob", "fwd", "bwd"],
+                    help="bob (the benchmark); fwd / bwd time the boundary's other calls alone")
     ap.add_argument("--bh", default=None,
                     help="B,H override (smaller profiling captures of the same kernels)")
     args = ap.parse_args()
@@ -394,6 +448,8 @@ def main():
         w = dataclasses.replace(w, B=B, H=H, name=f"{w.name}_B{B}H{H}")
     if args.impl == "reference":
         run_reference(args, w)
+    elif args.op != "bob":
+        run_gpu_op(args, w)
     else:
         run_gpu(args, w)
 
