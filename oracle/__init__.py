@@ -48,9 +48,9 @@ def _load(mutant: int = 0, out_dir: str | None = None):
     lib = ctypes.CDLL(build(mutant, out_dir))
     i64, dbl, cint = ctypes.c_int64, ctypes.c_double, ctypes.c_int
     p = ctypes.c_void_p
-    lib.fbob_oracle_fwd.argtypes = [i64, i64, dbl, cint, p, p, p, p, p, cint]
-    lib.fbob_oracle_bwd.argtypes = [i64, i64, dbl, cint, p, p, p, p, p, p, p, p, cint]
-    lib.fbob_oracle_bob.argtypes = [i64, i64, dbl, cint, p, p, p, p, p, p, p,
+    lib.fbob_oracle_fwd.argtypes = [i64, i64, dbl, cint, i64, i64, p, p, p, p, p, cint]
+    lib.fbob_oracle_bwd.argtypes = [i64, i64, dbl, cint, i64, i64, p, p, p, p, p, p, p, p, cint]
+    lib.fbob_oracle_bob.argtypes = [i64, i64, dbl, cint, i64, i64, p, p, p, p, p, p, p,
                                     p, i64, i64, i64, p, p, p, p, p, p, p, p, cint]
     for f in (lib.fbob_oracle_fwd, lib.fbob_oracle_bwd, lib.fbob_oracle_bob):
         f.restype = cint
@@ -66,6 +66,14 @@ def _ptr(x):
     return None if x is None else x.ctypes.data_as(ctypes.c_void_p)
 
 
+def _window(window):
+    """(wl, wr) of the sliding-window band i - wl <= j <= i + wr; -1 = unbounded."""
+    if window is None:
+        return -1, -1
+    wl, wr = (int(w) for w in window)
+    return wl, wr
+
+
 def _heads(x):
     x = np.asarray(x)
     if x.ndim == 2:
@@ -73,8 +81,10 @@ def _heads(x):
     return x
 
 
-def fwd(q, k, v, scale, causal, nthreads=0):
-    """Forward attention (eq. 1).  Returns O [B,H,N,d] and natural-log L [B,H,N]."""
+def fwd(q, k, v, scale, causal, nthreads=0, window=None):
+    """Forward attention (eq. 1).  Returns O [B,H,N,d] and natural-log L [B,H,N].
+    window: (wl, wr) sliding-window band (default: none)."""
+    wl, wr = _window(window)
     q, k, v = (_c(_heads(t)) for t in (q, k, v))
     B, H, N, d = q.shape
     lib = _load()
@@ -83,7 +93,7 @@ def fwd(q, k, v, scale, causal, nthreads=0):
     for b in range(B):
         for h in range(H):
             o_ = np.zeros((N, d)); l_ = np.zeros(N)
-            rc = lib.fbob_oracle_fwd(N, d, float(scale), int(bool(causal)),
+            rc = lib.fbob_oracle_fwd(N, d, float(scale), int(bool(causal)), wl, wr,
                                      _ptr(_c(q[b, h])), _ptr(_c(k[b, h])), _ptr(_c(v[b, h])),
                                      _ptr(o_), _ptr(l_), int(nthreads))
             assert rc == 0, rc
@@ -91,8 +101,9 @@ def fwd(q, k, v, scale, causal, nthreads=0):
     return O, L
 
 
-def bwd(q, k, v, dout, scale, causal, nthreads=0):
+def bwd(q, k, v, dout, scale, causal, nthreads=0, window=None):
     """First backward (eqs. 2-3).  Returns dQ, dK, dV [B,H,N,d] and D [B,H,N]."""
+    wl, wr = _window(window)
     q, k, v, dout = (_c(_heads(t)) for t in (q, k, v, dout))
     B, H, N, d = q.shape
     lib = _load()
@@ -101,7 +112,7 @@ def bwd(q, k, v, dout, scale, causal, nthreads=0):
     for b in range(B):
         for h in range(H):
             dq, dk, dv, dd = np.zeros((N, d)), np.zeros((N, d)), np.zeros((N, d)), np.zeros(N)
-            rc = lib.fbob_oracle_bwd(N, d, float(scale), int(bool(causal)),
+            rc = lib.fbob_oracle_bwd(N, d, float(scale), int(bool(causal)), wl, wr,
                                      _ptr(_c(q[b, h])), _ptr(_c(k[b, h])), _ptr(_c(v[b, h])),
                                      _ptr(_c(dout[b, h])), _ptr(dq), _ptr(dk), _ptr(dv),
                                      _ptr(dd), int(nthreads))
@@ -111,7 +122,7 @@ def bwd(q, k, v, dout, scale, causal, nthreads=0):
 
 
 def bob_head(q, k, v, dout, gq, gk, gv, scale, causal, rows=None, cols=None,
-             nthreads=0, mutant=0, mutant_dir=None):
+             nthreads=0, mutant=0, mutant_dir=None, window=None):
     """Backward-over-backward of one head ([N, d] float64 arrays).
 
     rows: query rows whose row-owned outputs are wanted (default: all).
@@ -119,7 +130,9 @@ def bob_head(q, k, v, dout, gq, gk, gv, scale, causal, rows=None, cols=None,
           Ktil, Vtil (default: all columns when rows is all rows, else none).
     Returns a dict with qbar, dobar, alpha, E, D, L (indexed like rows) and
     kbar, vbar ((c1-c0) x d; complete only if every contributing row is listed).
+    window: (wl, wr) sliding-window band i - wl <= j <= i + wr (-1 = unbounded).
     """
+    wl, wr = _window(window)
     q, k, v, dout, gq, gk, gv = (_c(t) for t in (q, k, v, dout, gq, gk, gv))
     N, d = q.shape
     if rows is None:
@@ -138,7 +151,7 @@ def bob_head(q, k, v, dout, gq, gk, gv, scale, causal, rows=None, cols=None,
         "kbar": np.zeros((nc, d)), "vbar": np.zeros((nc, d)),
     }
     lib = _load(mutant, mutant_dir)
-    rc = lib.fbob_oracle_bob(N, d, float(scale), int(bool(causal)),
+    rc = lib.fbob_oracle_bob(N, d, float(scale), int(bool(causal)), wl, wr,
                              _ptr(q), _ptr(k), _ptr(v), _ptr(dout), _ptr(gq), _ptr(gk), _ptr(gv),
                              _ptr(rows), nr, c0, c1,
                              _ptr(res["qbar"]), _ptr(res["dobar"]), _ptr(res["alpha"]),
@@ -148,7 +161,8 @@ def bob_head(q, k, v, dout, gq, gk, gv, scale, causal, rows=None, cols=None,
     return res
 
 
-def bob(q, k, v, dout, gq, gk, gv, scale, causal, nthreads=0, mutant=0, mutant_dir=None):
+def bob(q, k, v, dout, gq, gk, gv, scale, causal, nthreads=0, mutant=0, mutant_dir=None,
+        window=None):
     """Full backward-over-backward on [B,H,N,d] (or [N,d]) float64 arrays.
 
     Returns (qbar, kbar, vbar, dobar, alpha, E, D) with the input's batch shape.
@@ -161,7 +175,7 @@ def bob(q, k, v, dout, gq, gk, gv, scale, causal, nthreads=0, mutant=0, mutant_d
     for b in range(B):
         for h in range(H):
             r = bob_head(*(t[b, h] for t in ts), scale, causal, nthreads=nthreads,
-                         mutant=mutant, mutant_dir=mutant_dir)
+                         mutant=mutant, mutant_dir=mutant_dir, window=window)
             for n in ("qbar", "kbar", "vbar", "dobar", "alpha", "E", "D"):
                 out[n][b, h] = r[n]
     return (out["qbar"], out["kbar"], out["vbar"], out["dobar"],

@@ -30,9 +30,13 @@
  * scores of that row), alpha and E are formed as plain row sums before they are
  * used, and every output is the plain sum its defining equation states.
  *
- * Masking (Sec. 2): the valid column set of row i is V_i = {j < N} without a
- * mask and {j <= i} with the causal mask (square, top-left aligned, diagonal
- * included).  Entries outside V_i have P = 0 and contribute nothing.
+ * Masking (Sec. 2; sliding window, App. "Sliding-window attention"): the valid
+ * column set of row i is the band V_i = {j : lo_i <= j < hi_i} with
+ *   lo_i = max(0, i - wl)                    (wl < 0: lo_i = 0),
+ *   hi_i = min(N, i + wr + 1)                (wr < 0: hi_i = N),
+ * and the causal mask (square, top-left aligned, diagonal included) caps
+ * hi_i at i + 1.  wl = wr = -1 is the plain mask.  Every row keeps its
+ * diagonal.  Entries outside V_i have P = 0 and contribute nothing.
  *
  * Threads: rows are independent, so OpenMP splits rows across threads.  The
  * column-owned sums (Ktil, Vtil, dV, dK) are accumulated into one private
@@ -59,8 +63,15 @@ static double dot(const double* a, const double* b, int64_t d) {
     return s;
 }
 
-static int64_t valid_cols(int64_t i, int64_t N, int causal) {
-    return causal ? (i + 1 < N ? i + 1 : N) : N;
+/* the valid band [lo_i, hi_i) of row i (see the header comment) */
+typedef struct { int causal; int64_t wl, wr; } band_t;
+
+static void valid_cols(int64_t i, int64_t N, band_t m, int64_t* lo, int64_t* hi) {
+    int64_t a = m.wl < 0 ? 0 : i - m.wl;
+    int64_t b = m.wr < 0 ? N : i + m.wr + 1;
+    if (m.causal && b > i + 1) b = i + 1;
+    *lo = a < 0 ? 0 : a;
+    *hi = b > N ? N : b;
 }
 
 static int pick_threads(int nthreads) {
@@ -80,30 +91,34 @@ static int thread_id(void) {
 #endif
 }
 
-/* Row i of S and P (eq. 1): S_ij = tau q_i.k_j for j in V_i, L_i the
- * natural-log normaliser, P_ij = exp(S_ij - L_i).  Returns |V_i|. */
-static int64_t softmax_row(int64_t i, int64_t N, int64_t d, double tau, int causal,
-                           const double* Q, const double* K, double* S, double* P,
-                           double* L_out) {
-    const int64_t nv = valid_cols(i, N, causal);
+/* Row i of S and P (eq. 1): S_ij = tau q_i.k_j for j in V_i = [lo, hi), L_i
+ * the natural-log normaliser, P_ij = exp(S_ij - L_i).  S and P are indexed by
+ * the absolute column j. */
+static void softmax_row(int64_t i, int64_t N, int64_t d, double tau, band_t mk,
+                        const double* Q, const double* K, double* S, double* P,
+                        double* L_out, int64_t* lo_out, int64_t* hi_out) {
+    int64_t lo, hi;
+    valid_cols(i, N, mk, &lo, &hi);
     double m = -INFINITY;
-    for (int64_t j = 0; j < nv; ++j) {
+    for (int64_t j = lo; j < hi; ++j) {
         S[j] = tau * dot(Q + i * d, K + j * d, d);
         if (S[j] > m) m = S[j];
     }
     double z = 0.0;
-    for (int64_t j = 0; j < nv; ++j) z += exp(S[j] - m);
+    for (int64_t j = lo; j < hi; ++j) z += exp(S[j] - m);
     const double L = m + log(z);
-    for (int64_t j = 0; j < nv; ++j) P[j] = exp(S[j] - L);
+    for (int64_t j = lo; j < hi; ++j) P[j] = exp(S[j] - L);
     *L_out = L;
-    return nv;
+    *lo_out = lo;
+    *hi_out = hi;
 }
 
 /* ---------------------------------------------------------------- forward */
-int fbob_oracle_fwd(int64_t N, int64_t d, double tau, int causal,
+int fbob_oracle_fwd(int64_t N, int64_t d, double tau, int causal, int64_t wl, int64_t wr,
                     const double* Q, const double* K, const double* V,
                     double* O, double* L, int nthreads) {
     if (N < 0 || d <= 0) return 1;
+    const band_t mk = {causal, wl, wr};
     const int nt = pick_threads(nthreads);
 #pragma omp parallel num_threads(nt)
     {
@@ -112,11 +127,12 @@ int fbob_oracle_fwd(int64_t N, int64_t d, double tau, int causal,
 #pragma omp for schedule(static)
         for (int64_t i = 0; i < N; ++i) {
             double Li;
-            const int64_t nv = softmax_row(i, N, d, tau, causal, Q, K, S, P, &Li);
+            int64_t lo, hi;
+            softmax_row(i, N, d, tau, mk, Q, K, S, P, &Li, &lo, &hi);
             L[i] = Li;
             for (int64_t a = 0; a < d; ++a) {
                 double acc = 0.0;
-                for (int64_t j = 0; j < nv; ++j) acc += P[j] * V[j * d + a];
+                for (int64_t j = lo; j < hi; ++j) acc += P[j] * V[j * d + a];
                 O[i * d + a] = acc;
             }
         }
@@ -127,10 +143,11 @@ int fbob_oracle_fwd(int64_t N, int64_t d, double tau, int causal,
 }
 
 /* ------------------------------------------------------- first backward */
-int fbob_oracle_bwd(int64_t N, int64_t d, double tau, int causal,
+int fbob_oracle_bwd(int64_t N, int64_t d, double tau, int causal, int64_t wl, int64_t wr,
                     const double* Q, const double* K, const double* V, const double* dO,
                     double* dQ, double* dK, double* dV, double* Dvec, int nthreads) {
     if (N < 0 || d <= 0) return 1;
+    const band_t mk = {causal, wl, wr};
     const int nt = pick_threads(nthreads);
     const size_t nd = (size_t)N * (size_t)d;
     double* part = (double*)calloc((size_t)nt * 2 * (nd > 0 ? nd : 1), sizeof(double));
@@ -145,15 +162,16 @@ int fbob_oracle_bwd(int64_t N, int64_t d, double tau, int causal,
 #pragma omp for schedule(static)
         for (int64_t i = 0; i < N; ++i) {
             double Li;
-            const int64_t nv = softmax_row(i, N, d, tau, causal, Q, K, S, P, &Li);
+            int64_t lo, hi;
+            softmax_row(i, N, d, tau, mk, Q, K, S, P, &Li, &lo, &hi);
             double D = 0.0;                                   /* D_i = sum_j P_ij dP_ij */
-            for (int64_t j = 0; j < nv; ++j) {
+            for (int64_t j = lo; j < hi; ++j) {
                 dP[j] = dot(dO + i * d, V + j * d, d);        /* dP = dO V^T */
                 D += P[j] * dP[j];
             }
             Dvec[i] = D;
             for (int64_t a = 0; a < d; ++a) dQ[i * d + a] = 0.0;
-            for (int64_t j = 0; j < nv; ++j) {
+            for (int64_t j = lo; j < hi; ++j) {
                 const double dS = P[j] * (dP[j] - D);         /* dS = P o (dP - D) */
                 for (int64_t a = 0; a < d; ++a) {
                     dQ[i * d + a] += tau * dS * K[j * d + a];     /* dQ = tau dS K   */
@@ -187,16 +205,18 @@ int fbob_oracle_bwd(int64_t N, int64_t d, double tau, int causal,
  * [c0, c1): the key columns whose column-owned outputs Ktil, Vtil receive the
  *   contributions of the listed rows (written as a (c1-c0) x d block).  They
  *   are the complete Ktil_j, Vtil_j only when every row i with j in V_i is
- *   listed: all rows without a mask, rows i >= j with the causal mask.
+ *   listed: all rows without a mask, rows i >= j with the causal mask, and
+ *   rows j - wr <= i <= j + wl with a window.
  * Any output pointer may be NULL; c1 <= c0 skips the column-owned sums.
  */
-int fbob_oracle_bob(int64_t N, int64_t d, double tau, int causal,
+int fbob_oracle_bob(int64_t N, int64_t d, double tau, int causal, int64_t wl, int64_t wr,
                     const double* Q, const double* K, const double* V, const double* dO,
                     const double* UQ, const double* UK, const double* UV,
                     const int64_t* rows, int64_t nrows, int64_t c0, int64_t c1,
                     double* Qt, double* dOt, double* alpha_out, double* E_out,
                     double* D_out, double* L_out, double* Kt, double* Vt, int nthreads) {
     if (N < 0 || d <= 0 || nrows < 0) return 1;
+    const band_t mk = {causal, wl, wr};
     for (int64_t r = 0; r < nrows; ++r)
         if (rows[r] < 0 || rows[r] >= N) return 1;
     if (c0 < 0) c0 = 0;
@@ -230,16 +250,17 @@ int fbob_oracle_bob(int64_t N, int64_t d, double tau, int causal,
             const double* dout = dO + i * d;
             const double* uq = UQ + i * d;
             double Li;
-            /* eq. (1): scores and probabilities of row i */
-            const int64_t nv = softmax_row(i, N, d, tau, causal, Q, K, S, P, &Li);
+            int64_t lo, hi;
+            /* eq. (1): scores and probabilities of row i over V_i = [lo, hi) */
+            softmax_row(i, N, d, tau, mk, Q, K, S, P, &Li, &lo, &hi);
             /* eq. (2): dP = dO V^T and D_i = sum_j P_ij dP_ij */
             double D = 0.0;
-            for (int64_t j = 0; j < nv; ++j) {
+            for (int64_t j = lo; j < hi; ++j) {
                 dP[j] = dot(dout, V + j * d, d);
                 D += P[j] * dP[j];
             }
             /* App. C step 1: F = tau (U_Q K^T + Q U_K^T); step 4: C = dO U_V^T */
-            for (int64_t j = 0; j < nv; ++j) {
+            for (int64_t j = lo; j < hi; ++j) {
 #if FBOB_MUTANT == 1 /* planted: dropped Q U_K^T term */
                 F[j] = tau * dot(uq, K + j * d, d);
 #elif FBOB_MUTANT == 2 /* planted: transposed operand, U_Q paired with U_K */
@@ -251,9 +272,9 @@ int fbob_oracle_bob(int64_t N, int64_t d, double tau, int causal,
             }
             /* step 2: alpha_i = sum_j P_ij F_ij */
             double alpha = 0.0;
-            for (int64_t j = 0; j < nv; ++j) alpha += P[j] * F[j];
+            for (int64_t j = lo; j < hi; ++j) alpha += P[j] * F[j];
             /* step 5: Ptil = C + F o (dP - D) - alpha dP */
-            for (int64_t j = 0; j < nv; ++j) {
+            for (int64_t j = lo; j < hi; ++j) {
 #if FBOB_MUTANT == 3 /* planted: wrong sign on the alpha term */
                 Pt[j] = C[j] + F[j] * (dP[j] - D) + alpha * dP[j];
 #elif FBOB_MUTANT == 4 /* planted: dropped C (the dV-child contribution) */
@@ -264,8 +285,8 @@ int fbob_oracle_bob(int64_t N, int64_t d, double tau, int causal,
             }
             /* step 6: E_i = sum_j P_ij Ptil_ij, Stil = P o (Ptil - E) */
             double E = 0.0;
-            for (int64_t j = 0; j < nv; ++j) E += P[j] * Pt[j];
-            for (int64_t j = 0; j < nv; ++j) {
+            for (int64_t j = lo; j < hi; ++j) E += P[j] * Pt[j];
+            for (int64_t j = lo; j < hi; ++j) {
 #if FBOB_MUTANT == 5 /* planted: E row scalar dropped */
                 St[j] = P[j] * Pt[j];
 #else
@@ -279,7 +300,7 @@ int fbob_oracle_bob(int64_t N, int64_t d, double tau, int causal,
             if (Qt || dOt) {
                 for (int64_t a = 0; a < d; ++a) {
                     double qa = 0.0, oa = 0.0;
-                    for (int64_t j = 0; j < nv; ++j) {
+                    for (int64_t j = lo; j < hi; ++j) {
                         qa += St[j] * K[j * d + a] + dS[j] * UK[j * d + a];
 #if FBOB_MUTANT == 6 /* planted: h replaced by F (alpha dropped from h) */
                         oa += P[j] * UV[j * d + a] + P[j] * F[j] * V[j * d + a];
@@ -300,8 +321,9 @@ int fbob_oracle_bob(int64_t N, int64_t d, double tau, int causal,
             /* step 7 / step 3: column-owned sums over the listed rows:
              * Ktil_j += tau (Stil_ij q_i + dS_ij u_Q,i),  Vtil_j += P_ij h_ij do_i */
             if (my_Kt) {
-                const int64_t jend = nv < c1 ? nv : c1;
-                for (int64_t j = c0; j < jend; ++j) {
+                const int64_t jbeg = lo > c0 ? lo : c0;
+                const int64_t jend = hi < c1 ? hi : c1;
+                for (int64_t j = jbeg; j < jend; ++j) {
                     double* kt = my_Kt + (size_t)(j - c0) * d;
                     double* vt = my_Vt + (size_t)(j - c0) * d;
                     const double ph = P[j] * h[j];

@@ -14,28 +14,39 @@ from __future__ import annotations
 import numpy as np
 
 
-def mask(N, causal):
+def mask(N, causal, window=None):
+    """0/1 mask: causal keeps j <= i; window (wl, wr) keeps i - wl <= j <= i + wr
+    (a negative side is unbounded)."""
+    i = np.arange(N)[:, None]
+    j = np.arange(N)[None, :]
+    keep = np.ones((N, N), dtype=bool)
     if causal:
-        return np.tril(np.ones((N, N)))
-    return np.ones((N, N))
+        keep &= j <= i
+    if window is not None:
+        wl, wr = window
+        if wl >= 0:
+            keep &= j >= i - wl
+        if wr >= 0:
+            keep &= j <= i + wr
+    return keep.astype(np.float64)
 
 
-def softmax_probs(Q, K, tau, causal):
+def softmax_probs(Q, K, tau, causal, window=None):
     """P = softmax_row(tau Q K^T + M) for [..., N, d] inputs (real or complex).
 
     The shift uses the real part of the row max so the function stays
     complex-analytic (the shift cancels exactly in the ratio)."""
     N = Q.shape[-2]
     S = tau * (Q @ np.swapaxes(K, -1, -2))
-    Mk = mask(N, causal)
+    Mk = mask(N, causal, window)
     shift = np.max(np.where(Mk > 0, S.real, -np.inf), axis=-1, keepdims=True)
     Ex = np.exp(S - shift) * Mk
     return Ex / Ex.sum(axis=-1, keepdims=True)
 
 
-def first_backward(Q, K, V, dO, tau, causal):
+def first_backward(Q, K, V, dO, tau, causal, window=None):
     """g(Q, K, V, dO) = (dQ, dK, dV), eqs. (2)-(3), batched over leading dims."""
-    P = softmax_probs(Q, K, tau, causal)
+    P = softmax_probs(Q, K, tau, causal, window)
     dP = dO @ np.swapaxes(V, -1, -2)
     D = (P * dP).sum(axis=-1, keepdims=True)
     dS = P * (dP - D)
@@ -45,12 +56,12 @@ def first_backward(Q, K, V, dO, tau, causal):
     return dQ, dK, dV
 
 
-def attention(Q, K, V, tau, causal):
-    return softmax_probs(Q, K, tau, causal) @ V
+def attention(Q, K, V, tau, causal, window=None):
+    return softmax_probs(Q, K, tau, causal, window) @ V
 
 
-def phi(Q, K, V, dO, UQ, UK, UV, tau, causal):
-    dQ, dK, dV = first_backward(Q, K, V, dO, tau, causal)
+def phi(Q, K, V, dO, UQ, UK, UV, tau, causal, window=None):
+    dQ, dK, dV = first_backward(Q, K, V, dO, tau, causal, window)
     return ((dQ * UQ).sum(axis=(-1, -2)) + (dK * UK).sum(axis=(-1, -2))
             + (dV * UV).sum(axis=(-1, -2)))
 
@@ -70,7 +81,7 @@ def _perturbed(X, which, deltas):
     return out
 
 
-def bob_central_fd(Q, K, V, dO, UQ, UK, UV, tau, causal, rel_h=1e-5):
+def bob_central_fd(Q, K, V, dO, UQ, UK, UV, tau, causal, rel_h=1e-5, window=None):
     """grad_{Q,K,V,dO} Phi by central differences, one entry at a time."""
     X = [Q, K, V, dO]
     grads = []
@@ -79,13 +90,13 @@ def bob_central_fd(Q, K, V, dO, UQ, UK, UV, tau, causal, rel_h=1e-5):
         h = rel_h * np.maximum(1.0, np.abs(x))
         plus = _perturbed(X, which, h)
         minus = _perturbed(X, which, -h)
-        fp = phi(*plus, UQ, UK, UV, tau, causal)
-        fm = phi(*minus, UQ, UK, UV, tau, causal)
+        fp = phi(*plus, UQ, UK, UV, tau, causal, window)
+        fm = phi(*minus, UQ, UK, UV, tau, causal, window)
         grads.append(((fp - fm) / (2 * h)).reshape(X[which].shape))
     return grads
 
 
-def jacobian_complex_step(Q, K, V, dO, tau, causal, h=1e-30):
+def jacobian_complex_step(Q, K, V, dO, tau, causal, h=1e-30, window=None):
     """Explicit Jacobian of g: rows index vec(dQ, dK, dV) (3Nd), columns index
     vec(Q, K, V, dO) (4Nd); built column by column by complex step."""
     N, d = Q.shape
@@ -93,7 +104,7 @@ def jacobian_complex_step(Q, K, V, dO, tau, causal, h=1e-30):
     cols = []
     for which in range(4):
         pert = _perturbed(X, which, np.full(N * d, 1j * h))
-        dQ, dK, dV = first_backward(*pert, tau, causal)
+        dQ, dK, dV = first_backward(*pert, tau, causal, window)
         J = np.concatenate([dQ.reshape(N * d, -1), dK.reshape(N * d, -1),
                             dV.reshape(N * d, -1)], axis=1).imag / h   # [Nd(in), 3Nd(out)]
         cols.append(J.T)
