@@ -22,6 +22,11 @@
  *             N <= 2^24 and B*H <= 2^24.  scale must be finite and > 0
  *             (1/sqrt(d) in the paper).  causal is 0 or 1; with 1 the mask
  *             keeps j <= i (square, top-left aligned, diagonal included).
+ *             window_left, window_right (each -1 or >= 0) add a sliding-window
+ *             band: row i keeps i - window_left <= j <= i + window_right
+ *             (App. "Sliding-window attention"); -1 leaves that side
+ *             unbounded.  Every row keeps its diagonal.  Both -1 (and causal 0)
+ *             is the unmasked problem.
  *  Stream     Every call enqueues its kernels on `stream` (NULL = legacy
  *             default stream) and returns without synchronising.
  *  Memory     The library allocates and frees no device memory.  The caller
@@ -64,8 +69,10 @@ typedef enum fbob_status {
 
 typedef struct fbob_shape {
     int64_t B, H, N, d;
-    float scale;    /* tau */
-    int32_t causal; /* 0 or 1 */
+    float scale;          /* tau */
+    int32_t causal;       /* 0 or 1 */
+    int32_t window_left;  /* sliding window: row i keeps j >= i - window_left; -1 = unbounded */
+    int32_t window_right; /* and j <= i + window_right; -1 = unbounded (causal caps it at 0) */
 } fbob_shape;
 
 /*

@@ -33,11 +33,11 @@ class _AttnBwd(torch.autograd.Function):
     """(q, k, v, dout) -> (dq, dk, dv); its backward is BoB."""
 
     @staticmethod
-    def forward(ctx, q, k, v, o, lse, dout, scale, causal):
+    def forward(ctx, q, k, v, o, lse, dout, scale, causal, window):
         dout = _bf16(dout)
-        dq, dk, dv, _ = attn_bwd(q, k, v, o, lse, dout, scale, causal)
+        dq, dk, dv, _ = attn_bwd(q, k, v, o, lse, dout, scale, causal, window)
         ctx.save_for_backward(q, k, v, o, lse, dout)
-        ctx.scale, ctx.causal = scale, causal
+        ctx.scale, ctx.causal, ctx.window = scale, causal, window
         return dq, dk, dv
 
     @staticmethod
@@ -45,33 +45,35 @@ class _AttnBwd(torch.autograd.Function):
         q, k, v, o, lse, dout = ctx.saved_tensors
         g = [torch.zeros_like(q) if t is None else _bf16(t) for t in (gq, gk, gv)]
         q_bar, k_bar, v_bar, dout_bar, _ = attn_bob(q, k, v, o, lse, dout, *g, ctx.scale,
-                                                    ctx.causal)
-        return q_bar, k_bar, v_bar, None, None, dout_bar, None, None
+                                                    ctx.causal, ctx.window)
+        return q_bar, k_bar, v_bar, None, None, dout_bar, None, None, None
 
 
 class _Attn(torch.autograd.Function):
     """(q, k, v) -> O = softmax(scale Q K^T + M) V (eq. 1)."""
 
     @staticmethod
-    def forward(ctx, q, k, v, scale, causal):
-        o, lse = attn_fwd(q, k, v, scale, causal)
+    def forward(ctx, q, k, v, scale, causal, window):
+        o, lse = attn_fwd(q, k, v, scale, causal, window)
         ctx.save_for_backward(q, k, v, o, lse)
-        ctx.scale, ctx.causal = scale, causal
+        ctx.scale, ctx.causal, ctx.window = scale, causal, window
         return o
 
     @staticmethod
     def backward(ctx, dout):
         q, k, v, o, lse = ctx.saved_tensors
-        dq, dk, dv = _AttnBwd.apply(q, k, v, o.detach(), lse, dout, ctx.scale, ctx.causal)
-        return dq, dk, dv, None, None
+        dq, dk, dv = _AttnBwd.apply(q, k, v, o.detach(), lse, dout, ctx.scale, ctx.causal,
+                                    ctx.window)
+        return dq, dk, dv, None, None, None
 
 
 def attention(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, scale: float | None = None,
-              causal: bool = False) -> torch.Tensor:
-    """Softmax attention on libfbob, differentiable twice (see the module doc)."""
+              causal: bool = False, window: tuple | None = None) -> torch.Tensor:
+    """Softmax attention on libfbob, differentiable twice (see the module doc).
+    window: (left, right) sliding-window band, -1 = unbounded side."""
     for t in (q, k, v):
         _check(t)
     if scale is None:
         scale = 1.0 / math.sqrt(q.shape[-1])
     return _Attn.apply(q.contiguous(), k.contiguous(), v.contiguous(), float(scale),
-                       bool(causal))
+                       bool(causal), None if window is None else tuple(window))

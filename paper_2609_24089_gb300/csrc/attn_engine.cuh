@@ -199,7 +199,12 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
   const int rb = p.causal ? (p.nblk - 1 - rbi) : rbi;
   const int i0 = rb * BM;
   const int last_row = min(i0 + BM, N) - 1;
-  const int ntiles = p.causal ? (last_row / BN + 1) : (N + BN - 1) / BN;
+  // streamed key tiles: those overlapping the rows' bands [i - wl, i + wr]
+  // (negative w: unbounded; the causal mask has wr = 0)
+  const int key_lo = p.wl < 0 ? 0 : max(0, i0 - p.wl);
+  const int key_hi = p.wr < 0 ? N : min(N, last_row + p.wr + 1);  // exclusive
+  const int first_tile = key_lo / BN;
+  const int ntiles = (key_hi - 1) / BN - first_tile + 1;
   const int nsteps = OP == RowOp::Fwd ? 2 * ntiles : ntiles;
   const int first_b = OP == RowOp::Fwd ? ntiles : 0;  // first step with stage-B MMAs
 
@@ -256,7 +261,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         if (st >= C::NSTAGES) {
           if (!mbar_wait(&m->bar_empty[stage], ((st / C::NSTAGES) - 1) & 1, wctl)) break;
         }
-        const int j0 = (st % ntiles) * BN;
+        const int j0 = (first_tile + st % ntiles) * BN;
         const bool k_only = (OP == RowOp::Fwd) && st < ntiles;
         const int nt = k_only ? 1 : C::NSTREAM;
         uint8_t* dst = s_stream + stage * C::STAGE_BYTES;
@@ -551,6 +556,9 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
     const int r = 32 * (warp & 3) + (tid & 31);  // stationary row in the block
     const int gi = i0 + r;
     const bool row_ok = gi < N;
+    // this row's valid keys [jlo, jhi): its band, capped at N (none past N)
+    const int jlo = !row_ok ? 0 : (p.wl < 0 ? 0 : gi - p.wl);
+    const int jhi = !row_ok ? 0 : (p.wr < 0 ? N : min(N, gi + p.wr + 1));
     const uint32_t ta = lane_base_addr(tmem, warp);
     const size_t rowoff = ((size_t)bh * N + (size_t)(row_ok ? gi : 0)) * D;
     const float tau = p.scale;
@@ -631,7 +639,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
       }
       tc_fence_before();
       mbar_arrive(&m->bar_sf_free[sfb]);
-      const int jt = (st % ntiles) * BN;
+      const int jt = (first_tile + st % ntiles) * BN;
       const float2 sl2v = splat(sl2), nL2v = splat(-L2);
       if constexpr (kStats) {
         // ---- row statistics: copy DC of the whole tile, release it, then
@@ -657,14 +665,14 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
           const int j0 = jt + HB * h + 16 * wg;
-          const bool need_mask = (!row_ok) || (j0 + 16 > N) || (p.causal && j0 + 15 > gi);
-          const int lim = need_mask ? (row_ok ? (p.causal ? min(N, gi + 1) : N) - j0 : 0) : 16;
+          const int mlo = jlo - j0, mhi = jhi - j0;  // valid columns: mlo <= c < mhi
+          const bool need_mask = mlo > 0 || mhi < 16;
 #pragma unroll
           for (int c = 0; c < 16; c += 2) {
             float2 pr = probs2(pair(rS[h], c), sl2v, nL2v);
             if (need_mask) {
-              if (c >= lim) pr.x = 0.f;
-              if (c + 1 >= lim) pr.y = 0.f;
+              if (c < mlo || c >= mhi) pr.x = 0.f;
+              if (c + 1 < mlo || c + 1 >= mhi) pr.y = 0.f;
             }
             const float2 f = __fmul2_rn(pair(rF[h], c), tauv);
             const float2 t = __fadd2_rn(pair(rdP[h], c), nDv);
@@ -685,8 +693,8 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
           }
           const int c0 = HB * h + 16 * wg;  // tile column of this thread's 16
           const int j0 = jt + c0;           // first key of this thread's 16
-          const bool need_mask = (!row_ok) || (j0 + 16 > N) || (p.causal && j0 + 15 > gi);
-          const int lim = need_mask ? (row_ok ? (p.causal ? min(N, gi + 1) : N) - j0 : 0) : 16;
+          const int mlo = jlo - j0, mhi = jhi - j0;  // valid columns: mlo <= c < mhi
+          const bool need_mask = mlo > 0 || mhi < 16;
           if constexpr (kBob) {
             const uint32_t R = ta + kColDC + 64 * h + 16 * wg;  // [dP_h | C_h] columns
             uint32_t rdP[16], rC[16];
@@ -700,8 +708,8 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
             for (int c = 0; c < 16; c += 2) {
               float2 pr = probs2(pair(rS[h], c), sl2v, nL2v);
               if (need_mask) {
-                if (c >= lim) pr.x = 0.f;
-                if (c + 1 >= lim) pr.y = 0.f;
+                if (c < mlo || c >= mhi) pr.x = 0.f;
+                if (c + 1 < mlo || c + 1 >= mhi) pr.y = 0.f;
               }
               const float2 f = __fmul2_rn(pair(rF[h], c), tauv);
               const float2 dp = pair(rdP, c);
@@ -734,8 +742,8 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
             for (int c = 0; c < 16; c += 2) {
               float2 pr = probs2(pair(rS[h], c), sl2v, nL2v);
               if (need_mask) {
-                if (c >= lim) pr.x = 0.f;
-                if (c + 1 >= lim) pr.y = 0.f;
+                if (c < mlo || c >= mhi) pr.x = 0.f;
+                if (c + 1 < mlo || c + 1 >= mhi) pr.y = 0.f;
               }
               const float2 f = __fmul2_rn(pair(rF[h], c), tauv);
               const float2 dp = pair(rdP, c);
@@ -765,8 +773,8 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
             for (int c = 0; c < 16; c += 2) {
               float2 pr = probs2(pair(rS[h], c), sl2v, nL2v);
               if (need_mask) {
-                if (c >= lim) pr.x = 0.f;
-                if (c + 1 >= lim) pr.y = 0.f;
+                if (c < mlo || c >= mhi) pr.x = 0.f;
+                if (c + 1 < mlo || c + 1 >= mhi) pr.y = 0.f;
               }
               const float2 ds = __fmul2_rn(pr, __fadd2_rn(pair(rdP, c), nDv));
               odS[c / 2] = pack_bf16(ds.x, ds.y);
@@ -779,7 +787,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
 #pragma unroll
               for (int c = 0; c < 16; ++c) {
                 x[c] = bits_f(rS[h][c]) * sl2;
-                if (need_mask && c >= lim) x[c] = -INFINITY;
+                if (need_mask && (c < mlo || c >= mhi)) x[c] = -INFINITY;
                 mx = fmaxf(mx, x[c]);
               }
               if (mx != -INFINITY) {
@@ -795,8 +803,8 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
               for (int c = 0; c < 16; c += 2) {
                 float2 pr = probs2(pair(rS[h], c), sl2v, nL2v);
                 if (need_mask) {
-                  if (c >= lim) pr.x = 0.f;
-                  if (c + 1 >= lim) pr.y = 0.f;
+                  if (c < mlo || c >= mhi) pr.x = 0.f;
+                  if (c + 1 < mlo || c + 1 >= mhi) pr.y = 0.f;
                 }
                 oP[c / 2] = pack_bf16(pr.x, pr.y);
               }
@@ -946,9 +954,13 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
   const int cb = p.head_major ? lin % p.nblk : lin / p.BH;
   const int bh = p.head_major ? lin / p.nblk : lin % p.BH;
   const int j0 = cb * BM;
-  const int first_tile = p.causal ? (j0 / BN) : 0;
-  const int ntotal = (N + BN - 1) / BN;
-  const int nsteps = ntotal - first_tile;
+  // streamed query tiles: rows whose band holds a key of this block,
+  // j - wr <= i <= j + wl (negative w: unbounded; causal: wr = 0)
+  const int last_key = min(j0 + BM, N) - 1;
+  const int q_lo = p.wr < 0 ? 0 : max(0, j0 - p.wr);
+  const int q_hi = p.wl < 0 ? N : min(N, last_key + p.wl + 1);  // exclusive
+  const int first_tile = q_lo / BN;
+  const int nsteps = (q_hi - 1) / BN - first_tile + 1;
 
   if (tid == 0) {
     m->wctl.abort = 0;
@@ -1213,6 +1225,9 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
     const int r = 32 * (warp & 3) + (tid & 31);
     const int gj = j0 + r;  // stationary key row
     const bool row_ok = gj < N;
+    // query rows that see this key: [qlo, qhi) (none for a key past N)
+    const int qlo = !row_ok ? 0 : (p.wr < 0 ? 0 : gj - p.wr);
+    const int qhi = !row_ok ? 0 : (p.wl < 0 ? N : min(N, gj + p.wl + 1));
     const uint32_t ta = lane_base_addr(tmem, warp);
     const float tau = p.scale;
     const float2 sl2v = splat(tau * kLog2e), tauv = splat(tau);
@@ -1253,10 +1268,9 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
       for (int h = 0; h < 2; ++h) {
         const int cv = HB * h + 16 * wg;             // tile column of this thread's first
         const int ib = (first_tile + st) * BN + cv;  // first query row of this thread's 16
-        const bool need_mask = (!row_ok) || (ib + 16 > N) || (p.causal && ib < gj);
         // valid query columns c satisfy  lo <= c < hi
-        const int lo = p.causal ? gj - ib : 0;
-        const int hi = row_ok ? N - ib : 0;
+        const int lo = qlo - ib, hi = qhi - ib;
+        const bool need_mask = lo > 0 || hi < 16;
         const uint32_t R = ta + dcol + cv;
         if constexpr (kBob) {
           uint32_t rdP[16], rC[16];

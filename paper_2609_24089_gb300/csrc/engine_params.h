@@ -47,6 +47,7 @@ struct EngineParams {
   int BH;
   int nblk;  // stationary blocks per head
   int causal;
+  int wl, wr;  // valid band of row i: i - wl <= j <= i + wr (-1: unbounded); causal gives wr = 0
   float scale;
   long long bhn;  // BH * N (row_stats plane stride)
   unsigned long long wait_limit_ns;  // bound of every device-side wait

@@ -64,6 +64,7 @@ int check_shape(const fbob_shape* s, bool* empty) {
   if (s->B < 0 || s->H < 0 || s->N < 0 || s->d <= 0) return FBOB_ERR_INVALID_ARGUMENT;
   if (!(std::isfinite(s->scale) && s->scale > 0.f)) return FBOB_ERR_INVALID_ARGUMENT;
   if (s->causal != 0 && s->causal != 1) return FBOB_ERR_INVALID_ARGUMENT;
+  if (s->window_left < -1 || s->window_right < -1) return FBOB_ERR_INVALID_ARGUMENT;
   if (s->d != 64 && s->d != 128) return FBOB_ERR_UNSUPPORTED;
   if (s->N > kMaxN) return FBOB_ERR_INVALID_ARGUMENT;
   if (s->B > kMaxBH || s->H > kMaxBH || s->B * s->H > kMaxBH) return FBOB_ERR_INVALID_ARGUMENT;
@@ -119,6 +120,8 @@ EngineParams base_params(const fbob_shape* s) {
   p.N = (int)s->N;
   p.BH = (int)(s->B * s->H);
   p.causal = s->causal;
+  p.wl = s->window_left;
+  p.wr = s->causal ? 0 : s->window_right;
   p.scale = s->scale;
   p.bhn = s->B * s->H * s->N;
   debug_controls(&p);

@@ -66,22 +66,23 @@ def f64(bits):
     return synth.to_f64(bits)
 
 
-def oracle_o_l(bits, scale, causal):
+def oracle_o_l(bits, scale, causal, window=None):
     """O rounded to bf16 and L rounded to fp32, from the oracle's forward."""
-    O, L = oracle.fwd(f64(bits["q"]), f64(bits["k"]), f64(bits["v"]), scale, causal)
+    O, L = oracle.fwd(f64(bits["q"]), f64(bits["k"]), f64(bits["v"]), scale, causal,
+                      window=window)
     return synth.bf16_bits(O.astype(np.float32)), L.astype(np.float32)
 
 
-def run_bob(bits, scale, causal, o_l=None):
+def run_bob(bits, scale, causal, o_l=None, window=None):
     """Upload, (forward unless o_l is given), then backward-over-backward.
     Returns dict of host float64 arrays and the device status."""
     t = torch()
     q, k, v, do, gq, gk, gv = (dev(bits[n]) for n in synth.NAMES)
     if o_l is None:
-        o, lse = fbob.attn_fwd(q, k, v, scale, causal)
+        o, lse = fbob.attn_fwd(q, k, v, scale, causal, window)
     else:
         o, lse = dev(o_l[0]), dev_f32(o_l[1])
-    qb, kb, vb, dob, rs = fbob.attn_bob(q, k, v, o, lse, do, gq, gk, gv, scale, causal)
+    qb, kb, vb, dob, rs = fbob.attn_bob(q, k, v, o, lse, do, gq, gk, gv, scale, causal, window)
     status = fbob.fbob_device_status()
     t.cuda.synchronize()
     return {"qbar": host(qb), "kbar": host(kb), "vbar": host(vb), "dobar": host(dob),

@@ -111,3 +111,12 @@ def test_row_stats_and_direct_validate_like_pass1(lib):
     assert lib.fbob_launch_count(b"bob_row_stats") == 0
     assert pd(ctypes.byref(empty), *ptrs(11), None) == 0
     assert lib.fbob_launch_count(b"bob_pass1_direct") == 0
+
+
+def test_rejects_bad_windows(lib):
+    S = fbob.make_shape
+    assert bob(lib, S(1, 1, 128, 64, 0.125, 0, window=(-2, -1)), ptrs(14)) == 1
+    assert bob(lib, S(1, 1, 128, 64, 0.125, 1, window=(3, -5)), ptrs(14)) == 1
+    # valid windows pass validation (then stop at the empty problem, no CUDA call)
+    assert bob(lib, S(1, 1, 0, 64, 0.125, 0, window=(3, 4)), ptrs(14)) == 0
+    assert bob(lib, S(1, 1, 0, 64, 0.125, 1, window=(0, -1)), ptrs(14)) == 0
