@@ -33,6 +33,7 @@ class Workload:
     causal: bool
     seed: int
     sigma: tuple  # per tensor in NAMES order
+    window: tuple = (-1, -1)  # sliding-window band (left, right); -1 = unbounded
 
     @property
     def scale(self) -> float:
@@ -58,7 +59,24 @@ WORKLOADS = {
     "n64k_d128_causal_peaky": Workload(
         "n64k_d128_causal_peaky", 1, 8, 65536, 128, True, 3, _s(1.5, 1.5, 1, 1, 1, 1, 1)),
     "n256k_d64": Workload("n256k_d64", 1, 4, 262144, 64, False, 4, _s(1, 1, 1, 1, 1, 1, 1)),
+    # sliding-window variant of n16k_d128_causal with the window of the paper's
+    # sliding-window experiment, w = N/4 keys (row i keeps i - w < j <= i)
+    "n16k_d128_causal_swa4k": Workload(
+        "n16k_d128_causal_swa4k", 2, 16, 16384, 128, True, 5,
+        _s(1, 1, 1, *(4 * [1 / math.sqrt(128)])), (4095, -1)),
 }
+
+
+def band_pairs(w: Workload, rows=None) -> float:
+    """Valid (i, j) pairs of the listed rows (all rows by default) under the
+    workload's mask: the band i - wl <= j <= i + wr, capped at j <= i if causal."""
+    r = np.arange(w.N, dtype=np.int64) if rows is None else np.asarray(rows, dtype=np.int64)
+    wl, wr = w.window
+    lo = np.zeros_like(r) if wl < 0 else np.maximum(0, r - wl)
+    hi = np.full_like(r, w.N) if wr < 0 else np.minimum(w.N, r + wr + 1)
+    if w.causal:
+        hi = np.minimum(hi, r + 1)
+    return float(np.sum(hi - lo))
 
 
 def bf16_bits(x: np.ndarray) -> np.ndarray:

@@ -92,14 +92,14 @@ def run_bob(bits, scale, causal, o_l=None, window=None):
             "o": host(o), "lse": lse.cpu().numpy().astype(np.float64), "status": status}
 
 
-def oracle_bob_heads(bits, scale, causal, heads, rows=None, cols=None):
+def oracle_bob_heads(bits, scale, causal, heads, rows=None, cols=None, window=None):
     """Oracle on selected flat heads of a [B,H,N,d] bit tensor set."""
     B, H, N, d = bits["q"].shape
     out = []
     for hh in heads:
         b, h = divmod(hh, H)
         X = [f64(bits[n][b, h]) for n in synth.NAMES]
-        out.append(oracle.bob_head(*X, scale, causal, rows=rows, cols=cols))
+        out.append(oracle.bob_head(*X, scale, causal, rows=rows, cols=cols, window=window))
     return out
 
 

@@ -9,6 +9,9 @@ launch configuration the benchmark times.
                          rows >= N - 256 are summed
   n256k_d64              oracle on sampled rows; Ktil, Vtil through identities that
                          hold at any size (column sums vanish, Euler identities)
+  n16k_d128_causal_swa4k sliding window w = N/4: oracle on sampled rows and on a
+                         256-key block, complete once the rows whose band holds
+                         it (keys j .. j + 4095) are summed
 """
 import os
 
@@ -132,3 +135,21 @@ def test_n256k_d64_rows_and_identities():
         assert abs(float((Vt * X["v"]).sum()) - (a + bk)) <= 2e-2 * (abs(a) + abs(bk))
         lhs = float((Qt * X["q"]).sum()) - float((Kt * X["k"]).sum())
         assert abs(lhs - (bk - a)) <= 2e-2 * (abs(a) + abs(bk))
+
+
+def test_n16k_d128_causal_swa4k_rows_and_key_block():
+    w = synth.WORKLOADS["n16k_d128_causal_swa4k"]
+    bits = synth.workload_inputs(w)
+    r = G.run_bob(bits, w.scale, w.causal, window=w.window)
+    assert r["status"] == 0
+    N, wl = w.N, w.window[0]
+    heads = [5]
+    rows = sample_rows(N, 65)
+    check_rows(r, G.oracle_bob_heads(bits, w.scale, w.causal, heads, rows=rows, window=w.window),
+               heads, w.H, rows)
+    c0, c1 = N // 2, N // 2 + 256
+    blk = G.oracle_bob_heads(bits, w.scale, w.causal, heads, rows=np.arange(c0, min(N, c1 + wl)),
+                             cols=(c0, c1), window=w.window)
+    for hh, ref in zip(heads, blk):
+        G.check("kbar[block]", G.flat(r["kbar"], hh, w.H)[c0:c1], ref["kbar"])
+        G.check("vbar[block]", G.flat(r["vbar"], hh, w.H)[c0:c1], ref["vbar"])
