@@ -48,9 +48,10 @@ def _load(mutant: int = 0, out_dir: str | None = None):
     lib = ctypes.CDLL(build(mutant, out_dir))
     i64, dbl, cint = ctypes.c_int64, ctypes.c_double, ctypes.c_int
     p = ctypes.c_void_p
-    lib.fbob_oracle_fwd.argtypes = [i64, i64, dbl, cint, i64, i64, p, p, p, p, p, cint]
-    lib.fbob_oracle_bwd.argtypes = [i64, i64, dbl, cint, i64, i64, p, p, p, p, p, p, p, p, cint]
-    lib.fbob_oracle_bob.argtypes = [i64, i64, dbl, cint, i64, i64, p, p, p, p, p, p, p,
+    lib.fbob_oracle_fwd.argtypes = [i64, i64, dbl, cint, i64, i64, p, i64, p, p, p, p, p, cint]
+    lib.fbob_oracle_bwd.argtypes = [i64, i64, dbl, cint, i64, i64, p, i64,
+                                    p, p, p, p, p, p, p, p, cint]
+    lib.fbob_oracle_bob.argtypes = [i64, i64, dbl, cint, i64, i64, p, i64, p, p, p, p, p, p, p,
                                     p, i64, i64, i64, p, p, p, p, p, p, p, p, cint]
     for f in (lib.fbob_oracle_fwd, lib.fbob_oracle_bwd, lib.fbob_oracle_bob):
         f.restype = cint
@@ -74,6 +75,17 @@ def _window(window):
     return wl, wr
 
 
+def _segments(segments, N):
+    """Segment offsets of packed variable-length sequences as an int64 array
+    (seg[0] = 0, non-decreasing, seg[-1] = N), or None for one sequence."""
+    if segments is None:
+        return None, 0
+    seg = np.ascontiguousarray(segments, dtype=np.int64)
+    assert seg.ndim == 1 and seg.size >= 2 and seg[0] == 0 and seg[-1] == N
+    assert np.all(np.diff(seg) >= 0)
+    return seg, seg.size - 1
+
+
 def _heads(x):
     x = np.asarray(x)
     if x.ndim == 2:
@@ -81,12 +93,14 @@ def _heads(x):
     return x
 
 
-def fwd(q, k, v, scale, causal, nthreads=0, window=None):
+def fwd(q, k, v, scale, causal, nthreads=0, window=None, segments=None):
     """Forward attention (eq. 1).  Returns O [B,H,N,d] and natural-log L [B,H,N].
-    window: (wl, wr) sliding-window band (default: none)."""
+    window: (wl, wr) sliding-window band (default: none); segments: offsets of
+    packed sequences (default: one sequence)."""
     wl, wr = _window(window)
     q, k, v = (_c(_heads(t)) for t in (q, k, v))
     B, H, N, d = q.shape
+    seg, nseg = _segments(segments, N)
     lib = _load()
     O = np.zeros_like(q)
     L = np.zeros((B, H, N))
@@ -94,6 +108,7 @@ def fwd(q, k, v, scale, causal, nthreads=0, window=None):
         for h in range(H):
             o_ = np.zeros((N, d)); l_ = np.zeros(N)
             rc = lib.fbob_oracle_fwd(N, d, float(scale), int(bool(causal)), wl, wr,
+                                     _ptr(seg), nseg,
                                      _ptr(_c(q[b, h])), _ptr(_c(k[b, h])), _ptr(_c(v[b, h])),
                                      _ptr(o_), _ptr(l_), int(nthreads))
             assert rc == 0, rc
@@ -101,11 +116,12 @@ def fwd(q, k, v, scale, causal, nthreads=0, window=None):
     return O, L
 
 
-def bwd(q, k, v, dout, scale, causal, nthreads=0, window=None):
+def bwd(q, k, v, dout, scale, causal, nthreads=0, window=None, segments=None):
     """First backward (eqs. 2-3).  Returns dQ, dK, dV [B,H,N,d] and D [B,H,N]."""
     wl, wr = _window(window)
     q, k, v, dout = (_c(_heads(t)) for t in (q, k, v, dout))
     B, H, N, d = q.shape
+    seg, nseg = _segments(segments, N)
     lib = _load()
     outs = [np.zeros_like(q) for _ in range(3)]
     D = np.zeros((B, H, N))
@@ -113,6 +129,7 @@ def bwd(q, k, v, dout, scale, causal, nthreads=0, window=None):
         for h in range(H):
             dq, dk, dv, dd = np.zeros((N, d)), np.zeros((N, d)), np.zeros((N, d)), np.zeros(N)
             rc = lib.fbob_oracle_bwd(N, d, float(scale), int(bool(causal)), wl, wr,
+                                     _ptr(seg), nseg,
                                      _ptr(_c(q[b, h])), _ptr(_c(k[b, h])), _ptr(_c(v[b, h])),
                                      _ptr(_c(dout[b, h])), _ptr(dq), _ptr(dk), _ptr(dv),
                                      _ptr(dd), int(nthreads))
@@ -122,7 +139,7 @@ def bwd(q, k, v, dout, scale, causal, nthreads=0, window=None):
 
 
 def bob_head(q, k, v, dout, gq, gk, gv, scale, causal, rows=None, cols=None,
-             nthreads=0, mutant=0, mutant_dir=None, window=None):
+             nthreads=0, mutant=0, mutant_dir=None, window=None, segments=None):
     """Backward-over-backward of one head ([N, d] float64 arrays).
 
     rows: query rows whose row-owned outputs are wanted (default: all).
@@ -131,10 +148,12 @@ def bob_head(q, k, v, dout, gq, gk, gv, scale, causal, rows=None, cols=None,
     Returns a dict with qbar, dobar, alpha, E, D, L (indexed like rows) and
     kbar, vbar ((c1-c0) x d; complete only if every contributing row is listed).
     window: (wl, wr) sliding-window band i - wl <= j <= i + wr (-1 = unbounded).
+    segments: offsets of packed sequences; a row sees only its own sequence.
     """
     wl, wr = _window(window)
     q, k, v, dout, gq, gk, gv = (_c(t) for t in (q, k, v, dout, gq, gk, gv))
     N, d = q.shape
+    seg, nseg = _segments(segments, N)
     if rows is None:
         rows = np.arange(N, dtype=np.int64)
         if cols is None:
@@ -151,7 +170,7 @@ def bob_head(q, k, v, dout, gq, gk, gv, scale, causal, rows=None, cols=None,
         "kbar": np.zeros((nc, d)), "vbar": np.zeros((nc, d)),
     }
     lib = _load(mutant, mutant_dir)
-    rc = lib.fbob_oracle_bob(N, d, float(scale), int(bool(causal)), wl, wr,
+    rc = lib.fbob_oracle_bob(N, d, float(scale), int(bool(causal)), wl, wr, _ptr(seg), nseg,
                              _ptr(q), _ptr(k), _ptr(v), _ptr(dout), _ptr(gq), _ptr(gk), _ptr(gv),
                              _ptr(rows), nr, c0, c1,
                              _ptr(res["qbar"]), _ptr(res["dobar"]), _ptr(res["alpha"]),
@@ -162,7 +181,7 @@ def bob_head(q, k, v, dout, gq, gk, gv, scale, causal, rows=None, cols=None,
 
 
 def bob(q, k, v, dout, gq, gk, gv, scale, causal, nthreads=0, mutant=0, mutant_dir=None,
-        window=None):
+        window=None, segments=None):
     """Full backward-over-backward on [B,H,N,d] (or [N,d]) float64 arrays.
 
     Returns (qbar, kbar, vbar, dobar, alpha, E, D) with the input's batch shape.
@@ -175,7 +194,8 @@ def bob(q, k, v, dout, gq, gk, gv, scale, causal, nthreads=0, mutant=0, mutant_d
     for b in range(B):
         for h in range(H):
             r = bob_head(*(t[b, h] for t in ts), scale, causal, nthreads=nthreads,
-                         mutant=mutant, mutant_dir=mutant_dir, window=window)
+                         mutant=mutant, mutant_dir=mutant_dir, window=window,
+                         segments=segments)
             for n in ("qbar", "kbar", "vbar", "dobar", "alpha", "E", "D"):
                 out[n][b, h] = r[n]
     return (out["qbar"], out["kbar"], out["vbar"], out["dobar"],

@@ -35,8 +35,12 @@
  *   lo_i = max(0, i - wl)                    (wl < 0: lo_i = 0),
  *   hi_i = min(N, i + wr + 1)                (wr < 0: hi_i = N),
  * and the causal mask (square, top-left aligned, diagonal included) caps
- * hi_i at i + 1.  wl = wr = -1 is the plain mask.  Every row keeps its
- * diagonal.  Entries outside V_i have P = 0 and contribute nothing.
+ * hi_i at i + 1.  wl = wr = -1 is the plain mask.  Packed variable-length
+ * sequences (App. "Extensions"): with segment offsets seg[0..nseg] (seg[0] =
+ * 0, non-decreasing, seg[nseg] = N) row i also keeps only the columns of its
+ * own segment [seg[s], seg[s+1]), s the segment holding i; seg = NULL is one
+ * segment.  Every row keeps its diagonal.  Entries outside V_i have P = 0 and
+ * contribute nothing.
  *
  * Threads: rows are independent, so OpenMP splits rows across threads.  The
  * column-owned sums (Ktil, Vtil, dV, dK) are accumulated into one private
@@ -63,13 +67,21 @@ static double dot(const double* a, const double* b, int64_t d) {
     return s;
 }
 
-/* the valid band [lo_i, hi_i) of row i (see the header comment) */
-typedef struct { int causal; int64_t wl, wr; } band_t;
+/* the valid columns [lo_i, hi_i) of row i (see the header comment) */
+typedef struct { int causal; int64_t wl, wr; const int64_t* seg; int64_t nseg; } band_t;
 
 static void valid_cols(int64_t i, int64_t N, band_t m, int64_t* lo, int64_t* hi) {
     int64_t a = m.wl < 0 ? 0 : i - m.wl;
     int64_t b = m.wr < 0 ? N : i + m.wr + 1;
     if (m.causal && b > i + 1) b = i + 1;
+    if (m.seg) {  /* the segment holding row i: a plain scan */
+        for (int64_t s = 0; s < m.nseg; ++s)
+            if (m.seg[s] <= i && i < m.seg[s + 1]) {
+                if (a < m.seg[s]) a = m.seg[s];
+                if (b > m.seg[s + 1]) b = m.seg[s + 1];
+                break;
+            }
+    }
     *lo = a < 0 ? 0 : a;
     *hi = b > N ? N : b;
 }
@@ -115,10 +127,11 @@ static void softmax_row(int64_t i, int64_t N, int64_t d, double tau, band_t mk,
 
 /* ---------------------------------------------------------------- forward */
 int fbob_oracle_fwd(int64_t N, int64_t d, double tau, int causal, int64_t wl, int64_t wr,
+                    const int64_t* seg, int64_t nseg,
                     const double* Q, const double* K, const double* V,
                     double* O, double* L, int nthreads) {
     if (N < 0 || d <= 0) return 1;
-    const band_t mk = {causal, wl, wr};
+    const band_t mk = {causal, wl, wr, seg, nseg};
     const int nt = pick_threads(nthreads);
 #pragma omp parallel num_threads(nt)
     {
@@ -144,10 +157,11 @@ int fbob_oracle_fwd(int64_t N, int64_t d, double tau, int causal, int64_t wl, in
 
 /* ------------------------------------------------------- first backward */
 int fbob_oracle_bwd(int64_t N, int64_t d, double tau, int causal, int64_t wl, int64_t wr,
+                    const int64_t* seg, int64_t nseg,
                     const double* Q, const double* K, const double* V, const double* dO,
                     double* dQ, double* dK, double* dV, double* Dvec, int nthreads) {
     if (N < 0 || d <= 0) return 1;
-    const band_t mk = {causal, wl, wr};
+    const band_t mk = {causal, wl, wr, seg, nseg};
     const int nt = pick_threads(nthreads);
     const size_t nd = (size_t)N * (size_t)d;
     double* part = (double*)calloc((size_t)nt * 2 * (nd > 0 ? nd : 1), sizeof(double));
@@ -205,18 +219,19 @@ int fbob_oracle_bwd(int64_t N, int64_t d, double tau, int causal, int64_t wl, in
  * [c0, c1): the key columns whose column-owned outputs Ktil, Vtil receive the
  *   contributions of the listed rows (written as a (c1-c0) x d block).  They
  *   are the complete Ktil_j, Vtil_j only when every row i with j in V_i is
- *   listed: all rows without a mask, rows i >= j with the causal mask, and
- *   rows j - wr <= i <= j + wl with a window.
+ *   listed: all rows without a mask, rows i >= j with the causal mask,
+ *   rows j - wr <= i <= j + wl with a window, and only rows of j's segment.
  * Any output pointer may be NULL; c1 <= c0 skips the column-owned sums.
  */
 int fbob_oracle_bob(int64_t N, int64_t d, double tau, int causal, int64_t wl, int64_t wr,
+                    const int64_t* seg, int64_t nseg,
                     const double* Q, const double* K, const double* V, const double* dO,
                     const double* UQ, const double* UK, const double* UV,
                     const int64_t* rows, int64_t nrows, int64_t c0, int64_t c1,
                     double* Qt, double* dOt, double* alpha_out, double* E_out,
                     double* D_out, double* L_out, double* Kt, double* Vt, int nthreads) {
     if (N < 0 || d <= 0 || nrows < 0) return 1;
-    const band_t mk = {causal, wl, wr};
+    const band_t mk = {causal, wl, wr, seg, nseg};
     for (int64_t r = 0; r < nrows; ++r)
         if (rows[r] < 0 || rows[r] >= N) return 1;
     if (c0 < 0) c0 = 0;

@@ -14,12 +14,16 @@ from __future__ import annotations
 import numpy as np
 
 
-def mask(N, causal, window=None):
+def mask(N, causal, window=None, segments=None):
     """0/1 mask: causal keeps j <= i; window (wl, wr) keeps i - wl <= j <= i + wr
-    (a negative side is unbounded)."""
+    (a negative side is unbounded); segments (offsets of packed sequences)
+    keeps i and j in the same sequence (a block-diagonal mask)."""
     i = np.arange(N)[:, None]
     j = np.arange(N)[None, :]
     keep = np.ones((N, N), dtype=bool)
+    if segments is not None:
+        sid = np.searchsorted(np.asarray(segments)[1:], np.arange(N), side="right")
+        keep &= sid[:, None] == sid[None, :]
     if causal:
         keep &= j <= i
     if window is not None:
@@ -31,22 +35,22 @@ def mask(N, causal, window=None):
     return keep.astype(np.float64)
 
 
-def softmax_probs(Q, K, tau, causal, window=None):
+def softmax_probs(Q, K, tau, causal, window=None, segments=None):
     """P = softmax_row(tau Q K^T + M) for [..., N, d] inputs (real or complex).
 
     The shift uses the real part of the row max so the function stays
     complex-analytic (the shift cancels exactly in the ratio)."""
     N = Q.shape[-2]
     S = tau * (Q @ np.swapaxes(K, -1, -2))
-    Mk = mask(N, causal, window)
+    Mk = mask(N, causal, window, segments)
     shift = np.max(np.where(Mk > 0, S.real, -np.inf), axis=-1, keepdims=True)
     Ex = np.exp(S - shift) * Mk
     return Ex / Ex.sum(axis=-1, keepdims=True)
 
 
-def first_backward(Q, K, V, dO, tau, causal, window=None):
+def first_backward(Q, K, V, dO, tau, causal, window=None, segments=None):
     """g(Q, K, V, dO) = (dQ, dK, dV), eqs. (2)-(3), batched over leading dims."""
-    P = softmax_probs(Q, K, tau, causal, window)
+    P = softmax_probs(Q, K, tau, causal, window, segments)
     dP = dO @ np.swapaxes(V, -1, -2)
     D = (P * dP).sum(axis=-1, keepdims=True)
     dS = P * (dP - D)
@@ -56,12 +60,12 @@ def first_backward(Q, K, V, dO, tau, causal, window=None):
     return dQ, dK, dV
 
 
-def attention(Q, K, V, tau, causal, window=None):
-    return softmax_probs(Q, K, tau, causal, window) @ V
+def attention(Q, K, V, tau, causal, window=None, segments=None):
+    return softmax_probs(Q, K, tau, causal, window, segments) @ V
 
 
-def phi(Q, K, V, dO, UQ, UK, UV, tau, causal, window=None):
-    dQ, dK, dV = first_backward(Q, K, V, dO, tau, causal, window)
+def phi(Q, K, V, dO, UQ, UK, UV, tau, causal, window=None, segments=None):
+    dQ, dK, dV = first_backward(Q, K, V, dO, tau, causal, window, segments)
     return ((dQ * UQ).sum(axis=(-1, -2)) + (dK * UK).sum(axis=(-1, -2))
             + (dV * UV).sum(axis=(-1, -2)))
 
@@ -81,7 +85,8 @@ def _perturbed(X, which, deltas):
     return out
 
 
-def bob_central_fd(Q, K, V, dO, UQ, UK, UV, tau, causal, rel_h=1e-5, window=None):
+def bob_central_fd(Q, K, V, dO, UQ, UK, UV, tau, causal, rel_h=1e-5, window=None,
+                   segments=None):
     """grad_{Q,K,V,dO} Phi by central differences, one entry at a time."""
     X = [Q, K, V, dO]
     grads = []
@@ -90,8 +95,8 @@ def bob_central_fd(Q, K, V, dO, UQ, UK, UV, tau, causal, rel_h=1e-5, window=None
         h = rel_h * np.maximum(1.0, np.abs(x))
         plus = _perturbed(X, which, h)
         minus = _perturbed(X, which, -h)
-        fp = phi(*plus, UQ, UK, UV, tau, causal, window)
-        fm = phi(*minus, UQ, UK, UV, tau, causal, window)
+        fp = phi(*plus, UQ, UK, UV, tau, causal, window, segments)
+        fm = phi(*minus, UQ, UK, UV, tau, causal, window, segments)
         grads.append(((fp - fm) / (2 * h)).reshape(X[which].shape))
     return grads
 

@@ -112,3 +112,80 @@ def test_column_sums_vanish_and_sampling_agrees(case):
     c = oracle.bob_head(*X, tau, causal, rows=np.arange(lo, hi), cols=(c0, c1), window=win)
     assert np.allclose(c["kbar"], r["kbar"][c0:c1], atol=1e-12)
     assert np.allclose(c["vbar"], r["vbar"][c0:c1], atol=1e-12)
+
+
+# ---------------------------------------------------------------- varlen
+# Packed variable-length sequences (App. "Extensions"): segment offsets split
+# the N rows; a row sees only the columns of its own sequence.
+SEGMENTS = [  # N, d, causal, window, offsets
+    (40, 8, True, None, [0, 7, 20, 21, 40]),
+    (36, 8, False, None, [0, 13, 13, 36]),
+    (45, 4, True, (6, -1), [0, 30, 45]),
+    (30, 8, False, (3, 2), [0, 1, 2, 17, 30]),
+]
+
+
+def sids(c):
+    N, d, causal, win, seg = c
+    return f"N{N}{'c' if causal else ''}w{win}s{len(seg) - 1}"
+
+
+@pytest.mark.parametrize("case", SEGMENTS, ids=sids)
+def test_central_fd_with_segment_mask(case):
+    N, d, causal, win, seg = case
+    X = rand_problem(N, d, 700 + N)
+    tau = 1 / np.sqrt(d)
+    r = oracle.bob_head(*X, tau, causal, window=win, segments=seg)
+    fd = pins.bob_central_fd(*X, tau, causal, window=win, segments=seg)
+    for name, g in zip(("qbar", "kbar", "vbar", "dobar"), fd):
+        assert pins.rel_fro(g, r[name]) <= 1e-6, (name, pins.rel_fro(g, r[name]))
+
+
+@pytest.mark.parametrize("case", SEGMENTS[:2], ids=sids)
+def test_torch_double_backward_with_segment_mask(case):
+    torch = pytest.importorskip("torch")
+    N, d, causal, win, seg = case
+    X = rand_problem(N, d, 800 + N)
+    tau = 1 / np.sqrt(d)
+    keep = torch.tensor(pins.mask(N, causal, win, seg) > 0)
+    q, k, v, do = (torch.tensor(x, dtype=torch.float64, requires_grad=True) for x in X[:4])
+    uq, uk, uv = (torch.tensor(x, dtype=torch.float64) for x in X[4:])
+    s = (tau * q @ k.T).masked_fill(~keep, float("-inf"))
+    o = torch.softmax(s, dim=-1) @ v
+    dq, dk, dv = torch.autograd.grad(o, (q, k, v), do, create_graph=True)
+    phi = (dq * uq).sum() + (dk * uk).sum() + (dv * uv).sum()
+    grads = torch.autograd.grad(phi, (q, k, v, do))
+    r = oracle.bob_head(*X, tau, causal, window=win, segments=seg)
+    for name, g in zip(("qbar", "kbar", "vbar", "dobar"), grads):
+        assert pins.rel_fro(g.numpy(), r[name]) <= 1e-12, name
+    O, L = oracle.fwd(*X[:3], tau, causal, window=win, segments=seg)
+    assert np.allclose(O[0, 0], o.detach().numpy(), atol=1e-12)
+    dQ, dK, dV, _ = oracle.bwd(*X[:4], tau, causal, window=win, segments=seg)
+    for got, want in ((dQ, dq), (dK, dk), (dV, dv)):
+        assert np.allclose(got[0, 0], want.detach().numpy(), atol=1e-12)
+
+
+@pytest.mark.parametrize("case", SEGMENTS, ids=sids)
+def test_packed_sequences_are_independent_problems(case):
+    """A block-diagonal mask decouples the sequences: the packed BoB equals
+    the BoB of each sequence on its own."""
+    N, d, causal, win, seg = case
+    X = rand_problem(N, d, 900 + N)
+    tau = 1 / np.sqrt(d)
+    r = oracle.bob_head(*X, tau, causal, window=win, segments=seg)
+    for a, b in zip(seg[:-1], seg[1:]):
+        if b == a:
+            continue
+        part = oracle.bob_head(*(x[a:b] for x in X), tau, causal, window=win)
+        for n in ("qbar", "kbar", "vbar", "dobar", "alpha", "E", "D", "L"):
+            assert np.allclose(r[n][a:b], part[n], rtol=0, atol=1e-12), (n, a, b)
+
+
+def test_one_segment_is_no_segments():
+    N, d = 33, 8
+    X = rand_problem(N, d, 12)
+    tau = 1 / np.sqrt(d)
+    a = oracle.bob_head(*X, tau, True)
+    b = oracle.bob_head(*X, tau, True, segments=[0, N])
+    for n in ("qbar", "kbar", "vbar", "dobar", "alpha", "E", "D", "L"):
+        assert np.array_equal(a[n], b[n]), n
