@@ -27,6 +27,16 @@
  *             (App. "Sliding-window attention"); -1 leaves that side
  *             unbounded.  Every row keeps its diagonal.  Both -1 (and causal 0)
  *             is the unmasked problem.
+ *             seq_offsets (optional) packs variable-length sequences along N
+ *             (App. "Extensions"): a device array of num_seqs + 1 int32 with
+ *             seq_offsets[0] = 0, non-decreasing, seq_offsets[num_seqs] = N,
+ *             the same for every (b, h).  Row i then keeps only the columns of
+ *             its own sequence (intersected with the causal mask and the
+ *             window); causal and the window apply within a sequence in the
+ *             global index.  The contents are not checked on the host; offsets
+ *             that break these rules give unspecified values but no access
+ *             outside the caller's buffers.  NULL (with num_seqs 0) is one
+ *             sequence.
  *  Stream     Every call enqueues its kernels on `stream` (NULL = legacy
  *             default stream) and returns without synchronising.
  *  Memory     The library allocates and frees no device memory.  The caller
@@ -73,6 +83,8 @@ typedef struct fbob_shape {
     int32_t causal;       /* 0 or 1 */
     int32_t window_left;  /* sliding window: row i keeps j >= i - window_left; -1 = unbounded */
     int32_t window_right; /* and j <= i + window_right; -1 = unbounded (causal caps it at 0) */
+    const int32_t* seq_offsets; /* packed sequences: device int32 [num_seqs + 1], or NULL */
+    int64_t num_seqs;           /* number of packed sequences (0 when seq_offsets is NULL) */
 } fbob_shape;
 
 /*

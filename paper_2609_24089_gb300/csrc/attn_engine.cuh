@@ -113,6 +113,24 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
   }
 }
 
+// [lo, hi) of the packed sequence holding index i: [0, N) without offsets.
+// A binary search for the last s with off[s] <= i; the result is clamped to
+// [0, N) and to contain i, so offsets that break the documented rules give
+// wrong values but never an access outside the buffers or an empty row.
+__device__ __forceinline__ void seq_bounds(const EngineParams& p, int i, int& lo, int& hi) {
+  lo = 0;
+  hi = p.N;
+  if (p.seq_off == nullptr) return;
+  int a = 0, b = p.nseq;
+  while (b - a > 1) {
+    const int m = (a + b) >> 1;
+    if (p.seq_off[m] <= i) a = m;
+    else b = m;
+  }
+  lo = max(0, min(p.seq_off[a], i));
+  hi = min(p.N, max(p.seq_off[a + 1], i + 1));
+}
+
 __device__ __forceinline__ float bits_f(uint32_t u) { return __uint_as_float(u); }
 __device__ __forceinline__ float2 pair(const uint32_t (&r)[16], int c) {
   return make_float2(__uint_as_float(r[c]), __uint_as_float(r[c + 1]));
@@ -200,9 +218,13 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
   const int i0 = rb * BM;
   const int last_row = min(i0 + BM, N) - 1;
   // streamed key tiles: those overlapping the rows' bands [i - wl, i + wr]
-  // (negative w: unbounded; the causal mask has wr = 0)
-  const int key_lo = p.wl < 0 ? 0 : max(0, i0 - p.wl);
-  const int key_hi = p.wr < 0 ? N : min(N, last_row + p.wr + 1);  // exclusive
+  // (negative w: unbounded; the causal mask has wr = 0) within their packed
+  // sequences; both ends of a row's range grow with i
+  int seq_lo0, seq_hi0, seq_lo1, seq_hi1;
+  seq_bounds(p, i0, seq_lo0, seq_hi0);
+  seq_bounds(p, last_row, seq_lo1, seq_hi1);
+  const int key_lo = max(seq_lo0, p.wl < 0 ? 0 : i0 - p.wl);
+  const int key_hi = min(seq_hi1, p.wr < 0 ? N : last_row + p.wr + 1);  // exclusive
   const int first_tile = key_lo / BN;
   const int ntiles = (key_hi - 1) / BN - first_tile + 1;
   const int nsteps = OP == RowOp::Fwd ? 2 * ntiles : ntiles;
@@ -556,9 +578,13 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
     const int r = 32 * (warp & 3) + (tid & 31);  // stationary row in the block
     const int gi = i0 + r;
     const bool row_ok = gi < N;
-    // this row's valid keys [jlo, jhi): its band, capped at N (none past N)
-    const int jlo = !row_ok ? 0 : (p.wl < 0 ? 0 : gi - p.wl);
-    const int jhi = !row_ok ? 0 : (p.wr < 0 ? N : min(N, gi + p.wr + 1));
+    // this row's valid keys [jlo, jhi): its band within its sequence (none past N)
+    int jlo = 0, jhi = 0;
+    if (row_ok) {
+      seq_bounds(p, gi, jlo, jhi);
+      if (p.wl >= 0) jlo = max(jlo, gi - p.wl);
+      if (p.wr >= 0) jhi = min(jhi, gi + p.wr + 1);
+    }
     const uint32_t ta = lane_base_addr(tmem, warp);
     const size_t rowoff = ((size_t)bh * N + (size_t)(row_ok ? gi : 0)) * D;
     const float tau = p.scale;
@@ -956,9 +982,13 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
   const int j0 = cb * BM;
   // streamed query tiles: rows whose band holds a key of this block,
   // j - wr <= i <= j + wl (negative w: unbounded; causal: wr = 0)
+  // (within the keys' packed sequences)
   const int last_key = min(j0 + BM, N) - 1;
-  const int q_lo = p.wr < 0 ? 0 : max(0, j0 - p.wr);
-  const int q_hi = p.wl < 0 ? N : min(N, last_key + p.wl + 1);  // exclusive
+  int seq_lo0, seq_hi0, seq_lo1, seq_hi1;
+  seq_bounds(p, j0, seq_lo0, seq_hi0);
+  seq_bounds(p, last_key, seq_lo1, seq_hi1);
+  const int q_lo = max(seq_lo0, p.wr < 0 ? 0 : j0 - p.wr);
+  const int q_hi = min(seq_hi1, p.wl < 0 ? N : last_key + p.wl + 1);  // exclusive
   const int first_tile = q_lo / BN;
   const int nsteps = (q_hi - 1) / BN - first_tile + 1;
 
@@ -1225,9 +1255,13 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
     const int r = 32 * (warp & 3) + (tid & 31);
     const int gj = j0 + r;  // stationary key row
     const bool row_ok = gj < N;
-    // query rows that see this key: [qlo, qhi) (none for a key past N)
-    const int qlo = !row_ok ? 0 : (p.wr < 0 ? 0 : gj - p.wr);
-    const int qhi = !row_ok ? 0 : (p.wl < 0 ? N : min(N, gj + p.wl + 1));
+    // query rows that see this key: [qlo, qhi), within its sequence (none past N)
+    int qlo = 0, qhi = 0;
+    if (row_ok) {
+      seq_bounds(p, gj, qlo, qhi);
+      if (p.wr >= 0) qlo = max(qlo, gj - p.wr);
+      if (p.wl >= 0) qhi = min(qhi, gj + p.wl + 1);
+    }
     const uint32_t ta = lane_base_addr(tmem, warp);
     const float tau = p.scale;
     const float2 sl2v = splat(tau * kLog2e), tauv = splat(tau);

@@ -65,6 +65,10 @@ int check_shape(const fbob_shape* s, bool* empty) {
   if (!(std::isfinite(s->scale) && s->scale > 0.f)) return FBOB_ERR_INVALID_ARGUMENT;
   if (s->causal != 0 && s->causal != 1) return FBOB_ERR_INVALID_ARGUMENT;
   if (s->window_left < -1 || s->window_right < -1) return FBOB_ERR_INVALID_ARGUMENT;
+  if (s->seq_offsets == nullptr ? s->num_seqs != 0
+                                : (s->num_seqs < 1 || s->num_seqs > kMaxN ||
+                                   (reinterpret_cast<uintptr_t>(s->seq_offsets) & 3u) != 0))
+    return FBOB_ERR_INVALID_ARGUMENT;
   if (s->d != 64 && s->d != 128) return FBOB_ERR_UNSUPPORTED;
   if (s->N > kMaxN) return FBOB_ERR_INVALID_ARGUMENT;
   if (s->B > kMaxBH || s->H > kMaxBH || s->B * s->H > kMaxBH) return FBOB_ERR_INVALID_ARGUMENT;
@@ -122,6 +126,8 @@ EngineParams base_params(const fbob_shape* s) {
   p.causal = s->causal;
   p.wl = s->window_left;
   p.wr = s->causal ? 0 : s->window_right;
+  p.seq_off = s->seq_offsets;
+  p.nseq = (int)s->num_seqs;
   p.scale = s->scale;
   p.bhn = s->B * s->H * s->N;
   debug_controls(&p);

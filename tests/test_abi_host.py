@@ -120,3 +120,13 @@ def test_rejects_bad_windows(lib):
     # valid windows pass validation (then stop at the empty problem, no CUDA call)
     assert bob(lib, S(1, 1, 0, 64, 0.125, 0, window=(3, 4)), ptrs(14)) == 0
     assert bob(lib, S(1, 1, 0, 64, 0.125, 1, window=(0, -1)), ptrs(14)) == 0
+
+
+def test_rejects_bad_sequence_offsets(lib):
+    def shape(seq, nseq, N=128):
+        return fbob.fbob_shape(1, 1, N, 64, 0.125, 0, -1, -1, seq, nseq)
+    assert bob(lib, shape(None, 3), ptrs(14)) == 1               # count without offsets
+    assert bob(lib, shape(BASE, 0), ptrs(14)) == 1               # offsets without a count
+    assert bob(lib, shape(BASE + 2, 2), ptrs(14)) == 1           # misaligned offsets
+    assert bob(lib, shape(BASE, (1 << 24) + 1), ptrs(14)) == 1   # more sequences than N allows
+    assert bob(lib, shape(BASE, 2, N=0), ptrs(14)) == 0          # valid: empty problem, no call
