@@ -49,7 +49,7 @@ def bob_flops(w, contractions=19):
     """2 * contractions * B*H*N^2*d*rho: rho = 1/2 exactly for the causal mask
     and 1 without one (the fixed formula); with a sliding window rho is the
     exact fraction of valid (i, j) pairs."""
-    if w.window != (-1, -1):
+    if w.window != (-1, -1) or w.segments:
         rho = synth.band_pairs(w) / float(w.N) ** 2
     else:
         rho = 0.5 if w.causal else 1.0
@@ -154,12 +154,15 @@ def oracle_sample(w, bits_head, target_s, seed=0):
     X = [synth.to_f64(bits_head[n]) for n in synth.NAMES]
     rows_probe = np.linspace(0, w.N - 1, 16).astype(np.int64)
     t0 = time.perf_counter()
-    oracle.bob_head(*X, w.scale, w.causal, rows=rows_probe, cols=(0, w.N), window=w.window)
+    seg = list(w.segments) or None
+    oracle.bob_head(*X, w.scale, w.causal, rows=rows_probe, cols=(0, w.N), window=w.window,
+                    segments=seg)
     dt = time.perf_counter() - t0
     n = int(max(16, min(w.N, 16 * target_s / max(dt, 1e-6))))
     rows = np.unique(np.linspace(0, w.N - 1, n).astype(np.int64))
     t0 = time.perf_counter()
-    oracle.bob_head(*X, w.scale, w.causal, rows=rows, cols=(0, w.N), window=w.window)
+    oracle.bob_head(*X, w.scale, w.causal, rows=rows, cols=(0, w.N), window=w.window,
+                    segments=seg)
     dt = time.perf_counter() - t0
     flops = 2.0 * 19 * valid_pairs_rows(w, rows) * w.d
     return flops, dt, f"{len(rows)} evenly spaced query rows of head 0 (of {w.N}), all key columns"
@@ -224,8 +227,10 @@ def run_gpu(args, w):
     dev = {n: torch.from_numpy(bits[n].view(np.int16)).view(torch.bfloat16).cuda()
            for n in synth.NAMES}
     q, k, v, do, gq, gk, gv = (dev[n] for n in synth.NAMES)
-    o, lse = fbob.attn_fwd(q, k, v, w.scale, w.causal, w.window)
-    shp = fbob.make_shape(w.B, w.H, w.N, w.d, w.scale, w.causal, w.window)
+    segs = (torch.tensor(w.segments, dtype=torch.int32, device="cuda") if w.segments
+            else None)  # packed-sequence offsets (kept alive for every call below)
+    o, lse = fbob.attn_fwd(q, k, v, w.scale, w.causal, w.window, segs)
+    shp = fbob.make_shape(w.B, w.H, w.N, w.d, w.scale, w.causal, w.window, segs)
     outs = [torch.empty_like(q) for _ in range(4)]
     rs = torch.empty((3, w.B, w.H, w.N), dtype=torch.float32, device="cuda")
     torch.cuda.synchronize()
@@ -358,11 +363,12 @@ def run_gpu(args, w):
         "warmup": args.warmup, "ms_per_step": ms_max / K, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": w.name, "B": w.B, "H": w.H, "N": w.N, "d": w.d,
-                   "causal": w.causal, "window": list(w.window), "seed": w.seed,
+                   "causal": w.causal, "window": list(w.window),
+                   "packed_sequences": len(w.segments) - 1 if w.segments else 1, "seed": w.seed,
                    "l2": "no flush: inputs (%.2f GB) exceed the 129 MB L2" % (footprint / 1e9),
                    "parallelism": "replicas" if world > 1 else "single GPU",
                    "flop_formula": ("2*19*B*H*d*(valid (i,j) pairs of the band)"
-                                    if w.window != (-1, -1)
+                                    if w.window != (-1, -1) or w.segments
                                     else "2*19*B*H*N^2*d*(1/2 if causal)")},
         "frac_of_bf16_peak": value / world / peak,
         "roofline": roofline,
@@ -397,8 +403,10 @@ def run_gpu_op(args, w):
     dev = {n: torch.from_numpy(bits[n].view(np.int16)).view(torch.bfloat16).cuda()
            for n in ("q", "k", "v", "dout")}
     q, k, v, do = dev["q"], dev["k"], dev["v"], dev["dout"]
-    shp = fbob.make_shape(w.B, w.H, w.N, w.d, w.scale, w.causal, w.window)
-    o, lse = fbob.attn_fwd(q, k, v, w.scale, w.causal, w.window)
+    segs = (torch.tensor(w.segments, dtype=torch.int32, device="cuda") if w.segments
+            else None)
+    shp = fbob.make_shape(w.B, w.H, w.N, w.d, w.scale, w.causal, w.window, segs)
+    o, lse = fbob.attn_fwd(q, k, v, w.scale, w.causal, w.window, segs)
     dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
     dstat = torch.empty_like(lse)
     if args.op == "fwd":

@@ -34,6 +34,7 @@ class Workload:
     seed: int
     sigma: tuple  # per tensor in NAMES order
     window: tuple = (-1, -1)  # sliding-window band (left, right); -1 = unbounded
+    segments: tuple = ()      # offsets of packed sequences along N; () = one sequence
 
     @property
     def scale(self) -> float:
@@ -67,6 +68,23 @@ WORKLOADS = {
 }
 
 
+def packed_offsets(N: int, n: int, seed: int) -> tuple:
+    """Offsets of n packed sequences filling N: seeded lengths drawn
+    uniformly between N/(4n) and 7N/(4n), rescaled to sum to N."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    lens = rng.uniform(0.25, 1.75, n)
+    cuts = np.round(np.cumsum(lens) / lens.sum() * N).astype(np.int64)
+    cuts[-1] = N
+    return tuple(int(x) for x in np.concatenate([[0], cuts]))
+
+
+# packed variable-length variant of n16k_d128_causal: 12 causal sequences of
+# seeded lengths (about 340 to 2400 tokens) in the 16K rows of each head
+WORKLOADS["n16k_d128_causal_varlen"] = Workload(
+    "n16k_d128_causal_varlen", 2, 16, 16384, 128, True, 6,
+    _s(1, 1, 1, *(4 * [1 / math.sqrt(128)])), segments=packed_offsets(16384, 12, 6))
+
+
 def band_pairs(w: Workload, rows=None) -> float:
     """Valid (i, j) pairs of the listed rows (all rows by default) under the
     workload's mask: the band i - wl <= j <= i + wr, capped at j <= i if causal."""
@@ -76,6 +94,11 @@ def band_pairs(w: Workload, rows=None) -> float:
     hi = np.full_like(r, w.N) if wr < 0 else np.minimum(w.N, r + wr + 1)
     if w.causal:
         hi = np.minimum(hi, r + 1)
+    if w.segments:
+        seg = np.asarray(w.segments, dtype=np.int64)
+        s = np.searchsorted(seg[1:], r, side="right")
+        lo = np.maximum(lo, seg[s])
+        hi = np.minimum(hi, seg[s + 1])
     return float(np.sum(hi - lo))
 
 

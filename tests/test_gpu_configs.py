@@ -153,3 +153,23 @@ def test_n16k_d128_causal_swa4k_rows_and_key_block():
     for hh, ref in zip(heads, blk):
         G.check("kbar[block]", G.flat(r["kbar"], hh, w.H)[c0:c1], ref["kbar"])
         G.check("vbar[block]", G.flat(r["vbar"], hh, w.H)[c0:c1], ref["vbar"])
+
+
+def test_n16k_d128_causal_varlen_rows_and_sequence():
+    """Packed sequences at full size: sampled rows, and the key columns of one
+    whole sequence (complete once that sequence's rows are summed)."""
+    w = synth.WORKLOADS["n16k_d128_causal_varlen"]
+    seg = list(w.segments)
+    bits = synth.workload_inputs(w)
+    r = G.run_bob(bits, w.scale, w.causal, segments=seg)
+    assert r["status"] == 0
+    heads = [9]
+    rows = sample_rows(w.N, 66)
+    check_rows(r, G.oracle_bob_heads(bits, w.scale, w.causal, heads, rows=rows, segments=seg),
+               heads, w.H, rows)
+    a, b = seg[5], seg[6]
+    blk = G.oracle_bob_heads(bits, w.scale, w.causal, heads, rows=np.arange(a, b), cols=(a, b),
+                             segments=seg)
+    for hh, ref in zip(heads, blk):
+        G.check("kbar[sequence]", G.flat(r["kbar"], hh, w.H)[a:b], ref["kbar"])
+        G.check("vbar[sequence]", G.flat(r["vbar"], hh, w.H)[a:b], ref["vbar"])
