@@ -86,6 +86,13 @@ def _segments(segments, N):
     return seg, seg.size - 1
 
 
+def _group(H, Hkv):
+    """Query heads per key/value head (grouped-query attention: query head h
+    reads key/value head h // G)."""
+    assert Hkv >= 1 and H % Hkv == 0, (H, Hkv)
+    return H // Hkv
+
+
 def _heads(x):
     x = np.asarray(x)
     if x.ndim == 2:
@@ -100,6 +107,7 @@ def fwd(q, k, v, scale, causal, nthreads=0, window=None, segments=None):
     wl, wr = _window(window)
     q, k, v = (_c(_heads(t)) for t in (q, k, v))
     B, H, N, d = q.shape
+    G = _group(H, k.shape[1])
     seg, nseg = _segments(segments, N)
     lib = _load()
     O = np.zeros_like(q)
@@ -107,9 +115,10 @@ def fwd(q, k, v, scale, causal, nthreads=0, window=None, segments=None):
     for b in range(B):
         for h in range(H):
             o_ = np.zeros((N, d)); l_ = np.zeros(N)
+            hk = h // G
             rc = lib.fbob_oracle_fwd(N, d, float(scale), int(bool(causal)), wl, wr,
                                      _ptr(seg), nseg,
-                                     _ptr(_c(q[b, h])), _ptr(_c(k[b, h])), _ptr(_c(v[b, h])),
+                                     _ptr(_c(q[b, h])), _ptr(_c(k[b, hk])), _ptr(_c(v[b, hk])),
                                      _ptr(o_), _ptr(l_), int(nthreads))
             assert rc == 0, rc
             O[b, h], L[b, h] = o_, l_
@@ -117,24 +126,30 @@ def fwd(q, k, v, scale, causal, nthreads=0, window=None, segments=None):
 
 
 def bwd(q, k, v, dout, scale, causal, nthreads=0, window=None, segments=None):
-    """First backward (eqs. 2-3).  Returns dQ, dK, dV [B,H,N,d] and D [B,H,N]."""
+    """First backward (eqs. 2-3).  Returns dQ [B,H,N,d], dK, dV [B,Hkv,N,d] and
+    D [B,H,N]; with grouped-query attention (k, v with Hkv < H heads) dK and dV
+    of a key/value head are the sums over its query heads."""
     wl, wr = _window(window)
     q, k, v, dout = (_c(_heads(t)) for t in (q, k, v, dout))
     B, H, N, d = q.shape
+    G = _group(H, k.shape[1])
     seg, nseg = _segments(segments, N)
     lib = _load()
-    outs = [np.zeros_like(q) for _ in range(3)]
+    outs = [np.zeros_like(q), np.zeros_like(k), np.zeros_like(v)]
     D = np.zeros((B, H, N))
     for b in range(B):
         for h in range(H):
+            hk = h // G
             dq, dk, dv, dd = np.zeros((N, d)), np.zeros((N, d)), np.zeros((N, d)), np.zeros(N)
             rc = lib.fbob_oracle_bwd(N, d, float(scale), int(bool(causal)), wl, wr,
                                      _ptr(seg), nseg,
-                                     _ptr(_c(q[b, h])), _ptr(_c(k[b, h])), _ptr(_c(v[b, h])),
+                                     _ptr(_c(q[b, h])), _ptr(_c(k[b, hk])), _ptr(_c(v[b, hk])),
                                      _ptr(_c(dout[b, h])), _ptr(dq), _ptr(dk), _ptr(dv),
                                      _ptr(dd), int(nthreads))
             assert rc == 0, rc
-            outs[0][b, h], outs[1][b, h], outs[2][b, h], D[b, h] = dq, dk, dv, dd
+            outs[0][b, h], D[b, h] = dq, dd
+            outs[1][b, hk] += dk
+            outs[2][b, hk] += dv
     return outs[0], outs[1], outs[2], D
 
 
@@ -185,19 +200,31 @@ def bob(q, k, v, dout, gq, gk, gv, scale, causal, nthreads=0, mutant=0, mutant_d
     """Full backward-over-backward on [B,H,N,d] (or [N,d]) float64 arrays.
 
     Returns (qbar, kbar, vbar, dobar, alpha, E, D) with the input's batch shape.
+    Grouped-query attention: k, v, gk, gv may have Hkv < H heads (query head h
+    reads head h // (H / Hkv)).  Phi then splits into one term per query head,
+    each using its key/value head's tensors, so kbar and vbar of a key/value
+    head are the sums of the per-query-head results over its group.
     """
     ts = [_c(_heads(t)) for t in (q, k, v, dout, gq, gk, gv)]
     B, H, N, d = ts[0].shape
-    out = {n: np.zeros((B, H, N, d)) for n in ("qbar", "kbar", "vbar", "dobar")}
+    Hkv = ts[1].shape[1]
+    G = _group(H, Hkv)
+    out = {n: np.zeros((B, H, N, d)) for n in ("qbar", "dobar")}
+    for n in ("kbar", "vbar"):
+        out[n] = np.zeros((B, Hkv, N, d))
     for n in ("alpha", "E", "D"):
         out[n] = np.zeros((B, H, N))
+    kv_side = (1, 2, 5, 6)  # k, v, gk, gv
     for b in range(B):
         for h in range(H):
-            r = bob_head(*(t[b, h] for t in ts), scale, causal, nthreads=nthreads,
+            args = [t[b, h // G] if i in kv_side else t[b, h] for i, t in enumerate(ts)]
+            r = bob_head(*args, scale, causal, nthreads=nthreads,
                          mutant=mutant, mutant_dir=mutant_dir, window=window,
                          segments=segments)
-            for n in ("qbar", "kbar", "vbar", "dobar", "alpha", "E", "D"):
+            for n in ("qbar", "dobar", "alpha", "E", "D"):
                 out[n][b, h] = r[n]
+            out["kbar"][b, h // G] += r["kbar"]
+            out["vbar"][b, h // G] += r["vbar"]
     return (out["qbar"], out["kbar"], out["vbar"], out["dobar"],
             out["alpha"], out["E"], out["D"])
 
