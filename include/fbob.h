@@ -37,6 +37,12 @@
  *             that break these rules give unspecified values but no access
  *             outside the caller's buffers.  NULL (with num_seqs 0) is one
  *             sequence.
+ *  GQA        H_kv > 0 (a divisor of H) gives grouped-query attention: the
+ *             key/value-side tensors (k, v, gk, gv and k_bar, v_bar, dk, dv)
+ *             are [B, H_kv, N, d] and query head h reads key/value head
+ *             h / (H / H_kv).  dK, dV, k_bar and v_bar of a key/value head are
+ *             then sums over its H / H_kv query heads, summed inside one CTA in
+ *             a fixed order.  Query-side tensors and row vectors keep H heads.
  *  Stream     Every call enqueues its kernels on `stream` (NULL = legacy
  *             default stream) and returns without synchronising.
  *  Memory     The library allocates and frees no device memory.  The caller
@@ -85,6 +91,7 @@ typedef struct fbob_shape {
     int32_t window_right; /* and j <= i + window_right; -1 = unbounded (causal caps it at 0) */
     const int32_t* seq_offsets; /* packed sequences: device int32 [num_seqs + 1], or NULL */
     int64_t num_seqs;           /* number of packed sequences (0 when seq_offsets is NULL) */
+    int64_t H_kv; /* key/value heads (grouped-query attention); 0 = H */
 } fbob_shape;
 
 /*

@@ -33,7 +33,8 @@ class fbob_shape(ctypes.Structure):
     _fields_ = [("B", ctypes.c_int64), ("H", ctypes.c_int64), ("N", ctypes.c_int64),
                 ("d", ctypes.c_int64), ("scale", ctypes.c_float), ("causal", ctypes.c_int32),
                 ("window_left", ctypes.c_int32), ("window_right", ctypes.c_int32),
-                ("seq_offsets", ctypes.c_void_p), ("num_seqs", ctypes.c_int64)]
+                ("seq_offsets", ctypes.c_void_p), ("num_seqs", ctypes.c_int64),
+                ("H_kv", ctypes.c_int64)]
 
 
 _lib = None
@@ -80,11 +81,13 @@ def header_symbols() -> list:
     return sorted(set(re.findall(r"^\s*(?:const\s+)?\w+\**\s+\**(fbob_\w+)\s*\(", text, re.M)))
 
 
-def make_shape(B, H, N, d, scale, causal, window=None, segments=None) -> fbob_shape:
+def make_shape(B, H, N, d, scale, causal, window=None, segments=None,
+               kv_heads=None) -> fbob_shape:
     """window: (left, right) sliding-window band i - left <= j <= i + right;
     -1 (or None) leaves a side unbounded.  segments: contiguous int32 CUDA
     tensor of packed-sequence offsets [num_seqs + 1] (it must stay alive
-    until the calls using this shape have run), or None for one sequence."""
+    until the calls using this shape have run), or None for one sequence.
+    kv_heads: key/value heads for grouped-query attention (None: H)."""
     wl, wr = (-1, -1) if window is None else (int(window[0]), int(window[1]))
     if segments is None:
         seg, nseg = None, 0
@@ -94,8 +97,9 @@ def make_shape(B, H, N, d, scale, causal, window=None, segments=None) -> fbob_sh
                 or not segments.is_contiguous()):
             raise ValueError("segments must be a contiguous 1-D int32 CUDA tensor")
         seg, nseg = segments.data_ptr(), segments.numel() - 1
+    hkv = 0 if kv_heads is None or int(kv_heads) == int(H) else int(kv_heads)
     return fbob_shape(int(B), int(H), int(N), int(d), float(scale), int(causal), wl, wr,
-                      seg, nseg)
+                      seg, nseg, hkv)
 
 
 def _ptr(t):
@@ -120,9 +124,9 @@ def _check(rc, where):
         raise FbobError(rc, where)
 
 
-def _shape_of(q, scale, causal, window=None, segments=None):
+def _shape_of(q, k, scale, causal, window=None, segments=None):
     B, H, N, d = q.shape
-    return make_shape(B, H, N, d, scale, causal, window, segments)
+    return make_shape(B, H, N, d, scale, causal, window, segments, kv_heads=k.shape[1])
 
 
 # ------------------------------------------------ entry points, same names as the C ABI
@@ -190,7 +194,7 @@ def attn_fwd(q, k, v, scale, causal, window=None, segments=None):
     B, H, N, d = q.shape
     o = torch.empty_like(q)
     lse = torch.empty((B, H, N), dtype=torch.float32, device=q.device)
-    fbob_attn_fwd(_shape_of(q, scale, causal, window, segments), q, k, v, o, lse)
+    fbob_attn_fwd(_shape_of(q, k, scale, causal, window, segments), q, k, v, o, lse)
     return o, lse
 
 
@@ -199,8 +203,8 @@ def attn_bwd(q, k, v, o, lse, dout, scale, causal, window=None, segments=None):
     B, H, N, d = q.shape
     dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
     dstat = torch.empty((B, H, N), dtype=torch.float32, device=q.device)
-    fbob_attn_bwd(_shape_of(q, scale, causal, window, segments), q, k, v, o, lse, dout, dq, dk,
-                  dv, dstat)
+    fbob_attn_bwd(_shape_of(q, k, scale, causal, window, segments), q, k, v, o, lse, dout, dq,
+                  dk, dv, dstat)
     return dq, dk, dv, dstat
 
 
@@ -208,8 +212,8 @@ def attn_bob(q, k, v, o, lse, dout, gq, gk, gv, scale, causal, window=None, segm
     """Returns (q_bar, k_bar, v_bar, dout_bar, row_stats[3,B,H,N] = alpha, E, D)."""
     import torch
     B, H, N, d = q.shape
-    outs = [torch.empty_like(q) for _ in range(4)]
+    outs = [torch.empty_like(q), torch.empty_like(k), torch.empty_like(v), torch.empty_like(q)]
     row_stats = torch.empty((3, B, H, N), dtype=torch.float32, device=q.device)
-    fbob_attn_bob(_shape_of(q, scale, causal, window, segments), q, k, v, o, lse, dout, gq, gk,
-                  gv, *outs, row_stats)
+    fbob_attn_bob(_shape_of(q, k, scale, causal, window, segments), q, k, v, o, lse, dout, gq,
+                  gk, gv, *outs, row_stats)
     return (*outs, row_stats)

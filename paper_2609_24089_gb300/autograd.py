@@ -43,7 +43,8 @@ class _AttnBwd(torch.autograd.Function):
     @staticmethod
     def backward(ctx, gq, gk, gv):
         q, k, v, o, lse, dout = ctx.saved_tensors
-        g = [torch.zeros_like(q) if t is None else _bf16(t) for t in (gq, gk, gv)]
+        g = [torch.zeros_like(x) if t is None else _bf16(t)
+             for t, x in zip((gq, gk, gv), (q, k, v))]
         q_bar, k_bar, v_bar, dout_bar, _ = attn_bob(q, k, v, o, lse, dout, *g, ctx.scale,
                                                     ctx.causal, ctx.window, ctx.segments)
         return q_bar, k_bar, v_bar, None, None, dout_bar, None, None, None, None

@@ -215,6 +215,8 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
   const int rbi = p.head_major ? lin % p.nblk : lin / p.BH;
   const int bh = p.head_major ? lin / p.nblk : lin % p.BH;
   const int rb = p.causal ? (p.nblk - 1 - rbi) : rbi;
+  // key/value head of this query head (grouped-query attention: h / (H / Hkv))
+  const int bh_kv = p.Hkv == p.H ? bh : (bh / p.H) * p.Hkv + (bh % p.H) / (p.H / p.Hkv);
   const int i0 = rb * BM;
   const int last_row = min(i0 + BM, N) - 1;
   // streamed key tiles: those overlapping the rows' bands [i - wl, i + wr]
@@ -294,14 +296,14 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         for (int b = 0; b < C::KB; ++b)
           for (int t = 0; t < nt_a; ++t)
             tma_load_3d(dst + soff<C::NSTREAM, kB4>(t, 0, b), &p.tm[C::NSTAT + t],
-                        &m->bar_full[stage], 64 * b, j0, bh);
+                        &m->bar_full[stage], 64 * b, j0, bh_kv);
         if (kB4) {  // 32-row chunks (map box rows HB)
           mbar_arrive_expect_tx(&m->bar_full_b[stage], 2 * C::KB * BN * 128);
           for (int b = 0; b < C::KB; ++b)
             for (int t = 2; t < 4; ++t)
               for (int h = 0; h < 2; ++h)
                 tma_load_3d(dst + soff<C::NSTREAM, kB4>(t, h, b), &p.tm[C::NSTAT + t],
-                            &m->bar_full_b[stage], 64 * b, j0 + HB * h, bh);
+                            &m->bar_full_b[stage], 64 * b, j0 + HB * h, bh_kv);
         }
         issued[stage] = st;
       }
@@ -990,7 +992,12 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
   const int q_lo = max(seq_lo0, p.wr < 0 ? 0 : j0 - p.wr);
   const int q_hi = min(seq_hi1, p.wl < 0 ? N : last_key + p.wl + 1);  // exclusive
   const int first_tile = q_lo / BN;
-  const int nsteps = (q_hi - 1) / BN - first_tile + 1;
+  const int nsteps_h = (q_hi - 1) / BN - first_tile + 1;  // query tiles per query head
+  // grouped-query attention: this key/value head's G query heads are streamed
+  // one after the other (their sums accumulate in this CTA, in a fixed order)
+  const int G = p.H / p.Hkv;
+  const int bh_q0 = (bh / p.Hkv) * p.H + (bh % p.Hkv) * G;  // first query head
+  const int nsteps = G * nsteps_h;
 
   if (tid == 0) {
     m->wctl.abort = 0;
@@ -1043,7 +1050,8 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
       if (st >= C::NSTAGES) {
         if (!mbar_wait(&m->bar_empty[stage], ((st / C::NSTAGES) - 1) & 1, wctl)) break;
       }
-      const int ib = (first_tile + st) * BN;
+      const int ib = (first_tile + st % nsteps_h) * BN;
+      const int bhq = bh_q0 + st / nsteps_h;  // query head of this step
       uint8_t* dst = s_stream + stage * C::STAGE_BYTES;
       if (lane == 0) {
         // Q (and U_Q) first on bar_full, dO on bar_full_b
@@ -1052,11 +1060,11 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
         for (int b = 0; b < C::KB; ++b)
           for (int t = 0; t < na; ++t)
             tma_load_3d(dst + soff<C::NSTREAM, false>(t, 0, b), &p.tm[C::NSTAT + t],
-                        &m->bar_full[stage], 64 * b, ib, bh);
+                        &m->bar_full[stage], 64 * b, ib, bhq);
         mbar_arrive_expect_tx(&m->bar_full_b[stage], C::KB * BN * 128);
         for (int b = 0; b < C::KB; ++b)
           tma_load_3d(dst + soff<C::NSTREAM, false>(na, 0, b), &p.tm[C::NSTAT + na],
-                      &m->bar_full_b[stage], 64 * b, ib, bh);
+                      &m->bar_full_b[stage], 64 * b, ib, bhq);
       }
       // negated row vectors of the streamed query rows:
       // [0] -L*log2e, [1] -D, [2] -alpha, [3] -E
@@ -1066,7 +1074,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
         const int c = lane + 32 * q;
         const int gi = ib + c;
         const bool ok = gi < N;
-        const size_t ri = (size_t)bh * N + (ok ? gi : 0);
+        const size_t ri = (size_t)bhq * N + (ok ? gi : 0);
         vec[c] = ok ? -p.lse[ri] * kLog2e : 0.f;
         if constexpr (OP == ColOp::BwdDKDV) {
           vec[64 + c] = ok ? -p.vec_in[ri] : 0.f;
@@ -1301,7 +1309,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
 #pragma unroll
       for (int h = 0; h < 2; ++h) {
         const int cv = HB * h + 16 * wg;             // tile column of this thread's first
-        const int ib = (first_tile + st) * BN + cv;  // first query row of this thread's 16
+        const int ib = (first_tile + st % nsteps_h) * BN + cv;  // first query row of this thread's 16
         // valid query columns c satisfy  lo <= c < hi
         const int lo = qlo - ib, hi = qhi - ib;
         const bool need_mask = lo > 0 || hi < 16;

@@ -50,6 +50,7 @@ struct EngineParams {
   int wl, wr;  // valid band of row i: i - wl <= j <= i + wr (-1: unbounded); causal gives wr = 0
   const int* seq_off;  // packed sequences: offsets [nseq + 1], or nullptr for one sequence
   int nseq;
+  int H, Hkv;  // query and key/value heads per batch entry (grouped-query attention)
   float scale;
   long long bhn;  // BH * N (row_stats plane stride)
   unsigned long long wait_limit_ns;  // bound of every device-side wait

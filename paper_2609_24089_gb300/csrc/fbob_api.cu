@@ -65,6 +65,7 @@ int check_shape(const fbob_shape* s, bool* empty) {
   if (!(std::isfinite(s->scale) && s->scale > 0.f)) return FBOB_ERR_INVALID_ARGUMENT;
   if (s->causal != 0 && s->causal != 1) return FBOB_ERR_INVALID_ARGUMENT;
   if (s->window_left < -1 || s->window_right < -1) return FBOB_ERR_INVALID_ARGUMENT;
+  if (s->H_kv < 0 || (s->H_kv > 0 && (s->H % s->H_kv) != 0)) return FBOB_ERR_INVALID_ARGUMENT;
   if (s->seq_offsets == nullptr ? s->num_seqs != 0
                                 : (s->num_seqs < 1 || s->num_seqs > kMaxN ||
                                    (reinterpret_cast<uintptr_t>(s->seq_offsets) & 3u) != 0))
@@ -118,6 +119,9 @@ void debug_controls(EngineParams* p) {
 // kernels balance the causal work better with heads innermost.
 void choose_order(EngineParams* p, int head_major) { p->head_major = head_major; }
 
+// key/value heads per batch entry
+int64_t kv_heads(const fbob_shape* s) { return s->H_kv > 0 ? s->H_kv : s->H; }
+
 EngineParams base_params(const fbob_shape* s) {
   EngineParams p;
   std::memset(&p, 0, sizeof(p));
@@ -128,6 +132,8 @@ EngineParams base_params(const fbob_shape* s) {
   p.wr = s->causal ? 0 : s->window_right;
   p.seq_off = s->seq_offsets;
   p.nseq = (int)s->num_seqs;
+  p.H = (int)s->H;
+  p.Hkv = (int)kv_heads(s);
   p.scale = s->scale;
   p.bhn = s->B * s->H * s->N;
   debug_controls(&p);
@@ -152,8 +158,9 @@ bool row_bob_params(const fbob_shape* s, const void* q, const void* k, const voi
   const void* strm[4] = {k, gk, v, gv};
   for (int t = 0; t < 3; ++t)
     if (!make_map(&p->tm[t], stat[t], BH, N, d, BM)) return false;
+  const int64_t BHk = s->B * kv_heads(s);
   for (int t = 0; t < 4; ++t)
-    if (!make_map(&p->tm[3 + t], strm[t], BH, N, d, t < 2 ? BN : HB)) return false;
+    if (!make_map(&p->tm[3 + t], strm[t], BHk, N, d, t < 2 ? BN : HB)) return false;
   p->q = static_cast<const __nv_bfloat16*>(q);
   p->uq = static_cast<const __nv_bfloat16*>(gq);
   p->o = static_cast<const __nv_bfloat16*>(o);
@@ -209,8 +216,10 @@ int run_pass2(const fbob_shape* s, const void* q, const void* k, const void* v, 
   const int64_t BH = s->B * s->H, N = s->N, d = s->d;
   const void* stat[4] = {k, v, gk, gv};
   const void* strm[3] = {q, gq, dout};
+  const int64_t BHk = s->B * kv_heads(s);
+  p.BH = (int)BHk;  // one CTA column per key/value head
   for (int t = 0; t < 4; ++t)
-    if (!make_map(&p.tm[t], stat[t], BH, N, d, BM)) return FBOB_ERR_CUDA;
+    if (!make_map(&p.tm[t], stat[t], BHk, N, d, BM)) return FBOB_ERR_CUDA;
   for (int t = 0; t < 3; ++t)
     if (!make_map(&p.tm[4 + t], strm[t], BH, N, d, BN)) return FBOB_ERR_CUDA;
   p.lse = lse;
@@ -261,16 +270,17 @@ int fbob_attn_fwd(const fbob_shape* s, const void* q, const void* k, const void*
     return FBOB_OK;
   }
   const int64_t mat = s->B * s->H * s->N * s->d * 2, vec = s->B * s->H * s->N * 4;
+  const int64_t matk = s->B * kv_heads(s) * s->N * s->d * 2;
   const void* in[3] = {q, k, v};
-  const int64_t inb[3] = {mat, mat, mat};
+  const int64_t inb[3] = {mat, matk, matk};
   void* out[2] = {o, lse};
   const int64_t outb[2] = {mat, vec};
   rc = check_ptrs(in, inb, 3, out, outb, 2);
   if (rc != FBOB_OK) return rc;
   EngineParams p = base_params(s);
-  const int64_t BH = s->B * s->H;
-  if (!make_map(&p.tm[0], q, BH, s->N, s->d, BM) || !make_map(&p.tm[1], k, BH, s->N, s->d, BN) ||
-      !make_map(&p.tm[2], v, BH, s->N, s->d, BN))
+  const int64_t BH = s->B * s->H, BHk = s->B * kv_heads(s);
+  if (!make_map(&p.tm[0], q, BH, s->N, s->d, BM) ||
+      !make_map(&p.tm[1], k, BHk, s->N, s->d, BN) || !make_map(&p.tm[2], v, BHk, s->N, s->d, BN))
     return FBOB_ERR_CUDA;
   p.out0 = static_cast<__nv_bfloat16*>(o);
   p.vec_out = lse;
@@ -292,17 +302,18 @@ int fbob_attn_bwd(const fbob_shape* s, const void* q, const void* k, const void*
     return FBOB_OK;
   }
   const int64_t mat = s->B * s->H * s->N * s->d * 2, vec = s->B * s->H * s->N * 4;
+  const int64_t matk = s->B * kv_heads(s) * s->N * s->d * 2;
   const void* in[6] = {q, k, v, o, lse, dout};
-  const int64_t inb[6] = {mat, mat, mat, mat, vec, mat};
+  const int64_t inb[6] = {mat, matk, matk, mat, vec, mat};
   void* out[4] = {dq, dk, dv, dstat};
-  const int64_t outb[4] = {mat, mat, mat, vec};
+  const int64_t outb[4] = {mat, matk, matk, vec};
   rc = check_ptrs(in, inb, 6, out, outb, 4);
   if (rc != FBOB_OK) return rc;
-  const int64_t BH = s->B * s->H, N = s->N, d = s->d;
+  const int64_t BH = s->B * s->H, BHk = s->B * kv_heads(s), N = s->N, d = s->d;
   // dQ and D: row-block pass (writes D, which the column pass reads)
   EngineParams p = base_params(s);
   if (!make_map(&p.tm[0], q, BH, N, d, BM) || !make_map(&p.tm[1], dout, BH, N, d, BM) ||
-      !make_map(&p.tm[2], k, BH, N, d, BN) || !make_map(&p.tm[3], v, BH, N, d, BN))
+      !make_map(&p.tm[2], k, BHk, N, d, BN) || !make_map(&p.tm[3], v, BHk, N, d, BN))
     return FBOB_ERR_CUDA;
   p.o = static_cast<const __nv_bfloat16*>(o);
   p.dout = static_cast<const __nv_bfloat16*>(dout);
@@ -315,7 +326,8 @@ int fbob_attn_bwd(const fbob_shape* s, const void* q, const void* k, const void*
   if (rc != FBOB_OK) return rc;
   // dK and dV: column-block pass
   EngineParams c = base_params(s);
-  if (!make_map(&c.tm[0], k, BH, N, d, BM) || !make_map(&c.tm[1], v, BH, N, d, BM) ||
+  c.BH = (int)BHk;  // one CTA column per key/value head
+  if (!make_map(&c.tm[0], k, BHk, N, d, BM) || !make_map(&c.tm[1], v, BHk, N, d, BM) ||
       !make_map(&c.tm[2], q, BH, N, d, BN) || !make_map(&c.tm[3], dout, BH, N, d, BN))
     return FBOB_ERR_CUDA;
   c.lse = lse;
@@ -341,8 +353,9 @@ int fbob_attn_bob_pass1(const fbob_shape* s, const void* q, const void* k, const
     return FBOB_OK;
   }
   const int64_t mat = s->B * s->H * s->N * s->d * 2, vec = s->B * s->H * s->N * 4;
+  const int64_t matk = s->B * kv_heads(s) * s->N * s->d * 2;
   const void* in[9] = {q, k, v, o, lse, dout, gq, gk, gv};
-  const int64_t inb[9] = {mat, mat, mat, mat, vec, mat, mat, mat, mat};
+  const int64_t inb[9] = {mat, matk, matk, mat, vec, mat, mat, matk, matk};
   void* out[3] = {q_bar, dout_bar, row_stats};
   const int64_t outb[3] = {mat, mat, 3 * vec};
   rc = check_ptrs(in, inb, 9, out, outb, 3);
@@ -364,11 +377,12 @@ int fbob_attn_bob_pass2(const fbob_shape* s, const void* q, const void* k, const
     return FBOB_OK;
   }
   const int64_t mat = s->B * s->H * s->N * s->d * 2, vec = s->B * s->H * s->N * 4;
+  const int64_t matk = s->B * kv_heads(s) * s->N * s->d * 2;
   // row_stats is an input of pass 2; check it with the inputs
   const void* in2[9] = {q, k, v, lse, dout, gq, gk, gv, row_stats};
-  const int64_t inb2[9] = {mat, mat, mat, vec, mat, mat, mat, mat, 3 * vec};
+  const int64_t inb2[9] = {mat, matk, matk, vec, mat, mat, matk, matk, 3 * vec};
   void* out[2] = {k_bar, v_bar};
-  const int64_t outb[2] = {mat, mat};
+  const int64_t outb[2] = {matk, matk};
   rc = check_ptrs(in2, inb2, 9, out, outb, 2);
   if (rc != FBOB_OK) return rc;
   rc = run_pass2(s, q, k, v, lse, dout, gq, gk, gv, row_stats, k_bar, v_bar, stream);
@@ -388,8 +402,9 @@ int fbob_attn_bob_row_stats(const fbob_shape* s, const void* q, const void* k, c
     return FBOB_OK;
   }
   const int64_t mat = s->B * s->H * s->N * s->d * 2, vec = s->B * s->H * s->N * 4;
+  const int64_t matk = s->B * kv_heads(s) * s->N * s->d * 2;
   const void* in[9] = {q, k, v, o, lse, dout, gq, gk, gv};
-  const int64_t inb[9] = {mat, mat, mat, mat, vec, mat, mat, mat, mat};
+  const int64_t inb[9] = {mat, matk, matk, mat, vec, mat, mat, matk, matk};
   void* out[1] = {row_stats};
   const int64_t outb[1] = {3 * vec};
   rc = check_ptrs(in, inb, 9, out, outb, 1);
@@ -413,8 +428,9 @@ int fbob_attn_bob_pass1_direct(const fbob_shape* s, const void* q, const void* k
     return FBOB_OK;
   }
   const int64_t mat = s->B * s->H * s->N * s->d * 2, vec = s->B * s->H * s->N * 4;
+  const int64_t matk = s->B * kv_heads(s) * s->N * s->d * 2;
   const void* in[9] = {q, k, v, lse, dout, gq, gk, gv, row_stats};
-  const int64_t inb[9] = {mat, mat, mat, vec, mat, mat, mat, mat, 3 * vec};
+  const int64_t inb[9] = {mat, matk, matk, vec, mat, mat, matk, matk, 3 * vec};
   void* out[2] = {q_bar, dout_bar};
   const int64_t outb[2] = {mat, mat};
   rc = check_ptrs(in, inb, 9, out, outb, 2);
@@ -439,10 +455,11 @@ int fbob_attn_bob(const fbob_shape* s, const void* q, const void* k, const void*
     return FBOB_OK;
   }
   const int64_t mat = s->B * s->H * s->N * s->d * 2, vec = s->B * s->H * s->N * 4;
+  const int64_t matk = s->B * kv_heads(s) * s->N * s->d * 2;
   const void* in[9] = {q, k, v, o, lse, dout, gq, gk, gv};
-  const int64_t inb[9] = {mat, mat, mat, mat, vec, mat, mat, mat, mat};
+  const int64_t inb[9] = {mat, matk, matk, mat, vec, mat, mat, matk, matk};
   void* out[5] = {q_bar, k_bar, v_bar, dout_bar, row_stats};
-  const int64_t outb[5] = {mat, mat, mat, mat, 3 * vec};
+  const int64_t outb[5] = {mat, matk, matk, mat, 3 * vec};
   rc = check_ptrs(in, inb, 9, out, outb, 5);
   if (rc != FBOB_OK) return rc;
   // Pass 1 (row blocks): Qtil, dOtil and the row scalars alpha, E, D.

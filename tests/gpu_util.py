@@ -58,8 +58,14 @@ def check(name, got, ref, rel=REL_FRO, mx=MAX_ABS, zero_atol=1e-6):
     return r, m
 
 
-def inputs(B, H, N, d, seed, sigma=(1.0,) * 7, heads=None):
-    return synth.make_inputs(B, H, N, d, seed, sigma, heads=heads)
+def inputs(B, H, N, d, seed, sigma=(1.0,) * 7, heads=None, kv_heads=None):
+    """Seeded bf16 inputs; with kv_heads, k, v, gk, gv keep only the first
+    kv_heads heads (grouped-query attention)."""
+    bits = synth.make_inputs(B, H, N, d, seed, sigma, heads=heads)
+    if kv_heads is not None:
+        for n in ("k", "v", "gk", "gv"):
+            bits[n] = np.ascontiguousarray(bits[n][:, :kv_heads])
+    return bits
 
 
 def f64(bits):

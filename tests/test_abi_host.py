@@ -130,3 +130,12 @@ def test_rejects_bad_sequence_offsets(lib):
     assert bob(lib, shape(BASE + 2, 2), ptrs(14)) == 1           # misaligned offsets
     assert bob(lib, shape(BASE, (1 << 24) + 1), ptrs(14)) == 1   # more sequences than N allows
     assert bob(lib, shape(BASE, 2, N=0), ptrs(14)) == 0          # valid: empty problem, no call
+
+
+def test_rejects_bad_kv_heads(lib):
+    def shape(H, Hkv, N=128):
+        return fbob.fbob_shape(1, H, N, 64, 0.125, 0, -1, -1, None, 0, Hkv)
+    assert bob(lib, shape(4, 3), ptrs(14)) == 1       # not a divisor of H
+    assert bob(lib, shape(4, -1), ptrs(14)) == 1
+    assert bob(lib, shape(4, 2, N=0), ptrs(14)) == 0  # valid: empty problem, no call
+    assert bob(lib, shape(4, 0, N=0), ptrs(14)) == 0  # 0 = no grouping
