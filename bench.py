@@ -230,8 +230,9 @@ def run_gpu(args, w):
     segs = (torch.tensor(w.segments, dtype=torch.int32, device="cuda") if w.segments
             else None)  # packed-sequence offsets (kept alive for every call below)
     o, lse = fbob.attn_fwd(q, k, v, w.scale, w.causal, w.window, segs)
-    shp = fbob.make_shape(w.B, w.H, w.N, w.d, w.scale, w.causal, w.window, segs)
-    outs = [torch.empty_like(q) for _ in range(4)]
+    shp = fbob.make_shape(w.B, w.H, w.N, w.d, w.scale, w.causal, w.window, segs,
+                          kv_heads=w.kv_heads or None)
+    outs = [torch.empty_like(q), torch.empty_like(k), torch.empty_like(v), torch.empty_like(q)]
     rs = torch.empty((3, w.B, w.H, w.N), dtype=torch.float32, device="cuda")
     torch.cuda.synchronize()
     stream = torch.cuda.current_stream()
@@ -299,7 +300,7 @@ def run_gpu(args, w):
     pin = {n: torch.from_numpy(bits[n].view(np.int16)).view(torch.bfloat16).pin_memory()
            for n in synth.NAMES}
     o_h, lse_h = o.cpu().pin_memory(), lse.cpu().pin_memory()
-    res_h = [torch.empty(q.shape, dtype=torch.bfloat16).pin_memory() for _ in range(4)]
+    res_h = [torch.empty(t.shape, dtype=torch.bfloat16).pin_memory() for t in outs]
     rs_h = torch.empty(rs.shape, dtype=torch.float32).pin_memory()
     h2d = sum(t.numel() * t.element_size() for t in (*pin.values(), o_h, lse_h))
     d2h = sum(t.numel() * t.element_size() for t in (*res_h, rs_h))
@@ -364,7 +365,8 @@ def run_gpu(args, w):
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": w.name, "B": w.B, "H": w.H, "N": w.N, "d": w.d,
                    "causal": w.causal, "window": list(w.window),
-                   "packed_sequences": len(w.segments) - 1 if w.segments else 1, "seed": w.seed,
+                   "packed_sequences": len(w.segments) - 1 if w.segments else 1,
+                   "kv_heads": w.kv_heads or w.H, "seed": w.seed,
                    "l2": "no flush: inputs (%.2f GB) exceed the 129 MB L2" % (footprint / 1e9),
                    "parallelism": "replicas" if world > 1 else "single GPU",
                    "flop_formula": ("2*19*B*H*d*(valid (i,j) pairs of the band)"
@@ -405,7 +407,8 @@ def run_gpu_op(args, w):
     q, k, v, do = dev["q"], dev["k"], dev["v"], dev["dout"]
     segs = (torch.tensor(w.segments, dtype=torch.int32, device="cuda") if w.segments
             else None)
-    shp = fbob.make_shape(w.B, w.H, w.N, w.d, w.scale, w.causal, w.window, segs)
+    shp = fbob.make_shape(w.B, w.H, w.N, w.d, w.scale, w.causal, w.window, segs,
+                          kv_heads=w.kv_heads or None)
     o, lse = fbob.attn_fwd(q, k, v, w.scale, w.causal, w.window, segs)
     dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
     dstat = torch.empty_like(lse)

@@ -35,6 +35,7 @@ class Workload:
     sigma: tuple  # per tensor in NAMES order
     window: tuple = (-1, -1)  # sliding-window band (left, right); -1 = unbounded
     segments: tuple = ()      # offsets of packed sequences along N; () = one sequence
+    kv_heads: int = 0         # key/value heads (grouped-query attention); 0 = H
 
     @property
     def scale(self) -> float:
@@ -80,6 +81,11 @@ def packed_offsets(N: int, n: int, seed: int) -> tuple:
 
 # packed variable-length variant of n16k_d128_causal: 12 causal sequences of
 # seeded lengths (about 340 to 2400 tokens) in the 16K rows of each head
+# grouped-query variant of n16k_d128_causal: 4 key/value heads for 16 query heads
+WORKLOADS["n16k_d128_causal_gqa4"] = Workload(
+    "n16k_d128_causal_gqa4", 2, 16, 16384, 128, True, 7,
+    _s(1, 1, 1, *(4 * [1 / math.sqrt(128)])), kv_heads=4)
+
 WORKLOADS["n16k_d128_causal_varlen"] = Workload(
     "n16k_d128_causal_varlen", 2, 16, 16384, 128, True, 6,
     _s(1, 1, 1, *(4 * [1 / math.sqrt(128)])), segments=packed_offsets(16384, 12, 6))
@@ -138,4 +144,10 @@ def make_inputs(B, H, N, d, seed, sigma=(1.0,) * 7, heads=None):
 
 
 def workload_inputs(w: Workload, heads=None):
-    return make_inputs(w.B, w.H, w.N, w.d, w.seed, w.sigma, heads=heads)
+    """The workload's seven inputs; with kv_heads, k, v, gk, gv keep the first
+    kv_heads heads of each batch entry."""
+    bits = make_inputs(w.B, w.H, w.N, w.d, w.seed, w.sigma, heads=heads)
+    if w.kv_heads and heads is None:
+        for n in ("k", "v", "gk", "gv"):
+            bits[n] = np.ascontiguousarray(bits[n][:, :w.kv_heads])
+    return bits

@@ -173,3 +173,34 @@ def test_n16k_d128_causal_varlen_rows_and_sequence():
     for hh, ref in zip(heads, blk):
         G.check("kbar[sequence]", G.flat(r["kbar"], hh, w.H)[a:b], ref["kbar"])
         G.check("vbar[sequence]", G.flat(r["vbar"], hh, w.H)[a:b], ref["vbar"])
+
+
+def test_n16k_d128_causal_gqa4_rows_and_tail():
+    """Grouped-query workload at full size: sampled rows of one query head,
+    and the causal tail of one key/value head (its key columns >= N - 256 are
+    complete once rows >= N - 256 of its four query heads are summed)."""
+    w = synth.WORKLOADS["n16k_d128_causal_gqa4"]
+    bits = synth.workload_inputs(w)
+    r = G.run_bob(bits, w.scale, w.causal)
+    assert r["status"] == 0
+    N, H, Hkv = w.N, w.H, w.kv_heads
+    Gq = H // Hkv
+    hq = 6  # query head 6 of batch 0 reads key/value head 1
+    rows = sample_rows(N, 67)
+    X = {n: G.f64(bits[n][0, hq // Gq if n in ("k", "v", "gk", "gv") else hq])
+         for n in synth.NAMES}
+    ref = oracle.bob_head(*(X[n] for n in synth.NAMES), w.scale, w.causal, rows=rows)
+    for name in ROWS_OUT:
+        G.check(f"{name}[head {hq}]", r[name][0, hq][rows], ref[name])
+    t0 = N - 256
+    kb = np.zeros((256, w.d))
+    vb = np.zeros((256, w.d))
+    for g in range(Gq):
+        h = 1 * Gq + g
+        Y = {n: G.f64(bits[n][0, 1 if n in ("k", "v", "gk", "gv") else h]) for n in synth.NAMES}
+        t = oracle.bob_head(*(Y[n] for n in synth.NAMES), w.scale, w.causal,
+                            rows=np.arange(t0, N), cols=(t0, N))
+        kb += t["kbar"]
+        vb += t["vbar"]
+    G.check("kbar[kv head 1, tail]", r["kbar"][0, 1][t0:], kb)
+    G.check("vbar[kv head 1, tail]", r["vbar"][0, 1][t0:], vb)
