@@ -69,6 +69,9 @@ constexpr uint32_t kColDC1 = 128;  // second DC buffer (column engine, d = 64)
 // column, D/2 columns each) at kColQT and kColQT + D/2; second SF buffer
 constexpr uint32_t kColQT = 0;
 constexpr uint32_t kColSF1 = 128;
+// forward: slack (log2 units) by which a tile's row maximum may exceed the
+// running maximum before the accumulator is rescaled (P <= 2^kFwdSlack)
+constexpr float kFwdSlack = 8.f;
 
 // Shared-memory bookkeeping block (in the MISC area).
 struct Misc {
@@ -82,6 +85,7 @@ struct Misc {
   uint64_t bar_sa_dc[2];
   uint64_t bar_ew[4];   // [DC buffer][half]; a single DC buffer uses [0..1]
   uint64_t bar_xb[2];   // issuer X's stage-B MMAs completed (per half, or per DC buffer)
+  uint64_t bar_od[2];   // forward: issuer Y's O += P V MMAs of a tile completed (per P buffer)
   uint64_t bar_acc;
   uint32_t tmem_base;
   uint32_t pad;
@@ -229,8 +233,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
   const int key_hi = min(seq_hi1, p.wr < 0 ? N : last_row + p.wr + 1);  // exclusive
   const int first_tile = key_lo / BN;
   const int ntiles = (key_hi - 1) / BN - first_tile + 1;
-  const int nsteps = OP == RowOp::Fwd ? 2 * ntiles : ntiles;
-  const int first_b = OP == RowOp::Fwd ? ntiles : 0;  // first step with stage-B MMAs
+  const int nsteps = ntiles;
 
   if (tid == 0) {
     m->wctl.abort = 0;
@@ -251,6 +254,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
     for (int h = 0; h < 2; ++h) {
       mbar_init(&m->bar_sa_dc[h], 1);
       mbar_init(&m->bar_xb[h], 1);
+      mbar_init(&m->bar_od[h], 1);
     }
     for (int h = 0; h < 4; ++h) mbar_init(&m->bar_ew[h], kEwThreads);
     mbar_init(&m->bar_acc, 2);
@@ -285,9 +289,8 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         if (st >= C::NSTAGES) {
           if (!mbar_wait(&m->bar_empty[stage], ((st / C::NSTAGES) - 1) & 1, wctl)) break;
         }
-        const int j0 = (first_tile + st % ntiles) * BN;
-        const bool k_only = (OP == RowOp::Fwd) && st < ntiles;
-        const int nt = k_only ? 1 : C::NSTREAM;
+        const int j0 = (first_tile + st) * BN;
+        const int nt = C::NSTREAM;
         uint8_t* dst = s_stream + stage * C::STAGE_BYTES;
         // BoB: K and U_K first on bar_full (all issuer X needs), then V and
         // U_V on bar_full_b; the other operations use bar_full alone
@@ -338,7 +341,6 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
       // or dOtil (direct form) (part 0) and issuer Y the rest (part 1);
       // otherwise Y takes them all (part 2).
       auto stage_b = [&](uint32_t sb, int h, int st, int part) {
-        if (st < first_b) return;
         constexpr uint32_t kBoxBytes = C::NSTREAM * BN * 128;
         const uint64_t md0 = sdesc_sw128(sb, kBoxBytes, 1024);
 #pragma unroll
@@ -347,7 +349,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
           auto md = [&](int t, int bo) -> uint64_t {
             return md0 + (uint64_t)((soff<C::NSTREAM, kB4>(t, h, bo) + sub * 2048) >> 4);
           };
-          const uint32_t first = (st == first_b && s == 0) ? 0u : 1u;
+          const uint32_t first = (st == 0 && s == 0) ? 0u : 1u;
           if constexpr (kBob) {
             const uint32_t A = tmem + kColDC + 64 * h + 16 * sub;
             const uint32_t k_rows = sb + soff<C::NSTREAM, kB4>(0, h, 0) + sub * 2048;
@@ -383,8 +385,6 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
             }
           } else if constexpr (OP == RowOp::BwdDQ) {
             mma_ts(tmem + 0, tmem + kColDC + 16 * s, md(0, 0), id_b, first);  // dQ += dS K
-          } else {
-            mma_ts(tmem + 0, tmem + kColDC + 16 * s, md(1, 0), id_b, first);  // O += P V
           }
         }
       };
@@ -434,6 +434,26 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
               break;
             tc_fence_after();
             stage_sf(st, b ? kColSF1 : kColSF);
+            mma_commit(&m->bar_sa_sf[b]);
+            mma_commit(&m->bar_empty[stage]);
+          }
+          ok = false;
+        }
+        if constexpr (OP == RowOp::Fwd) {
+          // S(t) = Q K^T into buffer t & 1 (columns kColSF + 64 b): X runs up
+          // to a tile ahead of the elementwise warps
+          for (int st = 0; ok && st < nsteps; ++st) {
+            const int b = st & 1;
+            const int stage = st % C::NSTAGES;
+            if ((st >= 2 && !mbar_wait(&m->bar_sf_free[b], ((st - 2) >> 1) & 1, wctl)) ||
+                !mbar_wait(&m->bar_full[stage], (st / C::NSTAGES) & 1, wctl))
+              break;
+            tc_fence_after();
+            const uint64_t kd0 =
+                sdesc_sw128(smem_u32(s_stream + stage * C::STAGE_BYTES), 16, 1024);
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k)
+              mma_ss(tmem + kColSF + 64 * b, sd(0, k), kd(kd0, 0, 0, k), id_n64, k > 0);
             mma_commit(&m->bar_sa_sf[b]);
             mma_commit(&m->bar_empty[stage]);
           }
@@ -527,6 +547,31 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
             mma_commit(&m->bar_empty[ns]);
           }
           ok = false;  // no stage B
+        }
+        if constexpr (OP == RowOp::Fwd) {
+          // O_wg += P_wg V: the 16-key K-step s of a tile belongs to
+          // warpgroup s & 1, whose accumulator sits at columns (s & 1) D
+          constexpr uint32_t kBoxBytes = C::NSTREAM * BN * 128;
+          for (int st = 0; ok && st < nsteps; ++st) {
+            const int b = st & 1;
+            const int stage = st % C::NSTAGES;
+            if (!mbar_wait(&m->bar_full[stage], (st / C::NSTAGES) & 1, wctl) ||
+                !mbar_wait(&m->bar_ew[b], (st >> 1) & 1, wctl))
+              break;
+            tc_fence_after();
+            const uint64_t md0 =
+                sdesc_sw128(smem_u32(s_stream + stage * C::STAGE_BYTES), kBoxBytes, 1024);
+#pragma unroll
+            for (int s4 = 0; s4 < 4; ++s4) {
+              const uint64_t vd =
+                  md0 + (uint64_t)((soff<C::NSTREAM, false>(1, s4 >> 1, 0) + (s4 & 1) * 2048) >> 4);
+              mma_ts(tmem + (s4 & 1) * D, tmem + kColDC + 32 * b + 8 * s4, vd, id_b,
+                     (st == 0 && s4 < 2) ? 0u : 1u);
+            }
+            mma_commit(&m->bar_od[b]);
+            mma_commit(&m->bar_empty[stage]);
+          }
+          ok = false;
         }
         if (ok) {
           tc_fence_after();
@@ -627,7 +672,133 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
       tc_fence_before();
       mbar_arrive(&m->bar_stat);
     }
-    float mrow = -INFINITY, lrow = 0.f;             // forward sweep 1 (log2 domain)
+    if constexpr (OP == RowOp::Fwd) {
+      // ---- single-sweep forward (eq. 1) with an online softmax.  Warpgroup
+      // wg owns the keys of its columns (K-steps s with s & 1 == wg) and its
+      // own accumulator O_wg (TMEM columns wg D .. +D).  Its running row
+      // maximum m (log2 domain) is raised only when a tile's maximum exceeds
+      // it by more than kFwdSlack, so P = 2^(x - m) <= 2^kFwdSlack, and O_wg
+      // is rescaled only then, after the MMAs into it have completed.  The
+      // two warpgroups' (m, l, O) are combined once, in the epilogue.
+      float mrow = -INFINITY, lrow = 0.f;
+      bool ok = true;
+      const uint32_t ocol = (uint32_t)(wg * D);
+      for (int st = 0; ok && st < nsteps; ++st) {
+        const int b = st & 1;
+        const uint32_t par = (st >> 1) & 1;
+        if (!mbar_wait(&m->bar_sa_sf[b], par, wctl)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        uint32_t rS[2][16];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) tmem_ld16(ta + kColSF + 64 * b + HB * h + 16 * wg, rS[h]);
+        tmem_ld_wait(rS[0]);
+        reg_dep(rS[1]);
+        tc_fence_before();
+        mbar_arrive(&m->bar_sf_free[b]);
+        const int jt = (first_tile + st) * BN;
+        float x[2][16];
+        float mt = -INFINITY;
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const int j0 = jt + HB * h + 16 * wg;
+          const int mlo = jlo - j0, mhi = jhi - j0;  // valid columns: mlo <= c < mhi
+          const bool need_mask = mlo > 0 || mhi < 16;
+#pragma unroll
+          for (int c = 0; c < 16; ++c) {
+            x[h][c] = bits_f(rS[h][c]) * sl2;
+            if (need_mask && (c < mlo || c >= mhi)) x[h][c] = -INFINITY;
+            mt = fmaxf(mt, x[h][c]);
+          }
+        }
+        const bool raise = mt > mrow + kFwdSlack;  // also the first tile with a valid key
+        const bool rescale = raise && mrow != -INFINITY;
+        if (__any_sync(0xffffffffu, rescale)) {
+          // every MMA into O_wg so far (tiles < st) must have completed
+          if (!mbar_wait(&m->bar_od[(st - 1) & 1], ((st - 1) >> 1) & 1, wctl)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const float f = rescale ? ex2(mrow - mt) : 1.f;
+#pragma unroll 1
+          for (int q = 0; q < D / 16; ++q) {
+            uint32_t o[16];
+            tmem_ld16(ta + ocol + 16 * q, o);
+            tmem_ld_wait(o);
+            uint32_t lo8[8], hi8[8];
+#pragma unroll
+            for (int c = 0; c < 8; ++c) {
+              lo8[c] = __float_as_uint(bits_f(o[c]) * f);
+              hi8[c] = __float_as_uint(bits_f(o[8 + c]) * f);
+            }
+            tmem_st8(ta + ocol + 16 * q, lo8);
+            tmem_st8(ta + ocol + 16 * q + 8, hi8);
+          }
+          tmem_st_wait();
+          if (rescale) lrow *= f;
+        }
+        if (raise) mrow = mt;
+        float psum = 0.f;
+        uint32_t oP[2][8];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+#pragma unroll
+          for (int c = 0; c < 16; c += 2) {
+            // no valid key yet in this row: m = -inf and every x = -inf
+            const float p0 = mrow == -INFINITY ? 0.f : ex2(x[h][c] - mrow);
+            const float p1 = mrow == -INFINITY ? 0.f : ex2(x[h][c + 1] - mrow);
+            psum += p0 + p1;
+            oP[h][c / 2] = pack_bf16(p0, p1);
+          }
+        }
+        lrow += psum;
+        // P buffer b was last read by the MMAs of tile st - 2
+        if (st >= 2 && !mbar_wait(&m->bar_od[b], par ^ 1u, wctl)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+#pragma unroll
+        for (int h = 0; h < 2; ++h) tmem_st8(ta + kColDC + 32 * b + 8 * (2 * h + wg), oP[h]);
+        tmem_st_wait();
+        tc_fence_before();
+        mbar_arrive(&m->bar_ew[b]);
+      }
+      // ---- epilogue: O = (O_0 2^(m0-M) + O_1 2^(m1-M)) / l, L = M + log2 l
+      if (ok) ok = mbar_wait(&m->bar_acc, 0, wctl);
+      if (ok && *abort_flag) ok = false;
+      tc_fence_after();
+      s_xchg[wg * BM + r] = mrow;
+      s_xchg[(2 + wg) * BM + r] = lrow;
+      named_bar_sync(1, kEwThreads);
+      if (ok) {
+        const float m0 = s_xchg[r], m1 = s_xchg[BM + r];
+        const float mm = fmaxf(m0, m1);
+        const float f0 = m0 == -INFINITY ? 0.f : ex2(m0 - mm);
+        const float f1 = m1 == -INFINITY ? 0.f : ex2(m1 - mm);
+        const float lt = s_xchg[2 * BM + r] * f0 + s_xchg[3 * BM + r] * f1;
+        const float inv = row_ok ? 1.f / lt : 0.f;
+#pragma unroll 1
+        for (int q = 0; q < D / 32; ++q) {
+          const int cc = wg * (D / 2) + 16 * q;  // output columns of this warpgroup
+          uint32_t a0[16], a1[16];
+          tmem_ld16(ta + cc, a0);
+          tmem_ld16(ta + D + cc, a1);
+          tmem_ld_wait(a0);
+          reg_dep(a1);
+          if (row_ok) {
+            float v[16];
+#pragma unroll
+            for (int c = 0; c < 16; ++c) v[c] = (bits_f(a0[c]) * f0 + bits_f(a1[c]) * f1) * inv;
+            store_row16(p.out0 + rowoff + cc, v);
+          }
+        }
+        if (row_ok && wg == 0) p.vec_out[(size_t)bh * N + gi] = (mm + __log2f(lt)) * kLn2;
+      }
+    } else {
     float2 acc_a = splat(0.f), acc_e = splat(0.f);  // Pass 1 partial row sums
     bool ok = true;
     for (int st = 0; ok && st < nsteps; ++st) {
@@ -639,19 +810,6 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         break;
       }
       tc_fence_after();
-      if constexpr (OP == RowOp::Fwd) {
-        if (st == ntiles) {  // end of sweep 1: combine the two warpgroups' (max, sum)
-          s_xchg[wg * BM + r] = mrow;
-          s_xchg[(2 + wg) * BM + r] = lrow;
-          named_bar_sync(1, kEwThreads);
-          const float m0 = s_xchg[r], m1 = s_xchg[BM + r];
-          const float l0 = s_xchg[2 * BM + r], l1 = s_xchg[3 * BM + r];
-          const float mm = fmaxf(m0, m1);
-          const float l = (m0 == -INFINITY ? 0.f : l0 * ex2(m0 - mm)) +
-                          (m1 == -INFINITY ? 0.f : l1 * ex2(m1 - mm));
-          L2 = row_ok ? mm + __log2f(l) : 0.f;
-        }
-      }
       // ---- copy this thread's SF columns of both halves, then release SF
       uint32_t rS[2][16], rF[2][16];
 #pragma unroll
@@ -808,36 +966,6 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
               odS[c / 2] = pack_bf16(ds.x, ds.y);
             }
             tmem_st8(R, odS);
-          } else {
-            if (st < ntiles) {  // sweep 1: running max and sum in the log2 domain
-              float x[16];
-              float mx = mrow;
-#pragma unroll
-              for (int c = 0; c < 16; ++c) {
-                x[c] = bits_f(rS[h][c]) * sl2;
-                if (need_mask && (c < mlo || c >= mhi)) x[c] = -INFINITY;
-                mx = fmaxf(mx, x[c]);
-              }
-              if (mx != -INFINITY) {
-                float l = (mrow == -INFINITY) ? 0.f : lrow * ex2(mrow - mx);
-#pragma unroll
-                for (int c = 0; c < 16; ++c) l += ex2(x[c] - mx);
-                lrow = l;
-                mrow = mx;
-              }
-            } else {  // sweep 2: normalised probabilities into DC for O += P V
-              uint32_t oP[8];
-#pragma unroll
-              for (int c = 0; c < 16; c += 2) {
-                float2 pr = probs2(pair(rS[h], c), sl2v, nL2v);
-                if (need_mask) {
-                  if (c < mlo || c >= mhi) pr.x = 0.f;
-                  if (c + 1 < mlo || c + 1 >= mhi) pr.y = 0.f;
-                }
-                oP[c / 2] = pack_bf16(pr.x, pr.y);
-              }
-              tmem_st8(ta + kColDC + c0, oP);
-            }
           }
           tmem_st_wait();
           tc_fence_before();
@@ -924,8 +1052,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
           }
         }
       } else {
-        // O (forward) or dQ = tau * acc (first backward), columns [wg*D/2, +D/2)
-        const float mul = OP == RowOp::BwdDQ ? tau : 1.f;
+        // dQ = tau * acc (first backward), columns [wg*D/2, +D/2), and D
 #pragma unroll 1
         for (int q = 0; q < D / 32; ++q) {
           const int cc = wg * (D / 2) + 16 * q;
@@ -935,17 +1062,14 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
           if (row_ok) {
             float v[16];
 #pragma unroll
-            for (int c = 0; c < 16; ++c) v[c] = mul * bits_f(rA[c]);
+            for (int c = 0; c < 16; ++c) v[c] = tau * bits_f(rA[c]);
             store_row16(p.out0 + rowoff + cc, v);
           }
         }
-        if (row_ok && wg == 0) {
-          const size_t ri = (size_t)bh * N + gi;
-          if constexpr (OP == RowOp::Fwd) p.vec_out[ri] = L2 * kLn2;
-          else p.vec_out[ri] = Dr;
-        }
+        if (row_ok && wg == 0) p.vec_out[(size_t)bh * N + gi] = Dr;
       }
     }
+    }  // elementwise: operations other than the forward
   }
   tc_fence_before();
   __syncthreads();
