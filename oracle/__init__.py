@@ -47,14 +47,16 @@ def _load(mutant: int = 0, out_dir: str | None = None):
         return _LIBS[key]
     lib = ctypes.CDLL(build(mutant, out_dir))
     i64, dbl, cint = ctypes.c_int64, ctypes.c_double, ctypes.c_int
-    p = ctypes.c_void_p
-    lib.fbob_oracle_fwd.argtypes = [i64, i64, dbl, cint, i64, i64, p, i64, p, p, p, p, p, cint]
-    lib.fbob_oracle_bwd.argtypes = [i64, i64, dbl, cint, i64, i64, p, i64,
-                                    p, p, p, p, p, p, p, p, cint]
-    lib.fbob_oracle_bob.argtypes = [i64, i64, dbl, cint, i64, i64, p, i64, p, p, p, p, p, p, p,
-                                    p, i64, i64, i64, p, p, p, p, p, p, p, p, cint]
+    u64, p = ctypes.c_uint64, ctypes.c_void_p
+    mask = [i64, i64, dbl, cint, i64, i64, p, i64, dbl, u64, i64]
+    lib.fbob_oracle_fwd.argtypes = mask + [p, p, p, p, p, cint]
+    lib.fbob_oracle_bwd.argtypes = mask + [p, p, p, p, p, p, p, p, cint]
+    lib.fbob_oracle_bob.argtypes = mask + [p, p, p, p, p, p, p,
+                                           p, i64, i64, i64, p, p, p, p, p, p, p, p, cint]
     for f in (lib.fbob_oracle_fwd, lib.fbob_oracle_bwd, lib.fbob_oracle_bob):
         f.restype = cint
+    lib.fbob_oracle_philox.argtypes = [p, p, p]
+    lib.fbob_oracle_philox.restype = None
     _LIBS[key] = lib
     return lib
 
@@ -86,6 +88,25 @@ def _segments(segments, N):
     return seg, seg.size - 1
 
 
+def _dropout(dropout):
+    """(p, seed) of attention dropout (App. "Extensions"); p = 0: none."""
+    if dropout is None:
+        return 0.0, 0
+    pd, seed = dropout
+    pd = float(pd)
+    assert 0.0 <= pd < 1.0, pd
+    return pd, int(seed) & 0xFFFFFFFFFFFFFFFF
+
+
+def philox(ctr, key):
+    """Philox4x32-10 of a 4-word counter under a 2-word key (four uint32)."""
+    c = np.ascontiguousarray(ctr, dtype=np.uint32)
+    k = np.ascontiguousarray(key, dtype=np.uint32)
+    out = np.zeros(4, dtype=np.uint32)
+    _load().fbob_oracle_philox(_ptr(c), _ptr(k), _ptr(out))
+    return out
+
+
 def _group(H, Hkv):
     """Query heads per key/value head (grouped-query attention: query head h
     reads key/value head h // G)."""
@@ -100,11 +121,13 @@ def _heads(x):
     return x
 
 
-def fwd(q, k, v, scale, causal, nthreads=0, window=None, segments=None):
+def fwd(q, k, v, scale, causal, nthreads=0, window=None, segments=None, dropout=None):
     """Forward attention (eq. 1).  Returns O [B,H,N,d] and natural-log L [B,H,N].
     window: (wl, wr) sliding-window band (default: none); segments: offsets of
-    packed sequences (default: one sequence)."""
+    packed sequences (default: one sequence); dropout: (p, seed), the keep
+    mask of query head b*H + h drawn from Philox with that head index."""
     wl, wr = _window(window)
+    pd, seed = _dropout(dropout)
     q, k, v = (_c(_heads(t)) for t in (q, k, v))
     B, H, N, d = q.shape
     G = _group(H, k.shape[1])
@@ -117,7 +140,7 @@ def fwd(q, k, v, scale, causal, nthreads=0, window=None, segments=None):
             o_ = np.zeros((N, d)); l_ = np.zeros(N)
             hk = h // G
             rc = lib.fbob_oracle_fwd(N, d, float(scale), int(bool(causal)), wl, wr,
-                                     _ptr(seg), nseg,
+                                     _ptr(seg), nseg, pd, seed, b * H + h,
                                      _ptr(_c(q[b, h])), _ptr(_c(k[b, hk])), _ptr(_c(v[b, hk])),
                                      _ptr(o_), _ptr(l_), int(nthreads))
             assert rc == 0, rc
@@ -125,11 +148,12 @@ def fwd(q, k, v, scale, causal, nthreads=0, window=None, segments=None):
     return O, L
 
 
-def bwd(q, k, v, dout, scale, causal, nthreads=0, window=None, segments=None):
+def bwd(q, k, v, dout, scale, causal, nthreads=0, window=None, segments=None, dropout=None):
     """First backward (eqs. 2-3).  Returns dQ [B,H,N,d], dK, dV [B,Hkv,N,d] and
     D [B,H,N]; with grouped-query attention (k, v with Hkv < H heads) dK and dV
-    of a key/value head are the sums over its query heads."""
+    of a key/value head are the sums over its query heads.  dropout as in fwd."""
     wl, wr = _window(window)
+    pd, seed = _dropout(dropout)
     q, k, v, dout = (_c(_heads(t)) for t in (q, k, v, dout))
     B, H, N, d = q.shape
     G = _group(H, k.shape[1])
@@ -142,7 +166,7 @@ def bwd(q, k, v, dout, scale, causal, nthreads=0, window=None, segments=None):
             hk = h // G
             dq, dk, dv, dd = np.zeros((N, d)), np.zeros((N, d)), np.zeros((N, d)), np.zeros(N)
             rc = lib.fbob_oracle_bwd(N, d, float(scale), int(bool(causal)), wl, wr,
-                                     _ptr(seg), nseg,
+                                     _ptr(seg), nseg, pd, seed, b * H + h,
                                      _ptr(_c(q[b, h])), _ptr(_c(k[b, hk])), _ptr(_c(v[b, hk])),
                                      _ptr(_c(dout[b, h])), _ptr(dq), _ptr(dk), _ptr(dv),
                                      _ptr(dd), int(nthreads))
@@ -154,7 +178,8 @@ def bwd(q, k, v, dout, scale, causal, nthreads=0, window=None, segments=None):
 
 
 def bob_head(q, k, v, dout, gq, gk, gv, scale, causal, rows=None, cols=None,
-             nthreads=0, mutant=0, mutant_dir=None, window=None, segments=None):
+             nthreads=0, mutant=0, mutant_dir=None, window=None, segments=None,
+             dropout=None, head=0):
     """Backward-over-backward of one head ([N, d] float64 arrays).
 
     rows: query rows whose row-owned outputs are wanted (default: all).
@@ -164,8 +189,11 @@ def bob_head(q, k, v, dout, gq, gk, gv, scale, causal, rows=None, cols=None,
     kbar, vbar ((c1-c0) x d; complete only if every contributing row is listed).
     window: (wl, wr) sliding-window band i - wl <= j <= i + wr (-1 = unbounded).
     segments: offsets of packed sequences; a row sees only its own sequence.
+    dropout: (p, seed); head: the flat query-head index b*H + h that keys the
+    head's dropout mask.
     """
     wl, wr = _window(window)
+    pd, seed = _dropout(dropout)
     q, k, v, dout, gq, gk, gv = (_c(t) for t in (q, k, v, dout, gq, gk, gv))
     N, d = q.shape
     seg, nseg = _segments(segments, N)
@@ -186,6 +214,7 @@ def bob_head(q, k, v, dout, gq, gk, gv, scale, causal, rows=None, cols=None,
     }
     lib = _load(mutant, mutant_dir)
     rc = lib.fbob_oracle_bob(N, d, float(scale), int(bool(causal)), wl, wr, _ptr(seg), nseg,
+                             pd, seed, int(head),
                              _ptr(q), _ptr(k), _ptr(v), _ptr(dout), _ptr(gq), _ptr(gk), _ptr(gv),
                              _ptr(rows), nr, c0, c1,
                              _ptr(res["qbar"]), _ptr(res["dobar"]), _ptr(res["alpha"]),
@@ -196,7 +225,7 @@ def bob_head(q, k, v, dout, gq, gk, gv, scale, causal, rows=None, cols=None,
 
 
 def bob(q, k, v, dout, gq, gk, gv, scale, causal, nthreads=0, mutant=0, mutant_dir=None,
-        window=None, segments=None):
+        window=None, segments=None, dropout=None):
     """Full backward-over-backward on [B,H,N,d] (or [N,d]) float64 arrays.
 
     Returns (qbar, kbar, vbar, dobar, alpha, E, D) with the input's batch shape.
@@ -220,7 +249,7 @@ def bob(q, k, v, dout, gq, gk, gv, scale, causal, nthreads=0, mutant=0, mutant_d
             args = [t[b, h // G] if i in kv_side else t[b, h] for i, t in enumerate(ts)]
             r = bob_head(*args, scale, causal, nthreads=nthreads,
                          mutant=mutant, mutant_dir=mutant_dir, window=window,
-                         segments=segments)
+                         segments=segments, dropout=dropout, head=b * H + h)
             for n in ("qbar", "dobar", "alpha", "E", "D"):
                 out[n][b, h] = r[n]
             out["kbar"][b, h // G] += r["kbar"]

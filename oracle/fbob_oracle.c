@@ -42,6 +42,16 @@
  * segment.  Every row keeps its diagonal.  Entries outside V_i have P = 0 and
  * contribute nothing.
  *
+ * Dropout (App. "Extensions"): with keep mask R and sigma = 1/(1 - p) the
+ * forward uses sigma (R o P); the row scalars L, D, alpha, E stay defined over
+ * the ungated P; the gating acts on dP -> sigma R dP, C -> sigma R C, on
+ * dV = sigma (R o P)^T dO, and in the BoB on Vtil and dOtil:
+ *   Vtil_j = sigma sum_i R_ij P_ij h_ij do_i,
+ *   dOtil_i = sigma sum_j R_ij P_ij (u_V,j + h_ij v_j).
+ * R_ij = 1 iff word (j mod 4) of Philox4x32-10(counter = {j / 4, i, head, 0},
+ * key = {seed low 32 bits, seed high 32 bits}) is >= floor(p 2^32) (clamped
+ * to 2^32 - 1); p = 0 keeps everything and leaves every result unchanged.
+ *
  * Threads: rows are independent, so OpenMP splits rows across threads.  The
  * column-owned sums (Ktil, Vtil, dV, dK) are accumulated into one private
  * buffer per thread and reduced in thread order at the end.
@@ -65,6 +75,53 @@ static double dot(const double* a, const double* b, int64_t d) {
     double s = 0.0;
     for (int64_t t = 0; t < d; ++t) s += a[t] * b[t];
     return s;
+}
+
+/* Philox4x32-10 (Salmon, Moraes, Dror and Shaw, "Parallel random numbers:
+ * as easy as 1, 2, 3", SC'11): ten rounds of the Philox S-box on a 4 x 32-bit
+ * counter under a 2 x 32-bit key, the key raised by the Weyl constants
+ * 0x9E3779B9, 0xBB67AE85 before every round but the first. */
+void fbob_oracle_philox(const uint32_t ctr[4], const uint32_t key[2], uint32_t out[4]) {
+    uint32_t c0 = ctr[0], c1 = ctr[1], c2 = ctr[2], c3 = ctr[3];
+    uint32_t k0 = key[0], k1 = key[1];
+    for (int r = 0; r < 10; ++r) {
+        if (r > 0) {
+            k0 += 0x9E3779B9u;
+            k1 += 0xBB67AE85u;
+        }
+        const uint64_t p0 = (uint64_t)0xD2511F53u * (uint64_t)c0;
+        const uint64_t p1 = (uint64_t)0xCD9E8D57u * (uint64_t)c2;
+        const uint32_t n0 = (uint32_t)(p1 >> 32) ^ c1 ^ k0;
+        const uint32_t n1 = (uint32_t)p1;
+        const uint32_t n2 = (uint32_t)(p0 >> 32) ^ c3 ^ k1;
+        const uint32_t n3 = (uint32_t)p0;
+        c0 = n0; c1 = n1; c2 = n2; c3 = n3;
+    }
+    out[0] = c0; out[1] = c1; out[2] = c2; out[3] = c3;
+}
+
+/* dropout: the keep threshold and the gate g_ij = sigma R_ij (1 without dropout) */
+typedef struct { int on; uint32_t thr; double sigma; uint64_t seed; int64_t head; } drop_t;
+
+static drop_t make_drop(double p, uint64_t seed, int64_t head) {
+    drop_t r = {0, 0u, 1.0, seed, head};
+    if (p > 0.0) {
+        double t = floor(p * 4294967296.0);
+        if (t > 4294967295.0) t = 4294967295.0;
+        r.on = 1;
+        r.thr = (uint32_t)t;
+        r.sigma = 1.0 / (1.0 - p);
+    }
+    return r;
+}
+
+static double gate(drop_t g, int64_t i, int64_t j) {
+    if (!g.on) return 1.0;
+    const uint32_t ctr[4] = {(uint32_t)(j >> 2), (uint32_t)i, (uint32_t)g.head, 0u};
+    const uint32_t key[2] = {(uint32_t)g.seed, (uint32_t)(g.seed >> 32)};
+    uint32_t w[4];
+    fbob_oracle_philox(ctr, key, w);
+    return w[j & 3] >= g.thr ? g.sigma : 0.0;
 }
 
 /* the valid columns [lo_i, hi_i) of row i (see the header comment) */
@@ -127,11 +184,13 @@ static void softmax_row(int64_t i, int64_t N, int64_t d, double tau, band_t mk,
 
 /* ---------------------------------------------------------------- forward */
 int fbob_oracle_fwd(int64_t N, int64_t d, double tau, int causal, int64_t wl, int64_t wr,
-                    const int64_t* seg, int64_t nseg,
+                    const int64_t* seg, int64_t nseg, double p_drop, uint64_t seed,
+                    int64_t head,
                     const double* Q, const double* K, const double* V,
                     double* O, double* L, int nthreads) {
     if (N < 0 || d <= 0) return 1;
     const band_t mk = {causal, wl, wr, seg, nseg};
+    const drop_t dg = make_drop(p_drop, seed, head);
     const int nt = pick_threads(nthreads);
 #pragma omp parallel num_threads(nt)
     {
@@ -145,7 +204,7 @@ int fbob_oracle_fwd(int64_t N, int64_t d, double tau, int causal, int64_t wl, in
             L[i] = Li;
             for (int64_t a = 0; a < d; ++a) {
                 double acc = 0.0;
-                for (int64_t j = lo; j < hi; ++j) acc += P[j] * V[j * d + a];
+                for (int64_t j = lo; j < hi; ++j) acc += gate(dg, i, j) * P[j] * V[j * d + a];
                 O[i * d + a] = acc;
             }
         }
@@ -157,11 +216,13 @@ int fbob_oracle_fwd(int64_t N, int64_t d, double tau, int causal, int64_t wl, in
 
 /* ------------------------------------------------------- first backward */
 int fbob_oracle_bwd(int64_t N, int64_t d, double tau, int causal, int64_t wl, int64_t wr,
-                    const int64_t* seg, int64_t nseg,
+                    const int64_t* seg, int64_t nseg, double p_drop, uint64_t seed,
+                    int64_t head,
                     const double* Q, const double* K, const double* V, const double* dO,
                     double* dQ, double* dK, double* dV, double* Dvec, int nthreads) {
     if (N < 0 || d <= 0) return 1;
     const band_t mk = {causal, wl, wr, seg, nseg};
+    const drop_t dg = make_drop(p_drop, seed, head);
     const int nt = pick_threads(nthreads);
     const size_t nd = (size_t)N * (size_t)d;
     double* part = (double*)calloc((size_t)nt * 2 * (nd > 0 ? nd : 1), sizeof(double));
@@ -180,7 +241,8 @@ int fbob_oracle_bwd(int64_t N, int64_t d, double tau, int causal, int64_t wl, in
             softmax_row(i, N, d, tau, mk, Q, K, S, P, &Li, &lo, &hi);
             double D = 0.0;                                   /* D_i = sum_j P_ij dP_ij */
             for (int64_t j = lo; j < hi; ++j) {
-                dP[j] = dot(dO + i * d, V + j * d, d);        /* dP = dO V^T */
+                /* dP = dO V^T, gated by dropout: sigma R dP */
+                dP[j] = gate(dg, i, j) * dot(dO + i * d, V + j * d, d);
                 D += P[j] * dP[j];
             }
             Dvec[i] = D;
@@ -190,7 +252,7 @@ int fbob_oracle_bwd(int64_t N, int64_t d, double tau, int causal, int64_t wl, in
                 for (int64_t a = 0; a < d; ++a) {
                     dQ[i * d + a] += tau * dS * K[j * d + a];     /* dQ = tau dS K   */
                     my_dK[j * d + a] += tau * dS * Q[i * d + a];  /* dK = tau dS^T Q */
-                    my_dV[j * d + a] += P[j] * dO[i * d + a];     /* dV = P^T dO     */
+                    my_dV[j * d + a] += gate(dg, i, j) * P[j] * dO[i * d + a];  /* dV = (sigma R o P)^T dO */
                 }
             }
         }
@@ -224,7 +286,8 @@ int fbob_oracle_bwd(int64_t N, int64_t d, double tau, int causal, int64_t wl, in
  * Any output pointer may be NULL; c1 <= c0 skips the column-owned sums.
  */
 int fbob_oracle_bob(int64_t N, int64_t d, double tau, int causal, int64_t wl, int64_t wr,
-                    const int64_t* seg, int64_t nseg,
+                    const int64_t* seg, int64_t nseg, double p_drop, uint64_t seed,
+                    int64_t head,
                     const double* Q, const double* K, const double* V, const double* dO,
                     const double* UQ, const double* UK, const double* UV,
                     const int64_t* rows, int64_t nrows, int64_t c0, int64_t c1,
@@ -232,6 +295,7 @@ int fbob_oracle_bob(int64_t N, int64_t d, double tau, int causal, int64_t wl, in
                     double* D_out, double* L_out, double* Kt, double* Vt, int nthreads) {
     if (N < 0 || d <= 0 || nrows < 0) return 1;
     const band_t mk = {causal, wl, wr, seg, nseg};
+    const drop_t dg = make_drop(p_drop, seed, head);
     for (int64_t r = 0; r < nrows; ++r)
         if (rows[r] < 0 || rows[r] >= N) return 1;
     if (c0 < 0) c0 = 0;
@@ -256,6 +320,7 @@ int fbob_oracle_bob(int64_t N, int64_t d, double tau, int causal, int64_t wl, in
         double* St = (double*)malloc(sizeof(double) * n1);
         double* dS = (double*)malloc(sizeof(double) * n1);
         double* h = (double*)malloc(sizeof(double) * n1);
+        double* G = (double*)malloc(sizeof(double) * n1);
         double* my_Kt = part ? part + (size_t)thread_id() * 2 * cd : NULL;
         double* my_Vt = part ? my_Kt + cd : NULL;
 #pragma omp for schedule(static)
@@ -271,7 +336,8 @@ int fbob_oracle_bob(int64_t N, int64_t d, double tau, int causal, int64_t wl, in
             /* eq. (2): dP = dO V^T and D_i = sum_j P_ij dP_ij */
             double D = 0.0;
             for (int64_t j = lo; j < hi; ++j) {
-                dP[j] = dot(dout, V + j * d, d);
+                G[j] = gate(dg, i, j);                       /* sigma R_ij (dropout) */
+                dP[j] = G[j] * dot(dout, V + j * d, d);
                 D += P[j] * dP[j];
             }
             /* App. C step 1: F = tau (U_Q K^T + Q U_K^T); step 4: C = dO U_V^T */
@@ -283,7 +349,11 @@ int fbob_oracle_bob(int64_t N, int64_t d, double tau, int causal, int64_t wl, in
 #else
                 F[j] = tau * (dot(uq, K + j * d, d) + dot(q, UK + j * d, d));
 #endif
+#if FBOB_MUTANT == 9 /* planted: C left ungated under dropout */
                 C[j] = dot(dout, UV + j * d, d);
+#else
+                C[j] = G[j] * dot(dout, UV + j * d, d);
+#endif
             }
             /* step 2: alpha_i = sum_j P_ij F_ij */
             double alpha = 0.0;
@@ -318,11 +388,13 @@ int fbob_oracle_bob(int64_t N, int64_t d, double tau, int causal, int64_t wl, in
                     for (int64_t j = lo; j < hi; ++j) {
                         qa += St[j] * K[j * d + a] + dS[j] * UK[j * d + a];
 #if FBOB_MUTANT == 6 /* planted: h replaced by F (alpha dropped from h) */
-                        oa += P[j] * UV[j * d + a] + P[j] * F[j] * V[j * d + a];
+                        oa += G[j] * (P[j] * UV[j * d + a] + P[j] * F[j] * V[j * d + a]);
 #elif FBOB_MUTANT == 7 /* planted: wrong index, value row i used for every j */
-                        oa += P[j] * UV[j * d + a] + P[j] * h[j] * V[i * d + a];
+                        oa += G[j] * (P[j] * UV[j * d + a] + P[j] * h[j] * V[i * d + a]);
+#elif FBOB_MUTANT == 10 /* planted: the U_V term of dOtil left ungated */
+                        oa += P[j] * UV[j * d + a] + G[j] * P[j] * h[j] * V[j * d + a];
 #else
-                        oa += P[j] * UV[j * d + a] + P[j] * h[j] * V[j * d + a];
+                        oa += G[j] * (P[j] * UV[j * d + a] + P[j] * h[j] * V[j * d + a]);
 #endif
                     }
                     if (Qt) Qt[r * d + a] = tau * qa;
@@ -341,7 +413,7 @@ int fbob_oracle_bob(int64_t N, int64_t d, double tau, int causal, int64_t wl, in
                 for (int64_t j = jbeg; j < jend; ++j) {
                     double* kt = my_Kt + (size_t)(j - c0) * d;
                     double* vt = my_Vt + (size_t)(j - c0) * d;
-                    const double ph = P[j] * h[j];
+                    const double ph = G[j] * P[j] * h[j];
                     for (int64_t a = 0; a < d; ++a) {
 #if FBOB_MUTANT == 8 /* planted: U_Q term replaced by U_K of row i */
                         kt[a] += tau * (St[j] * q[a] + dS[j] * UK[i * d + a]);
@@ -354,6 +426,7 @@ int fbob_oracle_bob(int64_t N, int64_t d, double tau, int causal, int64_t wl, in
             }
         }
         free(S); free(P); free(dP); free(F); free(C); free(Pt); free(St); free(dS); free(h);
+        free(G);
     }
     if (part) {
         for (size_t e = 0; e < cd; ++e) {

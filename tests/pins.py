@@ -48,26 +48,71 @@ def softmax_probs(Q, K, tau, causal, window=None, segments=None):
     return Ex / Ex.sum(axis=-1, keepdims=True)
 
 
-def first_backward(Q, K, V, dO, tau, causal, window=None, segments=None):
-    """g(Q, K, V, dO) = (dQ, dK, dV), eqs. (2)-(3), batched over leading dims."""
+def first_backward(Q, K, V, dO, tau, causal, window=None, segments=None, gate=None):
+    """g(Q, K, V, dO) = (dQ, dK, dV), eqs. (2)-(3), batched over leading dims.
+    gate: [N, N] dropout gate sigma R of the forward O = (gate o P) V, which
+    turns the derivative with respect to P into gate o (dO V^T) and dV into
+    (gate o P)^T dO."""
     P = softmax_probs(Q, K, tau, causal, window, segments)
-    dP = dO @ np.swapaxes(V, -1, -2)
+    g = 1.0 if gate is None else gate
+    dP = g * (dO @ np.swapaxes(V, -1, -2))
     D = (P * dP).sum(axis=-1, keepdims=True)
     dS = P * (dP - D)
     dQ = tau * dS @ K
     dK = tau * np.swapaxes(dS, -1, -2) @ Q
-    dV = np.swapaxes(P, -1, -2) @ dO
+    dV = np.swapaxes(g * P, -1, -2) @ dO
     return dQ, dK, dV
 
 
-def attention(Q, K, V, tau, causal, window=None, segments=None):
-    return softmax_probs(Q, K, tau, causal, window, segments) @ V
+def attention(Q, K, V, tau, causal, window=None, segments=None, gate=None):
+    P = softmax_probs(Q, K, tau, causal, window, segments)
+    return (P if gate is None else gate * P) @ V
 
 
-def phi(Q, K, V, dO, UQ, UK, UV, tau, causal, window=None, segments=None):
-    dQ, dK, dV = first_backward(Q, K, V, dO, tau, causal, window, segments)
+def phi(Q, K, V, dO, UQ, UK, UV, tau, causal, window=None, segments=None, gate=None):
+    dQ, dK, dV = first_backward(Q, K, V, dO, tau, causal, window, segments, gate)
     return ((dQ * UQ).sum(axis=(-1, -2)) + (dK * UK).sum(axis=(-1, -2))
             + (dV * UV).sum(axis=(-1, -2)))
+
+
+_M0, _M1 = np.uint64(0xD2511F53), np.uint64(0xCD9E8D57)
+_W0, _W1 = np.uint32(0x9E3779B9), np.uint32(0xBB67AE85)
+_LO = np.uint64(0xFFFFFFFF)
+
+
+def philox4x32_10(c0, c1, c2, c3, k0, k1):
+    """Philox4x32-10 (Salmon et al., SC'11) on arrays of uint32 counter words
+    under a scalar key, vectorised in numpy: each round multiplies words 0 and
+    2 by the Philox multipliers, swaps the products' halves into the four
+    words, xors the key in, and raises the key by the Weyl constants."""
+    c = [np.asarray(x, dtype=np.uint32) for x in (c0, c1, c2, c3)]
+    k0, k1 = np.uint32(k0), np.uint32(k1)
+    with np.errstate(over="ignore"):
+        for r in range(10):
+            if r:
+                k0 = np.uint32(k0 + _W0)
+                k1 = np.uint32(k1 + _W1)
+            p0 = _M0 * c[0].astype(np.uint64)
+            p1 = _M1 * c[2].astype(np.uint64)
+            c = [((p1 >> np.uint64(32)).astype(np.uint32) ^ c[1] ^ k0),
+                 (p1 & _LO).astype(np.uint32),
+                 ((p0 >> np.uint64(32)).astype(np.uint32) ^ c[3] ^ k1),
+                 (p0 & _LO).astype(np.uint32)]
+    return c
+
+
+def dropout_gate(N, p, seed, head):
+    """[N, N] gate sigma R of one head: R_ij = 1 iff word j mod 4 of
+    Philox4x32-10(counter (j div 4, i, head, 0), key (seed mod 2^32,
+    seed div 2^32)) is at least floor(p 2^32); sigma = 1 / (1 - p)."""
+    i = np.arange(N, dtype=np.uint32)[:, None]
+    j = np.arange(N, dtype=np.uint32)[None, :]
+    z = np.zeros((N, N), dtype=np.uint32)
+    w = philox4x32_10(z + (j >> np.uint32(2)), z + i, z + np.uint32(head), z,
+                      seed & 0xFFFFFFFF, (seed >> 32) & 0xFFFFFFFF)
+    word = np.choose((j & np.uint32(3)).astype(np.int64) + 0 * z, w)
+    thr = min(int(np.floor(p * 2.0 ** 32)), 2 ** 32 - 1)
+    return (word >= np.uint32(thr)).astype(np.float64) / (1.0 - p)
 
 
 def _perturbed(X, which, deltas):
@@ -86,7 +131,7 @@ def _perturbed(X, which, deltas):
 
 
 def bob_central_fd(Q, K, V, dO, UQ, UK, UV, tau, causal, rel_h=1e-5, window=None,
-                   segments=None):
+                   segments=None, gate=None):
     """grad_{Q,K,V,dO} Phi by central differences, one entry at a time."""
     X = [Q, K, V, dO]
     grads = []
@@ -95,8 +140,8 @@ def bob_central_fd(Q, K, V, dO, UQ, UK, UV, tau, causal, rel_h=1e-5, window=None
         h = rel_h * np.maximum(1.0, np.abs(x))
         plus = _perturbed(X, which, h)
         minus = _perturbed(X, which, -h)
-        fp = phi(*plus, UQ, UK, UV, tau, causal, window, segments)
-        fm = phi(*minus, UQ, UK, UV, tau, causal, window, segments)
+        fp = phi(*plus, UQ, UK, UV, tau, causal, window, segments, gate)
+        fm = phi(*minus, UQ, UK, UV, tau, causal, window, segments, gate)
         grads.append(((fp - fm) / (2 * h)).reshape(X[which].shape))
     return grads
 
