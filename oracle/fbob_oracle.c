@@ -48,9 +48,15 @@
  * dV = sigma (R o P)^T dO, and in the BoB on Vtil and dOtil:
  *   Vtil_j = sigma sum_i R_ij P_ij h_ij do_i,
  *   dOtil_i = sigma sum_j R_ij P_ij (u_V,j + h_ij v_j).
- * R_ij = 1 iff word (j mod 4) of Philox4x32-10(counter = {j / 4, i, head, 0},
- * key = {seed low 32 bits, seed high 32 bits}) is >= floor(p 2^32) (clamped
- * to 2^32 - 1); p = 0 keeps everything and leaves every result unchanged.
+ * The paper asks for a counter-based generator such as Philox and leaves the
+ * bit layout open.  Here one Philox4x32-10 call covers a 4 x 4 block of
+ * (query, key) pairs with one random byte each: for the block (i / 4, j / 4)
+ * of query head `head` the counter is {j / 4, i / 4, head, 0} and the key
+ * {seed low 32 bits, seed high 32 bits}; the pair (i, j) takes byte (j mod 4)
+ * (bits 8 (j mod 4) .. + 7) of output word (i mod 4).  R_ij = 1 iff that byte
+ * is >= t, t = floor(256 p + 1/2) clamped to 255; the realised drop rate is
+ * t / 256 and sigma = 256 / (256 - t).  t = 0 (p < 1/512) keeps everything
+ * and leaves every result unchanged.
  *
  * Threads: rows are independent, so OpenMP splits rows across threads.  The
  * column-owned sums (Ktil, Vtil, dV, dK) are accumulated into one private
@@ -100,28 +106,29 @@ void fbob_oracle_philox(const uint32_t ctr[4], const uint32_t key[2], uint32_t o
     out[0] = c0; out[1] = c1; out[2] = c2; out[3] = c3;
 }
 
-/* dropout: the keep threshold and the gate g_ij = sigma R_ij (1 without dropout) */
+/* dropout: the byte threshold t and the gate g_ij = sigma R_ij (1 without dropout) */
 typedef struct { int on; uint32_t thr; double sigma; uint64_t seed; int64_t head; } drop_t;
 
 static drop_t make_drop(double p, uint64_t seed, int64_t head) {
     drop_t r = {0, 0u, 1.0, seed, head};
-    if (p > 0.0) {
-        double t = floor(p * 4294967296.0);
-        if (t > 4294967295.0) t = 4294967295.0;
+    double t = floor(256.0 * p + 0.5);
+    if (t > 255.0) t = 255.0;
+    if (t >= 1.0) {
         r.on = 1;
         r.thr = (uint32_t)t;
-        r.sigma = 1.0 / (1.0 - p);
+        r.sigma = 256.0 / (256.0 - t);
     }
     return r;
 }
 
 static double gate(drop_t g, int64_t i, int64_t j) {
     if (!g.on) return 1.0;
-    const uint32_t ctr[4] = {(uint32_t)(j >> 2), (uint32_t)i, (uint32_t)g.head, 0u};
+    const uint32_t ctr[4] = {(uint32_t)(j >> 2), (uint32_t)(i >> 2), (uint32_t)g.head, 0u};
     const uint32_t key[2] = {(uint32_t)g.seed, (uint32_t)(g.seed >> 32)};
     uint32_t w[4];
     fbob_oracle_philox(ctr, key, w);
-    return w[j & 3] >= g.thr ? g.sigma : 0.0;
+    const uint32_t byte = (w[i & 3] >> (8 * (j & 3))) & 0xFFu;
+    return byte >= g.thr ? g.sigma : 0.0;
 }
 
 /* the valid columns [lo_i, hi_i) of row i (see the header comment) */

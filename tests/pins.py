@@ -102,17 +102,26 @@ def philox4x32_10(c0, c1, c2, c3, k0, k1):
 
 
 def dropout_gate(N, p, seed, head):
-    """[N, N] gate sigma R of one head: R_ij = 1 iff word j mod 4 of
-    Philox4x32-10(counter (j div 4, i, head, 0), key (seed mod 2^32,
-    seed div 2^32)) is at least floor(p 2^32); sigma = 1 / (1 - p)."""
+    """[N, N] gate sigma R of one head.  The (query, key) pair (i, j) reads
+    byte j mod 4 of word i mod 4 of Philox4x32-10(counter (j div 4, i div 4,
+    head, 0), key (seed mod 2^32, seed div 2^32)); R_ij = 1 iff that byte is
+    at least t = min(255, floor(256 p + 1/2)), and sigma = 256 / (256 - t)."""
     i = np.arange(N, dtype=np.uint32)[:, None]
     j = np.arange(N, dtype=np.uint32)[None, :]
     z = np.zeros((N, N), dtype=np.uint32)
-    w = philox4x32_10(z + (j >> np.uint32(2)), z + i, z + np.uint32(head), z,
+    w = philox4x32_10(z + (j >> np.uint32(2)), z + (i >> np.uint32(2)), z + np.uint32(head), z,
                       seed & 0xFFFFFFFF, (seed >> 32) & 0xFFFFFFFF)
-    word = np.choose((j & np.uint32(3)).astype(np.int64) + 0 * z, w)
-    thr = min(int(np.floor(p * 2.0 ** 32)), 2 ** 32 - 1)
-    return (word >= np.uint32(thr)).astype(np.float64) / (1.0 - p)
+    word = np.choose((i & np.uint32(3)).astype(np.int64) + 0 * z, w)
+    byte = (word >> (np.uint32(8) * (j & np.uint32(3)))) & np.uint32(0xFF)
+    t = min(255, int(np.floor(256 * p + 0.5)))
+    if t == 0:
+        return np.ones((N, N))
+    return (byte >= np.uint32(t)).astype(np.float64) * (256.0 / (256 - t))
+
+
+def dropout_rate(p):
+    """The realised drop rate t / 256 of a requested rate p."""
+    return min(255, int(np.floor(256 * p + 0.5))) / 256
 
 
 def _perturbed(X, which, deltas):

@@ -51,8 +51,12 @@ def test_keep_rate_and_scale(p):
     g = pins.dropout_gate(N, p, 0x1234_5678_9ABC_DEF0, 5)
     keep = g > 0
     n = keep.size
-    assert abs(keep.mean() - (1 - p)) <= 5 * np.sqrt(p * (1 - p) / n)
-    assert np.allclose(g[keep], 1 / (1 - p))
+    pr = pins.dropout_rate(p)
+    assert abs(pr - p) <= 1 / 512
+    assert abs(keep.mean() - (1 - pr)) <= 5 * np.sqrt(pr * (1 - pr) / n)
+    assert np.allclose(g[keep], 1 / (1 - pr))
+    # the gate is unbiased: E[sigma R] = 1
+    assert abs(g.mean() - 1) <= 5 * np.sqrt(pr / (1 - pr) / n)
     # neighbouring words of one Philox block and neighbouring rows are uncorrelated
     a, b = keep[:, :-1].astype(float).ravel(), keep[:, 1:].astype(float).ravel()
     assert abs(np.corrcoef(a, b)[0, 1]) <= 5 / np.sqrt(a.size)
@@ -133,14 +137,32 @@ def test_torch_double_backward_with_dropout(H, Hkv, causal, p):
 
 
 @pytest.mark.parametrize("causal", [True, False])
-def test_zero_rate_is_no_dropout(causal):
+@pytest.mark.parametrize("p", [0.0, 0.0019])
+def test_zero_rate_is_no_dropout(causal, p):
+    # rates below 1/512 round to a zero byte threshold: nothing is dropped
     rng = np.random.default_rng(8)
     X = [rng.standard_normal((1, 2, 19, 8)) for _ in range(7)]
     tau = 0.3
     a = oracle.bob(*X, tau, causal)
-    b = oracle.bob(*X, tau, causal, dropout=(0.0, 77))
+    b = oracle.bob(*X, tau, causal, dropout=(p, 77))
     for x, y in zip(a, b):
         assert np.array_equal(x, y)
     assert all(np.array_equal(x, y) for x, y in zip(oracle.fwd(*X[:3], tau, causal),
                                                     oracle.fwd(*X[:3], tau, causal,
-                                                               dropout=(0.0, 77))))
+                                                               dropout=(p, 77))))
+
+
+def test_realised_rate_and_block_layout():
+    """The mask of one 4 x 4 block comes from one Philox call: byte j mod 4
+    of word i mod 4, compared with the rounded byte threshold."""
+    seed, head, p = (3 << 32) + 9, 2, 0.3
+    g = pins.dropout_gate(8, p, seed, head)
+    t = round(256 * p)
+    for I in range(2):
+        for J in range(2):
+            w = oracle.philox([J, I, head, 0], [seed & 0xFFFFFFFF, seed >> 32])
+            for a in range(4):
+                for b in range(4):
+                    byte = (int(w[a]) >> (8 * b)) & 0xFF
+                    assert (g[4 * I + a, 4 * J + b] > 0) == (byte >= t)
+    assert pins.dropout_rate(0.3) == 77 / 256 and pins.dropout_rate(0.999) == 255 / 256
