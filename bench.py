@@ -155,14 +155,15 @@ def oracle_sample(w, bits_head, target_s, seed=0):
     rows_probe = np.linspace(0, w.N - 1, 16).astype(np.int64)
     t0 = time.perf_counter()
     seg = list(w.segments) or None
+    drop = w.dropout or None  # head 0 of batch entry 0: dropout counter head 0
     oracle.bob_head(*X, w.scale, w.causal, rows=rows_probe, cols=(0, w.N), window=w.window,
-                    segments=seg)
+                    segments=seg, dropout=drop, head=0)
     dt = time.perf_counter() - t0
     n = int(max(16, min(w.N, 16 * target_s / max(dt, 1e-6))))
     rows = np.unique(np.linspace(0, w.N - 1, n).astype(np.int64))
     t0 = time.perf_counter()
     oracle.bob_head(*X, w.scale, w.causal, rows=rows, cols=(0, w.N), window=w.window,
-                    segments=seg)
+                    segments=seg, dropout=drop, head=0)
     dt = time.perf_counter() - t0
     flops = 2.0 * 19 * valid_pairs_rows(w, rows) * w.d
     return flops, dt, f"{len(rows)} evenly spaced query rows of head 0 (of {w.N}), all key columns"
@@ -229,9 +230,10 @@ def run_gpu(args, w):
     q, k, v, do, gq, gk, gv = (dev[n] for n in synth.NAMES)
     segs = (torch.tensor(w.segments, dtype=torch.int32, device="cuda") if w.segments
             else None)  # packed-sequence offsets (kept alive for every call below)
-    o, lse = fbob.attn_fwd(q, k, v, w.scale, w.causal, w.window, segs)
+    drop = w.dropout or None
+    o, lse = fbob.attn_fwd(q, k, v, w.scale, w.causal, w.window, segs, drop)
     shp = fbob.make_shape(w.B, w.H, w.N, w.d, w.scale, w.causal, w.window, segs,
-                          kv_heads=w.kv_heads or None)
+                          kv_heads=w.kv_heads or None, dropout=drop)
     outs = [torch.empty_like(q), torch.empty_like(k), torch.empty_like(v), torch.empty_like(q)]
     rs = torch.empty((3, w.B, w.H, w.N), dtype=torch.float32, device="cuda")
     torch.cuda.synchronize()
@@ -257,7 +259,7 @@ def run_gpu(args, w):
 
     # ---- timed region: K steps, each as its kernels (through their C-ABI
     # calls, the same ones fbob_attn_bob makes) with events between them
-    if w.d == 64:
+    if w.d == 64 and not drop:  # one-sweep Pass 1
         parts = [("pass1", lambda: fbob.fbob_attn_bob_pass1(
             shp, q, k, v, o, lse, do, gq, gk, gv, outs[0], outs[3], rs))]
     else:
@@ -367,6 +369,7 @@ def run_gpu(args, w):
                    "causal": w.causal, "window": list(w.window),
                    "packed_sequences": len(w.segments) - 1 if w.segments else 1,
                    "kv_heads": w.kv_heads or w.H, "seed": w.seed,
+                   "dropout": list(w.dropout) if w.dropout else None,
                    "l2": "no flush: inputs (%.2f GB) exceed the 129 MB L2" % (footprint / 1e9),
                    "parallelism": "replicas" if world > 1 else "single GPU",
                    "flop_formula": ("2*19*B*H*d*(valid (i,j) pairs of the band)"
@@ -407,9 +410,10 @@ def run_gpu_op(args, w):
     q, k, v, do = dev["q"], dev["k"], dev["v"], dev["dout"]
     segs = (torch.tensor(w.segments, dtype=torch.int32, device="cuda") if w.segments
             else None)
+    drop = w.dropout or None
     shp = fbob.make_shape(w.B, w.H, w.N, w.d, w.scale, w.causal, w.window, segs,
-                          kv_heads=w.kv_heads or None)
-    o, lse = fbob.attn_fwd(q, k, v, w.scale, w.causal, w.window, segs)
+                          kv_heads=w.kv_heads or None, dropout=drop)
+    o, lse = fbob.attn_fwd(q, k, v, w.scale, w.causal, w.window, segs, drop)
     dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
     dstat = torch.empty_like(lse)
     if args.op == "fwd":
@@ -440,7 +444,7 @@ def run_gpu_op(args, w):
         "data": "synthetic", "frac_of_bf16_peak": value / peak,
         "gpu_launches": fbob.fbob_launch_count(entry) * args.steps,
         "config": {"workload": w.name, "B": w.B, "H": w.H, "N": w.N, "d": w.d,
-                   "causal": w.causal},
+                   "causal": w.causal, "dropout": list(w.dropout) if w.dropout else None},
         "clocks": clk.summary()}), flush=True)
 
 

@@ -43,6 +43,21 @@
  *             h / (H / H_kv).  dK, dV, k_bar and v_bar of a key/value head are
  *             then sums over its H / H_kv query heads, summed inside one CTA in
  *             a fixed order.  Query-side tensors and row vectors keep H heads.
+ *  Dropout    dropout_p in [0, 1) with dropout_seed applies attention dropout
+ *             after the softmax (App. "Extensions"): O = sigma (R o P) V with a
+ *             keep mask R and sigma the inverse keep rate; the first backward
+ *             and the BoB differentiate that forward (dP, C, dV, Vtil and
+ *             dOtil carry sigma R; L, D, alpha and E stay over the ungated P).
+ *             R is regenerated in every kernel from Philox4x32-10 (Salmon et
+ *             al., SC'11), never stored: the 4 x 4 block (i/4, j/4) of query
+ *             head b*H + h uses counter {j/4, i/4, b*H + h, 0} and key
+ *             {seed low 32 bits, seed high 32 bits}; pair (i, j) takes byte
+ *             j%4 of output word i%4 and is kept iff that byte is >= t, with
+ *             t = round(256 dropout_p) (at most 255).  The realised drop rate
+ *             is t/256 and sigma = 256/(256 - t).  t = 0 (dropout_p < 1/512)
+ *             is no dropout.  i and j are positions along N (with packed
+ *             sequences, global positions).  The forward, first backward and
+ *             BoB of one problem must be given the same dropout_p and seed.
  *  Stream     Every call enqueues its kernels on `stream` (NULL = legacy
  *             default stream) and returns without synchronising.
  *  Memory     The library allocates and frees no device memory.  The caller
@@ -92,6 +107,8 @@ typedef struct fbob_shape {
     const int32_t* seq_offsets; /* packed sequences: device int32 [num_seqs + 1], or NULL */
     int64_t num_seqs;           /* number of packed sequences (0 when seq_offsets is NULL) */
     int64_t H_kv; /* key/value heads (grouped-query attention); 0 = H */
+    double dropout_p;      /* attention dropout rate in [0, 1); 0 = none */
+    uint64_t dropout_seed; /* Philox key of the dropout mask */
 } fbob_shape;
 
 /*
@@ -138,9 +155,10 @@ int fbob_attn_bob(const fbob_shape* shape, const void* q, const void* k, const v
 /*
  * Pass 1 of Algorithm 1 alone (row-block outer; Alg. 2, first loop):
  * writes q_bar, dout_bar and row_stats (alpha, E, D).  Same arguments and
- * rules as fbob_attn_bob; k_bar/v_bar are not touched.  d = 64 runs one
- * sweep with the affine fusion of Prop. 3.1 (one kernel); d = 128 runs
- * fbob_attn_bob_row_stats then fbob_attn_bob_pass1_direct (two kernels).
+ * rules as fbob_attn_bob; k_bar/v_bar are not touched.  d = 64 without
+ * dropout runs one sweep with the affine fusion of Prop. 3.1 (one kernel);
+ * d = 128, and any d with dropout, runs fbob_attn_bob_row_stats then
+ * fbob_attn_bob_pass1_direct (two kernels).
  */
 int fbob_attn_bob_pass1(const fbob_shape* shape, const void* q, const void* k, const void* v,
                         const void* o, const float* lse, const void* dout,

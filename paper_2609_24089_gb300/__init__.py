@@ -34,7 +34,8 @@ class fbob_shape(ctypes.Structure):
                 ("d", ctypes.c_int64), ("scale", ctypes.c_float), ("causal", ctypes.c_int32),
                 ("window_left", ctypes.c_int32), ("window_right", ctypes.c_int32),
                 ("seq_offsets", ctypes.c_void_p), ("num_seqs", ctypes.c_int64),
-                ("H_kv", ctypes.c_int64)]
+                ("H_kv", ctypes.c_int64), ("dropout_p", ctypes.c_double),
+                ("dropout_seed", ctypes.c_uint64)]
 
 
 _lib = None
@@ -82,12 +83,14 @@ def header_symbols() -> list:
 
 
 def make_shape(B, H, N, d, scale, causal, window=None, segments=None,
-               kv_heads=None) -> fbob_shape:
+               kv_heads=None, dropout=None) -> fbob_shape:
     """window: (left, right) sliding-window band i - left <= j <= i + right;
     -1 (or None) leaves a side unbounded.  segments: contiguous int32 CUDA
     tensor of packed-sequence offsets [num_seqs + 1] (it must stay alive
     until the calls using this shape have run), or None for one sequence.
-    kv_heads: key/value heads for grouped-query attention (None: H)."""
+    kv_heads: key/value heads for grouped-query attention (None: H).
+    dropout: (p, seed) attention dropout after the softmax (None: none); the
+    realised rate is round(256 p) / 256."""
     wl, wr = (-1, -1) if window is None else (int(window[0]), int(window[1]))
     if segments is None:
         seg, nseg = None, 0
@@ -98,8 +101,9 @@ def make_shape(B, H, N, d, scale, causal, window=None, segments=None,
             raise ValueError("segments must be a contiguous 1-D int32 CUDA tensor")
         seg, nseg = segments.data_ptr(), segments.numel() - 1
     hkv = 0 if kv_heads is None or int(kv_heads) == int(H) else int(kv_heads)
+    dp, seed = (0.0, 0) if dropout is None else (float(dropout[0]), int(dropout[1]))
     return fbob_shape(int(B), int(H), int(N), int(d), float(scale), int(causal), wl, wr,
-                      seg, nseg, hkv)
+                      seg, nseg, hkv, dp, seed & 0xFFFFFFFFFFFFFFFF)
 
 
 def _ptr(t):
@@ -124,9 +128,10 @@ def _check(rc, where):
         raise FbobError(rc, where)
 
 
-def _shape_of(q, k, scale, causal, window=None, segments=None):
+def _shape_of(q, k, scale, causal, window=None, segments=None, dropout=None):
     B, H, N, d = q.shape
-    return make_shape(B, H, N, d, scale, causal, window, segments, kv_heads=k.shape[1])
+    return make_shape(B, H, N, d, scale, causal, window, segments, kv_heads=k.shape[1],
+                      dropout=dropout)
 
 
 # ------------------------------------------------ entry points, same names as the C ABI
@@ -189,31 +194,32 @@ def fbob_launch_count(entry: str) -> int:
 
 
 # ------------------------------------------------ allocating helpers
-def attn_fwd(q, k, v, scale, causal, window=None, segments=None):
+def attn_fwd(q, k, v, scale, causal, window=None, segments=None, dropout=None):
     import torch
     B, H, N, d = q.shape
     o = torch.empty_like(q)
     lse = torch.empty((B, H, N), dtype=torch.float32, device=q.device)
-    fbob_attn_fwd(_shape_of(q, k, scale, causal, window, segments), q, k, v, o, lse)
+    fbob_attn_fwd(_shape_of(q, k, scale, causal, window, segments, dropout), q, k, v, o, lse)
     return o, lse
 
 
-def attn_bwd(q, k, v, o, lse, dout, scale, causal, window=None, segments=None):
+def attn_bwd(q, k, v, o, lse, dout, scale, causal, window=None, segments=None, dropout=None):
     import torch
     B, H, N, d = q.shape
     dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
     dstat = torch.empty((B, H, N), dtype=torch.float32, device=q.device)
-    fbob_attn_bwd(_shape_of(q, k, scale, causal, window, segments), q, k, v, o, lse, dout, dq,
-                  dk, dv, dstat)
+    fbob_attn_bwd(_shape_of(q, k, scale, causal, window, segments, dropout), q, k, v, o, lse,
+                  dout, dq, dk, dv, dstat)
     return dq, dk, dv, dstat
 
 
-def attn_bob(q, k, v, o, lse, dout, gq, gk, gv, scale, causal, window=None, segments=None):
+def attn_bob(q, k, v, o, lse, dout, gq, gk, gv, scale, causal, window=None, segments=None,
+             dropout=None):
     """Returns (q_bar, k_bar, v_bar, dout_bar, row_stats[3,B,H,N] = alpha, E, D)."""
     import torch
     B, H, N, d = q.shape
     outs = [torch.empty_like(q), torch.empty_like(k), torch.empty_like(v), torch.empty_like(q)]
     row_stats = torch.empty((3, B, H, N), dtype=torch.float32, device=q.device)
-    fbob_attn_bob(_shape_of(q, k, scale, causal, window, segments), q, k, v, o, lse, dout, gq,
-                  gk, gv, *outs, row_stats)
+    fbob_attn_bob(_shape_of(q, k, scale, causal, window, segments, dropout), q, k, v, o, lse,
+                  dout, gq, gk, gv, *outs, row_stats)
     return (*outs, row_stats)

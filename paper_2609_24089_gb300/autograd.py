@@ -33,11 +33,12 @@ class _AttnBwd(torch.autograd.Function):
     """(q, k, v, dout) -> (dq, dk, dv); its backward is BoB."""
 
     @staticmethod
-    def forward(ctx, q, k, v, o, lse, dout, scale, causal, window, segments):
+    def forward(ctx, q, k, v, o, lse, dout, scale, causal, window, segments, dropout):
         dout = _bf16(dout)
-        dq, dk, dv, _ = attn_bwd(q, k, v, o, lse, dout, scale, causal, window, segments)
+        dq, dk, dv, _ = attn_bwd(q, k, v, o, lse, dout, scale, causal, window, segments, dropout)
         ctx.save_for_backward(q, k, v, o, lse, dout)
         ctx.scale, ctx.causal, ctx.window, ctx.segments = scale, causal, window, segments
+        ctx.dropout = dropout
         return dq, dk, dv
 
     @staticmethod
@@ -46,37 +47,43 @@ class _AttnBwd(torch.autograd.Function):
         g = [torch.zeros_like(x) if t is None else _bf16(t)
              for t, x in zip((gq, gk, gv), (q, k, v))]
         q_bar, k_bar, v_bar, dout_bar, _ = attn_bob(q, k, v, o, lse, dout, *g, ctx.scale,
-                                                    ctx.causal, ctx.window, ctx.segments)
-        return q_bar, k_bar, v_bar, None, None, dout_bar, None, None, None, None
+                                                    ctx.causal, ctx.window, ctx.segments,
+                                                    ctx.dropout)
+        return q_bar, k_bar, v_bar, None, None, dout_bar, None, None, None, None, None
 
 
 class _Attn(torch.autograd.Function):
     """(q, k, v) -> O = softmax(scale Q K^T + M) V (eq. 1)."""
 
     @staticmethod
-    def forward(ctx, q, k, v, scale, causal, window, segments):
-        o, lse = attn_fwd(q, k, v, scale, causal, window, segments)
+    def forward(ctx, q, k, v, scale, causal, window, segments, dropout):
+        o, lse = attn_fwd(q, k, v, scale, causal, window, segments, dropout)
         ctx.save_for_backward(q, k, v, o, lse)
         ctx.scale, ctx.causal, ctx.window, ctx.segments = scale, causal, window, segments
+        ctx.dropout = dropout
         return o
 
     @staticmethod
     def backward(ctx, dout):
         q, k, v, o, lse = ctx.saved_tensors
         dq, dk, dv = _AttnBwd.apply(q, k, v, o.detach(), lse, dout, ctx.scale, ctx.causal,
-                                    ctx.window, ctx.segments)
-        return dq, dk, dv, None, None, None, None
+                                    ctx.window, ctx.segments, ctx.dropout)
+        return dq, dk, dv, None, None, None, None, None
 
 
 def attention(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, scale: float | None = None,
               causal: bool = False, window: tuple | None = None,
-              segments: torch.Tensor | None = None) -> torch.Tensor:
+              segments: torch.Tensor | None = None, dropout_p: float = 0.0,
+              seed: int = 0) -> torch.Tensor:
     """Softmax attention on libfbob, differentiable twice (see the module doc).
     window: (left, right) sliding-window band, -1 = unbounded side; segments:
-    int32 CUDA offsets of packed variable-length sequences."""
+    int32 CUDA offsets of packed variable-length sequences; dropout_p, seed:
+    attention dropout after the softmax with a keep mask regenerated from the
+    seed in every kernel (the same mask in the forward and both backwards)."""
     for t in (q, k, v):
         _check(t)
     if scale is None:
         scale = 1.0 / math.sqrt(q.shape[-1])
+    dropout = (float(dropout_p), int(seed)) if dropout_p else None
     return _Attn.apply(q.contiguous(), k.contiguous(), v.contiguous(), float(scale),
-                       bool(causal), None if window is None else tuple(window), segments)
+                       bool(causal), None if window is None else tuple(window), segments, dropout)

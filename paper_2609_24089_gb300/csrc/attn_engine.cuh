@@ -57,6 +57,7 @@
 // the device error word, drains its own asynchronous work and exits.
 #pragma once
 
+#include "dropout.cuh"
 #include "engine_params.h"
 #include "tc_ptx.cuh"
 
@@ -189,9 +190,11 @@ __device__ __forceinline__ float2 probs2(float2 s, float2 sl2, float2 nL2) {
 }
 
 // ============================================================== row engine
-template <RowOp OP, int D>
+// DROP: attention dropout (App. "Extensions"); the one-sweep Pass 1 has none
+template <RowOp OP, int D, bool DROP>
 __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant__ EngineParams p) {
   using C = RowCfg<OP, D>;
+  static_assert(!DROP || OP != RowOp::BobPass1, "dropout Pass 1 runs as statistics + direct");
   constexpr bool kBob = OP == RowOp::BobPass1;      // Pass 1, one sweep (Prop. 3.1)
   constexpr bool kStats = OP == RowOp::BobStats;    // row scalars alpha, E, D only
   constexpr bool kDirect = OP == RowOp::BobPass1D;  // Pass 1 with alpha, E given
@@ -636,6 +639,21 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
     const size_t rowoff = ((size_t)bh * N + (size_t)(row_ok ? gi : 0)) * D;
     const float tau = p.scale;
     const float sl2 = tau * kLog2e;
+    // dropout: keep bits of this row's 16 keys in each half of key tile jt
+    // (computed before the tile's scores are waited for); gate sigma R
+    const DropKey dkey = {p.drop_k0, p.drop_k1, p.drop_thr4};
+    const float dsig = p.drop_sigma;
+    auto tile_keep = [&](int jt, uint32_t (&kb)[2]) {
+#pragma unroll
+      for (int h = 0; h < 2; ++h) kb[h] = keep_row16(gi, jt + HB * h + 16 * wg, (uint32_t)bh, dkey);
+    };
+    // with dropout the lanes of a warp exchange keep bits, so a wait that
+    // gives up makes the whole warp leave together
+    auto ew_wait = [&](uint64_t* bar, uint32_t par) -> bool {
+      const bool w = mbar_wait(bar, par, wctl);
+      if constexpr (DROP) return __all_sync(0xffffffffu, w);
+      return w;
+    };
     float L2 = 0.f, Dr = 0.f, nal = 0.f, nE = 0.f;  // nal = -alpha, nE = -E (direct form)
     if constexpr (OP != RowOp::Fwd) {
       if (row_ok) {
@@ -686,7 +704,9 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
       for (int st = 0; ok && st < nsteps; ++st) {
         const int b = st & 1;
         const uint32_t par = (st >> 1) & 1;
-        if (!mbar_wait(&m->bar_sa_sf[b], par, wctl)) {
+        uint32_t kb[2];
+        if constexpr (DROP) tile_keep((first_tile + st) * BN, kb);
+        if (!ew_wait(&m->bar_sa_sf[b], par)) {
           ok = false;
           break;
         }
@@ -717,7 +737,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         const bool rescale = raise && mrow != -INFINITY;
         if (__any_sync(0xffffffffu, rescale)) {
           // every MMA into O_wg so far (tiles < st) must have completed
-          if (!mbar_wait(&m->bar_od[(st - 1) & 1], ((st - 1) >> 1) & 1, wctl)) {
+          if (!ew_wait(&m->bar_od[(st - 1) & 1], ((st - 1) >> 1) & 1)) {
             ok = false;
             break;
           }
@@ -748,15 +768,19 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
 #pragma unroll
           for (int c = 0; c < 16; c += 2) {
             // no valid key yet in this row: m = -inf and every x = -inf
-            const float p0 = mrow == -INFINITY ? 0.f : ex2(x[h][c] - mrow);
-            const float p1 = mrow == -INFINITY ? 0.f : ex2(x[h][c + 1] - mrow);
-            psum += p0 + p1;
+            float p0 = mrow == -INFINITY ? 0.f : ex2(x[h][c] - mrow);
+            float p1 = mrow == -INFINITY ? 0.f : ex2(x[h][c + 1] - mrow);
+            psum += p0 + p1;  // L over the ungated P
+            if constexpr (DROP) {  // O = sigma (R o P) V: sigma in the epilogue
+              if (!((kb[h] >> c) & 1u)) p0 = 0.f;
+              if (!((kb[h] >> (c + 1)) & 1u)) p1 = 0.f;
+            }
             oP[h][c / 2] = pack_bf16(p0, p1);
           }
         }
         lrow += psum;
         // P buffer b was last read by the MMAs of tile st - 2
-        if (st >= 2 && !mbar_wait(&m->bar_od[b], par ^ 1u, wctl)) {
+        if (st >= 2 && !ew_wait(&m->bar_od[b], par ^ 1u)) {
           ok = false;
           break;
         }
@@ -780,7 +804,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         const float f0 = m0 == -INFINITY ? 0.f : ex2(m0 - mm);
         const float f1 = m1 == -INFINITY ? 0.f : ex2(m1 - mm);
         const float lt = s_xchg[2 * BM + r] * f0 + s_xchg[3 * BM + r] * f1;
-        const float inv = row_ok ? 1.f / lt : 0.f;
+        const float inv = row_ok ? (DROP ? dsig : 1.f) / lt : 0.f;
 #pragma unroll 1
         for (int q = 0; q < D / 32; ++q) {
           const int cc = wg * (D / 2) + 16 * q;  // output columns of this warpgroup
@@ -805,7 +829,9 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
       // SF buffer of this tile (the statistics kernel alternates two)
       const int sfb = kStats ? (st & 1) : 0;
       const uint32_t sfcol = sfb ? kColSF1 : kColSF;
-      if (!mbar_wait(&m->bar_sa_sf[sfb], kStats ? ((st >> 1) & 1) : (st & 1), wctl)) {
+      uint32_t kb[2];
+      if constexpr (DROP) tile_keep((first_tile + st % ntiles) * BN, kb);
+      if (!ew_wait(&m->bar_sa_sf[sfb], kStats ? ((st >> 1) & 1) : (st & 1))) {
         ok = false;
         break;
       }
@@ -830,7 +856,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
       if constexpr (kStats) {
         // ---- row statistics: copy DC of the whole tile, release it, then
         // accumulate alpha = sum P F and E0 = sum P (C + F (dP - D))  (eq. 6)
-        if (!mbar_wait(&m->bar_sa_dc[0], st & 1, wctl)) {
+        if (!ew_wait(&m->bar_sa_dc[0], st & 1)) {
           ok = false;
           break;
         }
@@ -861,8 +887,14 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
               if (c + 1 < mlo || c + 1 >= mhi) pr.y = 0.f;
             }
             const float2 f = __fmul2_rn(pair(rF[h], c), tauv);
-            const float2 t = __fadd2_rn(pair(rdP[h], c), nDv);
-            const float2 pt0 = __ffma2_rn(f, t, pair(rC[h], c));  // Ptil0 = C + F (dP - D)
+            float2 dp = pair(rdP[h], c), cv = pair(rC[h], c);
+            if constexpr (DROP) {  // dP -> sigma R dP, C -> sigma R C
+              const float2 g = gate2(kb[h], c, dsig);
+              dp = __fmul2_rn(dp, g);
+              cv = __fmul2_rn(cv, g);
+            }
+            const float2 t = __fadd2_rn(dp, nDv);
+            const float2 pt0 = __ffma2_rn(f, t, cv);  // Ptil0 = C + F (dP - D)
             acc_a = __ffma2_rn(pr, f, acc_a);
             acc_e = __ffma2_rn(pr, pt0, acc_e);
           }
@@ -871,7 +903,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
           if (kDcHalves || h == 0) {
-            if (!mbar_wait(&m->bar_sa_dc[kDcHalves ? h : 0], st & 1, wctl)) {
+            if (!ew_wait(&m->bar_sa_dc[kDcHalves ? h : 0], st & 1)) {
               ok = false;
               break;
             }
@@ -932,14 +964,20 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
                 if (c + 1 < mlo || c + 1 >= mhi) pr.y = 0.f;
               }
               const float2 f = __fmul2_rn(pair(rF[h], c), tauv);
-              const float2 dp = pair(rdP, c);
+              float2 dp = pair(rdP, c), cv = pair(rC, c), gp = pr;
+              if constexpr (DROP) {  // dP, C and the dOtil operands gated by sigma R
+                const float2 g = gate2(kb[h], c, dsig);
+                dp = __fmul2_rn(dp, g);
+                cv = __fmul2_rn(cv, g);
+                gp = __fmul2_rn(pr, g);
+              }
               const float2 t = __fadd2_rn(dp, nDv);
               // Ptil = C + F (dP - D) - alpha dP ; Stil = P (Ptil - E) ; h = F - alpha
-              const float2 pt = __ffma2_rn(nalv, dp, __ffma2_rn(f, t, pair(rC, c)));
-              const float2 ph = __fmul2_rn(pr, __fadd2_rn(f, nalv));
+              const float2 pt = __ffma2_rn(nalv, dp, __ffma2_rn(f, t, cv));
+              const float2 ph = __fmul2_rn(gp, __fadd2_rn(f, nalv));
               const float2 stl = __fmul2_rn(pr, __fadd2_rn(pt, nEv));
               const float2 ds = __fmul2_rn(pr, t);
-              oP[c / 2] = pack_bf16(pr.x, pr.y);
+              oP[c / 2] = pack_bf16(gp.x, gp.y);
               oPh[c / 2] = pack_bf16(ph.x, ph.y);
               oSt[c / 2] = pack_bf16(stl.x, stl.y);
               odS[c / 2] = pack_bf16(ds.x, ds.y);
@@ -962,7 +1000,9 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
                 if (c < mlo || c >= mhi) pr.x = 0.f;
                 if (c + 1 < mlo || c + 1 >= mhi) pr.y = 0.f;
               }
-              const float2 ds = __fmul2_rn(pr, __fadd2_rn(pair(rdP, c), nDv));
+              float2 dp = pair(rdP, c);
+              if constexpr (DROP) dp = __fmul2_rn(dp, gate2(kb[h], c, dsig));
+              const float2 ds = __fmul2_rn(pr, __fadd2_rn(dp, nDv));
               odS[c / 2] = pack_bf16(ds.x, ds.y);
             }
             tmem_st8(R, odS);
@@ -1080,7 +1120,8 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
 }
 
 // ============================================================ column engine
-template <ColOp OP, int D>
+// DROP: attention dropout (App. "Extensions")
+template <ColOp OP, int D, bool DROP>
 __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant__ EngineParams p) {
   using C = ColCfg<OP, D>;
   constexpr bool kBob = OP == ColOp::BobPass2;
@@ -1397,12 +1438,30 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
     const uint32_t ta = lane_base_addr(tmem, warp);
     const float tau = p.scale;
     const float2 sl2v = splat(tau * kLog2e), tauv = splat(tau);
+    // dropout: keep bits of this key's 16 queries in each half of a query
+    // tile (computed before the tile's scores are waited for); gate sigma R
+    const DropKey dkey = {p.drop_k0, p.drop_k1, p.drop_thr4};
+    const float dsig = p.drop_sigma;
+    // with dropout the lanes of a warp exchange keep bits, so a wait that
+    // gives up makes the whole warp leave together
+    auto ew_wait = [&](uint64_t* bar, uint32_t par) -> bool {
+      const bool w = mbar_wait(bar, par, wctl);
+      if constexpr (DROP) return __all_sync(0xffffffffu, w);
+      return w;
+    };
     bool ok = true;
     for (int st = 0; ok && st < nsteps; ++st) {
       const int stage = st % C::NSTAGES;
+      uint32_t kb[2];
+      if constexpr (DROP) {
+        const int it = (first_tile + st % nsteps_h) * BN;
+        const uint32_t bhq = (uint32_t)(bh_q0 + st / nsteps_h);
+#pragma unroll
+        for (int h = 0; h < 2; ++h) kb[h] = keep_col16(gj, it + HB * h + 16 * wg, bhq, dkey);
+      }
       // the row vectors were written by the producer: acquire them explicitly
-      if (!mbar_wait(&m->bar_full_b[stage], (st / C::NSTAGES) & 1, wctl) ||
-          !mbar_wait(&m->bar_sa_sf[0], st & 1, wctl)) {
+      if (!ew_wait(&m->bar_full_b[stage], (st / C::NSTAGES) & 1) ||
+          !ew_wait(&m->bar_sa_sf[0], st & 1)) {
         ok = false;
         break;
       }
@@ -1424,7 +1483,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
       }
       tc_fence_before();
       mbar_arrive(&m->bar_sf_free[0]);
-      if (!mbar_wait(&m->bar_sa_dc[dc_sel(st)], dc_par(st), wctl)) {
+      if (!ew_wait(&m->bar_sa_dc[dc_sel(st)], dc_par(st))) {
         ok = false;
         break;
       }
@@ -1457,11 +1516,17 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
               if (c + 1 < lo || c + 1 >= hi) pr.y = 0.f;
             }
             const float2 f = __fmul2_rn(pair(rF[h], c), tauv);
-            const float2 dp = pair(rdP, c);
+            float2 dp = pair(rdP, c), cv = pair(rC, c), gp = pr;
+            if constexpr (DROP) {  // dP, C and the Vtil operand gated by sigma R
+              const float2 g = gate2(kb[h], c, dsig);
+              dp = __fmul2_rn(dp, g);
+              cv = __fmul2_rn(cv, g);
+              gp = __fmul2_rn(pr, g);
+            }
             const float2 t = __fadd2_rn(dp, nD);
             // Ptil = C + F (dP - D) - alpha dP ; Stil = P (Ptil - E) ; h = F - alpha
-            const float2 pt = __ffma2_rn(nal, dp, __ffma2_rn(f, t, pair(rC, c)));
-            const float2 ph = __fmul2_rn(pr, __fadd2_rn(f, nal));
+            const float2 pt = __ffma2_rn(nal, dp, __ffma2_rn(f, t, cv));
+            const float2 ph = __fmul2_rn(gp, __fadd2_rn(f, nal));
             const float2 stl = __fmul2_rn(pr, __fadd2_rn(pt, nE));
             const float2 ds = __fmul2_rn(pr, t);
             oPh[c / 2] = pack_bf16(ph.x, ph.y);
@@ -1485,8 +1550,14 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
               if (c < lo || c >= hi) pr.x = 0.f;
               if (c + 1 < lo || c + 1 >= hi) pr.y = 0.f;
             }
-            const float2 ds = __fmul2_rn(pr, __fadd2_rn(pair(rdP, c), nD));
-            oP[c / 2] = pack_bf16(pr.x, pr.y);
+            float2 dp = pair(rdP, c), gp = pr;
+            if constexpr (DROP) {  // dV = (sigma R o P)^T dO, dS = P (sigma R dP - D)
+              const float2 g = gate2(kb[h], c, dsig);
+              dp = __fmul2_rn(dp, g);
+              gp = __fmul2_rn(pr, g);
+            }
+            const float2 ds = __fmul2_rn(pr, __fadd2_rn(dp, nD));
+            oP[c / 2] = pack_bf16(gp.x, gp.y);
             odS[c / 2] = pack_bf16(ds.x, ds.y);
           }
           tmem_st8(R + 0, oP);

@@ -1,29 +1,33 @@
 // col_kernels.cu -- instantiations and launcher of the column-block engine:
 // first-backward dK and dV (eqs. 2-3), BoB Pass 2 (Algorithm 2, second
-// loop).
+// loop).  Each operation with and without dropout.
 #include "attn_engine.cuh"
 #include "launch.h"
 
 namespace fbob {
 
-template <ColOp OP, int D>
+template <ColOp OP, int D, bool DROP>
 static cudaError_t launch_one(const EngineParams& p, int nblocks, cudaStream_t s) {
   const int smem = launch_smem(ColCfg<OP, D>::SMEM_BYTES);
-  cudaError_t e = cudaFuncSetAttribute(col_engine<OP, D>,
+  cudaError_t e = cudaFuncSetAttribute(col_engine<OP, D, DROP>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  col_engine<OP, D><<<nblocks, kThreads, smem, s>>>(p);
+  col_engine<OP, D, DROP><<<nblocks, kThreads, smem, s>>>(p);
   return cudaGetLastError();
 }
 
-cudaError_t launch_col(ColOp op, int d, const EngineParams& p, int nblocks, cudaStream_t s) {
+template <ColOp OP>
+static cudaError_t launch_op(int d, bool drop, const EngineParams& p, int nblocks, cudaStream_t s) {
+  if (d == 64)
+    return drop ? launch_one<OP, 64, true>(p, nblocks, s) : launch_one<OP, 64, false>(p, nblocks, s);
+  return drop ? launch_one<OP, 128, true>(p, nblocks, s) : launch_one<OP, 128, false>(p, nblocks, s);
+}
+
+cudaError_t launch_col(ColOp op, int d, bool drop, const EngineParams& p, int nblocks,
+                       cudaStream_t s) {
   switch (op) {
-    case ColOp::BwdDKDV:
-      return d == 64 ? launch_one<ColOp::BwdDKDV, 64>(p, nblocks, s)
-                     : launch_one<ColOp::BwdDKDV, 128>(p, nblocks, s);
-    case ColOp::BobPass2:
-      return d == 64 ? launch_one<ColOp::BobPass2, 64>(p, nblocks, s)
-                     : launch_one<ColOp::BobPass2, 128>(p, nblocks, s);
+    case ColOp::BwdDKDV: return launch_op<ColOp::BwdDKDV>(d, drop, p, nblocks, s);
+    case ColOp::BobPass2: return launch_op<ColOp::BobPass2>(d, drop, p, nblocks, s);
   }
   return cudaErrorInvalidValue;
 }

@@ -56,6 +56,10 @@ struct EngineParams {
   unsigned long long wait_limit_ns;  // bound of every device-side wait
   int inject_stall;                  // fault injection: producers issue nothing
   int head_major;                    // CTA order: 1 = head-major, 0 = heads innermost
+  // dropout (kernels instantiated with it): Philox key, byte threshold t in
+  // each byte, and sigma = 256 / (256 - t)
+  uint32_t drop_k0, drop_k1, drop_thr4;
+  float drop_sigma;
 };
 
 // ---------------------------------------------------------------- configs

@@ -66,6 +66,7 @@ int check_shape(const fbob_shape* s, bool* empty) {
   if (s->causal != 0 && s->causal != 1) return FBOB_ERR_INVALID_ARGUMENT;
   if (s->window_left < -1 || s->window_right < -1) return FBOB_ERR_INVALID_ARGUMENT;
   if (s->H_kv < 0 || (s->H_kv > 0 && (s->H % s->H_kv) != 0)) return FBOB_ERR_INVALID_ARGUMENT;
+  if (!(s->dropout_p >= 0.0 && s->dropout_p < 1.0)) return FBOB_ERR_INVALID_ARGUMENT;
   if (s->seq_offsets == nullptr ? s->num_seqs != 0
                                 : (s->num_seqs < 1 || s->num_seqs > kMaxN ||
                                    (reinterpret_cast<uintptr_t>(s->seq_offsets) & 3u) != 0))
@@ -122,6 +123,14 @@ void choose_order(EngineParams* p, int head_major) { p->head_major = head_major;
 // key/value heads per batch entry
 int64_t kv_heads(const fbob_shape* s) { return s->H_kv > 0 ? s->H_kv : s->H; }
 
+// dropout byte threshold t = round(256 p), at most 255; 0 = no dropout
+uint32_t drop_threshold(const fbob_shape* s) {
+  const double t = std::floor(256.0 * s->dropout_p + 0.5);
+  return t >= 255.0 ? 255u : (uint32_t)t;
+}
+
+bool has_dropout(const fbob_shape* s) { return drop_threshold(s) != 0; }
+
 EngineParams base_params(const fbob_shape* s) {
   EngineParams p;
   std::memset(&p, 0, sizeof(p));
@@ -136,6 +145,11 @@ EngineParams base_params(const fbob_shape* s) {
   p.Hkv = (int)kv_heads(s);
   p.scale = s->scale;
   p.bhn = s->B * s->H * s->N;
+  const uint32_t t = drop_threshold(s);
+  p.drop_k0 = (uint32_t)(s->dropout_seed & 0xFFFFFFFFull);
+  p.drop_k1 = (uint32_t)(s->dropout_seed >> 32);
+  p.drop_thr4 = t * 0x01010101u;
+  p.drop_sigma = t ? (float)(256.0 / (256.0 - (double)t)) : 1.f;
   debug_controls(&p);
   return p;
 }
@@ -172,19 +186,23 @@ bool row_bob_params(const fbob_shape* s, const void* q, const void* k, const voi
 }
 
 // Row scalars alpha, E, D (eq. 6) into row_stats.
-int run_row_stats(EngineParams p, int d, float* row_stats, cudaStream_t st) {
+int run_row_stats(EngineParams p, int d, bool drop, float* row_stats, cudaStream_t st) {
   p.vec_out = row_stats;
-  return launch_status(launch_row(RowOp::BobStats, d, p, p.nblk * p.BH, st));
+  return launch_status(launch_row(RowOp::BobStats, d, drop, p, p.nblk * p.BH, st));
 }
 
 // Qtil, dOtil from eqs. (6)-(7) with the row scalars given in row_stats.
-int run_pass1_direct(EngineParams p, int d, const float* row_stats, void* q_bar,
+int run_pass1_direct(EngineParams p, int d, bool drop, const float* row_stats, void* q_bar,
                      void* dout_bar, cudaStream_t st) {
   p.vec_in = row_stats;
   p.out0 = static_cast<__nv_bfloat16*>(q_bar);
   p.out1 = static_cast<__nv_bfloat16*>(dout_bar);
-  return launch_status(launch_row(RowOp::BobPass1D, d, p, p.nblk * p.BH, st));
+  return launch_status(launch_row(RowOp::BobPass1D, d, drop, p, p.nblk * p.BH, st));
 }
+
+// Pass 1 in one sweep (the affine fusion, Prop. 3.1) at d = 64 without
+// dropout; otherwise row statistics + direct form
+bool pass1_one_sweep(const fbob_shape* s) { return s->d == 64 && !has_dropout(s); }
 
 int run_pass1(const fbob_shape* s, const void* q, const void* k, const void* v, const void* o,
               const float* lse, const void* dout, const void* gq, const void* gk,
@@ -192,22 +210,24 @@ int run_pass1(const fbob_shape* s, const void* q, const void* k, const void* v, 
               cudaStream_t st) {
   EngineParams p;
   if (!row_bob_params(s, q, k, v, o, lse, dout, gq, gk, gv, &p)) return FBOB_ERR_CUDA;
-  if (s->d == 64) {  // one sweep, affine fusion (Prop. 3.1)
+  if (pass1_one_sweep(s)) {  // one sweep, affine fusion (Prop. 3.1)
     p.out0 = static_cast<__nv_bfloat16*>(q_bar);
     p.out1 = static_cast<__nv_bfloat16*>(dout_bar);
     p.vec_out = row_stats;
-    return launch_status(launch_row(RowOp::BobPass1, (int)s->d, p, p.nblk * p.BH, st));
+    return launch_status(launch_row(RowOp::BobPass1, (int)s->d, false, p, p.nblk * p.BH, st));
   }
   // d = 128: the four accumulators of the one-sweep form do not fit TMEM next
-  // to the stage-A tiles.  First the row scalars (alpha, E, D), then Qtil and
-  // dOtil from eqs. (6)-(7) with those scalars known (two accumulators).
-  const int rc = run_row_stats(p, (int)s->d, row_stats, st);
+  // to the stage-A tiles; with dropout (any d) the direct form gates its
+  // operands tile by tile.  First the row scalars (alpha, E, D), then Qtil
+  // and dOtil from eqs. (6)-(7) with those scalars known (two accumulators).
+  const bool drop = has_dropout(s);
+  const int rc = run_row_stats(p, (int)s->d, drop, row_stats, st);
   if (rc != FBOB_OK) return rc;
-  return run_pass1_direct(p, (int)s->d, row_stats, q_bar, dout_bar, st);
+  return run_pass1_direct(p, (int)s->d, drop, row_stats, q_bar, dout_bar, st);
 }
 
 // kernels one pass-1 call enqueues
-int pass1_launches(int64_t d) { return d == 64 ? 1 : 2; }
+int pass1_launches(const fbob_shape* s) { return pass1_one_sweep(s) ? 1 : 2; }
 
 int run_pass2(const fbob_shape* s, const void* q, const void* k, const void* v, const float* lse,
               const void* dout, const void* gq, const void* gk, const void* gv,
@@ -228,7 +248,7 @@ int run_pass2(const fbob_shape* s, const void* q, const void* k, const void* v, 
   p.out1 = static_cast<__nv_bfloat16*>(v_bar);
   p.nblk = n_blocks(N, BM);
   choose_order(&p, 0);
-  return launch_status(launch_col(ColOp::BobPass2, (int)d, p, p.nblk * p.BH, st));
+  return launch_status(launch_col(ColOp::BobPass2, (int)d, has_dropout(s), p, p.nblk * p.BH, st));
 }
 
 }  // namespace
@@ -286,7 +306,7 @@ int fbob_attn_fwd(const fbob_shape* s, const void* q, const void* k, const void*
   p.vec_out = lse;
   p.nblk = n_blocks(s->N, BM);
   choose_order(&p, 0);
-  rc = launch_status(launch_row(RowOp::Fwd, (int)s->d, p, p.nblk * p.BH, stream));
+  rc = launch_status(launch_row(RowOp::Fwd, (int)s->d, has_dropout(s), p, p.nblk * p.BH, stream));
   if (rc == FBOB_OK) g_launches[kEntFwd] = 1;
   return rc;
 }
@@ -322,7 +342,7 @@ int fbob_attn_bwd(const fbob_shape* s, const void* q, const void* k, const void*
   p.vec_out = dstat;
   p.nblk = n_blocks(N, BM);
   choose_order(&p, 0);
-  rc = launch_status(launch_row(RowOp::BwdDQ, (int)d, p, p.nblk * p.BH, stream));
+  rc = launch_status(launch_row(RowOp::BwdDQ, (int)d, has_dropout(s), p, p.nblk * p.BH, stream));
   if (rc != FBOB_OK) return rc;
   // dK and dV: column-block pass
   EngineParams c = base_params(s);
@@ -336,7 +356,7 @@ int fbob_attn_bwd(const fbob_shape* s, const void* q, const void* k, const void*
   c.out1 = static_cast<__nv_bfloat16*>(dv);
   c.nblk = n_blocks(N, BM);
   choose_order(&c, 0);
-  rc = launch_status(launch_col(ColOp::BwdDKDV, (int)d, c, c.nblk * c.BH, stream));
+  rc = launch_status(launch_col(ColOp::BwdDKDV, (int)d, has_dropout(s), c, c.nblk * c.BH, stream));
   if (rc == FBOB_OK) g_launches[kEntBwd] = 2;
   return rc;
 }
@@ -361,7 +381,7 @@ int fbob_attn_bob_pass1(const fbob_shape* s, const void* q, const void* k, const
   rc = check_ptrs(in, inb, 9, out, outb, 3);
   if (rc != FBOB_OK) return rc;
   rc = run_pass1(s, q, k, v, o, lse, dout, gq, gk, gv, q_bar, dout_bar, row_stats, stream);
-  if (rc == FBOB_OK) g_launches[kEntPass1] = pass1_launches(s->d);
+  if (rc == FBOB_OK) g_launches[kEntPass1] = pass1_launches(s);
   return rc;
 }
 
@@ -411,7 +431,7 @@ int fbob_attn_bob_row_stats(const fbob_shape* s, const void* q, const void* k, c
   if (rc != FBOB_OK) return rc;
   EngineParams p;
   if (!row_bob_params(s, q, k, v, o, lse, dout, gq, gk, gv, &p)) return FBOB_ERR_CUDA;
-  rc = run_row_stats(p, (int)s->d, row_stats, stream);
+  rc = run_row_stats(p, (int)s->d, has_dropout(s), row_stats, stream);
   if (rc == FBOB_OK) g_launches[kEntRowStats] = 1;
   return rc;
 }
@@ -438,7 +458,7 @@ int fbob_attn_bob_pass1_direct(const fbob_shape* s, const void* q, const void* k
   EngineParams p;
   // (o is not read: D comes from row_stats)
   if (!row_bob_params(s, q, k, v, nullptr, lse, dout, gq, gk, gv, &p)) return FBOB_ERR_CUDA;
-  rc = run_pass1_direct(p, (int)s->d, row_stats, q_bar, dout_bar, stream);
+  rc = run_pass1_direct(p, (int)s->d, has_dropout(s), row_stats, q_bar, dout_bar, stream);
   if (rc == FBOB_OK) g_launches[kEntPass1D] = 1;
   return rc;
 }
@@ -468,7 +488,7 @@ int fbob_attn_bob(const fbob_shape* s, const void* q, const void* k, const void*
   // Pass 2 (column blocks): Ktil, Vtil from the saved row state.  Stream
   // order is the only synchronisation between the passes.
   rc = run_pass2(s, q, k, v, lse, dout, gq, gk, gv, row_stats, k_bar, v_bar, stream);
-  if (rc == FBOB_OK) g_launches[kEntBob] = pass1_launches(s->d) + 1;
+  if (rc == FBOB_OK) g_launches[kEntBob] = pass1_launches(s) + 1;
   return rc;
 }
 

@@ -12,8 +12,11 @@ namespace fbob {
 // least 120 KB, so that one CTA (holding all 512 TMEM columns) runs per SM.
 inline int launch_smem(int plan_bytes) { return plan_bytes > 120 * 1024 ? plan_bytes : 120 * 1024; }
 
-cudaError_t launch_row(RowOp op, int d, const EngineParams& p, int nblocks, cudaStream_t s);
-cudaError_t launch_col(ColOp op, int d, const EngineParams& p, int nblocks, cudaStream_t s);
+// drop: the instantiation with attention dropout (p.drop_* set)
+cudaError_t launch_row(RowOp op, int d, bool drop, const EngineParams& p, int nblocks,
+                       cudaStream_t s);
+cudaError_t launch_col(ColOp op, int d, bool drop, const EngineParams& p, int nblocks,
+                       cudaStream_t s);
 
 // Read and clear the error word of the row / column engine unit.
 cudaError_t take_row_error(uint32_t* word, cudaStream_t s);

@@ -1,37 +1,39 @@
 // row_kernels.cu -- instantiations and launcher of the row-block engine:
 // forward (eq. 1), first-backward dQ (eqs. 2-3), BoB Pass 1 (Algorithm 2,
-// first loop): one sweep at d = 64, row statistics + direct form at d = 128.
+// first loop): one sweep at d = 64, row statistics + direct form at d = 128
+// (and at d = 64 with dropout).  Each operation with and without dropout.
 #include "attn_engine.cuh"
 #include "launch.h"
 
 namespace fbob {
 
-template <RowOp OP, int D>
+template <RowOp OP, int D, bool DROP>
 static cudaError_t launch_one(const EngineParams& p, int nblocks, cudaStream_t s) {
   const int smem = launch_smem(RowCfg<OP, D>::SMEM_BYTES);
-  cudaError_t e = cudaFuncSetAttribute(row_engine<OP, D>,
+  cudaError_t e = cudaFuncSetAttribute(row_engine<OP, D, DROP>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  row_engine<OP, D><<<nblocks, kThreads, smem, s>>>(p);
+  row_engine<OP, D, DROP><<<nblocks, kThreads, smem, s>>>(p);
   return cudaGetLastError();
 }
 
-cudaError_t launch_row(RowOp op, int d, const EngineParams& p, int nblocks, cudaStream_t s) {
+template <RowOp OP>
+static cudaError_t launch_op(int d, bool drop, const EngineParams& p, int nblocks, cudaStream_t s) {
+  if (d == 64)
+    return drop ? launch_one<OP, 64, true>(p, nblocks, s) : launch_one<OP, 64, false>(p, nblocks, s);
+  return drop ? launch_one<OP, 128, true>(p, nblocks, s) : launch_one<OP, 128, false>(p, nblocks, s);
+}
+
+cudaError_t launch_row(RowOp op, int d, bool drop, const EngineParams& p, int nblocks,
+                       cudaStream_t s) {
   switch (op) {
-    case RowOp::Fwd:
-      return d == 64 ? launch_one<RowOp::Fwd, 64>(p, nblocks, s)
-                     : launch_one<RowOp::Fwd, 128>(p, nblocks, s);
-    case RowOp::BwdDQ:
-      return d == 64 ? launch_one<RowOp::BwdDQ, 64>(p, nblocks, s)
-                     : launch_one<RowOp::BwdDQ, 128>(p, nblocks, s);
-    case RowOp::BobPass1:  // the one-sweep form serves d = 64 only
-      return d == 64 ? launch_one<RowOp::BobPass1, 64>(p, nblocks, s) : cudaErrorInvalidValue;
-    case RowOp::BobStats:
-      return d == 64 ? launch_one<RowOp::BobStats, 64>(p, nblocks, s)
-                     : launch_one<RowOp::BobStats, 128>(p, nblocks, s);
-    case RowOp::BobPass1D:
-      return d == 64 ? launch_one<RowOp::BobPass1D, 64>(p, nblocks, s)
-                     : launch_one<RowOp::BobPass1D, 128>(p, nblocks, s);
+    case RowOp::Fwd: return launch_op<RowOp::Fwd>(d, drop, p, nblocks, s);
+    case RowOp::BwdDQ: return launch_op<RowOp::BwdDQ>(d, drop, p, nblocks, s);
+    case RowOp::BobPass1:  // the one-sweep form serves d = 64 without dropout only
+      return d == 64 && !drop ? launch_one<RowOp::BobPass1, 64, false>(p, nblocks, s)
+                              : cudaErrorInvalidValue;
+    case RowOp::BobStats: return launch_op<RowOp::BobStats>(d, drop, p, nblocks, s);
+    case RowOp::BobPass1D: return launch_op<RowOp::BobPass1D>(d, drop, p, nblocks, s);
   }
   return cudaErrorInvalidValue;
 }

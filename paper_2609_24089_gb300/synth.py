@@ -36,6 +36,7 @@ class Workload:
     window: tuple = (-1, -1)  # sliding-window band (left, right); -1 = unbounded
     segments: tuple = ()      # offsets of packed sequences along N; () = one sequence
     kv_heads: int = 0         # key/value heads (grouped-query attention); 0 = H
+    dropout: tuple = ()       # attention dropout (p, seed); () = none
 
     @property
     def scale(self) -> float:
@@ -85,6 +86,11 @@ def packed_offsets(N: int, n: int, seed: int) -> tuple:
 WORKLOADS["n16k_d128_causal_gqa4"] = Workload(
     "n16k_d128_causal_gqa4", 2, 16, 16384, 128, True, 7,
     _s(1, 1, 1, *(4 * [1 / math.sqrt(128)])), kv_heads=4)
+
+# dropout variant of n16k_d128_causal: p = 0.1 after the softmax
+WORKLOADS["n16k_d128_causal_drop10"] = Workload(
+    "n16k_d128_causal_drop10", 2, 16, 16384, 128, True, 8,
+    _s(1, 1, 1, *(4 * [1 / math.sqrt(128)])), dropout=(0.1, (8 << 32) | 8))
 
 WORKLOADS["n16k_d128_causal_varlen"] = Workload(
     "n16k_d128_causal_varlen", 2, 16, 16384, 128, True, 6,

@@ -139,3 +139,24 @@ def test_rejects_bad_kv_heads(lib):
     assert bob(lib, shape(4, -1), ptrs(14)) == 1
     assert bob(lib, shape(4, 2, N=0), ptrs(14)) == 0  # valid: empty problem, no call
     assert bob(lib, shape(4, 0, N=0), ptrs(14)) == 0  # 0 = no grouping
+
+
+def test_rejects_bad_dropout_rates(lib):
+    S = fbob.make_shape
+    for p in (1.0, 1.5, -0.01, float("nan"), float("inf")):
+        assert bob(lib, S(1, 1, 128, 64, 0.125, 0, dropout=(p, 3)), ptrs(14)) == 1, p
+        assert lib.fbob_attn_fwd(ctypes.byref(S(1, 1, 128, 64, 0.125, 0, dropout=(p, 3))),
+                                 *ptrs(5), None) == 1, p
+    # valid rates (and any 64-bit seed) pass validation, then stop at the empty problem
+    for p in (0.0, 0.001, 0.5, 0.999):
+        assert bob(lib, S(1, 1, 0, 64, 0.125, 1, dropout=(p, (1 << 64) - 1)), ptrs(14)) == 0
+
+
+def test_shape_struct_matches_the_header():
+    """The ctypes mirror lists the C struct's fields in the header's order."""
+    import re
+    text = open(fbob.HEADER).read()
+    body = re.search(r"typedef struct fbob_shape \{(.*?)\} fbob_shape;", text, re.S).group(1)
+    body = re.sub(r"/\*.*?\*/", "", body, flags=re.S)
+    declared = re.findall(r"(\w+)\s*(?=[,;])", body)
+    assert declared == [f[0] for f in fbob.fbob_shape._fields_]

@@ -204,3 +204,23 @@ def test_n16k_d128_causal_gqa4_rows_and_tail():
         vb += t["vbar"]
     G.check("kbar[kv head 1, tail]", r["kbar"][0, 1][t0:], kb)
     G.check("vbar[kv head 1, tail]", r["vbar"][0, 1][t0:], vb)
+
+
+def test_n16k_d128_causal_drop10_rows_and_tail():
+    """Dropout workload (p = 0.1) at full size: sampled rows of one head and
+    its causal tail, against the oracle with the same keep mask."""
+    w = synth.WORKLOADS["n16k_d128_causal_drop10"]
+    bits = synth.workload_inputs(w)
+    r = G.run_bob(bits, w.scale, w.causal, dropout=w.dropout)
+    assert r["status"] == 0
+    N = w.N
+    heads = [w.H + 3]  # batch entry 1, head 3
+    rows = sample_rows(N, 68)
+    check_rows(r, G.oracle_bob_heads(bits, w.scale, w.causal, heads, rows=rows,
+                                     dropout=w.dropout), heads, w.H, rows)
+    t0 = N - 256
+    tail = G.oracle_bob_heads(bits, w.scale, w.causal, heads, rows=np.arange(t0, N), cols=(t0, N),
+                              dropout=w.dropout)
+    for hh, ref in zip(heads, tail):
+        G.check("kbar[tail]", G.flat(r["kbar"], hh, w.H)[t0:], ref["kbar"])
+        G.check("vbar[tail]", G.flat(r["vbar"], hh, w.H)[t0:], ref["vbar"])
