@@ -259,7 +259,7 @@ def run_gpu(args, w):
 
     # ---- timed region: K steps, each as its kernels (through their C-ABI
     # calls, the same ones fbob_attn_bob makes) with events between them
-    if w.d == 64 and not drop:  # one-sweep Pass 1
+    if w.d <= 64 and not drop:  # one-sweep Pass 1 (as fbob_attn_bob_pass1 chooses)
         parts = [("pass1", lambda: fbob.fbob_attn_bob_pass1(
             shp, q, k, v, o, lse, do, gq, gk, gv, outs[0], outs[3], rs))]
     else:

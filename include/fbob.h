@@ -16,7 +16,9 @@
  *  Pointers   Device pointers (global memory of the current device), each
  *             16-byte aligned.  Outputs must not overlap any input or each
  *             other.
- *  Shapes     d in {64, 128}; other head dims return FBOB_ERR_UNSUPPORTED.
+ *  Shapes     d in {32, 64, 128}; other head dims return FBOB_ERR_UNSUPPORTED.
+ *             (d = 32 runs in the kernels' 64-wide tiles, the missing
+ *             columns loaded as zeros.)
  *             N >= 0 is arbitrary (tails are masked); B*H*N == 0 is a valid
  *             empty problem that launches nothing and returns FBOB_OK.
  *             N <= 2^24 and B*H <= 2^24.  scale must be finite and > 0
@@ -92,7 +94,7 @@ struct CUstream_st; /* cudaStream_t == struct CUstream_st* */
 typedef enum fbob_status {
     FBOB_OK = 0,
     FBOB_ERR_INVALID_ARGUMENT = 1, /* null/misaligned/overlapping pointer, bad shape, scale */
-    FBOB_ERR_UNSUPPORTED = 2,      /* valid request this build does not implement (d) */
+    FBOB_ERR_UNSUPPORTED = 2,      /* valid request this build does not implement (d not 32/64/128) */
     FBOB_ERR_CUDA = 3,             /* a CUDA runtime/driver call or launch failed */
     FBOB_ERR_DEVICE_TIMEOUT = 4,   /* a bounded device-side wait expired */
     FBOB_ERR_DEVICE_FAULT = 5      /* the device reported an error while synchronising */
@@ -155,7 +157,7 @@ int fbob_attn_bob(const fbob_shape* shape, const void* q, const void* k, const v
 /*
  * Pass 1 of Algorithm 1 alone (row-block outer; Alg. 2, first loop):
  * writes q_bar, dout_bar and row_stats (alpha, E, D).  Same arguments and
- * rules as fbob_attn_bob; k_bar/v_bar are not touched.  d = 64 without
+ * rules as fbob_attn_bob; k_bar/v_bar are not touched.  d <= 64 without
  * dropout runs one sweep with the affine fusion of Prop. 3.1 (one kernel);
  * d = 128, and any d with dropout, runs fbob_attn_bob_row_stats then
  * fbob_attn_bob_pass1_direct (two kernels).
@@ -180,8 +182,9 @@ int fbob_attn_bob_pass2(const fbob_shape* shape, const void* q, const void* k, c
 /*
  * Row scalars of BoB alone (eq. 6): writes row_stats [3,B,H,N] = (alpha, E, D)
  * with alpha_i = sum_j P_ij F_ij, E_i = sum_j P_ij Ptil_ij and D_i = do_i . o_i,
- * exactly as pass 1 writes them (stage A only; no N x d output).  At d = 128
- * fbob_attn_bob_pass1 is this call followed by fbob_attn_bob_pass1_direct.
+ * exactly as pass 1 writes them (stage A only; no N x d output).  At d = 128,
+ * and with dropout, fbob_attn_bob_pass1 is this call followed by
+ * fbob_attn_bob_pass1_direct.
  * Same arguments and rules as fbob_attn_bob_pass1.
  */
 int fbob_attn_bob_row_stats(const fbob_shape* shape, const void* q, const void* k,

@@ -190,10 +190,15 @@ __device__ __forceinline__ float2 probs2(float2 s, float2 sl2, float2 nL2) {
 }
 
 // ============================================================== row engine
-// DROP: attention dropout (App. "Extensions"); the one-sweep Pass 1 has none
-template <RowOp OP, int D, bool DROP>
+// D: head dimension of the tiles (64 or 128); DG <= D: head dimension of the
+// tensors in global memory.  DG = 32 runs in the D = 64 tiles: the TMA loads
+// fill columns 32..63 with zeros, which add nothing to any contraction, and
+// only the first DG columns are read or written directly.
+// DROP: attention dropout (App. "Extensions"); the one-sweep Pass 1 has none.
+template <RowOp OP, int D, bool DROP, int DG>
 __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant__ EngineParams p) {
   using C = RowCfg<OP, D>;
+  static_assert(DG == D || (DG == 32 && D == 64), "global head dim 32 runs in 64-wide tiles");
   static_assert(!DROP || OP != RowOp::BobPass1, "dropout Pass 1 runs as statistics + direct");
   constexpr bool kBob = OP == RowOp::BobPass1;      // Pass 1, one sweep (Prop. 3.1)
   constexpr bool kStats = OP == RowOp::BobStats;    // row scalars alpha, E, D only
@@ -636,7 +641,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
       if (p.wr >= 0) jhi = min(jhi, gi + p.wr + 1);
     }
     const uint32_t ta = lane_base_addr(tmem, warp);
-    const size_t rowoff = ((size_t)bh * N + (size_t)(row_ok ? gi : 0)) * D;
+    const size_t rowoff = ((size_t)bh * N + (size_t)(row_ok ? gi : 0)) * DG;
     const float tau = p.scale;
     const float sl2 = tau * kLog2e;
     // dropout: keep bits of this row's 16 keys in each half of key tile jt
@@ -664,7 +669,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
           nE = -p.vec_in[p.bhn + ri];
           Dr = p.vec_in[2 * p.bhn + ri];
         } else {
-          Dr = row_dot<D>(p.dout + rowoff, p.o + rowoff);
+          Dr = row_dot<DG>(p.dout + rowoff, p.o + rowoff);
         }
       }
     }
@@ -677,7 +682,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
 #pragma unroll 1
         for (int c = c0; c < c0 + ncols; c += 8) {
           uint4 a = make_uint4(0, 0, 0, 0), b = a;
-          if (row_ok) {
+          if (row_ok && 2 * c < DG) {  // zero columns past the tensor's head dim
             a = src[c / 4];
             b = src[c / 4 + 1];
           }
@@ -813,7 +818,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
           tmem_ld16(ta + D + cc, a1);
           tmem_ld_wait(a0);
           reg_dep(a1);
-          if (row_ok) {
+          if (row_ok && cc < DG) {
             float v[16];
 #pragma unroll
             for (int c = 0; c < 16; ++c) v[c] = (bits_f(a0[c]) * f0 + bits_f(a1[c]) * f1) * inv;
@@ -1041,7 +1046,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
           reg_dep(rO);
           reg_dep(rG);
           reg_dep(rW);
-          if (row_ok) {
+          if (row_ok && cbase + 16 * q < DG) {
             float ov[16], qt[16], dot[16];
             load_row16(p.o + rowoff + cbase + 16 * q, ov);
 #pragma unroll
@@ -1080,7 +1085,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
           tmem_ld16(ta + D + cc, rO);
           tmem_ld_wait(rQ);
           reg_dep(rO);
-          if (row_ok) {
+          if (row_ok && cc < DG) {
             float qt[16], dot[16];
 #pragma unroll
             for (int c = 0; c < 16; ++c) {
@@ -1099,7 +1104,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
           uint32_t rA[16];
           tmem_ld16(ta + cc, rA);
           tmem_ld_wait(rA);
-          if (row_ok) {
+          if (row_ok && cc < DG) {
             float v[16];
 #pragma unroll
             for (int c = 0; c < 16; ++c) v[c] = tau * bits_f(rA[c]);
@@ -1120,10 +1125,11 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
 }
 
 // ============================================================ column engine
-// DROP: attention dropout (App. "Extensions")
-template <ColOp OP, int D, bool DROP>
+// D, DG as in the row engine; DROP: attention dropout (App. "Extensions")
+template <ColOp OP, int D, bool DROP, int DG>
 __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant__ EngineParams p) {
   using C = ColCfg<OP, D>;
+  static_assert(DG == D || (DG == 32 && D == 64), "global head dim 32 runs in 64-wide tiles");
   constexpr bool kBob = OP == ColOp::BobPass2;
   extern __shared__ __align__(1024) uint8_t smem[];
   uint8_t* s_stat = smem;
@@ -1572,7 +1578,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
     if (ok && *abort_flag) ok = false;
     tc_fence_after();
     if (ok) {
-      const size_t rowoff = ((size_t)bh * N + (size_t)(row_ok ? gj : 0)) * D;
+      const size_t rowoff = ((size_t)bh * N + (size_t)(row_ok ? gj : 0)) * DG;
 #pragma unroll 1
       for (int q = 0; q < D / 32; ++q) {
         const int cc = wg * (D / 2) + 16 * q;
@@ -1581,7 +1587,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
         tmem_ld16(ta + D + cc, rV);
         tmem_ld_wait(rK);
         reg_dep(rV);
-        if (row_ok) {
+        if (row_ok && cc < DG) {
           float kv[16], vv[16];
 #pragma unroll
           for (int c = 0; c < 16; ++c) {

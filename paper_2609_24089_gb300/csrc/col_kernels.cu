@@ -1,26 +1,36 @@
 // col_kernels.cu -- instantiations and launcher of the column-block engine:
 // first-backward dK and dV (eqs. 2-3), BoB Pass 2 (Algorithm 2, second
-// loop).  Each operation with and without dropout.
+// loop).  Each operation with and without dropout, for head dims 32 (in
+// 64-wide tiles), 64 and 128.
 #include "attn_engine.cuh"
 #include "launch.h"
 
 namespace fbob {
 
-template <ColOp OP, int D, bool DROP>
+// D: tile head dimension; DG: the tensors' head dimension (32 runs in 64-wide tiles)
+template <ColOp OP, int D, bool DROP, int DG = D>
 static cudaError_t launch_one(const EngineParams& p, int nblocks, cudaStream_t s) {
   const int smem = launch_smem(ColCfg<OP, D>::SMEM_BYTES);
-  cudaError_t e = cudaFuncSetAttribute(col_engine<OP, D, DROP>,
+  cudaError_t e = cudaFuncSetAttribute(col_engine<OP, D, DROP, DG>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  col_engine<OP, D, DROP><<<nblocks, kThreads, smem, s>>>(p);
+  col_engine<OP, D, DROP, DG><<<nblocks, kThreads, smem, s>>>(p);
   return cudaGetLastError();
+}
+
+template <ColOp OP, bool DROP>
+static cudaError_t launch_d(int d, const EngineParams& p, int nblocks, cudaStream_t s) {
+  switch (d) {
+    case 32: return launch_one<OP, 64, DROP, 32>(p, nblocks, s);
+    case 64: return launch_one<OP, 64, DROP>(p, nblocks, s);
+    case 128: return launch_one<OP, 128, DROP>(p, nblocks, s);
+  }
+  return cudaErrorInvalidValue;
 }
 
 template <ColOp OP>
 static cudaError_t launch_op(int d, bool drop, const EngineParams& p, int nblocks, cudaStream_t s) {
-  if (d == 64)
-    return drop ? launch_one<OP, 64, true>(p, nblocks, s) : launch_one<OP, 64, false>(p, nblocks, s);
-  return drop ? launch_one<OP, 128, true>(p, nblocks, s) : launch_one<OP, 128, false>(p, nblocks, s);
+  return drop ? launch_d<OP, true>(d, p, nblocks, s) : launch_d<OP, false>(d, p, nblocks, s);
 }
 
 cudaError_t launch_col(ColOp op, int d, bool drop, const EngineParams& p, int nblocks,

@@ -37,7 +37,8 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 }
 
 // [BH, N, d] bf16 tensor viewed as 3-D (d innermost), box = 64 columns x `rows`,
-// 128-byte swizzle, zero fill out of bounds.
+// 128-byte swizzle, zero fill out of bounds (with d = 32 the box's columns
+// 32..63 lie outside the tensor and arrive as zeros).
 bool make_map(CUtensorMap* m, const void* base, int64_t BH, int64_t N, int64_t d, int rows) {
   auto enc = encode_fn();
   if (!enc) return false;
@@ -71,7 +72,7 @@ int check_shape(const fbob_shape* s, bool* empty) {
                                 : (s->num_seqs < 1 || s->num_seqs > kMaxN ||
                                    (reinterpret_cast<uintptr_t>(s->seq_offsets) & 3u) != 0))
     return FBOB_ERR_INVALID_ARGUMENT;
-  if (s->d != 64 && s->d != 128) return FBOB_ERR_UNSUPPORTED;
+  if (s->d != 32 && s->d != 64 && s->d != 128) return FBOB_ERR_UNSUPPORTED;
   if (s->N > kMaxN) return FBOB_ERR_INVALID_ARGUMENT;
   if (s->B > kMaxBH || s->H > kMaxBH || s->B * s->H > kMaxBH) return FBOB_ERR_INVALID_ARGUMENT;
   *empty = (s->B * s->H * s->N) == 0;
@@ -200,9 +201,9 @@ int run_pass1_direct(EngineParams p, int d, bool drop, const float* row_stats, v
   return launch_status(launch_row(RowOp::BobPass1D, d, drop, p, p.nblk * p.BH, st));
 }
 
-// Pass 1 in one sweep (the affine fusion, Prop. 3.1) at d = 64 without
+// Pass 1 in one sweep (the affine fusion, Prop. 3.1) at d <= 64 without
 // dropout; otherwise row statistics + direct form
-bool pass1_one_sweep(const fbob_shape* s) { return s->d == 64 && !has_dropout(s); }
+bool pass1_one_sweep(const fbob_shape* s) { return s->d <= 64 && !has_dropout(s); }
 
 int run_pass1(const fbob_shape* s, const void* q, const void* k, const void* v, const void* o,
               const float* lse, const void* dout, const void* gq, const void* gk,

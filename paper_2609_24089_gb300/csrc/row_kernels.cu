@@ -1,27 +1,37 @@
 // row_kernels.cu -- instantiations and launcher of the row-block engine:
 // forward (eq. 1), first-backward dQ (eqs. 2-3), BoB Pass 1 (Algorithm 2,
-// first loop): one sweep at d = 64, row statistics + direct form at d = 128
-// (and at d = 64 with dropout).  Each operation with and without dropout.
+// first loop): one sweep at d <= 64, row statistics + direct form at d = 128
+// (and at any d with dropout).  Each operation with and without dropout, for
+// head dims 32 (in 64-wide tiles), 64 and 128.
 #include "attn_engine.cuh"
 #include "launch.h"
 
 namespace fbob {
 
-template <RowOp OP, int D, bool DROP>
+// D: tile head dimension; DG: the tensors' head dimension (32 runs in 64-wide tiles)
+template <RowOp OP, int D, bool DROP, int DG = D>
 static cudaError_t launch_one(const EngineParams& p, int nblocks, cudaStream_t s) {
   const int smem = launch_smem(RowCfg<OP, D>::SMEM_BYTES);
-  cudaError_t e = cudaFuncSetAttribute(row_engine<OP, D, DROP>,
+  cudaError_t e = cudaFuncSetAttribute(row_engine<OP, D, DROP, DG>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  row_engine<OP, D, DROP><<<nblocks, kThreads, smem, s>>>(p);
+  row_engine<OP, D, DROP, DG><<<nblocks, kThreads, smem, s>>>(p);
   return cudaGetLastError();
+}
+
+template <RowOp OP, bool DROP>
+static cudaError_t launch_d(int d, const EngineParams& p, int nblocks, cudaStream_t s) {
+  switch (d) {
+    case 32: return launch_one<OP, 64, DROP, 32>(p, nblocks, s);
+    case 64: return launch_one<OP, 64, DROP>(p, nblocks, s);
+    case 128: return launch_one<OP, 128, DROP>(p, nblocks, s);
+  }
+  return cudaErrorInvalidValue;
 }
 
 template <RowOp OP>
 static cudaError_t launch_op(int d, bool drop, const EngineParams& p, int nblocks, cudaStream_t s) {
-  if (d == 64)
-    return drop ? launch_one<OP, 64, true>(p, nblocks, s) : launch_one<OP, 64, false>(p, nblocks, s);
-  return drop ? launch_one<OP, 128, true>(p, nblocks, s) : launch_one<OP, 128, false>(p, nblocks, s);
+  return drop ? launch_d<OP, true>(d, p, nblocks, s) : launch_d<OP, false>(d, p, nblocks, s);
 }
 
 cudaError_t launch_row(RowOp op, int d, bool drop, const EngineParams& p, int nblocks,
@@ -29,9 +39,11 @@ cudaError_t launch_row(RowOp op, int d, bool drop, const EngineParams& p, int nb
   switch (op) {
     case RowOp::Fwd: return launch_op<RowOp::Fwd>(d, drop, p, nblocks, s);
     case RowOp::BwdDQ: return launch_op<RowOp::BwdDQ>(d, drop, p, nblocks, s);
-    case RowOp::BobPass1:  // the one-sweep form serves d = 64 without dropout only
-      return d == 64 && !drop ? launch_one<RowOp::BobPass1, 64, false>(p, nblocks, s)
-                              : cudaErrorInvalidValue;
+    case RowOp::BobPass1:  // the one-sweep form serves d <= 64 without dropout only
+      if (drop) return cudaErrorInvalidValue;
+      return d == 64   ? launch_one<RowOp::BobPass1, 64, false>(p, nblocks, s)
+             : d == 32 ? launch_one<RowOp::BobPass1, 64, false, 32>(p, nblocks, s)
+                       : cudaErrorInvalidValue;
     case RowOp::BobStats: return launch_op<RowOp::BobStats>(d, drop, p, nblocks, s);
     case RowOp::BobPass1D: return launch_op<RowOp::BobPass1D>(d, drop, p, nblocks, s);
   }

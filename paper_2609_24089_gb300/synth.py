@@ -92,6 +92,12 @@ WORKLOADS["n16k_d128_causal_drop10"] = Workload(
     "n16k_d128_causal_drop10", 2, 16, 16384, 128, True, 8,
     _s(1, 1, 1, *(4 * [1 / math.sqrt(128)])), dropout=(0.1, (8 << 32) | 8))
 
+# head-dimension sweep at the shape of the paper's sensitivity table
+# (App. "Head-dimension sensitivity": N = 4096, B = 4, H = 12, causal)
+for _d in (32, 64, 128):
+    WORKLOADS[f"n4k_d{_d}_causal_b4h12"] = Workload(
+        f"n4k_d{_d}_causal_b4h12", 4, 12, 4096, _d, True, 9, _s(1, 1, 1, 1, 1, 1, 1))
+
 WORKLOADS["n16k_d128_causal_varlen"] = Workload(
     "n16k_d128_causal_varlen", 2, 16, 16384, 128, True, 6,
     _s(1, 1, 1, *(4 * [1 / math.sqrt(128)])), segments=packed_offsets(16384, 12, 6))

@@ -48,7 +48,8 @@ def bob(lib, shape, ps):
 
 def test_rejects_bad_shapes(lib):
     S = fbob.make_shape
-    assert bob(lib, S(1, 1, 128, 32, 0.17, 0), ptrs(14)) == 2          # d unsupported
+    assert bob(lib, S(1, 1, 128, 48, 0.14, 0), ptrs(14)) == 2          # d unsupported
+    assert bob(lib, S(1, 1, 128, 16, 0.25, 0), ptrs(14)) == 2
     assert bob(lib, S(1, 1, 128, 256, 0.06, 1), ptrs(14)) == 2
     assert bob(lib, S(1, 1, 128, 64, 0.0, 0), ptrs(14)) == 1           # scale <= 0
     assert bob(lib, S(1, 1, 128, 64, float("nan"), 0), ptrs(14)) == 1
@@ -160,3 +161,9 @@ def test_shape_struct_matches_the_header():
     body = re.sub(r"/\*.*?\*/", "", body, flags=re.S)
     declared = re.findall(r"(\w+)\s*(?=[,;])", body)
     assert declared == [f[0] for f in fbob.fbob_shape._fields_]
+
+
+def test_head_dim_32_passes_validation(lib):
+    S = fbob.make_shape
+    assert bob(lib, S(1, 1, 0, 32, 0.17, 1), ptrs(14)) == 0  # valid: empty problem, no call
+    assert bob(lib, S(1, 1, 128, 32, 0.17, 1), ptrs(14, misalign=3)) == 1

@@ -224,3 +224,16 @@ def test_n16k_d128_causal_drop10_rows_and_tail():
     for hh, ref in zip(heads, tail):
         G.check("kbar[tail]", G.flat(r["kbar"], hh, w.H)[t0:], ref["kbar"])
         G.check("vbar[tail]", G.flat(r["vbar"], hh, w.H)[t0:], ref["vbar"])
+
+
+def test_n4k_d32_causal_b4h12_two_heads():
+    """Head dim 32 at the head-dimension sweep's shape: two full heads."""
+    w = synth.WORKLOADS["n4k_d32_causal_b4h12"]
+    bits = synth.workload_inputs(w)
+    r = G.run_bob(bits, w.scale, w.causal)
+    assert r["status"] == 0
+    heads = [1, w.B * w.H - 2]
+    refs = G.oracle_bob_heads(bits, w.scale, w.causal, heads)
+    for hh, ref in zip(heads, refs):
+        for name in ("qbar", "kbar", "vbar", "dobar", "alpha", "E", "D"):
+            G.check(f"{name}[head {hh}]", G.flat(r[name], hh, w.H), ref[name])

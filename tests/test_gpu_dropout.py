@@ -22,6 +22,8 @@ CASES = [  # B, H, N, d, causal, p, seed, window, kv_heads
     (1, 1, 333, 128, False, 0.25, 99, (60, 45), None),
     (1, 4, 260, 128, True, 0.15, 5, None, 2),
     (2, 2, 130, 64, True, 0.9, 31337, None, None),
+    (1, 2, 280, 32, True, 0.3, 77, None, None),
+    (1, 4, 150, 32, False, 0.2, 78, (30, 30), 2),
 ]
 
 
@@ -92,7 +94,7 @@ def test_bob_with_dropout_packed_sequences():
         G.check(name, r[name], x)
 
 
-@pytest.mark.parametrize("d", [64, 128])
+@pytest.mark.parametrize("d", [32, 64, 128])
 def test_keep_mask_bit_exact_in_both_engines(d):
     """Zeros of O and dV are the keep mask, pair by pair.  Q = 0 makes P
     uniform over each row's keys; with V rows one-hot in (j mod d) and the

@@ -17,6 +17,7 @@ CASES = [  # B, H, H_kv, N, d, causal, window
     (1, 8, 2, 520, 128, True, (100, -1)),
     (1, 4, 1, 700, 64, False, None),
     (2, 2, 2, 200, 64, True, None),
+    (1, 6, 2, 270, 32, True, None),
 ]
 
 

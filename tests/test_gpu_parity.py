@@ -22,6 +22,9 @@ SHAPES = [  # B, H, N, d, causal
     (1, 1, 3, 128, True),
     (2, 2, 384, 128, False),
     (1, 2, 520, 64, True),
+    (1, 1, 128, 32, False),   # head dim 32 (in 64-wide tiles)
+    (1, 2, 301, 32, True),
+    (2, 1, 3, 32, False),
 ]
 
 
@@ -67,7 +70,8 @@ def test_bob_end_to_end(shape):
         G.check(name, r[name], x)
 
 
-@pytest.mark.parametrize("shape", [(1, 2, 300, 64, True), (2, 1, 200, 128, False)], ids=ids)
+@pytest.mark.parametrize("shape", [(1, 2, 300, 64, True), (2, 1, 200, 128, False),
+                                   (1, 1, 190, 32, True)], ids=ids)
 def test_pass2_alone_on_oracle_row_state(shape):
     """Algorithm 2's second loop fed the oracle's L, D, alpha, E."""
     B, H, N, d, causal = shape

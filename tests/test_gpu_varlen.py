@@ -18,6 +18,7 @@ CASES = [  # B, H, N, d, causal, window, offsets
     (2, 1, 333, 128, True, (40, -1), [0, 50, 50, 333]),
     (1, 2, 300, 64, False, (20, 20), [0, 10, 20, 30, 300]),
     (1, 1, 1000, 128, True, None, [0, 64, 65, 300, 301, 777, 1000]),
+    (1, 2, 400, 32, True, None, [0, 33, 200, 400]),
 ]
 
 

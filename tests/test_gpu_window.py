@@ -19,6 +19,7 @@ CASES = [  # B, H, N, d, causal, (wl, wr)
     (1, 1, 400, 128, True, (5, -1)),
     (1, 2, 700, 128, False, (130, 200)),
     (2, 1, 200, 128, False, (1, 1)),
+    (1, 2, 330, 32, True, (90, -1)),
 ]
 
 
