@@ -646,7 +646,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
     const float sl2 = tau * kLog2e;
     // dropout: keep bits of this row's 16 keys in each half of key tile jt
     // (computed before the tile's scores are waited for); gate sigma R
-    const DropKey dkey = {p.drop_k0, p.drop_k1, p.drop_thr4};
+    const DropKey dkey = {p.drop_rk, p.drop_tlow4, p.drop_tmask};
     const float dsig = p.drop_sigma;
     auto tile_keep = [&](int jt, uint32_t (&kb)[2]) {
 #pragma unroll
@@ -1446,7 +1446,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
     const float2 sl2v = splat(tau * kLog2e), tauv = splat(tau);
     // dropout: keep bits of this key's 16 queries in each half of a query
     // tile (computed before the tile's scores are waited for); gate sigma R
-    const DropKey dkey = {p.drop_k0, p.drop_k1, p.drop_thr4};
+    const DropKey dkey = {p.drop_rk, p.drop_tlow4, p.drop_tmask};
     const float dsig = p.drop_sigma;
     // with dropout the lanes of a warp exchange keep bits, so a wait that
     // gives up makes the whole warp leave together

@@ -22,35 +22,43 @@
 namespace fbob {
 
 // Philox4x32-10 (Salmon, Moraes, Dror and Shaw, SC'11): ten rounds of the
-// Philox S-box; the key is raised by the Weyl constants before each round
-// after the first.
-__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1) {
+// Philox S-box.  rk[2r], rk[2r + 1] is the key of round r: the seed raised r
+// times by the Weyl constants 0x9E3779B9, 0xBB67AE85 (formed on the host, so
+// the kernels read them from the parameter bank).
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, const uint32_t (&rk)[20]) {
 #pragma unroll
   for (int r = 0; r < 10; ++r) {
-    if (r > 0) {
-      k0 += 0x9E3779B9u;
-      k1 += 0xBB67AE85u;
-    }
     const uint32_t lo0 = 0xD2511F53u * c.x, hi0 = __umulhi(0xD2511F53u, c.x);
     const uint32_t lo1 = 0xCD9E8D57u * c.z, hi1 = __umulhi(0xCD9E8D57u, c.z);
-    c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
+    c = make_uint4(hi1 ^ c.y ^ rk[2 * r], lo1, hi0 ^ c.w ^ rk[2 * r + 1], lo0);
   }
   return c;
 }
 
 struct DropKey {
-  uint32_t k0, k1;  // Philox key (the seed)
-  uint32_t thr4;    // byte threshold t in each of the four bytes
+  const uint32_t (&rk)[20];  // round keys (kernel parameters)
+  uint32_t tlow4;            // (t mod 128) in each byte
+  uint32_t tmask;            // all ones if t < 128, else zero
 };
+
+// Per byte of x: most significant bit set iff the byte is >= t.  r's bytes
+// (x | 0x80) - (t mod 128) compare the low seven bits without borrows; the
+// top bits then decide: x >= t iff (x7 or r7) when t < 128, (x7 and r7)
+// otherwise, i.e. the majority of x7, r7 and the t < 128 flag.
+__device__ __forceinline__ uint32_t bytes_ge(uint32_t x, const DropKey& k) {
+  const uint32_t r = (x | 0x80808080u) - k.tlow4;
+  return (x & r) | (k.tmask & (x | r));
+}
 
 // Keep bits of block (I, J) of query head `head`: bit 4a + b keeps the pair
 // (query 4I + a, key 4J + b).
 __device__ __forceinline__ uint32_t keep_block(uint32_t I, uint32_t J, uint32_t head,
                                                const DropKey& k) {
-  const uint4 w = philox4x32_10(make_uint4(J, I, head, 0u), k.k0, k.k1);
-  // per byte 0xFF where byte >= t; byte b's bit b, summed into the top byte
+  const uint4 w = philox4x32_10(make_uint4(J, I, head, 0u), k.rk);
+  // bytes' top bits 7, 15, 23, 31 gathered to 28..31 by one multiply
+  // (partial products land on distinct lower bits, so nothing carries)
   auto nib = [&](uint32_t x) -> uint32_t {
-    return ((__vcmpgeu4(x, k.thr4) & 0x08040201u) * 0x01010101u) >> 24;
+    return ((bytes_ge(x, k) & 0x80808080u) * 0x00204081u) >> 28;
   };
   return nib(w.x) | (nib(w.y) << 4) | (nib(w.z) << 8) | (nib(w.w) << 12);
 }
@@ -65,7 +73,7 @@ __device__ __forceinline__ uint32_t keep_row16(int i, int j0, uint32_t head, con
 #pragma unroll
   for (int s = 0; s < 4; ++s) {  // block s holds keys j0 + 4s .. + 3
     const uint32_t ms = __shfl_sync(0xffffffffu, mine, s, 4);
-    own |= ((ms >> (4 * t)) & 0xFu) << (4 * s);
+    own += ((ms >> (4 * t)) & 0xFu) << (4 * s);
   }
   return own;
 }
@@ -81,8 +89,10 @@ __device__ __forceinline__ uint32_t keep_col16(int j, int i0, uint32_t head, con
 #pragma unroll
   for (int s = 0; s < 4; ++s) {  // block s holds queries i0 + 4s .. + 3
     const uint32_t ms = __shfl_sync(0xffffffffu, mine, s, 4);
-    const uint32_t x = (ms >> t) & 0x1111u;  // bits 4a + t, a = 0..3
-    own |= ((x | (x >> 3) | (x >> 6) | (x >> 9)) & 0xFu) << (4 * s);
+    // bits 4a + t (a = 0..3) to bits 12 + a: multiply by 2^12 + 2^9 + 2^6 + 2^3
+    // (the other partial products fall on distinct bits outside 12..15)
+    const uint32_t x = (ms >> t) & 0x1111u;
+    own += ((x * 0x1248u) >> 12 & 0xFu) << (4 * s);
   }
   return own;
 }

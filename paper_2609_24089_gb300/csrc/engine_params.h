@@ -56,9 +56,12 @@ struct EngineParams {
   unsigned long long wait_limit_ns;  // bound of every device-side wait
   int inject_stall;                  // fault injection: producers issue nothing
   int head_major;                    // CTA order: 1 = head-major, 0 = heads innermost
-  // dropout (kernels instantiated with it): Philox key, byte threshold t in
-  // each byte, and sigma = 256 / (256 - t)
-  uint32_t drop_k0, drop_k1, drop_thr4;
+  // dropout (kernels instantiated with it): Philox round keys (the seed
+  // raised r times by the Weyl constants, r = 0..9), the byte threshold t as
+  // (t mod 128) in each byte and a flag (all ones if t < 128), and
+  // sigma = 256 / (256 - t)
+  uint32_t drop_rk[20];
+  uint32_t drop_tlow4, drop_tmask;
   float drop_sigma;
 };
 

@@ -147,9 +147,16 @@ EngineParams base_params(const fbob_shape* s) {
   p.scale = s->scale;
   p.bhn = s->B * s->H * s->N;
   const uint32_t t = drop_threshold(s);
-  p.drop_k0 = (uint32_t)(s->dropout_seed & 0xFFFFFFFFull);
-  p.drop_k1 = (uint32_t)(s->dropout_seed >> 32);
-  p.drop_thr4 = t * 0x01010101u;
+  uint32_t k0 = (uint32_t)(s->dropout_seed & 0xFFFFFFFFull);
+  uint32_t k1 = (uint32_t)(s->dropout_seed >> 32);
+  for (int r = 0; r < 10; ++r) {  // Philox4x32-10 key schedule (Weyl sequence)
+    p.drop_rk[2 * r] = k0;
+    p.drop_rk[2 * r + 1] = k1;
+    k0 += 0x9E3779B9u;
+    k1 += 0xBB67AE85u;
+  }
+  p.drop_tlow4 = (t & 0x7Fu) * 0x01010101u;
+  p.drop_tmask = t < 128 ? 0xFFFFFFFFu : 0u;
   p.drop_sigma = t ? (float)(256.0 / (256.0 - (double)t)) : 1.f;
   debug_controls(&p);
   return p;
