@@ -207,6 +207,42 @@ int fbob_attn_bob_pass1_direct(const fbob_shape* shape, const void* q, const voi
                                struct CUstream_st* stream);
 
 /*
+ * fbob_attn_bob with every tensor in host memory: the same computation and
+ * the same results, bit for bit.  The B*H query heads are processed in
+ * chunks of whole key/value groups, and each chunk's inputs are copied in,
+ * computed and copied out on three streams through two slots of a
+ * caller-owned device workspace, so copies and kernels of neighbouring
+ * chunks overlap (each head is an independent problem, Alg. 1).
+ * In:  q, k, v, o, lse, dout, gq, gk, gv: host buffers with the layouts of
+ *      fbob_attn_bob.  Page-locked memory lets the copies run asynchronously;
+ *      pageable memory gives the same results, without the overlap.
+ * Out: q_bar, k_bar, v_bar, dout_bar, row_stats: host buffers, as in
+ *      fbob_attn_bob; they must not overlap any input or each other.
+ * workspace: device memory of workspace_bytes, 256-byte aligned, owned by the
+ *      caller and not used by anything else until `stream` has passed this
+ *      call.  fbob_attn_bob_host_workspace() gives the bytes for a chunk size;
+ *      the call takes about a quarter of the heads per chunk, or fewer when
+ *      the workspace is smaller, and returns FBOB_ERR_INVALID_ARGUMENT if it
+ *      cannot hold one key/value group.
+ * Stream: the copies start after the work already enqueued on `stream`, and
+ *      `stream` completes only after the last copy out; synchronise it before
+ *      reading the outputs.  Two streams and seven events are created per call
+ *      and released when their work completes.
+ */
+int fbob_attn_bob_host(const fbob_shape* shape, const void* q, const void* k, const void* v,
+                       const void* o, const float* lse, const void* dout,
+                       const void* gq, const void* gk, const void* gv,
+                       void* q_bar, void* k_bar, void* v_bar, void* dout_bar, float* row_stats,
+                       void* workspace, int64_t workspace_bytes, struct CUstream_st* stream);
+
+/*
+ * Device workspace bytes fbob_attn_bob_host needs to run chunks of
+ * chunk_heads query heads (rounded up to whole key/value groups), or -1 for
+ * an invalid shape or chunk_heads < 1.
+ */
+int64_t fbob_attn_bob_host_workspace(const fbob_shape* shape, int64_t chunk_heads);
+
+/*
  * Synchronises `stream`, then returns and clears the device error word of the
  * current device: FBOB_OK, FBOB_ERR_DEVICE_TIMEOUT (a bounded wait expired in
  * some kernel since the last call), or FBOB_ERR_DEVICE_FAULT / FBOB_ERR_CUDA

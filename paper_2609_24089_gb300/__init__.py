@@ -64,6 +64,8 @@ def load():
         "fbob_attn_bob_pass2": [S, P, P, P, P, P, P, P, P, P, P, P, P],
         "fbob_attn_bob_row_stats": [S, P, P, P, P, P, P, P, P, P, P, P],
         "fbob_attn_bob_pass1_direct": [S, P, P, P, P, P, P, P, P, P, P, P, P],
+        "fbob_attn_bob_host": [S] + [P] * 15 + [ctypes.c_int64, P],
+        "fbob_attn_bob_host_workspace": [S, ctypes.c_int64],
         "fbob_device_status": [P],
         "fbob_launch_count": [ctypes.c_char_p],
         "fbob_status_string": [ctypes.c_int],
@@ -71,7 +73,8 @@ def load():
     for name, argt in sig.items():
         f = getattr(lib, name)
         f.argtypes = argt
-        f.restype = ctypes.c_char_p if name == "fbob_status_string" else ctypes.c_int
+        f.restype = (ctypes.c_char_p if name == "fbob_status_string" else
+                     ctypes.c_int64 if name == "fbob_attn_bob_host_workspace" else ctypes.c_int)
     _lib = lib
     return lib
 
@@ -183,6 +186,21 @@ def fbob_attn_bob_pass1_direct(shape, q, k, v, lse, dout, gq, gk, gv, row_stats,
         ctypes.byref(shape),
         *map(_ptr, (q, k, v, lse, dout, gq, gk, gv, row_stats, q_bar, dout_bar)),
         _stream(stream)), "fbob_attn_bob_pass1_direct")
+
+
+def fbob_attn_bob_host(shape, q, k, v, o, lse, dout, gq, gk, gv, q_bar, k_bar, v_bar, dout_bar,
+                       row_stats, workspace, stream=None):
+    """Host tensors (pinned for overlap) in and out; workspace: a CUDA uint8
+    tensor (its size is passed as workspace_bytes)."""
+    _check(load().fbob_attn_bob_host(
+        ctypes.byref(shape),
+        *map(_ptr, (q, k, v, o, lse, dout, gq, gk, gv, q_bar, k_bar, v_bar, dout_bar, row_stats,
+                    workspace)),
+        workspace.numel() * workspace.element_size(), _stream(stream)), "fbob_attn_bob_host")
+
+
+def fbob_attn_bob_host_workspace(shape, chunk_heads) -> int:
+    return load().fbob_attn_bob_host_workspace(ctypes.byref(shape), int(chunk_heads))
 
 
 def fbob_device_status(stream=None) -> int:

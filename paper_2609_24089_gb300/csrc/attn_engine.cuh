@@ -650,7 +650,8 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
     const float dsig = p.drop_sigma;
     auto tile_keep = [&](int jt, uint32_t (&kb)[2]) {
 #pragma unroll
-      for (int h = 0; h < 2; ++h) kb[h] = keep_row16(gi, jt + HB * h + 16 * wg, (uint32_t)bh, dkey);
+      for (int h = 0; h < 2; ++h)
+        kb[h] = keep_row16(gi, jt + HB * h + 16 * wg, (uint32_t)(p.head0 + bh), dkey);
     };
     // with dropout the lanes of a warp exchange keep bits, so a wait that
     // gives up makes the whole warp leave together
@@ -1461,7 +1462,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
       uint32_t kb[2];
       if constexpr (DROP) {
         const int it = (first_tile + st % nsteps_h) * BN;
-        const uint32_t bhq = (uint32_t)(bh_q0 + st / nsteps_h);
+        const uint32_t bhq = (uint32_t)(p.head0 + bh_q0 + st / nsteps_h);
 #pragma unroll
         for (int h = 0; h < 2; ++h) kb[h] = keep_col16(gj, it + HB * h + 16 * wg, bhq, dkey);
       }

@@ -63,6 +63,7 @@ struct EngineParams {
   uint32_t drop_rk[20];
   uint32_t drop_tlow4, drop_tmask;
   float drop_sigma;
+  int head0;  // flat index b*H + h of the launch's first query head (dropout counter)
 };
 
 // ---------------------------------------------------------------- configs

@@ -18,9 +18,11 @@ namespace {
 constexpr int64_t kMaxN = int64_t(1) << 24;
 constexpr int64_t kMaxBH = int64_t(1) << 24;
 
-constexpr int kNumEntries = 7;
-std::atomic<int> g_launches[kNumEntries] = {{-1}, {-1}, {-1}, {-1}, {-1}, {-1}, {-1}};
-enum Entry { kEntFwd = 0, kEntBwd, kEntBob, kEntPass1, kEntPass2, kEntRowStats, kEntPass1D };
+constexpr int kNumEntries = 8;
+std::atomic<int> g_launches[kNumEntries] = {{-1}, {-1}, {-1}, {-1}, {-1}, {-1}, {-1}, {-1}};
+enum Entry {
+  kEntFwd = 0, kEntBwd, kEntBob, kEntPass1, kEntPass2, kEntRowStats, kEntPass1D, kEntBobHost
+};
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   static std::once_flag once;
@@ -212,12 +214,15 @@ int run_pass1_direct(EngineParams p, int d, bool drop, const float* row_stats, v
 // dropout; otherwise row statistics + direct form
 bool pass1_one_sweep(const fbob_shape* s) { return s->d <= 64 && !has_dropout(s); }
 
+// head0: flat index of the shape's first query head within a larger problem
+// (chunked host-buffer calls); it only enters the dropout counter.
 int run_pass1(const fbob_shape* s, const void* q, const void* k, const void* v, const void* o,
               const float* lse, const void* dout, const void* gq, const void* gk,
               const void* gv, void* q_bar, void* dout_bar, float* row_stats,
-              cudaStream_t st) {
+              cudaStream_t st, int64_t head0 = 0) {
   EngineParams p;
   if (!row_bob_params(s, q, k, v, o, lse, dout, gq, gk, gv, &p)) return FBOB_ERR_CUDA;
+  p.head0 = (int)head0;
   if (pass1_one_sweep(s)) {  // one sweep, affine fusion (Prop. 3.1)
     p.out0 = static_cast<__nv_bfloat16*>(q_bar);
     p.out1 = static_cast<__nv_bfloat16*>(dout_bar);
@@ -239,8 +244,10 @@ int pass1_launches(const fbob_shape* s) { return pass1_one_sweep(s) ? 1 : 2; }
 
 int run_pass2(const fbob_shape* s, const void* q, const void* k, const void* v, const float* lse,
               const void* dout, const void* gq, const void* gk, const void* gv,
-              const float* row_stats, void* k_bar, void* v_bar, cudaStream_t st) {
+              const float* row_stats, void* k_bar, void* v_bar, cudaStream_t st,
+              int64_t head0 = 0) {
   EngineParams p = base_params(s);
+  p.head0 = (int)head0;
   const int64_t BH = s->B * s->H, N = s->N, d = s->d;
   const void* stat[4] = {k, v, gk, gv};
   const void* strm[3] = {q, gq, dout};
@@ -258,6 +265,71 @@ int run_pass2(const fbob_shape* s, const void* q, const void* k, const void* v, 
   choose_order(&p, 0);
   return launch_status(launch_col(ColOp::BobPass2, (int)d, has_dropout(s), p, p.nblk * p.BH, st));
 }
+
+// ---- host-buffer BoB: chunks of query heads pipelined through a device
+// workspace of kSlots slots (copy in, compute, copy out on three streams)
+constexpr int kSlots = 2;
+constexpr int kBufs = 14;  // q k v o lse dout gq gk gv q_bar k_bar v_bar dout_bar row_stats
+
+int64_t align256(int64_t x) { return (x + 255) & ~int64_t(255); }
+
+// query heads per key/value head
+int64_t group(const fbob_shape* s) { return s->H / kv_heads(s); }
+
+// Byte offsets of the buffers of one slot holding `nq` query heads; returns
+// the slot's size.
+int64_t slot_layout(const fbob_shape* s, int64_t nq, int64_t* off) {
+  const int64_t nkv = nq / group(s), nd = s->N * s->d * 2;
+  const int64_t bytes[kBufs] = {nq * nd,  nkv * nd, nkv * nd, nq * nd,  nq * s->N * 4,
+                                nq * nd,  nq * nd,  nkv * nd, nkv * nd, nq * nd,
+                                nkv * nd, nkv * nd, nq * nd,  3 * nq * s->N * 4};
+  int64_t at = 0;
+  for (int t = 0; t < kBufs; ++t) {
+    off[t] = at;
+    at += align256(bytes[t]);
+  }
+  return at;
+}
+
+// Query heads per chunk: whole key/value groups, about a quarter of the
+// problem (so copies overlap compute), at most what the workspace holds.
+int64_t chunk_heads(const fbob_shape* s, int64_t ws_bytes) {
+  const int64_t G = group(s), units = s->B * s->H / G, cap = ws_bytes / kSlots;
+  int64_t off[kBufs];
+  // unpadded bytes of one group bound the fit from above; then step down to
+  // the largest chunk whose padded slot fits (a few steps: padding < 14 * 256)
+  const int64_t raw = slot_layout(s, G, off) - kBufs * 255;
+  int64_t u = (units + 3) / 4;
+  if (raw > 0 && cap / raw < u) u = cap / raw;
+  while (u > 0 && slot_layout(s, u * G, off) > cap) --u;
+  return u * G;
+}
+
+struct HostCall {
+  cudaStream_t cin = nullptr, cout = nullptr;
+  cudaEvent_t entry = nullptr, in[kSlots] = {}, comp[kSlots] = {}, out[kSlots] = {};
+  ~HostCall() {  // released once their pending work completes
+    if (entry) cudaEventDestroy(entry);
+    for (int t = 0; t < kSlots; ++t) {
+      if (in[t]) cudaEventDestroy(in[t]);
+      if (comp[t]) cudaEventDestroy(comp[t]);
+      if (out[t]) cudaEventDestroy(out[t]);
+    }
+    if (cin) cudaStreamDestroy(cin);
+    if (cout) cudaStreamDestroy(cout);
+  }
+  cudaError_t init() {
+    cudaError_t e = cudaStreamCreateWithFlags(&cin, cudaStreamNonBlocking);
+    if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&cout, cudaStreamNonBlocking);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&entry, cudaEventDisableTiming);
+    for (int t = 0; t < kSlots && e == cudaSuccess; ++t) {
+      e = cudaEventCreateWithFlags(&in[t], cudaEventDisableTiming);
+      if (e == cudaSuccess) e = cudaEventCreateWithFlags(&comp[t], cudaEventDisableTiming);
+      if (e == cudaSuccess) e = cudaEventCreateWithFlags(&out[t], cudaEventDisableTiming);
+    }
+    return e;
+  }
+};
 
 }  // namespace
 }  // namespace fbob
@@ -280,9 +352,9 @@ const char* fbob_status_string(int status) {
 
 int fbob_launch_count(const char* entry) {
   if (!entry) return -1;
-  static const char* names[kNumEntries] = {"fwd",       "bwd",           "bob",
-                                          "bob_pass1", "bob_pass2",     "bob_row_stats",
-                                          "bob_pass1_direct"};
+  static const char* names[kNumEntries] = {"fwd",           "bwd",       "bob",
+                                          "bob_pass1",     "bob_pass2", "bob_row_stats",
+                                          "bob_pass1_direct", "bob_host"};
   for (int t = 0; t < kNumEntries; ++t)
     if (std::strcmp(entry, names[t]) == 0) return g_launches[t].load();
   return -1;
@@ -498,6 +570,126 @@ int fbob_attn_bob(const fbob_shape* s, const void* q, const void* k, const void*
   rc = run_pass2(s, q, k, v, lse, dout, gq, gk, gv, row_stats, k_bar, v_bar, stream);
   if (rc == FBOB_OK) g_launches[kEntBob] = pass1_launches(s) + 1;
   return rc;
+}
+
+int64_t fbob_attn_bob_host_workspace(const fbob_shape* s, int64_t chunk_heads) {
+  bool empty = false;
+  if (check_shape(s, &empty) != FBOB_OK || chunk_heads < 1) return -1;
+  const int64_t G = group(s);
+  const int64_t nq = (chunk_heads + G - 1) / G * G;
+  int64_t off[kBufs];
+  return kSlots * slot_layout(s, nq, off);
+}
+
+int fbob_attn_bob_host(const fbob_shape* s, const void* q, const void* k, const void* v,
+                       const void* o, const float* lse, const void* dout, const void* gq,
+                       const void* gk, const void* gv, void* q_bar, void* k_bar, void* v_bar,
+                       void* dout_bar, float* row_stats, void* workspace,
+                       int64_t workspace_bytes, struct CUstream_st* stream) {
+  bool empty = false;
+  int rc = check_shape(s, &empty);
+  if (rc != FBOB_OK) return rc;
+  const void* hin[9] = {q, k, v, o, lse, dout, gq, gk, gv};
+  void* hout[5] = {q_bar, k_bar, v_bar, dout_bar, row_stats};
+  const int64_t mat = s->B * s->H * s->N * s->d * 2, vec = s->B * s->H * s->N * 4;
+  const int64_t matk = s->B * kv_heads(s) * s->N * s->d * 2;
+  const int64_t inb[9] = {mat, matk, matk, mat, vec, mat, mat, matk, matk};
+  const int64_t outb[5] = {mat, matk, matk, mat, 3 * vec};
+  for (int t = 0; t < 9; ++t)
+    if (!hin[t]) return FBOB_ERR_INVALID_ARGUMENT;
+  for (int a = 0; a < 5; ++a) {  // host outputs overlap nothing
+    if (!hout[a]) return FBOB_ERR_INVALID_ARGUMENT;
+    const Span sa = {reinterpret_cast<uintptr_t>(hout[a]),
+                     reinterpret_cast<uintptr_t>(hout[a]) + (uintptr_t)outb[a]};
+    for (int b = 0; b < 14; ++b) {
+      if (b == 9 + a) continue;
+      const void* pb = b < 9 ? hin[b] : hout[b - 9];
+      const int64_t nb = b < 9 ? inb[b] : outb[b - 9];
+      const Span sb = {reinterpret_cast<uintptr_t>(pb), reinterpret_cast<uintptr_t>(pb) + (uintptr_t)nb};
+      if (overlaps(sa, sb)) return FBOB_ERR_INVALID_ARGUMENT;
+    }
+  }
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u) || workspace_bytes < 0)
+    return FBOB_ERR_INVALID_ARGUMENT;
+  if (empty) {
+    g_launches[kEntBobHost] = 0;
+    return FBOB_OK;
+  }
+  const int64_t BH = s->B * s->H, G = group(s), N = s->N, nd = N * s->d * 2;
+  const int64_t hc = chunk_heads(s, workspace_bytes);
+  if (hc < 1) return FBOB_ERR_INVALID_ARGUMENT;  // the workspace holds no key/value group
+  int64_t off[kBufs];
+  const int64_t slot = slot_layout(s, hc, off);
+  HostCall hcall;
+  if (hcall.init() != cudaSuccess) return FBOB_ERR_CUDA;
+  cudaStream_t st = stream;
+  // the copy streams start after the work already on `stream` (it may use
+  // the workspace or the host buffers)
+  if (cudaEventRecord(hcall.entry, st) != cudaSuccess ||
+      cudaStreamWaitEvent(hcall.cin, hcall.entry, 0) != cudaSuccess ||
+      cudaStreamWaitEvent(hcall.cout, hcall.entry, 0) != cudaSuccess)
+    return FBOB_ERR_CUDA;
+  const int64_t nchunks = (BH + hc - 1) / hc;
+  auto h2d = [&](void* dst, const void* src, int64_t bytes) {
+    return cudaMemcpyAsync(dst, src, (size_t)bytes, cudaMemcpyHostToDevice, hcall.cin);
+  };
+  auto d2h = [&](void* dst, const void* src, int64_t bytes) {
+    return cudaMemcpyAsync(dst, src, (size_t)bytes, cudaMemcpyDeviceToHost, hcall.cout);
+  };
+  auto hb = [](const void* p, int64_t at) { return static_cast<const uint8_t*>(p) + at; };
+  auto hbm = [](void* p, int64_t at) { return static_cast<uint8_t*>(p) + at; };
+  int launches = 0;
+  for (int64_t c = 0; c < nchunks; ++c) {
+    const int sl = (int)(c % kSlots);
+    uint8_t* base = static_cast<uint8_t*>(workspace) + sl * slot;
+    void* w[kBufs];
+    for (int t = 0; t < kBufs; ++t) w[t] = base + off[t];
+    const int64_t f0 = c * hc, nq = (BH - f0) < hc ? (BH - f0) : hc, nkv = nq / G, k0 = f0 / G;
+    cudaError_t e = cudaSuccess;
+    // copy in once the slot's previous chunk has been computed
+    if (c >= kSlots) e = cudaStreamWaitEvent(hcall.cin, hcall.comp[sl], 0);
+    const int qside[5] = {0, 3, 5, 6};  // q, o, dout, gq
+    for (int t = 0; t < 4 && e == cudaSuccess; ++t)
+      e = h2d(w[qside[t]], hb(hin[qside[t]], f0 * nd), nq * nd);
+    const int kside[4] = {1, 2, 7, 8};  // k, v, gk, gv
+    for (int t = 0; t < 4 && e == cudaSuccess; ++t)
+      e = h2d(w[kside[t]], hb(hin[kside[t]], k0 * nd), nkv * nd);
+    if (e == cudaSuccess) e = h2d(w[4], hb(lse, f0 * N * 4), nq * N * 4);
+    if (e == cudaSuccess) e = cudaEventRecord(hcall.in[sl], hcall.cin);
+    // compute once the inputs are in and the slot's previous outputs are out
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(st, hcall.in[sl], 0);
+    if (e == cudaSuccess && c >= kSlots) e = cudaStreamWaitEvent(st, hcall.out[sl], 0);
+    if (e != cudaSuccess) return FBOB_ERR_CUDA;
+    fbob_shape cs = *s;
+    cs.B = 1;
+    cs.H = nq;
+    cs.H_kv = s->H_kv > 0 ? nkv : 0;
+    rc = run_pass1(&cs, w[0], w[1], w[2], w[3], static_cast<const float*>(w[4]), w[5], w[6],
+                   w[7], w[8], w[9], w[12], static_cast<float*>(w[13]), st, f0);
+    if (rc == FBOB_OK)
+      rc = run_pass2(&cs, w[0], w[1], w[2], static_cast<const float*>(w[4]), w[5], w[6], w[7],
+                     w[8], static_cast<const float*>(w[13]), w[10], w[11], st, f0);
+    if (rc != FBOB_OK) return rc;
+    launches += pass1_launches(&cs) + 1;
+    // copy out once computed
+    e = cudaEventRecord(hcall.comp[sl], st);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(hcall.cout, hcall.comp[sl], 0);
+    if (e == cudaSuccess) e = d2h(hbm(q_bar, f0 * nd), w[9], nq * nd);
+    if (e == cudaSuccess) e = d2h(hbm(dout_bar, f0 * nd), w[12], nq * nd);
+    if (e == cudaSuccess) e = d2h(hbm(k_bar, k0 * nd), w[10], nkv * nd);
+    if (e == cudaSuccess) e = d2h(hbm(v_bar, k0 * nd), w[11], nkv * nd);
+    if (e == cudaSuccess)  // row_stats planes: [3][B*H][N] on the host, [3][nq][N] in the slot
+      e = cudaMemcpy2DAsync(hbm(row_stats, f0 * N * 4), (size_t)(BH * N * 4), w[13],
+                            (size_t)(nq * N * 4), (size_t)(nq * N * 4), 3, cudaMemcpyDeviceToHost,
+                            hcall.cout);
+    if (e == cudaSuccess) e = cudaEventRecord(hcall.out[sl], hcall.cout);
+    if (e != cudaSuccess) return FBOB_ERR_CUDA;
+  }
+  // `stream` completes after the last copies out
+  for (int sl = 0; sl < kSlots && sl < nchunks; ++sl)
+    if (cudaStreamWaitEvent(st, hcall.out[sl], 0) != cudaSuccess) return FBOB_ERR_CUDA;
+  g_launches[kEntBobHost] = launches;
+  return FBOB_OK;
 }
 
 int fbob_device_status(struct CUstream_st* stream) {

@@ -167,3 +167,41 @@ def test_head_dim_32_passes_validation(lib):
     S = fbob.make_shape
     assert bob(lib, S(1, 1, 0, 32, 0.17, 1), ptrs(14)) == 0  # valid: empty problem, no call
     assert bob(lib, S(1, 1, 128, 32, 0.17, 1), ptrs(14, misalign=3)) == 1
+
+
+def test_host_buffer_bob_validates_before_any_cuda_call(lib):
+    S = fbob.make_shape
+    shp = S(2, 4, 256, 64, 0.125, 1, kv_heads=2)
+    host = ptrs(14)
+    ws = ctypes.c_void_p(BASE + 20 * STRIDE)
+    call = lib.fbob_attn_bob_host
+    # (every call below fails validation or is empty: none reaches a CUDA call)
+    # null host pointer, misaligned or null workspace, negative size, overlapping outputs
+    bad = list(host)
+    bad[3] = None
+    assert call(ctypes.byref(shp), *bad, ws, 1 << 30, None) == 1
+    assert call(ctypes.byref(shp), *host, ctypes.c_void_p(BASE + 20 * STRIDE + 16), 1 << 30,
+                None) == 1
+    assert call(ctypes.byref(shp), *host, None, 1 << 30, None) == 1
+    assert call(ctypes.byref(shp), *host, ws, -1, None) == 1
+    ov = list(host)
+    ov[10] = ov[9]  # k_bar aliases q_bar
+    assert call(ctypes.byref(shp), *ov, ws, 1 << 30, None) == 1
+    # a workspace that cannot hold one key/value group of 2 query heads
+    assert call(ctypes.byref(shp), *host, ws, 1024, None) == 1
+    # empty problem: valid, no CUDA call
+    assert call(ctypes.byref(S(0, 4, 256, 64, 0.125, 1)), *host, ws, 0, None) == 0
+    assert lib.fbob_launch_count(b"bob_host") == 0
+
+
+def test_host_workspace_size(lib):
+    S = fbob.make_shape
+    shp = S(2, 8, 1000, 128, 0.09, 1, kv_heads=2)   # groups of 4 query heads
+    one = lib.fbob_attn_bob_host_workspace(ctypes.byref(shp), 1)
+    assert one == lib.fbob_attn_bob_host_workspace(ctypes.byref(shp), 4)   # rounded up to a group
+    nd = 1000 * 128 * 2
+    # two slots of: 4 query-side + 2 output query-side + lse + row_stats, 4 + 2 key/value-side
+    want = 2 * (6 * 4 * nd + 6 * 1 * nd + 4 * 1000 * 4 + 3 * 4 * 1000 * 4)
+    assert want <= one <= want + 2 * 14 * 256
+    assert lib.fbob_attn_bob_host_workspace(ctypes.byref(shp), 0) == -1
+    assert lib.fbob_attn_bob_host_workspace(ctypes.byref(S(1, 1, 8, 48, 0.1, 0)), 1) == -1
