@@ -97,7 +97,9 @@ typedef enum fbob_status {
     FBOB_ERR_UNSUPPORTED = 2,      /* valid request this build does not implement (d not 32/64/128) */
     FBOB_ERR_CUDA = 3,             /* a CUDA runtime/driver call or launch failed */
     FBOB_ERR_DEVICE_TIMEOUT = 4,   /* a bounded device-side wait expired */
-    FBOB_ERR_DEVICE_FAULT = 5      /* the device reported an error while synchronising */
+    FBOB_ERR_DEVICE_FAULT = 5,     /* the device reported an error while synchronising */
+    FBOB_ERR_SCRATCH_LIMIT = 6     /* the problem needs more staging memory than the
+                                      fixed array of fbob_attn_bob_host_noalloc */
 } fbob_status;
 
 typedef struct fbob_shape {
@@ -241,6 +243,36 @@ int fbob_attn_bob_host(const fbob_shape* shape, const void* q, const void* k, co
  * an invalid shape or chunk_heads < 1.
  */
 int64_t fbob_attn_bob_host_workspace(const fbob_shape* shape, int64_t chunk_heads);
+
+/*
+ * fbob_attn_bob_host for callers that cannot allocate device memory while they
+ * run, such as a process that reserves its whole device footprint when it
+ * starts and may not grow it later, or one that cannot spare a workspace of
+ * its own.  No workspace argument and no allocation of any kind per call: the
+ * chunks of heads are staged in a fixed 64 MiB device array that the library
+ * declares statically.  The paper has no counterpart; it is the same
+ * computation (the same kernels on each head) behind a different interface,
+ * and its results equal fbob_attn_bob_host's bit for bit.
+ * Arguments and layouts as fbob_attn_bob_host (host buffers; page-locked for
+ * asynchronous copies).  The heads go in chunks of whole key/value groups, as
+ * many as fit in the array, one chunk after the other on `stream` (copy in,
+ * Pass 1, Pass 2, copy out; copies do not overlap the kernels).
+ * Limit: the staging of one key/value group, about 12 N d (H / H_kv) * 2
+ *      bytes, must fit in 64 MiB (for example N = 16384 at d = 128 without
+ *      grouping); larger problems return FBOB_ERR_SCRATCH_LIMIT and run
+ *      nothing (use fbob_attn_bob_host with a workspace).
+ * Set-up: the first call on each device looks up the array's device address
+ *      (with that device current), which also places the array on that
+ *      device; make that first call before any stream capture.
+ * Nothing in the array has to start at zero: each call writes every byte it
+ *      reads.  All calls on a device share the array, so calls that overlap in
+ *      time (on other streams or threads) race; serialise them.
+ */
+int fbob_attn_bob_host_noalloc(const fbob_shape* shape, const void* q, const void* k,
+                               const void* v, const void* o, const float* lse,
+                               const void* dout, const void* gq, const void* gk,
+                               const void* gv, void* q_bar, void* k_bar, void* v_bar,
+                               void* dout_bar, float* row_stats, struct CUstream_st* stream);
 
 /*
  * Synchronises `stream`, then returns and clears the device error word of the

@@ -19,7 +19,8 @@ HEADER = os.path.join(os.path.dirname(_HERE), "include", "fbob.h")
 
 FBOB_OK = 0
 STATUS = {0: "FBOB_OK", 1: "FBOB_ERR_INVALID_ARGUMENT", 2: "FBOB_ERR_UNSUPPORTED",
-          3: "FBOB_ERR_CUDA", 4: "FBOB_ERR_DEVICE_TIMEOUT", 5: "FBOB_ERR_DEVICE_FAULT"}
+          3: "FBOB_ERR_CUDA", 4: "FBOB_ERR_DEVICE_TIMEOUT", 5: "FBOB_ERR_DEVICE_FAULT",
+          6: "FBOB_ERR_SCRATCH_LIMIT"}
 STATUS_CODES = {v: k for k, v in STATUS.items()}
 
 
@@ -66,6 +67,7 @@ def load():
         "fbob_attn_bob_pass1_direct": [S, P, P, P, P, P, P, P, P, P, P, P, P],
         "fbob_attn_bob_host": [S] + [P] * 15 + [ctypes.c_int64, P],
         "fbob_attn_bob_host_workspace": [S, ctypes.c_int64],
+        "fbob_attn_bob_host_noalloc": [S] + [P] * 14 + [P],
         "fbob_device_status": [P],
         "fbob_launch_count": [ctypes.c_char_p],
         "fbob_status_string": [ctypes.c_int],
@@ -197,6 +199,15 @@ def fbob_attn_bob_host(shape, q, k, v, o, lse, dout, gq, gk, gv, q_bar, k_bar, v
         *map(_ptr, (q, k, v, o, lse, dout, gq, gk, gv, q_bar, k_bar, v_bar, dout_bar, row_stats,
                     workspace)),
         workspace.numel() * workspace.element_size(), _stream(stream)), "fbob_attn_bob_host")
+
+
+def fbob_attn_bob_host_noalloc(shape, q, k, v, o, lse, dout, gq, gk, gv, q_bar, k_bar, v_bar,
+                               dout_bar, row_stats, stream=None):
+    """As fbob_attn_bob_host, staged in the library's fixed device array."""
+    _check(load().fbob_attn_bob_host_noalloc(
+        ctypes.byref(shape),
+        *map(_ptr, (q, k, v, o, lse, dout, gq, gk, gv, q_bar, k_bar, v_bar, dout_bar, row_stats)),
+        _stream(stream)), "fbob_attn_bob_host_noalloc")
 
 
 def fbob_attn_bob_host_workspace(shape, chunk_heads) -> int:

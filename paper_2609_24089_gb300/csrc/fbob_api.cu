@@ -18,11 +18,19 @@ namespace {
 constexpr int64_t kMaxN = int64_t(1) << 24;
 constexpr int64_t kMaxBH = int64_t(1) << 24;
 
-constexpr int kNumEntries = 8;
-std::atomic<int> g_launches[kNumEntries] = {{-1}, {-1}, {-1}, {-1}, {-1}, {-1}, {-1}, {-1}};
+constexpr int kNumEntries = 9;
+std::atomic<int> g_launches[kNumEntries] = {{-1}, {-1}, {-1}, {-1}, {-1},
+                                            {-1}, {-1}, {-1}, {-1}};
 enum Entry {
-  kEntFwd = 0, kEntBwd, kEntBob, kEntPass1, kEntPass2, kEntRowStats, kEntPass1D, kEntBobHost
+  kEntFwd = 0, kEntBwd, kEntBob, kEntPass1, kEntPass2, kEntRowStats, kEntPass1D, kEntBobHost,
+  kEntBobHostNoAlloc
 };
+
+// Staging memory of fbob_attn_bob_host_noalloc: a fixed device array, so that
+// call allocates nothing.  Its module holds no kernels; the array is placed
+// when the module is loaded on a device (on the first address lookup).
+constexpr int64_t kNoAllocBytes = int64_t(64) << 20;
+__device__ __align__(256) uint8_t g_noalloc_scratch[kNoAllocBytes];
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   static std::once_flag once;
@@ -305,6 +313,53 @@ int64_t chunk_heads(const fbob_shape* s, int64_t ws_bytes) {
   return u * G;
 }
 
+// Device address of the static staging array on the current device, looked
+// up once per device.
+cudaError_t noalloc_scratch(uint8_t** ptr) {
+  static std::mutex mu;
+  static uint8_t* addr[64] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(mu);
+  if (!addr[dev]) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess) return e;
+    addr[dev] = static_cast<uint8_t*>(p);
+  }
+  *ptr = addr[dev];
+  return cudaSuccess;
+}
+
+// Validation shared by the host-buffer calls: shape, host pointers present,
+// host outputs overlapping nothing.
+int check_host_args(const fbob_shape* s, const void* const* hin, void* const* hout, bool* empty) {
+  int rc = check_shape(s, empty);
+  if (rc != FBOB_OK) return rc;
+  const int64_t mat = s->B * s->H * s->N * s->d * 2, vec = s->B * s->H * s->N * 4;
+  const int64_t matk = s->B * kv_heads(s) * s->N * s->d * 2;
+  const int64_t inb[9] = {mat, matk, matk, mat, vec, mat, mat, matk, matk};
+  const int64_t outb[5] = {mat, matk, matk, mat, 3 * vec};
+  for (int t = 0; t < 9; ++t)
+    if (!hin[t]) return FBOB_ERR_INVALID_ARGUMENT;
+  for (int a = 0; a < 5; ++a) {
+    if (!hout[a]) return FBOB_ERR_INVALID_ARGUMENT;
+    const Span sa = {reinterpret_cast<uintptr_t>(hout[a]),
+                     reinterpret_cast<uintptr_t>(hout[a]) + (uintptr_t)outb[a]};
+    for (int b = 0; b < 14; ++b) {
+      if (b == 9 + a) continue;
+      const void* pb = b < 9 ? hin[b] : hout[b - 9];
+      const int64_t nb = b < 9 ? inb[b] : outb[b - 9];
+      const Span sb = {reinterpret_cast<uintptr_t>(pb),
+                       reinterpret_cast<uintptr_t>(pb) + (uintptr_t)nb};
+      if (overlaps(sa, sb)) return FBOB_ERR_INVALID_ARGUMENT;
+    }
+  }
+  return FBOB_OK;
+}
+
 struct HostCall {
   cudaStream_t cin = nullptr, cout = nullptr;
   cudaEvent_t entry = nullptr, in[kSlots] = {}, comp[kSlots] = {}, out[kSlots] = {};
@@ -346,15 +401,16 @@ const char* fbob_status_string(int status) {
     case FBOB_ERR_CUDA: return "FBOB_ERR_CUDA";
     case FBOB_ERR_DEVICE_TIMEOUT: return "FBOB_ERR_DEVICE_TIMEOUT";
     case FBOB_ERR_DEVICE_FAULT: return "FBOB_ERR_DEVICE_FAULT";
+    case FBOB_ERR_SCRATCH_LIMIT: return "FBOB_ERR_SCRATCH_LIMIT";
     default: return "FBOB_UNKNOWN_STATUS";
   }
 }
 
 int fbob_launch_count(const char* entry) {
   if (!entry) return -1;
-  static const char* names[kNumEntries] = {"fwd",           "bwd",       "bob",
-                                          "bob_pass1",     "bob_pass2", "bob_row_stats",
-                                          "bob_pass1_direct", "bob_host"};
+  static const char* names[kNumEntries] = {
+      "fwd",       "bwd",       "bob",           "bob_pass1",          "bob_pass2",
+      "bob_row_stats", "bob_pass1_direct", "bob_host", "bob_host_noalloc"};
   for (int t = 0; t < kNumEntries; ++t)
     if (std::strcmp(entry, names[t]) == 0) return g_launches[t].load();
   return -1;
@@ -587,28 +643,10 @@ int fbob_attn_bob_host(const fbob_shape* s, const void* q, const void* k, const 
                        void* dout_bar, float* row_stats, void* workspace,
                        int64_t workspace_bytes, struct CUstream_st* stream) {
   bool empty = false;
-  int rc = check_shape(s, &empty);
-  if (rc != FBOB_OK) return rc;
   const void* hin[9] = {q, k, v, o, lse, dout, gq, gk, gv};
   void* hout[5] = {q_bar, k_bar, v_bar, dout_bar, row_stats};
-  const int64_t mat = s->B * s->H * s->N * s->d * 2, vec = s->B * s->H * s->N * 4;
-  const int64_t matk = s->B * kv_heads(s) * s->N * s->d * 2;
-  const int64_t inb[9] = {mat, matk, matk, mat, vec, mat, mat, matk, matk};
-  const int64_t outb[5] = {mat, matk, matk, mat, 3 * vec};
-  for (int t = 0; t < 9; ++t)
-    if (!hin[t]) return FBOB_ERR_INVALID_ARGUMENT;
-  for (int a = 0; a < 5; ++a) {  // host outputs overlap nothing
-    if (!hout[a]) return FBOB_ERR_INVALID_ARGUMENT;
-    const Span sa = {reinterpret_cast<uintptr_t>(hout[a]),
-                     reinterpret_cast<uintptr_t>(hout[a]) + (uintptr_t)outb[a]};
-    for (int b = 0; b < 14; ++b) {
-      if (b == 9 + a) continue;
-      const void* pb = b < 9 ? hin[b] : hout[b - 9];
-      const int64_t nb = b < 9 ? inb[b] : outb[b - 9];
-      const Span sb = {reinterpret_cast<uintptr_t>(pb), reinterpret_cast<uintptr_t>(pb) + (uintptr_t)nb};
-      if (overlaps(sa, sb)) return FBOB_ERR_INVALID_ARGUMENT;
-    }
-  }
+  int rc = check_host_args(s, hin, hout, &empty);
+  if (rc != FBOB_OK) return rc;
   if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u) || workspace_bytes < 0)
     return FBOB_ERR_INVALID_ARGUMENT;
   if (empty) {
@@ -689,6 +727,81 @@ int fbob_attn_bob_host(const fbob_shape* s, const void* q, const void* k, const 
   for (int sl = 0; sl < kSlots && sl < nchunks; ++sl)
     if (cudaStreamWaitEvent(st, hcall.out[sl], 0) != cudaSuccess) return FBOB_ERR_CUDA;
   g_launches[kEntBobHost] = launches;
+  return FBOB_OK;
+}
+
+int fbob_attn_bob_host_noalloc(const fbob_shape* s, const void* q, const void* k,
+                               const void* v, const void* o, const float* lse, const void* dout,
+                               const void* gq, const void* gk, const void* gv, void* q_bar,
+                               void* k_bar, void* v_bar, void* dout_bar, float* row_stats,
+                               struct CUstream_st* stream) {
+  bool empty = false;
+  const void* hin[9] = {q, k, v, o, lse, dout, gq, gk, gv};
+  void* hout[5] = {q_bar, k_bar, v_bar, dout_bar, row_stats};
+  int rc = check_host_args(s, hin, hout, &empty);
+  if (rc != FBOB_OK) return rc;
+  if (empty) {
+    g_launches[kEntBobHostNoAlloc] = 0;
+    return FBOB_OK;
+  }
+  // as many whole key/value groups per chunk as one slot of the array holds
+  const int64_t BH = s->B * s->H, G = group(s), N = s->N, nd = N * s->d * 2;
+  int64_t off[kBufs];
+  int64_t u = s->B * s->H / G;
+  const int64_t raw = slot_layout(s, G, off) - kBufs * 255;
+  if (raw > 0 && kNoAllocBytes / raw < u) u = kNoAllocBytes / raw;
+  while (u > 0 && slot_layout(s, u * G, off) > kNoAllocBytes) --u;
+  if (u < 1) return FBOB_ERR_SCRATCH_LIMIT;  // one group's staging exceeds the array
+  const int64_t hc = u * G;
+  slot_layout(s, hc, off);
+  uint8_t* base = nullptr;
+  if (noalloc_scratch(&base) != cudaSuccess) return FBOB_ERR_CUDA;
+  void* w[kBufs];
+  for (int t = 0; t < kBufs; ++t) w[t] = base + off[t];
+  cudaStream_t st = stream;
+  auto h2d = [&](void* dst, const void* src, int64_t bytes) {
+    return cudaMemcpyAsync(dst, src, (size_t)bytes, cudaMemcpyHostToDevice, st);
+  };
+  auto d2h = [&](void* dst, const void* src, int64_t bytes) {
+    return cudaMemcpyAsync(dst, src, (size_t)bytes, cudaMemcpyDeviceToHost, st);
+  };
+  auto hb = [](const void* p, int64_t at) { return static_cast<const uint8_t*>(p) + at; };
+  auto hbm = [](void* p, int64_t at) { return static_cast<uint8_t*>(p) + at; };
+  int launches = 0;
+  // one chunk after the other, all on `stream`: copy in, compute, copy out
+  for (int64_t f0 = 0; f0 < BH; f0 += hc) {
+    const int64_t nq = (BH - f0) < hc ? (BH - f0) : hc, nkv = nq / G, k0 = f0 / G;
+    cudaError_t e = cudaSuccess;
+    const int qside[4] = {0, 3, 5, 6};  // q, o, dout, gq
+    for (int t = 0; t < 4 && e == cudaSuccess; ++t)
+      e = h2d(w[qside[t]], hb(hin[qside[t]], f0 * nd), nq * nd);
+    const int kside[4] = {1, 2, 7, 8};  // k, v, gk, gv
+    for (int t = 0; t < 4 && e == cudaSuccess; ++t)
+      e = h2d(w[kside[t]], hb(hin[kside[t]], k0 * nd), nkv * nd);
+    if (e == cudaSuccess) e = h2d(w[4], hb(lse, f0 * N * 4), nq * N * 4);
+    if (e != cudaSuccess) return FBOB_ERR_CUDA;
+    fbob_shape cs = *s;
+    cs.B = 1;
+    cs.H = nq;
+    cs.H_kv = s->H_kv > 0 ? nkv : 0;
+    rc = run_pass1(&cs, w[0], w[1], w[2], w[3], static_cast<const float*>(w[4]), w[5], w[6],
+                   w[7], w[8], w[9], w[12], static_cast<float*>(w[13]), st, f0);
+    if (rc == FBOB_OK)
+      rc = run_pass2(&cs, w[0], w[1], w[2], static_cast<const float*>(w[4]), w[5], w[6], w[7],
+                     w[8], static_cast<const float*>(w[13]), w[10], w[11], st, f0);
+    if (rc != FBOB_OK) return rc;
+    launches += pass1_launches(&cs) + 1;
+    e = d2h(hbm(q_bar, f0 * nd), w[9], nq * nd);
+    if (e == cudaSuccess) e = d2h(hbm(dout_bar, f0 * nd), w[12], nq * nd);
+    if (e == cudaSuccess) e = d2h(hbm(k_bar, k0 * nd), w[10], nkv * nd);
+    if (e == cudaSuccess) e = d2h(hbm(v_bar, k0 * nd), w[11], nkv * nd);
+    if (e == cudaSuccess)
+      e = cudaMemcpy2DAsync(hbm(row_stats, f0 * N * 4), (size_t)(BH * N * 4), w[13],
+                            (size_t)(nq * N * 4), (size_t)(nq * N * 4), 3, cudaMemcpyDeviceToHost,
+                            st);
+    if (e != cudaSuccess) return FBOB_ERR_CUDA;
+  }
+  g_launches[kEntBobHostNoAlloc] = launches;
   return FBOB_OK;
 }
 

@@ -205,3 +205,17 @@ def test_host_workspace_size(lib):
     assert want <= one <= want + 2 * 14 * 256
     assert lib.fbob_attn_bob_host_workspace(ctypes.byref(shp), 0) == -1
     assert lib.fbob_attn_bob_host_workspace(ctypes.byref(S(1, 1, 8, 48, 0.1, 0)), 1) == -1
+
+
+def test_noalloc_host_bob_refuses_before_any_cuda_call(lib):
+    S = fbob.make_shape
+    call = lib.fbob_attn_bob_host_noalloc
+    host = ptrs(14)
+    # one key/value group of 4 heads at N = 16384, d = 128 needs ~193 MiB > 64 MiB
+    assert call(ctypes.byref(S(1, 8, 16384, 128, 0.09, 1, kv_heads=2)), *host, None) == 6
+    assert lib.fbob_status_string(6) == b"FBOB_ERR_SCRATCH_LIMIT"
+    bad = list(host)
+    bad[0] = None
+    assert call(ctypes.byref(S(1, 1, 128, 64, 0.125, 0)), *bad, None) == 1
+    assert call(ctypes.byref(S(0, 1, 128, 64, 0.125, 0)), *host, None) == 0  # empty: no call
+    assert lib.fbob_launch_count(b"bob_host_noalloc") == 0
