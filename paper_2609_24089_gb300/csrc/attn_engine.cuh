@@ -725,8 +725,8 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         tc_fence_before();
         mbar_arrive(&m->bar_sf_free[b]);
         const int jt = (first_tile + st) * BN;
-        float x[2][16];
-        float mt = -INFINITY;
+        float x[2][16];  // raw scores (masked: -inf); the log2 scale enters below
+        float mraw = -INFINITY;
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
           const int j0 = jt + HB * h + 16 * wg;
@@ -734,11 +734,12 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
           const bool need_mask = mlo > 0 || mhi < 16;
 #pragma unroll
           for (int c = 0; c < 16; ++c) {
-            x[h][c] = bits_f(rS[h][c]) * sl2;
+            x[h][c] = bits_f(rS[h][c]);
             if (need_mask && (c < mlo || c >= mhi)) x[h][c] = -INFINITY;
-            mt = fmaxf(mt, x[h][c]);
+            mraw = fmaxf(mraw, x[h][c]);
           }
         }
+        const float mt = mraw * sl2;  // the tile's row maximum in log2 units (sl2 > 0)
         const bool raise = mt > mrow + kFwdSlack;  // also the first tile with a valid key
         const bool rescale = raise && mrow != -INFINITY;
         if (__any_sync(0xffffffffu, rescale)) {
@@ -769,13 +770,15 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         if (raise) mrow = mt;
         float psum = 0.f;
         uint32_t oP[2][8];
+        // no valid key yet in this row: m = -inf and every score is -inf, so
+        // any finite stand-in for m gives P = 2^-inf = 0
+        const float nm = mrow == -INFINITY ? 0.f : -mrow;
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
 #pragma unroll
           for (int c = 0; c < 16; c += 2) {
-            // no valid key yet in this row: m = -inf and every x = -inf
-            float p0 = mrow == -INFINITY ? 0.f : ex2(x[h][c] - mrow);
-            float p1 = mrow == -INFINITY ? 0.f : ex2(x[h][c + 1] - mrow);
+            float p0 = ex2(fmaf(x[h][c], sl2, nm));  // P = 2^(s tau log2 e - m)
+            float p1 = ex2(fmaf(x[h][c + 1], sl2, nm));
             psum += p0 + p1;  // L over the ungated P
             if constexpr (DROP) {  // O = sigma (R o P) V: sigma in the epilogue
               if (!((kb[h] >> c) & 1u)) p0 = 0.f;
