@@ -189,6 +189,15 @@ __device__ __forceinline__ float2 probs2(float2 s, float2 sl2, float2 nL2) {
   return make_float2(ex2(a.x), ex2(a.y));
 }
 
+// Masked columns (c < lo or c >= hi) of a thread's 16 scores set to -inf, so
+// that P = 2^-inf = 0 there; only tiles that cross a band edge need it, which
+// keeps the mask out of the elementwise loops.
+__device__ __forceinline__ void mask16(uint32_t (&r)[16], int lo, int hi) {
+#pragma unroll
+  for (int c = 0; c < 16; ++c)
+    if (c < lo || c >= hi) r[c] = 0xFF800000u;
+}
+
 // ============================================================== row engine
 // D: head dimension of the tiles (64 or 128); DG <= D: head dimension of the
 // tensors in global memory.  DG = 32 runs in the D = 64 tiles: the TMA loads
@@ -731,11 +740,10 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         for (int h = 0; h < 2; ++h) {
           const int j0 = jt + HB * h + 16 * wg;
           const int mlo = jlo - j0, mhi = jhi - j0;  // valid columns: mlo <= c < mhi
-          const bool need_mask = mlo > 0 || mhi < 16;
+          if (mlo > 0 || mhi < 16) mask16(rS[h], mlo, mhi);
 #pragma unroll
           for (int c = 0; c < 16; ++c) {
             x[h][c] = bits_f(rS[h][c]);
-            if (need_mask && (c < mlo || c >= mhi)) x[h][c] = -INFINITY;
             mraw = fmaxf(mraw, x[h][c]);
           }
         }
@@ -887,14 +895,10 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         for (int h = 0; h < 2; ++h) {
           const int j0 = jt + HB * h + 16 * wg;
           const int mlo = jlo - j0, mhi = jhi - j0;  // valid columns: mlo <= c < mhi
-          const bool need_mask = mlo > 0 || mhi < 16;
+          if (mlo > 0 || mhi < 16) mask16(rS[h], mlo, mhi);
 #pragma unroll
           for (int c = 0; c < 16; c += 2) {
-            float2 pr = probs2(pair(rS[h], c), sl2v, nL2v);
-            if (need_mask) {
-              if (c < mlo || c >= mhi) pr.x = 0.f;
-              if (c + 1 < mlo || c + 1 >= mhi) pr.y = 0.f;
-            }
+            const float2 pr = probs2(pair(rS[h], c), sl2v, nL2v);
             const float2 f = __fmul2_rn(pair(rF[h], c), tauv);
             float2 dp = pair(rdP[h], c), cv = pair(rC[h], c);
             if constexpr (DROP) {  // dP -> sigma R dP, C -> sigma R C
@@ -921,7 +925,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
           const int c0 = HB * h + 16 * wg;  // tile column of this thread's 16
           const int j0 = jt + c0;           // first key of this thread's 16
           const int mlo = jlo - j0, mhi = jhi - j0;  // valid columns: mlo <= c < mhi
-          const bool need_mask = mlo > 0 || mhi < 16;
+          if (mlo > 0 || mhi < 16) mask16(rS[h], mlo, mhi);
           if constexpr (kBob) {
             const uint32_t R = ta + kColDC + 64 * h + 16 * wg;  // [dP_h | C_h] columns
             uint32_t rdP[16], rC[16];
@@ -933,11 +937,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
             uint32_t oP[8], oPF[8], oPPt[8], odS[8];
 #pragma unroll
             for (int c = 0; c < 16; c += 2) {
-              float2 pr = probs2(pair(rS[h], c), sl2v, nL2v);
-              if (need_mask) {
-                if (c < mlo || c >= mhi) pr.x = 0.f;
-                if (c + 1 < mlo || c + 1 >= mhi) pr.y = 0.f;
-              }
+              const float2 pr = probs2(pair(rS[h], c), sl2v, nL2v);
               const float2 f = __fmul2_rn(pair(rF[h], c), tauv);
               const float2 dp = pair(rdP, c);
               const float2 t = __fadd2_rn(dp, nDv);
@@ -967,11 +967,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
             uint32_t oP[8], oPh[8], oSt[8], odS[8];
 #pragma unroll
             for (int c = 0; c < 16; c += 2) {
-              float2 pr = probs2(pair(rS[h], c), sl2v, nL2v);
-              if (need_mask) {
-                if (c < mlo || c >= mhi) pr.x = 0.f;
-                if (c + 1 < mlo || c + 1 >= mhi) pr.y = 0.f;
-              }
+              const float2 pr = probs2(pair(rS[h], c), sl2v, nL2v);
               const float2 f = __fmul2_rn(pair(rF[h], c), tauv);
               float2 dp = pair(rdP, c), cv = pair(rC, c), gp = pr;
               if constexpr (DROP) {  // dP, C and the dOtil operands gated by sigma R
@@ -1004,11 +1000,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
             uint32_t odS[8];
 #pragma unroll
             for (int c = 0; c < 16; c += 2) {
-              float2 pr = probs2(pair(rS[h], c), sl2v, nL2v);
-              if (need_mask) {
-                if (c < mlo || c >= mhi) pr.x = 0.f;
-                if (c + 1 < mlo || c + 1 >= mhi) pr.y = 0.f;
-              }
+              const float2 pr = probs2(pair(rS[h], c), sl2v, nL2v);
               float2 dp = pair(rdP, c);
               if constexpr (DROP) dp = __fmul2_rn(dp, gate2(kb[h], c, dsig));
               const float2 ds = __fmul2_rn(pr, __fadd2_rn(dp, nDv));
@@ -1505,7 +1497,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
         const int ib = (first_tile + st % nsteps_h) * BN + cv;  // first query row of this thread's 16
         // valid query columns c satisfy  lo <= c < hi
         const int lo = qlo - ib, hi = qhi - ib;
-        const bool need_mask = lo > 0 || hi < 16;
+        if (lo > 0 || hi < 16) mask16(rS[h], lo, hi);
         const uint32_t R = ta + dcol + cv;
         if constexpr (kBob) {
           uint32_t rdP[16], rC[16];
@@ -1520,11 +1512,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
             const float2 nD = *reinterpret_cast<const float2*>(vec + 64 + cv + c);
             const float2 nal = *reinterpret_cast<const float2*>(vec + 128 + cv + c);
             const float2 nE = *reinterpret_cast<const float2*>(vec + 192 + cv + c);
-            float2 pr = probs2(pair(rS[h], c), sl2v, nL2);
-            if (need_mask) {
-              if (c < lo || c >= hi) pr.x = 0.f;
-              if (c + 1 < lo || c + 1 >= hi) pr.y = 0.f;
-            }
+            const float2 pr = probs2(pair(rS[h], c), sl2v, nL2);
             const float2 f = __fmul2_rn(pair(rF[h], c), tauv);
             float2 dp = pair(rdP, c), cv = pair(rC, c), gp = pr;
             if constexpr (DROP) {  // dP, C and the Vtil operand gated by sigma R
@@ -1555,11 +1543,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
           for (int c = 0; c < 16; c += 2) {
             const float2 nL2 = *reinterpret_cast<const float2*>(vec + cv + c);
             const float2 nD = *reinterpret_cast<const float2*>(vec + 64 + cv + c);
-            float2 pr = probs2(pair(rS[h], c), sl2v, nL2);
-            if (need_mask) {
-              if (c < lo || c >= hi) pr.x = 0.f;
-              if (c + 1 < lo || c + 1 >= hi) pr.y = 0.f;
-            }
+            const float2 pr = probs2(pair(rS[h], c), sl2v, nL2);
             float2 dp = pair(rdP, c), gp = pr;
             if constexpr (DROP) {  // dV = (sigma R o P)^T dO, dS = P (sigma R dP - D)
               const float2 g = gate2(kb[h], c, dsig);
