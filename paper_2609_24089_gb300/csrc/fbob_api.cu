@@ -360,6 +360,37 @@ int check_host_args(const fbob_shape* s, const void* const* hin, void* const* ho
   return FBOB_OK;
 }
 
+// Chunk boundaries (in query heads, whole key/value groups) for chunks of at
+// most hc heads.  Only the first chunk's copy in and the last chunk's copy
+// out cannot overlap any kernel, so when there are more than two full chunks
+// those two are made about a quarter as large; the rest share the remainder
+// evenly.  Returns the number of chunks; starts[] gets nchunks + 1 entries.
+int64_t plan_chunks(int64_t BH, int64_t G, int64_t hc, int64_t* starts, int64_t max_chunks) {
+  const int64_t U = BH / G, b = hc / G;  // groups in all, per full chunk
+  int64_t n = 0;
+  starts[n] = 0;
+  if (U <= 2 * b || max_chunks < 4) {
+    for (int64_t u = 0; u < U && n + 1 < max_chunks;) {
+      u += (U - u) < b ? (U - u) : b;
+      starts[++n] = u * G;
+    }
+    return n;
+  }
+  const int64_t e = (b + 3) / 4;          // end chunks
+  const int64_t mid = U - 2 * e;          // groups for the middle chunks
+  int64_t m = (mid + b - 1) / b;          // middle chunks
+  if (m + 2 > max_chunks) m = max_chunks - 2;
+  int64_t u = e;
+  starts[++n] = u * G;
+  for (int64_t c = 0; c < m; ++c) {
+    u += mid / m + (c < mid % m ? 1 : 0);
+    starts[++n] = u * G;
+  }
+  u += e;
+  starts[++n] = u * G;
+  return n;
+}
+
 struct HostCall {
   cudaStream_t cin = nullptr, cout = nullptr;
   cudaEvent_t entry = nullptr, in[kSlots] = {}, comp[kSlots] = {}, out[kSlots] = {};
@@ -667,7 +698,13 @@ int fbob_attn_bob_host(const fbob_shape* s, const void* q, const void* k, const 
       cudaStreamWaitEvent(hcall.cin, hcall.entry, 0) != cudaSuccess ||
       cudaStreamWaitEvent(hcall.cout, hcall.entry, 0) != cudaSuccess)
     return FBOB_ERR_CUDA;
-  const int64_t nchunks = (BH + hc - 1) / hc;
+  // at most 64 chunks: above that, full chunks of hc heads end to end
+  int64_t starts[65];
+  const int64_t nfull = (BH + hc - 1) / hc;
+  int64_t nchunks = 0;
+  if (nfull + 2 <= 64) {
+    nchunks = plan_chunks(BH, G, hc, starts, 64);
+  }
   auto h2d = [&](void* dst, const void* src, int64_t bytes) {
     return cudaMemcpyAsync(dst, src, (size_t)bytes, cudaMemcpyHostToDevice, hcall.cin);
   };
@@ -677,12 +714,15 @@ int fbob_attn_bob_host(const fbob_shape* s, const void* q, const void* k, const 
   auto hb = [](const void* p, int64_t at) { return static_cast<const uint8_t*>(p) + at; };
   auto hbm = [](void* p, int64_t at) { return static_cast<uint8_t*>(p) + at; };
   int launches = 0;
-  for (int64_t c = 0; c < nchunks; ++c) {
+  const int64_t nloop = nchunks ? nchunks : nfull;
+  for (int64_t c = 0; c < nloop; ++c) {
     const int sl = (int)(c % kSlots);
     uint8_t* base = static_cast<uint8_t*>(workspace) + sl * slot;
     void* w[kBufs];
     for (int t = 0; t < kBufs; ++t) w[t] = base + off[t];
-    const int64_t f0 = c * hc, nq = (BH - f0) < hc ? (BH - f0) : hc, nkv = nq / G, k0 = f0 / G;
+    const int64_t f0 = nchunks ? starts[c] : c * hc;
+    const int64_t f1 = nchunks ? starts[c + 1] : ((f0 + hc) < BH ? (f0 + hc) : BH);
+    const int64_t nq = f1 - f0, nkv = nq / G, k0 = f0 / G;
     cudaError_t e = cudaSuccess;
     // copy in once the slot's previous chunk has been computed
     if (c >= kSlots) e = cudaStreamWaitEvent(hcall.cin, hcall.comp[sl], 0);
@@ -724,7 +764,7 @@ int fbob_attn_bob_host(const fbob_shape* s, const void* q, const void* k, const 
     if (e != cudaSuccess) return FBOB_ERR_CUDA;
   }
   // `stream` completes after the last copies out
-  for (int sl = 0; sl < kSlots && sl < nchunks; ++sl)
+  for (int sl = 0; sl < kSlots && sl < nloop; ++sl)
     if (cudaStreamWaitEvent(st, hcall.out[sl], 0) != cudaSuccess) return FBOB_ERR_CUDA;
   g_launches[kEntBobHost] = launches;
   return FBOB_OK;
