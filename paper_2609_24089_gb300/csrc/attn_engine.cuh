@@ -3,14 +3,16 @@
 //
 // Two engines share one schedule skeleton:
 //   * row engine: a CTA owns BM = 128 query rows (TMEM lanes) and streams key
-//     tiles of BN = 64 rows.  Used by the forward (eq. 1), the dQ half of the
-//     first backward (eqs. 2-3) and BoB Pass 1 (Alg. 2, first loop): at
+//     tiles of BN = 64 rows.  Used by the dQ half of the first backward
+//     (eqs. 2-3) and BoB Pass 1 (Alg. 2, first loop): at
 //     d = 64 in one sweep with the affine fusion of Prop. 3.1 (four
 //     accumulators); at d = 128 as a row-statistics kernel (alpha, E, D; stage
 //     A only) followed by the direct form of eqs. (6)-(7) (two accumulators).
 //   * column engine: a CTA owns BM = 128 key rows and streams query tiles of
 //     BN = 64 rows, computing transposed tiles (key rows on lanes).  Used by
 //     the dK/dV half of the first backward and BoB Pass 2 (Alg. 2, second loop).
+// The forward (eq. 1) has its own engine with two query tiles per CTA
+// (fwd_engine.cuh).
 //
 // Roles (352 threads):
 //   warps 0-7  elementwise: two warpgroups; warp w reads TMEM lanes
@@ -70,9 +72,6 @@ constexpr uint32_t kColDC1 = 128;  // second DC buffer (column engine, d = 64)
 // column, D/2 columns each) at kColQT and kColQT + D/2; second SF buffer
 constexpr uint32_t kColQT = 0;
 constexpr uint32_t kColSF1 = 128;
-// forward: slack (log2 units) by which a tile's row maximum may exceed the
-// running maximum before the accumulator is rescaled (P <= 2^kFwdSlack)
-constexpr float kFwdSlack = 8.f;
 
 // Shared-memory bookkeeping block (in the MISC area).
 struct Misc {
@@ -86,7 +85,6 @@ struct Misc {
   uint64_t bar_sa_dc[2];
   uint64_t bar_ew[4];   // [DC buffer][half]; a single DC buffer uses [0..1]
   uint64_t bar_xb[2];   // issuer X's stage-B MMAs completed (per half, or per DC buffer)
-  uint64_t bar_od[2];   // forward: issuer Y's O += P V MMAs of a tile completed (per P buffer)
   uint64_t bar_acc;
   uint32_t tmem_base;
   uint32_t pad;
@@ -271,7 +269,6 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
     for (int h = 0; h < 2; ++h) {
       mbar_init(&m->bar_sa_dc[h], 1);
       mbar_init(&m->bar_xb[h], 1);
-      mbar_init(&m->bar_od[h], 1);
     }
     for (int h = 0; h < 4; ++h) mbar_init(&m->bar_ew[h], kEwThreads);
     mbar_init(&m->bar_acc, 2);
@@ -456,26 +453,6 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
           }
           ok = false;
         }
-        if constexpr (OP == RowOp::Fwd) {
-          // S(t) = Q K^T into buffer t & 1 (columns kColSF + 64 b): X runs up
-          // to a tile ahead of the elementwise warps
-          for (int st = 0; ok && st < nsteps; ++st) {
-            const int b = st & 1;
-            const int stage = st % C::NSTAGES;
-            if ((st >= 2 && !mbar_wait(&m->bar_sf_free[b], ((st - 2) >> 1) & 1, wctl)) ||
-                !mbar_wait(&m->bar_full[stage], (st / C::NSTAGES) & 1, wctl))
-              break;
-            tc_fence_after();
-            const uint64_t kd0 =
-                sdesc_sw128(smem_u32(s_stream + stage * C::STAGE_BYTES), 16, 1024);
-#pragma unroll
-            for (int k = 0; k < D / 16; ++k)
-              mma_ss(tmem + kColSF + 64 * b, sd(0, k), kd(kd0, 0, 0, k), id_n64, k > 0);
-            mma_commit(&m->bar_sa_sf[b]);
-            mma_commit(&m->bar_empty[stage]);
-          }
-          ok = false;
-        }
         ok = ok && mbar_wait(&m->bar_full[0], 0, wctl);
         if (ok) {
           tc_fence_after();
@@ -565,31 +542,6 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
           }
           ok = false;  // no stage B
         }
-        if constexpr (OP == RowOp::Fwd) {
-          // O_wg += P_wg V: the 16-key K-step s of a tile belongs to
-          // warpgroup s & 1, whose accumulator sits at columns (s & 1) D
-          constexpr uint32_t kBoxBytes = C::NSTREAM * BN * 128;
-          for (int st = 0; ok && st < nsteps; ++st) {
-            const int b = st & 1;
-            const int stage = st % C::NSTAGES;
-            if (!mbar_wait(&m->bar_full[stage], (st / C::NSTAGES) & 1, wctl) ||
-                !mbar_wait(&m->bar_ew[b], (st >> 1) & 1, wctl))
-              break;
-            tc_fence_after();
-            const uint64_t md0 =
-                sdesc_sw128(smem_u32(s_stream + stage * C::STAGE_BYTES), kBoxBytes, 1024);
-#pragma unroll
-            for (int s4 = 0; s4 < 4; ++s4) {
-              const uint64_t vd =
-                  md0 + (uint64_t)((soff<C::NSTREAM, false>(1, s4 >> 1, 0) + (s4 & 1) * 2048) >> 4);
-              mma_ts(tmem + (s4 & 1) * D, tmem + kColDC + 32 * b + 8 * s4, vd, id_b,
-                     (st == 0 && s4 < 2) ? 0u : 1u);
-            }
-            mma_commit(&m->bar_od[b]);
-            mma_commit(&m->bar_empty[stage]);
-          }
-          ok = false;
-        }
         if (ok) {
           tc_fence_after();
           const uint32_t sb0 = smem_u32(s_stream);
@@ -670,7 +622,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
       return w;
     };
     float L2 = 0.f, Dr = 0.f, nal = 0.f, nE = 0.f;  // nal = -alpha, nE = -E (direct form)
-    if constexpr (OP != RowOp::Fwd) {
+    {
       if (row_ok) {
         const size_t ri = (size_t)bh * N + gi;
         L2 = p.lse[ri] * kLog2e;
@@ -705,141 +657,6 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
       tc_fence_before();
       mbar_arrive(&m->bar_stat);
     }
-    if constexpr (OP == RowOp::Fwd) {
-      // ---- single-sweep forward (eq. 1) with an online softmax.  Warpgroup
-      // wg owns the keys of its columns (K-steps s with s & 1 == wg) and its
-      // own accumulator O_wg (TMEM columns wg D .. +D).  Its running row
-      // maximum m (log2 domain) is raised only when a tile's maximum exceeds
-      // it by more than kFwdSlack, so P = 2^(x - m) <= 2^kFwdSlack, and O_wg
-      // is rescaled only then, after the MMAs into it have completed.  The
-      // two warpgroups' (m, l, O) are combined once, in the epilogue.
-      float mrow = -INFINITY, lrow = 0.f;
-      bool ok = true;
-      const uint32_t ocol = (uint32_t)(wg * D);
-      for (int st = 0; ok && st < nsteps; ++st) {
-        const int b = st & 1;
-        const uint32_t par = (st >> 1) & 1;
-        uint32_t kb[2];
-        if constexpr (DROP) tile_keep((first_tile + st) * BN, kb);
-        if (!ew_wait(&m->bar_sa_sf[b], par)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-        uint32_t rS[2][16];
-#pragma unroll
-        for (int h = 0; h < 2; ++h) tmem_ld16(ta + kColSF + 64 * b + HB * h + 16 * wg, rS[h]);
-        tmem_ld_wait(rS[0]);
-        reg_dep(rS[1]);
-        tc_fence_before();
-        mbar_arrive(&m->bar_sf_free[b]);
-        const int jt = (first_tile + st) * BN;
-        float x[2][16];  // raw scores (masked: -inf); the log2 scale enters below
-        float mraw = -INFINITY;
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const int j0 = jt + HB * h + 16 * wg;
-          const int mlo = jlo - j0, mhi = jhi - j0;  // valid columns: mlo <= c < mhi
-          if (mlo > 0 || mhi < 16) mask16(rS[h], mlo, mhi);
-#pragma unroll
-          for (int c = 0; c < 16; ++c) {
-            x[h][c] = bits_f(rS[h][c]);
-            mraw = fmaxf(mraw, x[h][c]);
-          }
-        }
-        const float mt = mraw * sl2;  // the tile's row maximum in log2 units (sl2 > 0)
-        const bool raise = mt > mrow + kFwdSlack;  // also the first tile with a valid key
-        const bool rescale = raise && mrow != -INFINITY;
-        if (__any_sync(0xffffffffu, rescale)) {
-          // every MMA into O_wg so far (tiles < st) must have completed
-          if (!ew_wait(&m->bar_od[(st - 1) & 1], ((st - 1) >> 1) & 1)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          const float f = rescale ? ex2(mrow - mt) : 1.f;
-#pragma unroll 1
-          for (int q = 0; q < D / 16; ++q) {
-            uint32_t o[16];
-            tmem_ld16(ta + ocol + 16 * q, o);
-            tmem_ld_wait(o);
-            uint32_t lo8[8], hi8[8];
-#pragma unroll
-            for (int c = 0; c < 8; ++c) {
-              lo8[c] = __float_as_uint(bits_f(o[c]) * f);
-              hi8[c] = __float_as_uint(bits_f(o[8 + c]) * f);
-            }
-            tmem_st8(ta + ocol + 16 * q, lo8);
-            tmem_st8(ta + ocol + 16 * q + 8, hi8);
-          }
-          tmem_st_wait();
-          if (rescale) lrow *= f;
-        }
-        if (raise) mrow = mt;
-        float psum = 0.f;
-        uint32_t oP[2][8];
-        // no valid key yet in this row: m = -inf and every score is -inf, so
-        // any finite stand-in for m gives P = 2^-inf = 0
-        const float nm = mrow == -INFINITY ? 0.f : -mrow;
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-#pragma unroll
-          for (int c = 0; c < 16; c += 2) {
-            float p0 = ex2(fmaf(x[h][c], sl2, nm));  // P = 2^(s tau log2 e - m)
-            float p1 = ex2(fmaf(x[h][c + 1], sl2, nm));
-            psum += p0 + p1;  // L over the ungated P
-            if constexpr (DROP) {  // O = sigma (R o P) V: sigma in the epilogue
-              if (!((kb[h] >> c) & 1u)) p0 = 0.f;
-              if (!((kb[h] >> (c + 1)) & 1u)) p1 = 0.f;
-            }
-            oP[h][c / 2] = pack_bf16(p0, p1);
-          }
-        }
-        lrow += psum;
-        // P buffer b was last read by the MMAs of tile st - 2
-        if (st >= 2 && !ew_wait(&m->bar_od[b], par ^ 1u)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-#pragma unroll
-        for (int h = 0; h < 2; ++h) tmem_st8(ta + kColDC + 32 * b + 8 * (2 * h + wg), oP[h]);
-        tmem_st_wait();
-        tc_fence_before();
-        mbar_arrive(&m->bar_ew[b]);
-      }
-      // ---- epilogue: O = (O_0 2^(m0-M) + O_1 2^(m1-M)) / l, L = M + log2 l
-      if (ok) ok = mbar_wait(&m->bar_acc, 0, wctl);
-      if (ok && *abort_flag) ok = false;
-      tc_fence_after();
-      s_xchg[wg * BM + r] = mrow;
-      s_xchg[(2 + wg) * BM + r] = lrow;
-      named_bar_sync(1, kEwThreads);
-      if (ok) {
-        const float m0 = s_xchg[r], m1 = s_xchg[BM + r];
-        const float mm = fmaxf(m0, m1);
-        const float f0 = m0 == -INFINITY ? 0.f : ex2(m0 - mm);
-        const float f1 = m1 == -INFINITY ? 0.f : ex2(m1 - mm);
-        const float lt = s_xchg[2 * BM + r] * f0 + s_xchg[3 * BM + r] * f1;
-        const float inv = row_ok ? (DROP ? dsig : 1.f) / lt : 0.f;
-#pragma unroll 1
-        for (int q = 0; q < D / 32; ++q) {
-          const int cc = wg * (D / 2) + 16 * q;  // output columns of this warpgroup
-          uint32_t a0[16], a1[16];
-          tmem_ld16(ta + cc, a0);
-          tmem_ld16(ta + D + cc, a1);
-          tmem_ld_wait(a0);
-          reg_dep(a1);
-          if (row_ok && cc < DG) {
-            float v[16];
-#pragma unroll
-            for (int c = 0; c < 16; ++c) v[c] = (bits_f(a0[c]) * f0 + bits_f(a1[c]) * f1) * inv;
-            store_row16(p.out0 + rowoff + cc, v);
-          }
-        }
-        if (row_ok && wg == 0) p.vec_out[(size_t)bh * N + gi] = (mm + __log2f(lt)) * kLn2;
-      }
-    } else {
     float2 acc_a = splat(0.f), acc_e = splat(0.f);  // Pass 1 partial row sums
     bool ok = true;
     for (int st = 0; ok && st < nsteps; ++st) {
@@ -1110,7 +927,6 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         if (row_ok && wg == 0) p.vec_out[(size_t)bh * N + gi] = Dr;
       }
     }
-    }  // elementwise: operations other than the forward
   }
   tc_fence_before();
   __syncthreads();

@@ -28,6 +28,7 @@ constexpr float kLn2 = 0.6931471805599453f;
 // BobPass1: Pass 1 in one sweep with the affine fusion of Prop. 3.1 (d = 64).
 // BobStats + BobPass1D: Pass 1 in two kernels (d = 128): the row scalars
 // alpha, E (and D) first, then Qtil and dOtil directly from eqs. (6)-(7).
+// (Fwd names the forward for the launcher; it runs in fwd_engine.cuh.)
 enum class RowOp { Fwd, BwdDQ, BobPass1, BobStats, BobPass1D };
 enum class ColOp { BwdDKDV, BobPass2 };
 
@@ -75,7 +76,7 @@ constexpr bool row_bob(RowOp op) {
 template <RowOp OP, int D>
 struct RowCfg {
   static constexpr int KB = D / 64;  // 64-wide boxes per row
-  static constexpr int NSTAT = OP == RowOp::Fwd ? 1 : OP == RowOp::BwdDQ ? 2 : 3;
+  static constexpr int NSTAT = OP == RowOp::BwdDQ ? 2 : 3;
   static constexpr int NSTREAM = row_bob(OP) ? 4 : 2;
   // the one-sweep Pass 1 holds four D-column accumulators: d = 64 only
   static_assert(OP != RowOp::BobPass1 || D == 64, "one-sweep Pass 1 needs d = 64");

@@ -471,7 +471,7 @@ int fbob_attn_fwd(const fbob_shape* s, const void* q, const void* k, const void*
     return FBOB_ERR_CUDA;
   p.out0 = static_cast<__nv_bfloat16*>(o);
   p.vec_out = lse;
-  p.nblk = n_blocks(s->N, BM);
+  p.nblk = n_blocks(s->N, 2 * BM);  // two 128-row query tiles per CTA
   choose_order(&p, 0);
   rc = launch_status(launch_row(RowOp::Fwd, (int)s->d, has_dropout(s), p, p.nblk * p.BH, stream));
   if (rc == FBOB_OK) g_launches[kEntFwd] = 1;

@@ -1,0 +1,366 @@
+// fwd_engine.cuh -- forward attention (eq. 1) on sm_103a with two query
+// tiles per CTA.
+//
+// A CTA owns 2 x 128 query rows of one head (query tiles 0 and 1) and streams
+// 128-key tiles of K and V through a ring of stream stages.  Each query tile
+// has its own score buffer S_q (128 TMEM columns) and accumulator O_q, and
+// its own softmax warpgroup, whose thread i holds query row i whole.  Per key
+// tile T and query tile q:
+//   X   S_q(T) = Q_q K(T)^T                 (N = 128, issuer X)
+//   WGq m, l (online softmax), P = 2^(S tau log2 e - m) written as bf16 over
+//       the first 64 columns of S_q (all of S_q is in registers by then)
+//   Y   O_q += P_q(T) V(T)                  (A from TMEM, issuer Y)
+// X issues S_q(T+1) once O_q += P_q(T) V(T) has completed (it overwrites
+// P_q(T)).  The two query tiles' chains interleave, so the tensor pipe works
+// on one tile while the other's softmax runs.  The running maximum is raised
+// lazily (by more than kFwdSlack2, so P <= 2^kFwdSlack2); O_q is then
+// rescaled by its warpgroup after the MMAs into it have completed.
+//
+// Roles (352 threads): warps 0-3 softmax of query tile 0, warps 4-7 of tile
+// 1 (warp w reads TMEM lanes 32 (w % 4) .. +31), warp 8 TMA producer,
+// warp 9 issuer X, warp 10 issuer Y.  Every wait is bounded.
+#pragma once
+
+#include "attn_engine.cuh"
+
+namespace fbob {
+
+constexpr int kFwdRows = 2 * BM;  // query rows per CTA
+constexpr int BN2 = 128;          // keys per streamed tile
+constexpr float kFwdSlack2 = 8.f;
+
+template <int D>
+struct FwdCfg {
+  static constexpr int KB = D / 64;
+  static constexpr int STAT_BYTES = 2 * KB * BM * 128;     // Q_0, Q_1
+  static constexpr int STAGE_BYTES = 2 * KB * BN2 * 128;   // K, V
+  static constexpr int NSTAGES = D == 64 ? 4 : 2;
+  static constexpr int MISC_BYTES = 256;
+  static constexpr int SMEM_BYTES = STAT_BYTES + NSTAGES * STAGE_BYTES + MISC_BYTES;
+};
+
+struct FwdMisc {
+  uint64_t bar_stat;
+  uint64_t full[4];
+  uint64_t empty[4];
+  uint64_t s_full[2];  // S_q(T) computed (issuer X)
+  uint64_t p_full[2];  // P_q(T) written (128 softmax threads)
+  uint64_t o_done[2];  // O_q += P_q(T) V(T) completed (issuer Y)
+  uint64_t bar_acc;    // every MMA of both issuers completed (abort drain)
+  uint32_t tmem_base;
+  uint32_t pad;
+  WaitCtl wctl;
+};
+static_assert(sizeof(FwdMisc) <= 256, "FwdMisc must fit the MISC area");
+
+// TMEM columns: O_q at q D, S_q at 256 + 128 q.
+constexpr uint32_t kColS2 = 256;
+
+template <int D, bool DROP, int DG>
+__global__ void __launch_bounds__(kThreads, 1) fwd_engine(const __grid_constant__ EngineParams p) {
+  using C = FwdCfg<D>;
+  static_assert(DG == D || (DG == 32 && D == 64), "global head dim 32 runs in 64-wide tiles");
+  extern __shared__ __align__(1024) uint8_t smem[];
+  uint8_t* s_stat = smem;
+  uint8_t* s_stream = smem + C::STAT_BYTES;
+  FwdMisc* m = reinterpret_cast<FwdMisc*>(s_stream + C::NSTAGES * C::STAGE_BYTES);
+
+  const int tid = threadIdx.x;
+  const int warp = tid >> 5;
+  if ((smem_u32(smem) & 1023u) != 0) {
+    if (tid == 0) atomicOr(&g_fbob_error_word, kDevErrBadLaunch);
+    return;
+  }
+  // ---- tile decode: 256 query rows; with the causal mask the row blocks
+  // with the most keys go first
+  const int N = p.N;
+  const int lin = blockIdx.x;
+  const int rbi = p.head_major ? lin % p.nblk : lin / p.BH;
+  const int bh = p.head_major ? lin / p.nblk : lin % p.BH;
+  const int rb = p.causal ? (p.nblk - 1 - rbi) : rbi;
+  const int bh_kv = p.Hkv == p.H ? bh : (bh / p.H) * p.Hkv + (bh % p.H) / (p.H / p.Hkv);
+  const int i0 = rb * kFwdRows;
+  // per query tile: active, and its key tiles [tq0, tq1] (the union of its
+  // rows' bands within their sequences)
+  bool act[2];
+  int tq0[2], tq1[2];
+#pragma unroll
+  for (int q = 0; q < 2; ++q) {
+    const int first = i0 + BM * q;
+    act[q] = first < N;
+    tq0[q] = 0;
+    tq1[q] = -1;
+    if (act[q]) {
+      const int last = min(first + BM, N) - 1;
+      int s0, e0, s1, e1;
+      seq_bounds(p, first, s0, e0);
+      seq_bounds(p, last, s1, e1);
+      const int lo = max(s0, p.wl < 0 ? 0 : first - p.wl);
+      const int hi = min(e1, p.wr < 0 ? N : last + p.wr + 1);
+      tq0[q] = lo / BN2;
+      tq1[q] = (hi - 1) / BN2;
+    }
+  }
+  const int T0 = act[1] ? min(tq0[0], tq0[1]) : tq0[0];
+  const int T1 = act[1] ? max(tq1[0], tq1[1]) : tq1[0];
+  const int nsteps = T1 - T0 + 1;
+  auto part = [&](int q, int T) { return act[q] && T >= tq0[q] && T <= tq1[q]; };
+
+  if (tid == 0) {
+    m->wctl.abort = 0;
+    m->wctl.limit_ns = p.wait_limit_ns;
+    mbar_init(&m->bar_stat, 1);
+    for (int s = 0; s < C::NSTAGES; ++s) {
+      mbar_init(&m->full[s], 1);
+      mbar_init(&m->empty[s], 2);  // issuers X and Y
+    }
+    for (int q = 0; q < 2; ++q) {
+      mbar_init(&m->s_full[q], 1);
+      mbar_init(&m->p_full[q], BM);
+      mbar_init(&m->o_done[q], 1);
+    }
+    mbar_init(&m->bar_acc, 2);
+    fence_mbar_init();
+  }
+  if (warp == kMmaWarp) {
+    tmem_alloc(&m->tmem_base, kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = m->tmem_base;
+  WaitCtl* wctl = &m->wctl;
+  volatile int* abort_flag = &m->wctl.abort;
+
+  if (warp == kProducerWarp) {
+    // ------------------------------------------------------------ producer
+    if (elect_lane0() && !p.inject_stall) {
+      for (int t = 0; t < 3; ++t) tma_prefetch_desc(&p.tm[t]);
+      mbar_arrive_expect_tx(&m->bar_stat, C::STAT_BYTES);
+      for (int q = 0; q < 2; ++q)
+        for (int b = 0; b < C::KB; ++b)
+          tma_load_3d(s_stat + (q * C::KB + b) * (BM * 128), &p.tm[0], &m->bar_stat, 64 * b,
+                      i0 + BM * q, bh);
+      int issued[4] = {-1, -1, -1, -1};
+      for (int st = 0; st < nsteps; ++st) {
+        const int stage = st % C::NSTAGES;
+        if (st >= C::NSTAGES &&
+            !mbar_wait(&m->empty[stage], ((st / C::NSTAGES) - 1) & 1, wctl))
+          break;
+        const int j0 = (T0 + st) * BN2;
+        uint8_t* dst = s_stream + stage * C::STAGE_BYTES;
+        mbar_arrive_expect_tx(&m->full[stage], C::STAGE_BYTES);
+        for (int t = 0; t < 2; ++t)        // K, V
+          for (int b = 0; b < C::KB; ++b)
+            for (int h = 0; h < 2; ++h)    // two 64-row boxes
+              tma_load_3d(dst + (t * C::KB + b) * (BN2 * 128) + h * (BN * 128), &p.tm[1 + t],
+                          &m->full[stage], 64 * b, j0 + BN * h, bh_kv);
+        issued[stage] = st;
+      }
+      if (*abort_flag) {
+        for (int s = 0; s < C::NSTAGES; ++s)
+          if (issued[s] >= 0) drain_wait(&m->full[s], (issued[s] / C::NSTAGES) & 1);
+        drain_wait(&m->bar_stat, 0);
+      }
+    }
+  } else if (warp == kMmaWarp || warp == kMmaWarpY) {
+    // ------------------------------------------------------------ MMA issuers
+    if (elect_lane0()) {
+      constexpr uint32_t id_s = idesc_bf16(128, BN2, false);
+      constexpr uint32_t id_o = idesc_bf16(128, D, true);
+      bool ok = true;
+      if (warp == kMmaWarp) {
+        // ---------------- issuer X: S_q(T) = Q_q K(T)^T
+        const uint64_t qd0 = sdesc_sw128(smem_u32(s_stat), 16, 1024);
+        ok = mbar_wait(&m->bar_stat, 0, wctl);
+        for (int st = 0; ok && st < nsteps; ++st) {
+          const int T = T0 + st;
+          const int stage = st % C::NSTAGES;
+          if (!mbar_wait(&m->full[stage], (st / C::NSTAGES) & 1, wctl)) break;
+          const uint64_t kd0 =
+              sdesc_sw128(smem_u32(s_stream + stage * C::STAGE_BYTES), 16, 1024);
+          for (int q = 0; q < 2 && ok; ++q) {
+            if (!part(q, T)) continue;
+            const int k = T - tq0[q];
+            // S_q(T) overwrites P_q(T-1): wait for O_q += P_q(T-1) V
+            if (k >= 1 && !mbar_wait(&m->o_done[q], (k - 1) & 1, wctl)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk) {
+              const uint64_t qd =
+                  qd0 + (uint64_t)(((q * C::KB + kk / 4) * (BM * 128) + (kk % 4) * 32) >> 4);
+              const uint64_t kd = kd0 + (uint64_t)(((kk / 4) * (BN2 * 128) + (kk % 4) * 32) >> 4);
+              mma_ss(tmem + kColS2 + 128 * q, qd, kd, id_s, kk > 0);
+            }
+            mma_commit(&m->s_full[q]);
+          }
+          if (!ok) break;
+          mma_commit(&m->empty[stage]);
+        }
+      } else {
+        // ---------------- issuer Y: O_q += P_q(T) V(T)
+        for (int st = 0; ok && st < nsteps; ++st) {
+          const int T = T0 + st;
+          const int stage = st % C::NSTAGES;
+          if (!mbar_wait(&m->full[stage], (st / C::NSTAGES) & 1, wctl)) break;
+          // V of this stage: MN-major, 64-wide boxes BN2 * 128 bytes apart
+          const uint64_t vd0 = sdesc_sw128(
+              smem_u32(s_stream + stage * C::STAGE_BYTES) + C::KB * (BN2 * 128), BN2 * 128, 1024);
+          for (int q = 0; q < 2 && ok; ++q) {
+            if (!part(q, T)) continue;
+            const int k = T - tq0[q];
+            if (!mbar_wait(&m->p_full[q], k & 1, wctl)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+#pragma unroll
+            for (int ks = 0; ks < BN2 / 16; ++ks)
+              mma_ts(tmem + q * D, tmem + kColS2 + 128 * q + 8 * ks,
+                     vd0 + (uint64_t)((ks * 2048) >> 4), id_o, (k == 0 && ks == 0) ? 0u : 1u);
+            mma_commit(&m->o_done[q]);
+          }
+          if (!ok) break;
+          mma_commit(&m->empty[stage]);
+        }
+      }
+      mma_commit(&m->bar_acc);
+      if (*abort_flag) drain_wait(&m->bar_acc, 0);
+    }
+  } else {
+    // ------------------------------------------------------------ softmax
+    const int q = warp >> 2;                     // query tile of this warpgroup
+    const int r = 32 * (warp & 3) + (tid & 31);  // row in the tile (TMEM lane)
+    const int gi = i0 + BM * q + r;
+    const bool row_ok = gi < N;
+    int jlo = 0, jhi = 0;  // this row's valid keys [jlo, jhi)
+    if (row_ok) {
+      seq_bounds(p, gi, jlo, jhi);
+      if (p.wl >= 0) jlo = max(jlo, gi - p.wl);
+      if (p.wr >= 0) jhi = min(jhi, gi + p.wr + 1);
+    }
+    const uint32_t ta = lane_base_addr(tmem, warp);
+    const uint32_t scol = kColS2 + 128 * q, ocol = (uint32_t)(q * D);
+    const float sl2 = p.scale * kLog2e;
+    const DropKey dkey = {p.drop_rk, p.drop_tlow4, p.drop_tmask};
+    auto ew_wait = [&](uint64_t* bar, uint32_t par) -> bool {
+      const bool w = mbar_wait(bar, par, wctl);
+      return __all_sync(0xffffffffu, w);  // the warp leaves together
+    };
+    float mrow = -INFINITY, lrow = 0.f;
+    bool ok = act[q];
+    const int nq = act[q] ? tq1[q] - tq0[q] + 1 : 0;
+    for (int k = 0; ok && k < nq; ++k) {
+      const int jt = (tq0[q] + k) * BN2;
+      if (!ew_wait(&m->s_full[q], k & 1)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      uint32_t rS[8][16];
+#pragma unroll
+      for (int c = 0; c < 8; ++c) tmem_ld16(ta + scol + 16 * c, rS[c]);
+      tmem_ld_wait(rS[0]);
+#pragma unroll
+      for (int c = 1; c < 8; ++c) reg_dep(rS[c]);
+      float mraw = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < 8; ++c) {
+        const int mlo = jlo - (jt + 16 * c), mhi = jhi - (jt + 16 * c);
+        if (mlo > 0 || mhi < 16) mask16(rS[c], mlo, mhi);
+#pragma unroll
+        for (int e = 0; e < 16; ++e) mraw = fmaxf(mraw, bits_f(rS[c][e]));
+      }
+      const float mt = mraw * sl2;
+      const bool raise = mt > mrow + kFwdSlack2;  // also the first tile with a valid key
+      const bool rescale = raise && mrow != -INFINITY;
+      if (__any_sync(0xffffffffu, rescale)) {
+        // every MMA into O_q so far (tiles before k) must have completed
+        if (!ew_wait(&m->o_done[q], (k - 1) & 1)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const float f = rescale ? ex2(mrow - mt) : 1.f;
+#pragma unroll 1
+        for (int c = 0; c < D / 16; ++c) {
+          uint32_t o[16];
+          tmem_ld16(ta + ocol + 16 * c, o);
+          tmem_ld_wait(o);
+          uint32_t lo8[8], hi8[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            lo8[e] = __float_as_uint(bits_f(o[e]) * f);
+            hi8[e] = __float_as_uint(bits_f(o[8 + e]) * f);
+          }
+          tmem_st8(ta + ocol + 16 * c, lo8);
+          tmem_st8(ta + ocol + 16 * c + 8, hi8);
+        }
+        tmem_st_wait();
+        if (rescale) lrow *= f;
+      }
+      if (raise) mrow = mt;
+      // no valid key yet: every score is -inf, so any finite m gives P = 0
+      const float nm = mrow == -INFINITY ? 0.f : -mrow;
+      float ps0 = 0.f, ps1 = 0.f;
+#pragma unroll
+      for (int c = 0; c < 8; ++c) {
+        uint32_t oP[8];
+        // dropout keep bits of keys jt + 16c .. + 15 (the whole warp shuffles)
+        const uint32_t kbc =
+            DROP ? keep_row16(gi, jt + 16 * c, (uint32_t)(p.head0 + bh), dkey) : 0u;
+#pragma unroll
+        for (int e = 0; e < 16; e += 2) {
+          float p0 = ex2(fmaf(bits_f(rS[c][e]), sl2, nm));
+          float p1 = ex2(fmaf(bits_f(rS[c][e + 1]), sl2, nm));
+          ps0 += p0;
+          ps1 += p1;  // L over the ungated P
+          if constexpr (DROP) {  // O = sigma (R o P) V: sigma in the epilogue
+            if (!((kbc >> e) & 1u)) p0 = 0.f;
+            if (!((kbc >> (e + 1)) & 1u)) p1 = 0.f;
+          }
+          oP[e / 2] = pack_bf16(p0, p1);
+        }
+        // P of keys 16c .. 16c+15 over S columns 8c .. 8c+7 (already in registers)
+        tmem_st8(ta + scol + 8 * c, oP);
+      }
+      lrow += ps0 + ps1;
+      tmem_st_wait();
+      tc_fence_before();
+      mbar_arrive(&m->p_full[q]);
+    }
+    // ---- epilogue: O = O_q / l (times sigma with dropout), L = m + log2 l
+    if (ok && nq > 0) ok = ew_wait(&m->o_done[q], (nq - 1) & 1);
+    if (ok && *abort_flag) ok = false;
+    tc_fence_after();
+    if (ok) {
+      const float inv = row_ok ? (DROP ? p.drop_sigma : 1.f) / lrow : 0.f;
+      const size_t rowoff = ((size_t)bh * N + (size_t)(row_ok ? gi : 0)) * DG;
+#pragma unroll 1
+      for (int c = 0; c < D / 16; ++c) {
+        uint32_t o[16];
+        tmem_ld16(ta + ocol + 16 * c, o);
+        tmem_ld_wait(o);
+        if (row_ok && 16 * c < DG) {
+          float v[16];
+#pragma unroll
+          for (int e = 0; e < 16; ++e) v[e] = bits_f(o[e]) * inv;
+          store_row16(p.out0 + rowoff + 16 * c, v);
+        }
+      }
+      if (row_ok) p.vec_out[(size_t)bh * N + gi] = (mrow + __log2f(lrow)) * kLn2;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == kMmaWarp) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+}  // namespace fbob

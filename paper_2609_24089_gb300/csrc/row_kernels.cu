@@ -1,9 +1,10 @@
-// row_kernels.cu -- instantiations and launcher of the row-block engine:
-// forward (eq. 1), first-backward dQ (eqs. 2-3), BoB Pass 1 (Algorithm 2,
+// row_kernels.cu -- instantiations and launcher of the row-block kernels:
+// forward (eq. 1, fwd_engine.cuh), first-backward dQ (eqs. 2-3), BoB Pass 1 (Algorithm 2,
 // first loop): one sweep at d <= 64, row statistics + direct form at d = 128
 // (and at any d with dropout).  Each operation with and without dropout, for
 // head dims 32 (in 64-wide tiles), 64 and 128.
 #include "attn_engine.cuh"
+#include "fwd_engine.cuh"
 #include "launch.h"
 
 namespace fbob {
@@ -34,10 +35,32 @@ static cudaError_t launch_op(int d, bool drop, const EngineParams& p, int nblock
   return drop ? launch_d<OP, true>(d, p, nblocks, s) : launch_d<OP, false>(d, p, nblocks, s);
 }
 
+// the forward: two query tiles per CTA (fwd_engine.cuh)
+template <int D, bool DROP, int DG = D>
+static cudaError_t launch_fwd_one(const EngineParams& p, int nblocks, cudaStream_t s) {
+  const int smem = launch_smem(FwdCfg<D>::SMEM_BYTES);
+  cudaError_t e = cudaFuncSetAttribute(fwd_engine<D, DROP, DG>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  fwd_engine<D, DROP, DG><<<nblocks, kThreads, smem, s>>>(p);
+  return cudaGetLastError();
+}
+
+template <bool DROP>
+static cudaError_t launch_fwd(int d, const EngineParams& p, int nblocks, cudaStream_t s) {
+  switch (d) {
+    case 32: return launch_fwd_one<64, DROP, 32>(p, nblocks, s);
+    case 64: return launch_fwd_one<64, DROP>(p, nblocks, s);
+    case 128: return launch_fwd_one<128, DROP>(p, nblocks, s);
+  }
+  return cudaErrorInvalidValue;
+}
+
 cudaError_t launch_row(RowOp op, int d, bool drop, const EngineParams& p, int nblocks,
                        cudaStream_t s) {
   switch (op) {
-    case RowOp::Fwd: return launch_op<RowOp::Fwd>(d, drop, p, nblocks, s);
+    case RowOp::Fwd:
+      return drop ? launch_fwd<true>(d, p, nblocks, s) : launch_fwd<false>(d, p, nblocks, s);
     case RowOp::BwdDQ: return launch_op<RowOp::BwdDQ>(d, drop, p, nblocks, s);
     case RowOp::BobPass1:  // the one-sweep form serves d <= 64 without dropout only
       if (drop) return cudaErrorInvalidValue;
