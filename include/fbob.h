@@ -212,9 +212,10 @@ int fbob_attn_bob_pass1_direct(const fbob_shape* shape, const void* q, const voi
  * fbob_attn_bob with every tensor in host memory: the same computation and
  * the same results, bit for bit.  The B*H query heads are processed in
  * chunks of whole key/value groups, and each chunk's inputs are copied in,
- * computed and copied out on three streams through two slots of a
+ * computed and copied out on separate streams through two slots of a
  * caller-owned device workspace, so copies and kernels of neighbouring
- * chunks overlap (each head is an independent problem, Alg. 1).
+ * chunks overlap, and so do the kernels of consecutive chunks (each head is
+ * an independent problem, Alg. 1).
  * In:  q, k, v, o, lse, dout, gq, gk, gv: host buffers with the layouts of
  *      fbob_attn_bob.  Page-locked memory lets the copies run asynchronously;
  *      pageable memory gives the same results, without the overlap.
@@ -228,8 +229,8 @@ int fbob_attn_bob_pass1_direct(const fbob_shape* shape, const void* q, const voi
  *      cannot hold one key/value group.
  * Stream: the copies start after the work already enqueued on `stream`, and
  *      `stream` completes only after the last copy out; synchronise it before
- *      reading the outputs.  Two streams and seven events are created per call
- *      and released when their work completes.
+ *      reading the outputs.  Three streams and seven events are created per
+ *      call and released when their work completes.
  */
 int fbob_attn_bob_host(const fbob_shape* shape, const void* q, const void* k, const void* v,
                        const void* o, const float* lse, const void* dout,

@@ -392,7 +392,7 @@ int64_t plan_chunks(int64_t BH, int64_t G, int64_t hc, int64_t* starts, int64_t 
 }
 
 struct HostCall {
-  cudaStream_t cin = nullptr, cout = nullptr;
+  cudaStream_t cin = nullptr, cout = nullptr, cmp = nullptr;
   cudaEvent_t entry = nullptr, in[kSlots] = {}, comp[kSlots] = {}, out[kSlots] = {};
   ~HostCall() {  // released once their pending work completes
     if (entry) cudaEventDestroy(entry);
@@ -403,10 +403,12 @@ struct HostCall {
     }
     if (cin) cudaStreamDestroy(cin);
     if (cout) cudaStreamDestroy(cout);
+    if (cmp) cudaStreamDestroy(cmp);
   }
   cudaError_t init() {
     cudaError_t e = cudaStreamCreateWithFlags(&cin, cudaStreamNonBlocking);
     if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&cout, cudaStreamNonBlocking);
+    if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&cmp, cudaStreamNonBlocking);
     if (e == cudaSuccess) e = cudaEventCreateWithFlags(&entry, cudaEventDisableTiming);
     for (int t = 0; t < kSlots && e == cudaSuccess; ++t) {
       e = cudaEventCreateWithFlags(&in[t], cudaEventDisableTiming);
@@ -696,7 +698,8 @@ int fbob_attn_bob_host(const fbob_shape* s, const void* q, const void* k, const 
   // the workspace or the host buffers)
   if (cudaEventRecord(hcall.entry, st) != cudaSuccess ||
       cudaStreamWaitEvent(hcall.cin, hcall.entry, 0) != cudaSuccess ||
-      cudaStreamWaitEvent(hcall.cout, hcall.entry, 0) != cudaSuccess)
+      cudaStreamWaitEvent(hcall.cout, hcall.entry, 0) != cudaSuccess ||
+      cudaStreamWaitEvent(hcall.cmp, hcall.entry, 0) != cudaSuccess)
     return FBOB_ERR_CUDA;
   // at most 64 chunks: above that, full chunks of hc heads end to end
   int64_t starts[65];
@@ -723,6 +726,9 @@ int fbob_attn_bob_host(const fbob_shape* s, const void* q, const void* k, const 
     const int64_t f0 = nchunks ? starts[c] : c * hc;
     const int64_t f1 = nchunks ? starts[c + 1] : ((f0 + hc) < BH ? (f0 + hc) : BH);
     const int64_t nq = f1 - f0, nkv = nq / G, k0 = f0 / G;
+    // the slots' chunks alternate between two compute streams, so the next
+    // chunk's kernels fill the SMs the previous chunk's last wave leaves idle
+    cudaStream_t cs = sl ? hcall.cmp : st;
     cudaError_t e = cudaSuccess;
     // copy in once the slot's previous chunk has been computed
     if (c >= kSlots) e = cudaStreamWaitEvent(hcall.cin, hcall.comp[sl], 0);
@@ -735,22 +741,22 @@ int fbob_attn_bob_host(const fbob_shape* s, const void* q, const void* k, const 
     if (e == cudaSuccess) e = h2d(w[4], hb(lse, f0 * N * 4), nq * N * 4);
     if (e == cudaSuccess) e = cudaEventRecord(hcall.in[sl], hcall.cin);
     // compute once the inputs are in and the slot's previous outputs are out
-    if (e == cudaSuccess) e = cudaStreamWaitEvent(st, hcall.in[sl], 0);
-    if (e == cudaSuccess && c >= kSlots) e = cudaStreamWaitEvent(st, hcall.out[sl], 0);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(cs, hcall.in[sl], 0);
+    if (e == cudaSuccess && c >= kSlots) e = cudaStreamWaitEvent(cs, hcall.out[sl], 0);
     if (e != cudaSuccess) return FBOB_ERR_CUDA;
-    fbob_shape cs = *s;
-    cs.B = 1;
-    cs.H = nq;
-    cs.H_kv = s->H_kv > 0 ? nkv : 0;
-    rc = run_pass1(&cs, w[0], w[1], w[2], w[3], static_cast<const float*>(w[4]), w[5], w[6],
-                   w[7], w[8], w[9], w[12], static_cast<float*>(w[13]), st, f0);
+    fbob_shape csh = *s;
+    csh.B = 1;
+    csh.H = nq;
+    csh.H_kv = s->H_kv > 0 ? nkv : 0;
+    rc = run_pass1(&csh, w[0], w[1], w[2], w[3], static_cast<const float*>(w[4]), w[5], w[6],
+                   w[7], w[8], w[9], w[12], static_cast<float*>(w[13]), cs, f0);
     if (rc == FBOB_OK)
-      rc = run_pass2(&cs, w[0], w[1], w[2], static_cast<const float*>(w[4]), w[5], w[6], w[7],
-                     w[8], static_cast<const float*>(w[13]), w[10], w[11], st, f0);
+      rc = run_pass2(&csh, w[0], w[1], w[2], static_cast<const float*>(w[4]), w[5], w[6], w[7],
+                     w[8], static_cast<const float*>(w[13]), w[10], w[11], cs, f0);
     if (rc != FBOB_OK) return rc;
-    launches += pass1_launches(&cs) + 1;
+    launches += pass1_launches(&csh) + 1;
     // copy out once computed
-    e = cudaEventRecord(hcall.comp[sl], st);
+    e = cudaEventRecord(hcall.comp[sl], cs);
     if (e == cudaSuccess) e = cudaStreamWaitEvent(hcall.cout, hcall.comp[sl], 0);
     if (e == cudaSuccess) e = d2h(hbm(q_bar, f0 * nd), w[9], nq * nd);
     if (e == cudaSuccess) e = d2h(hbm(dout_bar, f0 * nd), w[12], nq * nd);
