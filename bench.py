@@ -169,6 +169,19 @@ def oracle_sample(w, bits_head, target_s, seed=0):
     return flops, dt, f"{len(rows)} evenly spaced query rows of head 0 (of {w.N}), all key columns"
 
 
+def job_rate(ms_local, world, flops_per_rank_step, steps, device="cuda"):
+    """Whole-job rate over `world` replicas: the slowest rank's elapsed time
+    (max over ranks; every rank gets it) and the units all ranks processed
+    divided by that time.  Returns (TFLOP/s, max ms)."""
+    import torch
+    t = torch.tensor([float(ms_local)], dtype=torch.float64, device=device)
+    if world > 1:
+        import torch.distributed as dist
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    ms_max = float(t.item())
+    return world * flops_per_rank_step * steps / (ms_max * 1e-3) / 1e12, ms_max
+
+
 def cores():
     return len(os.sched_getaffinity(0))
 
@@ -291,12 +304,8 @@ def run_gpu(args, w):
     ms = start.elapsed_time(stop)
     part_ms = {name: sum(e[j].elapsed_time(e[j + 1]) for e in ev) / K
                for j, (name, _) in enumerate(parts)}
-    ms_t = torch.tensor([ms], device="cuda")
-    if world > 1:
-        dist.all_reduce(ms_t, op=dist.ReduceOp.MAX)
-    ms_max = float(ms_t.item())
     flops = bob_flops(w)
-    value = world * flops * K / (ms_max * 1e-3) / 1e12
+    value, ms_max = job_rate(ms, world, flops, K)
 
     # ---- end to end through the public host-buffer call: every step copies
     # its inputs in from pinned host memory and its results out, pipelined
@@ -324,11 +333,7 @@ def run_gpu(args, w):
         e2e_step()
     ee.record(stream)
     barrier()
-    e2e_ms = es.elapsed_time(ee)
-    e_t = torch.tensor([e2e_ms], device="cuda")
-    if world > 1:
-        dist.all_reduce(e_t, op=dist.ReduceOp.MAX)
-    e2e_val = world * flops * K / (float(e_t.item()) * 1e-3) / 1e12
+    e2e_val, e2e_ms_max = job_rate(es.elapsed_time(ee), world, flops, K)
 
     if rank != 0:
         if world > 1:
@@ -373,7 +378,7 @@ def run_gpu(args, w):
         "roofline": roofline,
         "cpu_baseline": cpu,
         "e2e": {"value": e2e_val, "unit": "TFLOP/s", "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": d2h, "ms_per_step": float(e_t.item()) / K,
+                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms_max / K,
                 "call": "fbob_attn_bob_host (pinned host buffers, copies pipelined over head chunks)",
                 "workspace_bytes": ws_bytes},
         "gpu_launches": launches_per_step * K,
