@@ -63,8 +63,13 @@
  *  Stream     Every call enqueues its kernels on `stream` (NULL = legacy
  *             default stream) and returns without synchronising.
  *  Memory     The library allocates and frees no device memory.  The caller
- *             owns every buffer.  Library state is one device-side error word
- *             per device plus cached driver entry points.
+ *             owns every buffer (fbob_attn_bob_host's device workspace
+ *             included).  Library state is one device-side error word per
+ *             device, cached driver entry points, and the fixed 64 MiB staging
+ *             array of fbob_attn_bob_host_noalloc, placed on a device by that
+ *             call's first use there.  fbob_attn_bob_host creates three streams
+ *             and seven events per call and releases them when their work is
+ *             done; no other call creates any CUDA object.
  *  Errors     Host-side validation failures return immediately, before any
  *             CUDA call, and launch nothing.  A failed launch returns
  *             FBOB_ERR_CUDA.  Kernels never trap: every device-side wait is
