@@ -256,6 +256,13 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_engine(const __grid_constant_
     const int nq = act[q] ? tq1[q] - tq0[q] + 1 : 0;
     for (int k = 0; ok && k < nq; ++k) {
       const int jt = (tq0[q] + k) * BN2;
+      // dropout keep bits of the tile's 8 x 16 keys, formed while S_q(T) is computed
+      uint32_t kb[8];
+      if constexpr (DROP) {
+#pragma unroll
+        for (int c = 0; c < 8; ++c)
+          kb[c] = keep_row16(gi, jt + 16 * c, (uint32_t)(p.head0 + bh), dkey);
+      }
       if (!ew_wait(&m->s_full[q], k & 1)) {
         ok = false;
         break;
@@ -310,9 +317,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_engine(const __grid_constant_
 #pragma unroll
       for (int c = 0; c < 8; ++c) {
         uint32_t oP[8];
-        // dropout keep bits of keys jt + 16c .. + 15 (the whole warp shuffles)
-        const uint32_t kbc =
-            DROP ? keep_row16(gi, jt + 16 * c, (uint32_t)(p.head0 + bh), dkey) : 0u;
+        const uint32_t kbc = DROP ? kb[c] : 0u;
 #pragma unroll
         for (int e = 0; e < 16; e += 2) {
           float p0 = ex2(fmaf(bits_f(rS[c][e]), sl2, nm));
