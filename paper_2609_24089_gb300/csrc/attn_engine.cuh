@@ -67,7 +67,6 @@ namespace fbob {
 
 constexpr uint32_t kColSF = 256;   // stage-A area of issuer X
 constexpr uint32_t kColDC = 384;   // stage-A area of issuer Y
-constexpr uint32_t kColDC1 = 128;  // second DC buffer (column engine, d = 64)
 // row statistics kernel: Q and U_Q as MMA A operands in TMEM (bf16 pairs per
 // column, D/2 columns each) at kColQT and kColQT + D/2; second SF buffer
 constexpr uint32_t kColQT = 0;
@@ -958,7 +957,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
   // under the causal mask
   // DC buffer of tile t, and the phase parity of its per-buffer barriers
   auto dc_sel = [](int t) -> int { return C::DC2 ? (t & 1) : 0; };
-  auto dc_col = [](int t) -> uint32_t { return (C::DC2 && (t & 1)) ? kColDC1 : kColDC; };
+  auto dc_col = [](int t) -> uint32_t { return (C::DC2 && (t & 1)) ? C::DC1_COL : kColDC; };
   auto dc_par = [](int t) -> uint32_t { return C::DC2 ? ((t >> 1) & 1) : (t & 1); };
   const int N = p.N;
   const int lin = blockIdx.x;

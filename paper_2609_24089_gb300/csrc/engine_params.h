@@ -107,8 +107,11 @@ struct ColCfg {
   static constexpr int STAGE_BYTES = TILE_BYTES + 1024;  // + row vectors
   static constexpr int NSTAGES = (OP == ColOp::BobPass2 && D == 128) ? 2 : (D == 64 ? 4 : 3);
   // two DC buffers in TMEM (DC(t+1) is issued before stage B(t)): possible
-  // when the accumulators (2 D columns) leave columns 128..255 free
-  static constexpr bool DC2 = D == 64;
+  // when the accumulators (2 D columns) leave columns 128..255 free, or, in
+  // the first backward, whose DC tile (dP^T) takes 64 of the DC area's 128
+  // columns, in the DC area's second half
+  static constexpr bool DC2 = D == 64 || OP == ColOp::BwdDKDV;
+  static constexpr uint32_t DC1_COL = D == 64 ? 128u : 448u;  // second DC buffer
   // issuer X takes the value-accumulator MMAs of stage B.  With one DC buffer
   // issuer Y would have to wait for them before the next DC (measured slower);
   // with two that wait is two tiles back and off the critical path.
