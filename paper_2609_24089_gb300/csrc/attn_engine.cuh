@@ -397,7 +397,8 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
               mma_ts(tmem + D, A + 8, md(2, 0), id_b, 1);
             }
           } else if constexpr (OP == RowOp::BwdDQ) {
-            mma_ts(tmem + 0, tmem + kColDC + 16 * s, md(0, 0), id_b, first);  // dQ += dS K
+            const uint32_t dcb = C::DC2 ? 64u * (uint32_t)(st & 1) : 0u;  // dP buffer of tile st
+            mma_ts(tmem + 0, tmem + kColDC + dcb + 16 * s, md(0, 0), id_b, first);  // dQ += dS K
           }
         }
       };
@@ -499,7 +500,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         if (*abort_flag) drain_wait(&m->bar_acc, 0);
       } else {
         // ---------------- issuer Y: DC(t) and the remaining stage-B MMAs
-        auto stage_dc = [&](uint32_t sb, int h) {
+        auto stage_dc = [&](uint32_t sb, int h, uint32_t dcb = 0) {
           const uint64_t kd0 = sdesc_sw128(sb, 16, 1024);
           if constexpr (kStats) {  // whole tile: [dP_0|C_0|dP_1|C_1] = dO [V_0;U_V_0;V_1;U_V_1]^T
 #pragma unroll
@@ -512,7 +513,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
           } else if constexpr (OP == RowOp::BwdDQ) {  // dP = dO V^T (whole tile)
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)
-              mma_ss(tmem + kColDC, sd(1, k), kd(kd0, 1, 0, k), id_n64, k > 0);
+              mma_ss(tmem + kColDC + dcb, sd(1, k), kd(kd0, 1, 0, k), id_n64, k > 0);
           }
         };
         // issuer Y reads every streamed tensor: wait for both halves of a stage
@@ -540,6 +541,42 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
             mma_commit(&m->bar_empty[ns]);
           }
           ok = false;  // no stage B
+        }
+        if constexpr (C::DC2) {
+          // dP(t) in buffer t & 1 (columns kColDC + 64 (t & 1)), two tiles
+          // ahead: dP(t+2) goes into the buffer stage B(t) has just read
+          for (int t = 0; ok && t < 2 && t < nsteps; ++t) {
+            if (t == 1) ok = wait_stage(1 % C::NSTAGES, (1 / C::NSTAGES) & 1);
+            if (!ok) break;
+            tc_fence_after();
+            stage_dc(smem_u32(s_stream + (t % C::NSTAGES) * C::STAGE_BYTES), 0, 64u * t);
+            mma_commit(&m->bar_sa_dc[t]);
+          }
+          for (int st = 0; ok && st < nsteps; ++st) {
+            const int b = st & 1;
+            const uint32_t par = (st >> 1) & 1;
+            const int stage = st % C::NSTAGES;
+            const uint32_t sb = smem_u32(s_stream + stage * C::STAGE_BYTES);
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              if (!mbar_wait(&m->bar_ew[2 * b + h], par, wctl)) {
+                ok = false;
+                break;
+              }
+              tc_fence_after();
+              stage_b(sb, h, st, 2);
+            }
+            if (!ok) break;
+            mma_commit(&m->bar_empty[stage]);
+            const int nx = st + 2;
+            if (nx < nsteps) {
+              if (!wait_stage(nx % C::NSTAGES, (nx / C::NSTAGES) & 1)) break;
+              tc_fence_after();
+              stage_dc(smem_u32(s_stream + (nx % C::NSTAGES) * C::STAGE_BYTES), 0, 64u * b);
+              mma_commit(&m->bar_sa_dc[b]);
+            }
+          }
+          ok = false;
         }
         if (ok) {
           tc_fence_after();
@@ -731,8 +768,11 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
       } else {
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
+          // (the dQ kernel alternates two dP buffers: buffer st & 1, phase st >> 1)
+          const int dcbi = C::DC2 ? (st & 1) : 0;
           if (kDcHalves || h == 0) {
-            if (!ew_wait(&m->bar_sa_dc[kDcHalves ? h : 0], st & 1)) {
+            if (!ew_wait(&m->bar_sa_dc[kDcHalves ? h : dcbi],
+                         C::DC2 ? ((st >> 1) & 1) : (st & 1))) {
               ok = false;
               break;
             }
@@ -808,7 +848,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
             tmem_st8(R + 32, oSt);
             tmem_st8(R + 40, odS);
           } else if constexpr (OP == RowOp::BwdDQ) {
-            const uint32_t R = ta + kColDC + c0;
+            const uint32_t R = ta + kColDC + 64 * dcbi + c0;
             uint32_t rdP[16];
             tmem_ld16(R, rdP);
             tmem_ld_wait(rdP);
@@ -826,7 +866,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
           }
           tmem_st_wait();
           tc_fence_before();
-          mbar_arrive(&m->bar_ew[h]);
+          mbar_arrive(&m->bar_ew[C::DC2 ? 2 * dcbi + h : h]);
         }
       }
     }

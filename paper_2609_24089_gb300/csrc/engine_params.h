@@ -92,6 +92,9 @@ struct RowCfg {
   // the direct form at d = 128 (dOtil on X) Y's wait for X's share before
   // each DC cost 5 % more than it saved.
   static constexpr bool XSHARE = OP == RowOp::BobPass1 && D == 64;
+  // the dQ kernel's DC tile (dP, 64 columns) leaves the other half of the DC
+  // area free: two dP buffers, dP(t+2) issued right after stage B(t)
+  static constexpr bool DC2 = OP == RowOp::BwdDQ;
   static constexpr int MISC_BYTES = 2304;
   static constexpr int SMEM_BYTES = STAT_BYTES + NSTAGES * STAGE_BYTES + MISC_BYTES;
 };
