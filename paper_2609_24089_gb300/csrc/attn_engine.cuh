@@ -210,7 +210,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
   constexpr bool kStats = OP == RowOp::BobStats;    // row scalars alpha, E, D only
   constexpr bool kDirect = OP == RowOp::BobPass1D;  // Pass 1 with alpha, E given
   constexpr bool kB4 = row_bob(OP);                 // streamed K, U_K, V, U_V
-  constexpr bool kDcHalves = kBob || kDirect;       // DC issued per 32-column half
+  constexpr bool kDcHalves = C::DC_HALVES;           // DC issued per 32-column half
   extern __shared__ __align__(1024) uint8_t smem[];
   uint8_t* s_stat = smem;
   uint8_t* s_stream = smem + C::STAT_BYTES;
@@ -506,10 +506,14 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)  // (dO is the one stationary tile in shared memory)
               mma_ss(tmem + kColDC, sd(0, k), kd(kd0, 2, 0, k), id_n128, k > 0);
-          } else if constexpr (kB4) {  // [dP_h | C_h] = dO [V_h ; U_V_h]^T
+          } else if constexpr (kB4 && kDcHalves) {  // [dP_h | C_h] = dO [V_h ; U_V_h]^T
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)
               mma_ss(tmem + kColDC + 64 * h, sd(2, k), kd(kd0, 2, h, k), id_n64, k > 0);
+          } else if constexpr (kB4) {  // whole tile: [dP_0|C_0|dP_1|C_1] = dO [V_0;U_V_0;V_1;U_V_1]^T
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k)
+              mma_ss(tmem + kColDC, sd(2, k), kd(kd0, 2, 0, k), id_n128, k > 0);
           } else if constexpr (OP == RowOp::BwdDQ) {  // dP = dO V^T (whole tile)
 #pragma unroll
             for (int k = 0; k < D / 16; ++k)

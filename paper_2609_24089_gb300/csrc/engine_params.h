@@ -92,6 +92,12 @@ struct RowCfg {
   // the direct form at d = 128 (dOtil on X) Y's wait for X's share before
   // each DC cost 5 % more than it saved.
   static constexpr bool XSHARE = OP == RowOp::BobPass1 && D == 64;
+  // Pass 1's DC ([dP | C]) issued per 32-key half, so that stage B of half 0
+  // overlaps the elementwise work on half 1; otherwise one N = 128 MMA per
+  // K-step for the whole tile.  Measured for the direct form at d = 128:
+  // whole-tile DC is 5 % faster (16 N = 64 MMAs per tile cost issuer Y more
+  // than the overlap saved).
+  static constexpr bool DC_HALVES = OP == RowOp::BobPass1;
   // the dQ kernel's DC tile (dP, 64 columns) leaves the other half of the DC
   // area free: two dP buffers, dP(t+2) issued right after stage B(t)
   static constexpr bool DC2 = OP == RowOp::BwdDQ;
