@@ -32,7 +32,7 @@
 //   X  issues SF(t+1) as soon as the elementwise warps have copied SF(t)
 //      into registers, so the next tile's largest stage-A contractions run
 //      while the elementwise warps still work on tile t.
-//   Y  issues DC(t) (per 32-column half in Pass 1).
+//   Y  issues DC(t) (per 32-column half in the one-sweep Pass 1).
 //   elementwise: copy SF to registers and release it; then per half read DC,
 //      compute, and write the bf16 operand tiles of stage B over the DC
 //      columns just read; stage B of half 0 overlaps the elementwise work on
