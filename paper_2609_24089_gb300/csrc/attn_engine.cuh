@@ -26,13 +26,16 @@
 //
 // Tensor memory (512 columns): accumulators at 0..255; stage-A area "SF" at
 // 256..383 (scores, and F in the BoB passes), owned by issuer X; stage-A area
-// "DC" at 384..511 (dP, and C in the BoB passes), owned by issuer Y.
+// "DC" at 384..511 (dP, and C in the BoB passes), owned by issuer Y.  Where
+// the DC tile leaves room (the column engine at d = 64, both first-backward
+// kernels) DC is double-buffered and issued two tiles ahead.
 //
 // Per streamed tile t:
 //   X  issues SF(t+1) as soon as the elementwise warps have copied SF(t)
 //      into registers, so the next tile's largest stage-A contractions run
 //      while the elementwise warps still work on tile t.
-//   Y  issues DC(t) (per 32-column half in the one-sweep Pass 1).
+//   Y  issues DC(t) (per 32-column half in the one-sweep Pass 1, for the
+//      whole tile otherwise).
 //   elementwise: copy SF to registers and release it; then per half read DC,
 //      compute, and write the bf16 operand tiles of stage B over the DC
 //      columns just read; stage B of half 0 overlaps the elementwise work on

@@ -13,7 +13,7 @@
 // X issues S_q(T+1) once O_q += P_q(T) V(T) has completed (it overwrites
 // P_q(T)).  The two query tiles' chains interleave, so the tensor pipe works
 // on one tile while the other's softmax runs.  The running maximum is raised
-// lazily (by more than kFwdSlack2, so P <= 2^kFwdSlack2); O_q is then
+// lazily (by more than kFwdSlack, so P <= 2^kFwdSlack); O_q is then
 // rescaled by its warpgroup after the MMAs into it have completed.
 //
 // Roles (352 threads): warps 0-3 softmax of query tile 0, warps 4-7 of tile
@@ -27,7 +27,7 @@ namespace fbob {
 
 constexpr int kFwdRows = 2 * BM;  // query rows per CTA
 constexpr int BN2 = 128;          // keys per streamed tile
-constexpr float kFwdSlack2 = 8.f;
+constexpr float kFwdSlack = 8.f;
 
 template <int D>
 struct FwdCfg {
@@ -283,7 +283,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_engine(const __grid_constant_
         for (int e = 0; e < 16; ++e) mraw = fmaxf(mraw, bits_f(rS[c][e]));
       }
       const float mt = mraw * sl2;
-      const bool raise = mt > mrow + kFwdSlack2;  // also the first tile with a valid key
+      const bool raise = mt > mrow + kFwdSlack;  // also the first tile with a valid key
       const bool rescale = raise && mrow != -INFINITY;
       if (__any_sync(0xffffffffu, rescale)) {
         // every MMA into O_q so far (tiles before k) must have completed
