@@ -328,11 +328,12 @@ def run_gpu(args, w):
         e2e_step()
     barrier()
     es, ee = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    es.record(stream)
-    for _ in range(K):
-        e2e_step()
-    ee.record(stream)
-    barrier()
+    with ClockSampler(local) as e2e_clk:  # clocks of the e2e loop as well
+        es.record(stream)
+        for _ in range(K):
+            e2e_step()
+        ee.record(stream)
+        barrier()
     e2e_val, e2e_ms_max = job_rate(es.elapsed_time(ee), world, flops, K)
 
     if rank != 0:
@@ -380,7 +381,7 @@ def run_gpu(args, w):
         "e2e": {"value": e2e_val, "unit": "TFLOP/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms_max / K,
                 "call": "fbob_attn_bob_host (pinned host buffers, copies pipelined over head chunks)",
-                "workspace_bytes": ws_bytes},
+                "workspace_bytes": ws_bytes, "clocks": e2e_clk.summary()},
         "gpu_launches": launches_per_step * K,
         "clocks": clk.summary(),
         "peak_hbm_bytes": footprint,
