@@ -12,6 +12,11 @@ launch configuration the benchmark times.
   n16k_d128_causal_swa4k sliding window w = N/4: oracle on sampled rows and on a
                          256-key block, complete once the rows whose band holds
                          it (keys j .. j + 4095) are summed
+  n16k_d128_causal_varlen / _gqa4 / _drop10
+                         packed sequences, grouped-query heads, dropout: sampled
+                         rows plus one whole sequence or the causal tail
+  n4k_d{32,64,128}_causal_b4h12
+                         the head-dimension sweep's shape: two full heads each
 """
 import os
 
@@ -226,9 +231,10 @@ def test_n16k_d128_causal_drop10_rows_and_tail():
         G.check("vbar[tail]", G.flat(r["vbar"], hh, w.H)[t0:], ref["vbar"])
 
 
-def test_n4k_d32_causal_b4h12_two_heads():
-    """Head dim 32 at the head-dimension sweep's shape: two full heads."""
-    w = synth.WORKLOADS["n4k_d32_causal_b4h12"]
+@pytest.mark.parametrize("d", [32, 64, 128])
+def test_n4k_causal_b4h12_head_dim_sweep_two_heads(d):
+    """The head-dimension sweep's shape (B 4, H 12, N 4096, causal): two full heads."""
+    w = synth.WORKLOADS[f"n4k_d{d}_causal_b4h12"]
     bits = synth.workload_inputs(w)
     r = G.run_bob(bits, w.scale, w.causal)
     assert r["status"] == 0
