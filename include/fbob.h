@@ -235,7 +235,10 @@ int fbob_attn_bob_pass1_direct(const fbob_shape* shape, const void* q, const voi
  * Stream: the copies start after the work already enqueued on `stream`, and
  *      `stream` completes only after the last copy out; synchronise it before
  *      reading the outputs.  Three streams and seven events are created per
- *      call and released when their work completes.
+ *      call and released when their work completes.  If the call returns an
+ *      error after validation (a failed CUDA call), copies and kernels it has
+ *      already enqueued may still be running on its own streams: synchronise
+ *      the device before reusing the buffers or the workspace.
  */
 int fbob_attn_bob_host(const fbob_shape* shape, const void* q, const void* k, const void* v,
                        const void* o, const float* lse, const void* dout,
