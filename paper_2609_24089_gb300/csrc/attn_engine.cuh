@@ -209,6 +209,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
   using C = RowCfg<OP, D>;
   static_assert(DG == D || (DG == 32 && D == 64), "global head dim 32 runs in 64-wide tiles");
   static_assert(!DROP || OP != RowOp::BobPass1, "dropout Pass 1 runs as statistics + direct");
+  static_assert(C::NSTAGES >= 2 && C::NSTAGES <= 4, "the stage barriers hold four stages");
   constexpr bool kBob = OP == RowOp::BobPass1;      // Pass 1, one sweep (Prop. 3.1)
   constexpr bool kStats = OP == RowOp::BobStats;    // row scalars alpha, E, D only
   constexpr bool kDirect = OP == RowOp::BobPass1D;  // Pass 1 with alpha, E given
@@ -988,6 +989,7 @@ template <ColOp OP, int D, bool DROP, int DG>
 __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant__ EngineParams p) {
   using C = ColCfg<OP, D>;
   static_assert(DG == D || (DG == 32 && D == 64), "global head dim 32 runs in 64-wide tiles");
+  static_assert(C::NSTAGES >= 2 && C::NSTAGES <= 4, "the stage barriers hold four stages");
   constexpr bool kBob = OP == ColOp::BobPass2;
   extern __shared__ __align__(1024) uint8_t smem[];
   uint8_t* s_stat = smem;

@@ -60,6 +60,7 @@ template <int D, bool DROP, int DG>
 __global__ void __launch_bounds__(kThreads, 1) fwd_engine(const __grid_constant__ EngineParams p) {
   using C = FwdCfg<D>;
   static_assert(DG == D || (DG == 32 && D == 64), "global head dim 32 runs in 64-wide tiles");
+  static_assert(C::NSTAGES >= 2 && C::NSTAGES <= 4, "the stage barriers hold four stages");
   extern __shared__ __align__(1024) uint8_t smem[];
   uint8_t* s_stat = smem;
   uint8_t* s_stream = smem + C::STAT_BYTES;
