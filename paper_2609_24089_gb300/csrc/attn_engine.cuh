@@ -78,9 +78,9 @@ constexpr uint32_t kColSF1 = 128;
 // Shared-memory bookkeeping block (in the MISC area).
 struct Misc {
   uint64_t bar_stat;
-  uint64_t bar_full[4];    // first part of a stream stage landed (all issuer X reads)
-  uint64_t bar_full_b[4];  // rest of the stage (and, column engine, the row vectors)
-  uint64_t bar_empty[4];
+  uint64_t bar_full[kMaxStages];    // first part of a stream stage landed (all issuer X reads)
+  uint64_t bar_full_b[kMaxStages];  // rest of the stage (and, column engine, the row vectors)
+  uint64_t bar_empty[kMaxStages];
   uint64_t bar_sa_sf[2];   // X's stage A of a tile completed (per SF buffer)
   uint64_t bar_sf_free[2]; // elementwise warps copied SF to registers (per SF buffer)
   uint64_t bar_dc_free; // elementwise warps copied DC to registers (row statistics kernel)
@@ -209,7 +209,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
   using C = RowCfg<OP, D>;
   static_assert(DG == D || (DG == 32 && D == 64), "global head dim 32 runs in 64-wide tiles");
   static_assert(!DROP || OP != RowOp::BobPass1, "dropout Pass 1 runs as statistics + direct");
-  static_assert(C::NSTAGES >= 2 && C::NSTAGES <= 4, "the stage barriers hold four stages");
+  static_assert(C::NSTAGES >= 2 && C::NSTAGES <= kMaxStages, "the stage barriers hold kMaxStages stages");
   constexpr bool kBob = OP == RowOp::BobPass1;      // Pass 1, one sweep (Prop. 3.1)
   constexpr bool kStats = OP == RowOp::BobStats;    // row scalars alpha, E, D only
   constexpr bool kDirect = OP == RowOp::BobPass1D;  // Pass 1 with alpha, E given
@@ -300,7 +300,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         for (int b = 0; b < C::KB; ++b)
           tma_load_3d(s_stat + ((C::STAT_TMEM ? 0 : t) * C::KB + b) * (BM * 128), &p.tm[t],
                       &m->bar_stat, 64 * b, i0, bh);
-      int issued[4] = {-1, -1, -1, -1};
+      int issued[kMaxStages] = {-1, -1, -1, -1};
       for (int st = 0; st < nsteps; ++st) {
         const int stage = st % C::NSTAGES;
         if (st >= C::NSTAGES) {
@@ -989,7 +989,7 @@ template <ColOp OP, int D, bool DROP, int DG>
 __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant__ EngineParams p) {
   using C = ColCfg<OP, D>;
   static_assert(DG == D || (DG == 32 && D == 64), "global head dim 32 runs in 64-wide tiles");
-  static_assert(C::NSTAGES >= 2 && C::NSTAGES <= 4, "the stage barriers hold four stages");
+  static_assert(C::NSTAGES >= 2 && C::NSTAGES <= kMaxStages, "the stage barriers hold kMaxStages stages");
   constexpr bool kBob = OP == ColOp::BobPass2;
   extern __shared__ __align__(1024) uint8_t smem[];
   uint8_t* s_stat = smem;
@@ -1075,7 +1075,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
           tma_load_3d(s_stat + (t * C::KB + b) * (BM * 128), &p.tm[t], &m->bar_stat, 64 * b, j0,
                       bh);
     }
-    int issued[4] = {-1, -1, -1, -1};
+    int issued[kMaxStages] = {-1, -1, -1, -1};
     for (int st = 0; st < nprod; ++st) {
       const int stage = st % C::NSTAGES;
       if (st >= C::NSTAGES) {

@@ -20,6 +20,7 @@ constexpr int kProducerWarp = 8;
 constexpr int kMmaWarp = 9;   // MMA issuer X (and TMEM allocator)
 constexpr int kMmaWarpY = 10; // MMA issuer Y
 constexpr int kEwThreads = 256;
+constexpr int kMaxStages = 4;  // stream stages the barrier arrays hold
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kColA = 256;  // stage-A region of half h starts at kColA + 128 h
 constexpr float kLog2e = 1.4426950408889634f;

@@ -41,8 +41,8 @@ struct FwdCfg {
 
 struct FwdMisc {
   uint64_t bar_stat;
-  uint64_t full[4];
-  uint64_t empty[4];
+  uint64_t full[kMaxStages];
+  uint64_t empty[kMaxStages];
   uint64_t s_full[2];  // S_q(T) computed (issuer X)
   uint64_t p_full[2];  // P_q(T) written (128 softmax threads)
   uint64_t o_done[2];  // O_q += P_q(T) V(T) completed (issuer Y)
@@ -60,7 +60,7 @@ template <int D, bool DROP, int DG>
 __global__ void __launch_bounds__(kThreads, 1) fwd_engine(const __grid_constant__ EngineParams p) {
   using C = FwdCfg<D>;
   static_assert(DG == D || (DG == 32 && D == 64), "global head dim 32 runs in 64-wide tiles");
-  static_assert(C::NSTAGES >= 2 && C::NSTAGES <= 4, "the stage barriers hold four stages");
+  static_assert(C::NSTAGES >= 2 && C::NSTAGES <= kMaxStages, "the stage barriers hold kMaxStages stages");
   extern __shared__ __align__(1024) uint8_t smem[];
   uint8_t* s_stat = smem;
   uint8_t* s_stream = smem + C::STAT_BYTES;
@@ -143,7 +143,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_engine(const __grid_constant_
         for (int b = 0; b < C::KB; ++b)
           tma_load_3d(s_stat + (q * C::KB + b) * (BM * 128), &p.tm[0], &m->bar_stat, 64 * b,
                       i0 + BM * q, bh);
-      int issued[4] = {-1, -1, -1, -1};
+      int issued[kMaxStages] = {-1, -1, -1, -1};
       for (int st = 0; st < nsteps; ++st) {
         const int stage = st % C::NSTAGES;
         if (st >= C::NSTAGES &&
