@@ -4,21 +4,26 @@
 // A CTA owns 2 x 128 query rows of one head (query tiles 0 and 1) and streams
 // 128-key tiles of K and V through a ring of stream stages.  Each query tile
 // has its own score buffer S_q (128 TMEM columns) and accumulator O_q, and
-// its own softmax warpgroup, whose thread i holds query row i whole.  Per key
-// tile T and query tile q:
+// two softmax warpgroups, one per half of the key tile (64 keys each), whose
+// thread i holds query row i.  Per key tile T and query tile q:
 //   X   S_q(T) = Q_q K(T)^T                 (N = 128, issuer X)
-//   WGq m, l (online softmax), P = 2^(S tau log2 e - m) written as bf16 over
-//       the first 64 columns of S_q (all of S_q is in registers by then)
+//   WGs m, l (online softmax): each half's row maxima are exchanged through
+//       shared memory, so both halves take the same running maximum; then
+//       P = 2^(S tau log2 e - m) is written as bf16 over the first 64
+//       columns of S_q (both halves hold their S in registers by then)
 //   Y   O_q += P_q(T) V(T)                  (A from TMEM, issuer Y)
 // X issues S_q(T+1) once O_q += P_q(T) V(T) has completed (it overwrites
 // P_q(T)).  The two query tiles' chains interleave, so the tensor pipe works
 // on one tile while the other's softmax runs.  The running maximum is raised
 // lazily (by more than kFwdSlack, so P <= 2^kFwdSlack); O_q is then
-// rescaled by its warpgroup after the MMAs into it have completed.
+// rescaled by the first half's warpgroup after the MMAs into it have
+// completed.  Each half keeps the row sum of its own keys; the epilogue adds
+// the two.
 //
-// Roles (352 threads): warps 0-3 softmax of query tile 0, warps 4-7 of tile
-// 1 (warp w reads TMEM lanes 32 (w % 4) .. +31), warp 8 TMA producer,
-// warp 9 issuer X, warp 10 issuer Y.  Every wait is bounded.
+// Roles (608 threads): warps 0-7 softmax of query tile 0 (keys 0-63, then
+// 64-127), warps 8-15 of tile 1 (warp w reads TMEM lanes 32 (w % 4) .. +31),
+// warp 16 TMA producer, warp 17 issuer X, warp 18 issuer Y.  Every wait is
+// bounded.
 #pragma once
 
 #include "attn_engine.cuh"
@@ -28,6 +33,10 @@ namespace fbob {
 constexpr int kFwdRows = 2 * BM;  // query rows per CTA
 constexpr int BN2 = 128;          // keys per streamed tile
 constexpr float kFwdSlack = 8.f;
+// warps 0-15: softmax, four warpgroups (query tile q = g / 2, key half g % 2);
+// then the TMA producer and the two MMA issuers
+constexpr int kFwdProducer = 16, kFwdX = 17, kFwdY = 18;
+constexpr int kFwdThreads = 19 * 32;
 
 template <int D>
 struct FwdCfg {
@@ -35,7 +44,9 @@ struct FwdCfg {
   static constexpr int STAT_BYTES = 2 * KB * BM * 128;     // Q_0, Q_1
   static constexpr int STAGE_BYTES = 2 * KB * BN2 * 128;   // K, V
   static constexpr int NSTAGES = D == 64 ? 4 : 2;
-  static constexpr int MISC_BYTES = 256;
+  // bookkeeping, then the row-maximum exchange [tile parity][q][half][row]
+  // and the row-sum exchange [q][half][row]
+  static constexpr int MISC_BYTES = 256 + 8 * BM * 4 + 4 * BM * 4;
   static constexpr int SMEM_BYTES = STAT_BYTES + NSTAGES * STAGE_BYTES + MISC_BYTES;
 };
 
@@ -46,6 +57,8 @@ struct FwdMisc {
   uint64_t s_full[2];  // S_q(T) computed (issuer X)
   uint64_t p_full[2];  // P_q(T) written (128 softmax threads)
   uint64_t o_done[2];  // O_q += P_q(T) V(T) completed (issuer Y)
+  uint64_t xq[2][2];   // [q][tile parity]: both halves posted their row maxima
+  uint64_t xl[2];      // [q]: both halves posted their row sums (epilogue)
   uint64_t bar_acc;    // every MMA of both issuers completed (abort drain)
   uint32_t tmem_base;
   uint32_t pad;
@@ -57,7 +70,7 @@ static_assert(sizeof(FwdMisc) <= 256, "FwdMisc must fit the MISC area");
 constexpr uint32_t kColS2 = 256;
 
 template <int D, bool DROP, int DG>
-__global__ void __launch_bounds__(kThreads, 1) fwd_engine(const __grid_constant__ EngineParams p) {
+__global__ void __launch_bounds__(kFwdThreads, 1) fwd_engine(const __grid_constant__ EngineParams p) {
   using C = FwdCfg<D>;
   static_assert(DG == D || (DG == 32 && D == 64), "global head dim 32 runs in 64-wide tiles");
   static_assert(C::NSTAGES >= 2 && C::NSTAGES <= kMaxStages, "the stage barriers hold kMaxStages stages");
@@ -65,6 +78,8 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_engine(const __grid_constant_
   uint8_t* s_stat = smem;
   uint8_t* s_stream = smem + C::STAT_BYTES;
   FwdMisc* m = reinterpret_cast<FwdMisc*>(s_stream + C::NSTAGES * C::STAGE_BYTES);
+  float* s_xm = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(m) + 256);  // 8 x BM
+  float* s_xl = s_xm + 8 * BM;                                                  // 4 x BM
 
   const int tid = threadIdx.x;
   const int warp = tid >> 5;
@@ -117,13 +132,16 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_engine(const __grid_constant_
     }
     for (int q = 0; q < 2; ++q) {
       mbar_init(&m->s_full[q], 1);
-      mbar_init(&m->p_full[q], BM);
+      mbar_init(&m->p_full[q], 2 * BM);  // both key halves
       mbar_init(&m->o_done[q], 1);
+      mbar_init(&m->xq[q][0], 2 * BM);
+      mbar_init(&m->xq[q][1], 2 * BM);
+      mbar_init(&m->xl[q], 2 * BM);
     }
     mbar_init(&m->bar_acc, 2);
     fence_mbar_init();
   }
-  if (warp == kMmaWarp) {
+  if (warp == kFwdX) {
     tmem_alloc(&m->tmem_base, kTmemCols);
     tmem_relinquish();
   }
@@ -134,7 +152,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_engine(const __grid_constant_
   WaitCtl* wctl = &m->wctl;
   volatile int* abort_flag = &m->wctl.abort;
 
-  if (warp == kProducerWarp) {
+  if (warp == kFwdProducer) {
     // ------------------------------------------------------------ producer
     if (elect_lane0() && !p.inject_stall) {
       for (int t = 0; t < 3; ++t) tma_prefetch_desc(&p.tm[t]);
@@ -165,13 +183,13 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_engine(const __grid_constant_
         drain_wait(&m->bar_stat, 0);
       }
     }
-  } else if (warp == kMmaWarp || warp == kMmaWarpY) {
+  } else if (warp == kFwdX || warp == kFwdY) {
     // ------------------------------------------------------------ MMA issuers
     if (elect_lane0()) {
       constexpr uint32_t id_s = idesc_bf16(128, BN2, false);
       constexpr uint32_t id_o = idesc_bf16(128, D, true);
       bool ok = true;
-      if (warp == kMmaWarp) {
+      if (warp == kFwdX) {
         // ---------------- issuer X: S_q(T) = Q_q K(T)^T
         const uint64_t qd0 = sdesc_sw128(smem_u32(s_stat), 16, 1024);
         ok = mbar_wait(&m->bar_stat, 0, wctl);
@@ -234,8 +252,11 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_engine(const __grid_constant_
     }
   } else {
     // ------------------------------------------------------------ softmax
-    const int q = warp >> 2;                     // query tile of this warpgroup
-    const int r = 32 * (warp & 3) + (tid & 31);  // row in the tile (TMEM lane)
+    // warpgroup g: query tile q = g / 2, key half hf = g % 2 (keys 64 hf ..
+    // 64 hf + 63 of each tile); thread: one row of the tile (TMEM lane)
+    const int g = warp >> 2;
+    const int q = g >> 1, hf = g & 1;
+    const int r = 32 * (warp & 3) + (tid & 31);
     const int gi = i0 + BM * q + r;
     const bool row_ok = gi < N;
     int jlo = 0, jhi = 0;  // this row's valid keys [jlo, jhi)
@@ -252,16 +273,16 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_engine(const __grid_constant_
       const bool w = mbar_wait(bar, par, wctl);
       return __all_sync(0xffffffffu, w);  // the warp leaves together
     };
-    float mrow = -INFINITY, lrow = 0.f;
+    float mrow = -INFINITY, lrow = 0.f;  // (lrow: this half's keys)
     bool ok = act[q];
     const int nq = act[q] ? tq1[q] - tq0[q] + 1 : 0;
     for (int k = 0; ok && k < nq; ++k) {
-      const int jt = (tq0[q] + k) * BN2;
-      // dropout keep bits of the tile's 8 x 16 keys, formed while S_q(T) is computed
-      uint32_t kb[8];
+      const int jt = (tq0[q] + k) * BN2 + 64 * hf;  // first key of this half
+      // dropout keep bits of the half's 4 x 16 keys, formed while S_q(T) is computed
+      uint32_t kb[4];
       if constexpr (DROP) {
 #pragma unroll
-        for (int c = 0; c < 8; ++c)
+        for (int c = 0; c < 4; ++c)
           kb[c] = keep_row16(gi, jt + 16 * c, (uint32_t)(p.head0 + bh), dkey);
       }
       if (!ew_wait(&m->s_full[q], k & 1)) {
@@ -269,54 +290,69 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_engine(const __grid_constant_
         break;
       }
       tc_fence_after();
-      uint32_t rS[8][16];
+      uint32_t rS[4][16];
 #pragma unroll
-      for (int c = 0; c < 8; ++c) tmem_ld16(ta + scol + 16 * c, rS[c]);
+      for (int c = 0; c < 4; ++c) tmem_ld16(ta + scol + 64 * hf + 16 * c, rS[c]);
       tmem_ld_wait(rS[0]);
 #pragma unroll
-      for (int c = 1; c < 8; ++c) reg_dep(rS[c]);
+      for (int c = 1; c < 4; ++c) reg_dep(rS[c]);
       float mraw = -INFINITY;
 #pragma unroll
-      for (int c = 0; c < 8; ++c) {
+      for (int c = 0; c < 4; ++c) {
         const int mlo = jlo - (jt + 16 * c), mhi = jhi - (jt + 16 * c);
         if (mlo > 0 || mhi < 16) mask16(rS[c], mlo, mhi);
 #pragma unroll
         for (int e = 0; e < 16; ++e) mraw = fmaxf(mraw, bits_f(rS[c][e]));
       }
+      // the row maximum over both halves: post this half's, wait for both
+      // (which also means both halves hold their S in registers, so P may be
+      // written over S), read the other's
+      float* xm = s_xm + ((k & 1) * 4 + q * 2) * BM;
+      xm[hf * BM + r] = mraw;
+      tc_fence_before();
+      mbar_arrive(&m->xq[q][k & 1]);
+      if (!ew_wait(&m->xq[q][k & 1], (k >> 1) & 1)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      mraw = fmaxf(mraw, xm[(1 - hf) * BM + r]);
       const float mt = mraw * sl2;
       const bool raise = mt > mrow + kFwdSlack;  // also the first tile with a valid key
       const bool rescale = raise && mrow != -INFINITY;
-      if (__any_sync(0xffffffffu, rescale)) {
-        // every MMA into O_q so far (tiles before k) must have completed
-        if (!ew_wait(&m->o_done[q], (k - 1) & 1)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-        const float f = rescale ? ex2(mrow - mt) : 1.f;
-#pragma unroll 1
-        for (int c = 0; c < D / 16; ++c) {
-          uint32_t o[16];
-          tmem_ld16(ta + ocol + 16 * c, o);
-          tmem_ld_wait(o);
-          uint32_t lo8[8], hi8[8];
-#pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            lo8[e] = __float_as_uint(bits_f(o[e]) * f);
-            hi8[e] = __float_as_uint(bits_f(o[8 + e]) * f);
+      if (__any_sync(0xffffffffu, rescale)) {  // (the same decision in both halves)
+        if (hf == 0) {  // half 0 rescales O_q
+          // every MMA into O_q so far (tiles before k) must have completed
+          if (!ew_wait(&m->o_done[q], (k - 1) & 1)) {
+            ok = false;
+            break;
           }
-          tmem_st8(ta + ocol + 16 * c, lo8);
-          tmem_st8(ta + ocol + 16 * c + 8, hi8);
+          tc_fence_after();
+          const float f = rescale ? ex2(mrow - mt) : 1.f;
+#pragma unroll 1
+          for (int c = 0; c < D / 16; ++c) {
+            uint32_t o[16];
+            tmem_ld16(ta + ocol + 16 * c, o);
+            tmem_ld_wait(o);
+            uint32_t lo8[8], hi8[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+              lo8[e] = __float_as_uint(bits_f(o[e]) * f);
+              hi8[e] = __float_as_uint(bits_f(o[8 + e]) * f);
+            }
+            tmem_st8(ta + ocol + 16 * c, lo8);
+            tmem_st8(ta + ocol + 16 * c + 8, hi8);
+          }
+          tmem_st_wait();
         }
-        tmem_st_wait();
-        if (rescale) lrow *= f;
+        if (rescale) lrow *= ex2(mrow - mt);
       }
       if (raise) mrow = mt;
       // no valid key yet: every score is -inf, so any finite m gives P = 0
       const float nm = mrow == -INFINITY ? 0.f : -mrow;
       float ps0 = 0.f, ps1 = 0.f;
 #pragma unroll
-      for (int c = 0; c < 8; ++c) {
+      for (int c = 0; c < 4; ++c) {
         uint32_t oP[8];
         const uint32_t kbc = DROP ? kb[c] : 0u;
 #pragma unroll
@@ -331,39 +367,47 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_engine(const __grid_constant_
           }
           oP[e / 2] = pack_bf16(p0, p1);
         }
-        // P of keys 16c .. 16c+15 over S columns 8c .. 8c+7 (already in registers)
-        tmem_st8(ta + scol + 8 * c, oP);
+        // P of keys 64 hf + 16c .. + 15 over S columns 32 hf + 8c .. + 7
+        tmem_st8(ta + scol + 32 * hf + 8 * c, oP);
       }
       lrow += ps0 + ps1;
       tmem_st_wait();
       tc_fence_before();
       mbar_arrive(&m->p_full[q]);
     }
-    // ---- epilogue: O = O_q / l (times sigma with dropout), L = m + log2 l
+    // ---- epilogue: l over both halves; O = O_q / l (times sigma with
+    // dropout), each half storing half of the columns; L = m + log2 l
     if (ok && nq > 0) ok = ew_wait(&m->o_done[q], (nq - 1) & 1);
+    if (ok) {
+      s_xl[(q * 2 + hf) * BM + r] = lrow;
+      mbar_arrive(&m->xl[q]);
+      ok = ew_wait(&m->xl[q], 0);
+    }
     if (ok && *abort_flag) ok = false;
     tc_fence_after();
     if (ok) {
-      const float inv = row_ok ? (DROP ? p.drop_sigma : 1.f) / lrow : 0.f;
+      const float lt = lrow + s_xl[(q * 2 + 1 - hf) * BM + r];
+      const float inv = row_ok ? (DROP ? p.drop_sigma : 1.f) / lt : 0.f;
       const size_t rowoff = ((size_t)bh * N + (size_t)(row_ok ? gi : 0)) * DG;
 #pragma unroll 1
-      for (int c = 0; c < D / 16; ++c) {
+      for (int c = 0; c < D / 32; ++c) {
+        const int cc = hf * (D / 2) + 16 * c;
         uint32_t o[16];
-        tmem_ld16(ta + ocol + 16 * c, o);
+        tmem_ld16(ta + ocol + cc, o);
         tmem_ld_wait(o);
-        if (row_ok && 16 * c < DG) {
+        if (row_ok && cc < DG) {
           float v[16];
 #pragma unroll
           for (int e = 0; e < 16; ++e) v[e] = bits_f(o[e]) * inv;
-          store_row16(p.out0 + rowoff + 16 * c, v);
+          store_row16(p.out0 + rowoff + cc, v);
         }
       }
-      if (row_ok) p.vec_out[(size_t)bh * N + gi] = (mrow + __log2f(lrow)) * kLn2;
+      if (row_ok && hf == 0) p.vec_out[(size_t)bh * N + gi] = (mrow + __log2f(lt)) * kLn2;
     }
   }
   tc_fence_before();
   __syncthreads();
-  if (warp == kMmaWarp) {
+  if (warp == kFwdX) {
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
   }

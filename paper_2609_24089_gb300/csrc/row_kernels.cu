@@ -42,7 +42,7 @@ static cudaError_t launch_fwd_one(const EngineParams& p, int nblocks, cudaStream
   cudaError_t e = cudaFuncSetAttribute(fwd_engine<D, DROP, DG>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  fwd_engine<D, DROP, DG><<<nblocks, kThreads, smem, s>>>(p);
+  fwd_engine<D, DROP, DG><<<nblocks, kFwdThreads, smem, s>>>(p);
   return cudaGetLastError();
 }
 
