@@ -66,6 +66,13 @@ struct FwdMisc {
 };
 static_assert(sizeof(FwdMisc) <= 256, "FwdMisc must fit the MISC area");
 
+// max(a, b, c) in one three-input instruction
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
+
 // TMEM columns: O_q at q D, S_q at 256 + 128 q.
 constexpr uint32_t kColS2 = 256;
 
@@ -302,7 +309,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1) fwd_engine(const __grid_consta
         const int mlo = jlo - (jt + 16 * c), mhi = jhi - (jt + 16 * c);
         if (mlo > 0 || mhi < 16) mask16(rS[c], mlo, mhi);
 #pragma unroll
-        for (int e = 0; e < 16; ++e) mraw = fmaxf(mraw, bits_f(rS[c][e]));
+        for (int e = 0; e < 16; e += 2) mraw = fmax3(mraw, bits_f(rS[c][e]), bits_f(rS[c][e + 1]));
       }
       // the row maximum over both halves: post this half's, wait for both
       // (which also means both halves hold their S in registers, so P may be
