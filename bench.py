@@ -62,7 +62,9 @@ def valid_pairs_rows(w, rows):
 
 def source_hash() -> str:
     h = hashlib.sha256()
-    for f in sorted(os.listdir(CSRC)):
+    for f in sorted(os.listdir(CSRC)):  # the kernel sources (no build or cache folders)
+        if not f.endswith((".cu", ".cuh", ".h")) or not os.path.isfile(os.path.join(CSRC, f)):
+            continue
         with open(os.path.join(CSRC, f), "rb") as fh:
             h.update(f.encode() + fh.read())
     return h.hexdigest()[:16]
