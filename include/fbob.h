@@ -99,7 +99,7 @@ struct CUstream_st; /* cudaStream_t == struct CUstream_st* */
 typedef enum fbob_status {
     FBOB_OK = 0,
     FBOB_ERR_INVALID_ARGUMENT = 1, /* null/misaligned/overlapping pointer, bad shape, scale */
-    FBOB_ERR_UNSUPPORTED = 2,      /* valid request this build does not implement (d not 32/64/128) */
+    FBOB_ERR_UNSUPPORTED = 2,      /* valid request the library does not implement (d not 32/64/128) */
     FBOB_ERR_CUDA = 3,             /* a CUDA runtime/driver call or launch failed */
     FBOB_ERR_DEVICE_TIMEOUT = 4,   /* a bounded device-side wait expired */
     FBOB_ERR_DEVICE_FAULT = 5,     /* the device reported an error while synchronising */
