@@ -258,3 +258,28 @@ def test_bounded_wait_timeout_is_reported_and_context_survives(monkeypatch):
     ref = oracle.bob(*(G.f64(bits[n]) for n in synth.NAMES), scale, False)
     for name, x in zip(("qbar", "kbar", "vbar", "dobar"), ref):
         G.check(name, r[name], x)
+
+
+@pytest.mark.parametrize("d,causal,rising", [(64, False, True), (128, True, True),
+                                             (128, False, False)])
+def test_forward_running_maximum_raised_many_times(d, causal, rising):
+    """Scores that ramp along the keys by about 85 log2 units: the forward's
+    lazily raised row maximum goes up some ten times (and every tile's largest
+    score sits in its second key half, so the first half takes it from the
+    exchange); a falling ramp never raises it after the first tile."""
+    B, H, N = 1, 2, 1000
+    rng = np.random.default_rng(7 + d)
+    e = np.full(d, 1.0 / np.sqrt(d))
+    amp = np.sqrt(60.0 * np.sqrt(d))  # q . k / sqrt(d) spans about [0, 60]
+    ramp = np.arange(N) / N if rising else 1.0 - np.arange(N) / N
+    q = amp * e + 0.1 * rng.standard_normal((B, H, N, d))
+    k = (amp * ramp)[:, None] * e + 0.1 * rng.standard_normal((B, H, N, d))
+    v = rng.standard_normal((B, H, N, d))
+    bits = {n: synth.bf16_bits(x.astype(np.float32)) for n, x in (("q", q), ("k", k), ("v", v))}
+    scale = 1 / np.sqrt(d)
+    o, lse = fbob.attn_fwd(G.dev(bits["q"]), G.dev(bits["k"]), G.dev(bits["v"]), scale, causal)
+    assert fbob.fbob_device_status() == 0
+    O, L = oracle.fwd(G.f64(bits["q"]), G.f64(bits["k"]), G.f64(bits["v"]), scale, causal)
+    G.check("O", G.host(o), O)
+    assert np.abs(lse.cpu().numpy() - L).max() <= 1e-3
+    assert L.max() > 40.0  # the ramp reached the scores
