@@ -10,11 +10,14 @@
 //   WGs m, l (online softmax): each half's row maxima are exchanged through
 //       shared memory, so both halves take the same running maximum; then
 //       P = 2^(S tau log2 e - m) is written as bf16 over the first 64
-//       columns of S_q (both halves hold their S in registers by then)
+//       columns of S_q (both halves hold their S in registers by then), or
+//       at d = 64 into 64 TMEM columns of its own
 //   Y   O_q += P_q(T) V(T)                  (A from TMEM, issuer Y)
 // X issues S_q(T+1) once O_q += P_q(T) V(T) has completed (it overwrites
-// P_q(T)).  The two query tiles' chains interleave, so the tensor pipe works
-// on one tile while the other's softmax runs.  The running maximum is raised
+// P_q(T)); at d = 64 P_q has TMEM columns of its own, and S_q(T+1) follows
+// as soon as the softmax holds S_q(T) in registers.  The two query tiles'
+// chains interleave, so the tensor pipe works on one tile while the other's
+// softmax runs.  The running maximum is raised
 // lazily (by more than kFwdSlack, so P <= 2^kFwdSlack); O_q is then
 // rescaled by the first half's warpgroup after the MMAs into it have
 // completed.  Each half keeps the row sum of its own keys; the epilogue adds
@@ -44,6 +47,11 @@ struct FwdCfg {
   static constexpr int STAT_BYTES = 2 * KB * BM * 128;     // Q_0, Q_1
   static constexpr int STAGE_BYTES = 2 * KB * BN2 * 128;   // K, V
   static constexpr int NSTAGES = D == 64 ? 4 : 2;
+  // d = 64 leaves TMEM room for separate P buffers (O 2 x 64, S 2 x 128, P
+  // 2 x 64 columns): S_q(T+1) is then issued as soon as both softmax halves
+  // hold S_q(T) in registers, instead of after O_q += P_q(T) V(T) has
+  // completed, which takes the S MMA off each query tile's critical path
+  static constexpr bool SEP_P = D == 64;
   // bookkeeping, then the row-maximum exchange [tile parity][q][half][row]
   // and the row-sum exchange [q][half][row]
   static constexpr int MISC_BYTES = 256 + 8 * BM * 4 + 4 * BM * 4;
@@ -73,8 +81,10 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
   return r;
 }
 
-// TMEM columns: O_q at q D, S_q at 256 + 128 q.
+// TMEM columns: O_q at q D, S_q at 256 + 128 q; with FwdCfg::SEP_P, P_q at
+// 128 + 64 q (otherwise P_q is written over the first 64 columns of S_q).
 constexpr uint32_t kColS2 = 256;
+constexpr uint32_t kColP = 128;
 
 template <int D, bool DROP, int DG>
 __global__ void __launch_bounds__(kFwdThreads, 1) fwd_engine(const __grid_constant__ EngineParams p) {
@@ -209,10 +219,17 @@ __global__ void __launch_bounds__(kFwdThreads, 1) fwd_engine(const __grid_consta
           for (int q = 0; q < 2 && ok; ++q) {
             if (!part(q, T)) continue;
             const int k = T - tq0[q];
-            // S_q(T) overwrites P_q(T-1): wait for O_q += P_q(T-1) V
-            if (k >= 1 && !mbar_wait(&m->o_done[q], (k - 1) & 1, wctl)) {
-              ok = false;
-              break;
+            if (k >= 1) {
+              // SEP_P: S_q(T) overwrites S_q(T-1): wait until both softmax
+              // halves hold it (their row-maximum exchange of tile T-1);
+              // otherwise S_q(T) overwrites P_q(T-1): wait for O_q += P_q(T-1) V
+              const bool w = C::SEP_P
+                                 ? mbar_wait(&m->xq[q][(k - 1) & 1], ((k - 1) >> 1) & 1, wctl)
+                                 : mbar_wait(&m->o_done[q], (k - 1) & 1, wctl);
+              if (!w) {
+                ok = false;
+                break;
+              }
             }
             tc_fence_after();
 #pragma unroll
@@ -246,7 +263,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1) fwd_engine(const __grid_consta
             tc_fence_after();
 #pragma unroll
             for (int ks = 0; ks < BN2 / 16; ++ks)
-              mma_ts(tmem + q * D, tmem + kColS2 + 128 * q + 8 * ks,
+              mma_ts(tmem + q * D, tmem + (C::SEP_P ? kColP + 64 * q : kColS2 + 128 * q) + 8 * ks,
                      vd0 + (uint64_t)((ks * 2048) >> 4), id_o, (k == 0 && ks == 0) ? 0u : 1u);
             mma_commit(&m->o_done[q]);
           }
@@ -357,6 +374,15 @@ __global__ void __launch_bounds__(kFwdThreads, 1) fwd_engine(const __grid_consta
       if (raise) mrow = mt;
       // no valid key yet: every score is -inf, so any finite m gives P = 0
       const float nm = mrow == -INFINITY ? 0.f : -mrow;
+      // SEP_P: P_q(T) overwrites P_q(T-1): wait for O_q += P_q(T-1) V
+      if (C::SEP_P && k >= 1) {
+        if (!ew_wait(&m->o_done[q], (k - 1) & 1)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+      }
+      const uint32_t pcol = C::SEP_P ? kColP + 64 * q : scol;
       // pairs of scores through the packed f32x2 FMA and add (half the
       // instructions of scalar ones; the same roundings)
       const float2 sl2v = make_float2(sl2, sl2), nmv = make_float2(nm, nm);
@@ -377,8 +403,8 @@ __global__ void __launch_bounds__(kFwdThreads, 1) fwd_engine(const __grid_consta
           }
           oP[e / 2] = pack_bf16(p0, p1);
         }
-        // P of keys 64 hf + 16c .. + 15 over S columns 32 hf + 8c .. + 7
-        tmem_st8(ta + scol + 32 * hf + 8 * c, oP);
+        // P of keys 64 hf + 16c .. + 15 in P columns 32 hf + 8c .. + 7
+        tmem_st8(ta + pcol + 32 * hf + 8 * c, oP);
       }
       lrow += ps.x + ps.y;
       tmem_st_wait();
