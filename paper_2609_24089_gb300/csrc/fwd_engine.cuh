@@ -17,11 +17,10 @@
 // P_q(T)); at d = 64 P_q has TMEM columns of its own, and S_q(T+1) follows
 // as soon as the softmax holds S_q(T) in registers.  The two query tiles'
 // chains interleave, so the tensor pipe works on one tile while the other's
-// softmax runs.  The running maximum is raised
-// lazily (by more than kFwdSlack, so P <= 2^kFwdSlack); O_q is then
-// rescaled by the first half's warpgroup after the MMAs into it have
-// completed.  Each half keeps the row sum of its own keys; the epilogue adds
-// the two.
+// softmax runs.  The running maximum is raised lazily (by more than
+// kFwdSlack, so P <= 2^kFwdSlack); O_q is then rescaled by the first half's
+// warpgroup after the MMAs into it have completed.  Each half keeps the row
+// sum of its own keys; the epilogue adds the two.
 //
 // Roles (608 threads): warps 0-7 softmax of query tile 0 (keys 0-63, then
 // 64-127), warps 8-15 of tile 1 (warp w reads TMEM lanes 32 (w % 4) .. +31),
