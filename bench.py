@@ -357,10 +357,14 @@ def run_gpu(args, w):
     total = sum(part_ms.values())
     dflops = bob_flops(w, CONTRACTIONS[dom])
     achieved = dflops / (dur * 1e-3) / 1e12
-    peak = peaks["bf16_sustained"]
+    # denominator: the burst bf16 peak (each kernel is timed per launch, a few
+    # ms at most, at the clocks sampled below); the sustained figure (a
+    # seconds-long cuBLAS loop under the power cap) is kept as a second number
+    peak = peaks["bf16"]
     roofline = {"bound": "tensor", "kernel": KERNEL_NAMES[dom], "achieved": achieved,
                 "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
-                "peak_kind": f"bf16 sustained ({peaks['source']})",
+                "peak_kind": f"bf16 burst ({peaks['source']})",
+                "frac_of_sustained": achieved / peaks["bf16_sustained"],
                 "traffic": ncu_traffic(dom, w.name),
                 "credited_contractions": CONTRACTIONS[dom],
                 "launch_ms": dur, "share_of_step": dur / total,
@@ -386,6 +390,7 @@ def run_gpu(args, w):
                                     if w.window != (-1, -1) or w.segments
                                     else "2*19*B*H*N^2*d*(1/2 if causal)")},
         "frac_of_bf16_peak": value / world / peak,
+        "frac_of_bf16_sustained": value / world / peaks["bf16_sustained"],
         "roofline": roofline,
         "cpu_baseline": cpu,
         "e2e": {"value": e2e_val, "unit": "TFLOP/s", "h2d_bytes_per_step": h2d,
@@ -448,7 +453,7 @@ def run_gpu_op(args, w):
         raise RuntimeError("device status not OK")
     ms = start.elapsed_time(stop) / args.steps
     value = bob_flops(w, contractions) / (ms * 1e-3) / 1e12
-    peak = measured_peaks()["bf16_sustained"]
+    peak = measured_peaks()["bf16"]
     print(json.dumps({
         "metric": f"attention {args.op} TFLOP/s ({contractions} contractions x 2*B*H*N^2*d*rho)",
         "value": value, "unit": "TFLOP/s", "n_gpus": 1, "steps": args.steps,

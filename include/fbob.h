@@ -66,8 +66,11 @@
  *             owns every buffer (fbob_attn_bob_host's device workspace
  *             included).  Library state is one device-side error word per
  *             device, cached driver entry points, and the fixed 64 MiB staging
- *             array of fbob_attn_bob_host_noalloc, placed on a device by that
- *             call's first use there.  fbob_attn_bob_host creates three streams
+ *             array of fbob_attn_bob_host_noalloc.  Under lazy module loading
+ *             (the CUDA default) that array is placed on a device by that
+ *             call's first use there; with CUDA_MODULE_LOADING=EAGER every
+ *             context that loads the library reserves it at once, whether or
+ *             not the call is ever made.  fbob_attn_bob_host creates three streams
  *             and seven events per call and releases them when their work is
  *             done; no other call creates any CUDA object.
  *  Errors     Host-side validation failures return immediately, before any
@@ -270,9 +273,11 @@ int64_t fbob_attn_bob_host_workspace(const fbob_shape* shape, int64_t chunk_head
  *      bytes, must fit in 64 MiB (for example N = 16384 at d = 128 without
  *      grouping); larger problems return FBOB_ERR_SCRATCH_LIMIT and run
  *      nothing (use fbob_attn_bob_host with a workspace).
- * Set-up: the first call on each device looks up the array's device address
- *      (with that device current), which also places the array on that
- *      device; make that first call before any stream capture.
+ * Set-up: every call looks up the array's device address on the current
+ *      device (cudaGetSymbolAddress, no allocation), so an address is never
+ *      reused across a context teardown (cudaDeviceReset).  Under lazy module
+ *      loading the first lookup on a device also places the array there; make
+ *      that first call before any stream capture.
  * Nothing in the array has to start at zero: each call writes every byte it
  *      reads.  All calls on a device share the array, so calls that overlap in
  *      time (on other streams or threads) race; serialise them.
@@ -293,7 +298,7 @@ int fbob_device_status(struct CUstream_st* stream);
 
 /* Number of kernels the last successful call of the named entry point
  * enqueued ("fwd", "bwd", "bob", "bob_pass1", "bob_pass2", "bob_row_stats",
- * "bob_pass1_direct"); -1 if unknown. */
+ * "bob_pass1_direct", "bob_host", "bob_host_noalloc"); -1 if unknown. */
 int fbob_launch_count(const char* entry);
 
 /* Static, human-readable name of a status code. */

@@ -179,7 +179,7 @@ def bwd(q, k, v, dout, scale, causal, nthreads=0, window=None, segments=None, dr
 
 def bob_head(q, k, v, dout, gq, gk, gv, scale, causal, rows=None, cols=None,
              nthreads=0, mutant=0, mutant_dir=None, window=None, segments=None,
-             dropout=None, head=0):
+             dropout=None, head=0, row_outputs=True):
     """Backward-over-backward of one head ([N, d] float64 arrays).
 
     rows: query rows whose row-owned outputs are wanted (default: all).
@@ -191,6 +191,8 @@ def bob_head(q, k, v, dout, gq, gk, gv, scale, causal, rows=None, cols=None,
     segments: offsets of packed sequences; a row sees only its own sequence.
     dropout: (p, seed); head: the flat query-head index b*H + h that keys the
     head's dropout mask.
+    row_outputs: False skips the listed rows' qbar and dobar (left as zeros),
+    for callers that want only the column block (it halves the work per row).
     """
     wl, wr = _window(window)
     pd, seed = _dropout(dropout)
@@ -217,7 +219,8 @@ def bob_head(q, k, v, dout, gq, gk, gv, scale, causal, rows=None, cols=None,
                              pd, seed, int(head),
                              _ptr(q), _ptr(k), _ptr(v), _ptr(dout), _ptr(gq), _ptr(gk), _ptr(gv),
                              _ptr(rows), nr, c0, c1,
-                             _ptr(res["qbar"]), _ptr(res["dobar"]), _ptr(res["alpha"]),
+                             _ptr(res["qbar"] if row_outputs else None),
+                             _ptr(res["dobar"] if row_outputs else None), _ptr(res["alpha"]),
                              _ptr(res["E"]), _ptr(res["D"]), _ptr(res["L"]),
                              _ptr(res["kbar"]), _ptr(res["vbar"]), int(nthreads))
     assert rc == 0, rc

@@ -28,7 +28,9 @@ enum Entry {
 
 // Staging memory of fbob_attn_bob_host_noalloc: a fixed device array, so that
 // call allocates nothing.  Its module holds no kernels; the array is placed
-// when the module is loaded on a device (on the first address lookup).
+// when the module is loaded on a device: at the first address lookup under
+// lazy module loading (the CUDA default), at context creation under
+// CUDA_MODULE_LOADING=EAGER.
 constexpr int64_t kNoAllocBytes = int64_t(64) << 20;
 __device__ __align__(256) uint8_t g_noalloc_scratch[kNoAllocBytes];
 
@@ -314,22 +316,14 @@ int64_t chunk_heads(const fbob_shape* s, int64_t ws_bytes) {
 }
 
 // Device address of the static staging array on the current device, looked
-// up once per device.
+// up on every call: an address cached across calls could outlive the context
+// it belongs to (a cudaDeviceReset tears the module down and the next context
+// places the array again, possibly elsewhere).  The lookup allocates nothing.
 cudaError_t noalloc_scratch(uint8_t** ptr) {
-  static std::mutex mu;
-  static uint8_t* addr[64] = {};
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
+  void* p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
   if (e != cudaSuccess) return e;
-  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-  std::lock_guard<std::mutex> lock(mu);
-  if (!addr[dev]) {
-    void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-    if (e != cudaSuccess) return e;
-    addr[dev] = static_cast<uint8_t*>(p);
-  }
-  *ptr = addr[dev];
+  *ptr = static_cast<uint8_t*>(p);
   return cudaSuccess;
 }
 

@@ -7,8 +7,10 @@ launch configuration the benchmark times.
   n64k_d128_causal_peaky oracle on sampled rows (row-owned outputs) and on the
                          causal tail: key columns >= N - 256 are complete once
                          rows >= N - 256 are summed
-  n256k_d64              oracle on sampled rows; Ktil, Vtil through identities that
-                         hold at any size (column sums vanish, Euler identities)
+  n256k_d64              oracle on sampled rows; one 128-key block of Ktil, Vtil
+                         (keys 199936..200063 of head 1) against stored oracle
+                         values; every head through identities that hold at any
+                         size (column sums vanish, Euler identities)
   n16k_d128_causal_swa4k sliding window w = N/4: oracle on sampled rows and on a
                          256-key block, complete once the rows whose band holds
                          it (keys j .. j + 4095) are summed
@@ -27,6 +29,7 @@ import oracle
 import paper_2609_24089_gb300 as fbob
 from paper_2609_24089_gb300 import synth
 from tests import gpu_util as G
+from tests.golden import make_n256k_d64_key_block as key_block
 
 pytestmark = pytest.mark.gpu
 
@@ -120,6 +123,14 @@ def test_n256k_d64_rows_and_identities():
     r = {"qbar": G.host(qb), "dobar": G.host(dob), "alpha": rs[0].cpu().numpy(),
          "E": rs[1].cpu().numpy(), "D": rs[2].cpu().numpy()}
     check_rows(r, G.oracle_bob_heads(bits, w.scale, w.causal, heads, rows=rows), heads, H, rows)
+    # one complete 128-key block of Ktil and Vtil past 2^17, element by element
+    # against the stored fp64 oracle values (all 262,144 rows of head 1 summed;
+    # tests/golden/make_n256k_d64_key_block.py wrote them)
+    kref, vref = key_block.load()
+    c0, c1 = key_block.C0, key_block.C1
+    b, h = divmod(key_block.HEAD, H)
+    G.check("kbar[head 1, keys 199936..200063]", G.host(kb[b, h, c0:c1]), kref)
+    G.check("vbar[head 1, keys 199936..200063]", G.host(vb[b, h, c0:c1]), vref)
     # identities, per head, in fp64 over the bf16 outputs
     for hh in range(w.B * H):
         b, h = divmod(hh, H)

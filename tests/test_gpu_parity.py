@@ -238,26 +238,72 @@ def test_single_key_degenerate(d, causal):
     assert np.abs(r["vbar"]).max() <= 1e-4 * np.abs(X["dout"]).max() * np.abs(X["gq"]).max() * d
 
 
-def test_bounded_wait_timeout_is_reported_and_context_survives(monkeypatch):
+STALL_CASES = [  # entry, d, causal, dropout
+    ("bob", 64, False, None),     # one-sweep Pass 1, Pass 2 at d = 64
+    ("bob", 128, True, None),     # row statistics + direct Pass 1, Pass 2 at d = 128
+    ("bob", 32, True, None),      # head dim 32 in the d = 64 tiles
+    ("bob", 128, True, (0.1, 5)),  # the dropout instantiations of all three
+    ("bob", 64, False, (0.2, 9)),  # dropout at d = 64: statistics + direct form
+    ("fwd", 64, False, None),     # forward engine (608 threads, its own barriers)
+    ("fwd", 128, True, None),
+    ("fwd", 128, False, (0.1, 3)),
+    ("bwd", 64, True, None),      # first backward: dQ (row) and dK/dV (column) kernels
+    ("bwd", 128, False, None),
+    ("bwd", 128, True, (0.1, 4)),
+]
+
+
+def stall_id(c):
+    return "{}_d{}{}{}".format(c[0], c[1], "c" if c[2] else "", "_drop" if c[3] else "")
+
+
+@pytest.mark.parametrize("case", STALL_CASES, ids=stall_id)
+def test_bounded_wait_timeout_is_reported_and_context_survives(monkeypatch, case):
     """Failure detection without a GPU fault: with the producers' loads
     suppressed (FBOB_INJECT_STALL=1) every consumer wait runs into its bounded
     limit; the kernels record FBOB_ERR_DEVICE_TIMEOUT, release tensor memory
-    and exit, and the next call on the same context computes correct results."""
-    B, H, N, d = 1, 1, 256, 64
-    bits = G.inputs(B, H, N, d, seed=77)
+    and exit, and the next call on the same context computes correct results.
+    Every kernel family is covered: the BoB passes (each Pass 1 form, with and
+    without dropout), the forward and both first-backward kernels."""
+    entry, d, causal, drop = case
+    B, H, N = 1, 2, 300
+    bits = G.inputs(B, H, N, d, seed=77 + d)
     scale = 1 / np.sqrt(d)
-    o_l = G.oracle_o_l(bits, scale, False)
+    X = {n: G.f64(bits[n]) for n in synth.NAMES}
+    q, k, v, do = (G.dev(bits[n]) for n in ("q", "k", "v", "dout"))
+
+    def run():
+        if entry == "fwd":
+            o, lse = fbob.attn_fwd(q, k, v, scale, causal, dropout=drop)
+            return fbob.fbob_device_status(), (o, lse)
+        if entry == "bwd":
+            o_l = G.oracle_o_l(bits, scale, causal, dropout=drop)
+            o, lse = G.dev(o_l[0]), G.dev_f32(o_l[1])
+            out = fbob.attn_bwd(q, k, v, o, lse, do, scale, causal, dropout=drop)
+            return fbob.fbob_device_status(), out
+        r = G.run_bob(bits, scale, causal, o_l=G.oracle_o_l(bits, scale, causal, dropout=drop),
+                      dropout=drop)
+        return r["status"], r
+
     monkeypatch.setenv("FBOB_WAIT_LIMIT_MS", "50")
     monkeypatch.setenv("FBOB_INJECT_STALL", "1")
-    r = G.run_bob(bits, scale, False, o_l=o_l)
-    assert r["status"] == fbob.STATUS_CODES["FBOB_ERR_DEVICE_TIMEOUT"]
+    status, _ = run()
+    assert status == fbob.STATUS_CODES["FBOB_ERR_DEVICE_TIMEOUT"]
     monkeypatch.delenv("FBOB_INJECT_STALL")
     monkeypatch.delenv("FBOB_WAIT_LIMIT_MS")
-    r = G.run_bob(bits, scale, False, o_l=o_l)
-    assert r["status"] == 0
-    ref = oracle.bob(*(G.f64(bits[n]) for n in synth.NAMES), scale, False)
-    for name, x in zip(("qbar", "kbar", "vbar", "dobar"), ref):
-        G.check(name, r[name], x)
+    status, out = run()
+    assert status == 0
+    if entry == "fwd":
+        O, _ = oracle.fwd(X["q"], X["k"], X["v"], scale, causal, dropout=drop)
+        G.check("O", G.host(out[0]), O)
+    elif entry == "bwd":
+        ref = oracle.bwd(X["q"], X["k"], X["v"], X["dout"], scale, causal, dropout=drop)
+        for name, got, x in zip(("dQ", "dK", "dV"), out[:3], ref[:3]):
+            G.check(name, G.host(got), x)
+    else:
+        ref = oracle.bob(*(X[n] for n in synth.NAMES), scale, causal, dropout=drop)
+        for name, x in zip(("qbar", "kbar", "vbar", "dobar"), ref):
+            G.check(name, out[name], x)
 
 
 @pytest.mark.parametrize("d,causal,rising", [(64, False, True), (128, True, True),
