@@ -48,7 +48,7 @@ def _load(mutant: int = 0, out_dir: str | None = None):
     lib = ctypes.CDLL(build(mutant, out_dir))
     i64, dbl, cint = ctypes.c_int64, ctypes.c_double, ctypes.c_int
     u64, p = ctypes.c_uint64, ctypes.c_void_p
-    mask = [i64, i64, dbl, cint, i64, i64, p, i64, dbl, u64, i64]
+    mask = [i64, i64, dbl, cint, i64, i64, p, i64, dbl, u64, i64, p, i64]
     lib.fbob_oracle_fwd.argtypes = mask + [p, p, p, p, p, cint]
     lib.fbob_oracle_bwd.argtypes = mask + [p, p, p, p, p, p, p, p, cint]
     lib.fbob_oracle_bob.argtypes = mask + [p, p, p, p, p, p, p,
@@ -88,6 +88,19 @@ def _segments(segments, N):
     return seg, seg.size - 1
 
 
+def _blocks(block_mask, block_size, N):
+    """Block-sparse mask (App. "Extensions"): a [nb, nb] 0/1 array over square
+    blocks of block_size rows and columns, nb = ceil(N / block_size), as
+    uint8 bytes; None keeps every block."""
+    if block_mask is None:
+        return None, 0
+    bs = int(block_size)
+    nb = (N + bs - 1) // bs
+    bm = np.ascontiguousarray(np.asarray(block_mask) != 0, dtype=np.uint8)
+    assert bm.shape == (nb, nb), (bm.shape, nb)
+    return bm, bs
+
+
 def _dropout(dropout):
     """(p, seed) of attention dropout (App. "Extensions"); p = 0: none."""
     if dropout is None:
@@ -121,17 +134,20 @@ def _heads(x):
     return x
 
 
-def fwd(q, k, v, scale, causal, nthreads=0, window=None, segments=None, dropout=None):
+def fwd(q, k, v, scale, causal, nthreads=0, window=None, segments=None, dropout=None,
+        block_mask=None, block_size=128):
     """Forward attention (eq. 1).  Returns O [B,H,N,d] and natural-log L [B,H,N].
     window: (wl, wr) sliding-window band (default: none); segments: offsets of
     packed sequences (default: one sequence); dropout: (p, seed), the keep
-    mask of query head b*H + h drawn from Philox with that head index."""
+    mask of query head b*H + h drawn from Philox with that head index;
+    block_mask: [nb, nb] 0/1 blocks of block_size (default: none)."""
     wl, wr = _window(window)
     pd, seed = _dropout(dropout)
     q, k, v = (_c(_heads(t)) for t in (q, k, v))
     B, H, N, d = q.shape
     G = _group(H, k.shape[1])
     seg, nseg = _segments(segments, N)
+    bm, bs = _blocks(block_mask, block_size, N)
     lib = _load()
     O = np.zeros_like(q)
     L = np.zeros((B, H, N))
@@ -140,7 +156,7 @@ def fwd(q, k, v, scale, causal, nthreads=0, window=None, segments=None, dropout=
             o_ = np.zeros((N, d)); l_ = np.zeros(N)
             hk = h // G
             rc = lib.fbob_oracle_fwd(N, d, float(scale), int(bool(causal)), wl, wr,
-                                     _ptr(seg), nseg, pd, seed, b * H + h,
+                                     _ptr(seg), nseg, pd, seed, b * H + h, _ptr(bm), bs,
                                      _ptr(_c(q[b, h])), _ptr(_c(k[b, hk])), _ptr(_c(v[b, hk])),
                                      _ptr(o_), _ptr(l_), int(nthreads))
             assert rc == 0, rc
@@ -148,16 +164,19 @@ def fwd(q, k, v, scale, causal, nthreads=0, window=None, segments=None, dropout=
     return O, L
 
 
-def bwd(q, k, v, dout, scale, causal, nthreads=0, window=None, segments=None, dropout=None):
+def bwd(q, k, v, dout, scale, causal, nthreads=0, window=None, segments=None, dropout=None,
+        block_mask=None, block_size=128):
     """First backward (eqs. 2-3).  Returns dQ [B,H,N,d], dK, dV [B,Hkv,N,d] and
     D [B,H,N]; with grouped-query attention (k, v with Hkv < H heads) dK and dV
-    of a key/value head are the sums over its query heads.  dropout as in fwd."""
+    of a key/value head are the sums over its query heads.  dropout and
+    block_mask as in fwd."""
     wl, wr = _window(window)
     pd, seed = _dropout(dropout)
     q, k, v, dout = (_c(_heads(t)) for t in (q, k, v, dout))
     B, H, N, d = q.shape
     G = _group(H, k.shape[1])
     seg, nseg = _segments(segments, N)
+    bm, bs = _blocks(block_mask, block_size, N)
     lib = _load()
     outs = [np.zeros_like(q), np.zeros_like(k), np.zeros_like(v)]
     D = np.zeros((B, H, N))
@@ -166,7 +185,7 @@ def bwd(q, k, v, dout, scale, causal, nthreads=0, window=None, segments=None, dr
             hk = h // G
             dq, dk, dv, dd = np.zeros((N, d)), np.zeros((N, d)), np.zeros((N, d)), np.zeros(N)
             rc = lib.fbob_oracle_bwd(N, d, float(scale), int(bool(causal)), wl, wr,
-                                     _ptr(seg), nseg, pd, seed, b * H + h,
+                                     _ptr(seg), nseg, pd, seed, b * H + h, _ptr(bm), bs,
                                      _ptr(_c(q[b, h])), _ptr(_c(k[b, hk])), _ptr(_c(v[b, hk])),
                                      _ptr(_c(dout[b, h])), _ptr(dq), _ptr(dk), _ptr(dv),
                                      _ptr(dd), int(nthreads))
@@ -179,7 +198,7 @@ def bwd(q, k, v, dout, scale, causal, nthreads=0, window=None, segments=None, dr
 
 def bob_head(q, k, v, dout, gq, gk, gv, scale, causal, rows=None, cols=None,
              nthreads=0, mutant=0, mutant_dir=None, window=None, segments=None,
-             dropout=None, head=0, row_outputs=True):
+             dropout=None, head=0, row_outputs=True, block_mask=None, block_size=128):
     """Backward-over-backward of one head ([N, d] float64 arrays).
 
     rows: query rows whose row-owned outputs are wanted (default: all).
@@ -191,6 +210,8 @@ def bob_head(q, k, v, dout, gq, gk, gv, scale, causal, rows=None, cols=None,
     segments: offsets of packed sequences; a row sees only its own sequence.
     dropout: (p, seed); head: the flat query-head index b*H + h that keys the
     head's dropout mask.
+    block_mask: [nb, nb] 0/1 array over square blocks of block_size rows and
+    columns (nb = ceil(N / block_size)); a pair is kept only if its block is.
     row_outputs: False skips the listed rows' qbar and dobar (left as zeros),
     for callers that want only the column block (it halves the work per row).
     """
@@ -199,6 +220,7 @@ def bob_head(q, k, v, dout, gq, gk, gv, scale, causal, rows=None, cols=None,
     q, k, v, dout, gq, gk, gv = (_c(t) for t in (q, k, v, dout, gq, gk, gv))
     N, d = q.shape
     seg, nseg = _segments(segments, N)
+    bm, bs = _blocks(block_mask, block_size, N)
     if rows is None:
         rows = np.arange(N, dtype=np.int64)
         if cols is None:
@@ -216,7 +238,7 @@ def bob_head(q, k, v, dout, gq, gk, gv, scale, causal, rows=None, cols=None,
     }
     lib = _load(mutant, mutant_dir)
     rc = lib.fbob_oracle_bob(N, d, float(scale), int(bool(causal)), wl, wr, _ptr(seg), nseg,
-                             pd, seed, int(head),
+                             pd, seed, int(head), _ptr(bm), bs,
                              _ptr(q), _ptr(k), _ptr(v), _ptr(dout), _ptr(gq), _ptr(gk), _ptr(gv),
                              _ptr(rows), nr, c0, c1,
                              _ptr(res["qbar"] if row_outputs else None),
@@ -228,7 +250,7 @@ def bob_head(q, k, v, dout, gq, gk, gv, scale, causal, rows=None, cols=None,
 
 
 def bob(q, k, v, dout, gq, gk, gv, scale, causal, nthreads=0, mutant=0, mutant_dir=None,
-        window=None, segments=None, dropout=None):
+        window=None, segments=None, dropout=None, block_mask=None, block_size=128):
     """Full backward-over-backward on [B,H,N,d] (or [N,d]) float64 arrays.
 
     Returns (qbar, kbar, vbar, dobar, alpha, E, D) with the input's batch shape.
@@ -252,7 +274,8 @@ def bob(q, k, v, dout, gq, gk, gv, scale, causal, nthreads=0, mutant=0, mutant_d
             args = [t[b, h // G] if i in kv_side else t[b, h] for i, t in enumerate(ts)]
             r = bob_head(*args, scale, causal, nthreads=nthreads,
                          mutant=mutant, mutant_dir=mutant_dir, window=window,
-                         segments=segments, dropout=dropout, head=b * H + h)
+                         segments=segments, dropout=dropout, head=b * H + h,
+                         block_mask=block_mask, block_size=block_size)
             for n in ("qbar", "dobar", "alpha", "E", "D"):
                 out[n][b, h] = r[n]
             out["kbar"][b, h // G] += r["kbar"]

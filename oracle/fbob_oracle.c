@@ -39,7 +39,13 @@
  * sequences (App. "Extensions"): with segment offsets seg[0..nseg] (seg[0] =
  * 0, non-decreasing, seg[nseg] = N) row i also keeps only the columns of its
  * own segment [seg[s], seg[s+1]), s the segment holding i; seg = NULL is one
- * segment.  Every row keeps its diagonal.  Entries outside V_i have P = 0 and
+ * segment.  Block-sparse masks (App. "Extensions": a sparse mask only needs a
+ * well-defined set of allowed columns per row, with zero probability on the
+ * masked entries): with a block mask bm of nb x nb bytes over square blocks of
+ * bs rows and bs columns (nb = ceil(N / bs)), the pair (i, j) is kept only if
+ * also bm[(i / bs) * nb + j / bs] != 0; bm = NULL keeps every block.  Every
+ * row keeps its diagonal (for the block mask: every diagonal block is set).
+ * Entries outside V_i, and masked entries inside it, have P = 0 and
  * contribute nothing.
  *
  * Dropout (App. "Extensions"): with keep mask R and sigma = 1/(1 - p) the
@@ -131,8 +137,25 @@ static double gate(drop_t g, int64_t i, int64_t j) {
     return byte >= g.thr ? g.sigma : 0.0;
 }
 
-/* the valid columns [lo_i, hi_i) of row i (see the header comment) */
-typedef struct { int causal; int64_t wl, wr; const int64_t* seg; int64_t nseg; } band_t;
+/* the valid columns [lo_i, hi_i) of row i (see the header comment), and the
+ * block mask inside that range */
+typedef struct {
+    int causal; int64_t wl, wr; const int64_t* seg; int64_t nseg;
+    const uint8_t* bm; int64_t bs, nb;
+} band_t;
+
+static band_t make_band(int64_t N, int causal, int64_t wl, int64_t wr, const int64_t* seg,
+                        int64_t nseg, const uint8_t* bm, int64_t bs) {
+    band_t m = {causal, wl, wr, seg, nseg, bm, bs, 0};
+    if (bm && bs > 0) m.nb = (N + bs - 1) / bs;
+    else m.bm = NULL;
+    return m;
+}
+
+/* 1 if the block mask keeps the pair (i, j) (always without a block mask) */
+static int block_keeps(band_t m, int64_t i, int64_t j) {
+    return !m.bm || m.bm[(i / m.bs) * m.nb + j / m.bs] != 0;
+}
 
 static void valid_cols(int64_t i, int64_t N, band_t m, int64_t* lo, int64_t* hi) {
     int64_t a = m.wl < 0 ? 0 : i - m.wl;
@@ -178,12 +201,18 @@ static void softmax_row(int64_t i, int64_t N, int64_t d, double tau, band_t mk,
     double m = -INFINITY;
     for (int64_t j = lo; j < hi; ++j) {
         S[j] = tau * dot(Q + i * d, K + j * d, d);
-        if (S[j] > m) m = S[j];
+        if (block_keeps(mk, i, j) && S[j] > m) m = S[j];
     }
     double z = 0.0;
-    for (int64_t j = lo; j < hi; ++j) z += exp(S[j] - m);
+    for (int64_t j = lo; j < hi; ++j)
+#if FBOB_MUTANT == 11 /* planted: masked blocks left in the normaliser */
+        z += exp(S[j] - m);
+#else
+        if (block_keeps(mk, i, j)) z += exp(S[j] - m);
+#endif
     const double L = m + log(z);
-    for (int64_t j = lo; j < hi; ++j) P[j] = exp(S[j] - L);
+    /* masked entries of the block mask: zero probability */
+    for (int64_t j = lo; j < hi; ++j) P[j] = block_keeps(mk, i, j) ? exp(S[j] - L) : 0.0;
     *L_out = L;
     *lo_out = lo;
     *hi_out = hi;
@@ -192,11 +221,11 @@ static void softmax_row(int64_t i, int64_t N, int64_t d, double tau, band_t mk,
 /* ---------------------------------------------------------------- forward */
 int fbob_oracle_fwd(int64_t N, int64_t d, double tau, int causal, int64_t wl, int64_t wr,
                     const int64_t* seg, int64_t nseg, double p_drop, uint64_t seed,
-                    int64_t head,
+                    int64_t head, const uint8_t* bm, int64_t bs,
                     const double* Q, const double* K, const double* V,
                     double* O, double* L, int nthreads) {
     if (N < 0 || d <= 0) return 1;
-    const band_t mk = {causal, wl, wr, seg, nseg};
+    const band_t mk = make_band(N, causal, wl, wr, seg, nseg, bm, bs);
     const drop_t dg = make_drop(p_drop, seed, head);
     const int nt = pick_threads(nthreads);
 #pragma omp parallel num_threads(nt)
@@ -224,11 +253,11 @@ int fbob_oracle_fwd(int64_t N, int64_t d, double tau, int causal, int64_t wl, in
 /* ------------------------------------------------------- first backward */
 int fbob_oracle_bwd(int64_t N, int64_t d, double tau, int causal, int64_t wl, int64_t wr,
                     const int64_t* seg, int64_t nseg, double p_drop, uint64_t seed,
-                    int64_t head,
+                    int64_t head, const uint8_t* bm, int64_t bs,
                     const double* Q, const double* K, const double* V, const double* dO,
                     double* dQ, double* dK, double* dV, double* Dvec, int nthreads) {
     if (N < 0 || d <= 0) return 1;
-    const band_t mk = {causal, wl, wr, seg, nseg};
+    const band_t mk = make_band(N, causal, wl, wr, seg, nseg, bm, bs);
     const drop_t dg = make_drop(p_drop, seed, head);
     const int nt = pick_threads(nthreads);
     const size_t nd = (size_t)N * (size_t)d;
@@ -294,14 +323,14 @@ int fbob_oracle_bwd(int64_t N, int64_t d, double tau, int causal, int64_t wl, in
  */
 int fbob_oracle_bob(int64_t N, int64_t d, double tau, int causal, int64_t wl, int64_t wr,
                     const int64_t* seg, int64_t nseg, double p_drop, uint64_t seed,
-                    int64_t head,
+                    int64_t head, const uint8_t* bm, int64_t bs,
                     const double* Q, const double* K, const double* V, const double* dO,
                     const double* UQ, const double* UK, const double* UV,
                     const int64_t* rows, int64_t nrows, int64_t c0, int64_t c1,
                     double* Qt, double* dOt, double* alpha_out, double* E_out,
                     double* D_out, double* L_out, double* Kt, double* Vt, int nthreads) {
     if (N < 0 || d <= 0 || nrows < 0) return 1;
-    const band_t mk = {causal, wl, wr, seg, nseg};
+    const band_t mk = make_band(N, causal, wl, wr, seg, nseg, bm, bs);
     const drop_t dg = make_drop(p_drop, seed, head);
     for (int64_t r = 0; r < nrows; ++r)
         if (rows[r] < 0 || rows[r] >= N) return 1;

@@ -14,13 +14,18 @@ from __future__ import annotations
 import numpy as np
 
 
-def mask(N, causal, window=None, segments=None):
+def mask(N, causal, window=None, segments=None, block=None):
     """0/1 mask: causal keeps j <= i; window (wl, wr) keeps i - wl <= j <= i + wr
     (a negative side is unbounded); segments (offsets of packed sequences)
-    keeps i and j in the same sequence (a block-diagonal mask)."""
+    keeps i and j in the same sequence (a block-diagonal mask); block
+    (bm, bs) keeps (i, j) only where the [nb, nb] 0/1 block mask bm has its
+    block (i // bs, j // bs) set (a block-sparse mask)."""
     i = np.arange(N)[:, None]
     j = np.arange(N)[None, :]
     keep = np.ones((N, N), dtype=bool)
+    if block is not None:
+        bm, bs = block
+        keep &= np.asarray(bm)[i // bs, j // bs] != 0
     if segments is not None:
         sid = np.searchsorted(np.asarray(segments)[1:], np.arange(N), side="right")
         keep &= sid[:, None] == sid[None, :]
@@ -35,25 +40,26 @@ def mask(N, causal, window=None, segments=None):
     return keep.astype(np.float64)
 
 
-def softmax_probs(Q, K, tau, causal, window=None, segments=None):
+def softmax_probs(Q, K, tau, causal, window=None, segments=None, block=None):
     """P = softmax_row(tau Q K^T + M) for [..., N, d] inputs (real or complex).
 
     The shift uses the real part of the row max so the function stays
     complex-analytic (the shift cancels exactly in the ratio)."""
     N = Q.shape[-2]
     S = tau * (Q @ np.swapaxes(K, -1, -2))
-    Mk = mask(N, causal, window, segments)
+    Mk = mask(N, causal, window, segments, block)
     shift = np.max(np.where(Mk > 0, S.real, -np.inf), axis=-1, keepdims=True)
     Ex = np.exp(S - shift) * Mk
     return Ex / Ex.sum(axis=-1, keepdims=True)
 
 
-def first_backward(Q, K, V, dO, tau, causal, window=None, segments=None, gate=None):
+def first_backward(Q, K, V, dO, tau, causal, window=None, segments=None, gate=None,
+                   block=None):
     """g(Q, K, V, dO) = (dQ, dK, dV), eqs. (2)-(3), batched over leading dims.
     gate: [N, N] dropout gate sigma R of the forward O = (gate o P) V, which
     turns the derivative with respect to P into gate o (dO V^T) and dV into
     (gate o P)^T dO."""
-    P = softmax_probs(Q, K, tau, causal, window, segments)
+    P = softmax_probs(Q, K, tau, causal, window, segments, block)
     g = 1.0 if gate is None else gate
     dP = g * (dO @ np.swapaxes(V, -1, -2))
     D = (P * dP).sum(axis=-1, keepdims=True)
@@ -64,13 +70,14 @@ def first_backward(Q, K, V, dO, tau, causal, window=None, segments=None, gate=No
     return dQ, dK, dV
 
 
-def attention(Q, K, V, tau, causal, window=None, segments=None, gate=None):
-    P = softmax_probs(Q, K, tau, causal, window, segments)
+def attention(Q, K, V, tau, causal, window=None, segments=None, gate=None, block=None):
+    P = softmax_probs(Q, K, tau, causal, window, segments, block)
     return (P if gate is None else gate * P) @ V
 
 
-def phi(Q, K, V, dO, UQ, UK, UV, tau, causal, window=None, segments=None, gate=None):
-    dQ, dK, dV = first_backward(Q, K, V, dO, tau, causal, window, segments, gate)
+def phi(Q, K, V, dO, UQ, UK, UV, tau, causal, window=None, segments=None, gate=None,
+        block=None):
+    dQ, dK, dV = first_backward(Q, K, V, dO, tau, causal, window, segments, gate, block)
     return ((dQ * UQ).sum(axis=(-1, -2)) + (dK * UK).sum(axis=(-1, -2))
             + (dV * UV).sum(axis=(-1, -2)))
 
@@ -140,7 +147,7 @@ def _perturbed(X, which, deltas):
 
 
 def bob_central_fd(Q, K, V, dO, UQ, UK, UV, tau, causal, rel_h=1e-5, window=None,
-                   segments=None, gate=None):
+                   segments=None, gate=None, block=None):
     """grad_{Q,K,V,dO} Phi by central differences, one entry at a time."""
     X = [Q, K, V, dO]
     grads = []
@@ -149,8 +156,8 @@ def bob_central_fd(Q, K, V, dO, UQ, UK, UV, tau, causal, rel_h=1e-5, window=None
         h = rel_h * np.maximum(1.0, np.abs(x))
         plus = _perturbed(X, which, h)
         minus = _perturbed(X, which, -h)
-        fp = phi(*plus, UQ, UK, UV, tau, causal, window, segments, gate)
-        fm = phi(*minus, UQ, UK, UV, tau, causal, window, segments, gate)
+        fp = phi(*plus, UQ, UK, UV, tau, causal, window, segments, gate, block)
+        fm = phi(*minus, UQ, UK, UV, tau, causal, window, segments, gate, block)
         grads.append(((fp - fm) / (2 * h)).reshape(X[which].shape))
     return grads
 
