@@ -47,9 +47,11 @@ CSRC = os.path.join(ROOT, "paper_2609_24089_gb300", "csrc")
 
 def bob_flops(w, contractions=19):
     """2 * contractions * B*H*N^2*d*rho: rho = 1/2 exactly for the causal mask
-    and 1 without one (the fixed formula); with a sliding window rho is the
-    exact fraction of valid (i, j) pairs."""
-    if w.window != (-1, -1) or w.segments:
+    and 1 without one (the fixed formula); with a sliding window, packed
+    sequences or a block-sparse mask rho is the exact fraction of valid (i, j)
+    pairs (for the block mask: the pairs of the visited blocks V, App.
+    "Extensions")."""
+    if w.window != (-1, -1) or w.segments or w.blocks:
         rho = synth.band_pairs(w) / float(w.N) ** 2
     else:
         rho = 0.5 if w.causal else 1.0
@@ -166,14 +168,15 @@ def oracle_sample(w, bits_head, target_s, seed=0):
     t0 = time.perf_counter()
     seg = list(w.segments) or None
     drop = w.dropout or None  # head 0 of batch entry 0: dropout counter head 0
+    bm = synth.workload_blocks(w)
     oracle.bob_head(*X, w.scale, w.causal, rows=rows_probe, cols=(0, w.N), window=w.window,
-                    segments=seg, dropout=drop, head=0)
+                    segments=seg, dropout=drop, head=0, block_mask=bm)
     dt = time.perf_counter() - t0
     n = int(max(16, min(w.N, 16 * target_s / max(dt, 1e-6))))
     rows = np.unique(np.linspace(0, w.N - 1, n).astype(np.int64))
     t0 = time.perf_counter()
     oracle.bob_head(*X, w.scale, w.causal, rows=rows, cols=(0, w.N), window=w.window,
-                    segments=seg, dropout=drop, head=0)
+                    segments=seg, dropout=drop, head=0, block_mask=bm)
     dt = time.perf_counter() - t0
     flops = 2.0 * 19 * valid_pairs_rows(w, rows) * w.d
     return flops, dt, f"{len(rows)} evenly spaced query rows of head 0 (of {w.N}), all key columns"
@@ -254,9 +257,11 @@ def run_gpu(args, w):
     segs = (torch.tensor(w.segments, dtype=torch.int32, device="cuda") if w.segments
             else None)  # packed-sequence offsets (kept alive for every call below)
     drop = w.dropout or None
-    o, lse = fbob.attn_fwd(q, k, v, w.scale, w.causal, w.window, segs, drop)
+    bm = synth.workload_blocks(w)  # block-sparse mask (kept alive for every call below)
+    bmk = torch.from_numpy(bm).cuda() if bm is not None else None
+    o, lse = fbob.attn_fwd(q, k, v, w.scale, w.causal, w.window, segs, drop, bmk)
     shp = fbob.make_shape(w.B, w.H, w.N, w.d, w.scale, w.causal, w.window, segs,
-                          kv_heads=w.kv_heads or None, dropout=drop)
+                          kv_heads=w.kv_heads or None, dropout=drop, block_mask=bmk)
     outs = [torch.empty_like(q), torch.empty_like(k), torch.empty_like(v), torch.empty_like(q)]
     rs = torch.empty((3, w.B, w.H, w.N), dtype=torch.float32, device="cuda")
     torch.cuda.synchronize()
@@ -384,10 +389,14 @@ def run_gpu(args, w):
                    "packed_sequences": len(w.segments) - 1 if w.segments else 1,
                    "kv_heads": w.kv_heads or w.H, "seed": w.seed,
                    "dropout": list(w.dropout) if w.dropout else None,
+                   "block_mask": ({"local": w.blocks[0], "sinks": w.blocks[1],
+                                   "density": w.blocks[2], "seed": w.blocks[3],
+                                   "blocks_set": int(bm.sum()), "blocks": int(bm.size)}
+                                  if bm is not None else None),
                    "l2": "no flush: inputs (%.2f GB) exceed the 129 MB L2" % (footprint / 1e9),
                    "parallelism": "replicas" if world > 1 else "single GPU",
                    "flop_formula": ("2*19*B*H*d*(valid (i,j) pairs of the band)"
-                                    if w.window != (-1, -1) or w.segments
+                                    if w.window != (-1, -1) or w.segments or w.blocks
                                     else "2*19*B*H*N^2*d*(1/2 if causal)")},
         "frac_of_bf16_peak": value / world / peak,
         "frac_of_bf16_sustained": value / world / peaks["bf16_sustained"],
@@ -428,9 +437,11 @@ def run_gpu_op(args, w):
     segs = (torch.tensor(w.segments, dtype=torch.int32, device="cuda") if w.segments
             else None)
     drop = w.dropout or None
+    bm = synth.workload_blocks(w)
+    bmk = torch.from_numpy(bm).cuda() if bm is not None else None
     shp = fbob.make_shape(w.B, w.H, w.N, w.d, w.scale, w.causal, w.window, segs,
-                          kv_heads=w.kv_heads or None, dropout=drop)
-    o, lse = fbob.attn_fwd(q, k, v, w.scale, w.causal, w.window, segs, drop)
+                          kv_heads=w.kv_heads or None, dropout=drop, block_mask=bmk)
+    o, lse = fbob.attn_fwd(q, k, v, w.scale, w.causal, w.window, segs, drop, bmk)
     dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
     dstat = torch.empty_like(lse)
     if args.op == "fwd":

@@ -39,6 +39,20 @@
  *             that break these rules give unspecified values but no access
  *             outside the caller's buffers.  NULL (with num_seqs 0) is one
  *             sequence.
+ *             block_mask (optional) is a block-sparse mask (App.
+ *             "Extensions": each row keeps a set of allowed columns and the
+ *             streamed loops visit only the block pairs with an allowed
+ *             entry): a device array of nb x nb bytes, nb = ceil(N / 128),
+ *             row-major over (query block, key block) of 128 x 128 entries,
+ *             the same for every (b, h).  Pair (i, j) is kept only if byte
+ *             (i / 128) * nb + j / 128 is nonzero (and the causal mask, the
+ *             window and the packed sequences keep it).  Every diagonal block
+ *             must be set, so that every row keeps its diagonal; the contents
+ *             are not checked on the host, and a mask that breaks the rule
+ *             gives unspecified values but no access outside the caller's
+ *             buffers.  It must not overlap any output.  Each CTA scans its
+ *             row (or column) of the mask, O(nb) bytes.  NULL keeps every
+ *             block.
  *  GQA        H_kv > 0 (a divisor of H) gives grouped-query attention: the
  *             key/value-side tensors (k, v, gk, gv and k_bar, v_bar, dk, dv)
  *             are [B, H_kv, N, d] and query head h reads key/value head
@@ -121,6 +135,7 @@ typedef struct fbob_shape {
     int64_t H_kv; /* key/value heads (grouped-query attention); 0 = H */
     double dropout_p;      /* attention dropout rate in [0, 1); 0 = none */
     uint64_t dropout_seed; /* Philox key of the dropout mask */
+    const uint8_t* block_mask; /* block-sparse mask: device uint8 [nb][nb], nb = ceil(N/128), or NULL */
 } fbob_shape;
 
 /*

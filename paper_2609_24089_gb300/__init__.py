@@ -36,7 +36,7 @@ class fbob_shape(ctypes.Structure):
                 ("window_left", ctypes.c_int32), ("window_right", ctypes.c_int32),
                 ("seq_offsets", ctypes.c_void_p), ("num_seqs", ctypes.c_int64),
                 ("H_kv", ctypes.c_int64), ("dropout_p", ctypes.c_double),
-                ("dropout_seed", ctypes.c_uint64)]
+                ("dropout_seed", ctypes.c_uint64), ("block_mask", ctypes.c_void_p)]
 
 
 _lib = None
@@ -88,14 +88,16 @@ def header_symbols() -> list:
 
 
 def make_shape(B, H, N, d, scale, causal, window=None, segments=None,
-               kv_heads=None, dropout=None) -> fbob_shape:
+               kv_heads=None, dropout=None, block_mask=None) -> fbob_shape:
     """window: (left, right) sliding-window band i - left <= j <= i + right;
     -1 (or None) leaves a side unbounded.  segments: contiguous int32 CUDA
     tensor of packed-sequence offsets [num_seqs + 1] (it must stay alive
     until the calls using this shape have run), or None for one sequence.
     kv_heads: key/value heads for grouped-query attention (None: H).
     dropout: (p, seed) attention dropout after the softmax (None: none); the
-    realised rate is round(256 p) / 256."""
+    realised rate is round(256 p) / 256.  block_mask: contiguous uint8 CUDA
+    tensor [nb, nb] (nb = ceil(N / 128)) of 128 x 128 query-key blocks to
+    keep, every diagonal block set (kept alive like segments), or None."""
     wl, wr = (-1, -1) if window is None else (int(window[0]), int(window[1]))
     if segments is None:
         seg, nseg = None, 0
@@ -107,8 +109,16 @@ def make_shape(B, H, N, d, scale, causal, window=None, segments=None,
         seg, nseg = segments.data_ptr(), segments.numel() - 1
     hkv = 0 if kv_heads is None or int(kv_heads) == int(H) else int(kv_heads)
     dp, seed = (0.0, 0) if dropout is None else (float(dropout[0]), int(dropout[1]))
+    bm = None
+    if block_mask is not None:
+        import torch
+        nb = (int(N) + 127) // 128
+        if (not block_mask.is_cuda or block_mask.dtype != torch.uint8
+                or tuple(block_mask.shape) != (nb, nb) or not block_mask.is_contiguous()):
+            raise ValueError(f"block_mask must be a contiguous [{nb}, {nb}] uint8 CUDA tensor")
+        bm = block_mask.data_ptr()
     return fbob_shape(int(B), int(H), int(N), int(d), float(scale), int(causal), wl, wr,
-                      seg, nseg, hkv, dp, seed & 0xFFFFFFFFFFFFFFFF)
+                      seg, nseg, hkv, dp, seed & 0xFFFFFFFFFFFFFFFF, bm)
 
 
 def _ptr(t):
@@ -133,10 +143,10 @@ def _check(rc, where):
         raise FbobError(rc, where)
 
 
-def _shape_of(q, k, scale, causal, window=None, segments=None, dropout=None):
+def _shape_of(q, k, scale, causal, window=None, segments=None, dropout=None, block_mask=None):
     B, H, N, d = q.shape
     return make_shape(B, H, N, d, scale, causal, window, segments, kv_heads=k.shape[1],
-                      dropout=dropout)
+                      dropout=dropout, block_mask=block_mask)
 
 
 # ------------------------------------------------ entry points, same names as the C ABI
@@ -223,32 +233,35 @@ def fbob_launch_count(entry: str) -> int:
 
 
 # ------------------------------------------------ allocating helpers
-def attn_fwd(q, k, v, scale, causal, window=None, segments=None, dropout=None):
+def attn_fwd(q, k, v, scale, causal, window=None, segments=None, dropout=None,
+             block_mask=None):
     import torch
     B, H, N, d = q.shape
     o = torch.empty_like(q)
     lse = torch.empty((B, H, N), dtype=torch.float32, device=q.device)
-    fbob_attn_fwd(_shape_of(q, k, scale, causal, window, segments, dropout), q, k, v, o, lse)
+    fbob_attn_fwd(_shape_of(q, k, scale, causal, window, segments, dropout, block_mask),
+                  q, k, v, o, lse)
     return o, lse
 
 
-def attn_bwd(q, k, v, o, lse, dout, scale, causal, window=None, segments=None, dropout=None):
+def attn_bwd(q, k, v, o, lse, dout, scale, causal, window=None, segments=None, dropout=None,
+             block_mask=None):
     import torch
     B, H, N, d = q.shape
     dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
     dstat = torch.empty((B, H, N), dtype=torch.float32, device=q.device)
-    fbob_attn_bwd(_shape_of(q, k, scale, causal, window, segments, dropout), q, k, v, o, lse,
-                  dout, dq, dk, dv, dstat)
+    fbob_attn_bwd(_shape_of(q, k, scale, causal, window, segments, dropout, block_mask),
+                  q, k, v, o, lse, dout, dq, dk, dv, dstat)
     return dq, dk, dv, dstat
 
 
 def attn_bob(q, k, v, o, lse, dout, gq, gk, gv, scale, causal, window=None, segments=None,
-             dropout=None):
+             dropout=None, block_mask=None):
     """Returns (q_bar, k_bar, v_bar, dout_bar, row_stats[3,B,H,N] = alpha, E, D)."""
     import torch
     B, H, N, d = q.shape
     outs = [torch.empty_like(q), torch.empty_like(k), torch.empty_like(v), torch.empty_like(q)]
     row_stats = torch.empty((3, B, H, N), dtype=torch.float32, device=q.device)
-    fbob_attn_bob(_shape_of(q, k, scale, causal, window, segments, dropout), q, k, v, o, lse,
-                  dout, gq, gk, gv, *outs, row_stats)
+    fbob_attn_bob(_shape_of(q, k, scale, causal, window, segments, dropout, block_mask),
+                  q, k, v, o, lse, dout, gq, gk, gv, *outs, row_stats)
     return (*outs, row_stats)

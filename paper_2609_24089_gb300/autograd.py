@@ -33,12 +33,13 @@ class _AttnBwd(torch.autograd.Function):
     """(q, k, v, dout) -> (dq, dk, dv); its backward is BoB."""
 
     @staticmethod
-    def forward(ctx, q, k, v, o, lse, dout, scale, causal, window, segments, dropout):
+    def forward(ctx, q, k, v, o, lse, dout, scale, causal, window, segments, dropout, blocks):
         dout = _bf16(dout)
-        dq, dk, dv, _ = attn_bwd(q, k, v, o, lse, dout, scale, causal, window, segments, dropout)
+        dq, dk, dv, _ = attn_bwd(q, k, v, o, lse, dout, scale, causal, window, segments, dropout,
+                                 blocks)
         ctx.save_for_backward(q, k, v, o, lse, dout)
         ctx.scale, ctx.causal, ctx.window, ctx.segments = scale, causal, window, segments
-        ctx.dropout = dropout
+        ctx.dropout, ctx.blocks = dropout, blocks
         return dq, dk, dv
 
     @staticmethod
@@ -48,42 +49,45 @@ class _AttnBwd(torch.autograd.Function):
              for t, x in zip((gq, gk, gv), (q, k, v))]
         q_bar, k_bar, v_bar, dout_bar, _ = attn_bob(q, k, v, o, lse, dout, *g, ctx.scale,
                                                     ctx.causal, ctx.window, ctx.segments,
-                                                    ctx.dropout)
-        return q_bar, k_bar, v_bar, None, None, dout_bar, None, None, None, None, None
+                                                    ctx.dropout, ctx.blocks)
+        return q_bar, k_bar, v_bar, None, None, dout_bar, None, None, None, None, None, None
 
 
 class _Attn(torch.autograd.Function):
     """(q, k, v) -> O = softmax(scale Q K^T + M) V (eq. 1)."""
 
     @staticmethod
-    def forward(ctx, q, k, v, scale, causal, window, segments, dropout):
-        o, lse = attn_fwd(q, k, v, scale, causal, window, segments, dropout)
+    def forward(ctx, q, k, v, scale, causal, window, segments, dropout, blocks):
+        o, lse = attn_fwd(q, k, v, scale, causal, window, segments, dropout, blocks)
         ctx.save_for_backward(q, k, v, o, lse)
         ctx.scale, ctx.causal, ctx.window, ctx.segments = scale, causal, window, segments
-        ctx.dropout = dropout
+        ctx.dropout, ctx.blocks = dropout, blocks
         return o
 
     @staticmethod
     def backward(ctx, dout):
         q, k, v, o, lse = ctx.saved_tensors
         dq, dk, dv = _AttnBwd.apply(q, k, v, o.detach(), lse, dout, ctx.scale, ctx.causal,
-                                    ctx.window, ctx.segments, ctx.dropout)
-        return dq, dk, dv, None, None, None, None, None
+                                    ctx.window, ctx.segments, ctx.dropout, ctx.blocks)
+        return dq, dk, dv, None, None, None, None, None, None
 
 
 def attention(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, scale: float | None = None,
               causal: bool = False, window: tuple | None = None,
               segments: torch.Tensor | None = None, dropout_p: float = 0.0,
-              seed: int = 0) -> torch.Tensor:
+              seed: int = 0, block_mask: torch.Tensor | None = None) -> torch.Tensor:
     """Softmax attention on libfbob, differentiable twice (see the module doc).
     window: (left, right) sliding-window band, -1 = unbounded side; segments:
     int32 CUDA offsets of packed variable-length sequences; dropout_p, seed:
     attention dropout after the softmax with a keep mask regenerated from the
-    seed in every kernel (the same mask in the forward and both backwards)."""
+    seed in every kernel (the same mask in the forward and both backwards);
+    block_mask: uint8 CUDA [ceil(N/128)]^2 block-sparse mask of 128 x 128
+    (query block, key block) tiles, every diagonal block set."""
     for t in (q, k, v):
         _check(t)
     if scale is None:
         scale = 1.0 / math.sqrt(q.shape[-1])
     dropout = (float(dropout_p), int(seed)) if dropout_p else None
     return _Attn.apply(q.contiguous(), k.contiguous(), v.contiguous(), float(scale),
-                       bool(causal), None if window is None else tuple(window), segments, dropout)
+                       bool(causal), None if window is None else tuple(window), segments, dropout,
+                       block_mask)

@@ -136,6 +136,36 @@ __device__ __forceinline__ void seq_bounds(const EngineParams& p, int i, int& lo
   hi = min(p.N, max(p.seq_off[a + 1], i + 1));
 }
 
+// Streamed tiles of one CTA under a block-sparse mask (App. "Extensions":
+// the streamed loop visits only the block pairs with an unmasked entry).
+// Tiles of BN = 64 rows lie in 128-row mask blocks; tile t is visited if the
+// mask entry of its block (t / 2) is set.  mb points at the stationary
+// block's entry for streamed block 0 and stride steps to the next streamed
+// block (1 along a mask row, nbm down a column); mb == nullptr visits every
+// tile of the band t0 .. t1.
+struct TileSet {
+  const uint8_t* mb;
+  int stride;
+  int t0, t1;
+  __device__ __forceinline__ bool set(int t) const {
+    return mb == nullptr || mb[(size_t)(t >> 1) * stride] != 0;
+  }
+  // number of visited tiles
+  __device__ int count() const {
+    if (mb == nullptr) return t1 - t0 + 1;
+    int n = 0;
+    for (int b = t0 >> 1; b <= (t1 >> 1); ++b)
+      if (mb[(size_t)b * stride] != 0) n += min(2 * b + 1, t1) - max(2 * b, t0) + 1;
+    return n;
+  }
+  // first visited tile >= t (t1 + 1 if there is none)
+  __device__ __forceinline__ int next(int t) const {
+    if (mb == nullptr) return t;
+    while (t <= t1 && mb[(size_t)(t >> 1) * stride] == 0) t = (t | 1) + 1;
+    return t;
+  }
+};
+
 __device__ __forceinline__ float bits_f(uint32_t u) { return __uint_as_float(u); }
 __device__ __forceinline__ float2 pair(const uint32_t (&r)[16], int c) {
   return make_float2(__uint_as_float(r[c]), __uint_as_float(r[c + 1]));
@@ -250,8 +280,10 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
   const int key_lo = max(seq_lo0, p.wl < 0 ? 0 : i0 - p.wl);
   const int key_hi = min(seq_hi1, p.wr < 0 ? N : last_row + p.wr + 1);  // exclusive
   const int first_tile = key_lo / BN;
-  const int ntiles = (key_hi - 1) / BN - first_tile + 1;
-  const int nsteps = ntiles;
+  // (with a block-sparse mask only the tiles of this row block's set blocks)
+  const TileSet tiles = {p.bmask ? p.bmask + (size_t)rb * p.nbm : nullptr, 1, first_tile,
+                         (key_hi - 1) / BN};
+  const int nsteps = tiles.count();
 
   if (tid == 0) {
     m->wctl.abort = 0;
@@ -301,12 +333,14 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
           tma_load_3d(s_stat + ((C::STAT_TMEM ? 0 : t) * C::KB + b) * (BM * 128), &p.tm[t],
                       &m->bar_stat, 64 * b, i0, bh);
       int issued[kMaxStages] = {-1, -1, -1, -1};
+      int tile = first_tile - 1;
       for (int st = 0; st < nsteps; ++st) {
         const int stage = st % C::NSTAGES;
         if (st >= C::NSTAGES) {
           if (!mbar_wait(&m->bar_empty[stage], ((st / C::NSTAGES) - 1) & 1, wctl)) break;
         }
-        const int j0 = (first_tile + st) * BN;
+        tile = tiles.next(tile + 1);
+        const int j0 = tile * BN;
         const int nt = C::NSTREAM;
         uint8_t* dst = s_stream + stage * C::STAGE_BYTES;
         // BoB: K and U_K first on bar_full (all issuer X needs), then V and
@@ -457,7 +491,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
           }
           ok = false;
         }
-        ok = ok && mbar_wait(&m->bar_full[0], 0, wctl);
+        ok = ok && nsteps > 0 && mbar_wait(&m->bar_full[0], 0, wctl);
         if (ok) {
           tc_fence_after();
           stage_sf(0, kColSF);
@@ -529,7 +563,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
           return mbar_wait(&m->bar_full[stg], par, wctl) &&
                  (!kB4 || mbar_wait(&m->bar_full_b[stg], par, wctl));
         };
-        bool ok = mbar_wait(&m->bar_stat, 0, wctl) && wait_stage(0, 0);
+        bool ok = mbar_wait(&m->bar_stat, 0, wctl) && nsteps > 0 && wait_stage(0, 0);
         if constexpr (kStats) {
           // DC(t+1) once the elementwise warps hold DC(t) in registers
           if (ok) {
@@ -703,12 +737,15 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
     }
     float2 acc_a = splat(0.f), acc_e = splat(0.f);  // Pass 1 partial row sums
     bool ok = true;
+    int tile = first_tile - 1;
     for (int st = 0; ok && st < nsteps; ++st) {
+      tile = tiles.next(tile + 1);
+      const int jt = tile * BN;  // first key of the tile
       // SF buffer of this tile (the statistics kernel alternates two)
       const int sfb = kStats ? (st & 1) : 0;
       const uint32_t sfcol = sfb ? kColSF1 : kColSF;
       uint32_t kb[2];
-      if constexpr (DROP) tile_keep((first_tile + st % ntiles) * BN, kb);
+      if constexpr (DROP) tile_keep(jt, kb);
       if (!ew_wait(&m->bar_sa_sf[sfb], kStats ? ((st >> 1) & 1) : (st & 1))) {
         ok = false;
         break;
@@ -729,7 +766,6 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
       }
       tc_fence_before();
       mbar_arrive(&m->bar_sf_free[sfb]);
-      const int jt = (first_tile + st % ntiles) * BN;
       const float2 sl2v = splat(sl2), nL2v = splat(-L2);
       if constexpr (kStats) {
         // ---- row statistics: copy DC of the whole tile, release it, then
@@ -1023,7 +1059,10 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
   const int q_lo = max(seq_lo0, p.wr < 0 ? 0 : j0 - p.wr);
   const int q_hi = min(seq_hi1, p.wl < 0 ? N : last_key + p.wl + 1);  // exclusive
   const int first_tile = q_lo / BN;
-  const int nsteps_h = (q_hi - 1) / BN - first_tile + 1;  // query tiles per query head
+  // query tiles per query head (with a block-sparse mask only the tiles of
+  // the query blocks set in this key block's mask column)
+  const TileSet tiles = {p.bmask ? p.bmask + cb : nullptr, p.nbm, first_tile, (q_hi - 1) / BN};
+  const int nsteps_h = tiles.count();
   // grouped-query attention: this key/value head's G query heads are streamed
   // one after the other (their sums accumulate in this CTA, in a fixed order)
   const int G = p.H / p.Hkv;
@@ -1076,12 +1115,15 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
                       bh);
     }
     int issued[kMaxStages] = {-1, -1, -1, -1};
+    int tile = first_tile - 1;
     for (int st = 0; st < nprod; ++st) {
       const int stage = st % C::NSTAGES;
       if (st >= C::NSTAGES) {
         if (!mbar_wait(&m->bar_empty[stage], ((st / C::NSTAGES) - 1) & 1, wctl)) break;
       }
-      const int ib = (first_tile + st % nsteps_h) * BN;
+      if (st % nsteps_h == 0) tile = first_tile - 1;  // next query head: from the start
+      tile = tiles.next(tile + 1);
+      const int ib = tile * BN;
       const int bhq = bh_q0 + st / nsteps_h;  // query head of this step
       uint8_t* dst = s_stream + stage * C::STAGE_BYTES;
       if (lane == 0) {
@@ -1187,7 +1229,8 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
               mma_ss(R + 0, sd(0, k), kd(kd0, 0, k), id_n64, k > 0);
           }
         };
-        bool ok = mbar_wait(&m->bar_stat, 0, wctl) && mbar_wait(&m->bar_full[0], 0, wctl);
+        bool ok = mbar_wait(&m->bar_stat, 0, wctl) && nsteps > 0 &&
+                  mbar_wait(&m->bar_full[0], 0, wctl);
         if (ok) {
           tc_fence_after();
           stage_sf(0);
@@ -1316,11 +1359,14 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
       return w;
     };
     bool ok = true;
+    int tile = first_tile - 1;
     for (int st = 0; ok && st < nsteps; ++st) {
       const int stage = st % C::NSTAGES;
+      if (st % nsteps_h == 0) tile = first_tile - 1;  // next query head: from the start
+      tile = tiles.next(tile + 1);
+      const int it = tile * BN;  // first query row of the tile
       uint32_t kb[2];
       if constexpr (DROP) {
-        const int it = (first_tile + st % nsteps_h) * BN;
         const uint32_t bhq = (uint32_t)(p.head0 + bh_q0 + st / nsteps_h);
 #pragma unroll
         for (int h = 0; h < 2; ++h) kb[h] = keep_col16(gj, it + HB * h + 16 * wg, bhq, dkey);
@@ -1357,8 +1403,8 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
       const uint32_t dcol = dc_col(st);
 #pragma unroll
       for (int h = 0; h < 2; ++h) {
-        const int cv = HB * h + 16 * wg;             // tile column of this thread's first
-        const int ib = (first_tile + st % nsteps_h) * BN + cv;  // first query row of this thread's 16
+        const int cv = HB * h + 16 * wg;  // tile column of this thread's first
+        const int ib = it + cv;           // first query row of this thread's 16
         // valid query columns c satisfy  lo <= c < hi
         const int lo = qlo - ib, hi = qhi - ib;
         if (lo > 0 || hi < 16) mask16(rS[h], lo, hi);

@@ -52,6 +52,10 @@ struct EngineParams {
   int wl, wr;  // valid band of row i: i - wl <= j <= i + wr (-1: unbounded); causal gives wr = 0
   const int* seq_off;  // packed sequences: offsets [nseq + 1], or nullptr for one sequence
   int nseq;
+  // block-sparse mask: [nbm][nbm] bytes over 128 x 128 blocks (query block,
+  // key block), or nullptr; nbm = ceil(N / 128)
+  const uint8_t* bmask;
+  int nbm;
   int H, Hkv;  // query and key/value heads per batch entry (grouped-query attention)
   float scale;
   long long bhn;  // BH * N (row_stats plane stride)

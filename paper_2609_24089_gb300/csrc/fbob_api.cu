@@ -136,6 +136,8 @@ void choose_order(EngineParams* p, int head_major) { p->head_major = head_major;
 // key/value heads per batch entry
 int64_t kv_heads(const fbob_shape* s) { return s->H_kv > 0 ? s->H_kv : s->H; }
 
+int n_blocks(int64_t N, int rows) { return (int)((N + rows - 1) / rows); }
+
 // dropout byte threshold t = round(256 p), at most 255; 0 = no dropout
 uint32_t drop_threshold(const fbob_shape* s) {
   const double t = std::floor(256.0 * s->dropout_p + 0.5);
@@ -154,6 +156,8 @@ EngineParams base_params(const fbob_shape* s) {
   p.wr = s->causal ? 0 : s->window_right;
   p.seq_off = s->seq_offsets;
   p.nseq = (int)s->num_seqs;
+  p.bmask = s->block_mask;
+  p.nbm = n_blocks(s->N, BM);
   p.H = (int)s->H;
   p.Hkv = (int)kv_heads(s);
   p.scale = s->scale;
@@ -173,8 +177,6 @@ EngineParams base_params(const fbob_shape* s) {
   debug_controls(&p);
   return p;
 }
-
-int n_blocks(int64_t N, int rows) { return (int)((N + rows - 1) / rows); }
 
 int launch_status(cudaError_t e) { return e == cudaSuccess ? FBOB_OK : FBOB_ERR_CUDA; }
 

@@ -135,8 +135,25 @@ __global__ void __launch_bounds__(kFwdThreads, 1) fwd_engine(const __grid_consta
   }
   const int T0 = act[1] ? min(tq0[0], tq0[1]) : tq0[0];
   const int T1 = act[1] ? max(tq1[0], tq1[1]) : tq1[0];
-  const int nsteps = T1 - T0 + 1;
-  auto part = [&](int q, int T) { return act[q] && T >= tq0[q] && T <= tq1[q]; };
+  // block-sparse mask (128 x 128 blocks: a key tile is one key block, query
+  // tile q is query block 2 rb + q): query tile q takes key tile T only if
+  // that block pair is set, and a key tile neither takes is not streamed
+  const uint8_t* bm = p.bmask;
+  auto part = [&](int q, int T) {
+    return act[q] && T >= tq0[q] && T <= tq1[q] &&
+           (bm == nullptr || bm[(size_t)(2 * rb + q) * p.nbm + T] != 0);
+  };
+  // next streamed key tile >= T (T1 + 1 if none)
+  auto next_T = [&](int T) {
+    if (bm != nullptr)
+      while (T <= T1 && !part(0, T) && !part(1, T)) ++T;
+    return T;
+  };
+  int nsteps = T1 - T0 + 1;
+  if (bm != nullptr) {
+    nsteps = 0;
+    for (int T = T0; T <= T1; ++T) nsteps += (part(0, T) || part(1, T)) ? 1 : 0;
+  }
 
   if (tid == 0) {
     m->wctl.abort = 0;
@@ -178,12 +195,14 @@ __global__ void __launch_bounds__(kFwdThreads, 1) fwd_engine(const __grid_consta
           tma_load_3d(s_stat + (q * C::KB + b) * (BM * 128), &p.tm[0], &m->bar_stat, 64 * b,
                       i0 + BM * q, bh);
       int issued[kMaxStages] = {-1, -1, -1, -1};
+      int T = T0 - 1;
       for (int st = 0; st < nsteps; ++st) {
         const int stage = st % C::NSTAGES;
         if (st >= C::NSTAGES &&
             !mbar_wait(&m->empty[stage], ((st / C::NSTAGES) - 1) & 1, wctl))
           break;
-        const int j0 = (T0 + st) * BN2;
+        T = next_T(T + 1);
+        const int j0 = T * BN2;
         uint8_t* dst = s_stream + stage * C::STAGE_BYTES;
         mbar_arrive_expect_tx(&m->full[stage], C::STAGE_BYTES);
         for (int t = 0; t < 2; ++t)        // K, V
@@ -209,15 +228,16 @@ __global__ void __launch_bounds__(kFwdThreads, 1) fwd_engine(const __grid_consta
         // ---------------- issuer X: S_q(T) = Q_q K(T)^T
         const uint64_t qd0 = sdesc_sw128(smem_u32(s_stat), 16, 1024);
         ok = mbar_wait(&m->bar_stat, 0, wctl);
+        int T = T0 - 1, kq[2] = {0, 0};  // key tile; tiles each query tile has taken
         for (int st = 0; ok && st < nsteps; ++st) {
-          const int T = T0 + st;
+          T = next_T(T + 1);
           const int stage = st % C::NSTAGES;
           if (!mbar_wait(&m->full[stage], (st / C::NSTAGES) & 1, wctl)) break;
           const uint64_t kd0 =
               sdesc_sw128(smem_u32(s_stream + stage * C::STAGE_BYTES), 16, 1024);
           for (int q = 0; q < 2 && ok; ++q) {
             if (!part(q, T)) continue;
-            const int k = T - tq0[q];
+            const int k = kq[q]++;
             if (k >= 1) {
               // SEP_P: S_q(T) overwrites S_q(T-1): wait until both softmax
               // halves hold it (their row-maximum exchange of tile T-1);
@@ -245,8 +265,9 @@ __global__ void __launch_bounds__(kFwdThreads, 1) fwd_engine(const __grid_consta
         }
       } else {
         // ---------------- issuer Y: O_q += P_q(T) V(T)
+        int T = T0 - 1, kq[2] = {0, 0};
         for (int st = 0; ok && st < nsteps; ++st) {
-          const int T = T0 + st;
+          T = next_T(T + 1);
           const int stage = st % C::NSTAGES;
           if (!mbar_wait(&m->full[stage], (st / C::NSTAGES) & 1, wctl)) break;
           // V of this stage: MN-major, 64-wide boxes BN2 * 128 bytes apart
@@ -254,7 +275,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1) fwd_engine(const __grid_consta
               smem_u32(s_stream + stage * C::STAGE_BYTES) + C::KB * (BN2 * 128), BN2 * 128, 1024);
           for (int q = 0; q < 2 && ok; ++q) {
             if (!part(q, T)) continue;
-            const int k = T - tq0[q];
+            const int k = kq[q]++;
             if (!mbar_wait(&m->p_full[q], k & 1, wctl)) {
               ok = false;
               break;
@@ -298,9 +319,21 @@ __global__ void __launch_bounds__(kFwdThreads, 1) fwd_engine(const __grid_consta
     };
     float mrow = -INFINITY, lrow = 0.f;  // (lrow: this half's keys)
     bool ok = act[q];
-    const int nq = act[q] ? tq1[q] - tq0[q] + 1 : 0;
+    // key tiles this query tile takes (with a block-sparse mask, those of its
+    // set blocks)
+    int nq = act[q] ? tq1[q] - tq0[q] + 1 : 0;
+    if (bm != nullptr && act[q]) {
+      nq = 0;
+      for (int T = tq0[q]; T <= tq1[q]; ++T) nq += part(q, T) ? 1 : 0;
+    }
+    int Tq = tq0[q] - 1;
     for (int k = 0; ok && k < nq; ++k) {
-      const int jt = (tq0[q] + k) * BN2 + 64 * hf;  // first key of this half
+      ++Tq;
+      if (p.bmask != nullptr) {  // the next set block of this query block (gi / 128)
+        const uint8_t* bq = p.bmask + (size_t)(gi >> 7) * p.nbm;
+        while (Tq < p.nbm - 1 && bq[Tq] == 0) ++Tq;
+      }
+      const int jt = Tq * BN2 + 64 * hf;  // first key of this half
       // dropout keep bits of the half's 4 x 16 keys, formed while S_q(T) is computed
       uint32_t kb[4];
       if constexpr (DROP) {

@@ -37,6 +37,7 @@ class Workload:
     segments: tuple = ()      # offsets of packed sequences along N; () = one sequence
     kv_heads: int = 0         # key/value heads (grouped-query attention); 0 = H
     dropout: tuple = ()       # attention dropout (p, seed); () = none
+    blocks: tuple = ()        # block-sparse mask (local, sinks, density, seed); () = none
 
     @property
     def scale(self) -> float:
@@ -98,9 +99,39 @@ for _d in (32, 64, 128):
     WORKLOADS[f"n4k_d{_d}_causal_b4h12"] = Workload(
         f"n4k_d{_d}_causal_b4h12", 4, 12, 4096, _d, True, 9, _s(1, 1, 1, 1, 1, 1, 1))
 
+# block-sparse variant of n16k_d128_causal (App. "Extensions"): each query
+# block keeps its own and the 2 previous key blocks, the first key block, and
+# random blocks with probability 0.1 (about a quarter of the causal blocks)
+WORKLOADS["n16k_d128_causal_bsparse"] = Workload(
+    "n16k_d128_causal_bsparse", 2, 16, 16384, 128, True, 10,
+    _s(1, 1, 1, *(4 * [1 / math.sqrt(128)])), blocks=(2, 1, 0.1, 10))
+
 WORKLOADS["n16k_d128_causal_varlen"] = Workload(
     "n16k_d128_causal_varlen", 2, 16, 16384, 128, True, 6,
     _s(1, 1, 1, *(4 * [1 / math.sqrt(128)])), segments=packed_offsets(16384, 12, 6))
+
+
+def block_pattern(N: int, local: int, sinks: int, density: float, seed: int,
+                  block: int = 128) -> np.ndarray:
+    """[nb, nb] uint8 block-sparse mask over block x block tiles (nb =
+    ceil(N / block)): query block b keeps key blocks b - local .. b (its own
+    and `local` before it), the first `sinks` key blocks, and every other key
+    block with probability `density` (seeded); the diagonal is always set."""
+    nb = (N + block - 1) // block
+    rng = np.random.Generator(np.random.PCG64(seed))
+    bm = (rng.random((nb, nb)) < density)
+    b = np.arange(nb)
+    bm |= (b[None, :] <= b[:, None]) & (b[None, :] >= b[:, None] - local)
+    bm[:, :sinks] = True
+    return bm.astype(np.uint8)
+
+
+def workload_blocks(w: Workload):
+    """The workload's block mask ([nb, nb] uint8, 128 x 128 blocks), or None."""
+    if not w.blocks:
+        return None
+    local, sinks, density, seed = w.blocks
+    return block_pattern(w.N, int(local), int(sinks), float(density), int(seed))
 
 
 def band_pairs(w: Workload, rows=None) -> float:
@@ -117,7 +148,17 @@ def band_pairs(w: Workload, rows=None) -> float:
         s = np.searchsorted(seg[1:], r, side="right")
         lo = np.maximum(lo, seg[s])
         hi = np.minimum(hi, seg[s + 1])
-    return float(np.sum(hi - lo))
+    bm = workload_blocks(w)
+    if bm is None:
+        return float(np.sum(hi - lo))
+    # with a block mask: the part of each row's [lo, hi) inside its set blocks
+    total = 0.0
+    for kb in range(bm.shape[1]):
+        keep = bm[r // 128, kb] != 0
+        a = np.maximum(lo, kb * 128)
+        b = np.minimum(hi, min(w.N, (kb + 1) * 128))
+        total += float(np.sum(np.where(keep, np.maximum(b - a, 0), 0)))
+    return total
 
 
 def bf16_bits(x: np.ndarray) -> np.ndarray:

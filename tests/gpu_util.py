@@ -72,10 +72,10 @@ def f64(bits):
     return synth.to_f64(bits)
 
 
-def oracle_o_l(bits, scale, causal, window=None, segments=None, dropout=None):
+def oracle_o_l(bits, scale, causal, window=None, segments=None, dropout=None, block_mask=None):
     """O rounded to bf16 and L rounded to fp32, from the oracle's forward."""
     O, L = oracle.fwd(f64(bits["q"]), f64(bits["k"]), f64(bits["v"]), scale, causal,
-                      window=window, segments=segments, dropout=dropout)
+                      window=window, segments=segments, dropout=dropout, block_mask=block_mask)
     return synth.bf16_bits(O.astype(np.float32)), L.astype(np.float32)
 
 
@@ -87,18 +87,28 @@ def dev_segments(segments):
     return t.tensor(np.asarray(segments, dtype=np.int32), device="cuda")
 
 
-def run_bob(bits, scale, causal, o_l=None, window=None, segments=None, dropout=None):
+def dev_blocks(block_mask):
+    """Block mask as the uint8 CUDA tensor the library reads."""
+    if block_mask is None:
+        return None
+    t = torch()
+    return t.tensor(np.asarray(block_mask, dtype=np.uint8), device="cuda")
+
+
+def run_bob(bits, scale, causal, o_l=None, window=None, segments=None, dropout=None,
+            block_mask=None):
     """Upload, (forward unless o_l is given), then backward-over-backward.
     Returns dict of host float64 arrays and the device status."""
     t = torch()
     q, k, v, do, gq, gk, gv = (dev(bits[n]) for n in synth.NAMES)
     seg = dev_segments(segments)
+    bmk = dev_blocks(block_mask)
     if o_l is None:
-        o, lse = fbob.attn_fwd(q, k, v, scale, causal, window, seg, dropout)
+        o, lse = fbob.attn_fwd(q, k, v, scale, causal, window, seg, dropout, bmk)
     else:
         o, lse = dev(o_l[0]), dev_f32(o_l[1])
     qb, kb, vb, dob, rs = fbob.attn_bob(q, k, v, o, lse, do, gq, gk, gv, scale, causal, window,
-                                        seg, dropout)
+                                        seg, dropout, bmk)
     status = fbob.fbob_device_status()
     t.cuda.synchronize()
     return {"qbar": host(qb), "kbar": host(kb), "vbar": host(vb), "dobar": host(dob),
@@ -109,7 +119,7 @@ def run_bob(bits, scale, causal, o_l=None, window=None, segments=None, dropout=N
 
 
 def oracle_bob_heads(bits, scale, causal, heads, rows=None, cols=None, window=None,
-                     segments=None, dropout=None):
+                     segments=None, dropout=None, block_mask=None):
     """Oracle on selected flat heads of a [B,H,N,d] bit tensor set (the
     key/value side of a grouped-query set is read from head h // G)."""
     B, H, N, d = bits["q"].shape
@@ -119,7 +129,8 @@ def oracle_bob_heads(bits, scale, causal, heads, rows=None, cols=None, window=No
         b, h = divmod(hh, H)
         X = [f64(bits[n][b, h // G if n in ("k", "v", "gk", "gv") else h]) for n in synth.NAMES]
         out.append(oracle.bob_head(*X, scale, causal, rows=rows, cols=cols, window=window,
-                                   segments=segments, dropout=dropout, head=hh))
+                                   segments=segments, dropout=dropout, head=hh,
+                                   block_mask=block_mask))
     return out
 
 
