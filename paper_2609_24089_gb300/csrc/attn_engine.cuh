@@ -500,6 +500,10 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         for (int st = 0; ok && st < nsteps; ++st) {
           const int stage = st % C::NSTAGES;
           const bool more = st + 1 < nsteps;
+          // without XSHARE, X's last read of this stage was SF(t), already
+          // issued: release the stage when that completes (a commit after
+          // SF(t+1) would hold it until SF(t+1) completes, a tile later)
+          if (!C::XSHARE) mma_commit(&m->bar_empty[stage]);
           if (more) {  // SF(t+1) once the elementwise warps hold SF(t)
             if (!mbar_wait(&m->bar_sf_free[0], st & 1, wctl) ||
                 !mbar_wait(&m->bar_full[(st + 1) % C::NSTAGES], ((st + 1) / C::NSTAGES) & 1, wctl))
@@ -531,8 +535,8 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
               }
             }
             if (!ok) break;
+            mma_commit(&m->bar_empty[stage]);
           }
-          mma_commit(&m->bar_empty[stage]);
         }
         mma_commit(&m->bar_acc);
         if (*abort_flag) drain_wait(&m->bar_acc, 0);
@@ -1229,6 +1233,18 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
               mma_ss(R + 0, sd(0, k), kd(kd0, 0, k), id_n64, k > 0);
           }
         };
+        // with C::PH_SF: Vtil(t) += (P o h)^T dO from the operand tile the
+        // elementwise warps wrote into SF (K-step s at SF column 16 s)
+        auto stage_vt = [&](uint32_t sb, int st) {
+          constexpr uint32_t kBoxBytes = C::NSTREAM * BN * 128;
+          const uint64_t md0 = sdesc_sw128(sb, kBoxBytes, 1024);
+#pragma unroll
+          for (int s = 0; s < 4; ++s) {
+            const uint64_t md =
+                md0 + (uint64_t)((soff<C::NSTREAM, false>(2, s >> 1, 0) + (s & 1) * 2048) >> 4);
+            mma_ts(tmem + D, tmem + kColSF + 16 * s, md, id_b, (st == 0 && s == 0) ? 0u : 1u);
+          }
+        };
         bool ok = mbar_wait(&m->bar_stat, 0, wctl) && nsteps > 0 &&
                   mbar_wait(&m->bar_full[0], 0, wctl);
         if (ok) {
@@ -1238,6 +1254,30 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
         }
         for (int st = 0; ok && st < nsteps; ++st) {
           const int stage = st % C::NSTAGES;
+          if constexpr (C::PH_SF) {
+            // the elementwise warps hold SF(t) in registers and have written
+            // P o h over it: Vtil(t), then SF(t+1) (in issue order, so SF(t+1)
+            // overwrites the operand tile only after Vtil(t) has read it)
+            if (!mbar_wait(&m->bar_sf_free[0], st & 1, wctl) ||
+                !mbar_wait(&m->bar_full_b[stage], (st / C::NSTAGES) & 1, wctl))
+              break;
+            tc_fence_after();
+            stage_vt(smem_u32(s_stream + stage * C::STAGE_BYTES), st);
+            // X's last read of this stage: release it once Vtil(t) has read it
+            mma_commit(&m->bar_empty[stage]);
+            if (st + 1 < nsteps) {
+              if (!mbar_wait(&m->bar_full[(st + 1) % C::NSTAGES], ((st + 1) / C::NSTAGES) & 1,
+                             wctl))
+                break;
+              tc_fence_after();
+              stage_sf(st + 1);
+              mma_commit(&m->bar_sa_sf[0]);
+            }
+            continue;
+          }
+          // without XSHARE, X's last read of this stage was SF(t): release it
+          // when that completes, not after SF(t+1) as well
+          if (!C::XSHARE) mma_commit(&m->bar_empty[stage]);
           if (st + 1 < nsteps) {  // SF(t+1) once the elementwise warps hold SF(t)
             if (!mbar_wait(&m->bar_sf_free[0], st & 1, wctl) ||
                 !mbar_wait(&m->bar_full[(st + 1) % C::NSTAGES], ((st + 1) / C::NSTAGES) & 1, wctl))
@@ -1261,8 +1301,8 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
             }
             if (!ok) break;
             mma_commit(&m->bar_xb[dc_sel(st)]);
+            mma_commit(&m->bar_empty[stage]);
           }
-          mma_commit(&m->bar_empty[stage]);
         }
         mma_commit(&m->bar_acc);
         if (*abort_flag) drain_wait(&m->bar_acc, 0);
@@ -1312,7 +1352,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
               break;
             }
             tc_fence_after();
-            stage_b(sb, h, st, C::XSHARE ? 1 : 2);
+            stage_b(sb, h, st, (C::XSHARE || C::PH_SF) ? 1 : 2);
           }
           if (!ok) break;
           mma_commit(&m->bar_empty[stage]);
@@ -1392,6 +1432,78 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
       if constexpr (kBob) {
         reg_dep(rF[0]);
         reg_dep(rF[1]);
+      }
+      if constexpr (C::PH_SF) {
+        // ---- from SF alone: P, f = tau F and the Vtil operand P o h (h = F -
+        // alpha) of both halves; P o h goes over the S columns just copied
+        float2 pP[2][8], pF[2][8];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const int cv = HB * h + 16 * wg;
+          const int lo = qlo - (it + cv), hi = qhi - (it + cv);
+          if (lo > 0 || hi < 16) mask16(rS[h], lo, hi);
+          uint32_t oPh[8];
+#pragma unroll
+          for (int c = 0; c < 16; c += 2) {
+            const float2 nL2 = *reinterpret_cast<const float2*>(vec + cv + c);
+            const float2 nal = *reinterpret_cast<const float2*>(vec + 128 + cv + c);
+            const float2 pr = probs2(pair(rS[h], c), sl2v, nL2);
+            const float2 f = __fmul2_rn(pair(rF[h], c), tauv);
+            float2 gp = pr;
+            if constexpr (DROP) gp = __fmul2_rn(pr, gate2(kb[h], c, dsig));
+            const float2 ph = __fmul2_rn(gp, __fadd2_rn(f, nal));
+            pP[h][c / 2] = pr;
+            pF[h][c / 2] = f;
+            oPh[c / 2] = pack_bf16(ph.x, ph.y);
+          }
+          tmem_st8(ta + kColSF + cv, oPh);
+        }
+        tmem_st_wait();
+        tc_fence_before();
+        mbar_arrive(&m->bar_sf_free[0]);
+        if (!ew_wait(&m->bar_sa_dc[dc_sel(st)], dc_par(st))) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        // ---- with DC: Stil and dS into the DC columns just read
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const int cv = HB * h + 16 * wg;
+          const uint32_t R = ta + dc_col(st) + cv;
+          uint32_t rdP[16], rC[16];
+          tmem_ld16(R + 0, rdP);
+          tmem_ld16(R + 64, rC);
+          tmem_ld_wait(rdP);
+          reg_dep(rC);
+          uint32_t oSt[8], odS[8];
+#pragma unroll
+          for (int c = 0; c < 16; c += 2) {
+            const float2 nD = *reinterpret_cast<const float2*>(vec + 64 + cv + c);
+            const float2 nal = *reinterpret_cast<const float2*>(vec + 128 + cv + c);
+            const float2 nE = *reinterpret_cast<const float2*>(vec + 192 + cv + c);
+            const float2 pr = pP[h][c / 2], f = pF[h][c / 2];
+            float2 dp = pair(rdP, c), cc = pair(rC, c);
+            if constexpr (DROP) {  // dP and C gated by sigma R
+              const float2 g = gate2(kb[h], c, dsig);
+              dp = __fmul2_rn(dp, g);
+              cc = __fmul2_rn(cc, g);
+            }
+            const float2 t = __fadd2_rn(dp, nD);
+            // Ptil = C + F (dP - D) - alpha dP ; Stil = P (Ptil - E)
+            const float2 pt = __ffma2_rn(nal, dp, __ffma2_rn(f, t, cc));
+            const float2 stl = __fmul2_rn(pr, __fadd2_rn(pt, nE));
+            const float2 ds = __fmul2_rn(pr, t);
+            oSt[c / 2] = pack_bf16(stl.x, stl.y);
+            odS[c / 2] = pack_bf16(ds.x, ds.y);
+          }
+          tmem_st8(R + 8, oSt);
+          tmem_st8(R + 64, odS);
+          tmem_st_wait();
+          tc_fence_before();
+          mbar_arrive(&m->bar_ew[2 * dc_sel(st) + h]);
+        }
+        continue;
       }
       tc_fence_before();
       mbar_arrive(&m->bar_sf_free[0]);

@@ -130,6 +130,13 @@ struct ColCfg {
   // issuer Y would have to wait for them before the next DC (measured slower);
   // with two that wait is two tiles back and off the critical path.
   static constexpr bool XSHARE = DC2;
+  // BoB Pass 2 with one DC buffer (d = 128): the Vtil operand P o h needs
+  // only the scores tile, so the elementwise warps write it into the SF
+  // columns they have just copied, and issuer X accumulates Vtil from there
+  // (before SF(t+1), in its own issue order).  Issuer Y's chain per tile is
+  // then the Ktil MMAs and DC(t+1) alone, and the exponentials leave the
+  // elementwise work that waits for DC.
+  static constexpr bool PH_SF = OP == ColOp::BobPass2 && !DC2;
   static constexpr int MISC_BYTES = 256;
   static constexpr int SMEM_BYTES = STAT_BYTES + NSTAGES * STAGE_BYTES + MISC_BYTES;
 };
