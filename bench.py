@@ -39,9 +39,13 @@ DEFAULT_WORKLOAD = "n16k_d128_causal"
 # first loop) and Pass 2 is 8.  At d = 128 Pass 1 runs as two kernels: the
 # row-statistics kernel is credited with the 5 stage-A contractions and the
 # direct-form kernel with the other 6 (its stage-A recompute is not credited).
-CONTRACTIONS = {"pass1": 11, "row_stats": 5, "pass1_direct": 6, "pass2": 8}
-KERNEL_NAMES = {"pass1": "row_engine<BobPass1>", "row_stats": "row_engine<BobStats>",
-                "pass1_direct": "row_engine<BobPass1D>", "pass2": "col_engine<BobPass2>"}
+CONTRACTIONS = {"pass1": 11, "pass1_fused": 11, "row_stats": 5, "pass1_direct": 6, "pass2": 8}
+KERNEL_NAMES = {"pass1": "row_engine<BobPass1>", "pass1_fused": "row_engine<BobPass1>",
+                "row_stats": "row_engine<BobStats>", "pass1_direct": "row_engine<BobPass1D>",
+                "pass2": "col_engine<BobPass2>"}
+ENTRY_NAMES = {"pass1": "bob_pass1", "pass1_fused": "bob_pass1_fused",
+               "row_stats": "bob_row_stats", "pass1_direct": "bob_pass1_direct",
+               "pass2": "bob_pass2"}
 CSRC = os.path.join(ROOT, "paper_2609_24089_gb300", "csrc")
 
 
@@ -287,7 +291,11 @@ def run_gpu(args, w):
 
     # ---- timed region: K steps, each as its kernels (through their C-ABI
     # calls, the same ones fbob_attn_bob makes) with events between them
-    if w.d <= 64 and not drop:  # one-sweep Pass 1 (as fbob_attn_bob_pass1 chooses)
+    if args.pass1 == "fused" and not drop:  # one-sweep Pass 1 (Prop. 3.1) at any d
+        parts = [("pass1_fused", lambda: fbob.fbob_attn_bob_pass1_fused(
+            shp, q, k, v, o, lse, do, gq, gk, gv, outs[0], outs[3], rs))]
+    elif w.d <= 64 and not drop and args.pass1 != "stats_direct":
+        # one-sweep Pass 1 (as fbob_attn_bob_pass1 chooses)
         parts = [("pass1", lambda: fbob.fbob_attn_bob_pass1(
             shp, q, k, v, o, lse, do, gq, gk, gv, outs[0], outs[3], rs))]
     else:
@@ -313,9 +321,7 @@ def run_gpu(args, w):
     status = fbob.fbob_device_status()
     if status != 0:
         raise RuntimeError(f"device status {status} in timed region")
-    launches_per_step = sum(fbob.fbob_launch_count(
-        {"pass1": "bob_pass1", "row_stats": "bob_row_stats", "pass1_direct": "bob_pass1_direct",
-         "pass2": "bob_pass2"}[name]) for name, _ in parts)
+    launches_per_step = sum(fbob.fbob_launch_count(ENTRY_NAMES[name]) for name, _ in parts)
     ms = start.elapsed_time(stop)
     part_ms = {name: sum(e[j].elapsed_time(e[j + 1]) for e in ev) / K
                for j, (name, _) in enumerate(parts)}
@@ -410,6 +416,9 @@ def run_gpu(args, w):
         "clocks": clk.summary(),
         "peak_hbm_bytes": footprint,
         "call_alloc_bytes": call_delta,
+        "pass1_form": ("one sweep, affine fusion (Prop. 3.1)"
+                       if parts[0][0] in ("pass1", "pass1_fused")
+                       else "row statistics + direct form (eqs. 6-7)"),
         "pass_ms": {"pass1": total - part_ms["pass2"], "pass2": part_ms["pass2"]},
         "kernel_ms": part_ms,
     }
@@ -488,6 +497,9 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--op", default="bob", choices=["bob", "fwd", "bwd"],
                     help="bob (the benchmark); fwd / bwd time the boundary's other calls alone")
+    ap.add_argument("--pass1", default="auto", choices=["auto", "fused", "stats_direct"],
+                    help="Pass 1 form timed: auto (as fbob_attn_bob chooses), fused (one sweep "
+                         "with the affine fusion at any d) or stats_direct")
     ap.add_argument("--bh", default=None,
                     help="B,H override (smaller profiling captures of the same kernels)")
     args = ap.parse_args()

@@ -194,6 +194,23 @@ int fbob_attn_bob_pass1(const fbob_shape* shape, const void* q, const void* k, c
                         struct CUstream_st* stream);
 
 /*
+ * Pass 1 in one sweep with the affine fusion of Prop. 3.1 (eq. 8) at any
+ * supported d (the form fbob_attn_bob_pass1 takes at d <= 64): each row block
+ * streams K, U_K, V, U_V once and accumulates B = sum_j P_ij k_j, dOtil0 =
+ * sum_j P_ij (u_V,j + F_ij v_j), G = sum_j dS_ij k_j and Omega = sum_j
+ * (P o Ptil0)_ij k_j + dS_ij u_K,j with the running row sums alpha and E0;
+ * the epilogue forms E = E0 - alpha D, dOtil = dOtil0 - alpha o and Qtil =
+ * tau (Omega - alpha G - E0 B).  At d = 128 the four accumulators are split
+ * by output column over two CTAs per row block (each computes the whole
+ * stage A and its 64 columns of stage B).  One kernel.  Same arguments and
+ * outputs as fbob_attn_bob_pass1; dropout returns FBOB_ERR_UNSUPPORTED.
+ */
+int fbob_attn_bob_pass1_fused(const fbob_shape* shape, const void* q, const void* k,
+                              const void* v, const void* o, const float* lse, const void* dout,
+                              const void* gq, const void* gk, const void* gv, void* q_bar,
+                              void* dout_bar, float* row_stats, struct CUstream_st* stream);
+
+/*
  * Pass 2 of Algorithm 1 alone (column-block outer; Alg. 2, second loop):
  * reads row_stats (alpha, E, D, as pass 1 writes them) and lse, writes
  * k_bar and v_bar.  row_stats is an input here.
@@ -313,7 +330,8 @@ int fbob_device_status(struct CUstream_st* stream);
 
 /* Number of kernels the last successful call of the named entry point
  * enqueued ("fwd", "bwd", "bob", "bob_pass1", "bob_pass2", "bob_row_stats",
- * "bob_pass1_direct", "bob_host", "bob_host_noalloc"); -1 if unknown. */
+ * "bob_pass1_direct", "bob_host", "bob_host_noalloc", "bob_pass1_fused");
+ * -1 if unknown. */
 int fbob_launch_count(const char* entry);
 
 /* Static, human-readable name of a status code. */

@@ -62,6 +62,7 @@ def load():
         "fbob_attn_bwd": [S, P, P, P, P, P, P, P, P, P, P, P],
         "fbob_attn_bob": [S, P, P, P, P, P, P, P, P, P, P, P, P, P, P, P],
         "fbob_attn_bob_pass1": [S, P, P, P, P, P, P, P, P, P, P, P, P, P],
+        "fbob_attn_bob_pass1_fused": [S, P, P, P, P, P, P, P, P, P, P, P, P, P],
         "fbob_attn_bob_pass2": [S, P, P, P, P, P, P, P, P, P, P, P, P],
         "fbob_attn_bob_row_stats": [S, P, P, P, P, P, P, P, P, P, P, P],
         "fbob_attn_bob_pass1_direct": [S, P, P, P, P, P, P, P, P, P, P, P, P],
@@ -175,6 +176,14 @@ def fbob_attn_bob_pass1(shape, q, k, v, o, lse, dout, gq, gk, gv, q_bar, dout_ba
         ctypes.byref(shape),
         *map(_ptr, (q, k, v, o, lse, dout, gq, gk, gv, q_bar, dout_bar, row_stats)),
         _stream(stream)), "fbob_attn_bob_pass1")
+
+
+def fbob_attn_bob_pass1_fused(shape, q, k, v, o, lse, dout, gq, gk, gv, q_bar, dout_bar,
+                              row_stats, stream=None):
+    _check(load().fbob_attn_bob_pass1_fused(
+        ctypes.byref(shape),
+        *map(_ptr, (q, k, v, o, lse, dout, gq, gk, gv, q_bar, dout_bar, row_stats)),
+        _stream(stream)), "fbob_attn_bob_pass1_fused")
 
 
 def fbob_attn_bob_pass2(shape, q, k, v, lse, dout, gq, gk, gv, row_stats, k_bar, v_bar,

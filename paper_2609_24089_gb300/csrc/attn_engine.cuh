@@ -263,7 +263,10 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
   // in L2.  Otherwise heads are innermost, so with the causal mask the longest
   // row blocks of all heads go first (better balance, less sharing).
   const int N = p.N;
-  const int lin = blockIdx.x;
+  // one-sweep Pass 1 at d = 128: the C::SPLIT CTAs of a row block are
+  // neighbours in launch order; hc selects this CTA's 64 output columns
+  const int hc = C::SPLIT > 1 ? (int)(blockIdx.x % C::SPLIT) : 0;
+  const int lin = blockIdx.x / C::SPLIT;
   const int rbi = p.head_major ? lin % p.nblk : lin / p.BH;
   const int bh = p.head_major ? lin / p.nblk : lin % p.BH;
   const int rb = p.causal ? (p.nblk - 1 - rbi) : rbi;
@@ -375,8 +378,9 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
     if (elect_lane0()) {
       constexpr uint32_t id_n64 = idesc_bf16(128, 64, false);
       constexpr uint32_t id_n128 = idesc_bf16(128, 128, false);
-      constexpr uint32_t id_b = idesc_bf16(128, D, true);
-      constexpr uint32_t id_b2 = idesc_bf16(128, 2 * D, true);
+      // stage B of the one-sweep Pass 1 accumulates 64 output columns per CTA
+      constexpr uint32_t id_b = idesc_bf16(128, kBob ? 64 : D, true);
+      constexpr uint32_t id_b2 = idesc_bf16(128, 2 * (kBob ? 64 : D), true);
       // descriptors are formed once; per MMA only the start-address field moves
       const uint64_t sd0 = sdesc_sw128(smem_u32(s_stat), 16, 1024);
       auto sd = [&](int t, int k) -> uint64_t {
@@ -402,25 +406,27 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
           };
           const uint32_t first = (st == 0 && s == 0) ? 0u : 1u;
           if constexpr (kBob) {
+            // B operands: the 64-column box hc of K, U_V, V, U_K (this CTA's
+            // output columns)
             const uint32_t A = tmem + kColDC + 64 * h + 16 * sub;
-            const uint32_t k_rows = sb + soff<C::NSTREAM, kB4>(0, h, 0) + sub * 2048;
+            const uint32_t k_rows = sb + soff<C::NSTREAM, kB4>(0, h, hc) + sub * 2048;
             if (part != 1) {
               // [B | dOtil0] += P [K | U_V]   (second 64-wide block at U_V)
               const uint64_t fKUV = sdesc_sw128(
                   k_rows,
-                  soff<C::NSTREAM, kB4>(3, h, 0) - soff<C::NSTREAM, kB4>(0, h, 0),
+                  soff<C::NSTREAM, kB4>(3, h, hc) - soff<C::NSTREAM, kB4>(0, h, hc),
                   1024);
               mma_ts(tmem + 0, A + 0, fKUV, id_b2, first);
-              mma_ts(tmem + 64, A + 8, md(2, 0), id_b, 1);  // dOtil0 += (P o F) V
+              mma_ts(tmem + 64, A + 8, md(2, hc), id_b, 1);  // dOtil0 += (P o F) V
             }
             if (part != 0) {
               // [G | Omega] += dS [K | U_K] ;  Omega += (P o Pt0) K
               const uint64_t fKUK = sdesc_sw128(
                   k_rows,
-                  soff<C::NSTREAM, kB4>(1, h, 0) - soff<C::NSTREAM, kB4>(0, h, 0),
+                  soff<C::NSTREAM, kB4>(1, h, hc) - soff<C::NSTREAM, kB4>(0, h, hc),
                   1024);
               mma_ts(tmem + 128, A + 40, fKUK, id_b2, first);
-              mma_ts(tmem + 192, A + 32, md(0, 0), id_b, 1);
+              mma_ts(tmem + 192, A + 32, md(0, hc), id_b, 1);
             }
           } else if constexpr (kDirect) {
             // eqs. (6)-(7): Qtil += Stil K + dS U_K (part 1) ; dOtil += P U_V +
@@ -932,7 +938,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         const float alpha = s_xchg[r] + s_xchg[BM + r];
         const float E0 = s_xchg[2 * BM + r] + s_xchg[3 * BM + r];
         const float E = E0 - alpha * Dr;  // eq. (8): E = E0 - alpha D
-        const int cbase = 32 * wg;
+        const int cbase = 64 * hc + 32 * wg;  // output column of accumulator column 32 wg
 #pragma unroll 1
         for (int q = 0; q < 2; ++q) {
           const int cc = 32 * wg + 16 * q;  // accumulator column (0..63)
@@ -960,7 +966,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
             store_row16(p.out1 + rowoff + cbase + 16 * q, dot);
           }
         }
-        if (row_ok && wg == 0) {
+        if (row_ok && wg == 0 && hc == 0) {
           const size_t ri = (size_t)bh * N + gi;
           p.vec_out[ri] = alpha;
           p.vec_out[p.bhn + ri] = E;

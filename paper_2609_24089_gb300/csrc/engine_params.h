@@ -83,8 +83,12 @@ struct RowCfg {
   static constexpr int KB = D / 64;  // 64-wide boxes per row
   static constexpr int NSTAT = OP == RowOp::BwdDQ ? 2 : 3;
   static constexpr int NSTREAM = row_bob(OP) ? 4 : 2;
-  // the one-sweep Pass 1 holds four D-column accumulators: d = 64 only
-  static_assert(OP != RowOp::BobPass1 || D == 64, "one-sweep Pass 1 needs d = 64");
+  // the one-sweep Pass 1 (Prop. 3.1) holds four accumulators of 64 output
+  // columns next to the stage-A tiles (4 x 64 + 128 + 128 = 512 TMEM
+  // columns): at d = 128 the output columns are split over SPLIT = 2 CTAs per
+  // row block, each computing the whole stage A and its half of stage B
+  static constexpr int SPLIT = OP == RowOp::BobPass1 ? D / 64 : 1;
+  static_assert(OP != RowOp::BobPass1 || D == 64 || D == 128, "one-sweep Pass 1: d <= 128");
   // the row statistics kernel has no accumulators: Q and U_Q live in TMEM as
   // MMA A operands next to two SF buffers; only dO stays in shared memory,
   // which leaves room for another stream stage
@@ -96,7 +100,7 @@ struct RowCfg {
   // parts of SF(t+1).  Measured faster for the one-sweep Pass 1 (d = 64); for
   // the direct form at d = 128 (dOtil on X) Y's wait for X's share before
   // each DC cost 5 % more than it saved.
-  static constexpr bool XSHARE = OP == RowOp::BobPass1 && D == 64;
+  static constexpr bool XSHARE = OP == RowOp::BobPass1;
   // Pass 1's DC ([dP | C]) issued per 32-key half, so that stage B of half 0
   // overlaps the elementwise work on half 1; otherwise one N = 128 MMA per
   // K-step for the whole tile.  Measured for the direct form at d = 128:

@@ -18,12 +18,12 @@ namespace {
 constexpr int64_t kMaxN = int64_t(1) << 24;
 constexpr int64_t kMaxBH = int64_t(1) << 24;
 
-constexpr int kNumEntries = 9;
+constexpr int kNumEntries = 10;
 std::atomic<int> g_launches[kNumEntries] = {{-1}, {-1}, {-1}, {-1}, {-1},
-                                            {-1}, {-1}, {-1}, {-1}};
+                                            {-1}, {-1}, {-1}, {-1}, {-1}};
 enum Entry {
   kEntFwd = 0, kEntBwd, kEntBob, kEntPass1, kEntPass2, kEntRowStats, kEntPass1D, kEntBobHost,
-  kEntBobHostNoAlloc
+  kEntBobHostNoAlloc, kEntPass1Fused
 };
 
 // Staging memory of fbob_attn_bob_host_noalloc: a fixed device array, so that
@@ -222,8 +222,22 @@ int run_pass1_direct(EngineParams p, int d, bool drop, const float* row_stats, v
   return launch_status(launch_row(RowOp::BobPass1D, d, drop, p, p.nblk * p.BH, st));
 }
 
-// Pass 1 in one sweep (the affine fusion, Prop. 3.1) at d <= 64 without
-// dropout; otherwise row statistics + direct form
+// Pass 1 in one sweep with the affine fusion (Prop. 3.1, eq. 8): one kernel,
+// at d = 128 two CTAs per row block (64 output columns each).  No dropout.
+int run_pass1_fused(EngineParams p, int d, void* q_bar, void* dout_bar, float* row_stats,
+                    cudaStream_t st) {
+  p.out0 = static_cast<__nv_bfloat16*>(q_bar);
+  p.out1 = static_cast<__nv_bfloat16*>(dout_bar);
+  p.vec_out = row_stats;
+  const int split = d == 128 ? 2 : 1;
+  return launch_status(launch_row(RowOp::BobPass1, d, false, p, p.nblk * p.BH * split, st));
+}
+
+// The form fbob_attn_bob's Pass 1 takes: the one-sweep affine fusion at d <= 64
+// without dropout; otherwise row statistics + direct form (with dropout the
+// one-sweep fusion would need a fifth operand tile per half, the ungated P
+// of B next to the gated P of dOtil0; at d = 128 the statistics + direct
+// form was measured faster than the fused form over two CTAs per row block).
 bool pass1_one_sweep(const fbob_shape* s) { return s->d <= 64 && !has_dropout(s); }
 
 // head0: flat index of the shape's first query head within a larger problem
@@ -235,12 +249,7 @@ int run_pass1(const fbob_shape* s, const void* q, const void* k, const void* v, 
   EngineParams p;
   if (!row_bob_params(s, q, k, v, o, lse, dout, gq, gk, gv, &p)) return FBOB_ERR_CUDA;
   p.head0 = (int)head0;
-  if (pass1_one_sweep(s)) {  // one sweep, affine fusion (Prop. 3.1)
-    p.out0 = static_cast<__nv_bfloat16*>(q_bar);
-    p.out1 = static_cast<__nv_bfloat16*>(dout_bar);
-    p.vec_out = row_stats;
-    return launch_status(launch_row(RowOp::BobPass1, (int)s->d, false, p, p.nblk * p.BH, st));
-  }
+  if (pass1_one_sweep(s)) return run_pass1_fused(p, (int)s->d, q_bar, dout_bar, row_stats, st);
   // d = 128: the four accumulators of the one-sweep form do not fit TMEM next
   // to the stage-A tiles; with dropout (any d) the direct form gates its
   // operands tile by tile.  First the row scalars (alpha, E, D), then Qtil
@@ -439,7 +448,7 @@ int fbob_launch_count(const char* entry) {
   if (!entry) return -1;
   static const char* names[kNumEntries] = {
       "fwd",       "bwd",       "bob",           "bob_pass1",          "bob_pass2",
-      "bob_row_stats", "bob_pass1_direct", "bob_host", "bob_host_noalloc"};
+      "bob_row_stats", "bob_pass1_direct", "bob_host", "bob_host_noalloc", "bob_pass1_fused"};
   for (int t = 0; t < kNumEntries; ++t)
     if (std::strcmp(entry, names[t]) == 0) return g_launches[t].load();
   return -1;
@@ -547,6 +556,33 @@ int fbob_attn_bob_pass1(const fbob_shape* s, const void* q, const void* k, const
   if (rc != FBOB_OK) return rc;
   rc = run_pass1(s, q, k, v, o, lse, dout, gq, gk, gv, q_bar, dout_bar, row_stats, stream);
   if (rc == FBOB_OK) g_launches[kEntPass1] = pass1_launches(s);
+  return rc;
+}
+
+int fbob_attn_bob_pass1_fused(const fbob_shape* s, const void* q, const void* k, const void* v,
+                              const void* o, const float* lse, const void* dout, const void* gq,
+                              const void* gk, const void* gv, void* q_bar, void* dout_bar,
+                              float* row_stats, struct CUstream_st* stream) {
+  bool empty = false;
+  int rc = check_shape(s, &empty);
+  if (rc != FBOB_OK) return rc;
+  if (has_dropout(s)) return FBOB_ERR_UNSUPPORTED;
+  if (empty) {
+    g_launches[kEntPass1Fused] = 0;
+    return FBOB_OK;
+  }
+  const int64_t mat = s->B * s->H * s->N * s->d * 2, vec = s->B * s->H * s->N * 4;
+  const int64_t matk = s->B * kv_heads(s) * s->N * s->d * 2;
+  const void* in[9] = {q, k, v, o, lse, dout, gq, gk, gv};
+  const int64_t inb[9] = {mat, matk, matk, mat, vec, mat, mat, matk, matk};
+  void* out[3] = {q_bar, dout_bar, row_stats};
+  const int64_t outb[3] = {mat, mat, 3 * vec};
+  rc = check_ptrs(in, inb, 9, out, outb, 3);
+  if (rc != FBOB_OK) return rc;
+  EngineParams p;
+  if (!row_bob_params(s, q, k, v, o, lse, dout, gq, gk, gv, &p)) return FBOB_ERR_CUDA;
+  rc = run_pass1_fused(p, (int)s->d, q_bar, dout_bar, row_stats, stream);
+  if (rc == FBOB_OK) g_launches[kEntPass1Fused] = 1;
   return rc;
 }
 

@@ -1,7 +1,7 @@
 // row_kernels.cu -- instantiations and launcher of the row-block kernels:
 // forward (eq. 1, fwd_engine.cuh), first-backward dQ (eqs. 2-3), BoB Pass 1 (Algorithm 2,
-// first loop): one sweep at d <= 64, row statistics + direct form at d = 128
-// (and at any d with dropout).  Each operation with and without dropout, for
+// first loop): one sweep with the affine fusion (at d = 128 over two CTAs per
+// row block), or row statistics + direct form.  Each operation with and without dropout, for
 // head dims 32 (in 64-wide tiles), 64 and 128.
 #include "attn_engine.cuh"
 #include "fwd_engine.cuh"
@@ -62,11 +62,13 @@ cudaError_t launch_row(RowOp op, int d, bool drop, const EngineParams& p, int nb
     case RowOp::Fwd:
       return drop ? launch_fwd<true>(d, p, nblocks, s) : launch_fwd<false>(d, p, nblocks, s);
     case RowOp::BwdDQ: return launch_op<RowOp::BwdDQ>(d, drop, p, nblocks, s);
-    case RowOp::BobPass1:  // the one-sweep form serves d <= 64 without dropout only
+    case RowOp::BobPass1:  // the one-sweep form (no dropout); at d = 128 nblocks
+                           // counts both CTAs of each row block
       if (drop) return cudaErrorInvalidValue;
-      return d == 64   ? launch_one<RowOp::BobPass1, 64, false>(p, nblocks, s)
-             : d == 32 ? launch_one<RowOp::BobPass1, 64, false, 32>(p, nblocks, s)
-                       : cudaErrorInvalidValue;
+      return d == 64    ? launch_one<RowOp::BobPass1, 64, false>(p, nblocks, s)
+             : d == 32  ? launch_one<RowOp::BobPass1, 64, false, 32>(p, nblocks, s)
+             : d == 128 ? launch_one<RowOp::BobPass1, 128, false>(p, nblocks, s)
+                        : cudaErrorInvalidValue;
     case RowOp::BobStats: return launch_op<RowOp::BobStats>(d, drop, p, nblocks, s);
     case RowOp::BobPass1D: return launch_op<RowOp::BobPass1D>(d, drop, p, nblocks, s);
   }
