@@ -139,7 +139,9 @@ struct ColCfg {
   // columns they have just copied, and issuer X accumulates Vtil from there
   // (before SF(t+1), in its own issue order).  Issuer Y's chain per tile is
   // then the Ktil MMAs and DC(t+1) alone, and the exponentials leave the
-  // elementwise work that waits for DC.
+  // elementwise work that waits for DC.  Measured 2.5 % faster at d = 128;
+  // at d = 64 (two DC buffers, XSHARE) it was 10 % slower: there SF(t+1)
+  // waiting for P o h is the longer delay.
   static constexpr bool PH_SF = OP == ColOp::BobPass2 && !DC2;
   static constexpr int MISC_BYTES = 256;
   static constexpr int SMEM_BYTES = STAT_BYTES + NSTAGES * STAGE_BYTES + MISC_BYTES;
