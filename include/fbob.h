@@ -21,7 +21,8 @@
  *             columns loaded as zeros.)
  *             N >= 0 is arbitrary (tails are masked); B*H*N == 0 is a valid
  *             empty problem that launches nothing and returns FBOB_OK.
- *             N <= 2^24 and B*H <= 2^24.  scale must be finite and > 0
+ *             N <= 2^24, B*H <= 2^24 and ceil(N/128) * B*H * 2 < 2^31 (the
+ *             launch grids).  scale must be finite and > 0
  *             (1/sqrt(d) in the paper).  causal is 0 or 1; with 1 the mask
  *             keeps j <= i (square, top-left aligned, diagonal included).
  *             window_left, window_right (each -1 or >= 0) add a sliding-window

@@ -87,6 +87,9 @@ int check_shape(const fbob_shape* s, bool* empty) {
   if (s->d != 32 && s->d != 64 && s->d != 128) return FBOB_ERR_UNSUPPORTED;
   if (s->N > kMaxN) return FBOB_ERR_INVALID_ARGUMENT;
   if (s->B > kMaxBH || s->H > kMaxBH || s->B * s->H > kMaxBH) return FBOB_ERR_INVALID_ARGUMENT;
+  // the largest launch (two CTAs per 128-row block for the split one-sweep
+  // Pass 1) must fit a grid
+  if ((s->N + 127) / 128 * s->B * s->H * 2 > (int64_t)0x7FFFFFFF) return FBOB_ERR_INVALID_ARGUMENT;
   *empty = (s->B * s->H * s->N) == 0;
   return FBOB_OK;
 }
@@ -202,7 +205,7 @@ bool row_bob_params(const fbob_shape* s, const void* q, const void* k, const voi
   p->o = static_cast<const __nv_bfloat16*>(o);
   p->dout = static_cast<const __nv_bfloat16*>(dout);
   p->lse = lse;
-  p->nblk = n_blocks(N, BM);
+  p->nblk = n_blocks(s->N, BM);
   choose_order(p, 1);
   return true;
 }
@@ -282,7 +285,7 @@ int run_pass2(const fbob_shape* s, const void* q, const void* k, const void* v, 
   p.vec_in = row_stats;
   p.out0 = static_cast<__nv_bfloat16*>(k_bar);
   p.out1 = static_cast<__nv_bfloat16*>(v_bar);
-  p.nblk = n_blocks(N, BM);
+  p.nblk = n_blocks(s->N, BM);
   choose_order(&p, 0);
   return launch_status(launch_col(ColOp::BobPass2, (int)d, has_dropout(s), p, p.nblk * p.BH, st));
 }
@@ -514,7 +517,7 @@ int fbob_attn_bwd(const fbob_shape* s, const void* q, const void* k, const void*
   p.lse = lse;
   p.out0 = static_cast<__nv_bfloat16*>(dq);
   p.vec_out = dstat;
-  p.nblk = n_blocks(N, BM);
+  p.nblk = n_blocks(s->N, BM);
   choose_order(&p, 0);
   rc = launch_status(launch_row(RowOp::BwdDQ, (int)d, has_dropout(s), p, p.nblk * p.BH, stream));
   if (rc != FBOB_OK) return rc;
@@ -528,7 +531,7 @@ int fbob_attn_bwd(const fbob_shape* s, const void* q, const void* k, const void*
   c.vec_in = dstat;
   c.out0 = static_cast<__nv_bfloat16*>(dk);
   c.out1 = static_cast<__nv_bfloat16*>(dv);
-  c.nblk = n_blocks(N, BM);
+  c.nblk = n_blocks(s->N, BM);
   choose_order(&c, 0);
   rc = launch_status(launch_col(ColOp::BwdDKDV, (int)d, has_dropout(s), c, c.nblk * c.BH, stream));
   if (rc == FBOB_OK) g_launches[kEntBwd] = 2;

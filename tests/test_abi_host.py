@@ -57,6 +57,8 @@ def test_rejects_bad_shapes(lib):
     assert bob(lib, S(1, 1, 128, 64, 0.125, 2), ptrs(14)) == 1         # causal not 0/1
     assert bob(lib, S(-1, 1, 128, 64, 0.125, 0), ptrs(14)) == 1
     assert bob(lib, S(1, 1, (1 << 24) + 1, 64, 0.125, 0), ptrs(14)) == 1
+    # launch grids past 2^31 CTAs: ceil(N/128) * B*H * 2 >= 2^31
+    assert bob(lib, S(1 << 12, 1 << 12, 1 << 14, 64, 0.125, 0), ptrs(14)) == 1
     assert lib.fbob_attn_bob(None, *ptrs(14), None) == 1               # null shape
 
 
