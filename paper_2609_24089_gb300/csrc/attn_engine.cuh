@@ -166,6 +166,20 @@ struct TileSet {
   }
 };
 
+// CTA order: heads in groups of p.head_group; within a group the blocks are
+// outermost (with the causal mask the longest first) and the group's heads
+// innermost.  head_group 1 is head-major (the CTAs in flight share one head's
+// streamed tiles in L2); head_group >= BH puts every head's longest block
+// first (the best balance, the least sharing).
+__device__ __forceinline__ void cta_order(const EngineParams& p, int lin, int& rbi, int& bh) {
+  const int G = p.head_group;
+  const int grp = lin / (p.nblk * G);
+  const int gsz = min(G, p.BH - grp * G);
+  const int rem = lin - grp * p.nblk * G;
+  rbi = rem / gsz;
+  bh = grp * G + rem % gsz;
+}
+
 __device__ __forceinline__ float bits_f(uint32_t u) { return __uint_as_float(u); }
 __device__ __forceinline__ float2 pair(const uint32_t (&r)[16], int c) {
   return make_float2(__uint_as_float(r[c]), __uint_as_float(r[c + 1]));
@@ -198,19 +212,47 @@ __device__ __forceinline__ void load_row16(const __nv_bfloat16* src, float (&v)[
   }
 }
 
-// fp32 dot product of one bf16 row pair of length D (D = do_i . o_i).
-template <int D>
-__device__ __forceinline__ float row_dot(const __nv_bfloat16* a, const __nv_bfloat16* b) {
-  float acc = 0.f;
+// D_i = do_i . o_i (fp32) for the 128 rows of a row block, computed by the
+// 256 elementwise threads together and returned to thread r (any warpgroup)
+// for row r.  Each row's DG bf16 values are read by DG / 8 consecutive lanes,
+// 16 bytes each, so a warp's loads cover whole rows (coalesced); the lanes'
+// partial sums are added by shuffles and passed on through s_d[128].  Every
+// elementwise thread must call it (it ends in a named barrier).
+template <int DG>
+__device__ __forceinline__ float block_row_dots(const __nv_bfloat16* dout, const __nv_bfloat16* o,
+                                                size_t head_off, int i0, int row_end, float* s_d,
+                                                int ew_tid) {
+  constexpr int LPR = DG / 8;     // lanes per row
+  constexpr int RPI = 32 / LPR;   // rows per warp instruction
+  const int warp = ew_tid >> 5, lane = ew_tid & 31;
+  const int sub = lane / LPR, part = lane % LPR;
+  float acc[16 / RPI];
 #pragma unroll
-  for (int c = 0; c < D; c += 16) {
-    float x[16], y[16];
-    load_row16(a + c, x);
-    load_row16(b + c, y);
+  for (int k = 0; k < 16 / RPI; ++k) {  // this warp's 16 rows, RPI at a time
+    const int r = 16 * warp + RPI * k + sub;
+    acc[k] = 0.f;
+    if (i0 + r < row_end) {
+      const size_t off = head_off + (size_t)(i0 + r) * DG + 8 * part;
+      const uint4 va = *reinterpret_cast<const uint4*>(dout + off);
+      const uint4 vb = *reinterpret_cast<const uint4*>(o + off);
+      const uint32_t wa[4] = {va.x, va.y, va.z, va.w};
+      const uint32_t wb[4] = {vb.x, vb.y, vb.z, vb.w};
 #pragma unroll
-    for (int t = 0; t < 16; ++t) acc = fmaf(x[t], y[t], acc);
+      for (int t = 0; t < 4; ++t) {
+        acc[k] = fmaf(__uint_as_float(wa[t] << 16), __uint_as_float(wb[t] << 16), acc[k]);
+        acc[k] = fmaf(__uint_as_float(wa[t] & 0xFFFF0000u), __uint_as_float(wb[t] & 0xFFFF0000u),
+                      acc[k]);
+      }
+    }
   }
-  return acc;
+#pragma unroll
+  for (int k = 0; k < 16 / RPI; ++k) {
+#pragma unroll
+    for (int s = LPR / 2; s > 0; s >>= 1) acc[k] += __shfl_xor_sync(0xffffffffu, acc[k], s);
+    if (part == 0) s_d[16 * warp + RPI * k + sub] = acc[k];
+  }
+  named_bar_sync(2, kEwThreads);
+  return s_d[32 * (warp & 3) + lane];
 }
 
 // p = exp2(s * sl2 - L2) for a pair of scores.
@@ -250,6 +292,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
   uint8_t* s_stream = smem + C::STAT_BYTES;
   Misc* m = reinterpret_cast<Misc*>(s_stream + C::NSTAGES * C::STAGE_BYTES);
   float* s_xchg = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(m) + 256);  // 4 x BM floats
+  float* s_d = s_xchg + 4 * BM;  // BM floats: the rows' D (block_row_dots)
 
   const int tid = threadIdx.x;
   const int warp = tid >> 5;
@@ -258,17 +301,14 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
     return;
   }
 
-  // ---- tile decode.  Head-major order: the CTAs in flight work on the row
-  // blocks of one or two heads and stream the same K/V tiles, which then stay
-  // in L2.  Otherwise heads are innermost, so with the causal mask the longest
-  // row blocks of all heads go first (better balance, less sharing).
+  // ---- tile decode (CTA order: cta_order).
   const int N = p.N;
   // one-sweep Pass 1 at d = 128: the C::SPLIT CTAs of a row block are
   // neighbours in launch order; hc selects this CTA's 64 output columns
   const int hc = C::SPLIT > 1 ? (int)(blockIdx.x % C::SPLIT) : 0;
   const int lin = blockIdx.x / C::SPLIT;
-  const int rbi = p.head_major ? lin % p.nblk : lin / p.BH;
-  const int bh = p.head_major ? lin / p.nblk : lin % p.BH;
+  int rbi, bh;
+  cta_order(p, lin, rbi, bh);
   const int rb = p.causal ? (p.nblk - 1 - rbi) : rbi;
   // key/value head of this query head (grouped-query attention: h / (H / Hkv))
   const int bh_kv = p.Hkv == p.H ? bh : (bh / p.H) * p.Hkv + (bh % p.H) / (p.H / p.Hkv);
@@ -718,32 +758,37 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
           nal = -p.vec_in[ri];
           nE = -p.vec_in[p.bhn + ri];
           Dr = p.vec_in[2 * p.bhn + ri];
-        } else {
-          Dr = row_dot<DG>(p.dout + rowoff, p.o + rowoff);
         }
       }
     }
+    // D = do . o (the statistics kernel first puts Q and U_Q into TMEM, so
+    // that issuer X can start while D is summed)
+    if constexpr (!kDirect && !C::STAT_TMEM)
+      Dr = block_row_dots<DG>(p.dout, p.o, (size_t)bh * N * DG, i0, N, s_d, tid);
     if constexpr (C::STAT_TMEM) {
       // stationary rows straight into TMEM as MMA A operands (word c of a
       // bf16 row = elements 2c, 2c+1 = column c of its operand): warpgroup 0
       // writes Q, warpgroup 1 U_Q
-      auto put_row = [&](const __nv_bfloat16* row, uint32_t col, int c0, int ncols) {
+      // (every load of the row first, so the CTA waits for one memory round
+      // trip instead of one per 8 columns)
+      auto put_row = [&](const __nv_bfloat16* row, uint32_t col) {
         const uint4* src = reinterpret_cast<const uint4*>(row);
-#pragma unroll 1
-        for (int c = c0; c < c0 + ncols; c += 8) {
-          uint4 a = make_uint4(0, 0, 0, 0), b = a;
-          if (row_ok && 2 * c < DG) {  // zero columns past the tensor's head dim
-            a = src[c / 4];
-            b = src[c / 4 + 1];
-          }
+        uint4 v[D / 8];  // the row's D bf16 values, 8 per uint4
+#pragma unroll
+        for (int u = 0; u < D / 8; ++u)  // zero columns past the tensor's head dim
+          v[u] = (row_ok && 8 * u < DG) ? src[u] : make_uint4(0, 0, 0, 0);
+#pragma unroll
+        for (int c = 0; c < D / 2; c += 8) {
+          const uint4 a = v[c / 4], b = v[c / 4 + 1];
           const uint32_t w[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
           tmem_st8(ta + col + c, w);
         }
       };
-      put_row((wg == 0 ? p.q : p.uq) + rowoff, kColQT + wg * (D / 2), 0, D / 2);
+      put_row((wg == 0 ? p.q : p.uq) + rowoff, kColQT + wg * (D / 2));
       tmem_st_wait();
       tc_fence_before();
       mbar_arrive(&m->bar_stat);
+      Dr = block_row_dots<DG>(p.dout, p.o, (size_t)bh * N * DG, i0, N, s_d, tid);
     }
     float2 acc_a = splat(0.f), acc_e = splat(0.f);  // Pass 1 partial row sums
     bool ok = true;
@@ -1056,8 +1101,8 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
   auto dc_par = [](int t) -> uint32_t { return C::DC2 ? ((t >> 1) & 1) : (t & 1); };
   const int N = p.N;
   const int lin = blockIdx.x;
-  const int cb = p.head_major ? lin % p.nblk : lin / p.BH;
-  const int bh = p.head_major ? lin / p.nblk : lin % p.BH;
+  int cb, bh;
+  cta_order(p, lin, cb, bh);
   const int j0 = cb * BM;
   // streamed query tiles: rows whose band holds a key of this block,
   // j - wr <= i <= j + wl (negative w: unbounded; causal: wr = 0)

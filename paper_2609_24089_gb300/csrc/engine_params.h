@@ -61,7 +61,7 @@ struct EngineParams {
   long long bhn;  // BH * N (row_stats plane stride)
   unsigned long long wait_limit_ns;  // bound of every device-side wait
   int inject_stall;                  // fault injection: producers issue nothing
-  int head_major;                    // CTA order: 1 = head-major, 0 = heads innermost
+  int head_group;                    // CTA order: heads per group (attn_engine.cuh, cta_order)
   // dropout (kernels instantiated with it): Philox round keys (the seed
   // raised r times by the Weyl constants, r = 0..9), the byte threshold t as
   // (t mod 128) in each byte and a flag (all ones if t < 128), and
@@ -110,7 +110,8 @@ struct RowCfg {
   // the dQ kernel's DC tile (dP, 64 columns) leaves the other half of the DC
   // area free: two dP buffers, dP(t+2) issued right after stage B(t)
   static constexpr bool DC2 = OP == RowOp::BwdDQ;
-  static constexpr int MISC_BYTES = 2304;
+  // bookkeeping (256), the row-sum exchange (4 x BM floats), the rows' D (BM floats)
+  static constexpr int MISC_BYTES = 2816;
   static constexpr int SMEM_BYTES = STAT_BYTES + NSTAGES * STAGE_BYTES + MISC_BYTES;
 };
 

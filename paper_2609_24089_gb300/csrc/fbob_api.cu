@@ -131,10 +131,16 @@ void debug_controls(EngineParams* p) {
   p->inject_stall = (inj && inj[0] == '1') ? 1 : 0;
 }
 
-// CTA order per kernel, from measurements on GB300: head-major helps Pass 1
-// (CTAs in flight share one head's K/V stream in L2); Pass 2 and the helper
-// kernels balance the causal work better with heads innermost.
-void choose_order(EngineParams* p, int head_major) { p->head_major = head_major; }
+// CTA order per kernel (heads per group, cta_order in attn_engine.cuh), from
+// measurements on GB300: groups of four heads suit Pass 1 (the CTAs in flight
+// share four heads' K/V streams in L2, and no head's longest row blocks are
+// left to the end: 0.4 % faster than head-major, 2 % faster than all heads);
+// Pass 2 and the helper kernels balance the causal work better with every
+// head's longest block first (all heads).
+void choose_order(EngineParams* p, int heads_per_group) {
+  p->head_group = heads_per_group < 1 ? 1 : (heads_per_group > p->BH ? p->BH : heads_per_group);
+  if (p->head_group < 1) p->head_group = 1;
+}
 
 // key/value heads per batch entry
 int64_t kv_heads(const fbob_shape* s) { return s->H_kv > 0 ? s->H_kv : s->H; }
@@ -206,7 +212,7 @@ bool row_bob_params(const fbob_shape* s, const void* q, const void* k, const voi
   p->dout = static_cast<const __nv_bfloat16*>(dout);
   p->lse = lse;
   p->nblk = n_blocks(s->N, BM);
-  choose_order(p, 1);
+  choose_order(p, 4);
   return true;
 }
 
@@ -286,7 +292,7 @@ int run_pass2(const fbob_shape* s, const void* q, const void* k, const void* v, 
   p.out0 = static_cast<__nv_bfloat16*>(k_bar);
   p.out1 = static_cast<__nv_bfloat16*>(v_bar);
   p.nblk = n_blocks(s->N, BM);
-  choose_order(&p, 0);
+  choose_order(&p, p.BH);
   return launch_status(launch_col(ColOp::BobPass2, (int)d, has_dropout(s), p, p.nblk * p.BH, st));
 }
 
@@ -482,7 +488,7 @@ int fbob_attn_fwd(const fbob_shape* s, const void* q, const void* k, const void*
   p.out0 = static_cast<__nv_bfloat16*>(o);
   p.vec_out = lse;
   p.nblk = n_blocks(s->N, 2 * BM);  // two 128-row query tiles per CTA
-  choose_order(&p, 0);
+  choose_order(&p, p.BH);
   rc = launch_status(launch_row(RowOp::Fwd, (int)s->d, has_dropout(s), p, p.nblk * p.BH, stream));
   if (rc == FBOB_OK) g_launches[kEntFwd] = 1;
   return rc;
@@ -518,7 +524,7 @@ int fbob_attn_bwd(const fbob_shape* s, const void* q, const void* k, const void*
   p.out0 = static_cast<__nv_bfloat16*>(dq);
   p.vec_out = dstat;
   p.nblk = n_blocks(s->N, BM);
-  choose_order(&p, 0);
+  choose_order(&p, p.BH);
   rc = launch_status(launch_row(RowOp::BwdDQ, (int)d, has_dropout(s), p, p.nblk * p.BH, stream));
   if (rc != FBOB_OK) return rc;
   // dK and dV: column-block pass
@@ -532,7 +538,7 @@ int fbob_attn_bwd(const fbob_shape* s, const void* q, const void* k, const void*
   c.out0 = static_cast<__nv_bfloat16*>(dk);
   c.out1 = static_cast<__nv_bfloat16*>(dv);
   c.nblk = n_blocks(s->N, BM);
-  choose_order(&c, 0);
+  choose_order(&c, c.BH);
   rc = launch_status(launch_col(ColOp::BwdDKDV, (int)d, has_dropout(s), c, c.nblk * c.BH, stream));
   if (rc == FBOB_OK) g_launches[kEntBwd] = 2;
   return rc;

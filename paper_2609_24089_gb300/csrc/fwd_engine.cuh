@@ -107,8 +107,8 @@ __global__ void __launch_bounds__(kFwdThreads, 1) fwd_engine(const __grid_consta
   // with the most keys go first
   const int N = p.N;
   const int lin = blockIdx.x;
-  const int rbi = p.head_major ? lin % p.nblk : lin / p.BH;
-  const int bh = p.head_major ? lin / p.nblk : lin % p.BH;
+  int rbi, bh;
+  cta_order(p, lin, rbi, bh);
   const int rb = p.causal ? (p.nblk - 1 - rbi) : rbi;
   const int bh_kv = p.Hkv == p.H ? bh : (bh / p.H) * p.Hkv + (bh % p.H) / (p.H / p.Hkv);
   const int i0 = rb * kFwdRows;
