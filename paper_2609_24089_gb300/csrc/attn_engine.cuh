@@ -1170,16 +1170,48 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
                       bh);
     }
     int issued[kMaxStages] = {-1, -1, -1, -1};
+    // query tile and head of step st (the tile cursor restarts for each of
+    // the key/value head's query heads)
     int tile = first_tile - 1;
+    auto advance = [&](int st, int& ib, int& bhq) {
+      if (st % nsteps_h == 0) tile = first_tile - 1;
+      tile = tiles.next(tile + 1);
+      ib = tile * BN;
+      bhq = bh_q0 + st / nsteps_h;
+    };
+    // negated row vectors of a step's streamed query rows, two rows per lane:
+    // [0] -L*log2e, [1] -D, [2] -alpha, [3] -E (the first backward: L, D).
+    // They are loaded one step ahead, so their latency passes while the
+    // producer waits for the stage they go to.
+    constexpr int NV = C::NVEC;
+    auto load_vec = [&](int ib, int bhq, float (&v)[2][NV]) {
+#pragma unroll
+      for (int q = 0; q < 2; ++q) {
+        const int gi = ib + lane + 32 * q;
+        const bool ok = gi < N;
+        const size_t ri = (size_t)bhq * N + (ok ? gi : 0);
+        v[q][0] = ok ? -p.lse[ri] * kLog2e : 0.f;
+        if constexpr (OP == ColOp::BwdDKDV) {
+          v[q][1] = ok ? -p.vec_in[ri] : 0.f;
+        } else {
+          v[q][1] = ok ? -p.vec_in[2 * p.bhn + ri] : 0.f;  // D
+          v[q][2] = ok ? -p.vec_in[ri] : 0.f;              // alpha
+          v[q][3] = ok ? -p.vec_in[p.bhn + ri] : 0.f;      // E
+        }
+      }
+    };
+    int ib_n = 0, bhq_n = 0;
+    float vn[2][NV];
+    if (nprod > 0) {
+      advance(0, ib_n, bhq_n);
+      load_vec(ib_n, bhq_n, vn);
+    }
     for (int st = 0; st < nprod; ++st) {
       const int stage = st % C::NSTAGES;
       if (st >= C::NSTAGES) {
         if (!mbar_wait(&m->bar_empty[stage], ((st / C::NSTAGES) - 1) & 1, wctl)) break;
       }
-      if (st % nsteps_h == 0) tile = first_tile - 1;  // next query head: from the start
-      tile = tiles.next(tile + 1);
-      const int ib = tile * BN;
-      const int bhq = bh_q0 + st / nsteps_h;  // query head of this step
+      const int ib = ib_n, bhq = bhq_n;  // this step's query tile and head
       uint8_t* dst = s_stream + stage * C::STAGE_BYTES;
       if (lane == 0) {
         // Q (and U_Q) first on bar_full, dO on bar_full_b
@@ -1194,26 +1226,17 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
           tma_load_3d(dst + soff<C::NSTREAM, false>(na, 0, b), &p.tm[C::NSTAT + na],
                       &m->bar_full_b[stage], 64 * b, ib, bhq);
       }
-      // negated row vectors of the streamed query rows:
-      // [0] -L*log2e, [1] -D, [2] -alpha, [3] -E
       float* vec = reinterpret_cast<float*>(dst + C::TILE_BYTES);
 #pragma unroll
-      for (int q = 0; q < 2; ++q) {
-        const int c = lane + 32 * q;
-        const int gi = ib + c;
-        const bool ok = gi < N;
-        const size_t ri = (size_t)bhq * N + (ok ? gi : 0);
-        vec[c] = ok ? -p.lse[ri] * kLog2e : 0.f;
-        if constexpr (OP == ColOp::BwdDKDV) {
-          vec[64 + c] = ok ? -p.vec_in[ri] : 0.f;
-        } else {
-          vec[64 + c] = ok ? -p.vec_in[2 * p.bhn + ri] : 0.f;  // D
-          vec[128 + c] = ok ? -p.vec_in[ri] : 0.f;             // alpha
-          vec[192 + c] = ok ? -p.vec_in[p.bhn + ri] : 0.f;     // E
-        }
-      }
+      for (int q = 0; q < 2; ++q)
+#pragma unroll
+        for (int k = 0; k < NV; ++k) vec[64 * k + lane + 32 * q] = vn[q][k];
       mbar_arrive(&m->bar_full_b[stage]);
       issued[stage] = st;
+      if (st + 1 < nprod) {  // the next step's coordinates and row vectors
+        advance(st + 1, ib_n, bhq_n);
+        load_vec(ib_n, bhq_n, vn);
+      }
     }
     if (lane == 0 && *abort_flag) {
       for (int s = 0; s < C::NSTAGES; ++s)
