@@ -40,6 +40,11 @@ CASES = [  # B, H, N, d, causal, window, density, empty block rows, kv heads, dr
     (1, 1, 129, 128, False, None, 0.0, (), None, None),
 ]
 
+SEG_CASES = [  # B, H, N, d, causal, segments, density
+    (1, 2, 700, 128, True, [0, 100, 356, 357, 700], 0.5),
+    (1, 1, 600, 64, False, [0, 300, 600], 0.4),
+]
+
 
 def ids(c):
     B, H, N, d, causal, win, dens, er, hkv, drop = c
@@ -129,3 +134,21 @@ def test_n16k_d128_causal_bsparse_rows_and_key_block():
                              block_mask=bm)
     G.check("kbar[block 40]", G.flat(r["kbar"], heads[0], w.H)[c0:c1], blk[0]["kbar"])
     G.check("vbar[block 40]", G.flat(r["vbar"], heads[0], w.H)[c0:c1], blk[0]["vbar"])
+
+
+@pytest.mark.parametrize("case", SEG_CASES, ids=lambda c: f"N{c[2]}d{c[3]}{'c' if c[4] else ''}s{len(c[5]) - 1}")
+def test_bob_block_sparse_with_packed_sequences(case):
+    """A block mask together with packed sequences: each pair must pass both."""
+    B, H, N, d, causal, seg, dens = case
+    bits = G.inputs(B, H, N, d, seed=9 * N + d)
+    bm = random_blocks(N, dens, N + d)
+    scale = 1 / np.sqrt(d)
+    r = G.run_bob(bits, scale, causal, segments=seg, block_mask=bm)
+    assert r["status"] == 0
+    ref = oracle.bob(*(G.f64(bits[n]) for n in synth.NAMES), scale, causal, segments=seg,
+                     block_mask=bm)
+    for name, x in zip(("qbar", "kbar", "vbar", "dobar", "alpha", "E", "D"), ref):
+        G.check(name, r[name], x)
+    O, _ = oracle.fwd(*(G.f64(bits[n]) for n in ("q", "k", "v")), scale, causal, segments=seg,
+                      block_mask=bm)
+    G.check("O", r["o"], O)

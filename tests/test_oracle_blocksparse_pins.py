@@ -144,3 +144,16 @@ def test_diagonal_only_block_of_size_one_closed_form():
     for n in ("qbar", "kbar", "vbar"):
         assert np.abs(r[n]).max() <= 1e-12, n
     assert np.allclose(r["dobar"], X[6], atol=1e-12)
+
+
+def test_central_fd_with_block_mask_and_packed_sequences():
+    """A block mask and packed sequences at once (both restrict the same rows)."""
+    N, d, bs = 36, 8, 6
+    seg = [0, 10, 25, 36]
+    X = rand_problem(N, d, 1400)
+    bm = block_mask(N, bs, 0.5, 14, (2,))
+    tau = 1 / np.sqrt(d)
+    r = oracle.bob_head(*X, tau, True, segments=seg, block_mask=bm, block_size=bs)
+    fd = pins.bob_central_fd(*X, tau, True, segments=seg, block=(bm, bs))
+    for name, g in zip(("qbar", "kbar", "vbar", "dobar"), fd):
+        assert pins.rel_fro(g, r[name]) <= 1e-6, (name, pins.rel_fro(g, r[name]))
