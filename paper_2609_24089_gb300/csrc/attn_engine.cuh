@@ -1179,24 +1179,26 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
       ib = tile * BN;
       bhq = bh_q0 + st / nsteps_h;
     };
-    // negated row vectors of a step's streamed query rows, two rows per lane:
-    // [0] -L*log2e, [1] -D, [2] -alpha, [3] -E (the first backward: L, D).
-    // They are loaded one step ahead, so their latency passes while the
-    // producer waits for the stage they go to.
+    // row vectors of a step's streamed query rows, two rows per lane, as
+    // loaded: [0] L, [1] D, [2] alpha, [3] E (the first backward: L, D).
+    // They are loaded one step ahead and only written (negated, L scaled by
+    // log2 e) into the stage at the next step: no arithmetic touches them
+    // here, so the loads stay in flight while the producer moves on (a use
+    // right after the load would stall the producer for the whole load
+    // latency every step).  Rows past N read the head's last row; the write
+    // zeroes them.
     constexpr int NV = C::NVEC;
     auto load_vec = [&](int ib, int bhq, float (&v)[2][NV]) {
 #pragma unroll
       for (int q = 0; q < 2; ++q) {
-        const int gi = ib + lane + 32 * q;
-        const bool ok = gi < N;
-        const size_t ri = (size_t)bhq * N + (ok ? gi : 0);
-        v[q][0] = ok ? -p.lse[ri] * kLog2e : 0.f;
+        const size_t ri = (size_t)bhq * N + min(ib + lane + 32 * q, N - 1);
+        v[q][0] = p.lse[ri];
         if constexpr (OP == ColOp::BwdDKDV) {
-          v[q][1] = ok ? -p.vec_in[ri] : 0.f;
+          v[q][1] = p.vec_in[ri];
         } else {
-          v[q][1] = ok ? -p.vec_in[2 * p.bhn + ri] : 0.f;  // D
-          v[q][2] = ok ? -p.vec_in[ri] : 0.f;              // alpha
-          v[q][3] = ok ? -p.vec_in[p.bhn + ri] : 0.f;      // E
+          v[q][1] = p.vec_in[2 * p.bhn + ri];  // D
+          v[q][2] = p.vec_in[ri];              // alpha
+          v[q][3] = p.vec_in[p.bhn + ri];      // E
         }
       }
     };
@@ -1228,9 +1230,12 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
       }
       float* vec = reinterpret_cast<float*>(dst + C::TILE_BYTES);
 #pragma unroll
-      for (int q = 0; q < 2; ++q)
+      for (int q = 0; q < 2; ++q) {
+        const bool ok = ib + lane + 32 * q < N;
 #pragma unroll
-        for (int k = 0; k < NV; ++k) vec[64 * k + lane + 32 * q] = vn[q][k];
+        for (int k = 0; k < NV; ++k)
+          vec[64 * k + lane + 32 * q] = ok ? -(k == 0 ? vn[q][k] * kLog2e : vn[q][k]) : 0.f;
+      }
       mbar_arrive(&m->bar_full_b[stage]);
       issued[stage] = st;
       if (st + 1 < nprod) {  // the next step's coordinates and row vectors
