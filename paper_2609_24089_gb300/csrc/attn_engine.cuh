@@ -88,6 +88,7 @@ struct Misc {
   uint64_t bar_ew[4];   // [DC buffer][half]; a single DC buffer uses [0..1]
   uint64_t bar_xb[2];   // issuer X's stage-B MMAs completed (per half, or per DC buffer)
   uint64_t bar_acc;
+  uint64_t bar_xsf[2];  // issuer X's part of SF(t) completed (per SF buffer; row statistics kernel)
   uint32_t tmem_base;
   uint32_t pad;
   WaitCtl wctl;
@@ -347,6 +348,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
     for (int h = 0; h < 2; ++h) {
       mbar_init(&m->bar_sa_dc[h], 1);
       mbar_init(&m->bar_xb[h], 1);
+      mbar_init(&m->bar_xsf[h], 1);
     }
     for (int h = 0; h < 4; ++h) mbar_init(&m->bar_ew[h], kEwThreads);
     mbar_init(&m->bar_acc, 2);
@@ -499,7 +501,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
             for (int k = 0; k < D / 16; ++k)  // [S | F] = Q [K ; U_K]^T
               mma_ts(R + 0, tmem + kColQT + 8 * k, kd(kd0, 0, 0, k), id_n128, k > 0);
 #pragma unroll
-            for (int k = 0; k < D / 16; ++k)  // F += U_Q K^T
+            for (int k = 0; k < D / 32; ++k)  // F += U_Q K^T, first half of the K-steps
               mma_ts(R + 64, tmem + kColQT + D / 2 + 8 * k, kd(kd0, 0, 0, k), id_n64, 1);
           } else if constexpr (kB4) {
             // stationary: 0 Q, 1 U_Q, 2 dO ; stream: 0 K, 1 U_K, 2 V, 3 U_V
@@ -523,7 +525,9 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         if constexpr (kStats) {
           // two SF buffers (tile t in buffer t & 1), so X runs up to a tile
           // ahead of the elementwise warps; no stage B, so a stage is released
-          // as soon as the MMAs reading it complete
+          // as soon as the MMAs reading it complete.  Issuer Y adds the second
+          // half of F += U_Q K^T once X's part has completed (12 MMAs per tile
+          // on each issuer), and signals SF(t)
           for (int st = 0; ok && st < nsteps; ++st) {
             const int b = st & 1;
             const int stage = st % C::NSTAGES;
@@ -532,7 +536,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
               break;
             tc_fence_after();
             stage_sf(st, b ? kColSF1 : kColSF);
-            mma_commit(&m->bar_sa_sf[b]);
+            mma_commit(&m->bar_xsf[b]);
             mma_commit(&m->bar_empty[stage]);
           }
           ok = false;
@@ -615,22 +619,34 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         };
         bool ok = mbar_wait(&m->bar_stat, 0, wctl) && nsteps > 0 && wait_stage(0, 0);
         if constexpr (kStats) {
-          // DC(t+1) once the elementwise warps hold DC(t) in registers
+          // tile t: the second half of F += U_Q K^T once issuer X's part of
+          // SF(t) has completed (then SF(t) is whole), and DC(t), for t + 1
+          // once the elementwise warps hold DC(t) in registers
+          auto tile_y = [&](int t) -> bool {
+            const int b = t & 1;
+            if (!mbar_wait(&m->bar_xsf[b], (t >> 1) & 1, wctl)) return false;
+            tc_fence_after();
+            const uint32_t sb = smem_u32(s_stream + (t % C::NSTAGES) * C::STAGE_BYTES);
+            const uint64_t kd0 = sdesc_sw128(sb, 16, 1024);
+            const uint32_t R = tmem + (b ? kColSF1 : kColSF);
+#pragma unroll
+            for (int k = D / 32; k < D / 16; ++k)  // F += U_Q K^T, second half
+              mma_ts(R + 64, tmem + kColQT + D / 2 + 8 * k, kd(kd0, 0, 0, k), id_n64, 1);
+            mma_commit(&m->bar_sa_sf[b]);
+            stage_dc(sb, 0);
+            mma_commit(&m->bar_sa_dc[0]);
+            mma_commit(&m->bar_empty[t % C::NSTAGES]);
+            return true;
+          };
           if (ok) {
             tc_fence_after();
-            stage_dc(smem_u32(s_stream), 0);
-            mma_commit(&m->bar_sa_dc[0]);
-            mma_commit(&m->bar_empty[0]);
+            ok = tile_y(0);
           }
           for (int st = 0; ok && st + 1 < nsteps; ++st) {
             const int ns = (st + 1) % C::NSTAGES;
             if (!mbar_wait(&m->bar_dc_free, st & 1, wctl) ||
-                !wait_stage(ns, ((st + 1) / C::NSTAGES) & 1))
+                !wait_stage(ns, ((st + 1) / C::NSTAGES) & 1) || !tile_y(st + 1))
               break;
-            tc_fence_after();
-            stage_dc(smem_u32(s_stream + ns * C::STAGE_BYTES), 0);
-            mma_commit(&m->bar_sa_dc[0]);
-            mma_commit(&m->bar_empty[ns]);
           }
           ok = false;  // no stage B
         }
