@@ -88,7 +88,10 @@ struct Misc {
   uint64_t bar_ew[4];   // [DC buffer][half]; a single DC buffer uses [0..1]
   uint64_t bar_xb[2];   // issuer X's stage-B MMAs completed (per half, or per DC buffer)
   uint64_t bar_acc;
-  uint64_t bar_xsf[2];  // issuer X's part of SF(t) completed (per SF buffer; row statistics kernel)
+  // issuer X's per-tile signal to issuer Y, per parity of the tile: its part
+  // of SF(t) completed (row statistics kernel), or SF(t+1) issued (Pass 2
+  // with P o h in SF)
+  uint64_t bar_xsig[2];
   uint32_t tmem_base;
   uint32_t pad;
   WaitCtl wctl;
@@ -348,7 +351,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
     for (int h = 0; h < 2; ++h) {
       mbar_init(&m->bar_sa_dc[h], 1);
       mbar_init(&m->bar_xb[h], 1);
-      mbar_init(&m->bar_xsf[h], 1);
+      mbar_init(&m->bar_xsig[h], 1);
     }
     for (int h = 0; h < 4; ++h) mbar_init(&m->bar_ew[h], kEwThreads);
     mbar_init(&m->bar_acc, 2);
@@ -536,7 +539,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
               break;
             tc_fence_after();
             stage_sf(st, b ? kColSF1 : kColSF);
-            mma_commit(&m->bar_xsf[b]);
+            mma_commit(&m->bar_xsig[b]);
             mma_commit(&m->bar_empty[stage]);
           }
           ok = false;
@@ -624,7 +627,7 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
           // once the elementwise warps hold DC(t) in registers
           auto tile_y = [&](int t) -> bool {
             const int b = t & 1;
-            if (!mbar_wait(&m->bar_xsf[b], (t >> 1) & 1, wctl)) return false;
+            if (!mbar_wait(&m->bar_xsig[b], (t >> 1) & 1, wctl)) return false;
             tc_fence_after();
             const uint32_t sb = smem_u32(s_stream + (t % C::NSTAGES) * C::STAGE_BYTES);
             const uint64_t kd0 = sdesc_sw128(sb, 16, 1024);
@@ -1156,6 +1159,7 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
     for (int h = 0; h < 2; ++h) {
       mbar_init(&m->bar_sa_dc[h], 1);
       mbar_init(&m->bar_xb[h], 1);
+      mbar_init(&m->bar_xsig[h], 1);
     }
     for (int h = 0; h < 4; ++h) mbar_init(&m->bar_ew[h], kEwThreads);
     mbar_init(&m->bar_acc, 2);
@@ -1367,6 +1371,8 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
               tc_fence_after();
               stage_sf(st + 1);
               mma_commit(&m->bar_sa_sf[0]);
+              // SF(t+1) is in the tensor pipe ahead of issuer Y's MMAs of tile t
+              mbar_arrive(&m->bar_xsig[st & 1]);
             }
             continue;
           }
@@ -1458,6 +1464,9 @@ __global__ void __launch_bounds__(kThreads, 1) col_engine(const __grid_constant_
             if (!wait_stage(nx % C::NSTAGES, (nx / C::NSTAGES) & 1) ||
                 (C::XSHARE && !mbar_wait(&m->bar_xb[dc_sel(st)], dc_par(st), wctl)))
               break;
+            // with P o h in SF: the elementwise warps wait for SF(t+1) first and
+            // DC(t+1) only after P o h, so DC(t+1) enters the pipe after SF(t+1)
+            if (C::PH_SF && !mbar_wait(&m->bar_xsig[st & 1], (st >> 1) & 1, wctl)) break;
             tc_fence_after();
             stage_dc(nx);
           }
