@@ -132,14 +132,23 @@ void debug_controls(EngineParams* p) {
 }
 
 // CTA order per kernel (heads per group, cta_order in attn_engine.cuh), from
-// measurements on GB300: groups of four heads suit Pass 1 (the CTAs in flight
-// share four heads' K/V streams in L2, and no head's longest row blocks are
-// left to the end: 0.4 % faster than head-major, 2 % faster than all heads);
-// Pass 2 and the helper kernels balance the causal work better with every
-// head's longest block first (all heads).
+// measurements on GB300.  Pass 1 takes heads in groups whose streamed K, U_K,
+// V, U_V (4 N d bf16 per head) fit in about 96 MiB of the 129 MB L2, at most
+// four: the CTAs in flight then share a few heads' streams in L2 and no
+// head's longest row blocks are left to the end (n16k_d128_causal, 16.8 MB
+// per head: groups of four, 0.4 % faster than one head at a time and 2 %
+// faster than all heads; N = 262,144 at d = 64, 134 MB per head: one head at
+// a time, 4.4 % faster than groups of four).  Pass 2 and the helper kernels
+// balance the causal work better with every head's longest block first (all
+// heads).
 void choose_order(EngineParams* p, int heads_per_group) {
   p->head_group = heads_per_group < 1 ? 1 : (heads_per_group > p->BH ? p->BH : heads_per_group);
   if (p->head_group < 1) p->head_group = 1;
+}
+int pass1_heads_per_group(const fbob_shape* s) {
+  const double per_head = 8.0 * (double)s->N * (double)s->d;  // bytes streamed per head
+  const double g = 96.0 * 1048576.0 / (per_head > 1.0 ? per_head : 1.0);
+  return g >= 4.0 ? 4 : (g >= 1.0 ? (int)g : 1);
 }
 
 // key/value heads per batch entry
@@ -212,7 +221,7 @@ bool row_bob_params(const fbob_shape* s, const void* q, const void* k, const voi
   p->dout = static_cast<const __nv_bfloat16*>(dout);
   p->lse = lse;
   p->nblk = n_blocks(s->N, BM);
-  choose_order(p, 4);
+  choose_order(p, pass1_heads_per_group(s));
   return true;
 }
 
