@@ -341,8 +341,9 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
     for (int s = 0; s < C::NSTAGES; ++s) {
       mbar_init(&m->bar_full[s], 1);
       mbar_init(&m->bar_full_b[s], 1);
-      mbar_init(&m->bar_empty[s], 2);  // released by both MMA issuers
     }
+    // released by both MMA issuers, per stage or (C::HALF_REL) per 32-key half
+    for (int s = 0; s < (C::HALF_REL ? 2 : 1) * C::NSTAGES; ++s) mbar_init(&m->bar_empty[s], 2);
     for (int b = 0; b < 2; ++b) {
       mbar_init(&m->bar_sa_sf[b], 1);
       mbar_init(&m->bar_sf_free[b], kEwThreads);
@@ -382,10 +383,12 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
                       &m->bar_stat, 64 * b, i0, bh);
       int issued[kMaxStages] = {-1, -1, -1, -1};
       int tile = first_tile - 1;
-      for (int st = 0; st < nsteps; ++st) {
+      bool go = true;
+      for (int st = 0; go && st < nsteps; ++st) {
         const int stage = st % C::NSTAGES;
-        if (st >= C::NSTAGES) {
-          if (!mbar_wait(&m->bar_empty[stage], ((st / C::NSTAGES) - 1) & 1, wctl)) break;
+        const uint32_t epar = ((st / C::NSTAGES) - 1) & 1;
+        if (st >= C::NSTAGES && !C::HALF_REL) {
+          if (!mbar_wait(&m->bar_empty[stage], epar, wctl)) break;
         }
         tile = tiles.next(tile + 1);
         const int j0 = tile * BN;
@@ -394,20 +397,40 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
         // BoB: K and U_K first on bar_full (all issuer X needs), then V and
         // U_V on bar_full_b; the other operations use bar_full alone
         const int nt_a = kB4 ? 2 : nt;
-        mbar_arrive_expect_tx(&m->bar_full[stage], nt_a * C::KB * BN * 128);
-        for (int b = 0; b < C::KB; ++b)
-          for (int t = 0; t < nt_a; ++t)
-            tma_load_3d(dst + soff<C::NSTREAM, kB4>(t, 0, b), &p.tm[C::NSTAT + t],
-                        &m->bar_full[stage], 64 * b, j0, bh_kv);
-        if (kB4) {  // 32-row chunks (map box rows HB)
-          mbar_arrive_expect_tx(&m->bar_full_b[stage], 2 * C::KB * BN * 128);
+        if (!kB4) {
+          mbar_arrive_expect_tx(&m->bar_full[stage], nt_a * C::KB * BN * 128);
           for (int b = 0; b < C::KB; ++b)
-            for (int t = 2; t < 4; ++t)
-              for (int h = 0; h < 2; ++h)
+            for (int t = 0; t < nt_a; ++t)
+              tma_load_3d(dst + soff<C::NSTREAM, kB4>(t, 0, b), &p.tm[C::NSTAT + t],
+                          &m->bar_full[stage], 64 * b, j0, bh_kv);
+          issued[stage] = st;
+        } else {
+          // every streamed tensor in 32-row chunks (map box rows HB), half h
+          // of the tile (keys 32 h ..) after the other; with C::HALF_REL each
+          // half of the stage is refilled as soon as its own release comes.
+          // The full barriers are armed only once half 0 is released: that
+          // release implies the stage's previous phase completed.
+          for (int h = 0; h < 2; ++h) {
+            if (C::HALF_REL && st >= C::NSTAGES &&
+                !mbar_wait(&m->bar_empty[2 * stage + h], epar, wctl)) {
+              go = false;
+              break;
+            }
+            if (h == 0) {
+              mbar_arrive_expect_tx(&m->bar_full[stage], 2 * C::KB * BN * 128);
+              mbar_arrive_expect_tx(&m->bar_full_b[stage], 2 * C::KB * BN * 128);
+              issued[stage] = st;  // (a stage left half loaded drains by its time limit)
+            }
+            for (int b = 0; b < C::KB; ++b)
+              for (int t = 0; t < 2; ++t)
+                tma_load_3d(dst + soff<C::NSTREAM, kB4>(t, h, b), &p.tm[C::NSTAT + t],
+                            &m->bar_full[stage], 64 * b, j0 + HB * h, bh_kv);
+            for (int b = 0; b < C::KB; ++b)
+              for (int t = 2; t < 4; ++t)
                 tma_load_3d(dst + soff<C::NSTREAM, kB4>(t, h, b), &p.tm[C::NSTAT + t],
                             &m->bar_full_b[stage], 64 * b, j0 + HB * h, bh_kv);
+          }
         }
-        issued[stage] = st;
       }
       if (*abort_flag) {  // drain loads still in flight
         for (int s = 0; s < C::NSTAGES; ++s)
@@ -556,7 +579,14 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
           // without XSHARE, X's last read of this stage was SF(t), already
           // issued: release the stage when that completes (a commit after
           // SF(t+1) would hold it until SF(t+1) completes, a tile later)
-          if (!C::XSHARE) mma_commit(&m->bar_empty[stage]);
+          if (!C::XSHARE) {
+            if (C::HALF_REL) {
+              mma_commit(&m->bar_empty[2 * stage]);
+              mma_commit(&m->bar_empty[2 * stage + 1]);
+            } else {
+              mma_commit(&m->bar_empty[stage]);
+            }
+          }
           if (more) {  // SF(t+1) once the elementwise warps hold SF(t)
             if (!mbar_wait(&m->bar_sf_free[0], st & 1, wctl) ||
                 !mbar_wait(&m->bar_full[(st + 1) % C::NSTAGES], ((st + 1) / C::NSTAGES) & 1, wctl))
@@ -713,7 +743,11 @@ __global__ void __launch_bounds__(kThreads, 1) row_engine(const __grid_constant_
             }
             tc_fence_after();
             stage_b(sb, h, st, C::XSHARE ? 1 : 2);
-            if (h == 1) mma_commit(&m->bar_empty[stage]);
+            // issuer Y's last read of the stage (of its half h with C::HALF_REL)
+            if (C::HALF_REL)
+              mma_commit(&m->bar_empty[2 * stage + h]);
+            else if (h == 1)
+              mma_commit(&m->bar_empty[stage]);
             if (more && (kDcHalves || h == 1)) {
               if ((h == 0 || !kDcHalves) && !wait_stage(nstage, ((st + 1) / C::NSTAGES) & 1)) {
                 ok = false;

@@ -110,6 +110,12 @@ struct RowCfg {
   // the dQ kernel's DC tile (dP, 64 columns) leaves the other half of the DC
   // area free: two dP buffers, dP(t+2) issued right after stage B(t)
   static constexpr bool DC2 = OP == RowOp::BwdDQ;
+  // the direct form's stream stages are released per 32-key half: half h of
+  // tile t's stage is free once stage B(t) of half h has run, and the
+  // producer refills it with half h of tile t + NSTAGES at once (with only
+  // two 64 KB stages its loads otherwise land late for issuer X)
+  // (d = 128; at d = 64 three stages already keep the loads ahead)
+  static constexpr bool HALF_REL = OP == RowOp::BobPass1D && 2 * NSTAGES <= kMaxStages;
   // bookkeeping (256), the row-sum exchange (4 x BM floats), the rows' D (BM floats)
   static constexpr int MISC_BYTES = 2816;
   static constexpr int SMEM_BYTES = STAT_BYTES + NSTAGES * STAGE_BYTES + MISC_BYTES;

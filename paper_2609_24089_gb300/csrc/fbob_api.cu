@@ -213,8 +213,9 @@ bool row_bob_params(const fbob_shape* s, const void* q, const void* k, const voi
   for (int t = 0; t < 3; ++t)
     if (!make_map(&p->tm[t], stat[t], BH, N, d, BM)) return false;
   const int64_t BHk = s->B * kv_heads(s);
+  // streamed tiles in 32-row chunks (two per 64-key tile)
   for (int t = 0; t < 4; ++t)
-    if (!make_map(&p->tm[3 + t], strm[t], BHk, N, d, t < 2 ? BN : HB)) return false;
+    if (!make_map(&p->tm[3 + t], strm[t], BHk, N, d, HB)) return false;
   p->q = static_cast<const __nv_bfloat16*>(q);
   p->uq = static_cast<const __nv_bfloat16*>(gq);
   p->o = static_cast<const __nv_bfloat16*>(o);
