@@ -43,6 +43,11 @@ CONTRACTIONS = {"pass1": 11, "pass1_fused": 11, "row_stats": 5, "pass1_direct": 
 KERNEL_NAMES = {"pass1": "row_engine<BobPass1>", "pass1_fused": "row_engine<BobPass1>",
                 "row_stats": "row_engine<BobStats>", "pass1_direct": "row_engine<BobPass1D>",
                 "pass2": "col_engine<BobPass2>"}
+# head dimension 256 (wide_engine.cuh): the direct form and Pass 2 are two
+# kernels each (dOtil and Qtil; Vtil and Ktil), timed together per entry call
+WIDE_KERNEL_NAMES = {"row_stats": "wide_engine<Stats>",
+                     "pass1_direct": "wide_engine<DOut> + wide_engine<DQ>",
+                     "pass2": "wide_engine<P2V> + wide_engine<P2K>"}
 ENTRY_NAMES = {"pass1": "bob_pass1", "pass1_fused": "bob_pass1_fused",
                "row_stats": "bob_row_stats", "pass1_direct": "bob_pass1_direct",
                "pass2": "bob_pass2"}
@@ -291,7 +296,7 @@ def run_gpu(args, w):
 
     # ---- timed region: K steps, each as its kernels (through their C-ABI
     # calls, the same ones fbob_attn_bob makes) with events between them
-    if args.pass1 == "fused" and not drop:  # one-sweep Pass 1 (Prop. 3.1) at any d
+    if args.pass1 == "fused" and not drop and w.d <= 128:  # one-sweep Pass 1 (Prop. 3.1)
         parts = [("pass1_fused", lambda: fbob.fbob_attn_bob_pass1_fused(
             shp, q, k, v, o, lse, do, gq, gk, gv, outs[0], outs[3], rs))]
     elif w.d <= 64 and not drop and args.pass1 != "stats_direct":
@@ -372,7 +377,8 @@ def run_gpu(args, w):
     # ms at most, at the clocks sampled below); the sustained figure (a
     # seconds-long cuBLAS loop under the power cap) is kept as a second number
     peak = peaks["bf16"]
-    roofline = {"bound": "tensor", "kernel": KERNEL_NAMES[dom], "achieved": achieved,
+    kname = WIDE_KERNEL_NAMES[dom] if w.d == 256 else KERNEL_NAMES[dom]
+    roofline = {"bound": "tensor", "kernel": kname, "achieved": achieved,
                 "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
                 "peak_kind": f"bf16 burst ({peaks['source']})",
                 "frac_of_sustained": achieved / peaks["bf16_sustained"],

@@ -10,7 +10,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libfbob.so")
-UNITS = ("fbob_api.cu", "row_kernels.cu", "col_kernels.cu")
+UNITS = ("fbob_api.cu", "row_kernels.cu", "col_kernels.cu", "wide_kernels.cu")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr"]
 

@@ -32,11 +32,18 @@ constexpr float kLn2 = 0.6931471805599453f;
 // (Fwd names the forward for the launcher; it runs in fwd_engine.cuh.)
 enum class RowOp { Fwd, BwdDQ, BobPass1, BobStats, BobPass1D };
 enum class ColOp { BwdDKDV, BobPass2 };
+// Head dimension 256 (wide_engine.cuh): FwdL, FwdO the forward's two sweeps
+// (L, then O); Stats, DOut, DQ BoB Pass 1 (alpha E D, dOtil, Qtil); P2V, P2K
+// BoB Pass 2 (Vtil, Ktil); BwdDQ, BwdDV, BwdDK the first backward.
+enum class WOp { FwdL, FwdO, Stats, DOut, DQ, BwdDQ, P2V, P2K, BwdDV, BwdDK };
 
 // ---------------------------------------------------------------- parameters
 struct EngineParams {
   CUtensorMap tm[7];  // stationary maps first (box rows BM), then streamed (box rows BN)
-  const __nv_bfloat16* q;     // Q and U_Q (row statistics kernel: stationary A operands)
+  // Q and U_Q; in the kernels that hold stationary MMA A operands in TMEM
+  // (the row statistics kernel, every head-dimension-256 kernel) the sources
+  // of those operands: Q, U_Q in the row kernels, K, V in the column kernels
+  const __nv_bfloat16* q;
   const __nv_bfloat16* uq;
   const __nv_bfloat16* o;     // forward output O (row engine: D and dOtil)
   const __nv_bfloat16* dout;  // dO (row engine: D = do.o)

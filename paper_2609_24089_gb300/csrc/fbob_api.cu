@@ -84,7 +84,7 @@ int check_shape(const fbob_shape* s, bool* empty) {
                                 : (s->num_seqs < 1 || s->num_seqs > kMaxN ||
                                    (reinterpret_cast<uintptr_t>(s->seq_offsets) & 3u) != 0))
     return FBOB_ERR_INVALID_ARGUMENT;
-  if (s->d != 32 && s->d != 64 && s->d != 128) return FBOB_ERR_UNSUPPORTED;
+  if (s->d != 32 && s->d != 64 && s->d != 128 && s->d != 256) return FBOB_ERR_UNSUPPORTED;
   if (s->N > kMaxN) return FBOB_ERR_INVALID_ARGUMENT;
   if (s->B > kMaxBH || s->H > kMaxBH || s->B * s->H > kMaxBH) return FBOB_ERR_INVALID_ARGUMENT;
   // the largest launch (two CTAs per 128-row block for the split one-sweep
@@ -198,6 +198,108 @@ EngineParams base_params(const fbob_shape* s) {
 
 int launch_status(cudaError_t e) { return e == cudaSuccess ? FBOB_OK : FBOB_ERR_CUDA; }
 
+// ---- head dimension 256 (wide_engine.cuh): stationary shared-memory
+// operands in 128-row boxes, streamed tensors in 32-row boxes; the kernels'
+// TMEM operands are read through p.q / p.uq
+
+int run_wide(WOp op, const EngineParams& p, bool drop, int nblocks, cudaStream_t st) {
+  return launch_status(launch_wide(op, drop, p, nblocks, st));
+}
+
+// maps[t] = (tensor, heads, box rows)
+struct MapSpec {
+  const void* base;
+  int64_t heads;
+  int rows;
+};
+bool wide_maps(EngineParams* p, const fbob_shape* s, const MapSpec* spec, int n) {
+  for (int t = 0; t < n; ++t)
+    if (!make_map(&p->tm[t], spec[t].base, spec[t].heads, s->N, s->d, spec[t].rows)) return false;
+  return true;
+}
+
+// Pass 1 at d = 256: `parts` 1 = the row scalars alpha, E, D (eq. 6); 2 =
+// dOtil and Qtil from eqs. (6)-(7) with row_stats given; 3 = both.
+int run_pass1_wide(const fbob_shape* s, const void* q, const void* k, const void* v,
+                   const void* o, const float* lse, const void* dout, const void* gq,
+                   const void* gk, const void* gv, void* q_bar, void* dout_bar, float* row_stats,
+                   cudaStream_t st, int64_t head0, int parts) {
+  const int64_t BH = s->B * s->H, BHk = s->B * kv_heads(s);
+  EngineParams p = base_params(s);
+  p.head0 = (int)head0;
+  p.lse = lse;
+  p.nblk = n_blocks(s->N, BM);
+  choose_order(&p, pass1_heads_per_group(s));
+  const bool drop = has_dropout(s);
+  const int nb = p.nblk * p.BH;
+  int rc = FBOB_OK;
+  if (parts & 1) {  // alpha, E, D: Q, U_Q in TMEM; dO; K, U_K, V, U_V streamed
+    EngineParams a = p;
+    a.q = static_cast<const __nv_bfloat16*>(q);
+    a.uq = static_cast<const __nv_bfloat16*>(gq);
+    a.o = static_cast<const __nv_bfloat16*>(o);
+    a.dout = static_cast<const __nv_bfloat16*>(dout);
+    a.vec_out = row_stats;
+    const MapSpec m[5] = {{dout, BH, BM}, {k, BHk, HB}, {gk, BHk, HB}, {v, BHk, HB}, {gv, BHk, HB}};
+    if (!wide_maps(&a, s, m, 5)) return FBOB_ERR_CUDA;
+    rc = run_wide(WOp::Stats, a, drop, nb, st);
+    if (rc != FBOB_OK) return rc;
+  }
+  if (parts & 2) {
+    // dOtil: Q in TMEM; U_Q; K, U_K, V, U_V streamed
+    EngineParams a = p;
+    a.q = static_cast<const __nv_bfloat16*>(q);
+    a.vec_in = row_stats;
+    a.out0 = static_cast<__nv_bfloat16*>(dout_bar);
+    const MapSpec ma[5] = {{gq, BH, BM}, {k, BHk, HB}, {gk, BHk, HB}, {v, BHk, HB}, {gv, BHk, HB}};
+    if (!wide_maps(&a, s, ma, 5)) return FBOB_ERR_CUDA;
+    rc = run_wide(WOp::DOut, a, drop, nb, st);
+    if (rc != FBOB_OK) return rc;
+    // Qtil: Q in TMEM; U_Q, dO; K, U_K streamed; V, U_V in a ring of their own
+    EngineParams b = p;
+    b.q = static_cast<const __nv_bfloat16*>(q);
+    b.vec_in = row_stats;
+    b.out0 = static_cast<__nv_bfloat16*>(q_bar);
+    const MapSpec mb[6] = {{gq, BH, BM}, {dout, BH, BM}, {k, BHk, HB},
+                           {gk, BHk, HB}, {v, BHk, HB},  {gv, BHk, HB}};
+    if (!wide_maps(&b, s, mb, 6)) return FBOB_ERR_CUDA;
+    rc = run_wide(WOp::DQ, b, drop, nb, st);
+  }
+  return rc;
+}
+
+// Pass 2 at d = 256: Vtil (K in TMEM; U_K; Q, U_Q, dO streamed), then Ktil
+// over two CTAs per key block (K, V in TMEM; U_K, U_V; Q, U_Q streamed; dO
+// in a ring of its own).
+int run_pass2_wide(const fbob_shape* s, const void* q, const void* k, const void* v,
+                   const float* lse, const void* dout, const void* gq, const void* gk,
+                   const void* gv, const float* row_stats, void* k_bar, void* v_bar,
+                   cudaStream_t st, int64_t head0) {
+  const int64_t BH = s->B * s->H, BHk = s->B * kv_heads(s);
+  EngineParams p = base_params(s);
+  p.head0 = (int)head0;
+  p.BH = (int)BHk;  // one CTA column per key/value head
+  p.lse = lse;
+  p.vec_in = row_stats;
+  p.nblk = n_blocks(s->N, BM);
+  choose_order(&p, p.BH);
+  const bool drop = has_dropout(s);
+  EngineParams a = p;
+  a.q = static_cast<const __nv_bfloat16*>(k);
+  a.out0 = static_cast<__nv_bfloat16*>(v_bar);
+  const MapSpec ma[4] = {{gk, BHk, BM}, {q, BH, HB}, {gq, BH, HB}, {dout, BH, HB}};
+  if (!wide_maps(&a, s, ma, 4)) return FBOB_ERR_CUDA;
+  int rc = run_wide(WOp::P2V, a, drop, p.nblk * p.BH, st);
+  if (rc != FBOB_OK) return rc;
+  EngineParams b = p;
+  b.q = static_cast<const __nv_bfloat16*>(k);
+  b.uq = static_cast<const __nv_bfloat16*>(v);
+  b.out0 = static_cast<__nv_bfloat16*>(k_bar);
+  const MapSpec mb[5] = {{gk, BHk, BM}, {gv, BHk, BM}, {q, BH, HB}, {gq, BH, HB}, {dout, BH, HB}};
+  if (!wide_maps(&b, s, mb, 5)) return FBOB_ERR_CUDA;
+  return run_wide(WOp::P2K, b, drop, 2 * p.nblk * p.BH, st);
+}
+
 // ---- the individual launches (arguments already validated)
 
 // Tensor maps and pointers shared by the row-block BoB kernels: stationary
@@ -265,6 +367,9 @@ int run_pass1(const fbob_shape* s, const void* q, const void* k, const void* v, 
               const float* lse, const void* dout, const void* gq, const void* gk,
               const void* gv, void* q_bar, void* dout_bar, float* row_stats,
               cudaStream_t st, int64_t head0 = 0) {
+  if (s->d == 256)
+    return run_pass1_wide(s, q, k, v, o, lse, dout, gq, gk, gv, q_bar, dout_bar, row_stats, st,
+                          head0, 3);
   EngineParams p;
   if (!row_bob_params(s, q, k, v, o, lse, dout, gq, gk, gv, &p)) return FBOB_ERR_CUDA;
   p.head0 = (int)head0;
@@ -279,13 +384,18 @@ int run_pass1(const fbob_shape* s, const void* q, const void* k, const void* v, 
   return run_pass1_direct(p, (int)s->d, drop, row_stats, q_bar, dout_bar, st);
 }
 
-// kernels one pass-1 call enqueues
-int pass1_launches(const fbob_shape* s) { return pass1_one_sweep(s) ? 1 : 2; }
+// kernels one pass-1 / pass-2 call enqueues
+int pass1_launches(const fbob_shape* s) {
+  return s->d == 256 ? 3 : pass1_one_sweep(s) ? 1 : 2;
+}
+int pass2_launches(const fbob_shape* s) { return s->d == 256 ? 2 : 1; }
 
 int run_pass2(const fbob_shape* s, const void* q, const void* k, const void* v, const float* lse,
               const void* dout, const void* gq, const void* gk, const void* gv,
               const float* row_stats, void* k_bar, void* v_bar, cudaStream_t st,
               int64_t head0 = 0) {
+  if (s->d == 256)
+    return run_pass2_wide(s, q, k, v, lse, dout, gq, gk, gv, row_stats, k_bar, v_bar, st, head0);
   EngineParams p = base_params(s);
   p.head0 = (int)head0;
   const int64_t BH = s->B * s->H, N = s->N, d = s->d;
@@ -490,6 +600,28 @@ int fbob_attn_fwd(const fbob_shape* s, const void* q, const void* k, const void*
   const int64_t outb[2] = {mat, vec};
   rc = check_ptrs(in, inb, 3, out, outb, 2);
   if (rc != FBOB_OK) return rc;
+  if (s->d == 256) {
+    // two sweeps: L (over the ungated probabilities), then O with L known
+    const int64_t BHk = s->B * kv_heads(s);
+    EngineParams p = base_params(s);
+    p.q = static_cast<const __nv_bfloat16*>(q);
+    p.nblk = n_blocks(s->N, BM);
+    choose_order(&p, p.BH);
+    EngineParams a = p;
+    a.vec_out = lse;
+    const MapSpec ma[1] = {{k, BHk, HB}};
+    if (!wide_maps(&a, s, ma, 1)) return FBOB_ERR_CUDA;
+    rc = run_wide(WOp::FwdL, a, false, p.nblk * p.BH, stream);
+    if (rc != FBOB_OK) return rc;
+    EngineParams b = p;
+    b.lse = lse;
+    b.out0 = static_cast<__nv_bfloat16*>(o);
+    const MapSpec mb[2] = {{k, BHk, HB}, {v, BHk, HB}};
+    if (!wide_maps(&b, s, mb, 2)) return FBOB_ERR_CUDA;
+    rc = run_wide(WOp::FwdO, b, has_dropout(s), p.nblk * p.BH, stream);
+    if (rc == FBOB_OK) g_launches[kEntFwd] = 2;
+    return rc;
+  }
   EngineParams p = base_params(s);
   const int64_t BH = s->B * s->H, BHk = s->B * kv_heads(s);
   if (!make_map(&p.tm[0], q, BH, s->N, s->d, BM) ||
@@ -522,6 +654,44 @@ int fbob_attn_bwd(const fbob_shape* s, const void* q, const void* k, const void*
   const int64_t outb[4] = {mat, matk, matk, vec};
   rc = check_ptrs(in, inb, 6, out, outb, 4);
   if (rc != FBOB_OK) return rc;
+  if (s->d == 256) {
+    // dQ and D (row blocks), then dV and dK (key blocks, one kernel each)
+    const int64_t BH = s->B * s->H, BHk = s->B * kv_heads(s);
+    const bool drop = has_dropout(s);
+    EngineParams p = base_params(s);
+    p.q = static_cast<const __nv_bfloat16*>(q);
+    p.o = static_cast<const __nv_bfloat16*>(o);
+    p.dout = static_cast<const __nv_bfloat16*>(dout);
+    p.lse = lse;
+    p.out0 = static_cast<__nv_bfloat16*>(dq);
+    p.vec_out = dstat;
+    p.nblk = n_blocks(s->N, BM);
+    choose_order(&p, p.BH);
+    const MapSpec mq[3] = {{dout, BH, BM}, {k, BHk, HB}, {v, BHk, HB}};
+    if (!wide_maps(&p, s, mq, 3)) return FBOB_ERR_CUDA;
+    rc = run_wide(WOp::BwdDQ, p, drop, p.nblk * p.BH, stream);
+    if (rc != FBOB_OK) return rc;
+    EngineParams c = base_params(s);
+    c.BH = (int)BHk;  // one CTA column per key/value head
+    c.q = static_cast<const __nv_bfloat16*>(k);
+    c.lse = lse;
+    c.vec_in = dstat;
+    c.nblk = n_blocks(s->N, BM);
+    choose_order(&c, c.BH);
+    EngineParams cv = c;
+    cv.out0 = static_cast<__nv_bfloat16*>(dv);
+    const MapSpec mv[2] = {{q, BH, HB}, {dout, BH, HB}};
+    if (!wide_maps(&cv, s, mv, 2)) return FBOB_ERR_CUDA;
+    rc = run_wide(WOp::BwdDV, cv, drop, c.nblk * c.BH, stream);
+    if (rc != FBOB_OK) return rc;
+    EngineParams ck = c;
+    ck.out0 = static_cast<__nv_bfloat16*>(dk);
+    const MapSpec mk[3] = {{v, BHk, BM}, {q, BH, HB}, {dout, BH, HB}};
+    if (!wide_maps(&ck, s, mk, 3)) return FBOB_ERR_CUDA;
+    rc = run_wide(WOp::BwdDK, ck, drop, c.nblk * c.BH, stream);
+    if (rc == FBOB_OK) g_launches[kEntBwd] = 3;
+    return rc;
+  }
   const int64_t BH = s->B * s->H, BHk = s->B * kv_heads(s), N = s->N, d = s->d;
   // dQ and D: row-block pass (writes D, which the column pass reads)
   EngineParams p = base_params(s);
@@ -585,7 +755,9 @@ int fbob_attn_bob_pass1_fused(const fbob_shape* s, const void* q, const void* k,
   bool empty = false;
   int rc = check_shape(s, &empty);
   if (rc != FBOB_OK) return rc;
-  if (has_dropout(s)) return FBOB_ERR_UNSUPPORTED;
+  // with dropout, or at d = 256 (four 256-column accumulators), the one-sweep
+  // form does not fit
+  if (has_dropout(s) || s->d == 256) return FBOB_ERR_UNSUPPORTED;
   if (empty) {
     g_launches[kEntPass1Fused] = 0;
     return FBOB_OK;
@@ -626,7 +798,7 @@ int fbob_attn_bob_pass2(const fbob_shape* s, const void* q, const void* k, const
   rc = check_ptrs(in2, inb2, 9, out, outb, 2);
   if (rc != FBOB_OK) return rc;
   rc = run_pass2(s, q, k, v, lse, dout, gq, gk, gv, row_stats, k_bar, v_bar, stream);
-  if (rc == FBOB_OK) g_launches[kEntPass2] = 1;
+  if (rc == FBOB_OK) g_launches[kEntPass2] = pass2_launches(s);
   return rc;
 }
 
@@ -649,6 +821,12 @@ int fbob_attn_bob_row_stats(const fbob_shape* s, const void* q, const void* k, c
   const int64_t outb[1] = {3 * vec};
   rc = check_ptrs(in, inb, 9, out, outb, 1);
   if (rc != FBOB_OK) return rc;
+  if (s->d == 256) {
+    rc = run_pass1_wide(s, q, k, v, o, lse, dout, gq, gk, gv, nullptr, nullptr, row_stats, stream,
+                        0, 1);
+    if (rc == FBOB_OK) g_launches[kEntRowStats] = 1;
+    return rc;
+  }
   EngineParams p;
   if (!row_bob_params(s, q, k, v, o, lse, dout, gq, gk, gv, &p)) return FBOB_ERR_CUDA;
   rc = run_row_stats(p, (int)s->d, has_dropout(s), row_stats, stream);
@@ -675,6 +853,12 @@ int fbob_attn_bob_pass1_direct(const fbob_shape* s, const void* q, const void* k
   const int64_t outb[2] = {mat, mat};
   rc = check_ptrs(in, inb, 9, out, outb, 2);
   if (rc != FBOB_OK) return rc;
+  if (s->d == 256) {
+    rc = run_pass1_wide(s, q, k, v, nullptr, lse, dout, gq, gk, gv, q_bar, dout_bar,
+                        const_cast<float*>(row_stats), stream, 0, 2);
+    if (rc == FBOB_OK) g_launches[kEntPass1D] = 2;
+    return rc;
+  }
   EngineParams p;
   // (o is not read: D comes from row_stats)
   if (!row_bob_params(s, q, k, v, nullptr, lse, dout, gq, gk, gv, &p)) return FBOB_ERR_CUDA;
@@ -708,7 +892,7 @@ int fbob_attn_bob(const fbob_shape* s, const void* q, const void* k, const void*
   // Pass 2 (column blocks): Ktil, Vtil from the saved row state.  Stream
   // order is the only synchronisation between the passes.
   rc = run_pass2(s, q, k, v, lse, dout, gq, gk, gv, row_stats, k_bar, v_bar, stream);
-  if (rc == FBOB_OK) g_launches[kEntBob] = pass1_launches(s) + 1;
+  if (rc == FBOB_OK) g_launches[kEntBob] = pass1_launches(s) + pass2_launches(s);
   return rc;
 }
 
@@ -805,7 +989,7 @@ int fbob_attn_bob_host(const fbob_shape* s, const void* q, const void* k, const 
       rc = run_pass2(&csh, w[0], w[1], w[2], static_cast<const float*>(w[4]), w[5], w[6], w[7],
                      w[8], static_cast<const float*>(w[13]), w[10], w[11], cs, f0);
     if (rc != FBOB_OK) return rc;
-    launches += pass1_launches(&csh) + 1;
+    launches += pass1_launches(&csh) + pass2_launches(&csh);
     // copy out once computed
     e = cudaEventRecord(hcall.comp[sl], cs);
     if (e == cudaSuccess) e = cudaStreamWaitEvent(hcall.cout, hcall.comp[sl], 0);
@@ -887,7 +1071,7 @@ int fbob_attn_bob_host_noalloc(const fbob_shape* s, const void* q, const void* k
       rc = run_pass2(&cs, w[0], w[1], w[2], static_cast<const float*>(w[4]), w[5], w[6], w[7],
                      w[8], static_cast<const float*>(w[13]), w[10], w[11], st, f0);
     if (rc != FBOB_OK) return rc;
-    launches += pass1_launches(&cs) + 1;
+    launches += pass1_launches(&cs) + pass2_launches(&cs);
     e = d2h(hbm(q_bar, f0 * nd), w[9], nq * nd);
     if (e == cudaSuccess) e = d2h(hbm(dout_bar, f0 * nd), w[12], nq * nd);
     if (e == cudaSuccess) e = d2h(hbm(k_bar, k0 * nd), w[10], nkv * nd);
@@ -905,10 +1089,11 @@ int fbob_attn_bob_host_noalloc(const fbob_shape* s, const void* q, const void* k
 int fbob_device_status(struct CUstream_st* stream) {
   cudaError_t e = cudaStreamSynchronize(stream);
   if (e != cudaSuccess) return FBOB_ERR_DEVICE_FAULT;
-  uint32_t w1 = 0, w2 = 0;
-  if (take_row_error(&w1, stream) != cudaSuccess || take_col_error(&w2, stream) != cudaSuccess)
+  uint32_t w1 = 0, w2 = 0, w3 = 0;
+  if (take_row_error(&w1, stream) != cudaSuccess || take_col_error(&w2, stream) != cudaSuccess ||
+      take_wide_error(&w3, stream) != cudaSuccess)
     return FBOB_ERR_CUDA;
-  const uint32_t w = w1 | w2;
+  const uint32_t w = w1 | w2 | w3;
   if (w & kDevErrTimeout) return FBOB_ERR_DEVICE_TIMEOUT;
   if (w) return FBOB_ERR_DEVICE_FAULT;
   return FBOB_OK;

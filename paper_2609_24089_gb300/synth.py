@@ -95,7 +95,7 @@ WORKLOADS["n16k_d128_causal_drop10"] = Workload(
 
 # head-dimension sweep at the shape of the paper's sensitivity table
 # (App. "Head-dimension sensitivity": N = 4096, B = 4, H = 12, causal)
-for _d in (32, 64, 128):
+for _d in (32, 64, 128, 256):
     WORKLOADS[f"n4k_d{_d}_causal_b4h12"] = Workload(
         f"n4k_d{_d}_causal_b4h12", 4, 12, 4096, _d, True, 9, _s(1, 1, 1, 1, 1, 1, 1))
 
@@ -105,6 +105,11 @@ for _d in (32, 64, 128):
 WORKLOADS["n16k_d128_causal_bsparse"] = Workload(
     "n16k_d128_causal_bsparse", 2, 16, 16384, 128, True, 10,
     _s(1, 1, 1, *(4 * [1 / math.sqrt(128)])), blocks=(2, 1, 0.1, 10))
+
+# head dimension 256 (App. "Head-dimension sensitivity" names it as the next
+# specialisation): the causal headline shape at one batch entry and 8 heads
+WORKLOADS["n16k_d256_causal"] = Workload(
+    "n16k_d256_causal", 1, 8, 16384, 256, True, 11, _s(1, 1, 1, *(4 * [1 / math.sqrt(256)])))
 
 WORKLOADS["n16k_d128_causal_varlen"] = Workload(
     "n16k_d128_causal_varlen", 2, 16, 16384, 128, True, 6,

@@ -50,7 +50,12 @@ def test_rejects_bad_shapes(lib):
     S = fbob.make_shape
     assert bob(lib, S(1, 1, 128, 48, 0.14, 0), ptrs(14)) == 2          # d unsupported
     assert bob(lib, S(1, 1, 128, 16, 0.25, 0), ptrs(14)) == 2
-    assert bob(lib, S(1, 1, 128, 256, 0.06, 1), ptrs(14)) == 2
+    assert bob(lib, S(1, 1, 128, 512, 0.04, 1), ptrs(14)) == 2
+    assert bob(lib, S(1, 1, 128, 96, 0.1, 1), ptrs(14)) == 2
+    # d = 256 is supported, except by the one-sweep Pass 1 (four 256-column
+    # accumulators do not fit TMEM), which refuses it before any CUDA call
+    fused = lib.fbob_attn_bob_pass1_fused
+    assert fused(ctypes.byref(S(1, 1, 128, 256, 0.0625, 1)), *ptrs(13), None) == 2
     assert bob(lib, S(1, 1, 128, 64, 0.0, 0), ptrs(14)) == 1           # scale <= 0
     assert bob(lib, S(1, 1, 128, 64, float("nan"), 0), ptrs(14)) == 1
     assert bob(lib, S(1, 1, 128, 64, float("inf"), 0), ptrs(14)) == 1

@@ -212,7 +212,7 @@ def test_lemma_d2_embedding_on_gpu():
         assert np.abs(r[n]).max() == 0.0, n
 
 
-@pytest.mark.parametrize("d,causal", [(64, False), (128, True)])
+@pytest.mark.parametrize("d,causal", [(64, False), (128, True), (256, True)])
 def test_single_key_degenerate(d, causal):
     """N = 1: P = 1, so Qtil = Ktil = Vtil = 0 and dOtil = U_V exactly.  The
     fused form Qtil = tau (Omega - alpha R - E B) cancels to zero only up to
@@ -250,6 +250,10 @@ STALL_CASES = [  # entry, d, causal, dropout
     ("bwd", 64, True, None),      # first backward: dQ (row) and dK/dV (column) kernels
     ("bwd", 128, False, None),
     ("bwd", 128, True, (0.1, 4)),
+    ("bob", 256, True, None),     # head dim 256: the five wide kernels of BoB
+    ("bob", 256, False, (0.1, 6)),
+    ("fwd", 256, True, None),     # the forward's two sweeps
+    ("bwd", 256, False, (0.1, 7)),  # dQ, dV and dK kernels
 ]
 
 
