@@ -16,9 +16,12 @@
  *  Pointers   Device pointers (global memory of the current device), each
  *             16-byte aligned.  Outputs must not overlap any input or each
  *             other.
- *  Shapes     d in {32, 64, 128}; other head dims return FBOB_ERR_UNSUPPORTED.
- *             (d = 32 runs in the kernels' 64-wide tiles, the missing
- *             columns loaded as zeros.)
+ *  Shapes     d in {32, 64, 128, 256}; other head dims return
+ *             FBOB_ERR_UNSUPPORTED.  (d = 32 runs in the kernels' 64-wide
+ *             tiles, the missing columns loaded as zeros.  d = 256, App.
+ *             "Head-dimension sensitivity", runs in kernels of its own with
+ *             32-row streamed tiles and one accumulator per kernel; each
+ *             entry point below states its launches there.)
  *             N >= 0 is arbitrary (tails are masked); B*H*N == 0 is a valid
  *             empty problem that launches nothing and returns FBOB_OK.
  *             N <= 2^24, B*H <= 2^24 and ceil(N/128) * B*H * 2 < 2^31 (the
@@ -117,7 +120,7 @@ struct CUstream_st; /* cudaStream_t == struct CUstream_st* */
 typedef enum fbob_status {
     FBOB_OK = 0,
     FBOB_ERR_INVALID_ARGUMENT = 1, /* null/misaligned/overlapping pointer, bad shape, scale */
-    FBOB_ERR_UNSUPPORTED = 2,      /* valid request the library does not implement (d not 32/64/128) */
+    FBOB_ERR_UNSUPPORTED = 2,      /* valid request the library does not implement (d not 32/64/128/256) */
     FBOB_ERR_CUDA = 3,             /* a CUDA runtime/driver call or launch failed */
     FBOB_ERR_DEVICE_TIMEOUT = 4,   /* a bounded device-side wait expired */
     FBOB_ERR_DEVICE_FAULT = 5,     /* the device reported an error while synchronising */
@@ -144,6 +147,7 @@ typedef struct fbob_shape {
  *   S = scale * Q K^T + M,  P = softmax_row(S),  O = P V,
  *   lse_i = L_i = log sum_{j valid} exp(S_ij)   (natural log, fp32).
  * In:  q, k, v  bf16 [B,H,N,d].   Out: o bf16 [B,H,N,d], lse fp32 [B,H,N].
+ * One kernel; at d = 256 two sweeps (lse, then o with lse known).
  */
 int fbob_attn_fwd(const fbob_shape* shape, const void* q, const void* k, const void* v,
                   void* o, float* lse, struct CUstream_st* stream);
@@ -155,6 +159,8 @@ int fbob_attn_fwd(const fbob_shape* shape, const void* q, const void* k, const v
  * P is recomputed from q, k and lse.  D (fp32, from the given o and dout) is
  * written to dstat [B,H,N].
  * In:  q, k, v, o, dout bf16; lse fp32.   Out: dq, dk, dv bf16; dstat fp32.
+ * Two kernels (dq and dstat by row blocks, dk and dv by key blocks); at
+ * d = 256 three (dq and dstat, dv, dk).
  */
 int fbob_attn_bwd(const fbob_shape* shape, const void* q, const void* k, const void* v,
                   const void* o, const float* lse, const void* dout,
@@ -164,9 +170,12 @@ int fbob_attn_bwd(const fbob_shape* shape, const void* q, const void* k, const v
  * Backward-over-backward, Sec. 3.1 eqs. (4)-(5) and closed form eqs. (6)-(7):
  *   Phi = <dQ, U_Q> + <dK, U_K> + <dV, U_V>,
  *   (q_bar, k_bar, v_bar, dout_bar) = grad_{Q, K, V, dO} Phi,
- * computed by the two-pass schedule of Algorithm 1 (row-block pass, then
- * column-block pass) with the affine fusion of Prop. 3.1 / eq. (8).  No N x N
- * tensor is written to memory.
+ * computed by the row-block pass, then the column-block pass of Algorithm 1:
+ * pass 1 as fbob_attn_bob_pass1 describes (one sweep with the affine fusion
+ * of Prop. 3.1 / eq. (8) at d <= 64 without dropout; otherwise the row
+ * scalars first, then the direct form of eqs. (6)-(7)), pass 2 as
+ * fbob_attn_bob_pass2: 2 kernels at d <= 64, 3 at d = 128 or with dropout,
+ * 5 at d = 256.  No N x N tensor is written to memory.
  * In:  q, k, v, o, dout, gq, gk, gv  bf16 [B,H,N,d]; lse fp32 [B,H,N] (natural
  *      log, as written by fbob_attn_fwd).
  * Out: q_bar, k_bar, v_bar, dout_bar bf16 [B,H,N,d];
@@ -186,7 +195,7 @@ int fbob_attn_bob(const fbob_shape* shape, const void* q, const void* k, const v
  * rules as fbob_attn_bob; k_bar/v_bar are not touched.  d <= 64 without
  * dropout runs one sweep with the affine fusion of Prop. 3.1 (one kernel);
  * d = 128, and any d with dropout, runs fbob_attn_bob_row_stats then
- * fbob_attn_bob_pass1_direct (two kernels).
+ * fbob_attn_bob_pass1_direct (two kernels; three at d = 256).
  */
 int fbob_attn_bob_pass1(const fbob_shape* shape, const void* q, const void* k, const void* v,
                         const void* o, const float* lse, const void* dout,
@@ -204,7 +213,9 @@ int fbob_attn_bob_pass1(const fbob_shape* shape, const void* q, const void* k, c
  * tau (Omega - alpha G - E0 B).  At d = 128 the four accumulators are split
  * by output column over two CTAs per row block (each computes the whole
  * stage A and its 64 columns of stage B).  One kernel.  Same arguments and
- * outputs as fbob_attn_bob_pass1; dropout returns FBOB_ERR_UNSUPPORTED.
+ * outputs as fbob_attn_bob_pass1; dropout, and d = 256 (four 256-column
+ * accumulators exceed tensor memory), return FBOB_ERR_UNSUPPORTED before any
+ * CUDA call.
  */
 int fbob_attn_bob_pass1_fused(const fbob_shape* shape, const void* q, const void* k,
                               const void* v, const void* o, const float* lse, const void* dout,
@@ -214,7 +225,8 @@ int fbob_attn_bob_pass1_fused(const fbob_shape* shape, const void* q, const void
 /*
  * Pass 2 of Algorithm 1 alone (column-block outer; Alg. 2, second loop):
  * reads row_stats (alpha, E, D, as pass 1 writes them) and lse, writes
- * k_bar and v_bar.  row_stats is an input here.
+ * k_bar and v_bar.  row_stats is an input here.  One kernel; at d = 256 two
+ * (v_bar, then k_bar over two CTAs per key block, 128 output columns each).
  */
 int fbob_attn_bob_pass2(const fbob_shape* shape, const void* q, const void* k, const void* v,
                         const float* lse, const void* dout,
@@ -239,7 +251,8 @@ int fbob_attn_bob_row_stats(const fbob_shape* shape, const void* q, const void* 
  * Pass 1 given its row scalars: q_bar and dout_bar from eqs. (6)-(7) directly,
  *   q_bar = scale (Stil K + dS U_K),  dout_bar = P U_V + (P o h) V,
  * with alpha, E, D read from row_stats (as fbob_attn_bob_row_stats or pass 1
- * writes them; input here) and P from lse.  O is not needed.
+ * writes them; input here) and P from lse.  O is not needed.  One kernel; at
+ * d = 256 two (dout_bar, then q_bar).
  * In:  q, k, v, dout, gq, gk, gv bf16; lse fp32; row_stats fp32 [3,B,H,N].
  * Out: q_bar, dout_bar bf16 [B,H,N,d].
  */
