@@ -43,9 +43,11 @@ CONTRACTIONS = {"pass1": 11, "pass1_fused": 11, "row_stats": 5, "pass1_direct": 
 KERNEL_NAMES = {"pass1": "row_engine<BobPass1>", "pass1_fused": "row_engine<BobPass1>",
                 "row_stats": "row_engine<BobStats>", "pass1_direct": "row_engine<BobPass1D>",
                 "pass2": "col_engine<BobPass2>"}
-# head dimension 256 (wide_engine.cuh): the direct form and Pass 2 are two
-# kernels each (dOtil and Qtil; Vtil and Ktil), timed together per entry call
-WIDE_KERNEL_NAMES = {"row_stats": "wide_engine<Stats>",
+# head dimension 256 (wide_engine.cuh): Pass 1 is two kernels (the row scalars
+# with dOtil in one sweep, then Qtil), the direct form two (dOtil, Qtil) and
+# Pass 2 two (Vtil, Ktil), timed together per entry call
+WIDE_KERNEL_NAMES = {"pass1": "wide_engine<StatsDO> + wide_engine<DQ>",
+                     "row_stats": "wide_engine<Stats>",
                      "pass1_direct": "wide_engine<DOut> + wide_engine<DQ>",
                      "pass2": "wide_engine<P2V> + wide_engine<P2K>"}
 ENTRY_NAMES = {"pass1": "bob_pass1", "pass1_fused": "bob_pass1_fused",
@@ -299,6 +301,10 @@ def run_gpu(args, w):
     if args.pass1 == "fused" and not drop and w.d <= 128:  # one-sweep Pass 1 (Prop. 3.1)
         parts = [("pass1_fused", lambda: fbob.fbob_attn_bob_pass1_fused(
             shp, q, k, v, o, lse, do, gq, gk, gv, outs[0], outs[3], rs))]
+    elif w.d == 256 and args.pass1 != "stats_direct":
+        # d = 256: row scalars with dOtil in one sweep, then Qtil (as fbob_attn_bob_pass1)
+        parts = [("pass1", lambda: fbob.fbob_attn_bob_pass1(
+            shp, q, k, v, o, lse, do, gq, gk, gv, outs[0], outs[3], rs))]
     elif w.d <= 64 and not drop and args.pass1 != "stats_direct":
         # one-sweep Pass 1 (as fbob_attn_bob_pass1 chooses)
         parts = [("pass1", lambda: fbob.fbob_attn_bob_pass1(
@@ -422,7 +428,9 @@ def run_gpu(args, w):
         "clocks": clk.summary(),
         "peak_hbm_bytes": footprint,
         "call_alloc_bytes": call_delta,
-        "pass1_form": ("one sweep, affine fusion (Prop. 3.1)"
+        "pass1_form": ("row scalars and dOtil in one sweep (eq. 8), then Qtil (eqs. 6-7)"
+                       if w.d == 256 and parts[0][0] == "pass1"
+                       else "one sweep, affine fusion (Prop. 3.1)"
                        if parts[0][0] in ("pass1", "pass1_fused")
                        else "row statistics + direct form (eqs. 6-7)"),
         "pass_ms": {"pass1": total - part_ms["pass2"], "pass2": part_ms["pass2"]},

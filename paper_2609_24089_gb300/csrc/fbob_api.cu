@@ -219,7 +219,9 @@ bool wide_maps(EngineParams* p, const fbob_shape* s, const MapSpec* spec, int n)
 }
 
 // Pass 1 at d = 256: `parts` 1 = the row scalars alpha, E, D (eq. 6); 2 =
-// dOtil and Qtil from eqs. (6)-(7) with row_stats given; 3 = both.
+// dOtil and Qtil from eqs. (6)-(7) with row_stats given; 3 = the whole pass:
+// alpha, E, D with dOtil in one sweep (dOtil0 = P U_V + (P o F) V needs no
+// row scalar; dOtil = dOtil0 - alpha o, eq. 8), then Qtil.
 int run_pass1_wide(const fbob_shape* s, const void* q, const void* k, const void* v,
                    const void* o, const float* lse, const void* dout, const void* gq,
                    const void* gk, const void* gv, void* q_bar, void* dout_bar, float* row_stats,
@@ -233,7 +235,21 @@ int run_pass1_wide(const fbob_shape* s, const void* q, const void* k, const void
   const bool drop = has_dropout(s);
   const int nb = p.nblk * p.BH;
   int rc = FBOB_OK;
-  if (parts & 1) {  // alpha, E, D: Q, U_Q in TMEM; dO; K, U_K, V, U_V streamed
+  if (parts == 3) {
+    // alpha, E, D and dOtil: Q in TMEM; U_Q, dO; (K, U_K) and (V, U_V) streamed as pairs
+    EngineParams a = p;
+    a.q = static_cast<const __nv_bfloat16*>(q);
+    a.o = static_cast<const __nv_bfloat16*>(o);
+    a.dout = static_cast<const __nv_bfloat16*>(dout);
+    a.vec_out = row_stats;
+    a.out0 = static_cast<__nv_bfloat16*>(dout_bar);
+    const MapSpec ma[6] = {{gq, BH, BM}, {dout, BH, BM}, {k, BHk, HB},
+                           {gk, BHk, HB}, {v, BHk, HB},  {gv, BHk, HB}};
+    if (!wide_maps(&a, s, ma, 6)) return FBOB_ERR_CUDA;
+    rc = run_wide(WOp::StatsDO, a, drop, nb, st);
+    if (rc != FBOB_OK) return rc;
+  }
+  if (parts == 1) {  // alpha, E, D: Q, U_Q in TMEM; dO; K, U_K, V, U_V streamed
     EngineParams a = p;
     a.q = static_cast<const __nv_bfloat16*>(q);
     a.uq = static_cast<const __nv_bfloat16*>(gq);
@@ -245,7 +261,7 @@ int run_pass1_wide(const fbob_shape* s, const void* q, const void* k, const void
     rc = run_wide(WOp::Stats, a, drop, nb, st);
     if (rc != FBOB_OK) return rc;
   }
-  if (parts & 2) {
+  if (parts == 2) {
     // dOtil: Q in TMEM; U_Q; K, U_K, V, U_V streamed
     EngineParams a = p;
     a.q = static_cast<const __nv_bfloat16*>(q);
@@ -255,6 +271,8 @@ int run_pass1_wide(const fbob_shape* s, const void* q, const void* k, const void
     if (!wide_maps(&a, s, ma, 5)) return FBOB_ERR_CUDA;
     rc = run_wide(WOp::DOut, a, drop, nb, st);
     if (rc != FBOB_OK) return rc;
+  }
+  if (parts & 2) {
     // Qtil: Q in TMEM; U_Q, dO; K, U_K streamed; V, U_V in a ring of their own
     EngineParams b = p;
     b.q = static_cast<const __nv_bfloat16*>(q);
@@ -386,7 +404,7 @@ int run_pass1(const fbob_shape* s, const void* q, const void* k, const void* v, 
 
 // kernels one pass-1 / pass-2 call enqueues
 int pass1_launches(const fbob_shape* s) {
-  return s->d == 256 ? 3 : pass1_one_sweep(s) ? 1 : 2;
+  return s->d == 256 ? 2 : pass1_one_sweep(s) ? 1 : 2;
 }
 int pass2_launches(const fbob_shape* s) { return s->d == 256 ? 2 : 1; }
 

@@ -47,8 +47,10 @@ namespace fbob {
 
 // WOp (engine_params.h): FwdL: L (eq. 1, first sweep); FwdO: O with L known
 // (second sweep).  Stats: alpha, E, D (eq. 6); DOut: dOtil; DQ: Qtil (eqs.
-// 6-7).  BwdDQ: dQ and D; BwdDV: dV; BwdDK: dK (eqs. 2-3).  P2V: Vtil; P2K:
-// Ktil (Alg. 2, second loop; eq. 7).
+// 6-7).  StatsDO: alpha, E, D and dOtil in one sweep: dOtil0 = P U_V +
+// (P o F) V needs no row scalar, and dOtil = dOtil0 - alpha o (Prop. 3.1,
+// eq. 8).  BwdDQ: dQ and D; BwdDV: dV; BwdDK: dK (eqs. 2-3).  P2V: Vtil;
+// P2K: Ktil (Alg. 2, second loop; eq. 7).
 
 constexpr int WD = 256;               // head dimension of these kernels
 constexpr int WKB = WD / 64;          // 64-column boxes per row
@@ -62,17 +64,27 @@ constexpr int kWStat = WKB * BM * 128;  // one stationary 128 x 256 bf16 tensor 
 // vectors of the streamed rows (column kernels).  SF: SFW columns per buffer,
 // NSF buffers; DC likewise.  ACC_N accumulator columns.  SPLIT CTAs per
 // stationary block (each its ACC_N output columns).
+//
+// PAIR (StatsDO): the four streamed tensors travel as two pairs, (K, U_K)
+// read only by SF and (V, U_V) read by DC and stage B, through one ring of
+// NSA 32 KB slots in the order KU(0), VU(0), KU(1), VU(1), ...; each slot is
+// released by the one issuer that reads its pair last (X after SF, Y after
+// stage B), so with three slots tile t+1's pairs load while tile t runs
+// (KU(t+1) reuses the slot of VU(t-1), VU(t+1) that of KU(t)).
 template <WOp OP>
 struct WCfg {
+  static constexpr bool PAIR = OP == WOp::StatsDO;
   static constexpr bool ROW = OP == WOp::FwdL || OP == WOp::FwdO || OP == WOp::Stats ||
-                              OP == WOp::DOut || OP == WOp::DQ || OP == WOp::BwdDQ;
+                              OP == WOp::DOut || OP == WOp::DQ || OP == WOp::BwdDQ || PAIR;
   static constexpr int NTT = (OP == WOp::Stats || OP == WOp::P2K) ? 2 : 1;
   static constexpr int NTS = (OP == WOp::FwdL || OP == WOp::FwdO || OP == WOp::BwdDV) ? 0
-                             : (OP == WOp::DQ || OP == WOp::P2K)                     ? 2
+                             : (OP == WOp::DQ || OP == WOp::P2K || PAIR)             ? 2
                                                                                      : 1;
+  // (PAIR: tensors per slot; the maps hold K, U_K, then V, U_V)
   static constexpr int NTA = (OP == WOp::Stats || OP == WOp::DOut) ? 4
                              : OP == WOp::P2V                        ? 3
-                             : (OP == WOp::FwdO || OP == WOp::DQ || OP == WOp::P2K || OP == WOp::BwdDV)
+                             : (OP == WOp::FwdO || OP == WOp::DQ || OP == WOp::P2K ||
+                                OP == WOp::BwdDV || PAIR)
                                  ? 2
                                  : 1;
   static constexpr int NTB = OP == WOp::DQ ? 2
@@ -85,18 +97,18 @@ struct WCfg {
                                                  : 0;
   static constexpr int NSA = (OP == WOp::Stats || OP == WOp::DOut || OP == WOp::DQ || OP == WOp::P2K)
                                  ? 2
-                             : OP == WOp::P2V ? 3
-                                              : 4;
+                             : (OP == WOp::P2V || PAIR) ? 3
+                                                        : 4;
   static constexpr int NSB = NTB == 0 ? 0 : OP == WOp::DQ ? 1 : OP == WOp::P2K ? 2 : 4;
   static constexpr int SFW = (OP == WOp::Stats || OP == WOp::DOut || OP == WOp::DQ ||
-                              OP == WOp::P2V || OP == WOp::P2K)
+                              OP == WOp::P2V || OP == WOp::P2K || PAIR)
                                  ? 64   // [S | F]
                                  : 32;  // S
-  static constexpr int NSF = (OP == WOp::DQ || OP == WOp::P2K) ? 1 : 2;
-  static constexpr int DCW = (OP == WOp::Stats || OP == WOp::DQ || OP == WOp::P2K) ? 64  // [dP | C]
+  static constexpr int NSF = (OP == WOp::DQ || OP == WOp::P2K || PAIR) ? 1 : 2;
+  static constexpr int DCW = (OP == WOp::Stats || OP == WOp::DQ || OP == WOp::P2K || PAIR) ? 64  // [dP | C]
                              : (OP == WOp::BwdDQ || OP == WOp::BwdDK)              ? 32  // dP
                                                                                    : 0;
-  static constexpr int NDC = DCW == 0 ? 0 : (OP == WOp::DQ || OP == WOp::P2K) ? 1 : 2;
+  static constexpr int NDC = DCW == 0 ? 0 : (OP == WOp::DQ || OP == WOp::P2K || PAIR) ? 1 : 2;
   static constexpr int NDC1 = NDC > 0 ? NDC : 1;  // (divisor where there is no DC)
   static constexpr int ACC_N = (OP == WOp::FwdL || OP == WOp::Stats) ? 0 : OP == WOp::P2K ? 128 : 256;
   static constexpr int SPLIT = OP == WOp::P2K ? 2 : 1;
@@ -104,14 +116,15 @@ struct WCfg {
   static constexpr bool OPS_SF = OP == WOp::FwdO || OP == WOp::DOut || OP == WOp::P2V ||
                                  OP == WOp::BwdDV;
   static constexpr bool OPS_DC = OP == WOp::DQ || OP == WOp::BwdDQ || OP == WOp::P2K ||
-                                 OP == WOp::BwdDK;
+                                 OP == WOp::BwdDK || PAIR;
   static constexpr bool HAS_B = ACC_N > 0;
-  // issuer Y reads ring A (stage B, or the statistics kernel's DC)
-  static constexpr bool Y_READS_A = HAS_B || OP == WOp::Stats;
+  // issuer Y reads ring A (stage B, or the statistics kernel's DC); with
+  // PAIR each slot has one releasing issuer
+  static constexpr bool Y_READS_A = (HAS_B || OP == WOp::Stats) && !PAIR;
   // D = do . o summed in the prologue; alpha / E0 row sums (or the online
   // maximum and sum) exchanged between the two warpgroups
-  static constexpr bool ROW_DOTS = OP == WOp::Stats || OP == WOp::BwdDQ;
-  static constexpr bool XCHG = OP == WOp::Stats || OP == WOp::FwdL;
+  static constexpr bool ROW_DOTS = OP == WOp::Stats || OP == WOp::BwdDQ || PAIR;
+  static constexpr bool XCHG = OP == WOp::Stats || OP == WOp::FwdL || PAIR;
 
   // TMEM columns
   static constexpr uint32_t ACC_COL = 128u * NTT;
@@ -284,6 +297,28 @@ __global__ void __launch_bounds__(kThreads, 1) wide_engine(const __grid_constant
       tile = tiles.next(tile + 1);
       const int row = tile * WBN;
       const int hs = stream_head(st);
+      if constexpr (C::PAIR) {
+        // pair pr of tile st (0: K, U_K; 1: V, U_V) at ring position 2 st + pr
+        bool go = true;
+        for (int pr = 0; pr < 2; ++pr) {
+          const int pos = 2 * st + pr, sl = pos % C::NSA, use = pos / C::NSA;
+          if (use >= 1 && !mbar_wait(&m->empty_a[sl], (use - 1) & 1, wctl)) {
+            go = false;
+            break;
+          }
+          if (lane == 0) {
+            uint8_t* dst = s_a + sl * C::STAGE_A;
+            mbar_arrive_expect_tx(&m->full_a[sl], C::STAGE_A);
+            for (int b = 0; b < WKB; ++b)
+              for (int t = 0; t < 2; ++t)
+                tma_load_3d(dst + (b * 2 + t) * kWBox, &p.tm[C::NTS + 2 * pr + t], &m->full_a[sl],
+                            64 * b, row, hs);
+          }
+          issued_a[sl] = pos;
+        }
+        if (!go) break;
+        continue;
+      }
       // ring A
       const int sa = st % C::NSA;
       if (st >= C::NSA && !mbar_wait(&m->empty_a[sa], ((st / C::NSA) - 1) & 1, wctl)) break;
@@ -369,12 +404,14 @@ __global__ void __launch_bounds__(kThreads, 1) wide_engine(const __grid_constant
       if (warp == kMmaWarp) {
         // ---------------- issuer X: SF(t)
         for (int st = 0; ok && st < nsteps; ++st) {
-          const int b = st % C::NSF, sa = st % C::NSA;
+          // ring slot of this tile's SF operands and its use count
+          const int apos = C::PAIR ? 2 * st : st;
+          const int b = st % C::NSF, sa = apos % C::NSA;
           if (st >= C::NSF) {
             uint64_t* freed = C::OPS_SF ? &m->sb[b] : &m->sf_read[b];
             if (!mbar_wait(freed, ((st / C::NSF) - 1) & 1, wctl)) break;
           }
-          if (!mbar_wait(&m->full_a[sa], (st / C::NSA) & 1, wctl)) break;
+          if (!mbar_wait(&m->full_a[sa], (apos / C::NSA) & 1, wctl)) break;
           tc_fence_after();
           const uint32_t stg = smem_u32(s_a + sa * C::STAGE_A);
           const uint32_t R = tmem + C::SF_COL + b * C::SFW;
@@ -408,7 +445,13 @@ __global__ void __launch_bounds__(kThreads, 1) wide_engine(const __grid_constant
             return false;
           uint32_t stg;
           int nt, t0;
-          if constexpr (C::NTB > 0) {
+          if constexpr (C::PAIR) {  // V, U_V: pair 1 of tile u
+            const int pos = 2 * u + 1, sl = pos % C::NSA;
+            if (!mbar_wait(&m->full_a[sl], (pos / C::NSA) & 1, wctl)) return false;
+            stg = smem_u32(s_a + sl * C::STAGE_A);
+            nt = 2;
+            t0 = 0;
+          } else if constexpr (C::NTB > 0) {
             const int sbx = u % C::NSB;
             if (!mbar_wait(&m->full_b[sbx], (u / C::NSB) & 1, wctl)) return false;
             stg = smem_u32(s_b + sbx * C::STAGE_B);
@@ -432,13 +475,18 @@ __global__ void __launch_bounds__(kThreads, 1) wide_engine(const __grid_constant
               mma_ss(R + 32, sd(1, k), kd(stg, nt, 0, k), id_n32, k > 0);
           } else {
             // [dP | C] = dO [V ; U_V]^T ; dP = dO V^T ; dP^T = V dO^T
-            constexpr int kA = OP == WOp::DQ ? 1 : 0;  // stationary dO (V for dK)
+            constexpr int kA = (OP == WOp::DQ || C::PAIR) ? 1 : 0;  // stationary dO (V for dK)
 #pragma unroll
             for (int k = 0; k < WD / 16; ++k) mma_ss(R, sd(kA, k), kd(stg, nt, t0, k), id_dc, k > 0);
           }
           mma_commit(&m->dc[b]);
-          if constexpr (C::NTB > 0) mma_commit(&m->empty_b[u % C::NSB]);
-          else mma_commit(&m->empty_a[u % C::NSA]);
+          if constexpr (C::PAIR) {
+            // (V, U_V stay for stage B, which releases them)
+          } else if constexpr (C::NTB > 0) {
+            mma_commit(&m->empty_b[u % C::NSB]);
+          } else {
+            mma_commit(&m->empty_a[u % C::NSA]);
+          }
           return true;
         };
         if constexpr (C::NDC > 0) {
@@ -448,7 +496,8 @@ __global__ void __launch_bounds__(kThreads, 1) wide_engine(const __grid_constant
           if constexpr (C::HAS_B) {
             if (!mbar_wait(&m->ew[st & 1], (st >> 1) & 1, wctl)) break;
             tc_fence_after();
-            const int sa = st % C::NSA;
+            // (PAIR: the slot of V, U_V)
+            const int sa = (C::PAIR ? 2 * st + 1 : st) % C::NSA;
             const uint32_t stg = smem_u32(s_a + sa * C::STAGE_A);
             const uint32_t A = tmem + (C::OPS_SF ? C::SF_COL + (st % C::NSF) * C::SFW
                                                  : C::DC_COL + (st % C::NDC1) * C::DCW);
@@ -475,6 +524,9 @@ __global__ void __launch_bounds__(kThreads, 1) wide_engine(const __grid_constant
                 mma_ts(acc, As, md(stg, C::NTA, 1, s, 0), id_b, first);
               } else if constexpr (OP == WOp::BwdDK) {  // dK += dS^T Q
                 mma_ts(acc, As, md(stg, C::NTA, 0, s, 0), id_b, first);
+              } else if constexpr (C::PAIR) {  // dOtil0 += P U_V + (P o F) V
+                mma_ts(acc, As, md(stg, 2, 1, s, 0), id_b, first);
+                mma_ts(acc, As + 8, md(stg, 2, 0, s, 0), id_b, 1);
               }
             }
             if constexpr (C::OPS_SF) mma_commit(&m->sb[st % C::NSF]);
@@ -659,6 +711,22 @@ __global__ void __launch_bounds__(kThreads, 1) wide_engine(const __grid_constant
           if constexpr (OP == WOp::FwdO || OP == WOp::BwdDV) {  // (sigma R o P)
             const float2 gp = DROP ? __fmul2_rn(pr, g) : pr;
             o0[c / 2] = pack_bf16(gp.x, gp.y);
+          } else if constexpr (C::PAIR) {
+            // alpha += P F ; E0 += P (C + F (dP - D)) (dP, C gated); the
+            // dOtil0 operands sigma R o P and sigma R o P o F
+            const float2 f = __fmul2_rn(pair(rF, c), tauv);
+            float2 dp = pair(rdP, c), cv = pair(rC, c), gp = pr;
+            if constexpr (DROP) {
+              dp = __fmul2_rn(dp, g);
+              cv = __fmul2_rn(cv, g);
+              gp = __fmul2_rn(pr, g);
+            }
+            const float2 pt0 = __ffma2_rn(f, __fadd2_rn(dp, cD), cv);
+            acc_a = __ffma2_rn(pr, f, acc_a);
+            acc_e = __ffma2_rn(pr, pt0, acc_e);
+            const float2 pf = __fmul2_rn(gp, f);
+            o0[c / 2] = pack_bf16(gp.x, gp.y);
+            o1[c / 2] = pack_bf16(pf.x, pf.y);
           } else if constexpr (OP == WOp::Stats) {
             // alpha += P F ; E0 += P (C + F (dP - D))  (dP, C gated)
             const float2 f = __fmul2_rn(pair(rF, c), tauv);
@@ -706,7 +774,8 @@ __global__ void __launch_bounds__(kThreads, 1) wide_engine(const __grid_constant
           // operand tiles over this thread's own SF (or dP) columns just read
           const uint32_t R = C::OPS_SF ? Rsf : Rdc;
           tmem_st8(R, o0);
-          if constexpr (OP == WOp::DOut || OP == WOp::DQ || OP == WOp::P2K) tmem_st8(R + 8, o1);
+          if constexpr (OP == WOp::DOut || OP == WOp::DQ || OP == WOp::P2K || C::PAIR)
+            tmem_st8(R + 8, o1);
           tmem_st_wait();
           tc_fence_before();
           mbar_arrive(&m->ew[st & 1]);
@@ -718,7 +787,7 @@ __global__ void __launch_bounds__(kThreads, 1) wide_engine(const __grid_constant
     if (ok && *abort_flag) ok = false;
     tc_fence_after();
     if constexpr (C::XCHG) {
-      if constexpr (OP == WOp::Stats) {
+      if constexpr (OP == WOp::Stats || C::PAIR) {
         s_xchg[wg * BM + r] = acc_a.x + acc_a.y;
         s_xchg[(2 + wg) * BM + r] = acc_e.x + acc_e.y;
       } else {
@@ -743,6 +812,29 @@ __global__ void __launch_bounds__(kThreads, 1) wide_engine(const __grid_constant
           p.vec_out[ri] = alpha;
           p.vec_out[p.bhn + ri] = E0 - alpha * Dr;  // E = E0 - alpha D
           p.vec_out[2 * p.bhn + ri] = Dr;
+        }
+      } else if constexpr (C::PAIR) {
+        // eq. (8): E = E0 - alpha D, dOtil = dOtil0 - alpha o
+        const float alpha = s_xchg[r] + s_xchg[BM + r];
+        const float E0 = s_xchg[2 * BM + r] + s_xchg[3 * BM + r];
+        if (row_ok && wg == 0) {
+          p.vec_out[ri] = alpha;
+          p.vec_out[p.bhn + ri] = E0 - alpha * Dr;
+          p.vec_out[2 * p.bhn + ri] = Dr;
+        }
+#pragma unroll 1
+        for (int q = 0; q < WD / 32; ++q) {
+          const int cc = wg * (WD / 2) + 16 * q;
+          uint32_t rA[16];
+          tmem_ld16(ta + C::ACC_COL + cc, rA);
+          tmem_ld_wait(rA);
+          if (row_ok) {
+            float ov[16], v[16];
+            load_row16(p.o + rowoff + cc, ov);
+#pragma unroll
+            for (int c = 0; c < 16; ++c) v[c] = nsteps > 0 ? bits_f(rA[c]) - alpha * ov[c] : 0.f;
+            store_row16(p.out0 + rowoff + cc, v);
+          }
         }
       } else {
         // the accumulator's ACC_N columns: warpgroup g stores half of them

@@ -34,6 +34,7 @@ cudaError_t launch_wide(WOp op, bool drop, const EngineParams& p, int nblocks, c
     case WOp::P2K: return launch_op<WOp::P2K>(drop, p, nblocks, s);
     case WOp::BwdDV: return launch_op<WOp::BwdDV>(drop, p, nblocks, s);
     case WOp::BwdDK: return launch_op<WOp::BwdDK>(drop, p, nblocks, s);
+    case WOp::StatsDO: return launch_op<WOp::StatsDO>(drop, p, nblocks, s);
   }
   return cudaErrorInvalidValue;
 }

@@ -18,6 +18,8 @@ CASES = [  # B, H, Hkv, N, d, causal, window, segments, dropout
     (2, 3, None, 200, 64, True, None, None, (0.2, 99)),
     (1, 4, 4, 333, 128, True, (50, -1), [0, 100, 333], None),
     (3, 2, 1, 190, 32, True, None, None, (0.1, 5)),
+    (1, 4, 2, 260, 256, True, None, None, None),       # head dimension 256: four kernels
+    (2, 2, None, 150, 256, False, (60, 30), None, (0.1, 8)),
 ]
 
 
@@ -73,7 +75,7 @@ def test_host_buffers_equal_device_buffers(case, chunk):
     units = B * H // Gq                      # key/value groups
     u = min(-(-units // 4), -(-max(heads, 1) // Gq))  # groups per full chunk the call takes
     nchunks = expected_chunks(B * H, Gq, u * Gq)
-    per_chunk = (1 if (d <= 64 and not drop) else 2) + 1
+    per_chunk = 4 if d == 256 else (1 if (d <= 64 and not drop) else 2) + 1
     assert fbob.fbob_launch_count("bob_host") == nchunks * per_chunk
     for name, got, want in zip(("qbar", "kbar", "vbar", "dobar", "row_stats"), hout, ref):
         assert torch.equal(got, want.cpu()), name
