@@ -273,11 +273,6 @@ __global__ void __launch_bounds__(kThreads, 1) wide_engine(const __grid_constant
   WaitCtl* wctl = &m->wctl;
   volatile int* abort_flag = &m->wctl.abort;
 
-  // streamed tile and head of step st (the cursor restarts for each query head)
-  struct Cursor {
-    int tile;
-  };
-
   if (warp == kProducerWarp) {
     // ------------------------------------------------------------ producer
     const int lane = tid & 31;
