@@ -211,6 +211,35 @@ def cores():
 
 
 # ----------------------------------------------------------------- reference arm
+def caller_bytes(w) -> int:
+    """HBM the caller's tensors of one BoB take: q, dout, gq, o and q_bar,
+    dout_bar [B,H,N,d] bf16; k, v, gk, gv and k_bar, v_bar [B,Hkv,N,d] bf16;
+    lse [B,H,N] and row_stats [3,B,H,N] fp32."""
+    q_side = w.B * w.H * w.N * w.d * 2
+    kv_side = w.B * (w.kv_heads or w.H) * w.N * w.d * 2
+    return 6 * q_side + 6 * kv_side + 4 * w.B * w.H * w.N * 4
+
+
+def workload_config(w, world: int) -> dict:
+    """The `config` object of both arms' JSON lines (identical for the same
+    workload and launch)."""
+    bm = synth.workload_blocks(w)
+    return {"workload": w.name, "B": w.B, "H": w.H, "N": w.N, "d": w.d,
+            "causal": w.causal, "window": list(w.window),
+            "packed_sequences": len(w.segments) - 1 if w.segments else 1,
+            "kv_heads": w.kv_heads or w.H, "seed": w.seed,
+            "dropout": list(w.dropout) if w.dropout else None,
+            "block_mask": ({"local": w.blocks[0], "sinks": w.blocks[1],
+                            "density": w.blocks[2], "seed": w.blocks[3],
+                            "blocks_set": int(bm.sum()), "blocks": int(bm.size)}
+                           if bm is not None else None),
+            "l2": "no flush: inputs (%.2f GB) exceed the 129 MB L2" % (caller_bytes(w) / 1e9),
+            "parallelism": "replicas" if world > 1 else "single GPU",
+            "flop_formula": ("2*19*B*H*d*(valid (i,j) pairs of the band)"
+                             if w.window != (-1, -1) or w.segments or w.blocks
+                             else "2*19*B*H*N^2*d*(1/2 if causal)")}
+
+
 def run_reference(args, w):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
@@ -231,8 +260,7 @@ def run_reference(args, w):
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1e3 * dt / len(per), "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": w.name, "B": w.B, "H": w.H, "N": w.N, "d": w.d,
-                       "causal": w.causal},
+            "config": workload_config(w, int(os.environ.get("WORLD_SIZE", "1"))),
             "cpu_baseline": {"value": val, "unit": "TFLOP/s", "cores": cores(), "kind": "oracle",
                              "sample": desc + " per step"},
             "e2e": {"value": val, "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
@@ -402,20 +430,7 @@ def run_gpu(args, w):
         "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": K,
         "warmup": args.warmup, "ms_per_step": ms_max / K, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": w.name, "B": w.B, "H": w.H, "N": w.N, "d": w.d,
-                   "causal": w.causal, "window": list(w.window),
-                   "packed_sequences": len(w.segments) - 1 if w.segments else 1,
-                   "kv_heads": w.kv_heads or w.H, "seed": w.seed,
-                   "dropout": list(w.dropout) if w.dropout else None,
-                   "block_mask": ({"local": w.blocks[0], "sinks": w.blocks[1],
-                                   "density": w.blocks[2], "seed": w.blocks[3],
-                                   "blocks_set": int(bm.sum()), "blocks": int(bm.size)}
-                                  if bm is not None else None),
-                   "l2": "no flush: inputs (%.2f GB) exceed the 129 MB L2" % (footprint / 1e9),
-                   "parallelism": "replicas" if world > 1 else "single GPU",
-                   "flop_formula": ("2*19*B*H*d*(valid (i,j) pairs of the band)"
-                                    if w.window != (-1, -1) or w.segments or w.blocks
-                                    else "2*19*B*H*N^2*d*(1/2 if causal)")},
+        "config": workload_config(w, world),
         "frac_of_bf16_peak": value / world / peak,
         "frac_of_bf16_sustained": value / world / peaks["bf16_sustained"],
         "roofline": roofline,
