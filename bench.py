@@ -75,15 +75,22 @@ def valid_pairs_rows(w, rows):
 
 # the forward's own engine: no BoB kernel instantiates anything from it, so
 # its edits leave the BoB kernels' recorded traffic valid
+# Sources each BoB kernel family is not built from: the forward's engine (no
+# BoB kernel uses its templates) and, for head dims up to 128, the
+# head-dimension-256 engine (its own translation unit; the other kernels do not
+# include it).  Shared headers and the host code stay in every family's hash.
 NOT_BOB_SOURCES = ("fwd_engine.cuh",)
+WIDE_ONLY_SOURCES = ("wide_engine.cuh", "wide_kernels.cu")
 
 
-def source_hash() -> str:
-    """Hash of the BoB kernels' sources (the kernel sources of csrc, without
-    build or cache folders and without NOT_BOB_SOURCES)."""
+def source_hash(d: int = 128) -> str:
+    """Hash of the sources the BoB kernels of head dim d are built from (the
+    kernel and host sources of csrc, without build or cache folders, without
+    NOT_BOB_SOURCES, and without WIDE_ONLY_SOURCES when d <= 128)."""
     h = hashlib.sha256()
     for f in sorted(os.listdir(CSRC)):
         if (not f.endswith((".cu", ".cuh", ".h")) or f in NOT_BOB_SOURCES
+                or (d <= 128 and f in WIDE_ONLY_SOURCES)
                 or not os.path.isfile(os.path.join(CSRC, f))):
             continue
         with open(os.path.join(CSRC, f), "rb") as fh:
@@ -101,13 +108,13 @@ def measured_peaks():
     return {"bf16": 1900.0, "bf16_sustained": 1700.0, "hbm": 6800.0, "source": "fallback"}
 
 
-def ncu_traffic(kernel_key, workload):
+def ncu_traffic(kernel_key, workload, d=128):
     """Per-launch DRAM bytes from the committed ncu summary, if it was taken on
     the current kernel source (else None)."""
     p = os.path.join(ROOT, "profiles", "traffic.txt")
     if not os.path.exists(p):
         return None
-    cur = source_hash()
+    cur = source_hash(d)
     with open(p) as fh:
         for line in fh:
             f = line.split()
@@ -416,7 +423,7 @@ def run_gpu(args, w):
                 "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
                 "peak_kind": f"bf16 burst ({peaks['source']})",
                 "frac_of_sustained": achieved / peaks["bf16_sustained"],
-                "traffic": ncu_traffic(dom, w.name),
+                "traffic": ncu_traffic(dom, w.name, w.d),
                 "credited_contractions": CONTRACTIONS[dom],
                 "launch_ms": dur, "share_of_step": dur / total,
                 "other_kernels_ms": {n: t for n, t in part_ms.items() if n != dom}}
