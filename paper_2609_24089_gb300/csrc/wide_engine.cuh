@@ -12,11 +12,14 @@
 //     stage of four tensors is 64 KB;
 //   * one or two stationary operands live in TMEM as MMA A operands (128
 //     columns each: bf16 pairs), written there once per CTA;
-//   * one accumulator per kernel.  BoB Pass 1 runs as three kernels: the row
-//     scalars alpha, E, D (eq. 6), then dOtil = P U_V + (P o h) V and
-//     Qtil = tau (Stil K + dS U_K) (eqs. 6-7) with those scalars known.  Pass
-//     2 runs as Vtil = (P o h)^T dO and Ktil = tau (Stil^T Q + dS^T U_Q), the
-//     latter over two CTAs per key block, each owning 128 output columns.
+//   * one accumulator per kernel.  BoB Pass 1 runs as two kernels: the row
+//     scalars alpha, E, D (eq. 6) together with dOtil (its alpha-free part
+//     dOtil0 = P U_V + (P o F) V accumulated in the same sweep, dOtil =
+//     dOtil0 - alpha o, eq. 8), then Qtil = tau (Stil K + dS U_K) (eqs. 6-7)
+//     with those scalars known.  (The per-pass entry points also run the row
+//     scalars alone and dOtil = P U_V + (P o h) V given them.)  Pass 2 runs
+//     as Vtil = (P o h)^T dO and Ktil = tau (Stil^T Q + dS^T U_Q), the latter
+//     over two CTAs per key block, each owning 128 output columns.
 //     The forward is two sweeps (L, then O with L known) and the first
 //     backward three kernels (dQ and D, dV, dK);
 //   * where a kernel reads a streamed tensor only in its stage A, that tensor
@@ -279,7 +282,8 @@ __global__ void __launch_bounds__(kThreads, 1) wide_engine(const __grid_constant
     const bool stall = p.inject_stall != 0;
     int issued_a[kMaxStages] = {-1, -1, -1, -1}, issued_b[kMaxStages] = {-1, -1, -1, -1};
     if (lane == 0 && !stall) {
-      for (int t = 0; t < C::NTS + C::NTA + C::NTB; ++t) tma_prefetch_desc(&p.tm[t]);
+      constexpr int kMaps = C::NTS + (C::PAIR ? 2 * C::NTA : C::NTA + C::NTB);
+      for (int t = 0; t < kMaps; ++t) tma_prefetch_desc(&p.tm[t]);
       mbar_arrive_expect_tx(&m->bar_stat, C::STAT_BYTES);
       for (int t = 0; t < C::NTS; ++t)
         for (int b = 0; b < WKB; ++b)

@@ -196,10 +196,11 @@ def test_runs_are_bitwise_identical():
         assert np.array_equal(a[n], b[n]), n
 
 
-def test_lemma_d2_embedding_on_gpu():
+@pytest.mark.parametrize("d", [64, 256])
+def test_lemma_d2_embedding_on_gpu(d):
     """V = dO = U_Q = U_K = 0, U_V = W: dOtil = softmax(tau Q K^T) W exactly
     (Lemma D.2) and the other outputs vanish."""
-    B, H, N, d = 1, 2, 200, 64
+    B, H, N = 1, 2, 200
     bits = G.inputs(B, H, N, d, seed=21)
     z = np.zeros_like(bits["q"])
     for n in ("v", "dout", "gq", "gk"):
@@ -311,7 +312,7 @@ def test_bounded_wait_timeout_is_reported_and_context_survives(monkeypatch, case
 
 
 @pytest.mark.parametrize("d,causal,rising", [(64, False, True), (128, True, True),
-                                             (128, False, False)])
+                                             (128, False, False), (256, True, True)])
 def test_forward_running_maximum_raised_many_times(d, causal, rising):
     """Scores that ramp along the keys by about 85 log2 units: the forward's
     lazily raised row maximum goes up some ten times (and every tile's largest
