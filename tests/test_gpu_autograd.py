@@ -10,7 +10,8 @@ from tests import gpu_util as G
 
 
 @pytest.mark.gpu
-@pytest.mark.parametrize("shape", [(1, 2, 200, 64, True), (1, 1, 257, 128, False)],
+@pytest.mark.parametrize("shape", [(1, 2, 200, 64, True), (1, 1, 257, 128, False),
+                                   (1, 2, 150, 256, True)],
                          ids=lambda s: "B{}H{}N{}d{}{}".format(*s[:4], "c" if s[4] else ""))
 def test_hessian_vector_product_through_autograd(shape):
     t = G.torch()
