@@ -147,7 +147,7 @@ typedef struct fbob_shape {
  *   S = scale * Q K^T + M,  P = softmax_row(S),  O = P V,
  *   lse_i = L_i = log sum_{j valid} exp(S_ij)   (natural log, fp32).
  * In:  q, k, v  bf16 [B,H,N,d].   Out: o bf16 [B,H,N,d], lse fp32 [B,H,N].
- * One kernel; at d = 256 two sweeps (lse, then o with lse known).
+ * One kernel (an online softmax over the key tiles).
  */
 int fbob_attn_fwd(const fbob_shape* shape, const void* q, const void* k, const void* v,
                   void* o, float* lse, struct CUstream_st* stream);

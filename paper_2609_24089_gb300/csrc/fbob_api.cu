@@ -619,25 +619,18 @@ int fbob_attn_fwd(const fbob_shape* s, const void* q, const void* k, const void*
   rc = check_ptrs(in, inb, 3, out, outb, 2);
   if (rc != FBOB_OK) return rc;
   if (s->d == 256) {
-    // two sweeps: L (over the ungated probabilities), then O with L known
+    // one sweep with an online softmax (wide_engine.cuh)
     const int64_t BHk = s->B * kv_heads(s);
     EngineParams p = base_params(s);
     p.q = static_cast<const __nv_bfloat16*>(q);
     p.nblk = n_blocks(s->N, BM);
+    p.vec_out = lse;
+    p.out0 = static_cast<__nv_bfloat16*>(o);
     choose_order(&p, p.BH);
-    EngineParams a = p;
-    a.vec_out = lse;
-    const MapSpec ma[1] = {{k, BHk, HB}};
-    if (!wide_maps(&a, s, ma, 1)) return FBOB_ERR_CUDA;
-    rc = run_wide(WOp::FwdL, a, false, p.nblk * p.BH, stream);
-    if (rc != FBOB_OK) return rc;
-    EngineParams b = p;
-    b.lse = lse;
-    b.out0 = static_cast<__nv_bfloat16*>(o);
-    const MapSpec mb[2] = {{k, BHk, HB}, {v, BHk, HB}};
-    if (!wide_maps(&b, s, mb, 2)) return FBOB_ERR_CUDA;
-    rc = run_wide(WOp::FwdO, b, has_dropout(s), p.nblk * p.BH, stream);
-    if (rc == FBOB_OK) g_launches[kEntFwd] = 2;
+    const MapSpec m[2] = {{k, BHk, HB}, {v, BHk, HB}};
+    if (!wide_maps(&p, s, m, 2)) return FBOB_ERR_CUDA;
+    rc = run_wide(WOp::Fwd, p, has_dropout(s), p.nblk * p.BH, stream);
+    if (rc == FBOB_OK) g_launches[kEntFwd] = 1;
     return rc;
   }
   EngineParams p = base_params(s);

@@ -20,8 +20,10 @@
 //     scalars alone and dOtil = P U_V + (P o h) V given them.)  Pass 2 runs
 //     as Vtil = (P o h)^T dO and Ktil = tau (Stil^T Q + dS^T U_Q), the latter
 //     over two CTAs per key block, each owning 128 output columns.
-//     The forward is two sweeps (L, then O with L known) and the first
-//     backward three kernels (dQ and D, dV, dK);
+//     The forward is one sweep with an online softmax (the two warpgroups
+//     share each tile's row maximum through shared memory; O in TMEM is
+//     rescaled only when the running maximum grows by more than 8 in log2
+//     units) and the first backward three kernels (dQ and D, dV, dK);
 //   * where a kernel reads a streamed tensor only in its stage A, that tensor
 //     has a ring of its own (ring B), released as soon as the stage-A MMAs
 //     reading it complete.
@@ -48,8 +50,8 @@
 
 namespace fbob {
 
-// WOp (engine_params.h): FwdL: L (eq. 1, first sweep); FwdO: O with L known
-// (second sweep).  Stats: alpha, E, D (eq. 6); DOut: dOtil; DQ: Qtil (eqs.
+// WOp (engine_params.h): Fwd: O and L (eq. 1).  Stats: alpha, E, D (eq.
+// 6); DOut: dOtil; DQ: Qtil (eqs.
 // 6-7).  StatsDO: alpha, E, D and dOtil in one sweep: dOtil0 = P U_V +
 // (P o F) V needs no row scalar, and dOtil = dOtil0 - alpha o (Prop. 3.1,
 // eq. 8).  BwdDQ: dQ and D; BwdDV: dV; BwdDK: dK (eqs. 2-3).  P2V: Vtil;
@@ -77,16 +79,16 @@ constexpr int kWStat = WKB * BM * 128;  // one stationary 128 x 256 bf16 tensor 
 template <WOp OP>
 struct WCfg {
   static constexpr bool PAIR = OP == WOp::StatsDO;
-  static constexpr bool ROW = OP == WOp::FwdL || OP == WOp::FwdO || OP == WOp::Stats ||
+  static constexpr bool ROW = OP == WOp::Fwd || OP == WOp::Stats ||
                               OP == WOp::DOut || OP == WOp::DQ || OP == WOp::BwdDQ || PAIR;
   static constexpr int NTT = (OP == WOp::Stats || OP == WOp::P2K) ? 2 : 1;
-  static constexpr int NTS = (OP == WOp::FwdL || OP == WOp::FwdO || OP == WOp::BwdDV) ? 0
+  static constexpr int NTS = (OP == WOp::Fwd || OP == WOp::BwdDV) ? 0
                              : (OP == WOp::DQ || OP == WOp::P2K || PAIR)             ? 2
                                                                                      : 1;
   // (PAIR: tensors per slot; the maps hold K, U_K, then V, U_V)
   static constexpr int NTA = (OP == WOp::Stats || OP == WOp::DOut) ? 4
                              : OP == WOp::P2V                        ? 3
-                             : (OP == WOp::FwdO || OP == WOp::DQ || OP == WOp::P2K ||
+                             : (OP == WOp::Fwd || OP == WOp::DQ || OP == WOp::P2K ||
                                 OP == WOp::BwdDV || PAIR)
                                  ? 2
                                  : 1;
@@ -113,10 +115,10 @@ struct WCfg {
                                                                                    : 0;
   static constexpr int NDC = DCW == 0 ? 0 : (OP == WOp::DQ || OP == WOp::P2K || PAIR) ? 1 : 2;
   static constexpr int NDC1 = NDC > 0 ? NDC : 1;  // (divisor where there is no DC)
-  static constexpr int ACC_N = (OP == WOp::FwdL || OP == WOp::Stats) ? 0 : OP == WOp::P2K ? 128 : 256;
+  static constexpr int ACC_N = OP == WOp::Stats ? 0 : OP == WOp::P2K ? 128 : 256;
   static constexpr int SPLIT = OP == WOp::P2K ? 2 : 1;
   // stage-B operand tiles written over the SF columns (else over DC)
-  static constexpr bool OPS_SF = OP == WOp::FwdO || OP == WOp::DOut || OP == WOp::P2V ||
+  static constexpr bool OPS_SF = OP == WOp::Fwd || OP == WOp::DOut || OP == WOp::P2V ||
                                  OP == WOp::BwdDV;
   static constexpr bool OPS_DC = OP == WOp::DQ || OP == WOp::BwdDQ || OP == WOp::P2K ||
                                  OP == WOp::BwdDK || PAIR;
@@ -124,10 +126,12 @@ struct WCfg {
   // issuer Y reads ring A (stage B, or the statistics kernel's DC); with
   // PAIR each slot has one releasing issuer
   static constexpr bool Y_READS_A = (HAS_B || OP == WOp::Stats) && !PAIR;
-  // D = do . o summed in the prologue; alpha / E0 row sums (or the online
-  // maximum and sum) exchanged between the two warpgroups
+  // D = do . o summed in the prologue; alpha / E0 row sums (or the
+  // forward's row sums) exchanged between the two warpgroups; the forward's
+  // per-tile row maxima exchanged likewise (MX)
   static constexpr bool ROW_DOTS = OP == WOp::Stats || OP == WOp::BwdDQ || PAIR;
-  static constexpr bool XCHG = OP == WOp::Stats || OP == WOp::FwdL || PAIR;
+  static constexpr bool XCHG = OP == WOp::Stats || OP == WOp::Fwd || PAIR;
+  static constexpr bool MX = OP == WOp::Fwd;
 
   // TMEM columns
   static constexpr uint32_t ACC_COL = 128u * NTT;
@@ -144,7 +148,8 @@ struct WCfg {
   static constexpr int OFF_B = OFF_A + NSA * STAGE_A;
   static constexpr int OFF_VEC = OFF_B + NSB * STAGE_B;
   static constexpr int OFF_MISC = OFF_VEC + NSA * VEC_BYTES;
-  static constexpr int MISC_BYTES = 512 + (XCHG ? 4 * BM * 4 : 0) + (ROW_DOTS ? BM * 4 : 0);
+  static constexpr int MISC_BYTES =
+      512 + (XCHG ? 4 * BM * 4 : 0) + (ROW_DOTS ? BM * 4 : 0) + (MX ? 4 * BM * 4 : 0);
   static constexpr int SMEM_BYTES = OFF_MISC + MISC_BYTES;
   static_assert(SMEM_BYTES <= 232448, "shared-memory plan exceeds 227 KB");
   static_assert(NSA <= kMaxStages && NSB <= kMaxStages, "ring bound");
@@ -158,6 +163,7 @@ struct WMisc {
   uint64_t dc[2], dc_read[2];
   uint64_t ew[2];  // the elementwise warps wrote the stage-B operands of tile t (t & 1)
   uint64_t sb[2];  // stage B(t) completed (per SF buffer)
+  uint64_t mx[2];  // forward: both warpgroups posted tile t's row maxima (t & 1)
   uint64_t acc;
   uint32_t tmem_base;
   uint32_t pad;
@@ -198,6 +204,7 @@ __global__ void __launch_bounds__(kThreads, 1) wide_engine(const __grid_constant
   WMisc* m = reinterpret_cast<WMisc*>(smem + C::OFF_MISC);
   float* s_xchg = reinterpret_cast<float*>(smem + C::OFF_MISC + 512);  // 4 x BM floats
   float* s_d = s_xchg + (C::XCHG ? 4 * BM : 0);                        // BM floats
+  float* s_mx = s_d + (C::ROW_DOTS ? BM : 0);  // forward: [tile & 1][warpgroup][row]
 
   const int tid = threadIdx.x;
   const int warp = tid >> 5;
@@ -261,6 +268,7 @@ __global__ void __launch_bounds__(kThreads, 1) wide_engine(const __grid_constant
       mbar_init(&m->dc_read[b], kEwThreads);
       mbar_init(&m->ew[b], kEwThreads);
       mbar_init(&m->sb[b], 1);
+      mbar_init(&m->mx[b], kEwThreads);
     }
     mbar_init(&m->acc, 2);
     fence_mbar_init();
@@ -504,7 +512,7 @@ __global__ void __launch_bounds__(kThreads, 1) wide_engine(const __grid_constant
             for (int s = 0; s < 2; ++s) {  // K-step s: streamed rows 16 s .. (warpgroup s)
               const uint32_t first = (st == 0 && s == 0) ? 0u : 1u;
               const uint32_t As = A + 16 * s;
-              if constexpr (OP == WOp::FwdO) {  // O += P V
+              if constexpr (OP == WOp::Fwd) {  // O += P V
                 mma_ts(acc, As, md(stg, C::NTA, 1, s, 0), id_b, first);
               } else if constexpr (OP == WOp::DOut) {  // dOtil += P U_V + (P o h) V
                 mma_ts(acc, As, md(stg, C::NTA, 3, s, 0), id_b, first);
@@ -538,9 +546,7 @@ __global__ void __launch_bounds__(kThreads, 1) wide_engine(const __grid_constant
           }
         }
       }
-      // (issuer Y of the first forward sweep issues nothing: a plain arrive)
-      if (warp == kMmaWarpY && !C::HAS_B && C::NDC == 0) mbar_arrive(&m->acc);
-      else mma_commit(&m->acc);
+      mma_commit(&m->acc);
       if (*abort_flag) drain_wait(&m->acc, 0);
     }
   } else {
@@ -569,10 +575,12 @@ __global__ void __launch_bounds__(kThreads, 1) wide_engine(const __grid_constant
     const float2 sl2v = splat(sl2), tauv = splat(tau);
     const DropKey dkey = {p.drop_rk, p.drop_tlow4, p.drop_tmask};
     const float dsig = p.drop_sigma;
+    // every lane of a warp takes a wait's outcome together: the TMEM loads
+    // and stores after it are warp-collective (and with dropout the lanes
+    // exchange keep bits), so no lane may leave the loop alone
     auto ew_wait = [&](uint64_t* bar, uint32_t par) -> bool {
       const bool w = mbar_wait(bar, par, wctl);
-      if constexpr (DROP) return __all_sync(0xffffffffu, w);
-      return w;
+      return __all_sync(0xffffffffu, w);
     };
 
     // ---- stationary operands into TMEM (bf16 pairs: word c of a row =
@@ -601,7 +609,7 @@ __global__ void __launch_bounds__(kThreads, 1) wide_engine(const __grid_constant
     // ---- row scalars of a stationary row (row kernels)
     float nL2 = 0.f, nal = 0.f, nE = 0.f, Dr = 0.f;
     if constexpr (kRow) {
-      if (row_ok && OP != WOp::FwdL) {
+      if (row_ok && OP != WOp::Fwd) {
         const size_t ri = (size_t)bh_stat * N + gr;
         nL2 = -p.lse[ri] * kLog2e;
         if constexpr (OP == WOp::DOut || OP == WOp::DQ) {
@@ -616,7 +624,7 @@ __global__ void __launch_bounds__(kThreads, 1) wide_engine(const __grid_constant
     const float2 nL2v = splat(nL2), nalv = splat(nal), nEv = splat(nE), nDv = splat(-Dr);
 
     float2 acc_a = splat(0.f), acc_e = splat(0.f);      // row sums (statistics)
-    float run_m = -INFINITY, run_l = 0.f;               // online max / sum (L)
+    float run_m = -INFINITY, run_l = 0.f;  // forward: running maximum (log2 units) and sum
     bool ok = true;
     int tile = first_tile - 1;
     for (int st = 0; ok && st < nsteps; ++st) {
@@ -674,19 +682,72 @@ __global__ void __launch_bounds__(kThreads, 1) wide_engine(const __grid_constant
       const int mlo = vlo - c0, mhi = vhi - c0;  // valid columns: mlo <= c < mhi
       if (mlo > 0 || mhi < 16) mask16(rS, mlo, mhi);
 
-      if constexpr (OP == WOp::FwdL) {
-        // online log-sum-exp over this thread's columns (log2 units)
+      if constexpr (OP == WOp::Fwd) {
+        // this thread's tile maximum (log2 units), shared with the other
+        // warpgroup's half of the row behind mx[t & 1] (bounded wait)
         float mt = -INFINITY;
 #pragma unroll
         for (int c = 0; c < 16; ++c) mt = fmaxf(mt, bits_f(rS[c]));
-        const float mn = fmaxf(run_m, mt * sl2);
-        if (mn != -INFINITY) {
-          float s = 0.f;
-#pragma unroll
-          for (int c = 0; c < 16; ++c) s += ex2(fmaf(bits_f(rS[c]), sl2, -mn));
-          run_l = run_l * ex2(run_m - mn) + s;
-          run_m = mn;
+        mt *= sl2;
+        float* mxs = s_mx + (st & 1) * 2 * BM;
+        mxs[wg * BM + r] = mt;
+        mbar_arrive(&m->mx[st & 1]);
+        if (!ew_wait(&m->mx[st & 1], (st >> 1) & 1)) {
+          ok = false;
+          break;
         }
+        const float mrow = fmaxf(mt, mxs[(1 - wg) * BM + r]);
+        // the running maximum is raised only when a tile's exceeds it by
+        // more than 8 (so P <= 2^8): then the row sum and O (once the MMAs
+        // into it so far have completed) are scaled by 2^(old - new); both
+        // warpgroups take the same decision from the same maxima.  The
+        // TMEM loads and stores are warp-collective, so a warp rescales
+        // together whenever one of its rows needs it (the others by 1)
+        const bool raise = mrow > run_m + 8.f;
+        const float sc = raise ? ex2(run_m - mrow) : 1.f;  // 0 while run_m is -inf
+        // (a row whose maximum was -inf so far holds only zeros in O)
+        if (__any_sync(0xffffffffu, raise && run_m != -INFINITY) && st > 0) {
+          if (!ew_wait(&m->sb[(st - 1) % C::NSF], ((st - 1) / C::NSF) & 1)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+#pragma unroll 1
+          for (int q = 0; q < 8; ++q) {
+            const uint32_t ca = ta + C::ACC_COL + 128 * wg + 16 * q;
+            uint32_t rO[16];
+            tmem_ld16(ca, rO);
+            tmem_ld_wait(rO);
+            uint32_t w0[8], w1[8];
+#pragma unroll
+            for (int c = 0; c < 8; ++c) {
+              w0[c] = __float_as_uint(bits_f(rO[c]) * sc);
+              w1[c] = __float_as_uint(bits_f(rO[8 + c]) * sc);
+            }
+            tmem_st8(ca, w0);
+            tmem_st8(ca + 8, w1);
+          }
+        }
+        if (raise) {
+          run_l *= sc;
+          run_m = mrow;
+        }
+        const float2 mu = splat(run_m == -INFINITY ? 0.f : -run_m);
+        uint32_t o0[8];
+        float2 ls = splat(0.f);
+#pragma unroll
+        for (int c = 0; c < 16; c += 2) {
+          const float2 pr = probs2(pair(rS, c), sl2v, mu);
+          ls = __fadd2_rn(ls, pr);
+          float2 gp = pr;
+          if constexpr (DROP) gp = __fmul2_rn(pr, gate2(kb, c, dsig));  // O = (sigma R o P) V
+          o0[c / 2] = pack_bf16(gp.x, gp.y);
+        }
+        run_l += ls.x + ls.y;
+        tmem_st8(Rsf, o0);
+        tmem_st_wait();
+        tc_fence_before();
+        mbar_arrive(&m->ew[st & 1]);
       } else {
         uint32_t o0[8], o1[8];
 #pragma unroll
@@ -707,7 +768,7 @@ __global__ void __launch_bounds__(kThreads, 1) wide_engine(const __grid_constant
           const float2 pr = probs2(pair(rS, c), sl2v, cL2);
           float2 g = splat(1.f);
           if constexpr (DROP) g = gate2(kb, c, dsig);
-          if constexpr (OP == WOp::FwdO || OP == WOp::BwdDV) {  // (sigma R o P)
+          if constexpr (OP == WOp::BwdDV) {  // (sigma R o P)
             const float2 gp = DROP ? __fmul2_rn(pr, g) : pr;
             o0[c / 2] = pack_bf16(gp.x, gp.y);
           } else if constexpr (C::PAIR) {
@@ -784,25 +845,36 @@ __global__ void __launch_bounds__(kThreads, 1) wide_engine(const __grid_constant
     // ---------------------------------------------------------- epilogue
     if (ok) ok = mbar_wait(&m->acc, 0, wctl);
     if (ok && *abort_flag) ok = false;
+    ok = __all_sync(0xffffffffu, ok);  // (the TMEM loads below are warp-collective)
     tc_fence_after();
     if constexpr (C::XCHG) {
       if constexpr (OP == WOp::Stats || C::PAIR) {
         s_xchg[wg * BM + r] = acc_a.x + acc_a.y;
         s_xchg[(2 + wg) * BM + r] = acc_e.x + acc_e.y;
-      } else {
-        s_xchg[wg * BM + r] = run_m;
-        s_xchg[(2 + wg) * BM + r] = run_l;
+      } else {  // the forward: each warpgroup's row sum (the maxima agree)
+        s_xchg[wg * BM + r] = run_l;
       }
       named_bar_sync(1, kEwThreads);
     }
     if (ok) {
       const size_t ri = (size_t)bh_stat * N + gr;
-      if constexpr (OP == WOp::FwdL) {
-        if (row_ok && wg == 0) {
-          const float m0 = s_xchg[r], m1 = s_xchg[BM + r];
-          const float mx = fmaxf(m0, m1);
-          const float l = s_xchg[2 * BM + r] * ex2(m0 - mx) + s_xchg[3 * BM + r] * ex2(m1 - mx);
-          p.vec_out[ri] = (mx + log2f(l)) * kLn2;  // natural-log L
+      if constexpr (OP == WOp::Fwd) {
+        // O = (sum of P V) / l and the natural-log L = (m + log2 l) ln 2
+        const float l = s_xchg[r] + s_xchg[BM + r];
+        const float il = l > 0.f ? 1.f / l : 0.f;
+        if (row_ok && wg == 0) p.vec_out[ri] = (run_m + log2f(l)) * kLn2;
+#pragma unroll 1
+        for (int q = 0; q < WD / 32; ++q) {
+          const int cc = wg * (WD / 2) + 16 * q;
+          uint32_t rA[16];
+          tmem_ld16(ta + C::ACC_COL + cc, rA);
+          tmem_ld_wait(rA);
+          if (row_ok) {
+            float v[16];
+#pragma unroll
+            for (int c = 0; c < 16; ++c) v[c] = bits_f(rA[c]) * il;
+            store_row16(p.out0 + rowoff + cc, v);
+          }
         }
       } else if constexpr (OP == WOp::Stats) {
         if (row_ok && wg == 0) {

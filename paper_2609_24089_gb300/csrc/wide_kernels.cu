@@ -1,7 +1,6 @@
 // wide_kernels.cu -- instantiations and launcher of the head-dimension-256
 // kernels (wide_engine.cuh): forward (eq. 1), first backward (eqs. 2-3) and
-// both passes of BoB (Alg. 2), each with and without dropout (the first
-// forward sweep, L over the ungated probabilities, has no dropout form).
+// both passes of BoB (Alg. 2), each with and without dropout.
 #include "launch.h"
 #include "wide_engine.cuh"
 
@@ -24,8 +23,7 @@ static cudaError_t launch_op(bool drop, const EngineParams& p, int nblocks, cuda
 
 cudaError_t launch_wide(WOp op, bool drop, const EngineParams& p, int nblocks, cudaStream_t s) {
   switch (op) {
-    case WOp::FwdL: return drop ? cudaErrorInvalidValue : launch_one<WOp::FwdL, false>(p, nblocks, s);
-    case WOp::FwdO: return launch_op<WOp::FwdO>(drop, p, nblocks, s);
+    case WOp::Fwd: return launch_op<WOp::Fwd>(drop, p, nblocks, s);
     case WOp::Stats: return launch_op<WOp::Stats>(drop, p, nblocks, s);
     case WOp::DOut: return launch_op<WOp::DOut>(drop, p, nblocks, s);
     case WOp::DQ: return launch_op<WOp::DQ>(drop, p, nblocks, s);
