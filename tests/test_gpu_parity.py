@@ -253,7 +253,7 @@ STALL_CASES = [  # entry, d, causal, dropout
     ("bwd", 128, True, (0.1, 4)),
     ("bob", 256, True, None),     # head dim 256: the five wide kernels of BoB
     ("bob", 256, False, (0.1, 6)),
-    ("fwd", 256, True, None),     # the forward's two sweeps
+    ("fwd", 256, True, None),     # the d = 256 forward (online softmax)
     ("bwd", 256, False, (0.1, 7)),  # dQ, dV and dK kernels
 ]
 
