@@ -80,7 +80,7 @@ def valid_pairs_rows(w, rows):
 # head-dimension-256 engine (its own translation unit; the other kernels do not
 # include it).  Shared headers and the host code stay in every family's hash.
 NOT_BOB_SOURCES = ("fwd_engine.cuh",)
-WIDE_ONLY_SOURCES = ("wide_engine.cuh", "wide_kernels.cu")
+WIDE_ONLY_SOURCES = ("wide_engine.cuh", "wide_kernels.cu", "wide_launch.h")
 
 
 def source_hash(d: int = 128) -> str:

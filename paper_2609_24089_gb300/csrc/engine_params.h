@@ -32,11 +32,6 @@ constexpr float kLn2 = 0.6931471805599453f;
 // (Fwd names the forward for the launcher; it runs in fwd_engine.cuh.)
 enum class RowOp { Fwd, BwdDQ, BobPass1, BobStats, BobPass1D };
 enum class ColOp { BwdDKDV, BobPass2 };
-// Head dimension 256 (wide_engine.cuh): Fwd the forward (O and L, online
-// softmax); Stats, DOut, DQ BoB Pass 1 (alpha E D, dOtil, Qtil); StatsDO alpha
-// E D and dOtil in one sweep; P2V, P2K BoB Pass 2 (Vtil, Ktil); BwdDQ, BwdDV,
-// BwdDK the first backward.
-enum class WOp { Fwd = 1, Stats, DOut, DQ, BwdDQ, P2V, P2K, BwdDV, BwdDK, StatsDO };
 
 // ---------------------------------------------------------------- parameters
 struct EngineParams {

@@ -11,6 +11,7 @@
 
 #include "../../include/fbob.h"
 #include "launch.h"
+#include "wide_launch.h"
 
 namespace fbob {
 namespace {

@@ -18,12 +18,9 @@ cudaError_t launch_row(RowOp op, int d, bool drop, const EngineParams& p, int nb
 cudaError_t launch_col(ColOp op, int d, bool drop, const EngineParams& p, int nblocks,
                        cudaStream_t s);
 
-// head dimension 256 (wide_engine.cuh)
-cudaError_t launch_wide(WOp op, bool drop, const EngineParams& p, int nblocks, cudaStream_t s);
-
-// Read and clear the error word of the row / column / wide engine unit.
+// Read and clear the error word of the row / column engine unit (the
+// head-dimension-256 unit: wide_launch.h).
 cudaError_t take_row_error(uint32_t* word, cudaStream_t s);
 cudaError_t take_col_error(uint32_t* word, cudaStream_t s);
-cudaError_t take_wide_error(uint32_t* word, cudaStream_t s);
 
 }  // namespace fbob

@@ -47,10 +47,11 @@
 #pragma once
 
 #include "attn_engine.cuh"
+#include "wide_launch.h"
 
 namespace fbob {
 
-// WOp (engine_params.h): Fwd: O and L (eq. 1).  Stats: alpha, E, D (eq.
+// WOp (wide_launch.h): Fwd: O and L (eq. 1).  Stats: alpha, E, D (eq.
 // 6); DOut: dOtil; DQ: Qtil (eqs.
 // 6-7).  StatsDO: alpha, E, D and dOtil in one sweep: dOtil0 = P U_V +
 // (P o F) V needs no row scalar, and dOtil = dOtil0 - alpha o (Prop. 3.1,

@@ -3,6 +3,7 @@
 // both passes of BoB (Alg. 2), each with and without dropout.
 #include "launch.h"
 #include "wide_engine.cuh"
+#include "wide_launch.h"
 
 namespace fbob {
 
