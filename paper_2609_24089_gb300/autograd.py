@@ -9,7 +9,7 @@ BoB returns the total derivatives of Phi = <dQ,U_Q> + <dK,U_K> + <dV,U_V>
 with respect to Q, K, V and dO, the paths through O and L included (Sec. 3.1).
 The first-backward node therefore takes O and L as plain, non-differentiable
 inputs.  Inputs are contiguous CUDA bf16 tensors [B, H, N, d] with d in
-{32, 64, 128}; there is no CPU or PyTorch fallback.
+{32, 64, 128, 256}; there is no CPU or PyTorch fallback.
 """
 from __future__ import annotations
 
